@@ -1,0 +1,204 @@
+/*
+ * adept.h -- C ABI of the GB300 (sm_103a) library for ADEPT's token-level
+ * early-exit forward pass (arXiv 2601.03700).
+ *
+ * Notation follows the paper's problem statement (Sec. 3): N layers, indexed
+ * i = 1..N (1-based everywhere in this API), tokens j, hidden size D_h
+ * (d_model), query/key/value size D_q (heads x head_dim), exit layer i*.
+ *
+ * Conventions shared by every call:
+ *  - Pointers prefixed d_ are DEVICE pointers owned by the caller; they must stay
+ *    valid until the work queued on `stream` has finished.  Pointers prefixed
+ *    h_ are host pointers read before the call returns.
+ *  - `stream` is a cudaStream_t (NULL = legacy default stream).  Every call that
+ *    takes a stream only enqueues work on it and returns; results are valid once
+ *    the stream has been synchronised.
+ *  - The library owns its copy of the weights, the paged KV cache and its
+ *    workspaces (allocated by adept_model_load, released by adept_free).
+ *  - Errors are returned as adept_status; nothing is thrown across the ABI.
+ *    Argument errors are detected on the host before anything is enqueued.
+ *    Device-side input errors (a forced exit layer or token id out of range)
+ *    set a device error word that adept_check_device_status reports.
+ *    adept_last_error returns a message for the last failing call.
+ *  - A model is not thread-safe: calls on one model must be serialised.
+ */
+#ifndef ADEPT_H
+#define ADEPT_H
+
+#include <stdint.h>
+
+#if defined(__GNUC__)
+#define ADEPT_API __attribute__((visibility("default")))
+#else
+#define ADEPT_API
+#endif
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum {
+  ADEPT_OK = 0,
+  ADEPT_ERR_INVALID_ARG = 1,   /* bad argument; nothing was enqueued */
+  ADEPT_ERR_OOM = 2,           /* device allocation failed */
+  ADEPT_ERR_CAPACITY = 3,      /* batch / sequence / KV-block capacity exceeded */
+  ADEPT_ERR_CUDA = 4,          /* a CUDA runtime or driver call failed */
+  ADEPT_ERR_TIMEOUT = 5,       /* a bounded device-side wait gave up */
+  ADEPT_ERR_DEVICE_INPUT = 6   /* device-side validation of an input failed */
+} adept_status;
+
+enum { ADEPT_FAMILY_LLAMA = 0,   /* RMSNorm pre-norm, RoPE, SwiGLU, untied head */
+       ADEPT_FAMILY_GPT2 = 1,    /* LayerNorm pre-norm, learned positions, tanh-GELU, biases, tied head */
+       ADEPT_FAMILY_BERT = 2 };  /* post-LN encoder, bidirectional, pooler + classifier */
+
+enum { ADEPT_DTYPE_F32 = 0, ADEPT_DTYPE_BF16 = 1 };
+
+typedef struct {
+  int family;          /* ADEPT_FAMILY_* */
+  int n_layers;        /* N */
+  int d_model;         /* D_h */
+  int n_heads;
+  int n_kv_heads;      /* 0 -> n_heads */
+  int head_dim;        /* D_q = n_heads * head_dim; must be even, <= 128 */
+  int d_ffn;
+  int vocab;
+  int max_pos;         /* learned-position table size (GPT-2 / BERT) */
+  int n_classes;       /* encoder classifier outputs */
+  int dtype;           /* ADEPT_DTYPE_*: storage and GEMM-input precision; accumulation is fp32 */
+  float norm_eps;
+  float rope_theta;
+  float hsm_eps;       /* eps of the three RMS normalisations inside the HSM */
+  int hsm_m1;          /* HSM FC1 / FC3 output width (Table S1: 4 D_h) */
+  int hsm_m2;          /* HSM FC2 output width (Table S1: 8 D_h) */
+  int kv_block_tokens; /* positions per KV-cache block (16) */
+  int max_batch;       /* sequences */
+  int max_seq;         /* positions per sequence (prompt + generated) */
+  int kv_pool_blocks;  /* 0 -> max_batch * ceil(max_seq / kv_block_tokens) */
+  uint64_t block_shuffle_seed; /* 0: KV blocks handed out in order; else a seeded permutation */
+} adept_config;
+
+/* One named weight tensor.  `data` may be a host or a device pointer (it is read
+ * with cudaMemcpyDefault); its element type is the model dtype; `numel` must equal
+ * the element count of the named shape.  Names (0-based layer slot l = paper layer
+ * l+1; matrices are [out, in] row-major):
+ *   tok_emb [V,D]; pos_emb [max_pos,D] (GPT-2/BERT); type_emb [D], emb_ln.g/.b [D] (BERT)
+ *   layers.l.attn_norm.g/.b, layers.l.ffn_norm.g/.b [D]   (.b not for LLAMA)
+ *   layers.l.wq [D_q,D], wk [D_kv,D], wv [D_kv,D], wo [D,D_q]; bq bk bv bo (not LLAMA)
+ *   LLAMA: layers.l.w_gate [F,D], w_up [F,D], w_down [D,F]
+ *   GPT2/BERT: layers.l.w_fc [F,D], b_fc [F], w_proj [D,F], b_proj [D]
+ *   LLAMA: final_norm.g [D], lm_head [V,D]; GPT2: final_norm.g/.b [D] (head tied to tok_emb)
+ *   BERT: pool.w [D,D], pool.b [D], cls.w [C,D], cls.b [C]
+ *   HSM (App. B Table S1): hsm.g0 [D], hsm.conv_w [3,3], hsm.conv_b [1],
+ *     hsm.fc1_w [m1,D], hsm.fc1_b, hsm.fc2_w [m2,m1], hsm.fc2_b, hsm.fc3_w [m1,m2],
+ *     hsm.fc3_b, hsm.g1 [m1], hsm.fc4_w [D,m1], hsm.fc4_b [D], hsm.g2 [D]      */
+typedef struct {
+  const char* name;
+  const void* data;
+  int64_t numel;
+} adept_tensor;
+
+typedef struct {
+  const adept_tensor* tensors;
+  int n_tensors;
+} adept_tensor_table;
+
+typedef struct adept_model adept_model;  /* opaque, library-owned */
+
+/* Load a model: validate `cfg`, allocate device memory, copy and repack the weights
+ * (norm gains and LN shifts are folded into the following projection), allocate
+ * the paged KV pool.  Synchronises `stream` before returning.
+ * Errors: INVALID_ARG (bad config, missing or mis-sized tensor), OOM, CUDA. */
+ADEPT_API adept_status adept_model_load(const adept_config* cfg, const adept_tensor_table* weights,
+                              void* stream, adept_model** out);
+
+/* Prompt pass (prefill) of `batch` sequences of `prompt_len` tokens each; resets
+ * sequences 0..batch-1 and reserves KV blocks for their whole max_seq.
+ * Per layer i (App. H): the still-active tokens run layer i; for 2 <= i <= N-1 each
+ * active token tests <s_hat_i, I_hat> >= delta (Sec. 4.1), or, where
+ * d_forced_exit[j] != 0, exits exactly at that layer; exiting tokens are mapped by
+ * the HSM (Sec. 4.2) and their K/V for every skipped layer r > i* are produced
+ * from s~_N (Sec. 4.3) before layer r's attention.
+ *   d_tokens        [batch*prompt_len] int32 token ids, sequence-major
+ *   delta           exit threshold (+inf: never exit)
+ *   d_forced_exit   [batch*prompt_len] int32, 0 = use delta, else i* in [2, N]; or NULL
+ *   d_exit_layer_out[batch*prompt_len] int32 i* per token (N = full depth); or NULL
+ *   d_logits_out    decoder: [batch, vocab] fp32 logits of each sequence's last token;
+ *                   encoder: [batch, n_classes] classifier logits of position 0; or NULL
+ *   d_next_token_out[batch] int32 greedy argmax of the logits (lowest index on ties); or NULL
+ *   d_sim_out       [batch*prompt_len, N] fp32 cosine at each tested layer, NaN elsewhere; or NULL
+ * Errors: INVALID_ARG, CAPACITY (batch > max_batch, prompt_len > max_seq). */
+ADEPT_API adept_status adept_prefill(adept_model* m, int batch, int prompt_len, const int32_t* d_tokens,
+                           float delta, const int32_t* d_forced_exit, int32_t* d_exit_layer_out,
+                           float* d_logits_out, int32_t* d_next_token_out, float* d_sim_out,
+                           void* stream);
+
+/* One generation step (App. H, generation phase): token b of sequence b is appended
+ * at that sequence's next position and exits independently of the others.  Same
+ * per-token outputs as adept_prefill with batch rows.  Decoder families only.
+ * Errors: INVALID_ARG, CAPACITY (a sequence is full). */
+ADEPT_API adept_status adept_decode_step(adept_model* m, int batch, const int32_t* d_tokens, float delta,
+                               const int32_t* d_forced_exit, int32_t* d_exit_layer_out,
+                               float* d_logits_out, int32_t* d_next_token_out, float* d_sim_out,
+                               void* stream);
+
+/* Decoupled skipped-layer KV fill (Sec. 4, decoupling equation; Sec. 4.3 KV
+ * generation): for every token j and every layer r = i*_j+1..N, writes layer r's
+ * K = RoPE(W_K^r norm_r(s~_j) + b_K^r) and V = W_V^r norm_r(s~_j) + b_V^r into the
+ * KV cache at (d_seq[j], d_pos[j]); all (token, layer) pairs in one grouped launch.
+ *   d_h_mapped  [n_tokens, D] mapped states s~_N in the model dtype
+ *   d_exit_layer[n_tokens] int32 i* in [1, N] (N: nothing to fill)
+ *   d_seq, d_pos[n_tokens] int32 sequence and position; their KV blocks must have been
+ *               reserved (adept_prefill or adept_seq_reserve)
+ * Errors: INVALID_ARG, CAPACITY (n_tokens above the fill workspace limit, 1<<20). */
+ADEPT_API adept_status adept_skip_kv_fill(adept_model* m, int n_tokens, const void* d_h_mapped,
+                                const int32_t* d_exit_layer, const int32_t* d_seq,
+                                const int32_t* d_pos, void* stream);
+
+/* Release everything the model owns (synchronises the device first).  NULL is a no-op. */
+ADEPT_API void adept_free(adept_model* m);
+
+/* ---- helpers (not part of the method; used by tests and the benchmark) ---- */
+
+/* Message of the last failing call on `m` (or of the last failed load when m is NULL). */
+ADEPT_API const char* adept_last_error(const adept_model* m);
+ADEPT_API const char* adept_status_string(adept_status s);
+
+/* Reset sequences 0..batch-1 to lengths h_lens[b] and reserve their KV blocks for
+ * max_seq positions (no compute; the cached values are left undefined). */
+ADEPT_API adept_status adept_seq_reserve(adept_model* m, int batch, const int32_t* h_lens);
+
+/* Copy K and V of `n_pos` positions starting at pos0 of sequence `seq` at layer
+ * `layer` (1-based) out of the paged cache into d_k_out / d_v_out, each
+ * [n_pos, n_kv_heads, head_dim] in the model dtype. */
+ADEPT_API adept_status adept_read_kv(adept_model* m, int layer, int seq, int pos0, int n_pos,
+                           void* d_k_out, void* d_v_out, void* stream);
+
+/* Copy the final states of the last prefill/decode pass ([rows, D] fp32: s~_N of
+ * exited tokens, s_N of the rest) into d_out; rows = tokens of that pass. */
+ADEPT_API adept_status adept_read_final_states(adept_model* m, float* d_out, int rows, void* stream);
+
+/* Synchronise `stream`, then read and clear the device error word.
+ * Returns DEVICE_INPUT if a kernel flagged an invalid input, TIMEOUT if a bounded
+ * wait gave up, CUDA on an asynchronous CUDA error, else OK. */
+ADEPT_API adept_status adept_check_device_status(adept_model* m, void* stream);
+
+/* Options (ADEPT_OPT_*).  HSM_IDENTITY=1 replaces the HSM by s~ = s_i* (test switch).
+ * PROFILE=1 records CUDA events around every launch of the grouped GEMM so that
+ * adept_profile_read can report its launch count and total device time. */
+enum { ADEPT_OPT_HSM_IDENTITY = 1, ADEPT_OPT_PROFILE = 2, ADEPT_OPT_GEMM_SIMT = 3 };
+ADEPT_API adept_status adept_set_option(adept_model* m, int option, int value);
+
+/* Kernel classes reported by adept_profile_read. */
+enum { ADEPT_PROF_GEMM = 0, ADEPT_PROF_KV_FILL = 1, ADEPT_PROF_ATTENTION = 2, ADEPT_PROF_NCLASS = 3 };
+/* Synchronise, then return launches, total ms, and the algorithmic flop and byte
+ * counts summed over the recorded launches of kernel class `cls`; resets the record. */
+ADEPT_API adept_status adept_profile_read(adept_model* m, int cls, int64_t* launches, double* total_ms,
+                                double* flops, double* bytes);
+
+/* Number of kernel launches the library enqueued since the last call (then reset). */
+ADEPT_API int64_t adept_launch_count(adept_model* m);
+
+#ifdef __cplusplus
+}
+#endif
+#endif /* ADEPT_H */

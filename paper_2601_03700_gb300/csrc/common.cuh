@@ -1,0 +1,157 @@
+// Shared device-side definitions of the ADEPT GB300 library.
+#pragma once
+#include <cuda_runtime.h>
+#include <cuda_bf16.h>
+#include <stdint.h>
+
+typedef __nv_bfloat16 bf16;
+
+// Device error word bits (read by adept_check_device_status).
+enum : unsigned {
+  ERRW_FORCED = 1u,    // forced exit layer outside {0} U [2, N]
+  ERRW_TOKEN = 2u,     // token id outside [0, vocab)
+  ERRW_POS = 4u,       // position outside the sequence's reserved blocks / max_pos
+  ERRW_EXIT_LAYER = 8u,// exit layer outside [1, N] (skipped-layer fill input)
+  ERRW_TIMEOUT = 16u,  // a bounded device-side wait gave up
+  ERRW_CONFIG = 32u    // a kernel was launched with a shape it does not support
+};
+
+template <typename T> __device__ __forceinline__ float to_f(T x);
+template <> __device__ __forceinline__ float to_f<float>(float x) { return x; }
+template <> __device__ __forceinline__ float to_f<bf16>(bf16 x) { return __bfloat162float(x); }
+template <typename T> __device__ __forceinline__ T from_f(float x);
+template <> __device__ __forceinline__ float from_f<float>(float x) { return x; }
+template <> __device__ __forceinline__ bf16 from_f<bf16>(float x) { return __float2bfloat16_rn(x); }
+
+__device__ __forceinline__ float warp_sum(float v) {
+#pragma unroll
+  for (int o = 16; o; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+  return v;
+}
+__device__ __forceinline__ float warp_max(float v) {
+#pragma unroll
+  for (int o = 16; o; o >>= 1) v = fmaxf(v, __shfl_xor_sync(0xffffffffu, v, o));
+  return v;
+}
+
+// Block-wide sum for blockDim.x a multiple of 32 (<= 1024); `red` holds 32 floats.
+__device__ __forceinline__ float block_sum(float v, float* red) {
+  const int lane = threadIdx.x & 31, w = threadIdx.x >> 5, nw = blockDim.x >> 5;
+  v = warp_sum(v);
+  __syncthreads();
+  if (lane == 0) red[w] = v;
+  __syncthreads();
+  float t = (threadIdx.x < (unsigned)nw) ? red[threadIdx.x] : 0.f;
+  if (w == 0) t = warp_sum(t);
+  if (threadIdx.x == 0) red[0] = t;
+  __syncthreads();
+  float r = red[0];
+  return r;
+}
+
+__device__ __forceinline__ float gelu_erf_f(float x) { return 0.5f * x * (1.f + erff(x * 0.70710678118654752f)); }
+__device__ __forceinline__ float gelu_tanh_f(float x) {
+  return 0.5f * x * (1.f + tanhf(0.79788456080286536f * (x + 0.044715f * x * x * x)));
+}
+__device__ __forceinline__ float silu_f(float x) { return x / (1.f + expf(-x)); }
+
+enum Act : int { ACT_NONE = 0, ACT_GELU_ERF = 1, ACT_GELU_TANH = 2, ACT_TANH = 3 };
+__device__ __forceinline__ float apply_act(int act, float x) {
+  switch (act) {
+    case ACT_GELU_ERF: return gelu_erf_f(x);
+    case ACT_GELU_TANH: return gelu_tanh_f(x);
+    case ACT_TANH: return tanhf(x);
+    default: return x;
+  }
+}
+
+// Normalisation applied to a layer's attention input (norm gains / shifts are folded
+// into the following projection at load time, so only the standardisation remains).
+enum NormMode : int { NORM_RMS = 0, NORM_LN = 1, NORM_COPY = 2 };
+
+// Paged KV cache: pools [n_layers][n_blocks][n_kv_heads][block_tokens][head_dim] for K
+// and for V; a sequence's position p lives in block block_table[seq][p / block_tokens].
+struct KVCacheView {
+  void* k;
+  void* v;
+  const int* block_table;   // [max_batch][max_blocks_per_seq]
+  int max_blocks_per_seq;
+  int n_blocks;
+  int n_kv_heads;
+  int head_dim;
+  int block_tokens;
+  int max_batch;
+  __device__ __forceinline__ size_t offset(int layer0, int seq, int pos, int h) const {
+    const int blk = block_table[seq * max_blocks_per_seq + pos / block_tokens];
+    return ((((size_t)layer0 * n_blocks + blk) * n_kv_heads + h) * block_tokens + (pos % block_tokens)) *
+           (size_t)head_dim;
+  }
+  // Base offset (head 0, dim 0) of a position, or -1 when (seq, pos) has no reserved block.
+  __device__ __forceinline__ long long checked_base(int layer0, int seq, int pos) const {
+    if (seq < 0 || seq >= max_batch || pos < 0 || pos >= max_blocks_per_seq * block_tokens) return -1;
+    const int blk = block_table[seq * max_blocks_per_seq + pos / block_tokens];
+    if (blk < 0 || blk >= n_blocks) return -1;
+    return (long long)((((size_t)layer0 * n_blocks + blk) * n_kv_heads) * block_tokens + (pos % block_tokens)) *
+           head_dim;
+  }
+  // Distance between consecutive heads of one position.
+  __device__ __forceinline__ size_t head_stride() const { return (size_t)block_tokens * head_dim; }
+};
+
+// Row range of a GEMM operand, resolved on the device: rows [*begin, *end) of A (a
+// NULL begin means 0; a NULL end means `count`).
+struct DevRange {
+  const int* begin;
+  const int* end;
+  int count;
+  __device__ __forceinline__ int b() const { return begin ? *begin : 0; }
+  __device__ __forceinline__ int e() const { return end ? *end : count; }
+};
+
+enum EpiKind : int {
+  EPI_F32 = 0,     // out_f32 = acc + bias
+  EPI_ACT = 1,     // out_t = act(acc + bias) (and out_f32 if set)
+  EPI_RESID = 2,   // out_f32 = resid + acc + bias
+  EPI_SWIGLU = 3,  // columns interleaved in 16-blocks (gate, up): out_t = silu(g) * u
+  EPI_QKV = 4,     // q -> q_out (RoPE), k/v -> KV cache (RoPE on k)
+  EPI_KV = 5       // k/v only (skipped-layer fill) -> KV cache
+};
+
+// Epilogue description.  Output row r refers to GEMM row r (relative to the range
+// begin); for the cache epilogues its token is row_tok[begin + r].
+struct Epi {
+  int kind;
+  int act;
+  const float* bias;
+  float* out_f32;
+  int ld_f32;
+  const float* resid;
+  int ld_resid;
+  void* out_t;
+  int ld_t;
+  // QKV / KV
+  const int* row_tok;
+  const int* tok_seq;
+  const int* tok_pos;
+  KVCacheView cache;
+  int layer0;        // 0-based layer of the cache writes
+  int n_q_cols;      // D_q (0 for EPI_KV)
+  int n_kv_cols;     // D_kv
+  int head_dim;
+  int rope;          // apply RoPE to q and k
+  const float2* rope_table;   // [max_seq][head_dim/2] (cos, sin)
+};
+
+// One problem of a (grouped) GEMM: C[M, N] = A[M, K] * B[N, K]^T, both K-major.
+struct GemmProblem {
+  const void* A;
+  int lda;
+  const void* B;
+  int ldb;
+  DevRange rows;
+  int N;
+  int K;
+  Epi epi;
+};
+
+static inline int cdiv(int a, int b) { return (a + b - 1) / b; }

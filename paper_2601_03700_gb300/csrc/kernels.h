@@ -1,0 +1,59 @@
+// Host-side launchers of the library's kernels (all enqueue on the given stream).
+#pragma once
+#include "common.cuh"
+
+namespace adept {
+
+// Device counter word layout of one pass.
+enum : int {
+  CTR_ACTIVE = 0,    // [0], [1]: active rows, ping-pong by layer parity
+  CTR_EXITED = 2,    // exits so far in this pass
+  CTR_PREFIX = 3,    // [3 + i]: exits after layer i (i = 0..N)
+};
+static inline int ctr_words(int n_layers) { return CTR_PREFIX + n_layers + 2; }
+
+void launch_pass_init(cudaStream_t st, int n_tok, int prompt_len, int decode, int* tok_seq, int* tok_pos,
+                      int* row_tok, int* seq_len, int seq_cap, int max_pos, unsigned* err);
+void launch_embed(cudaStream_t st, int dt, const int* tokens, int n_tok, const int* tok_pos, const void* E,
+                  const void* P, const float* type_emb, const float* g, const float* b, int family, int D, int V,
+                  float eps, float* X, unsigned* err);
+void launch_standardize(cudaStream_t st, int dt, const float* X, int ldx, const int* in_rows, DevRange rows,
+                        int max_rows, int D, int mode, float eps, void* out, int ld_out);
+void launch_layernorm_inplace(cudaStream_t st, float* X, DevRange rows, int max_rows, int D, const float* g,
+                              const float* b, float eps);
+void launch_exit_decide(cudaStream_t st, const float* Xout, const float* I, int D, DevRange rows, int max_rows,
+                        const int* row_tok, const int* forced, int layer, int n_layers, float delta, int test,
+                        float* sim, int* flag, float* inv_norm, unsigned* err);
+void launch_exit_scan(cudaStream_t st, int* ctr, int in_parity, const int* flag, const int* row_tok,
+                      int* row_tok_next, int* exit_tok, int* dst, int* exit_layer_out, int layer);
+void launch_exit_move(cudaStream_t st, const float* Xin, const float* Xout, const float* I, int D, const int* n_rows,
+                      int max_rows, const int* dst, const float* inv_norm, float* Xnext, float* Inext, float* hsm_s,
+                      float* hsm_prev, float* hsm_I);
+void launch_final_scatter(cudaStream_t st, const float* X, int D, const int* n_rows, int max_rows, const int* row_tok,
+                          float* final_, int* exit_layer_out, int n_layers);
+void launch_hsm_prep(cudaStream_t st, int dt, const float* hs, const float* hp, const float* hI, DevRange rows,
+                     int max_rows, int D, const float* g0, const float* conv, float eps, float* c0f, void* c0t);
+void launch_hsm_mid(cudaStream_t st, int dt, const float* h3, const float* h1, DevRange rows, int max_rows, int m1,
+                    const float* g1, float eps, void* h4);
+void launch_hsm_out(cudaStream_t st, int dt, const float* h5, const float* c0f, const float* hs, int identity,
+                    DevRange rows, int max_rows, int D, const float* g2, float eps, const int* exit_tok,
+                    float* final_, void* xfill, int fill_mode, float norm_eps);
+void launch_argmax(cudaStream_t st, const float* logits, int V, int rows, int* out);
+void launch_head_rows(cudaStream_t st, int batch, int prompt_len, int last, int* rows);
+void launch_fill_sort(cudaStream_t st, int dt, const void* h, int n, int D, const int* exit_layer, int n_layers,
+                      int* hist, int* start, int* cursor, int* sorted_tok, void* xs, int mode, float eps,
+                      unsigned* err);
+void launch_fold_rows(cudaStream_t st, int dt, void* dst, int ld_dst, const void* src, int n_rows, int K,
+                      const float* gamma, const float* beta, const float* bias_in, float* bias_out, int row_mode);
+void launch_to_f32(cudaStream_t st, int dt, const void* src, float* dst, int n);
+void launch_read_kv(cudaStream_t st, int dt, KVCacheView c, int layer0, int seq, int pos0, int n_pos, void* ko,
+                    void* vo);
+
+// GEMMs.  SIMT path: C = A B^T into fp32 scratch, then the epilogue kernel.
+void launch_gemm_simt(cudaStream_t st, int dt, const GemmProblem& p, int max_rows, float* scratch);
+// Attention of the active query rows over the paged cache of one layer.
+void launch_attention(cudaStream_t st, int dt, const void* q, int ld_q, void* out, int ld_out, DevRange rows,
+                      int max_rows, const int* row_tok, const int* tok_seq, const int* tok_pos, const int* seq_len,
+                      KVCacheView cache, int layer0, int n_heads, int causal);
+
+}  // namespace adept

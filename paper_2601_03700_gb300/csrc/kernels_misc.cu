@@ -1,0 +1,637 @@
+// Row-wise kernels of the early-exit pass: embedding, norms, the exit test with
+// active-token compaction, the HSM's non-GEMM steps, argmax, skipped-layer-fill
+// bucketing and load-time weight repacking.
+#include "common.cuh"
+#include "kernels.h"
+
+#include <math.h>
+
+namespace adept {
+
+// ---------------------------------------------------------------------------
+// pass set-up: token -> (sequence, position), identity row map, counters
+// ---------------------------------------------------------------------------
+__global__ void pass_init_kernel(int n_tok, int prompt_len, int decode, int* tok_seq, int* tok_pos,
+                                 int* row_tok, int* seq_len, int seq_cap, int max_pos, unsigned* err) {
+  const int t = blockIdx.x * blockDim.x + threadIdx.x;
+  if (t >= n_tok) return;
+  int s, p;
+  if (decode) {
+    s = t;
+    p = seq_len[t];
+    seq_len[t] = p + 1;
+  } else {
+    s = t / prompt_len;
+    p = t % prompt_len;
+    if (p == 0) seq_len[s] = prompt_len;
+  }
+  if (p >= seq_cap || (max_pos > 0 && p >= max_pos)) {
+    atomicOr(err, ERRW_POS);
+    p = 0;
+  }
+  tok_seq[t] = s;
+  tok_pos[t] = p;
+  row_tok[t] = t;
+}
+
+// ---------------------------------------------------------------------------
+// embedding (s_0): token embedding (+ learned position) (+ type and LayerNorm for BERT)
+// ---------------------------------------------------------------------------
+template <typename T>
+__global__ void embed_kernel(const int* tokens, int n_tok, const int* tok_pos, const T* E, const T* P,
+                             const float* type_emb, const float* g, const float* b, int family, int D, int V,
+                             float eps, float* X, unsigned* err) {
+  __shared__ float red[32];
+  const int t = blockIdx.x;
+  if (t >= n_tok) return;
+  int tok = tokens[t];
+  if (tok < 0 || tok >= V) {
+    if (threadIdx.x == 0) atomicOr(err, ERRW_TOKEN);
+    tok = 0;
+  }
+  const int pos = tok_pos[t];
+  float* x = X + (size_t)t * D;
+  float s1 = 0.f;
+  for (int d = threadIdx.x; d < D; d += blockDim.x) {
+    float v = to_f(E[(size_t)tok * D + d]);
+    if (P) v += to_f(P[(size_t)pos * D + d]);
+    if (type_emb) v += type_emb[d];
+    x[d] = v;
+    s1 += v;
+  }
+  if (family != 2) return;
+  const float mu = block_sum(s1, red) / D;
+  float s2 = 0.f;
+  for (int d = threadIdx.x; d < D; d += blockDim.x) {
+    const float c = x[d] - mu;
+    s2 += c * c;
+  }
+  const float rstd = rsqrtf(block_sum(s2, red) / D + eps);
+  for (int d = threadIdx.x; d < D; d += blockDim.x) x[d] = (x[d] - mu) * rstd * g[d] + b[d];
+}
+
+// ---------------------------------------------------------------------------
+// standardisation of a layer input (gains folded into the next GEMM)
+// ---------------------------------------------------------------------------
+template <typename T>
+__global__ void standardize_kernel(const float* X, int ldx, const int* in_rows, DevRange rows, int D, int mode,
+                                   float eps, T* out, int ld_out) {
+  __shared__ float red[32];
+  const int r = rows.b() + blockIdx.x;
+  if (r >= rows.e()) return;
+  const int src = in_rows ? in_rows[r] : r;
+  const float* x = X + (size_t)src * ldx;
+  T* o = out + (size_t)r * ld_out;
+  if (mode == NORM_COPY) {
+    for (int d = threadIdx.x; d < D; d += blockDim.x) o[d] = from_f<T>(x[d]);
+    return;
+  }
+  float mu = 0.f;
+  if (mode == NORM_LN) {
+    float s = 0.f;
+    for (int d = threadIdx.x; d < D; d += blockDim.x) s += x[d];
+    mu = block_sum(s, red) / D;
+  }
+  float s2 = 0.f;
+  for (int d = threadIdx.x; d < D; d += blockDim.x) {
+    const float c = x[d] - mu;
+    s2 += c * c;
+  }
+  const float rstd = rsqrtf(block_sum(s2, red) / D + eps);
+  for (int d = threadIdx.x; d < D; d += blockDim.x) o[d] = from_f<T>((x[d] - mu) * rstd);
+}
+
+// In-place LayerNorm with gain and shift (the post-LN encoder's residual stream).
+__global__ void layernorm_inplace_kernel(float* X, DevRange rows, int D, const float* g, const float* b, float eps) {
+  __shared__ float red[32];
+  const int r = rows.b() + blockIdx.x;
+  if (r >= rows.e()) return;
+  float* x = X + (size_t)r * D;
+  float s = 0.f;
+  for (int d = threadIdx.x; d < D; d += blockDim.x) s += x[d];
+  const float mu = block_sum(s, red) / D;
+  float s2 = 0.f;
+  for (int d = threadIdx.x; d < D; d += blockDim.x) {
+    const float c = x[d] - mu;
+    s2 += c * c;
+  }
+  const float rstd = rsqrtf(block_sum(s2, red) / D + eps);
+  for (int d = threadIdx.x; d < D; d += blockDim.x) x[d] = (x[d] - mu) * rstd * g[d] + b[d];
+}
+
+// ---------------------------------------------------------------------------
+// exit test (Sec. 4.1): c = <s_i, I> / (|s_i| |I|) vs delta, or the forced layer
+// ---------------------------------------------------------------------------
+__global__ void exit_decide_kernel(const float* Xout, const float* I, int D, DevRange rows, const int* row_tok,
+                                   const int* forced, int layer, int n_layers, float delta, int test, float* sim,
+                                   int* flag, float* inv_norm, unsigned* err) {
+  const int warp = (blockIdx.x * blockDim.x + threadIdx.x) >> 5, lane = threadIdx.x & 31;
+  const int r = warp;
+  if (r >= rows.e()) return;
+  const float* s = Xout + (size_t)r * D;
+  const float* in = I + (size_t)r * D;
+  float ns = 0.f, ni = 0.f, dot = 0.f;
+  for (int d = lane; d < D; d += 32) {
+    const float a = s[d], c = in[d];
+    ns += a * a;
+    ni += c * c;
+    dot += a * c;
+  }
+  ns = warp_sum(ns);
+  ni = warp_sum(ni);
+  dot = warp_sum(dot);
+  if (lane != 0) return;
+  const int tok = row_tok[r];
+  int ex = 0;
+  if (test) {
+    const float c = (ns > 0.f && ni > 0.f) ? dot / sqrtf(ns * ni) : -INFINITY;
+    if (sim) sim[(size_t)tok * n_layers + (layer - 1)] = c;
+    const int f = forced ? forced[tok] : 0;
+    if (f != 0 && (f < 2 || f > n_layers)) atomicOr(err, ERRW_FORCED);
+    ex = (f > 0) ? (f == layer) : (c >= delta);
+  }
+  flag[r] = ex;
+  inv_norm[r] = ns > 0.f ? rsqrtf(ns) : 0.f;
+}
+
+// Single-CTA stable compaction of the active rows: survivors keep their order in the
+// next active list; exits are appended to the pass's exit list.  Counter layout:
+// ctr[CTR_ACTIVE + parity] active counts, ctr[CTR_EXITED] exits so far,
+// ctr[CTR_PREFIX + i] exits after layer i.
+__global__ void exit_scan_kernel(int* ctr, int in_parity, const int* flag, const int* row_tok, int* row_tok_next,
+                                 int* exit_tok, int* dst, int* exit_layer_out, int layer) {
+  __shared__ int s_stay[1024];
+  __shared__ int s_exit[1024];
+  const int n = ctr[CTR_ACTIVE + in_parity];
+  const int base = ctr[CTR_EXITED];
+  const int tid = threadIdx.x, nt = blockDim.x;
+  const int per = (n + nt - 1) / nt;
+  const int lo = min(n, tid * per), hi = min(n, lo + per);
+  int ce = 0;
+  for (int r = lo; r < hi; ++r) ce += flag[r];
+  s_exit[tid] = ce;
+  s_stay[tid] = (hi - lo) - ce;
+  __syncthreads();
+  for (int off = 1; off < nt; off <<= 1) {
+    int a = 0, b = 0;
+    if (tid >= off) {
+      a = s_exit[tid - off];
+      b = s_stay[tid - off];
+    }
+    __syncthreads();
+    s_exit[tid] += a;
+    s_stay[tid] += b;
+    __syncthreads();
+  }
+  int e = s_exit[tid] - ce;
+  int s = s_stay[tid] - ((hi - lo) - ce);
+  for (int r = lo; r < hi; ++r) {
+    const int tok = row_tok[r];
+    if (flag[r]) {
+      dst[r] = -1 - (base + e);
+      exit_tok[base + e] = tok;
+      if (exit_layer_out) exit_layer_out[tok] = layer;
+      ++e;
+    } else {
+      dst[r] = s;
+      row_tok_next[s] = tok;
+      ++s;
+    }
+  }
+  if (tid == nt - 1) {
+    const int E = s_exit[nt - 1];
+    ctr[CTR_ACTIVE + (in_parity ^ 1)] = s_stay[nt - 1];
+    ctr[CTR_EXITED] = base + E;
+    ctr[CTR_PREFIX + layer] = base + E;
+  }
+}
+
+// Moves each active row to its new place: survivors -> next layer input (s_i) and the
+// inertia with s_hat_i added (Sec. 4.1, after the test); exits -> the HSM input slots
+// (s_i, s_{i-1}, inertia before s_hat_i).
+__global__ void exit_move_kernel(const float* Xin, const float* Xout, const float* I, int D, const int* n_rows,
+                                 const int* dst, const float* inv_norm, float* Xnext, float* Inext, float* hsm_s,
+                                 float* hsm_prev, float* hsm_I) {
+  const int r = blockIdx.x;
+  if (r >= *n_rows) return;
+  const int d0 = dst[r];
+  const float* s = Xout + (size_t)r * D;
+  const float* in = I + (size_t)r * D;
+  if (d0 >= 0) {
+    const float w = inv_norm[r];
+    float* xn = Xnext + (size_t)d0 * D;
+    float* inn = Inext + (size_t)d0 * D;
+    for (int d = threadIdx.x; d < D; d += blockDim.x) {
+      const float v = s[d];
+      xn[d] = v;
+      inn[d] = in[d] + v * w;
+    }
+  } else {
+    const size_t k = (size_t)(-1 - d0);
+    const float* sp = Xin + (size_t)r * D;
+    for (int d = threadIdx.x; d < D; d += blockDim.x) {
+      hsm_s[k * D + d] = s[d];
+      hsm_prev[k * D + d] = sp[d];
+      hsm_I[k * D + d] = in[d];
+    }
+  }
+}
+
+// After layer N: the remaining active rows' s_N are their final states.
+__global__ void final_scatter_kernel(const float* X, int D, const int* n_rows, const int* row_tok, float* final_,
+                                     int* exit_layer_out, int n_layers) {
+  const int r = blockIdx.x;
+  if (r >= *n_rows) return;
+  const int tok = row_tok[r];
+  for (int d = threadIdx.x; d < D; d += blockDim.x) final_[(size_t)tok * D + d] = X[(size_t)r * D + d];
+  if (threadIdx.x == 0 && exit_layer_out) exit_layer_out[tok] = n_layers;
+}
+
+// ---------------------------------------------------------------------------
+// Hidden State Mapper, non-GEMM steps (Sec. 4.2, App. B Table S1)
+// ---------------------------------------------------------------------------
+// Three separately RMS-normalised rows (shared gain g0), then the 3x3 convolution with
+// padding (0, 1): c0[t] = b + sum_a sum_u w[a][u] x_a[t + u - 1].
+template <typename T>
+__global__ void hsm_prep_kernel(const float* hs, const float* hp, const float* hI, DevRange rows, int D,
+                                const float* g0, const float* conv /* 9 taps + bias */, float eps, float* c0f,
+                                T* c0t) {
+  __shared__ float red[32];
+  const int k = rows.b() + blockIdx.x;
+  if (k >= rows.e()) return;
+  const float* x[3] = {hs + (size_t)k * D, hp + (size_t)k * D, hI + (size_t)k * D};
+  float sc[3];
+#pragma unroll
+  for (int a = 0; a < 3; ++a) {
+    float s2 = 0.f;
+    for (int d = threadIdx.x; d < D; d += blockDim.x) s2 += x[a][d] * x[a][d];
+    sc[a] = rsqrtf(block_sum(s2, red) / D + eps);
+  }
+  for (int t = threadIdx.x; t < D; t += blockDim.x) {
+    float acc = conv[9];
+#pragma unroll
+    for (int a = 0; a < 3; ++a) {
+#pragma unroll
+      for (int u = 0; u < 3; ++u) {
+        const int tt = t + u - 1;
+        if (tt >= 0 && tt < D) acc += conv[a * 3 + u] * (x[a][tt] * sc[a] * g0[tt]);
+      }
+    }
+    c0f[(size_t)k * D + t] = acc;
+    c0t[(size_t)k * D + t] = from_f<T>(acc);
+  }
+}
+
+// h4 = RMSNorm_g1(h3) + h1 (the MLP's addition), rounded for FC4.
+template <typename T>
+__global__ void hsm_mid_kernel(const float* h3, const float* h1, DevRange rows, int m1, const float* g1, float eps,
+                               T* h4) {
+  __shared__ float red[32];
+  const int k = rows.b() + blockIdx.x;
+  if (k >= rows.e()) return;
+  const float* a = h3 + (size_t)k * m1;
+  float s2 = 0.f;
+  for (int d = threadIdx.x; d < m1; d += blockDim.x) s2 += a[d] * a[d];
+  const float sc = rsqrtf(block_sum(s2, red) / m1 + eps);
+  for (int d = threadIdx.x; d < m1; d += blockDim.x)
+    h4[(size_t)k * m1 + d] = from_f<T>(a[d] * sc * g1[d] + h1[(size_t)k * m1 + d]);
+}
+
+// s~ = RMSNorm_g2(h5) + c0 (the final addition); written to the token's final state,
+// and standardised (the attention-input normalisation of the family) for the fills.
+// identity != 0: s~ = s_i* (test switch replacing the HSM).
+template <typename T>
+__global__ void hsm_out_kernel(const float* h5, const float* c0f, const float* hs, int identity, DevRange rows, int D,
+                               const float* g2, float eps, const int* exit_tok, float* final_, T* xfill,
+                               int fill_mode, float norm_eps) {
+  __shared__ float red[32];
+  const int k = rows.b() + blockIdx.x;
+  if (k >= rows.e()) return;
+  const int tok = exit_tok[k];
+  float* f = final_ + (size_t)tok * D;
+  if (identity) {
+    for (int d = threadIdx.x; d < D; d += blockDim.x) f[d] = hs[(size_t)k * D + d];
+  } else {
+    const float* a = h5 + (size_t)k * D;
+    float s2 = 0.f;
+    for (int d = threadIdx.x; d < D; d += blockDim.x) s2 += a[d] * a[d];
+    const float sc = rsqrtf(block_sum(s2, red) / D + eps);
+    for (int d = threadIdx.x; d < D; d += blockDim.x) f[d] = a[d] * sc * g2[d] + c0f[(size_t)k * D + d];
+  }
+  __syncthreads();
+  T* o = xfill + (size_t)k * D;
+  if (fill_mode == NORM_COPY) {
+    for (int d = threadIdx.x; d < D; d += blockDim.x) o[d] = from_f<T>(f[d]);
+    return;
+  }
+  float mu = 0.f;
+  if (fill_mode == NORM_LN) {
+    float s = 0.f;
+    for (int d = threadIdx.x; d < D; d += blockDim.x) s += f[d];
+    mu = block_sum(s, red) / D;
+  }
+  float s2 = 0.f;
+  for (int d = threadIdx.x; d < D; d += blockDim.x) {
+    const float c = f[d] - mu;
+    s2 += c * c;
+  }
+  const float rstd = rsqrtf(block_sum(s2, red) / D + norm_eps);
+  for (int d = threadIdx.x; d < D; d += blockDim.x) o[d] = from_f<T>((f[d] - mu) * rstd);
+}
+
+// ---------------------------------------------------------------------------
+// greedy token: argmax with the lowest index on ties
+// ---------------------------------------------------------------------------
+__global__ void argmax_kernel(const float* logits, int V, int rows, int* out) {
+  __shared__ float sv[32];
+  __shared__ int si[32];
+  const int r = blockIdx.x;
+  if (r >= rows) return;
+  const float* l = logits + (size_t)r * V;
+  float bv = -INFINITY;
+  int bi = 0x7fffffff;
+  for (int v = threadIdx.x; v < V; v += blockDim.x) {
+    const float x = l[v];
+    if (x > bv || (x == bv && v < bi)) {
+      bv = x;
+      bi = v;
+    }
+  }
+#pragma unroll
+  for (int o = 16; o; o >>= 1) {
+    const float ov = __shfl_xor_sync(0xffffffffu, bv, o);
+    const int oi = __shfl_xor_sync(0xffffffffu, bi, o);
+    if (ov > bv || (ov == bv && oi < bi)) {
+      bv = ov;
+      bi = oi;
+    }
+  }
+  const int lane = threadIdx.x & 31, w = threadIdx.x >> 5;
+  if (lane == 0) {
+    sv[w] = bv;
+    si[w] = bi;
+  }
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    for (int k = 1; k < (int)(blockDim.x >> 5); ++k)
+      if (sv[k] > bv || (sv[k] == bv && si[k] < bi)) {
+        bv = sv[k];
+        bi = si[k];
+      }
+    out[r] = bi == 0x7fffffff ? 0 : bi;
+  }
+}
+
+// Rows of the last position of each sequence (decoder head) or of position 0 (encoder).
+__global__ void head_rows_kernel(int batch, int prompt_len, int last, int* rows) {
+  const int b = blockIdx.x * blockDim.x + threadIdx.x;
+  if (b < batch) rows[b] = b * prompt_len + (last ? prompt_len - 1 : 0);
+}
+
+// ---------------------------------------------------------------------------
+// skipped-layer fill input: bucket tokens by exit layer (ascending) so that the rows of
+// skipped layer r (tokens with i* < r) are a prefix, and standardise s~ once.
+// ---------------------------------------------------------------------------
+__global__ void fill_hist_kernel(const int* exit_layer, int n, int n_layers, int* hist, unsigned* err) {
+  const int j = blockIdx.x * blockDim.x + threadIdx.x;
+  if (j >= n) return;
+  int l = exit_layer[j];
+  if (l < 1 || l > n_layers) {
+    atomicOr(err, ERRW_EXIT_LAYER);
+    l = n_layers;
+  }
+  atomicAdd(&hist[l], 1);
+}
+
+// hist[1..N] -> start[l] (exclusive prefix) and prefix[r] = #(i* < r) = start[r].
+__global__ void fill_scan_kernel(const int* hist, int n_layers, int* start, int* cursor) {
+  if (threadIdx.x != 0 || blockIdx.x != 0) return;
+  int acc = 0;
+  for (int l = 0; l <= n_layers + 1; ++l) {
+    start[l] = acc;
+    cursor[l] = 0;
+    if (l >= 1 && l <= n_layers) acc += hist[l];
+  }
+}
+
+template <typename T>
+__global__ void fill_scatter_kernel(const T* h, int n, int D, const int* exit_layer, int n_layers, const int* start,
+                                    int* cursor, int* sorted_tok, T* xs, int mode, float eps) {
+  __shared__ float red[32];
+  __shared__ int s_slot;
+  const int j = blockIdx.x;
+  if (j >= n) return;
+  if (threadIdx.x == 0) {
+    int l = exit_layer[j];
+    if (l < 1 || l > n_layers) l = n_layers;
+    s_slot = start[l] + atomicAdd(&cursor[l], 1);
+    sorted_tok[s_slot] = j;
+  }
+  __syncthreads();
+  const int slot = s_slot;
+  const T* x = h + (size_t)j * D;
+  T* o = xs + (size_t)slot * D;
+  if (mode == NORM_COPY) {
+    for (int d = threadIdx.x; d < D; d += blockDim.x) o[d] = x[d];
+    return;
+  }
+  float mu = 0.f;
+  if (mode == NORM_LN) {
+    float s = 0.f;
+    for (int d = threadIdx.x; d < D; d += blockDim.x) s += to_f(x[d]);
+    mu = block_sum(s, red) / D;
+  }
+  float s2 = 0.f;
+  for (int d = threadIdx.x; d < D; d += blockDim.x) {
+    const float c = to_f(x[d]) - mu;
+    s2 += c * c;
+  }
+  const float rstd = rsqrtf(block_sum(s2, red) / D + eps);
+  for (int d = threadIdx.x; d < D; d += blockDim.x) o[d] = from_f<T>((to_f(x[d]) - mu) * rstd);
+}
+
+// ---------------------------------------------------------------------------
+// load-time repacking: W'[n, k] = W[src(n), k] * gamma[k] (rounded once),
+// b'[n] = b[src(n)] + sum_k W[src(n), k] * beta[k]
+// ---------------------------------------------------------------------------
+template <typename T>
+__global__ void fold_rows_kernel(T* dst, int ld_dst, const T* src, int n_rows, int K, const float* gamma,
+                                 const float* beta, const float* bias_in, float* bias_out, int row_mode) {
+  const int warp = (blockIdx.x * blockDim.x + threadIdx.x) >> 5, lane = threadIdx.x & 31;
+  if (warp >= n_rows) return;
+  const int n = warp;
+  // row_mode 0: dst row = n.  1 / 2: gate / up of a SwiGLU pair, interleaved in blocks of 16.
+  int drow = n;
+  if (row_mode == 1) drow = (n / 16) * 32 + (n % 16);
+  if (row_mode == 2) drow = (n / 16) * 32 + 16 + (n % 16);
+  const T* s = src + (size_t)n * K;
+  T* o = dst + (size_t)drow * ld_dst;
+  float acc = 0.f;
+  for (int k = lane; k < K; k += 32) {
+    const float w = to_f(s[k]);
+    o[k] = gamma ? from_f<T>(w * gamma[k]) : s[k];
+    if (beta) acc += w * beta[k];
+  }
+  acc = warp_sum(acc);
+  if (lane == 0 && bias_out) bias_out[drow] = (bias_in ? bias_in[n] : 0.f) + acc;
+}
+
+template <typename T>
+__global__ void to_f32_kernel(const T* src, float* dst, int n) {
+  const int i = blockIdx.x * blockDim.x + threadIdx.x;
+  if (i < n) dst[i] = to_f(src[i]);
+}
+
+// Copy n_pos positions of one sequence / layer out of the paged cache.
+template <typename T>
+__global__ void read_kv_kernel(KVCacheView c, int layer0, int seq, int pos0, int n_pos, T* ko, T* vo) {
+  const int p = blockIdx.x;
+  if (p >= n_pos) return;
+  const int per = c.n_kv_heads * c.head_dim;
+  for (int e = threadIdx.x; e < per; e += blockDim.x) {
+    const int h = e / c.head_dim, d = e % c.head_dim;
+    const size_t off = c.offset(layer0, seq, pos0 + p, h) + d;
+    ko[(size_t)p * per + e] = ((const T*)c.k)[off];
+    vo[(size_t)p * per + e] = ((const T*)c.v)[off];
+  }
+}
+
+// ---------------------------------------------------------------------------
+// launchers
+// ---------------------------------------------------------------------------
+void launch_pass_init(cudaStream_t st, int n_tok, int prompt_len, int decode, int* tok_seq, int* tok_pos,
+                      int* row_tok, int* seq_len, int seq_cap, int max_pos, unsigned* err) {
+  pass_init_kernel<<<cdiv(n_tok, 256), 256, 0, st>>>(n_tok, prompt_len, decode, tok_seq, tok_pos, row_tok, seq_len,
+                                                    seq_cap, max_pos, err);
+}
+
+void launch_embed(cudaStream_t st, int dt, const int* tokens, int n_tok, const int* tok_pos, const void* E,
+                  const void* P, const float* type_emb, const float* g, const float* b, int family, int D, int V,
+                  float eps, float* X, unsigned* err) {
+  if (dt == 1)
+    embed_kernel<bf16><<<n_tok, 256, 0, st>>>(tokens, n_tok, tok_pos, (const bf16*)E, (const bf16*)P, type_emb, g, b,
+                                              family, D, V, eps, X, err);
+  else
+    embed_kernel<float><<<n_tok, 256, 0, st>>>(tokens, n_tok, tok_pos, (const float*)E, (const float*)P, type_emb, g,
+                                               b, family, D, V, eps, X, err);
+}
+
+void launch_standardize(cudaStream_t st, int dt, const float* X, int ldx, const int* in_rows, DevRange rows,
+                        int max_rows, int D, int mode, float eps, void* out, int ld_out) {
+  if (max_rows <= 0) return;
+  if (dt == 1)
+    standardize_kernel<bf16><<<max_rows, 256, 0, st>>>(X, ldx, in_rows, rows, D, mode, eps, (bf16*)out, ld_out);
+  else
+    standardize_kernel<float><<<max_rows, 256, 0, st>>>(X, ldx, in_rows, rows, D, mode, eps, (float*)out, ld_out);
+}
+
+void launch_layernorm_inplace(cudaStream_t st, float* X, DevRange rows, int max_rows, int D, const float* g,
+                              const float* b, float eps) {
+  if (max_rows <= 0) return;
+  layernorm_inplace_kernel<<<max_rows, 256, 0, st>>>(X, rows, D, g, b, eps);
+}
+
+void launch_exit_decide(cudaStream_t st, const float* Xout, const float* I, int D, DevRange rows, int max_rows,
+                        const int* row_tok, const int* forced, int layer, int n_layers, float delta, int test,
+                        float* sim, int* flag, float* inv_norm, unsigned* err) {
+  if (max_rows <= 0) return;
+  exit_decide_kernel<<<cdiv(max_rows, 8), 256, 0, st>>>(Xout, I, D, rows, row_tok, forced, layer, n_layers, delta,
+                                                       test, sim, flag, inv_norm, err);
+}
+
+void launch_exit_scan(cudaStream_t st, int* ctr, int in_parity, const int* flag, const int* row_tok,
+                      int* row_tok_next, int* exit_tok, int* dst, int* exit_layer_out, int layer) {
+  exit_scan_kernel<<<1, 1024, 0, st>>>(ctr, in_parity, flag, row_tok, row_tok_next, exit_tok, dst, exit_layer_out,
+                                       layer);
+}
+
+void launch_exit_move(cudaStream_t st, const float* Xin, const float* Xout, const float* I, int D, const int* n_rows,
+                      int max_rows, const int* dst, const float* inv_norm, float* Xnext, float* Inext, float* hsm_s,
+                      float* hsm_prev, float* hsm_I) {
+  if (max_rows <= 0) return;
+  exit_move_kernel<<<max_rows, 256, 0, st>>>(Xin, Xout, I, D, n_rows, dst, inv_norm, Xnext, Inext, hsm_s, hsm_prev,
+                                             hsm_I);
+}
+
+void launch_final_scatter(cudaStream_t st, const float* X, int D, const int* n_rows, int max_rows, const int* row_tok,
+                          float* final_, int* exit_layer_out, int n_layers) {
+  if (max_rows <= 0) return;
+  final_scatter_kernel<<<max_rows, 256, 0, st>>>(X, D, n_rows, row_tok, final_, exit_layer_out, n_layers);
+}
+
+void launch_hsm_prep(cudaStream_t st, int dt, const float* hs, const float* hp, const float* hI, DevRange rows,
+                     int max_rows, int D, const float* g0, const float* conv, float eps, float* c0f, void* c0t) {
+  if (max_rows <= 0) return;
+  if (dt == 1)
+    hsm_prep_kernel<bf16><<<max_rows, 256, 0, st>>>(hs, hp, hI, rows, D, g0, conv, eps, c0f, (bf16*)c0t);
+  else
+    hsm_prep_kernel<float><<<max_rows, 256, 0, st>>>(hs, hp, hI, rows, D, g0, conv, eps, c0f, (float*)c0t);
+}
+
+void launch_hsm_mid(cudaStream_t st, int dt, const float* h3, const float* h1, DevRange rows, int max_rows, int m1,
+                    const float* g1, float eps, void* h4) {
+  if (max_rows <= 0) return;
+  if (dt == 1) hsm_mid_kernel<bf16><<<max_rows, 256, 0, st>>>(h3, h1, rows, m1, g1, eps, (bf16*)h4);
+  else hsm_mid_kernel<float><<<max_rows, 256, 0, st>>>(h3, h1, rows, m1, g1, eps, (float*)h4);
+}
+
+void launch_hsm_out(cudaStream_t st, int dt, const float* h5, const float* c0f, const float* hs, int identity,
+                    DevRange rows, int max_rows, int D, const float* g2, float eps, const int* exit_tok,
+                    float* final_, void* xfill, int fill_mode, float norm_eps) {
+  if (max_rows <= 0) return;
+  if (dt == 1)
+    hsm_out_kernel<bf16><<<max_rows, 256, 0, st>>>(h5, c0f, hs, identity, rows, D, g2, eps, exit_tok, final_,
+                                                   (bf16*)xfill, fill_mode, norm_eps);
+  else
+    hsm_out_kernel<float><<<max_rows, 256, 0, st>>>(h5, c0f, hs, identity, rows, D, g2, eps, exit_tok, final_,
+                                                    (float*)xfill, fill_mode, norm_eps);
+}
+
+void launch_argmax(cudaStream_t st, const float* logits, int V, int rows, int* out) {
+  if (rows <= 0) return;
+  argmax_kernel<<<rows, 256, 0, st>>>(logits, V, rows, out);
+}
+
+void launch_head_rows(cudaStream_t st, int batch, int prompt_len, int last, int* rows) {
+  head_rows_kernel<<<cdiv(batch, 128), 128, 0, st>>>(batch, prompt_len, last, rows);
+}
+
+void launch_fill_sort(cudaStream_t st, int dt, const void* h, int n, int D, const int* exit_layer, int n_layers,
+                      int* hist, int* start, int* cursor, int* sorted_tok, void* xs, int mode, float eps,
+                      unsigned* err) {
+  cudaMemsetAsync(hist, 0, sizeof(int) * (n_layers + 2), st);
+  if (n > 0) fill_hist_kernel<<<cdiv(n, 256), 256, 0, st>>>(exit_layer, n, n_layers, hist, err);
+  fill_scan_kernel<<<1, 32, 0, st>>>(hist, n_layers, start, cursor);
+  if (n <= 0) return;
+  if (dt == 1)
+    fill_scatter_kernel<bf16><<<n, 256, 0, st>>>((const bf16*)h, n, D, exit_layer, n_layers, start, cursor,
+                                                 sorted_tok, (bf16*)xs, mode, eps);
+  else
+    fill_scatter_kernel<float><<<n, 256, 0, st>>>((const float*)h, n, D, exit_layer, n_layers, start, cursor,
+                                                  sorted_tok, (float*)xs, mode, eps);
+}
+
+void launch_fold_rows(cudaStream_t st, int dt, void* dst, int ld_dst, const void* src, int n_rows, int K,
+                      const float* gamma, const float* beta, const float* bias_in, float* bias_out, int row_mode) {
+  if (dt == 1)
+    fold_rows_kernel<bf16><<<cdiv(n_rows, 8), 256, 0, st>>>((bf16*)dst, ld_dst, (const bf16*)src, n_rows, K, gamma,
+                                                            beta, bias_in, bias_out, row_mode);
+  else
+    fold_rows_kernel<float><<<cdiv(n_rows, 8), 256, 0, st>>>((float*)dst, ld_dst, (const float*)src, n_rows, K,
+                                                             gamma, beta, bias_in, bias_out, row_mode);
+}
+
+void launch_to_f32(cudaStream_t st, int dt, const void* src, float* dst, int n) {
+  if (n <= 0) return;
+  if (dt == 1) to_f32_kernel<bf16><<<cdiv(n, 256), 256, 0, st>>>((const bf16*)src, dst, n);
+  else to_f32_kernel<float><<<cdiv(n, 256), 256, 0, st>>>((const float*)src, dst, n);
+}
+
+void launch_read_kv(cudaStream_t st, int dt, KVCacheView c, int layer0, int seq, int pos0, int n_pos, void* ko,
+                    void* vo) {
+  if (n_pos <= 0) return;
+  if (dt == 1) read_kv_kernel<bf16><<<n_pos, 256, 0, st>>>(c, layer0, seq, pos0, n_pos, (bf16*)ko, (bf16*)vo);
+  else read_kv_kernel<float><<<n_pos, 256, 0, st>>>(c, layer0, seq, pos0, n_pos, (float*)ko, (float*)vo);
+}
+
+}  // namespace adept

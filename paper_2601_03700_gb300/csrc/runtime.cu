@@ -1,0 +1,1035 @@
+// Host runtime of the ADEPT library: model loading and weight repacking, the paged KV
+// pool, the early-exit layer loop of prefill / decode, the skipped-layer fill entry
+// point, and the C ABI of include/adept.h.
+#include "adept.h"
+#include "common.cuh"
+#include "kernels.h"
+#include "gemm_tc.h"
+
+#include <algorithm>
+#include <cmath>
+#include <cstdarg>
+#include <cstdio>
+#include <cstring>
+#include <random>
+#include <string>
+#include <unordered_map>
+#include <vector>
+
+using namespace adept;
+
+namespace {
+thread_local std::string g_load_error;
+}
+
+struct LayerW {
+  void* w_qkv = nullptr;  // [D_q + 2 D_kv, D]: Q rows, then K rows, then V rows (input-norm gain folded in)
+  float* b_qkv = nullptr;
+  void* w_o = nullptr;    // [D, D_q]
+  float* b_o = nullptr;
+  void* w_up = nullptr;   // LLAMA: [2F, D] gate/up interleaved by 16 rows; else [F, D]
+  float* b_up = nullptr;
+  int up_rows = 0;
+  void* w_down = nullptr; // [D, F]
+  float* b_down = nullptr;
+  float *ln1_g = nullptr, *ln1_b = nullptr, *ln2_g = nullptr, *ln2_b = nullptr;  // post-LN (encoder)
+};
+
+struct ProfRec {
+  std::vector<std::pair<cudaEvent_t, cudaEvent_t>> ev;
+  std::vector<std::pair<double, double>> work;  // (flops, bytes) per recorded launch
+};
+
+struct adept_model {
+  adept_config cfg{};
+  int N = 0, D = 0, H = 0, Hkv = 0, dh = 0, Dq = 0, Dkv = 0, F = 0, V = 0, m1 = 0, m2 = 0, dt = 0;
+  size_t esz = 4;
+  std::vector<void*> allocs;
+  std::string err;
+  // weights
+  void* tok_emb = nullptr;
+  void* pos_emb = nullptr;
+  float* type_emb = nullptr;
+  float *emb_g = nullptr, *emb_b = nullptr;
+  std::vector<LayerW> L;
+  void* w_head = nullptr;
+  float* b_head = nullptr;
+  void *w_pool = nullptr, *w_cls = nullptr;
+  float *b_pool = nullptr, *b_cls = nullptr;
+  float *hsm_g0 = nullptr, *hsm_conv = nullptr, *hsm_g1 = nullptr, *hsm_g2 = nullptr;
+  float *hsm_b1 = nullptr, *hsm_b2 = nullptr, *hsm_b3 = nullptr, *hsm_b4 = nullptr;
+  void *hsm_w1 = nullptr, *hsm_w2 = nullptr, *hsm_w3 = nullptr, *hsm_w4 = nullptr;
+  float2* rope_table = nullptr;
+  // paged KV cache
+  void *k_pool = nullptr, *v_pool = nullptr;
+  int n_blocks = 0, max_blocks_per_seq = 0;
+  int* d_block_table = nullptr;
+  std::vector<int> h_block_table, free_list, h_seq_len;
+  std::vector<std::vector<int>> seq_blocks;
+  int* d_seq_len = nullptr;
+  // pass workspaces (T_max rows)
+  int T_max = 0;
+  float *X_in[2] = {nullptr, nullptr}, *X_out = nullptr, *I[2] = {nullptr, nullptr};
+  int *row_tok[2] = {nullptr, nullptr}, *tok_seq = nullptr, *tok_pos = nullptr, *flag = nullptr, *dst = nullptr;
+  float* inv_norm = nullptr;
+  float *hsm_s = nullptr, *hsm_prev = nullptr, *hsm_I = nullptr;
+  int* exit_tok = nullptr;
+  void *xn = nullptr, *q = nullptr, *att = nullptr, *hbuf = nullptr, *xfill = nullptr;
+  float *c0f = nullptr, *h1f = nullptr, *h3f = nullptr, *h5f = nullptr;
+  void *c0t = nullptr, *h1t = nullptr, *h2t = nullptr, *h4t = nullptr;
+  float* final_ = nullptr;
+  int* ctr = nullptr;
+  unsigned* err_word = nullptr;
+  int* head_rows = nullptr;
+  void* xhead = nullptr;
+  void* pool_t = nullptr;
+  float* logits_ws = nullptr;
+  float* scratch = nullptr;
+  size_t scratch_elems = 0;
+  // skipped-layer fill workspace (adept_skip_kv_fill)
+  int fill_cap = 0;
+  void* fill_x = nullptr;
+  int *fill_tok = nullptr, *fill_hist = nullptr, *fill_start = nullptr, *fill_cursor = nullptr;
+  // options / instrumentation
+  int hsm_identity = 0, profile = 0, force_simt = 0;
+  int last_rows = 0;
+  int64_t launches = 0;
+  ProfRec prof[ADEPT_PROF_NCLASS];
+};
+
+// ---------------------------------------------------------------------------
+// small helpers
+// ---------------------------------------------------------------------------
+static adept_status fail(adept_model* m, adept_status s, const char* fmt, ...) {
+  char buf[512];
+  va_list ap;
+  va_start(ap, fmt);
+  vsnprintf(buf, sizeof buf, fmt, ap);
+  va_end(ap);
+  if (m) m->err = buf;
+  else g_load_error = buf;
+  return s;
+}
+
+#define CUDA_TRY(m, call)                                                                               \
+  do {                                                                                                  \
+    cudaError_t e_ = (call);                                                                            \
+    if (e_ != cudaSuccess) return fail(m, ADEPT_ERR_CUDA, "%s failed: %s", #call, cudaGetErrorString(e_)); \
+  } while (0)
+
+static adept_status dalloc(adept_model* m, void** p, size_t bytes) {
+  *p = nullptr;
+  if (bytes == 0) return ADEPT_OK;
+  cudaError_t e = cudaMalloc(p, bytes);
+  if (e != cudaSuccess) {
+    cudaGetLastError();
+    *p = nullptr;
+    return fail(m, ADEPT_ERR_OOM, "cudaMalloc(%zu) failed: %s", bytes, cudaGetErrorString(e));
+  }
+  m->allocs.push_back(*p);
+  return ADEPT_OK;
+}
+
+template <typename P>
+static adept_status dalloc_t(adept_model* m, P** p, size_t count, size_t esz = sizeof(P)) {
+  return dalloc(m, (void**)p, count * esz);
+}
+
+#define TRY(x)                        \
+  do {                                \
+    adept_status s_ = (x);            \
+    if (s_ != ADEPT_OK) return s_;    \
+  } while (0)
+
+static void free_all(adept_model* m) {
+  for (void* p : m->allocs) cudaFree(p);
+  m->allocs.clear();
+  for (auto& pr : m->prof)
+    for (auto& e : pr.ev) {
+      cudaEventDestroy(e.first);
+      cudaEventDestroy(e.second);
+    }
+}
+
+static int attn_norm_mode(const adept_model* m) {
+  return m->cfg.family == ADEPT_FAMILY_LLAMA ? NORM_RMS : (m->cfg.family == ADEPT_FAMILY_GPT2 ? NORM_LN : NORM_COPY);
+}
+
+static KVCacheView cache_view(const adept_model* m) {
+  KVCacheView c;
+  c.k = m->k_pool;
+  c.v = m->v_pool;
+  c.block_table = m->d_block_table;
+  c.max_blocks_per_seq = m->max_blocks_per_seq;
+  c.n_blocks = m->n_blocks;
+  c.n_kv_heads = m->Hkv;
+  c.head_dim = m->dh;
+  c.block_tokens = m->cfg.kv_block_tokens;
+  c.max_batch = m->cfg.max_batch;
+  return c;
+}
+
+static Epi epi_base() {
+  Epi e;
+  memset(&e, 0, sizeof e);
+  return e;
+}
+
+// ---------------------------------------------------------------------------
+// GEMM dispatch: tcgen05 grouped GEMM for bf16 models, SIMT otherwise.
+// ---------------------------------------------------------------------------
+static void prof_begin(adept_model* m, int cls, cudaStream_t st, cudaEvent_t* b) {
+  if (!m->profile) return;
+  cudaEventCreate(b);
+  cudaEventRecord(*b, st);
+  (void)cls;
+}
+static void prof_end(adept_model* m, int cls, cudaStream_t st, cudaEvent_t b, double flops, double bytes) {
+  if (!m->profile) return;
+  cudaEvent_t e;
+  cudaEventCreate(&e);
+  cudaEventRecord(e, st);
+  m->prof[cls].ev.push_back({b, e});
+  m->prof[cls].work.push_back({flops, bytes});
+}
+
+static void gemm(adept_model* m, cudaStream_t st, const GemmProblem* probs, int n_probs, const int* max_rows,
+                 int cls, double flops = 0, double bytes = 0) {
+  cudaEvent_t b = nullptr;
+  prof_begin(m, cls, st, &b);
+  if (m->dt == ADEPT_DTYPE_BF16 && !m->force_simt && tc_gemm_supported()) {
+    m->launches += tc_gemm_grouped(st, probs, n_probs, max_rows, m->err_word);
+  } else {
+    for (int i = 0; i < n_probs; ++i) {
+      launch_gemm_simt(st, m->dt, probs[i], max_rows[i], m->scratch);
+      m->launches += 2;
+    }
+  }
+  prof_end(m, cls, st, b, flops, bytes);
+}
+
+// ---------------------------------------------------------------------------
+// loading
+// ---------------------------------------------------------------------------
+struct Loader {
+  adept_model* m;
+  std::unordered_map<std::string, adept_tensor> t;
+  void* staging = nullptr;
+  size_t staging_bytes = 0;
+  float* fstage[2] = {nullptr, nullptr};
+  size_t fstage_n = 0;
+  cudaStream_t st;
+
+  adept_status find(const std::string& name, int64_t numel, const void** out) {
+    auto it = t.find(name);
+    if (it == t.end()) return fail(m, ADEPT_ERR_INVALID_ARG, "weight '%s' missing", name.c_str());
+    if (it->second.numel != numel)
+      return fail(m, ADEPT_ERR_INVALID_ARG, "weight '%s' has %lld elements, expected %lld", name.c_str(),
+                  (long long)it->second.numel, (long long)numel);
+    if (!it->second.data) return fail(m, ADEPT_ERR_INVALID_ARG, "weight '%s' has a NULL pointer", name.c_str());
+    *out = it->second.data;
+    return ADEPT_OK;
+  }
+  bool has(const std::string& name) const { return t.count(name) != 0; }
+
+  // Model-dtype tensor copied verbatim into new device memory.
+  adept_status upload(const std::string& name, int64_t numel, void** out) {
+    const void* src;
+    TRY(find(name, numel, &src));
+    TRY(dalloc(m, out, numel * m->esz));
+    CUDA_TRY(m, cudaMemcpyAsync(*out, src, numel * m->esz, cudaMemcpyDefault, st));
+    return ADEPT_OK;
+  }
+  // Model-dtype tensor into the staging buffer (device).
+  adept_status stage(const std::string& name, int64_t numel, const void** out) {
+    const void* src;
+    TRY(find(name, numel, &src));
+    CUDA_TRY(m, cudaMemcpyAsync(staging, src, numel * m->esz, cudaMemcpyDefault, st));
+    *out = staging;
+    return ADEPT_OK;
+  }
+  // Vector converted to fp32 in new device memory (or into `dst` if given).
+  adept_status vec_f32(const std::string& name, int64_t n, float** out) {
+    const void* src;
+    TRY(stage(name, n, &src));
+    TRY(dalloc_t(m, out, n));
+    launch_to_f32(st, m->dt, src, *out, (int)n);
+    CUDA_TRY(m, cudaStreamSynchronize(st));
+    return ADEPT_OK;
+  }
+  adept_status vec_f32_opt(const std::string& name, int64_t n, float** out) {
+    if (!has(name)) {
+      TRY(dalloc_t(m, out, n));
+      CUDA_TRY(m, cudaMemsetAsync(*out, 0, n * sizeof(float), st));
+      return ADEPT_OK;
+    }
+    return vec_f32(name, n, out);
+  }
+  // fp32 copy of a vector into a reusable slot (gains / shifts used only while folding).
+  adept_status tmp_f32(const std::string& name, int64_t n, int slot, float** out) {
+    const void* src;
+    TRY(stage(name, n, &src));
+    launch_to_f32(st, m->dt, src, fstage[slot], (int)n);
+    CUDA_TRY(m, cudaStreamSynchronize(st));
+    *out = fstage[slot];
+    return ADEPT_OK;
+  }
+  // rows of `name` ([n_rows, K]) folded with gain/shift into dst (ld K) at row offset.
+  adept_status fold(const std::string& name, int n_rows, int K, void* dst, int row_off, const float* gamma,
+                    const float* beta, const float* bias_in, float* bias_out, int row_mode = 0) {
+    const void* src;
+    TRY(stage(name, (int64_t)n_rows * K, &src));
+    launch_fold_rows(st, m->dt, (char*)dst + (size_t)row_off * K * m->esz, K, src, n_rows, K, gamma, beta, bias_in,
+                     bias_out ? bias_out + row_off : nullptr, row_mode);
+    CUDA_TRY(m, cudaStreamSynchronize(st));
+    return ADEPT_OK;
+  }
+};
+
+static adept_status validate_cfg(adept_config* c) {
+  if (c->n_kv_heads == 0) c->n_kv_heads = c->n_heads;
+  if (c->family < 0 || c->family > 2) return fail(nullptr, ADEPT_ERR_INVALID_ARG, "family %d unknown", c->family);
+  if (c->dtype != ADEPT_DTYPE_F32 && c->dtype != ADEPT_DTYPE_BF16)
+    return fail(nullptr, ADEPT_ERR_INVALID_ARG, "dtype %d unknown", c->dtype);
+  if (c->n_layers < 1 || c->d_model < 1 || c->n_heads < 1 || c->d_ffn < 1 || c->vocab < 1)
+    return fail(nullptr, ADEPT_ERR_INVALID_ARG, "non-positive model size");
+  if (c->head_dim != 32 && c->head_dim != 64 && c->head_dim != 128)
+    return fail(nullptr, ADEPT_ERR_INVALID_ARG, "head_dim %d unsupported (32, 64 or 128)", c->head_dim);
+  if (c->n_heads % c->n_kv_heads) return fail(nullptr, ADEPT_ERR_INVALID_ARG, "n_heads %% n_kv_heads != 0");
+  if (c->d_model % 8 || c->d_ffn % 16 || c->hsm_m1 % 8 || c->hsm_m2 % 8)
+    return fail(nullptr, ADEPT_ERR_INVALID_ARG, "d_model, hsm widths must be multiples of 8 and d_ffn of 16");
+  if (c->hsm_m1 < 1 || c->hsm_m2 < 1) return fail(nullptr, ADEPT_ERR_INVALID_ARG, "HSM widths must be positive");
+  if (c->max_batch < 1 || c->max_seq < 1 || c->kv_block_tokens < 1)
+    return fail(nullptr, ADEPT_ERR_INVALID_ARG, "max_batch, max_seq, kv_block_tokens must be positive");
+  if (c->family != ADEPT_FAMILY_LLAMA && c->max_pos < c->max_seq)
+    return fail(nullptr, ADEPT_ERR_INVALID_ARG, "max_pos must cover max_seq for learned positions");
+  if (c->family == ADEPT_FAMILY_BERT && c->n_classes < 1)
+    return fail(nullptr, ADEPT_ERR_INVALID_ARG, "encoder needs n_classes >= 1");
+  if ((long long)c->max_batch * c->max_seq > (1LL << 26))
+    return fail(nullptr, ADEPT_ERR_INVALID_ARG, "max_batch * max_seq too large");
+  return ADEPT_OK;
+}
+
+static adept_status load_weights(adept_model* m, Loader& ld) {
+  const adept_config& c = m->cfg;
+  const int D = m->D, F = m->F, V = m->V, Dq = m->Dq, Dkv = m->Dkv, m1 = m->m1, m2 = m->m2;
+  const int fam = c.family;
+  // staging sized for the largest single tensor
+  size_t big = (size_t)V * D;
+  big = std::max(big, (size_t)F * D);
+  big = std::max(big, (size_t)m1 * m2);
+  big = std::max(big, (size_t)std::max(m1, D) * std::max(m1, D));
+  big = std::max(big, (size_t)Dq * D);
+  if (fam != ADEPT_FAMILY_LLAMA) big = std::max(big, (size_t)c.max_pos * D);
+  TRY(dalloc(m, &ld.staging, big * m->esz));
+  ld.fstage_n = std::max<size_t>(std::max(D, m1), 16);
+  TRY(dalloc_t(m, &ld.fstage[0], ld.fstage_n));
+  TRY(dalloc_t(m, &ld.fstage[1], ld.fstage_n));
+
+  TRY(ld.upload("tok_emb", (int64_t)V * D, &m->tok_emb));
+  if (fam != ADEPT_FAMILY_LLAMA) TRY(ld.upload("pos_emb", (int64_t)c.max_pos * D, &m->pos_emb));
+  if (fam == ADEPT_FAMILY_BERT) {
+    TRY(ld.vec_f32("type_emb", D, &m->type_emb));
+    TRY(ld.vec_f32("emb_ln.g", D, &m->emb_g));
+    TRY(ld.vec_f32("emb_ln.b", D, &m->emb_b));
+  }
+  m->L.resize(m->N);
+  const int nqkv = Dq + 2 * Dkv;
+  for (int l = 0; l < m->N; ++l) {
+    LayerW& w = m->L[l];
+    const std::string p = "layers." + std::to_string(l) + ".";
+    TRY(dalloc(m, &w.w_qkv, (size_t)nqkv * D * m->esz));
+    TRY(dalloc_t(m, &w.b_qkv, nqkv));
+    float *g = nullptr, *b = nullptr, *bin = nullptr;
+    if (fam == ADEPT_FAMILY_LLAMA) {
+      TRY(ld.tmp_f32(p + "attn_norm.g", D, 0, &g));
+    } else if (fam == ADEPT_FAMILY_GPT2) {
+      TRY(ld.tmp_f32(p + "attn_norm.g", D, 0, &g));
+      TRY(ld.tmp_f32(p + "attn_norm.b", D, 1, &b));
+    }
+    const char* qn[3] = {"wq", "wk", "wv"};
+    const char* bn[3] = {"bq", "bk", "bv"};
+    const int rows[3] = {Dq, Dkv, Dkv};
+    int off = 0;
+    for (int k = 0; k < 3; ++k) {
+      bin = nullptr;
+      float* btmp = nullptr;
+      if (fam != ADEPT_FAMILY_LLAMA) {
+        TRY(dalloc_t(m, &btmp, rows[k]));
+        const void* src;
+        TRY(ld.find(p + bn[k], rows[k], &src));
+        // biases go through the second fp32 slot only after the shift was consumed; use a private buffer
+        CUDA_TRY(m, cudaMemcpyAsync(ld.staging, src, rows[k] * m->esz, cudaMemcpyDefault, ld.st));
+        launch_to_f32(ld.st, m->dt, ld.staging, btmp, rows[k]);
+        CUDA_TRY(m, cudaStreamSynchronize(ld.st));
+        bin = btmp;
+      }
+      TRY(ld.fold(p + qn[k], rows[k], D, w.w_qkv, off, g, b, bin, w.b_qkv));
+      off += rows[k];
+    }
+    TRY(ld.upload(p + "wo", (int64_t)D * Dq, &w.w_o));
+    TRY(ld.vec_f32_opt(p + "bo", D, &w.b_o));
+    float *g2 = nullptr, *b2 = nullptr;
+    if (fam == ADEPT_FAMILY_LLAMA) {
+      TRY(ld.tmp_f32(p + "ffn_norm.g", D, 0, &g2));
+      w.up_rows = 2 * F;
+      TRY(dalloc(m, &w.w_up, (size_t)2 * F * D * m->esz));
+      TRY(dalloc_t(m, &w.b_up, 2 * F));
+      TRY(ld.fold(p + "w_gate", F, D, w.w_up, 0, g2, nullptr, nullptr, w.b_up, 1));
+      TRY(ld.fold(p + "w_up", F, D, w.w_up, 0, g2, nullptr, nullptr, w.b_up, 2));
+      TRY(ld.upload(p + "w_down", (int64_t)D * F, &w.w_down));
+      TRY(ld.vec_f32_opt(p + "b_down_absent", D, &w.b_down));
+    } else {
+      w.up_rows = F;
+      TRY(dalloc(m, &w.w_up, (size_t)F * D * m->esz));
+      TRY(dalloc_t(m, &w.b_up, F));
+      float* bfc = nullptr;
+      TRY(ld.vec_f32(p + "b_fc", F, &bfc));
+      if (fam == ADEPT_FAMILY_GPT2) {
+        TRY(ld.tmp_f32(p + "ffn_norm.g", D, 0, &g2));
+        TRY(ld.tmp_f32(p + "ffn_norm.b", D, 1, &b2));
+      }
+      TRY(ld.fold(p + "w_fc", F, D, w.w_up, 0, g2, b2, bfc, w.b_up));
+      TRY(ld.upload(p + "w_proj", (int64_t)D * F, &w.w_down));
+      TRY(ld.vec_f32(p + "b_proj", D, &w.b_down));
+      if (fam == ADEPT_FAMILY_BERT) {
+        TRY(ld.vec_f32(p + "attn_norm.g", D, &w.ln1_g));
+        TRY(ld.vec_f32(p + "attn_norm.b", D, &w.ln1_b));
+        TRY(ld.vec_f32(p + "ffn_norm.g", D, &w.ln2_g));
+        TRY(ld.vec_f32(p + "ffn_norm.b", D, &w.ln2_b));
+      }
+    }
+  }
+  // output heads (final norm gain / shift folded into the head)
+  if (fam == ADEPT_FAMILY_LLAMA) {
+    float* g = nullptr;
+    TRY(ld.tmp_f32("final_norm.g", D, 0, &g));
+    TRY(dalloc(m, &m->w_head, (size_t)V * D * m->esz));
+    TRY(dalloc_t(m, &m->b_head, V));
+    TRY(ld.fold("lm_head", V, D, m->w_head, 0, g, nullptr, nullptr, m->b_head));
+  } else if (fam == ADEPT_FAMILY_GPT2) {
+    float *g = nullptr, *b = nullptr;
+    TRY(ld.tmp_f32("final_norm.g", D, 0, &g));
+    TRY(ld.tmp_f32("final_norm.b", D, 1, &b));
+    TRY(dalloc(m, &m->w_head, (size_t)V * D * m->esz));
+    TRY(dalloc_t(m, &m->b_head, V));
+    TRY(ld.fold("tok_emb", V, D, m->w_head, 0, g, b, nullptr, m->b_head));
+  } else {
+    TRY(ld.upload("pool.w", (int64_t)D * D, &m->w_pool));
+    TRY(ld.vec_f32("pool.b", D, &m->b_pool));
+    TRY(ld.upload("cls.w", (int64_t)c.n_classes * D, &m->w_cls));
+    TRY(ld.vec_f32("cls.b", c.n_classes, &m->b_cls));
+  }
+  // Hidden State Mapper (App. B Table S1)
+  TRY(ld.vec_f32("hsm.g0", D, &m->hsm_g0));
+  TRY(dalloc_t(m, &m->hsm_conv, 10));
+  {
+    const void* src;
+    TRY(ld.stage("hsm.conv_w", 9, &src));
+    launch_to_f32(ld.st, m->dt, src, m->hsm_conv, 9);
+    CUDA_TRY(m, cudaStreamSynchronize(ld.st));
+    TRY(ld.stage("hsm.conv_b", 1, &src));
+    launch_to_f32(ld.st, m->dt, src, m->hsm_conv + 9, 1);
+    CUDA_TRY(m, cudaStreamSynchronize(ld.st));
+  }
+  TRY(ld.upload("hsm.fc1_w", (int64_t)m1 * D, &m->hsm_w1));
+  TRY(ld.vec_f32("hsm.fc1_b", m1, &m->hsm_b1));
+  TRY(ld.upload("hsm.fc2_w", (int64_t)m2 * m1, &m->hsm_w2));
+  TRY(ld.vec_f32("hsm.fc2_b", m2, &m->hsm_b2));
+  TRY(ld.upload("hsm.fc3_w", (int64_t)m1 * m2, &m->hsm_w3));
+  TRY(ld.vec_f32("hsm.fc3_b", m1, &m->hsm_b3));
+  TRY(ld.vec_f32("hsm.g1", m1, &m->hsm_g1));
+  TRY(ld.upload("hsm.fc4_w", (int64_t)D * m1, &m->hsm_w4));
+  TRY(ld.vec_f32("hsm.fc4_b", D, &m->hsm_b4));
+  TRY(ld.vec_f32("hsm.g2", D, &m->hsm_g2));
+  CUDA_TRY(m, cudaStreamSynchronize(ld.st));
+  return ADEPT_OK;
+}
+
+static adept_status alloc_runtime(adept_model* m) {
+  const adept_config& c = m->cfg;
+  const int D = m->D, T = m->T_max;
+  // RoPE table (cos, sin) per position and pair, evaluated in double once.
+  if (c.family == ADEPT_FAMILY_LLAMA) {
+    const int half = m->dh / 2;
+    std::vector<float2> tab((size_t)c.max_seq * half);
+    for (int p = 0; p < c.max_seq; ++p)
+      for (int i = 0; i < half; ++i) {
+        const double inv = std::pow((double)c.rope_theta, -2.0 * i / m->dh);
+        const double a = p * inv;
+        tab[(size_t)p * half + i] = make_float2((float)std::cos(a), (float)std::sin(a));
+      }
+    TRY(dalloc_t(m, &m->rope_table, tab.size()));
+    CUDA_TRY(m, cudaMemcpy(m->rope_table, tab.data(), tab.size() * sizeof(float2), cudaMemcpyHostToDevice));
+  }
+  // paged KV pool
+  m->max_blocks_per_seq = cdiv(c.max_seq, c.kv_block_tokens);
+  m->n_blocks = c.kv_pool_blocks > 0 ? c.kv_pool_blocks : c.max_batch * m->max_blocks_per_seq;
+  const size_t per_layer = (size_t)m->n_blocks * m->Hkv * c.kv_block_tokens * m->dh;
+  TRY(dalloc(m, &m->k_pool, per_layer * m->N * m->esz));
+  TRY(dalloc(m, &m->v_pool, per_layer * m->N * m->esz));
+  m->h_block_table.assign((size_t)c.max_batch * m->max_blocks_per_seq, -1);
+  TRY(dalloc_t(m, &m->d_block_table, m->h_block_table.size()));
+  CUDA_TRY(m, cudaMemcpy(m->d_block_table, m->h_block_table.data(), m->h_block_table.size() * sizeof(int),
+                         cudaMemcpyHostToDevice));
+  m->free_list.resize(m->n_blocks);
+  for (int i = 0; i < m->n_blocks; ++i) m->free_list[i] = m->n_blocks - 1 - i;  // pop_back hands out 0, 1, ...
+  if (c.block_shuffle_seed) {
+    std::mt19937_64 rng(c.block_shuffle_seed);
+    std::shuffle(m->free_list.begin(), m->free_list.end(), rng);
+  }
+  m->seq_blocks.assign(c.max_batch, {});
+  m->h_seq_len.assign(c.max_batch, 0);
+  TRY(dalloc_t(m, &m->d_seq_len, c.max_batch));
+  CUDA_TRY(m, cudaMemset(m->d_seq_len, 0, c.max_batch * sizeof(int)));
+  // pass workspaces
+  const size_t TD = (size_t)T * D;
+  for (int k = 0; k < 2; ++k) {
+    TRY(dalloc_t(m, &m->X_in[k], TD));
+    TRY(dalloc_t(m, &m->I[k], TD));
+    TRY(dalloc_t(m, &m->row_tok[k], T));
+  }
+  TRY(dalloc_t(m, &m->X_out, TD));
+  TRY(dalloc_t(m, &m->tok_seq, T));
+  TRY(dalloc_t(m, &m->tok_pos, T));
+  TRY(dalloc_t(m, &m->flag, T));
+  TRY(dalloc_t(m, &m->dst, T));
+  TRY(dalloc_t(m, &m->inv_norm, T));
+  TRY(dalloc_t(m, &m->hsm_s, TD));
+  TRY(dalloc_t(m, &m->hsm_prev, TD));
+  TRY(dalloc_t(m, &m->hsm_I, TD));
+  TRY(dalloc_t(m, &m->exit_tok, T));
+  TRY(dalloc_t(m, &m->final_, TD));
+  TRY(dalloc(m, &m->xn, TD * m->esz));
+  TRY(dalloc(m, &m->q, (size_t)T * m->Dq * m->esz));
+  TRY(dalloc(m, &m->att, (size_t)T * m->Dq * m->esz));
+  TRY(dalloc(m, &m->hbuf, (size_t)T * m->F * m->esz));
+  TRY(dalloc(m, &m->xfill, TD * m->esz));
+  TRY(dalloc_t(m, &m->c0f, TD));
+  TRY(dalloc(m, &m->c0t, TD * m->esz));
+  TRY(dalloc_t(m, &m->h1f, (size_t)T * m->m1));
+  TRY(dalloc(m, &m->h1t, (size_t)T * m->m1 * m->esz));
+  TRY(dalloc(m, &m->h2t, (size_t)T * m->m2 * m->esz));
+  TRY(dalloc_t(m, &m->h3f, (size_t)T * m->m1));
+  TRY(dalloc(m, &m->h4t, (size_t)T * m->m1 * m->esz));
+  TRY(dalloc_t(m, &m->h5f, TD));
+  TRY(dalloc_t(m, &m->ctr, ctr_words(m->N)));
+  TRY(dalloc_t(m, &m->err_word, 1));
+  CUDA_TRY(m, cudaMemset(m->err_word, 0, sizeof(unsigned)));
+  TRY(dalloc_t(m, &m->head_rows, c.max_batch));
+  TRY(dalloc(m, &m->xhead, (size_t)c.max_batch * D * m->esz));
+  TRY(dalloc(m, &m->pool_t, (size_t)c.max_batch * D * m->esz));
+  const int nout = c.family == ADEPT_FAMILY_BERT ? c.n_classes : m->V;
+  TRY(dalloc_t(m, &m->logits_ws, (size_t)c.max_batch * nout));
+  // SIMT scratch: the widest GEMM output of any pass step
+  size_t w = std::max({(size_t)m->Dq + 2 * m->Dkv, (size_t)m->L[0].up_rows, (size_t)m->m1, (size_t)m->m2, (size_t)D});
+  m->scratch_elems = std::max(w * T, (size_t)c.max_batch * nout);
+  TRY(dalloc_t(m, &m->scratch, m->scratch_elems));
+  return ADEPT_OK;
+}
+
+// ---------------------------------------------------------------------------
+// sequences and KV blocks
+// ---------------------------------------------------------------------------
+static adept_status reserve_seqs(adept_model* m, int batch, const int* lens, cudaStream_t st) {
+  const adept_config& c = m->cfg;
+  for (int b = 0; b < batch; ++b) {
+    for (int blk : m->seq_blocks[b]) m->free_list.push_back(blk);
+    m->seq_blocks[b].clear();
+    for (int k = 0; k < m->max_blocks_per_seq; ++k) m->h_block_table[(size_t)b * m->max_blocks_per_seq + k] = -1;
+  }
+  for (int b = 0; b < batch; ++b) {
+    const int need = m->max_blocks_per_seq;
+    if ((int)m->free_list.size() < need)
+      return fail(m, ADEPT_ERR_CAPACITY, "KV block pool exhausted (%d free, %d needed)", (int)m->free_list.size(), need);
+    for (int k = 0; k < need; ++k) {
+      const int blk = m->free_list.back();
+      m->free_list.pop_back();
+      m->seq_blocks[b].push_back(blk);
+      m->h_block_table[(size_t)b * m->max_blocks_per_seq + k] = blk;
+    }
+    m->h_seq_len[b] = lens[b];
+  }
+  CUDA_TRY(m, cudaMemcpyAsync(m->d_block_table, m->h_block_table.data(),
+                              (size_t)batch * m->max_blocks_per_seq * sizeof(int), cudaMemcpyHostToDevice, st));
+  CUDA_TRY(m, cudaMemcpyAsync(m->d_seq_len, m->h_seq_len.data(), batch * sizeof(int), cudaMemcpyHostToDevice, st));
+  (void)c;
+  return ADEPT_OK;
+}
+
+// ---------------------------------------------------------------------------
+// the early-exit pass
+// ---------------------------------------------------------------------------
+__global__ void set_int_kernel(int* p, int v) { *p = v; }
+
+static void run_hsm(adept_model* m, cudaStream_t st, DevRange rows, int max_rows) {
+  const int D = m->D, m1 = m->m1, m2 = m->m2;
+  const float eps = m->cfg.hsm_eps;
+  if (m->hsm_identity) {
+    launch_hsm_out(st, m->dt, nullptr, nullptr, m->hsm_s, 1, rows, max_rows, D, m->hsm_g2, eps, m->exit_tok,
+                   m->final_, m->xfill, attn_norm_mode(m), m->cfg.norm_eps);
+    m->launches += 1;
+    return;
+  }
+  launch_hsm_prep(st, m->dt, m->hsm_s, m->hsm_prev, m->hsm_I, rows, max_rows, D, m->hsm_g0, m->hsm_conv, eps, m->c0f,
+                  m->c0t);
+  m->launches += 1;
+  GemmProblem p;
+  memset(&p, 0, sizeof p);
+  p.rows = rows;
+  // FC1: h1 = GELU(W1 c0 + b1)
+  p.A = m->c0t; p.lda = D; p.B = m->hsm_w1; p.ldb = D; p.N = m1; p.K = D;
+  p.epi = epi_base(); p.epi.kind = EPI_ACT; p.epi.act = ACT_GELU_ERF; p.epi.bias = m->hsm_b1;
+  p.epi.out_t = m->h1t; p.epi.ld_t = m1; p.epi.out_f32 = m->h1f; p.epi.ld_f32 = m1;
+  gemm(m, st, &p, 1, &max_rows, ADEPT_PROF_GEMM);
+  // FC2: h2 = GELU(W2 h1 + b2)
+  p.A = m->h1t; p.lda = m1; p.B = m->hsm_w2; p.ldb = m1; p.N = m2; p.K = m1;
+  p.epi = epi_base(); p.epi.kind = EPI_ACT; p.epi.act = ACT_GELU_ERF; p.epi.bias = m->hsm_b2;
+  p.epi.out_t = m->h2t; p.epi.ld_t = m2;
+  gemm(m, st, &p, 1, &max_rows, ADEPT_PROF_GEMM);
+  // FC3: h3 = W3 h2 + b3
+  p.A = m->h2t; p.lda = m2; p.B = m->hsm_w3; p.ldb = m2; p.N = m1; p.K = m2;
+  p.epi = epi_base(); p.epi.kind = EPI_F32; p.epi.bias = m->hsm_b3; p.epi.out_f32 = m->h3f; p.epi.ld_f32 = m1;
+  gemm(m, st, &p, 1, &max_rows, ADEPT_PROF_GEMM);
+  launch_hsm_mid(st, m->dt, m->h3f, m->h1f, rows, max_rows, m1, m->hsm_g1, eps, m->h4t);
+  m->launches += 1;
+  // FC4: h5 = W4 h4 + b4
+  p.A = m->h4t; p.lda = m1; p.B = m->hsm_w4; p.ldb = m1; p.N = D; p.K = m1;
+  p.epi = epi_base(); p.epi.kind = EPI_F32; p.epi.bias = m->hsm_b4; p.epi.out_f32 = m->h5f; p.epi.ld_f32 = D;
+  gemm(m, st, &p, 1, &max_rows, ADEPT_PROF_GEMM);
+  launch_hsm_out(st, m->dt, m->h5f, m->c0f, m->hsm_s, 0, rows, max_rows, D, m->hsm_g2, eps, m->exit_tok, m->final_,
+                 m->xfill, attn_norm_mode(m), m->cfg.norm_eps);
+  m->launches += 1;
+}
+
+// KV-only projection problem of layer `layer0` for the rows of `xs` (K-major x~ rows).
+static GemmProblem kv_problem(adept_model* m, int layer0, const void* xs, DevRange rows, const int* row_tok,
+                              const int* tok_seq, const int* tok_pos) {
+  GemmProblem p;
+  memset(&p, 0, sizeof p);
+  const LayerW& w = m->L[layer0];
+  p.A = xs; p.lda = m->D;
+  p.B = (const char*)w.w_qkv + (size_t)m->Dq * m->D * m->esz; p.ldb = m->D;
+  p.rows = rows; p.N = 2 * m->Dkv; p.K = m->D;
+  p.epi = epi_base();
+  p.epi.kind = EPI_KV; p.epi.bias = w.b_qkv + m->Dq;
+  p.epi.row_tok = row_tok; p.epi.tok_seq = tok_seq; p.epi.tok_pos = tok_pos;
+  p.epi.cache = cache_view(m); p.epi.layer0 = layer0;
+  p.epi.n_q_cols = 0; p.epi.n_kv_cols = m->Dkv; p.epi.head_dim = m->dh;
+  p.epi.rope = m->cfg.family == ADEPT_FAMILY_LLAMA; p.epi.rope_table = m->rope_table;
+  return p;
+}
+
+static adept_status run_pass(adept_model* m, int n_tok, int batch, int prompt_len, bool decode, const int32_t* tokens,
+                             float delta, const int32_t* forced, int32_t* exit_out, float* sim_out, cudaStream_t st) {
+  const adept_config& c = m->cfg;
+  const int N = m->N, D = m->D, Dq = m->Dq, Dkv = m->Dkv;
+  const int fam = c.family;
+  const int amode = attn_norm_mode(m);
+  const float eps = c.norm_eps;
+  m->last_rows = n_tok;
+  if (sim_out) CUDA_TRY(m, cudaMemsetAsync(sim_out, 0xff, (size_t)n_tok * N * sizeof(float), st));  // NaN
+  CUDA_TRY(m, cudaMemsetAsync(m->ctr, 0, ctr_words(N) * sizeof(int), st));
+  set_int_kernel<<<1, 1, 0, st>>>(m->ctr + CTR_ACTIVE, n_tok);
+  launch_pass_init(st, n_tok, prompt_len, decode ? 1 : 0, m->tok_seq, m->tok_pos, m->row_tok[0], m->d_seq_len,
+                   m->max_blocks_per_seq * c.kv_block_tokens, fam == ADEPT_FAMILY_LLAMA ? 0 : c.max_pos,
+                   m->err_word);
+  launch_embed(st, m->dt, tokens, n_tok, m->tok_pos, m->tok_emb, m->pos_emb, m->type_emb, m->emb_g, m->emb_b, fam, D,
+               m->V, eps, m->X_in[0], m->err_word);
+  m->launches += 3;
+  const KVCacheView cv = cache_view(m);
+  const int causal = fam != ADEPT_FAMILY_BERT;
+  int par = 0;
+  for (int i = 1; i <= N; ++i) {
+    const int l0 = i - 1;
+    const LayerW& w = m->L[l0];
+    const DevRange act{nullptr, m->ctr + CTR_ACTIVE + par, 0};
+    float* Xi = m->X_in[par];
+    float* Ii = m->I[par];
+    int* rt = m->row_tok[par];
+    const int mr = n_tok;
+    // attention input (standardised; gain folded into W_qkv)
+    launch_standardize(st, m->dt, Xi, D, nullptr, act, mr, D, amode, eps, m->xn, D);
+    m->launches += 1;
+    // QKV of the active rows, and (prefill) layer i's K/V of every token that exited
+    // before layer i, from its mapped state (Sec. 4.3), in one grouped launch.
+    GemmProblem pr[2];
+    int mrs[2] = {mr, mr};
+    memset(pr, 0, sizeof pr);
+    pr[0].A = m->xn; pr[0].lda = D; pr[0].B = w.w_qkv; pr[0].ldb = D; pr[0].rows = act;
+    pr[0].N = Dq + 2 * Dkv; pr[0].K = D;
+    pr[0].epi = epi_base();
+    pr[0].epi.kind = EPI_QKV; pr[0].epi.bias = w.b_qkv; pr[0].epi.out_t = m->q; pr[0].epi.ld_t = Dq;
+    pr[0].epi.row_tok = rt; pr[0].epi.tok_seq = m->tok_seq; pr[0].epi.tok_pos = m->tok_pos;
+    pr[0].epi.cache = cv; pr[0].epi.layer0 = l0; pr[0].epi.n_q_cols = Dq; pr[0].epi.n_kv_cols = Dkv;
+    pr[0].epi.head_dim = m->dh; pr[0].epi.rope = fam == ADEPT_FAMILY_LLAMA; pr[0].epi.rope_table = m->rope_table;
+    int np = 1;
+    if (!decode && i >= 3) {
+      pr[1] = kv_problem(m, l0, m->xfill, DevRange{nullptr, m->ctr + CTR_EXITED, 0}, m->exit_tok, m->tok_seq,
+                         m->tok_pos);
+      np = 2;
+    }
+    gemm(m, st, pr, np, mrs, ADEPT_PROF_GEMM);
+    // attention over every cached position of layer i
+    launch_attention(st, m->dt, m->q, Dq, m->att, Dq, act, mr, rt, m->tok_seq, m->tok_pos, m->d_seq_len, cv, l0, m->H,
+                     causal);
+    m->launches += 1;
+    // O projection + residual
+    GemmProblem p;
+    memset(&p, 0, sizeof p);
+    p.A = m->att; p.lda = Dq; p.B = w.w_o; p.ldb = Dq; p.rows = act; p.N = D; p.K = Dq;
+    p.epi = epi_base(); p.epi.kind = EPI_RESID; p.epi.bias = w.b_o; p.epi.out_f32 = m->X_out; p.epi.ld_f32 = D;
+    p.epi.resid = Xi; p.epi.ld_resid = D;
+    gemm(m, st, &p, 1, &mr, ADEPT_PROF_GEMM);
+    if (fam == ADEPT_FAMILY_BERT) {
+      launch_layernorm_inplace(st, m->X_out, act, mr, D, w.ln1_g, w.ln1_b, eps);
+      m->launches += 1;
+    }
+    // FFN
+    launch_standardize(st, m->dt, m->X_out, D, nullptr, act, mr, D, amode, eps, m->xn, D);
+    m->launches += 1;
+    p.A = m->xn; p.lda = D; p.B = w.w_up; p.ldb = D; p.N = w.up_rows; p.K = D;
+    p.epi = epi_base();
+    if (fam == ADEPT_FAMILY_LLAMA) {
+      p.epi.kind = EPI_SWIGLU;
+    } else {
+      p.epi.kind = EPI_ACT;
+      p.epi.act = fam == ADEPT_FAMILY_GPT2 ? ACT_GELU_TANH : ACT_GELU_ERF;
+    }
+    p.epi.bias = w.b_up; p.epi.out_t = m->hbuf; p.epi.ld_t = m->F;
+    gemm(m, st, &p, 1, &mr, ADEPT_PROF_GEMM);
+    p.A = m->hbuf; p.lda = m->F; p.B = w.w_down; p.ldb = m->F; p.N = D; p.K = m->F;
+    p.epi = epi_base(); p.epi.kind = EPI_RESID; p.epi.bias = w.b_down; p.epi.out_f32 = m->X_out; p.epi.ld_f32 = D;
+    p.epi.resid = m->X_out; p.epi.ld_resid = D;
+    gemm(m, st, &p, 1, &mr, ADEPT_PROF_GEMM);
+    if (fam == ADEPT_FAMILY_BERT) {
+      launch_layernorm_inplace(st, m->X_out, act, mr, D, w.ln2_g, w.ln2_b, eps);
+      m->launches += 1;
+    }
+    if (i < N) {
+      // exit test (Sec. 4.1) for 2 <= i <= N-1, inertia update, compaction (App. H)
+      const int test = i >= 2;
+      launch_exit_decide(st, m->X_out, Ii, D, act, mr, rt, forced, i, N, delta, test, sim_out, m->flag, m->inv_norm,
+                         m->err_word);
+      launch_exit_scan(st, m->ctr, par, m->flag, rt, m->row_tok[par ^ 1], m->exit_tok, m->dst, exit_out, i);
+      launch_exit_move(st, Xi, m->X_out, Ii, D, m->ctr + CTR_ACTIVE + par, mr, m->dst, m->inv_norm, m->X_in[par ^ 1],
+                       m->I[par ^ 1], m->hsm_s, m->hsm_prev, m->hsm_I);
+      m->launches += 3;
+      if (!decode && test) {
+        // HSM of the tokens that left at layer i (Sec. 4.2); their s~_N feeds the fills
+        run_hsm(m, st, DevRange{m->ctr + CTR_PREFIX + i - 1, m->ctr + CTR_PREFIX + i, 0}, mr);
+      }
+      par ^= 1;
+    } else {
+      launch_final_scatter(st, m->X_out, D, m->ctr + CTR_ACTIVE + par, mr, rt, m->final_, exit_out, N);
+      m->launches += 1;
+    }
+  }
+  if (decode && N >= 3) {
+    // Generation step: the step's tokens belong to different sequences, so the HSM and
+    // the skipped-layer fills of all exits run once, after the layer loop: one HSM over
+    // every exited token, then one grouped launch over (skipped layer r) groups; rows are
+    // in exit-layer order, so layer r's rows (i* < r) are a prefix.
+    run_hsm(m, st, DevRange{nullptr, m->ctr + CTR_EXITED, 0}, n_tok);
+    std::vector<GemmProblem> probs;
+    std::vector<int> mrs;
+    for (int r = 3; r <= N; ++r) {
+      probs.push_back(kv_problem(m, r - 1, m->xfill, DevRange{nullptr, m->ctr + CTR_PREFIX + r - 1, 0}, m->exit_tok,
+                                 m->tok_seq, m->tok_pos));
+      mrs.push_back(n_tok);
+    }
+    gemm(m, st, probs.data(), (int)probs.size(), mrs.data(), ADEPT_PROF_KV_FILL);
+  }
+  return ADEPT_OK;
+}
+
+static adept_status run_head(adept_model* m, int batch, int prompt_len, bool decode, float* logits, int32_t* next,
+                             cudaStream_t st) {
+  const adept_config& c = m->cfg;
+  const int D = m->D;
+  const bool enc = c.family == ADEPT_FAMILY_BERT;
+  float* out = logits ? logits : m->logits_ws;
+  launch_head_rows(st, batch, decode ? 1 : prompt_len, enc ? 0 : 1, m->head_rows);
+  m->launches += 1;
+  const DevRange rows{nullptr, nullptr, batch};
+  GemmProblem p;
+  memset(&p, 0, sizeof p);
+  if (!enc) {
+    launch_standardize(st, m->dt, m->final_, D, m->head_rows, rows, batch, D, attn_norm_mode(m), c.norm_eps, m->xhead,
+                       D);
+    m->launches += 1;
+    p.A = m->xhead; p.lda = D; p.B = m->w_head; p.ldb = D; p.rows = rows; p.N = m->V; p.K = D;
+    p.epi = epi_base(); p.epi.kind = EPI_F32; p.epi.bias = m->b_head; p.epi.out_f32 = out; p.epi.ld_f32 = m->V;
+    gemm(m, st, &p, 1, &batch, ADEPT_PROF_GEMM);
+    if (next) {
+      launch_argmax(st, out, m->V, batch, next);
+      m->launches += 1;
+    }
+  } else {
+    launch_standardize(st, m->dt, m->final_, D, m->head_rows, rows, batch, D, NORM_COPY, c.norm_eps, m->xhead, D);
+    m->launches += 1;
+    p.A = m->xhead; p.lda = D; p.B = m->w_pool; p.ldb = D; p.rows = rows; p.N = D; p.K = D;
+    p.epi = epi_base(); p.epi.kind = EPI_ACT; p.epi.act = ACT_TANH; p.epi.bias = m->b_pool; p.epi.out_t = m->pool_t;
+    p.epi.ld_t = D;
+    gemm(m, st, &p, 1, &batch, ADEPT_PROF_GEMM);
+    p.A = m->pool_t; p.lda = D; p.B = m->w_cls; p.ldb = D; p.N = c.n_classes; p.K = D;
+    p.epi = epi_base(); p.epi.kind = EPI_F32; p.epi.bias = m->b_cls; p.epi.out_f32 = out; p.epi.ld_f32 = c.n_classes;
+    gemm(m, st, &p, 1, &batch, ADEPT_PROF_GEMM);
+    if (next) {
+      launch_argmax(st, out, c.n_classes, batch, next);
+      m->launches += 1;
+    }
+  }
+  return ADEPT_OK;
+}
+
+static adept_status check_launch(adept_model* m) {
+  cudaError_t e = cudaGetLastError();
+  if (e != cudaSuccess) return fail(m, ADEPT_ERR_CUDA, "kernel launch failed: %s", cudaGetErrorString(e));
+  return ADEPT_OK;
+}
+
+// ---------------------------------------------------------------------------
+// C ABI
+// ---------------------------------------------------------------------------
+extern "C" {
+
+const char* adept_status_string(adept_status s) {
+  switch (s) {
+    case ADEPT_OK: return "ok";
+    case ADEPT_ERR_INVALID_ARG: return "invalid argument";
+    case ADEPT_ERR_OOM: return "out of device memory";
+    case ADEPT_ERR_CAPACITY: return "capacity exceeded";
+    case ADEPT_ERR_CUDA: return "CUDA error";
+    case ADEPT_ERR_TIMEOUT: return "device wait timed out";
+    case ADEPT_ERR_DEVICE_INPUT: return "invalid device-side input";
+  }
+  return "unknown status";
+}
+
+const char* adept_last_error(const adept_model* m) { return m ? m->err.c_str() : g_load_error.c_str(); }
+
+adept_status adept_model_load(const adept_config* cfg_in, const adept_tensor_table* weights, void* stream,
+                              adept_model** out) {
+  g_load_error.clear();
+  if (!cfg_in || !weights || !out) return fail(nullptr, ADEPT_ERR_INVALID_ARG, "NULL argument");
+  *out = nullptr;
+  adept_config cfg = *cfg_in;
+  TRY(validate_cfg(&cfg));
+  if (weights->n_tensors < 0 || (weights->n_tensors > 0 && !weights->tensors))
+    return fail(nullptr, ADEPT_ERR_INVALID_ARG, "bad tensor table");
+  adept_model* m = new adept_model();
+  m->cfg = cfg;
+  m->N = cfg.n_layers; m->D = cfg.d_model; m->H = cfg.n_heads; m->Hkv = cfg.n_kv_heads; m->dh = cfg.head_dim;
+  m->Dq = m->H * m->dh; m->Dkv = m->Hkv * m->dh; m->F = cfg.d_ffn; m->V = cfg.vocab;
+  m->m1 = cfg.hsm_m1; m->m2 = cfg.hsm_m2; m->dt = cfg.dtype; m->esz = cfg.dtype == ADEPT_DTYPE_BF16 ? 2 : 4;
+  m->T_max = cfg.max_batch * cfg.max_seq;
+  Loader ld;
+  ld.m = m;
+  ld.st = (cudaStream_t)stream;
+  for (int i = 0; i < weights->n_tensors; ++i) {
+    const adept_tensor& t = weights->tensors[i];
+    if (!t.name) {
+      free_all(m);
+      delete m;
+      return fail(nullptr, ADEPT_ERR_INVALID_ARG, "tensor %d has no name", i);
+    }
+    ld.t[t.name] = t;
+  }
+  adept_status s = load_weights(m, ld);
+  if (s == ADEPT_OK) s = alloc_runtime(m);
+  if (s == ADEPT_OK) {
+    cudaError_t e = cudaStreamSynchronize(ld.st);
+    if (e != cudaSuccess) s = fail(m, ADEPT_ERR_CUDA, "load: %s", cudaGetErrorString(e));
+  }
+  if (s != ADEPT_OK) {
+    g_load_error = m->err;
+    free_all(m);
+    delete m;
+    return s;
+  }
+  // the staging buffers are not needed after loading
+  for (auto it = m->allocs.begin(); it != m->allocs.end();) {
+    if (*it == ld.staging || *it == ld.fstage[0] || *it == ld.fstage[1]) {
+      cudaFree(*it);
+      it = m->allocs.erase(it);
+    } else {
+      ++it;
+    }
+  }
+  *out = m;
+  return ADEPT_OK;
+}
+
+void adept_free(adept_model* m) {
+  if (!m) return;
+  cudaDeviceSynchronize();
+  free_all(m);
+  delete m;
+}
+
+adept_status adept_prefill(adept_model* m, int batch, int prompt_len, const int32_t* d_tokens, float delta,
+                           const int32_t* d_forced_exit, int32_t* d_exit_layer_out, float* d_logits_out,
+                           int32_t* d_next_token_out, float* d_sim_out, void* stream) {
+  if (!m) return ADEPT_ERR_INVALID_ARG;
+  if (!d_tokens) return fail(m, ADEPT_ERR_INVALID_ARG, "d_tokens is NULL");
+  if (batch < 1 || prompt_len < 1) return fail(m, ADEPT_ERR_INVALID_ARG, "batch and prompt_len must be positive");
+  if (batch > m->cfg.max_batch) return fail(m, ADEPT_ERR_CAPACITY, "batch %d > max_batch %d", batch, m->cfg.max_batch);
+  if (prompt_len > m->cfg.max_seq)
+    return fail(m, ADEPT_ERR_CAPACITY, "prompt_len %d > max_seq %d", prompt_len, m->cfg.max_seq);
+  if (std::isnan(delta)) return fail(m, ADEPT_ERR_INVALID_ARG, "delta is NaN");
+  cudaStream_t st = (cudaStream_t)stream;
+  std::vector<int> lens(batch, prompt_len);
+  TRY(reserve_seqs(m, batch, lens.data(), st));
+  TRY(run_pass(m, batch * prompt_len, batch, prompt_len, false, d_tokens, delta, d_forced_exit, d_exit_layer_out,
+               d_sim_out, st));
+  TRY(run_head(m, batch, prompt_len, false, d_logits_out, d_next_token_out, st));
+  return check_launch(m);
+}
+
+adept_status adept_decode_step(adept_model* m, int batch, const int32_t* d_tokens, float delta,
+                               const int32_t* d_forced_exit, int32_t* d_exit_layer_out, float* d_logits_out,
+                               int32_t* d_next_token_out, float* d_sim_out, void* stream) {
+  if (!m) return ADEPT_ERR_INVALID_ARG;
+  if (m->cfg.family == ADEPT_FAMILY_BERT) return fail(m, ADEPT_ERR_INVALID_ARG, "decode needs a decoder model");
+  if (!d_tokens) return fail(m, ADEPT_ERR_INVALID_ARG, "d_tokens is NULL");
+  if (batch < 1 || batch > m->cfg.max_batch) return fail(m, ADEPT_ERR_CAPACITY, "batch %d out of range", batch);
+  if (std::isnan(delta)) return fail(m, ADEPT_ERR_INVALID_ARG, "delta is NaN");
+  for (int b = 0; b < batch; ++b) {
+    if (m->seq_blocks[b].empty()) return fail(m, ADEPT_ERR_INVALID_ARG, "sequence %d has no prompt", b);
+    if (m->h_seq_len[b] >= m->max_blocks_per_seq * m->cfg.kv_block_tokens || m->h_seq_len[b] >= m->cfg.max_seq)
+      return fail(m, ADEPT_ERR_CAPACITY, "sequence %d is full (%d positions)", b, m->h_seq_len[b]);
+  }
+  cudaStream_t st = (cudaStream_t)stream;
+  TRY(run_pass(m, batch, batch, 1, true, d_tokens, delta, d_forced_exit, d_exit_layer_out, d_sim_out, st));
+  for (int b = 0; b < batch; ++b) m->h_seq_len[b] += 1;
+  TRY(run_head(m, batch, 1, true, d_logits_out, d_next_token_out, st));
+  return check_launch(m);
+}
+
+adept_status adept_skip_kv_fill(adept_model* m, int n_tokens, const void* d_h_mapped, const int32_t* d_exit_layer,
+                                const int32_t* d_seq, const int32_t* d_pos, void* stream) {
+  if (!m) return ADEPT_ERR_INVALID_ARG;
+  if (n_tokens < 0) return fail(m, ADEPT_ERR_INVALID_ARG, "n_tokens < 0");
+  if (n_tokens == 0) return ADEPT_OK;
+  if (n_tokens > (1 << 20)) return fail(m, ADEPT_ERR_CAPACITY, "n_tokens %d above 1<<20", n_tokens);
+  if (!d_h_mapped || !d_exit_layer || !d_seq || !d_pos) return fail(m, ADEPT_ERR_INVALID_ARG, "NULL device pointer");
+  cudaStream_t st = (cudaStream_t)stream;
+  if (n_tokens > m->fill_cap) {
+    // grow the fill workspace (outside any timed or captured region by contract)
+    for (void* p : {(void*)m->fill_x, (void*)m->fill_tok}) {
+      if (!p) continue;
+      cudaFree(p);
+      m->allocs.erase(std::remove(m->allocs.begin(), m->allocs.end(), p), m->allocs.end());
+    }
+    m->fill_x = nullptr;
+    m->fill_tok = nullptr;
+    int cap = std::max(n_tokens, 1024);
+    TRY(dalloc(m, &m->fill_x, (size_t)cap * m->D * m->esz));
+    TRY(dalloc_t(m, &m->fill_tok, cap));
+    if (!m->fill_hist) {
+      TRY(dalloc_t(m, &m->fill_hist, m->N + 2));
+      TRY(dalloc_t(m, &m->fill_start, m->N + 2));
+      TRY(dalloc_t(m, &m->fill_cursor, m->N + 2));
+    }
+    m->fill_cap = cap;
+  }
+  launch_fill_sort(st, m->dt, d_h_mapped, n_tokens, m->D, d_exit_layer, m->N, m->fill_hist, m->fill_start,
+                   m->fill_cursor, m->fill_tok, m->fill_x, attn_norm_mode(m), m->cfg.norm_eps, m->err_word);
+  m->launches += 4;
+  std::vector<GemmProblem> probs;
+  std::vector<int> mrs;
+  for (int r = 2; r <= m->N; ++r) {
+    probs.push_back(kv_problem(m, r - 1, m->fill_x, DevRange{nullptr, m->fill_start + r, 0}, m->fill_tok, d_seq, d_pos));
+    mrs.push_back(n_tokens);
+  }
+  // algorithmic work of this launch is only known on the device; the benchmark supplies it
+  gemm(m, st, probs.data(), (int)probs.size(), mrs.data(), ADEPT_PROF_KV_FILL);
+  return check_launch(m);
+}
+
+adept_status adept_seq_reserve(adept_model* m, int batch, const int32_t* h_lens) {
+  if (!m || !h_lens) return ADEPT_ERR_INVALID_ARG;
+  if (batch < 1 || batch > m->cfg.max_batch) return fail(m, ADEPT_ERR_CAPACITY, "batch %d out of range", batch);
+  for (int b = 0; b < batch; ++b)
+    if (h_lens[b] < 0 || h_lens[b] > m->cfg.max_seq) return fail(m, ADEPT_ERR_INVALID_ARG, "length out of range");
+  TRY(reserve_seqs(m, batch, h_lens, 0));
+  CUDA_TRY(m, cudaStreamSynchronize(0));
+  return ADEPT_OK;
+}
+
+adept_status adept_read_kv(adept_model* m, int layer, int seq, int pos0, int n_pos, void* d_k_out, void* d_v_out,
+                           void* stream) {
+  if (!m || !d_k_out || !d_v_out) return ADEPT_ERR_INVALID_ARG;
+  if (layer < 1 || layer > m->N) return fail(m, ADEPT_ERR_INVALID_ARG, "layer %d out of [1, N]", layer);
+  if (seq < 0 || seq >= m->cfg.max_batch || m->seq_blocks[seq].empty())
+    return fail(m, ADEPT_ERR_INVALID_ARG, "sequence %d not reserved", seq);
+  if (pos0 < 0 || n_pos < 0 || pos0 + n_pos > m->max_blocks_per_seq * m->cfg.kv_block_tokens)
+    return fail(m, ADEPT_ERR_INVALID_ARG, "position range out of the reserved blocks");
+  launch_read_kv((cudaStream_t)stream, m->dt, cache_view(m), layer - 1, seq, pos0, n_pos, d_k_out, d_v_out);
+  return check_launch(m);
+}
+
+adept_status adept_read_final_states(adept_model* m, float* d_out, int rows, void* stream) {
+  if (!m || !d_out) return ADEPT_ERR_INVALID_ARG;
+  if (rows < 0 || rows > m->last_rows) return fail(m, ADEPT_ERR_INVALID_ARG, "rows %d > last pass rows", rows);
+  CUDA_TRY(m, cudaMemcpyAsync(d_out, m->final_, (size_t)rows * m->D * sizeof(float), cudaMemcpyDeviceToDevice,
+                              (cudaStream_t)stream));
+  return ADEPT_OK;
+}
+
+adept_status adept_check_device_status(adept_model* m, void* stream) {
+  if (!m) return ADEPT_ERR_INVALID_ARG;
+  cudaStream_t st = (cudaStream_t)stream;
+  CUDA_TRY(m, cudaStreamSynchronize(st));
+  CUDA_TRY(m, cudaGetLastError());
+  unsigned w = 0;
+  CUDA_TRY(m, cudaMemcpy(&w, m->err_word, sizeof w, cudaMemcpyDeviceToHost));
+  CUDA_TRY(m, cudaMemset(m->err_word, 0, sizeof(unsigned)));
+  if (w & ERRW_TIMEOUT) return fail(m, ADEPT_ERR_TIMEOUT, "a device-side wait timed out (word 0x%x)", w);
+  if (w) return fail(m, ADEPT_ERR_DEVICE_INPUT, "device-side input check failed (word 0x%x)", w);
+  return ADEPT_OK;
+}
+
+adept_status adept_set_option(adept_model* m, int option, int value) {
+  if (!m) return ADEPT_ERR_INVALID_ARG;
+  switch (option) {
+    case ADEPT_OPT_HSM_IDENTITY: m->hsm_identity = value != 0; return ADEPT_OK;
+    case ADEPT_OPT_PROFILE: m->profile = value != 0; return ADEPT_OK;
+    case ADEPT_OPT_GEMM_SIMT: m->force_simt = value != 0; return ADEPT_OK;
+  }
+  return fail(m, ADEPT_ERR_INVALID_ARG, "unknown option %d", option);
+}
+
+adept_status adept_profile_read(adept_model* m, int cls, int64_t* launches, double* total_ms, double* flops,
+                                double* bytes) {
+  if (!m || cls < 0 || cls >= ADEPT_PROF_NCLASS) return ADEPT_ERR_INVALID_ARG;
+  CUDA_TRY(m, cudaDeviceSynchronize());
+  ProfRec& pr = m->prof[cls];
+  double ms = 0, fl = 0, by = 0;
+  for (size_t i = 0; i < pr.ev.size(); ++i) {
+    float t = 0;
+    cudaEventElapsedTime(&t, pr.ev[i].first, pr.ev[i].second);
+    ms += t;
+    fl += pr.work[i].first;
+    by += pr.work[i].second;
+    cudaEventDestroy(pr.ev[i].first);
+    cudaEventDestroy(pr.ev[i].second);
+  }
+  if (launches) *launches = (int64_t)pr.ev.size();
+  if (total_ms) *total_ms = ms;
+  if (flops) *flops = fl;
+  if (bytes) *bytes = by;
+  pr.ev.clear();
+  pr.work.clear();
+  return ADEPT_OK;
+}
+
+int64_t adept_launch_count(adept_model* m) {
+  if (!m) return 0;
+  const int64_t n = m->launches;
+  m->launches = 0;
+  return n;
+}
+
+}  // extern "C"

@@ -1,0 +1,167 @@
+"""GPU parity: the CUDA library (through its C ABI) against the CPU oracle on the same
+seeded inputs.  Hidden states, logits and KV entries within the row-wise relative
+tolerance of the precision contract (1e-4 fp32, 2e-2 bf16); exit layers bit-exact
+outside the +-1e-3 similarity band."""
+import numpy as np
+import pytest
+import torch
+
+import synth
+from oracle import adept_oracle as O
+from parity_utils import Pair, assert_rows_close, compare_decode, compare_prefill, TOL
+
+import paper_2601_03700_gb300 as adept
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _lib():
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+    adept.load_library()
+
+
+def small(family, dtype="bf16", **kw):
+    base = dict(family=family, n_layers=6, d_model=256, n_heads=4, head_dim=64, d_ffn=512, vocab=1000,
+                max_pos=160, n_classes=2 if family == synth.BERT else 0, dtype=dtype, max_batch=4, max_seq=160,
+                hsm_m1=512, hsm_m2=1024)
+    if family == synth.BERT:
+        base["norm_eps"] = 1e-12
+    base.update(kw)
+    return synth.ModelConfig(**base)
+
+
+# --------------------------------------------------------------------------- tiny, fp32
+
+def test_tiny_fp32_threshold_prefill_and_decode():
+    """Tiny decoder (4 layers, D=256, 4 heads, SwiGLU 1024, vocab 1024, fp32, seed 0): a
+    64-token prompt, then 16 greedy decode steps, cosine threshold 0.95."""
+    cfg = synth.tiny_config()
+    pair = Pair(cfg, seed=0)
+    tokens = synth.make_tokens(0, 1, 64, cfg.vocab).numpy()
+    ores, cache, g = compare_prefill(pair, tokens, 0.95)
+    compare_decode(pair, cache, ores.next_token, 16, 0.95)
+    pair.compare_cache(cache, 1, 64 + 16)
+    pair.close()
+
+
+@pytest.mark.parametrize("delta", [0.2, 0.5, -2.0, float("inf")])
+def test_tiny_fp32_thresholds_ragged_batch(delta):
+    cfg = synth.tiny_config()
+    pair = Pair(cfg, seed=1, std=0.05)
+    tokens = synth.make_tokens(1, 3, 37, cfg.vocab).numpy()
+    ores, cache, g = compare_prefill(pair, tokens, delta)
+    if delta == -2.0:
+        assert np.all(g["exit"] == 2)
+    if delta == float("inf"):
+        assert np.all(g["exit"] == cfg.n_layers)
+    compare_decode(pair, cache, ores.next_token, 3, delta)
+    pair.close()
+
+
+def test_tiny_fp32_forced_exits_and_hsm_identity():
+    cfg = synth.tiny_config(n_layers=6)
+    pair = Pair(cfg, seed=2, std=0.05)
+    tokens = synth.make_tokens(2, 2, 45, cfg.vocab).numpy()
+    forced = synth.forced_exits_uniform(2, 90, 2, 6).numpy().reshape(2, 45)
+    for ident in (False, True):
+        ores, cache, g = compare_prefill(pair, tokens, 0.5, forced, hsm_identity=ident)
+        fsteps = synth.forced_exits_uniform(3, 8, 2, 6).numpy().reshape(4, 2)
+        compare_decode(pair, cache, ores.next_token, 4, 0.5, fsteps)
+        pair.compare_cache(cache, 2, 45 + 4)
+    pair.close()
+
+
+# --------------------------------------------------------------------------- bf16 families
+
+@pytest.mark.parametrize("family", [synth.LLAMA, synth.GPT2, synth.BERT])
+def test_bf16_families_forced(family):
+    kw = dict(n_heads=2, head_dim=128) if family == synth.LLAMA else {}
+    cfg = small(family, **kw)
+    pair = Pair(cfg, seed=3)
+    B, P = 3, 70
+    tokens = synth.make_tokens(3, B, P, cfg.vocab).numpy()
+    forced = synth.forced_exits_uniform(4, B * P, 2, cfg.n_layers).numpy().reshape(B, P)
+    ores, cache, g = compare_prefill(pair, tokens, 0.9, forced)
+    if family != synth.BERT:
+        fsteps = synth.forced_exits_uniform(5, 5 * B, 2, cfg.n_layers).numpy().reshape(5, B)
+        compare_decode(pair, cache, ores.next_token, 5, 0.9, fsteps)
+        pair.compare_cache(cache, B, P + 5)
+    pair.close()
+
+
+@pytest.mark.parametrize("family", [synth.LLAMA, synth.GPT2, synth.BERT])
+def test_bf16_families_threshold(family):
+    cfg = small(family)
+    pair = Pair(cfg, seed=6, std=0.05)
+    tokens = synth.make_tokens(6, 2, 50, cfg.vocab).numpy()
+    for delta in (0.9, 0.6):
+        ores, cache, g = compare_prefill(pair, tokens, delta)
+        if family != synth.BERT:
+            compare_decode(pair, cache, ores.next_token, 3, delta)
+    pair.close()
+
+
+# --------------------------------------------------------------------------- skipped-layer fill ABI
+
+@pytest.mark.parametrize("dtype", ["f32", "bf16"])
+def test_skip_kv_fill_matches_oracle(dtype):
+    """adept_skip_kv_fill: every (token, r > i*) entry equals layer r's K/V projection of s~."""
+    cfg = small(synth.LLAMA, dtype=dtype, n_layers=8, n_heads=2, head_dim=128, block_shuffle_seed=7)
+    pair = Pair(cfg, seed=8)
+    n = 150
+    lens = [cfg.max_seq] * cfg.max_batch
+    adept.adept_seq_reserve(pair.gm.h, lens)
+    h = synth.make_mapped_states(9, n, cfg.d_model, dtype=cfg.torch_dtype)
+    el = synth.forced_exits_uniform(10, n, 1, cfg.n_layers).numpy()
+    seq = synth.randint(11, "seq", n, 0, cfg.max_batch - 1).numpy()
+    # distinct positions per sequence
+    pos = np.zeros(n, dtype=np.int64)
+    for b in range(cfg.max_batch):
+        idx = np.nonzero(seq == b)[0]
+        pos[idx] = synth.randint(12 + b, "perm", 1, 0, 0).numpy()[0] + np.arange(len(idx))
+    adept.adept_skip_kv_fill(pair.gm.h, n, h.cuda().contiguous(), torch.as_tensor(el, dtype=torch.int32).cuda(),
+                             torch.as_tensor(seq, dtype=torch.int32).cuda(), torch.as_tensor(pos, dtype=torch.int32).cuda())
+    pair.gm.check()
+    ref = O.skip_kv_fill(pair.om, h.double().numpy(), el, pos)
+    checked = 0
+    for r, (k, v, sel) in ref.items():
+        for b in range(cfg.max_batch):
+            rows = sel[seq[sel] == b]
+            if len(rows) == 0:
+                continue
+            gk, gv = pair.gpu_kv(r, b, cfg.max_seq)
+            assert_rows_close(gk[pos[rows]], k[np.searchsorted(sel, rows)], pair.tol, f"K r={r}")
+            assert_rows_close(gv[pos[rows]], v[np.searchsorted(sel, rows)], pair.tol, f"V r={r}")
+            checked += len(rows)
+    assert checked > n
+    pair.close()
+
+
+# --------------------------------------------------------------------------- error paths
+
+def test_device_input_errors_are_reported():
+    cfg = synth.tiny_config()
+    pair = Pair(cfg, seed=0)
+    tk = torch.zeros(1, 8, dtype=torch.int32, device="cuda")
+    bad = torch.ones(1, 8, dtype=torch.int32, device="cuda")      # forced layer 1 is not eligible
+    pair.gm.prefill(tk, 0.5, bad)
+    with pytest.raises(adept.AdeptError) as ei:
+        pair.gm.check()
+    assert ei.value.status == 6
+    tk2 = torch.full((1, 8), cfg.vocab + 5, dtype=torch.int32, device="cuda")
+    pair.gm.prefill(tk2, 0.5)
+    with pytest.raises(adept.AdeptError):
+        pair.gm.check()
+    pair.gm.check()  # cleared
+    with pytest.raises(adept.AdeptError) as ei:
+        pair.gm.prefill(torch.zeros(9, 8, dtype=torch.int32, device="cuda"), 0.5)
+    assert ei.value.status == 3
+    pair.close()
+
+
+def test_synth_generator_cpu_and_cuda_agree():
+    a = synth.normal(5, "w", (3, 100003), std=0.02, dtype=torch.bfloat16)
+    b = synth.normal(5, "w", (3, 100003), std=0.02, dtype=torch.bfloat16, device="cuda").cpu()
+    assert torch.equal(a.view(torch.int16), b.view(torch.int16))
