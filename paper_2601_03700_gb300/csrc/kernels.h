@@ -26,9 +26,9 @@ void launch_exit_decide(cudaStream_t st, const float* Xout, const float* I, int 
                         float* sim, int* flag, float* inv_norm, unsigned* err);
 void launch_exit_scan(cudaStream_t st, int* ctr, int in_parity, const int* flag, const int* row_tok,
                       int* row_tok_next, int* exit_tok, int* dst, int* exit_layer_out, int layer);
-void launch_exit_move(cudaStream_t st, const float* Xin, const float* Xout, const float* I, int D, const int* n_rows,
-                      int max_rows, const int* dst, const float* inv_norm, float* Xnext, float* Inext, float* hsm_s,
-                      float* hsm_prev, float* hsm_I);
+void launch_exit_move(cudaStream_t st, const float* Xin, const float* Xout, const float* I, int first, int D,
+                      const int* n_rows, int max_rows, const int* dst, const float* inv_norm, float* Xnext,
+                      float* Inext, float* hsm_s, float* hsm_prev, float* hsm_I);
 void launch_final_scatter(cudaStream_t st, const float* X, int D, const int* n_rows, int max_rows, const int* row_tok,
                           float* final_, int* exit_layer_out, int n_layers);
 void launch_hsm_prep(cudaStream_t st, int dt, const float* hs, const float* hp, const float* hI, DevRange rows,

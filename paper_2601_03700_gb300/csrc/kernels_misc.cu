@@ -208,10 +208,11 @@ __global__ void exit_scan_kernel(int* ctr, int in_parity, const int* flag, const
 
 // Moves each active row to its new place: survivors -> next layer input (s_i) and the
 // inertia with s_hat_i added (Sec. 4.1, after the test); exits -> the HSM input slots
-// (s_i, s_{i-1}, inertia before s_hat_i).
-__global__ void exit_move_kernel(const float* Xin, const float* Xout, const float* I, int D, const int* n_rows,
-                                 const int* dst, const float* inv_norm, float* Xnext, float* Inext, float* hsm_s,
-                                 float* hsm_prev, float* hsm_I) {
+// (s_i, s_{i-1}, inertia before s_hat_i).  first != 0 (layer 1): the inertia starts
+// as s_hat_1 (the sum over earlier layers is empty).
+__global__ void exit_move_kernel(const float* Xin, const float* Xout, const float* I, int first, int D,
+                                 const int* n_rows, const int* dst, const float* inv_norm, float* Xnext, float* Inext,
+                                 float* hsm_s, float* hsm_prev, float* hsm_I) {
   const int r = blockIdx.x;
   if (r >= *n_rows) return;
   const int d0 = dst[r];
@@ -224,7 +225,7 @@ __global__ void exit_move_kernel(const float* Xin, const float* Xout, const floa
     for (int d = threadIdx.x; d < D; d += blockDim.x) {
       const float v = s[d];
       xn[d] = v;
-      inn[d] = in[d] + v * w;
+      inn[d] = (first ? 0.f : in[d]) + v * w;
     }
   } else {
     const size_t k = (size_t)(-1 - d0);
@@ -545,12 +546,12 @@ void launch_exit_scan(cudaStream_t st, int* ctr, int in_parity, const int* flag,
                                        layer);
 }
 
-void launch_exit_move(cudaStream_t st, const float* Xin, const float* Xout, const float* I, int D, const int* n_rows,
-                      int max_rows, const int* dst, const float* inv_norm, float* Xnext, float* Inext, float* hsm_s,
-                      float* hsm_prev, float* hsm_I) {
+void launch_exit_move(cudaStream_t st, const float* Xin, const float* Xout, const float* I, int first, int D,
+                      const int* n_rows, int max_rows, const int* dst, const float* inv_norm, float* Xnext,
+                      float* Inext, float* hsm_s, float* hsm_prev, float* hsm_I) {
   if (max_rows <= 0) return;
-  exit_move_kernel<<<max_rows, 256, 0, st>>>(Xin, Xout, I, D, n_rows, dst, inv_norm, Xnext, Inext, hsm_s, hsm_prev,
-                                             hsm_I);
+  exit_move_kernel<<<max_rows, 256, 0, st>>>(Xin, Xout, I, first, D, n_rows, dst, inv_norm, Xnext, Inext, hsm_s,
+                                             hsm_prev, hsm_I);
 }
 
 void launch_final_scatter(cudaStream_t st, const float* X, int D, const int* n_rows, int max_rows, const int* row_tok,

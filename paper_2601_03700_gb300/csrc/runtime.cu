@@ -712,7 +712,7 @@ static adept_status run_pass(adept_model* m, int n_tok, int batch, int prompt_le
       launch_exit_decide(st, m->X_out, Ii, D, act, mr, rt, forced, i, N, delta, test, sim_out, m->flag, m->inv_norm,
                          m->err_word);
       launch_exit_scan(st, m->ctr, par, m->flag, rt, m->row_tok[par ^ 1], m->exit_tok, m->dst, exit_out, i);
-      launch_exit_move(st, Xi, m->X_out, Ii, D, m->ctr + CTR_ACTIVE + par, mr, m->dst, m->inv_norm, m->X_in[par ^ 1],
+      launch_exit_move(st, Xi, m->X_out, Ii, i == 1, D, m->ctr + CTR_ACTIVE + par, mr, m->dst, m->inv_norm, m->X_in[par ^ 1],
                        m->I[par ^ 1], m->hsm_s, m->hsm_prev, m->hsm_I);
       m->launches += 3;
       if (!decode && test) {

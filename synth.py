@@ -136,6 +136,8 @@ class ModelConfig:
     max_batch: int = 8
     max_seq: int = 1024
     n_kv_heads: int = 0        # 0 -> n_heads
+    kv_pool_blocks: int = 0    # 0 -> max_batch * ceil(max_seq / kv_block_tokens)
+    block_shuffle_seed: int = 0  # 0: KV blocks handed out in order; else a seeded permutation
 
     def __post_init__(self):
         if self.n_kv_heads == 0:

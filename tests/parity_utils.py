@@ -135,7 +135,8 @@ def check_greedy(g_next, g_logits, o_logits):
     return int(sure.sum())
 
 
-def compare_decode(pair: Pair, cache: O.OracleCache, first_tokens, steps: int, delta: float, forced_steps=None):
+def compare_decode(pair: Pair, cache: O.OracleCache, first_tokens, steps: int, delta: float, forced_steps=None,
+                   hsm_identity=False):
     """Greedy decode for `steps` steps, fed with the oracle's tokens (teacher forcing), so
     both sides stay on one trajectory; per step: exit layers, similarities, final states,
     logits and greedy tokens; at the end every cached position of every layer."""
@@ -143,7 +144,7 @@ def compare_decode(pair: Pair, cache: O.OracleCache, first_tokens, steps: int, d
     tok = np.asarray(first_tokens)
     for s in range(steps):
         f = None if forced_steps is None else np.asarray(forced_steps[s])
-        o = O.decode_step(pair.om, cache, tok, delta, f)
+        o = O.decode_step(pair.om, cache, tok, delta, f, hsm_mode="identity" if hsm_identity else "hsm")
         use_forced = f
         if f is None and band_tokens(o.sim, delta).any():
             use_forced = o.exit_layer

@@ -68,7 +68,7 @@ def test_tiny_fp32_forced_exits_and_hsm_identity():
     for ident in (False, True):
         ores, cache, g = compare_prefill(pair, tokens, 0.5, forced, hsm_identity=ident)
         fsteps = synth.forced_exits_uniform(3, 8, 2, 6).numpy().reshape(4, 2)
-        compare_decode(pair, cache, ores.next_token, 4, 0.5, fsteps)
+        compare_decode(pair, cache, ores.next_token, 4, 0.5, fsteps, hsm_identity=ident)
         pair.compare_cache(cache, 2, 45 + 4)
     pair.close()
 
