@@ -1,0 +1,490 @@
+#!/usr/bin/env python
+"""Benchmark of the early-exit forward pass on one GB300 (N GPUs: independent replicas).
+
+Workload (one step): a GPT-2-small-shaped decoder in bf16 (12 layers, D=768, 12 heads,
+FFN 3072, vocab 50257, random-init N(0, 0.02)); a prompt pass over 8 x 512 uniform
+random token ids, then 128 greedy generation steps; each token's exit layer is forced
+from the integer-uniform law on [4, 12] (12 = full depth).  value = (prompt + generated
+tokens) / s over the timed steps, inputs resident in HBM, L2 flushed between steps.
+
+Also reported: the skipped-layer KV fill at Llama-7B layer shapes (32 layers,
+D=4096, 32 KV heads x 128) on a grid of exited-token counts and exit layers, against
+its roofline; and the CPU oracle on a bounded sample of the same workload.
+
+--impl reference times that oracle (the slow plain statement of the method) as the
+reference arm.
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import math
+import os
+import subprocess
+import sys
+import tempfile
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+import numpy as np  # noqa: E402
+import torch  # noqa: E402
+
+import synth  # noqa: E402
+
+PEAKS_FALLBACK = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
+METRIC = "early-exit prefill+decode tokens/s at 1 GB300; skipped-layer KV-fill % of roofline"
+B, P, STEPS, LO, HI, DELTA = 8, 512, 128, 4, 12, 0.9
+L2_BYTES = 129 * 2 ** 20
+
+
+def load_peaks():
+    try:
+        with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
+            d = json.load(f)
+        return d, "measured"
+    except Exception:
+        return PEAKS_FALLBACK, "fallback"
+
+
+def workload_cfg():
+    return synth.gpt2_small_config(max_batch=B, max_seq=P + STEPS, max_pos=1024)
+
+
+# ----------------------------------------------------------------------------- algorithmic work
+
+def gemm_work(M, N, K, esz=2, extra_out_bytes=0, extra_in_bytes=0):
+    """(flops, bytes) of C[M,N] = A[M,K] B[N,K]^T: weights read once, A read, C written."""
+    if M <= 0:
+        return 0.0, 0.0
+    return 2.0 * M * N * K, float(N * K * esz + M * K * esz + extra_out_bytes + extra_in_bytes)
+
+
+def pass_work(cfg, exit_layers, decode: bool):
+    """Algorithmic (flops, bytes) of the GEMMs of one pass given each token's exit layer.
+
+    Counts what the method needs: layer i's projections for the tokens active at i,
+    layer i's K/V of the tokens that left before i (prompt pass), the HSM of the
+    exiting tokens, and the head; weights are read once per launch."""
+    N, D, F = cfg.n_layers, cfg.d_model, cfg.d_ffn
+    dq, dkv, m1, m2 = cfg.d_q, cfg.d_kv, cfg.hsm_m1, cfg.hsm_m2
+    up = 2 * F if cfg.family == synth.LLAMA else F
+    e = np.asarray(exit_layers).reshape(-1)
+    fl = by = 0.0
+    for i in range(1, N + 1):
+        act = int(np.sum(e >= i))
+        ex = int(np.sum(e < i))
+        for w in (gemm_work(act, dq + 2 * dkv, D, extra_out_bytes=act * (dq + 2 * dkv) * 2),
+                  gemm_work(act, D, dq, extra_out_bytes=act * D * 8),
+                  gemm_work(act, up, D, extra_out_bytes=act * F * 2),
+                  gemm_work(act, D, F, extra_out_bytes=act * D * 8)):
+            fl += w[0]
+            by += w[1]
+        if not decode and ex > 0 and i >= 3:
+            fl += 2.0 * ex * 2 * dkv * D
+            by += ex * D * 2 + ex * 2 * dkv * 2
+        E = int(np.sum(e == i)) if i < N else 0
+        if not decode and E > 0:
+            for w in (gemm_work(E, m1, D), gemm_work(E, m2, m1), gemm_work(E, m1, m2), gemm_work(E, D, m1)):
+                fl += w[0]
+                by += w[1]
+    if decode:
+        E = int(np.sum(e < N))
+        for w in (gemm_work(E, m1, D), gemm_work(E, m2, m1), gemm_work(E, m1, m2), gemm_work(E, D, m1)):
+            fl += w[0]
+            by += w[1]
+    rows = len(e) if decode else B
+    w = gemm_work(rows, cfg.vocab, D, extra_out_bytes=rows * cfg.vocab * 4)
+    return fl + w[0], by + w[1]
+
+
+def decode_fill_work(cfg, exit_layers):
+    """Grouped skipped-layer fill at the end of a generation step: (flops, bytes)."""
+    N, D, dkv = cfg.n_layers, cfg.d_model, cfg.d_kv
+    e = np.asarray(exit_layers).reshape(-1)
+    fl = by = 0.0
+    for r in range(3, N + 1):
+        n = int(np.sum(e < r))
+        if n:
+            fl += 2.0 * n * 2 * dkv * D
+            by += 2 * dkv * D * 2 + n * D * 2 + n * 2 * dkv * 2
+    return fl, by
+
+
+def fill_micro_work(T, istar, n_layers=32, d=4096, dkv=4096):
+    """Skipped-layer fill of T tokens exiting at i*, all deeper layers: flops and the
+    algorithmic bytes (each layer's W_K/W_V once, s~ once, K/V written once)."""
+    L = n_layers - istar
+    flops = 2.0 * T * L * d * 2 * dkv
+    bytes_ = L * 2 * dkv * d * 2 + T * d * 2 + T * L * 2 * dkv * 2
+    return flops, bytes_
+
+
+# ----------------------------------------------------------------------------- clocks
+
+class Clocks:
+    """Samples nvidia-smi clocks and throttle reasons while the timed region runs."""
+    Q = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+         "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+         "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index: int):
+        self.f = tempfile.NamedTemporaryFile("w+", suffix=".csv", delete=False)
+        self.p = None
+        try:
+            self.p = subprocess.Popen(["nvidia-smi", f"--id={gpu_index}", f"--query-gpu={self.Q}",
+                                       "--format=csv,noheader,nounits", "-lms", "100"],
+                                      stdout=self.f, stderr=subprocess.DEVNULL)
+        except Exception:
+            self.p = None
+
+    def stop(self):
+        out = {"sm_mhz": None, "sm_max_mhz": None, "reasons": []}
+        if self.p is None:
+            out["reasons"] = ["nvidia-smi unavailable"]
+            return out
+        time.sleep(0.25)
+        self.p.terminate()
+        try:
+            self.p.wait(timeout=5)
+        except Exception:
+            self.p.kill()
+        self.f.flush()
+        self.f.seek(0)
+        rows = [l.strip().split(", ") for l in self.f.read().splitlines() if l.strip()]
+        os.unlink(self.f.name)
+        sm, mx, reasons = [], [], set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for r in rows:
+            try:
+                sm.append(float(r[1]))
+                mx.append(float(r[2]))
+                for k, n in enumerate(names):
+                    if r[5 + k].strip().lower() == "active":
+                        reasons.add(n)
+            except Exception:
+                continue
+        if sm:
+            srt = sorted(sm)
+            top = [s for s in srt if s >= 0.5 * srt[-1]] or srt
+            out["sm_mhz"] = float(np.median(top))
+            out["sm_max_mhz"] = max(mx)
+            out["samples"] = len(sm)
+        out["reasons"] = sorted(reasons)
+        return out
+
+
+# ----------------------------------------------------------------------------- our arm
+
+def make_inputs(cfg, device):
+    tokens = synth.make_tokens(0, B, P, cfg.vocab).to(device)
+    fp = synth.forced_exits_uniform(0, B * P, LO, HI, name="forced_prompt").view(B, P).to(device)
+    fd = synth.forced_exits_uniform(0, STEPS * B, LO, HI, name="forced_decode").view(STEPS, B).to(device)
+    return tokens, fp, fd
+
+
+class Runner:
+    def __init__(self, adept, cfg, device):
+        self.a = adept
+        self.cfg = cfg
+        torch.manual_seed(0)
+        W = synth.make_weights(cfg, seed=0, device=device)
+        self.m = adept.Model(cfg, W)
+        del W
+        torch.cuda.empty_cache()
+        self.tokens, self.fp, self.fd = make_inputs(cfg, device)
+        self.exit_p = torch.empty(B * P, dtype=torch.int32, device=device)
+        self.exit_d = torch.empty(STEPS, B, dtype=torch.int32, device=device)
+        self.logits = torch.empty(B, cfg.vocab, dtype=torch.float32, device=device)
+        self.nxt = torch.empty(STEPS + 1, B, dtype=torch.int32, device=device)
+
+    def step(self, tokens=None, fp=None, fd=None):
+        a, h = self.a, self.m.h
+        tokens = self.tokens if tokens is None else tokens
+        fp = self.fp if fp is None else fp
+        fd = self.fd if fd is None else fd
+        a.adept_prefill(h, B, P, tokens.view(-1), DELTA, fp.view(-1), self.exit_p, self.logits, self.nxt[0], None)
+        for s in range(STEPS):
+            a.adept_decode_step(h, B, self.nxt[s], DELTA, fd[s], self.exit_d[s], self.logits, self.nxt[s + 1], None)
+
+
+def run_fill_micro(adept, device, peaks, grid_T, grid_i, reps=3):
+    """Skipped-layer fill through adept_skip_kv_fill at Llama-7B layer shapes."""
+    Tmax = max(grid_T)
+    seqs = 32
+    cfg = synth.llama7b_config(max_batch=seqs, max_seq=max(2048, (Tmax + seqs - 1) // seqs), max_pass_tokens=64,
+                               block_shuffle_seed=1234)
+    W = synth.make_weights(cfg, seed=0, device=device)
+    m = adept.Model(cfg, W)
+    del W
+    torch.cuda.empty_cache()
+    adept.adept_seq_reserve(m.h, [cfg.max_seq] * seqs)
+    h_all = synth.make_mapped_states(5, Tmax, cfg.d_model, device=device)
+    j = torch.arange(Tmax, device=device, dtype=torch.int32)
+    seq_all = (j % seqs).to(torch.int32).contiguous()
+    pos_all = (j // seqs).to(torch.int32).contiguous()
+    flush = torch.empty(2 * L2_BYTES // 4, dtype=torch.float32, device=device)
+    rows = []
+    st = torch.cuda.current_stream()
+    for istar in grid_i:
+        for T in grid_T:
+            el = torch.full((T,), istar, dtype=torch.int32, device=device)
+            args = (m.h, T, h_all[:T].contiguous(), el, seq_all[:T].contiguous(), pos_all[:T].contiguous())
+            adept.adept_skip_kv_fill(*args)
+            torch.cuda.synchronize()
+            adept.adept_set_option(m.h, adept.OPT_PROFILE, 1)
+            adept.adept_profile_read(m.h, adept.PROF_KV_FILL)
+            ts = []
+            for _ in range(reps):
+                flush.zero_()
+                e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+                e0.record(st)
+                adept.adept_skip_kv_fill(*args)
+                e1.record(st)
+                torch.cuda.synchronize()
+                ts.append(e0.elapsed_time(e1))
+            n, kms, _, _ = adept.adept_profile_read(m.h, adept.PROF_KV_FILL)
+            adept.adept_set_option(m.h, adept.OPT_PROFILE, 0)
+            adept.adept_check_device_status(m.h)
+            fl, by = fill_micro_work(T, istar)
+            t = float(np.median(ts)) / 1e3
+            tk = kms / max(n, 1) / 1e3
+            roof = max(fl / (peaks["bf16_tflops"] * 1e12), by / (peaks["hbm_gbs"] * 1e9))
+            rows.append({"T": T, "exit_layer": istar, "ms": round(t * 1e3, 4), "gemm_ms": round(tk * 1e3, 4),
+                         "tflops": round(fl / t / 1e12, 2), "gbs": round(by / t / 1e9, 1),
+                         "roofline_ms": round(roof * 1e3, 4), "frac": round(roof / t, 4),
+                         "bound": "tensor" if fl / (peaks["bf16_tflops"] * 1e12) > by / (peaks["hbm_gbs"] * 1e9) else "hbm"})
+    m.close()
+    del h_all
+    torch.cuda.empty_cache()
+    return rows
+
+
+def ours(args, rank, world, device):
+    import paper_2601_03700_gb300 as adept
+    if not os.path.exists(adept.LIB_PATH):
+        from paper_2601_03700_gb300 import build as _b
+        _b.build()
+    adept.load_library()
+    peaks, peaks_src = load_peaks()
+    cfg = workload_cfg()
+    run = Runner(adept, cfg, device)
+    flush = torch.empty(2 * L2_BYTES // 4, dtype=torch.float32, device=device)
+    st = torch.cuda.current_stream()
+    for _ in range(args.warmup):
+        run.step()
+    torch.cuda.synchronize()
+    adept.adept_check_device_status(run.m.h)
+    # --------------------------------------------------------------- timed region
+    adept.adept_set_option(run.m.h, adept.OPT_PROFILE, 1)
+    for c in range(4):
+        adept.adept_profile_read(run.m.h, c)
+    adept.adept_launch_count(run.m.h)
+    clocks = Clocks(torch.cuda.current_device()) if rank == 0 else None
+    if world > 1:
+        torch.distributed.barrier()
+    torch.cuda.synchronize()
+    total_ms = 0.0
+    for _ in range(args.steps):
+        flush.zero_()
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record(st)
+        run.step()
+        e1.record(st)
+        torch.cuda.synchronize()
+        total_ms += e0.elapsed_time(e1)
+    if world > 1:
+        torch.distributed.barrier()
+    clk = clocks.stop() if clocks else None
+    launches = adept.adept_launch_count(run.m.h)
+    prof = {c: adept.adept_profile_read(run.m.h, c) for c in range(4)}
+    adept.adept_set_option(run.m.h, adept.OPT_PROFILE, 0)
+    adept.adept_check_device_status(run.m.h)
+    t = torch.tensor([total_ms], dtype=torch.float64, device=device)
+    if world > 1:
+        torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
+    total_ms = float(t.item())
+    tok_per_step = B * P + B * STEPS
+    value = world * tok_per_step * args.steps / (total_ms / 1e3)
+    # --------------------------------------------------------------- end-to-end through the API with host buffers
+    tok_h = run.tokens.cpu().pin_memory()
+    fp_h = run.fp.cpu().pin_memory()
+    fd_h = run.fd.cpu().pin_memory()
+    out_h = torch.empty(STEPS + 1, B, dtype=torch.int32).pin_memory()
+    ex_h = torch.empty(B * P + STEPS * B, dtype=torch.int32).pin_memory()
+    tok_d, fp_d, fd_d = torch.empty_like(run.tokens), torch.empty_like(run.fp), torch.empty_like(run.fd)
+    e2e_t = 0.0
+    for _ in range(max(1, args.steps)):
+        flush.zero_()
+        torch.cuda.synchronize()
+        t0 = time.perf_counter()
+        tok_d.copy_(tok_h, non_blocking=True)
+        fp_d.copy_(fp_h, non_blocking=True)
+        fd_d.copy_(fd_h, non_blocking=True)
+        run.step(tok_d, fp_d, fd_d)
+        out_h.copy_(run.nxt, non_blocking=True)
+        ex_h[:B * P].copy_(run.exit_p, non_blocking=True)
+        ex_h[B * P:].copy_(run.exit_d.view(-1), non_blocking=True)
+        torch.cuda.synchronize()
+        e2e_t += time.perf_counter() - t0
+    e2e = world * tok_per_step * max(1, args.steps) / e2e_t
+    h2d = (tok_h.numel() + fp_h.numel() + fd_h.numel()) * 4
+    d2h = (out_h.numel() + ex_h.numel()) * 4
+    # --------------------------------------------------------------- dominant kernel roofline
+    e_p = run.exit_p.cpu().numpy()
+    e_d = run.exit_d.cpu().numpy()
+    wp = pass_work(cfg, e_p, decode=False)
+    wd = [pass_work(cfg, e_d[s], decode=True) for s in range(STEPS)]
+    wf = [decode_fill_work(cfg, e_d[s]) for s in range(STEPS)]
+    work = {adept.PROF_GEMM_PREFILL: wp, adept.PROF_GEMM_DECODE: (sum(w[0] for w in wd), sum(w[1] for w in wd)),
+            adept.PROF_KV_FILL: (sum(w[0] for w in wf), sum(w[1] for w in wf))}
+    names = {adept.PROF_GEMM_PREFILL: "gemm_prefill", adept.PROF_GEMM_DECODE: "gemm_decode",
+             adept.PROF_KV_FILL: "kv_fill_decode", adept.PROF_ATTENTION: "attention"}
+    per_class = {}
+    for c, (n, ms, _, _) in prof.items():
+        per_class[names[c]] = {"launches": n, "ms_per_step": round(ms / max(args.steps, 1), 4)}
+    dom = max((c for c in work), key=lambda c: prof[c][1])
+    n, ms, _, _ = prof[dom]
+    fl, by = work[dom]
+    fl_s = fl * args.steps
+    by_s = by * args.steps
+    t_f = fl_s / (peaks["bf16_tflops"] * 1e12)
+    t_b = by_s / (peaks["hbm_gbs"] * 1e9)
+    if t_f >= t_b:
+        roof = {"bound": "tensor", "achieved": round(fl_s / (ms / 1e3) / 1e12, 3), "peak": peaks["bf16_tflops"],
+                "unit": "TFLOP/s"}
+    else:
+        roof = {"bound": "hbm", "achieved": round(by_s / (ms / 1e3) / 1e9, 2), "peak": peaks["hbm_gbs"],
+                "unit": "GB/s"}
+    roof["frac"] = round(roof["achieved"] / roof["peak"], 4)
+    roof["traffic"] = None
+    roof["kernel"] = names[dom]
+    roof["launches"] = n
+    roof["peak_source"] = peaks_src + " (MEASURED_PEAKS.json burst)" if peaks_src == "measured" else peaks_src
+    line = {
+        "metric": METRIC, "value": round(value, 2), "unit": "tokens/s", "n_gpus": world, "steps": args.steps,
+        "warmup": args.warmup, "ms_per_step": round(total_ms / args.steps, 3), "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
+        "config": {"workload": "gpt2-small-shaped decoder, bf16, random-init N(0,0.02); batch 8 x 512-token "
+                               "uniform random prompts + 128 greedy decode steps; forced exit layer per token "
+                               "~ U{4..12}", "model": "gpt2-small-shape", "global_batch": B * world,
+                   "seq_len": P, "decode_steps": STEPS, "parallelism": f"replicas{world}" if world > 1 else "single",
+                   "l2": "flushed between timed steps (256 MiB write)"},
+        "e2e": {"value": round(e2e, 2), "unit": "tokens/s", "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h},
+        "gpu_launches": int(launches),
+        "roofline": roof,
+        "kernel_classes": per_class,
+        "exit_depth": {"prompt_mean": round(float(e_p.mean()), 3), "decode_mean": round(float(e_d.mean()), 3)},
+        "clocks": clk,
+    }
+    run.m.close()
+    del run
+    torch.cuda.empty_cache()
+    if rank == 0 and not args.no_kv_fill:
+        grid_T = [int(x) for x in args.fill_T.split(",")]
+        grid_i = [int(x) for x in args.fill_i.split(",")]
+        rows = run_fill_micro(adept, device, peaks, grid_T, grid_i)
+        line["kv_fill"] = {"shape": "Llama-7B layers: 32 x (D=4096 -> K,V 2x4096), bf16, paged 16-token blocks",
+                           "peak": {"tflops": peaks["bf16_tflops"], "gbs": peaks["hbm_gbs"], "source": peaks_src},
+                           "grid": rows,
+                           "mean_frac": round(float(np.mean([r["frac"] for r in rows])), 4)}
+    if rank == 0 and not args.no_cpu_baseline:
+        line["cpu_baseline"] = cpu_baseline(args.cpu_tokens)
+    return line
+
+
+# ----------------------------------------------------------------------------- oracle (CPU) arms
+
+def oracle_sample(n_seq: int, prompt: int, steps: int):
+    """Runs the oracle on a bounded sample of the workload: n_seq prompts of `prompt`
+    tokens and `steps` generation steps, same model, same exit law.  Returns
+    (tokens processed, seconds)."""
+    from oracle import adept_oracle as O
+    cfg = workload_cfg()
+    W = synth.make_weights(cfg, seed=0)
+    om = O.OracleModel(cfg, W)
+    del W
+    tokens, fp, fd = make_inputs(cfg, "cpu")
+    tk = tokens[:n_seq, :prompt].numpy()
+    f = fp[:n_seq, :prompt].numpy()
+    cache = O.OracleCache(cfg, n_seq, prompt + steps + 1)
+    t0 = time.perf_counter()
+    r = O.prefill(om, cache, tk, DELTA, f)
+    nxt = r.next_token
+    for s in range(steps):
+        r = O.decode_step(om, cache, nxt, DELTA, fd[s, :n_seq].numpy())
+        nxt = r.next_token
+    dt = time.perf_counter() - t0
+    return n_seq * (prompt + steps), dt
+
+
+def cores():
+    try:
+        return len(os.sched_getaffinity(0))
+    except Exception:
+        return os.cpu_count() or 1
+
+
+def cpu_baseline(n_tokens: int):
+    n_seq, prompt, steps = 1, n_tokens, 8
+    tok, dt = oracle_sample(n_seq, prompt, steps)
+    return {"value": round(tok / dt, 3), "unit": "tokens/s", "cores": cores(), "kind": "oracle",
+            "sample": f"{n_seq} prompt x {prompt} tokens + {steps} decode steps of the same model and exit law "
+                      f"(fp64 NumPy oracle, {dt:.1f} s)"}
+
+
+def reference_arm(args, rank, world):
+    if rank != 0:
+        return None
+    tot_tok, tot_s = 0, 0.0
+    for _ in range(args.warmup):
+        oracle_sample(1, 32, 1)
+    for _ in range(args.steps):
+        tok, dt = oracle_sample(1, args.cpu_tokens, 8)
+        tot_tok += tok
+        tot_s += dt
+    v = tot_tok / tot_s
+    return {"metric": METRIC, "value": round(v, 3), "unit": "tokens/s", "n_gpus": world, "steps": args.steps,
+            "warmup": args.warmup, "ms_per_step": round(tot_s / args.steps * 1e3, 3), "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic", "impl": "reference",
+            "config": {"workload": "gpt2-small-shaped decoder (same model and exit law), bounded sample: "
+                                   f"1 prompt x {args.cpu_tokens} tokens + 8 decode steps per step"},
+            "cpu_baseline": {"value": round(v, 3), "unit": "tokens/s", "cores": cores(), "kind": "oracle",
+                             "sample": f"1 prompt x {args.cpu_tokens} + 8 decode steps per step"},
+            "e2e": {"value": round(v, 3), "unit": "tokens/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=5)
+    ap.add_argument("--warmup", type=int, default=3)
+    ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
+    ap.add_argument("--no-kv-fill", action="store_true")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--fill-T", default="1,16,256,1024,4096,16384,65536")
+    ap.add_argument("--fill-i", default="4,8,16,24")
+    ap.add_argument("--cpu-tokens", type=int, default=512)
+    args = ap.parse_args()
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    if args.impl == "reference":
+        line = reference_arm(args, rank, world)
+        if line is not None:
+            print(json.dumps(line), flush=True)
+        return
+    if world > 1:
+        torch.cuda.set_device(local)
+        torch.distributed.init_process_group("nccl")
+    device = torch.device("cuda", torch.cuda.current_device())
+    line = ours(args, rank, world, device)
+    if rank == 0:
+        print(json.dumps(line), flush=True)
+    if world > 1:
+        torch.distributed.destroy_process_group()
+
+
+if __name__ == "__main__":
+    main()

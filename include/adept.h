@@ -74,6 +74,7 @@ typedef struct {
   int max_batch;       /* sequences */
   int max_seq;         /* positions per sequence (prompt + generated) */
   int kv_pool_blocks;  /* 0 -> max_batch * ceil(max_seq / kv_block_tokens) */
+  int max_pass_tokens; /* rows of the per-pass workspaces; 0 -> max_batch * max_seq */
   uint64_t block_shuffle_seed; /* 0: KV blocks handed out in order; else a seeded permutation */
 } adept_config;
 
@@ -188,10 +189,15 @@ ADEPT_API adept_status adept_check_device_status(adept_model* m, void* stream);
 enum { ADEPT_OPT_HSM_IDENTITY = 1, ADEPT_OPT_PROFILE = 2, ADEPT_OPT_GEMM_SIMT = 3 };
 ADEPT_API adept_status adept_set_option(adept_model* m, int option, int value);
 
-/* Kernel classes reported by adept_profile_read. */
-enum { ADEPT_PROF_GEMM = 0, ADEPT_PROF_KV_FILL = 1, ADEPT_PROF_ATTENTION = 2, ADEPT_PROF_NCLASS = 3 };
-/* Synchronise, then return launches, total ms, and the algorithmic flop and byte
- * counts summed over the recorded launches of kernel class `cls`; resets the record. */
+/* Kernel classes reported by adept_profile_read: the GEMMs of prompt passes (layer
+ * projections, HSM, head, and the per-layer skipped-layer fills co-launched with
+ * layer i's QKV), the GEMMs of generation steps, the grouped skipped-layer fill
+ * launches (end of a generation step and adept_skip_kv_fill), and attention. */
+enum { ADEPT_PROF_GEMM_PREFILL = 0, ADEPT_PROF_KV_FILL = 1, ADEPT_PROF_ATTENTION = 2,
+       ADEPT_PROF_GEMM_DECODE = 3, ADEPT_PROF_NCLASS = 4 };
+/* Synchronise, then return the number of recorded launches of kernel class `cls` and
+ * their total device time in ms (CUDA events on the launching stream); resets the
+ * record.  flops / bytes are reserved (returned as 0). */
 ADEPT_API adept_status adept_profile_read(adept_model* m, int cls, int64_t* launches, double* total_ms,
                                 double* flops, double* bytes);
 

@@ -20,7 +20,7 @@ ADEPT_OK = 0
 STATUS_NAMES = {0: "OK", 1: "INVALID_ARG", 2: "OOM", 3: "CAPACITY", 4: "CUDA", 5: "TIMEOUT", 6: "DEVICE_INPUT"}
 FAMILY = {"llama": 0, "gpt2": 1, "bert": 2}
 OPT_HSM_IDENTITY, OPT_PROFILE, OPT_GEMM_SIMT = 1, 2, 3
-PROF_GEMM, PROF_KV_FILL, PROF_ATTENTION = 0, 1, 2
+PROF_GEMM_PREFILL, PROF_KV_FILL, PROF_ATTENTION, PROF_GEMM_DECODE = 0, 1, 2, 3
 
 # every symbol declared in include/adept.h
 ABI_SYMBOLS = [
@@ -45,7 +45,8 @@ class AdeptConfig(ctypes.Structure):
         ("n_classes", ctypes.c_int), ("dtype", ctypes.c_int), ("norm_eps", ctypes.c_float),
         ("rope_theta", ctypes.c_float), ("hsm_eps", ctypes.c_float), ("hsm_m1", ctypes.c_int),
         ("hsm_m2", ctypes.c_int), ("kv_block_tokens", ctypes.c_int), ("max_batch", ctypes.c_int),
-        ("max_seq", ctypes.c_int), ("kv_pool_blocks", ctypes.c_int), ("block_shuffle_seed", ctypes.c_uint64),
+        ("max_seq", ctypes.c_int), ("kv_pool_blocks", ctypes.c_int), ("max_pass_tokens", ctypes.c_int),
+        ("block_shuffle_seed", ctypes.c_uint64),
     ]
 
 
@@ -137,7 +138,8 @@ def make_config(cfg) -> AdeptConfig:
         norm_eps=float(g("norm_eps", 1e-5)), rope_theta=float(g("rope_theta", 10000.0)),
         hsm_eps=float(g("hsm_eps", 1e-6)), hsm_m1=g("hsm_m1"), hsm_m2=g("hsm_m2"),
         kv_block_tokens=g("kv_block_tokens", 16), max_batch=g("max_batch"), max_seq=g("max_seq"),
-        kv_pool_blocks=g("kv_pool_blocks", 0) or 0, block_shuffle_seed=int(g("block_shuffle_seed", 0) or 0))
+        kv_pool_blocks=g("kv_pool_blocks", 0) or 0, max_pass_tokens=g("max_pass_tokens", 0) or 0,
+        block_shuffle_seed=int(g("block_shuffle_seed", 0) or 0))
 
 
 # ---------------------------------------------------------------------------

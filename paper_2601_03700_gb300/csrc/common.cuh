@@ -146,6 +146,7 @@ struct Epi {
 struct GemmProblem {
   const void* A;
   int lda;
+  int a_rows;       // rows allocated in A (the TMA view's extent; reads past it return zeros)
   const void* B;
   int ldb;
   DevRange rows;

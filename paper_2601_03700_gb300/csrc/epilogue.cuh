@@ -1,0 +1,190 @@
+// GEMM epilogues applied to 32 consecutive output columns of one row.  Shared by the
+// tcgen05 GEMM (a thread owns one accumulator row in tensor memory), the skinny GEMM
+// and the SIMT GEMM, so every path has one definition of each fused epilogue.
+//
+// Column layouts the epilogues rely on (fixed by the load-time repacking):
+//  * RoPE families: inside each Q / K head the weight rows are interleaved so that
+//    output columns (2i, 2i+1) hold the rotate-half pair (i, i + head_dim/2).
+//  * SwiGLU: gate and up rows interleaved in blocks of 16, so a 32-column chunk
+//    holds 16 gate and the matching 16 up columns.
+#pragma once
+#include "common.cuh"
+
+namespace adept {
+
+template <typename T> struct Vec16;
+template <> struct Vec16<float> {
+  static __device__ __forceinline__ void store(float* p, const float* v) {
+    float4* q = reinterpret_cast<float4*>(p);
+#pragma unroll
+    for (int j = 0; j < 4; ++j) q[j] = make_float4(v[4 * j], v[4 * j + 1], v[4 * j + 2], v[4 * j + 3]);
+  }
+};
+template <> struct Vec16<bf16> {
+  static __device__ __forceinline__ void store(bf16* p, const float* v) {
+    uint4 w[2];
+    uint32_t* u = reinterpret_cast<uint32_t*>(w);
+#pragma unroll
+    for (int j = 0; j < 8; ++j) {
+      __nv_bfloat162 h = __floats2bfloat162_rn(v[2 * j], v[2 * j + 1]);
+      u[j] = *reinterpret_cast<uint32_t*>(&h);
+    }
+    uint4* q = reinterpret_cast<uint4*>(p);
+    q[0] = w[0];
+    q[1] = w[1];
+  }
+};
+
+// 16 values to T* p (p 32-byte aligned for bf16, 64-byte for fp32).
+template <typename T>
+__device__ __forceinline__ void store16(T* p, const float* v) {
+  Vec16<T>::store(p, v);
+}
+
+// Per-row facts the cache epilogues need: the token's position and the cache offset
+// of its slot (-1 if the position has no reserved block).
+struct EpiRow {
+  long long cbase;
+  int pos;
+};
+
+__device__ __forceinline__ EpiRow epi_row(const Epi& e, int ra) {
+  EpiRow r{-1, 0};
+  if (e.kind == EPI_QKV || e.kind == EPI_KV) {
+    const int tok = e.row_tok[ra];
+    r.pos = e.tok_pos[tok];
+    r.cbase = e.cache.checked_base(e.layer0, e.tok_seq[tok], r.pos);
+  }
+  return r;
+}
+
+// Rotary embedding of 16 adjacent pairs (columns 2j, 2j+1 -> features i0+j, i0+j+half),
+// written as two runs of 16 at dst[i0] and dst[i0 + half].
+template <typename T>
+__device__ __forceinline__ void rope_pairs(T* dst, int i0, int half, const float* v, const float2* tab) {
+  float a[16], b[16];
+#pragma unroll
+  for (int j = 0; j < 16; ++j) {
+    const float2 cs = tab[i0 + j];
+    const float x1 = v[2 * j], x2 = v[2 * j + 1];
+    a[j] = x1 * cs.x - x2 * cs.y;
+    b[j] = x2 * cs.x + x1 * cs.y;
+  }
+  store16<T>(dst + i0, a);
+  store16<T>(dst + i0 + half, b);
+}
+
+template <typename T>
+__device__ __forceinline__ void epi_chunk32(const Epi& e, int ra, int c0, int N, float (&v)[32], const EpiRow& rr) {
+  const bool full = c0 + 32 <= N;
+  if (e.bias) {
+#pragma unroll
+    for (int j = 0; j < 32; ++j)
+      if (full || c0 + j < N) v[j] += e.bias[c0 + j];
+  }
+  switch (e.kind) {
+    case EPI_F32: {
+      float* o = e.out_f32 + (size_t)ra * e.ld_f32 + c0;
+      if (full && ((e.ld_f32 & 15) == 0)) {
+        store16<float>(o, v);
+        store16<float>(o + 16, v + 16);
+      } else {
+        for (int j = 0; j < 32; ++j)
+          if (c0 + j < N) o[j] = v[j];
+      }
+      return;
+    }
+    case EPI_ACT: {
+#pragma unroll
+      for (int j = 0; j < 32; ++j) v[j] = apply_act(e.act, v[j]);
+      T* o = (T*)e.out_t + (size_t)ra * e.ld_t + c0;
+      if (full && ((e.ld_t & 15) == 0)) {
+        store16<T>(o, v);
+        store16<T>(o + 16, v + 16);
+      } else {
+        for (int j = 0; j < 32; ++j)
+          if (c0 + j < N) o[j] = from_f<T>(v[j]);
+      }
+      if (e.out_f32) {
+        float* f = e.out_f32 + (size_t)ra * e.ld_f32 + c0;
+        if (full && ((e.ld_f32 & 15) == 0)) {
+          store16<float>(f, v);
+          store16<float>(f + 16, v + 16);
+        } else {
+          for (int j = 0; j < 32; ++j)
+            if (c0 + j < N) f[j] = v[j];
+        }
+      }
+      return;
+    }
+    case EPI_RESID: {
+      const float* r = e.resid + (size_t)ra * e.ld_resid + c0;
+      float* o = e.out_f32 + (size_t)ra * e.ld_f32 + c0;
+      if (full && ((e.ld_f32 & 15) == 0) && ((e.ld_resid & 15) == 0)) {
+        const float4* r4 = reinterpret_cast<const float4*>(r);
+#pragma unroll
+        for (int j = 0; j < 8; ++j) {
+          const float4 x = r4[j];
+          v[4 * j] += x.x;
+          v[4 * j + 1] += x.y;
+          v[4 * j + 2] += x.z;
+          v[4 * j + 3] += x.w;
+        }
+        store16<float>(o, v);
+        store16<float>(o + 16, v + 16);
+      } else {
+        for (int j = 0; j < 32; ++j)
+          if (c0 + j < N) o[j] = r[j] + v[j];
+      }
+      return;
+    }
+    case EPI_SWIGLU: {
+      float h[16];
+#pragma unroll
+      for (int j = 0; j < 16; ++j) h[j] = silu_f(v[j]) * v[16 + j];
+      T* o = (T*)e.out_t + (size_t)ra * e.ld_t + (c0 >> 1);
+      if ((e.ld_t & 15) == 0) {
+        store16<T>(o, h);
+      } else {
+        for (int j = 0; j < 16; ++j) o[j] = from_f<T>(h[j]);
+      }
+      return;
+    }
+    default:
+      break;
+  }
+  // EPI_QKV / EPI_KV: [0, n_q) query, [n_q, n_q + n_kv) key, [n_q + n_kv, n_q + 2 n_kv) value.
+  const int dh = e.head_dim, half = dh >> 1;
+  const int nq = e.n_q_cols, nkv = e.n_kv_cols;
+  if (c0 < nq) {
+    const int h = c0 / dh, d0 = c0 % dh;
+    T* q = (T*)e.out_t + (size_t)ra * e.ld_t + h * dh;
+    if (e.rope) {
+      rope_pairs<T>(q, d0 >> 1, half, v, e.rope_table + (size_t)rr.pos * half);
+    } else {
+      store16<T>(q + d0, v);
+      store16<T>(q + d0 + 16, v + 16);
+    }
+    return;
+  }
+  if (rr.cbase < 0) return;
+  if (c0 < nq + nkv) {
+    const int c = c0 - nq, h = c / dh, d0 = c % dh;
+    T* k = (T*)e.cache.k + rr.cbase + (size_t)h * e.cache.head_stride();
+    if (e.rope) {
+      rope_pairs<T>(k, d0 >> 1, half, v, e.rope_table + (size_t)rr.pos * half);
+    } else {
+      store16<T>(k + d0, v);
+      store16<T>(k + d0 + 16, v + 16);
+    }
+    return;
+  }
+  {
+    const int c = c0 - nq - nkv, h = c / dh, d0 = c % dh;
+    T* vv = (T*)e.cache.v + rr.cbase + (size_t)h * e.cache.head_stride() + d0;
+    store16<T>(vv, v);
+    store16<T>(vv + 16, v + 16);
+  }
+}
+
+}  // namespace adept

@@ -1,7 +1,440 @@
-// Grouped tcgen05 GEMM (placeholder until the tensor-core kernel lands).
+// Grouped tcgen05 GEMM for sm_103a: C[M, N] = A[M, K] * B[N, K]^T per problem (bf16
+// operands, both K-major; fp32 accumulation in tensor memory), one persistent launch
+// over the tiles of every problem of the group, fused epilogues (epilogue.cuh).
+//
+// CTA = 6 warps:  warp 0 lane 0  TMA producer (A and B tiles, 128-byte swizzle)
+//                 warp 1         tensor-memory allocator; lane 0 issues tcgen05.mma
+//                 warps 2..5     epilogue: tcgen05.ld of the accumulator rows -> global
+// Shared-memory ring of STAGES (A, B) k-blocks with full / empty mbarriers; two
+// accumulator buffers in tensor memory so the epilogue of tile t overlaps the
+// main loop of tile t+1.  Every mbarrier wait is bounded: on time-out the CTA sets
+// ERRW_TIMEOUT in the device error word, stops, drains its MMAs and frees TMEM.
 #include "gemm_tc.h"
+#include "epilogue.cuh"
+
+#include <cuda.h>
+#include <cudaTypedefs.h>
+
+#include <mutex>
 
 namespace adept {
-bool tc_gemm_supported() { return false; }
-int tc_gemm_grouped(cudaStream_t, const GemmProblem*, int, const int*, unsigned*) { return 0; }
+
+constexpr int TC_MAXG = 32;
+constexpr int TC_BM = 128;
+constexpr int TC_BK = 64;               // one 128-byte swizzle row of bf16
+constexpr int TC_THREADS = 192;
+constexpr long long TC_TIMEOUT_CYCLES = 4000000000LL;   // ~2 s at 2 GHz
+
+struct TcGroup {
+  CUtensorMap ta;   // A: [rows, K] bf16, box 64 x 128
+  CUtensorMap tb;   // B: [N, K] bf16, box 64 x BN
+  DevRange rows;
+  int N;
+  int K;
+  Epi epi;
+};
+
+struct TcParams {
+  TcGroup g[TC_MAXG];
+  int n_groups;
+  unsigned* err;
+};
+
+// ---------------------------------------------------------------------------- PTX wrappers
+__device__ __forceinline__ uint32_t smem_u32(const void* p) { return (uint32_t)__cvta_generic_to_shared(p); }
+
+__device__ __forceinline__ void mbar_init(uint64_t* bar, uint32_t count) {
+  asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(smem_u32(bar)), "r"(count) : "memory");
+}
+__device__ __forceinline__ void mbar_expect_tx(uint64_t* bar, uint32_t bytes) {
+  asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(smem_u32(bar)), "r"(bytes) : "memory");
+}
+__device__ __forceinline__ void mbar_arrive(uint64_t* bar) {
+  asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(smem_u32(bar)) : "memory");
+}
+__device__ __forceinline__ bool mbar_try_wait(uint64_t* bar, uint32_t parity) {
+  uint32_t ok;
+  asm volatile(
+      "{\n.reg .pred p;\nmbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\nselp.u32 %0, 1, 0, p;\n}\n"
+      : "=r"(ok)
+      : "r"(smem_u32(bar)), "r"(parity)
+      : "memory");
+  return ok != 0;
+}
+// Bounded wait for the phase of `parity`; false on time-out or when another role aborted.
+__device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, volatile int* abort_flag, unsigned* err) {
+  if (mbar_try_wait(bar, parity)) return true;
+  const long long t0 = clock64();
+  while (true) {
+    if (mbar_try_wait(bar, parity)) return true;
+    if (*abort_flag) return false;
+    if (clock64() - t0 > TC_TIMEOUT_CYCLES) {
+      atomicOr(err, ERRW_TIMEOUT);
+      *abort_flag = 1;
+      return false;
+    }
+  }
+}
+
+__device__ __forceinline__ void tma_load_2d(const CUtensorMap* tm, uint64_t* bar, void* dst, int x, int y) {
+  asm volatile(
+      "cp.async.bulk.tensor.2d.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1, {%2, %3}], [%4];" ::"r"(
+          smem_u32(dst)),
+      "l"((uint64_t)tm), "r"(x), "r"(y), "r"(smem_u32(bar))
+      : "memory");
+}
+
+__device__ __forceinline__ void tmem_alloc(uint32_t* slot, uint32_t ncols) {
+  asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(smem_u32(slot)), "r"(ncols)
+               : "memory");
+}
+__device__ __forceinline__ void tmem_relinquish() {
+  asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+}
+__device__ __forceinline__ void tmem_dealloc(uint32_t taddr, uint32_t ncols) {
+  asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(taddr), "r"(ncols) : "memory");
+}
+__device__ __forceinline__ void tc_fence_before() { asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory"); }
+__device__ __forceinline__ void tc_fence_after() { asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory"); }
+
+// D[tmem] (+)= A[smem] * B[smem]^T, M = 128, N from the instruction descriptor, K = 16.
+__device__ __forceinline__ void umma_bf16(uint32_t d, uint64_t a, uint64_t b, uint32_t idesc, uint32_t accumulate) {
+  asm volatile(
+      "{\n.reg .pred p;\nsetp.ne.b32 p, %4, 0;\ntcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n}\n" ::"r"(d),
+      "l"(a), "l"(b), "r"(idesc), "r"(accumulate)
+      : "memory");
+}
+// Arrive on `bar` once every tcgen05.mma issued so far by this thread has completed.
+__device__ __forceinline__ void umma_commit(uint64_t* bar) {
+  asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(smem_u32(bar))
+               : "memory");
+}
+
+// 32 consecutive fp32 accumulator columns of this thread's row (lane quarter of the warp).
+__device__ __forceinline__ void tmem_ld32(uint32_t taddr, float (&v)[32]) {
+  uint32_t r[32];
+  asm volatile(
+      "tcgen05.ld.sync.aligned.32x32b.x32.b32 {%0, %1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, %13, %14, %15, "
+      "%16, %17, %18, %19, %20, %21, %22, %23, %24, %25, %26, %27, %28, %29, %30, %31}, [%32];"
+      : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7]), "=r"(r[8]),
+        "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]), "=r"(r[15]), "=r"(r[16]),
+        "=r"(r[17]), "=r"(r[18]), "=r"(r[19]), "=r"(r[20]), "=r"(r[21]), "=r"(r[22]), "=r"(r[23]), "=r"(r[24]),
+        "=r"(r[25]), "=r"(r[26]), "=r"(r[27]), "=r"(r[28]), "=r"(r[29]), "=r"(r[30]), "=r"(r[31])
+      : "r"(taddr)
+      : "memory");
+  asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+#pragma unroll
+  for (int j = 0; j < 32; ++j) v[j] = __uint_as_float(r[j]);
+}
+
+// Shared-memory matrix descriptor: K-major operand in 128-byte-swizzled atoms of
+// 8 rows x 128 bytes (stride between atoms 1024 bytes), descriptor version 1.
+__device__ __forceinline__ uint64_t sdesc_sw128(uint32_t saddr) {
+  uint64_t d = 0;
+  d |= (uint64_t)((saddr >> 4) & 0x3FFF);
+  d |= (uint64_t)1 << 16;                 // leading-dimension byte offset (unused for this layout)
+  d |= (uint64_t)(1024 >> 4) << 32;       // stride-dimension byte offset
+  d |= (uint64_t)1 << 46;                 // version
+  d |= (uint64_t)2 << 61;                 // swizzle: 128 B
+  return d;
+}
+
+// Instruction descriptor of kind::f16: D fp32, A and B bf16, both K-major, M = 128.
+template <int BN>
+__device__ __forceinline__ constexpr uint32_t idesc_bf16() {
+  return (1u << 4) | (1u << 7) | (1u << 10) | ((uint32_t)(BN >> 3) << 17) | ((uint32_t)(TC_BM >> 4) << 24);
+}
+
+// ---------------------------------------------------------------------------- kernel
+template <int BN, int STAGES>
+__global__ void __launch_bounds__(TC_THREADS, 1) gemm_tc_kernel(const __grid_constant__ TcParams p) {
+  constexpr int A_BYTES = TC_BM * TC_BK * 2;
+  constexpr int B_BYTES = BN * TC_BK * 2;
+  constexpr uint32_t TX = A_BYTES + B_BYTES;
+  constexpr uint32_t TMEM_COLS = 2 * BN;
+  constexpr uint32_t IDESC = idesc_bf16<BN>();
+
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = (uint8_t*)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
+  uint8_t* sA = smem;
+  uint8_t* sB = smem + STAGES * A_BYTES;
+  uint64_t* full = (uint64_t*)(smem + STAGES * (A_BYTES + B_BYTES));
+  uint64_t* empty = full + STAGES;
+  uint64_t* accf = empty + STAGES;
+  uint64_t* acce = accf + 2;
+  uint64_t* drain = acce + 2;
+  uint32_t* tmem_slot = (uint32_t*)(drain + 1);
+  volatile int* abort_flag = (volatile int*)(tmem_slot + 1);
+
+  __shared__ int s_tile0[TC_MAXG + 1];
+  __shared__ int s_mbeg[TC_MAXG], s_M[TC_MAXG], s_tn[TC_MAXG];
+
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int ng = p.n_groups;
+  if (threadIdx.x == 0) {
+    int acc = 0;
+    for (int g = 0; g < ng; ++g) {
+      const int b = p.g[g].rows.b();
+      const int M = max(0, p.g[g].rows.e() - b);
+      const int tn = (p.g[g].N + BN - 1) / BN;
+      s_mbeg[g] = b;
+      s_M[g] = M;
+      s_tn[g] = tn;
+      s_tile0[g] = acc;
+      acc += ((M + TC_BM - 1) / TC_BM) * tn;
+    }
+    s_tile0[ng] = acc;
+    for (int s = 0; s < STAGES; ++s) {
+      mbar_init(&full[s], 1);
+      mbar_init(&empty[s], 1);
+    }
+    for (int b = 0; b < 2; ++b) {
+      mbar_init(&accf[b], 1);
+      mbar_init(&acce[b], 4);
+    }
+    mbar_init(drain, 1);
+    *abort_flag = 0;
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+  }
+  __syncthreads();
+  const int total = s_tile0[ng];
+  if ((int)blockIdx.x >= total) return;  // uniform: nothing allocated yet
+
+  if (warp == 1) {
+    tmem_alloc(tmem_slot, TMEM_COLS);
+    tmem_relinquish();
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = *tmem_slot;
+
+  auto locate = [&](int t, int& g, int& mb, int& nb) {
+    g = 0;
+    while (g + 1 < ng && t >= s_tile0[g + 1]) ++g;
+    const int local = t - s_tile0[g];
+    nb = local % s_tn[g];
+    mb = local / s_tn[g];
+  };
+
+  if (warp == 0) {
+    if (lane == 0) {
+      // ------------------------------------------------------------ TMA producer
+      int stage = 0;
+      uint32_t phase = 0;
+      uint32_t issued = 0, last_par = 0;   // per stage: issued at least once / parity of its last issue
+      for (int t = blockIdx.x; t < total && !*abort_flag; t += gridDim.x) {
+        int g, mb, nb;
+        locate(t, g, mb, nb);
+        const TcGroup& G = p.g[g];
+        const int nk = (G.K + TC_BK - 1) / TC_BK;
+        const int ya = s_mbeg[g] + mb * TC_BM, yb = nb * BN;
+        for (int kb = 0; kb < nk; ++kb) {
+          if (!mbar_wait(&empty[stage], phase ^ 1, abort_flag, p.err)) break;
+          mbar_expect_tx(&full[stage], TX);
+          tma_load_2d(&G.ta, &full[stage], sA + stage * A_BYTES, kb * TC_BK, ya);
+          tma_load_2d(&G.tb, &full[stage], sB + stage * B_BYTES, kb * TC_BK, yb);
+          issued |= 1u << stage;
+          last_par = (last_par & ~(1u << stage)) | (phase << stage);
+          if (++stage == STAGES) {
+            stage = 0;
+            phase ^= 1;
+          }
+        }
+      }
+      // every copy this thread issued has landed before the CTA may exit
+      for (int s = 0; s < STAGES; ++s) {
+        if (!(issued >> s & 1u)) continue;
+        const uint32_t par = (last_par >> s) & 1u;
+        const long long t0 = clock64();
+        while (!mbar_try_wait(&full[s], par)) {
+          if (clock64() - t0 > TC_TIMEOUT_CYCLES) {
+            atomicOr(p.err, ERRW_TIMEOUT);
+            break;
+          }
+        }
+      }
+    }
+  } else if (warp == 1) {
+    if (lane == 0) {
+      // ------------------------------------------------------------ MMA issuer
+      int stage = 0, ab = 0;
+      uint32_t phase = 0, aph = 0;
+      bool ok = true;
+      for (int t = blockIdx.x; t < total && ok; t += gridDim.x) {
+        int g, mb, nb;
+        locate(t, g, mb, nb);
+        const int nk = (p.g[g].K + TC_BK - 1) / TC_BK;
+        if (!(ok = mbar_wait(&acce[ab], aph ^ 1, abort_flag, p.err))) break;
+        tc_fence_after();
+        const uint32_t d = tmem + (uint32_t)(ab * BN);
+        for (int kb = 0; kb < nk; ++kb) {
+          if (!(ok = mbar_wait(&full[stage], phase, abort_flag, p.err))) break;
+          tc_fence_after();
+          const uint64_t ad = sdesc_sw128(smem_u32(sA + stage * A_BYTES));
+          const uint64_t bd = sdesc_sw128(smem_u32(sB + stage * B_BYTES));
+#pragma unroll
+          for (int k = 0; k < TC_BK / 16; ++k)
+            umma_bf16(d, ad + (uint64_t)(2 * k), bd + (uint64_t)(2 * k), IDESC, (kb | k) != 0 ? 1u : 0u);
+          umma_commit(&empty[stage]);
+          if (++stage == STAGES) {
+            stage = 0;
+            phase ^= 1;
+          }
+        }
+        if (!ok) break;
+        umma_commit(&accf[ab]);
+        ab ^= 1;
+        if (ab == 0) aph ^= 1;
+      }
+      // drain: every MMA issued by this thread has completed before TMEM is freed
+      umma_commit(drain);
+      const long long t0 = clock64();
+      while (!mbar_try_wait(drain, 0)) {
+        if (clock64() - t0 > TC_TIMEOUT_CYCLES) {
+          atomicOr(p.err, ERRW_TIMEOUT);
+          break;
+        }
+      }
+    }
+  } else {
+    // -------------------------------------------------------------- epilogue warps 2..5
+    const int q = warp & 3;                 // TMEM lane quarter this warp may access
+    const int row_in_tile = q * 32 + lane;
+    int ab = 0;
+    uint32_t aph = 0;
+    for (int t = blockIdx.x; t < total; t += gridDim.x) {
+      int g, mb, nb;
+      locate(t, g, mb, nb);
+      const TcGroup& G = p.g[g];
+      const bool got = mbar_wait(&accf[ab], aph, abort_flag, p.err);
+      if (!__all_sync(0xffffffffu, got)) break;   // warp-uniform: tcgen05.ld below is .sync.aligned
+      tc_fence_after();
+      const int r = mb * TC_BM + row_in_tile;
+      const bool valid = r < s_M[g];
+      const int ra = s_mbeg[g] + r;
+      EpiRow rr{-1, 0};
+      if (valid) rr = epi_row(G.epi, ra);
+      const uint32_t tb = tmem + ((uint32_t)(q * 32) << 16) + (uint32_t)(ab * BN);
+#pragma unroll 1
+      for (int c = 0; c < BN; c += 32) {
+        float v[32];
+        tmem_ld32(tb + (uint32_t)c, v);
+        const int c0 = nb * BN + c;
+        if (valid && c0 < G.N) epi_chunk32<bf16>(G.epi, ra, c0, G.N, v, rr);
+      }
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&acce[ab]);
+      ab ^= 1;
+      if (ab == 0) aph ^= 1;
+    }
+  }
+  __syncthreads();
+  if (warp == 1) {
+    __syncwarp();
+    tc_fence_after();
+    tmem_dealloc(tmem, TMEM_COLS);
+  }
+}
+
+// ---------------------------------------------------------------------------- host side
+static PFN_cuTensorMapEncodeTiled_v12000 g_encode = nullptr;
+static int g_num_sms = 0;
+static int g_cc_major = 0;
+
+static void init_once() {
+  static std::once_flag f;
+  std::call_once(f, [] {
+    void* fn = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &fn, 12000, cudaEnableDefault, &q) == cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      g_encode = (PFN_cuTensorMapEncodeTiled_v12000)fn;
+    else
+      cudaGetLastError();
+    int dev = 0;
+    cudaGetDevice(&dev);
+    cudaDeviceGetAttribute(&g_num_sms, cudaDevAttrMultiProcessorCount, dev);
+    cudaDeviceGetAttribute(&g_cc_major, cudaDevAttrComputeCapabilityMajor, dev);
+  });
+}
+
+bool tc_gemm_supported() {
+  init_once();
+  return g_encode != nullptr && g_cc_major == 10;
+}
+
+static bool make_map(CUtensorMap* m, const void* base, uint64_t inner, uint64_t outer, uint64_t row_bytes,
+                     uint32_t box_outer) {
+  if (((uintptr_t)base & 15) || (row_bytes & 15) || outer == 0 || inner == 0) return false;
+  cuuint64_t dims[2] = {inner, outer};
+  cuuint64_t strides[1] = {row_bytes};
+  cuuint32_t box[2] = {(cuuint32_t)TC_BK, box_outer};
+  cuuint32_t estr[2] = {1, 1};
+  return g_encode(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), dims, strides, box, estr,
+                  CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                  CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+template <int BN, int STAGES>
+static int launch_bn(cudaStream_t st, const TcParams& prm, int grid) {
+  constexpr size_t smem = (size_t)STAGES * (TC_BM + BN) * TC_BK * 2 + 1024 + 256;
+  static bool attr = false;
+  if (!attr) {
+    cudaFuncSetAttribute(gemm_tc_kernel<BN, STAGES>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    attr = true;
+  }
+  gemm_tc_kernel<BN, STAGES><<<grid, TC_THREADS, smem, st>>>(prm);
+  return 1;
+}
+
+int tc_gemm_grouped(cudaStream_t st, const GemmProblem* probs, int n_probs, const int* max_rows, unsigned* err_word) {
+  init_once();
+  if (n_probs <= 0) return 0;
+  if (n_probs > TC_MAXG) return -1;
+  // the cache / SwiGLU epilogues work on whole 32-column chunks
+  for (int i = 0; i < n_probs; ++i) {
+    const GemmProblem& q = probs[i];
+    if (q.K % 8 || q.lda % 8 || q.ldb % 8 || q.a_rows <= 0) return -1;
+    if ((q.epi.kind == EPI_QKV || q.epi.kind == EPI_KV || q.epi.kind == EPI_SWIGLU) && (q.N % 32)) return -1;
+  }
+  // tile width: the widest that still gives every SM a tile
+  long long tiles[4] = {0, 0, 0, 0};
+  const int bns[4] = {256, 128, 64, 32};
+  for (int i = 0; i < n_probs; ++i) {
+    const long long tm = (max_rows[i] + TC_BM - 1) / TC_BM;
+    for (int k = 0; k < 4; ++k) tiles[k] += tm * ((probs[i].N + bns[k] - 1) / bns[k]);
+  }
+  int pick = 3;
+  for (int k = 0; k < 4; ++k)
+    if (tiles[k] >= g_num_sms) {
+      pick = k;
+      break;
+    }
+  const int BN = bns[pick];
+  static TcParams prm;  // large: keep off the stack (calls on a model are serialised)
+  memset(&prm, 0, sizeof prm);
+  prm.n_groups = n_probs;
+  prm.err = err_word;
+  for (int i = 0; i < n_probs; ++i) {
+    const GemmProblem& q = probs[i];
+    TcGroup& G = prm.g[i];
+    if (!make_map(&G.ta, q.A, (uint64_t)q.K, (uint64_t)q.a_rows, (uint64_t)q.lda * 2, TC_BM)) return -1;
+    if (!make_map(&G.tb, q.B, (uint64_t)q.K, (uint64_t)q.N, (uint64_t)q.ldb * 2, (uint32_t)BN)) return -1;
+    G.rows = q.rows;
+    G.N = q.N;
+    G.K = q.K;
+    G.epi = q.epi;
+  }
+  const int grid = (int)std::min<long long>(tiles[pick], (long long)g_num_sms);
+  if (grid <= 0) return 0;
+  switch (BN) {
+    case 256: return launch_bn<256, 4>(st, prm, grid);
+    case 128: return launch_bn<128, 6>(st, prm, grid);
+    case 64: return launch_bn<64, 8>(st, prm, grid);
+    default: return launch_bn<32, 10>(st, prm, grid);
+  }
+}
+
 }  // namespace adept

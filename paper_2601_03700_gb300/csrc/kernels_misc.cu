@@ -462,9 +462,15 @@ __global__ void fold_rows_kernel(T* dst, int ld_dst, const T* src, int n_rows, i
   if (warp >= n_rows) return;
   const int n = warp;
   // row_mode 0: dst row = n.  1 / 2: gate / up of a SwiGLU pair, interleaved in blocks of 16.
+  // row_mode >= 8: rotary head of row_mode features -- the rotate-half pair (i, i + hd/2)
+  // lands on adjacent rows (2i, 2i + 1).
   int drow = n;
   if (row_mode == 1) drow = (n / 16) * 32 + (n % 16);
   if (row_mode == 2) drow = (n / 16) * 32 + 16 + (n % 16);
+  if (row_mode >= 8) {
+    const int hd = row_mode, half = hd / 2, h = n / hd, i = n % hd;
+    drow = h * hd + (i < half ? 2 * i : 2 * (i - half) + 1);
+  }
   const T* s = src + (size_t)n * K;
   T* o = dst + (size_t)drow * ld_dst;
   float acc = 0.f;

@@ -92,6 +92,7 @@ struct adept_model {
   int *fill_tok = nullptr, *fill_hist = nullptr, *fill_start = nullptr, *fill_cursor = nullptr;
   // options / instrumentation
   int hsm_identity = 0, profile = 0, force_simt = 0;
+  int gemm_cls = ADEPT_PROF_GEMM_PREFILL;
   int last_rows = 0;
   int64_t launches = 0;
   ProfRec prof[ADEPT_PROF_NCLASS];
@@ -193,14 +194,39 @@ static void prof_end(adept_model* m, int cls, cudaStream_t st, cudaEvent_t b, do
   m->prof[cls].work.push_back({flops, bytes});
 }
 
+// The SIMT path stages C in fp32 scratch: make room for `elems` floats.
+static bool ensure_scratch(adept_model* m, size_t elems) {
+  if (elems <= m->scratch_elems) return true;
+  if (m->scratch) {
+    cudaFree(m->scratch);
+    m->allocs.erase(std::remove(m->allocs.begin(), m->allocs.end(), (void*)m->scratch), m->allocs.end());
+    m->scratch = nullptr;
+    m->scratch_elems = 0;
+  }
+  if (dalloc_t(m, &m->scratch, elems) != ADEPT_OK) return false;
+  m->scratch_elems = elems;
+  return true;
+}
+
 static void gemm(adept_model* m, cudaStream_t st, const GemmProblem* probs, int n_probs, const int* max_rows,
                  int cls, double flops = 0, double bytes = 0) {
   cudaEvent_t b = nullptr;
   prof_begin(m, cls, st, &b);
   if (m->dt == ADEPT_DTYPE_BF16 && !m->force_simt && tc_gemm_supported()) {
-    m->launches += tc_gemm_grouped(st, probs, n_probs, max_rows, m->err_word);
-  } else {
+    const int nl = tc_gemm_grouped(st, probs, n_probs, max_rows, m->err_word);
+    if (nl >= 0) {
+      m->launches += nl;
+      prof_end(m, cls, st, b, flops, bytes);
+      return;
+    }
+    // shapes the tensor-core path does not take run on the SIMT path
+  }
+  {
     for (int i = 0; i < n_probs; ++i) {
+      if (!ensure_scratch(m, (size_t)max_rows[i] * probs[i].N)) {
+        cudaStreamSynchronize(st);
+        if (!ensure_scratch(m, (size_t)max_rows[i] * probs[i].N)) continue;  // error already recorded
+      }
       launch_gemm_simt(st, m->dt, probs[i], max_rows[i], m->scratch);
       m->launches += 2;
     }
@@ -364,7 +390,8 @@ static adept_status load_weights(adept_model* m, Loader& ld) {
         CUDA_TRY(m, cudaStreamSynchronize(ld.st));
         bin = btmp;
       }
-      TRY(ld.fold(p + qn[k], rows[k], D, w.w_qkv, off, g, b, bin, w.b_qkv));
+      const int rmode = (fam == ADEPT_FAMILY_LLAMA && k < 2) ? m->dh : 0;  // RoPE pairs made adjacent
+      TRY(ld.fold(p + qn[k], rows[k], D, w.w_qkv, off, g, b, bin, w.b_qkv, rmode));
       off += rows[k];
     }
     TRY(ld.upload(p + "wo", (int64_t)D * Dq, &w.w_o));
@@ -577,38 +604,39 @@ static void run_hsm(adept_model* m, cudaStream_t st, DevRange rows, int max_rows
   GemmProblem p;
   memset(&p, 0, sizeof p);
   p.rows = rows;
+  p.a_rows = m->T_max;
   // FC1: h1 = GELU(W1 c0 + b1)
   p.A = m->c0t; p.lda = D; p.B = m->hsm_w1; p.ldb = D; p.N = m1; p.K = D;
   p.epi = epi_base(); p.epi.kind = EPI_ACT; p.epi.act = ACT_GELU_ERF; p.epi.bias = m->hsm_b1;
   p.epi.out_t = m->h1t; p.epi.ld_t = m1; p.epi.out_f32 = m->h1f; p.epi.ld_f32 = m1;
-  gemm(m, st, &p, 1, &max_rows, ADEPT_PROF_GEMM);
+  gemm(m, st, &p, 1, &max_rows, m->gemm_cls);
   // FC2: h2 = GELU(W2 h1 + b2)
   p.A = m->h1t; p.lda = m1; p.B = m->hsm_w2; p.ldb = m1; p.N = m2; p.K = m1;
   p.epi = epi_base(); p.epi.kind = EPI_ACT; p.epi.act = ACT_GELU_ERF; p.epi.bias = m->hsm_b2;
   p.epi.out_t = m->h2t; p.epi.ld_t = m2;
-  gemm(m, st, &p, 1, &max_rows, ADEPT_PROF_GEMM);
+  gemm(m, st, &p, 1, &max_rows, m->gemm_cls);
   // FC3: h3 = W3 h2 + b3
   p.A = m->h2t; p.lda = m2; p.B = m->hsm_w3; p.ldb = m2; p.N = m1; p.K = m2;
   p.epi = epi_base(); p.epi.kind = EPI_F32; p.epi.bias = m->hsm_b3; p.epi.out_f32 = m->h3f; p.epi.ld_f32 = m1;
-  gemm(m, st, &p, 1, &max_rows, ADEPT_PROF_GEMM);
+  gemm(m, st, &p, 1, &max_rows, m->gemm_cls);
   launch_hsm_mid(st, m->dt, m->h3f, m->h1f, rows, max_rows, m1, m->hsm_g1, eps, m->h4t);
   m->launches += 1;
   // FC4: h5 = W4 h4 + b4
   p.A = m->h4t; p.lda = m1; p.B = m->hsm_w4; p.ldb = m1; p.N = D; p.K = m1;
   p.epi = epi_base(); p.epi.kind = EPI_F32; p.epi.bias = m->hsm_b4; p.epi.out_f32 = m->h5f; p.epi.ld_f32 = D;
-  gemm(m, st, &p, 1, &max_rows, ADEPT_PROF_GEMM);
+  gemm(m, st, &p, 1, &max_rows, m->gemm_cls);
   launch_hsm_out(st, m->dt, m->h5f, m->c0f, m->hsm_s, 0, rows, max_rows, D, m->hsm_g2, eps, m->exit_tok, m->final_,
                  m->xfill, attn_norm_mode(m), m->cfg.norm_eps);
   m->launches += 1;
 }
 
 // KV-only projection problem of layer `layer0` for the rows of `xs` (K-major x~ rows).
-static GemmProblem kv_problem(adept_model* m, int layer0, const void* xs, DevRange rows, const int* row_tok,
-                              const int* tok_seq, const int* tok_pos) {
+static GemmProblem kv_problem(adept_model* m, int layer0, const void* xs, int a_rows, DevRange rows,
+                              const int* row_tok, const int* tok_seq, const int* tok_pos) {
   GemmProblem p;
   memset(&p, 0, sizeof p);
   const LayerW& w = m->L[layer0];
-  p.A = xs; p.lda = m->D;
+  p.A = xs; p.lda = m->D; p.a_rows = a_rows;
   p.B = (const char*)w.w_qkv + (size_t)m->Dq * m->D * m->esz; p.ldb = m->D;
   p.rows = rows; p.N = 2 * m->Dkv; p.K = m->D;
   p.epi = epi_base();
@@ -622,6 +650,7 @@ static GemmProblem kv_problem(adept_model* m, int layer0, const void* xs, DevRan
 
 static adept_status run_pass(adept_model* m, int n_tok, int batch, int prompt_len, bool decode, const int32_t* tokens,
                              float delta, const int32_t* forced, int32_t* exit_out, float* sim_out, cudaStream_t st) {
+  m->gemm_cls = decode ? ADEPT_PROF_GEMM_DECODE : ADEPT_PROF_GEMM_PREFILL;
   const adept_config& c = m->cfg;
   const int N = m->N, D = m->D, Dq = m->Dq, Dkv = m->Dkv;
   const int fam = c.family;
@@ -656,7 +685,7 @@ static adept_status run_pass(adept_model* m, int n_tok, int batch, int prompt_le
     GemmProblem pr[2];
     int mrs[2] = {mr, mr};
     memset(pr, 0, sizeof pr);
-    pr[0].A = m->xn; pr[0].lda = D; pr[0].B = w.w_qkv; pr[0].ldb = D; pr[0].rows = act;
+    pr[0].A = m->xn; pr[0].lda = D; pr[0].a_rows = m->T_max; pr[0].B = w.w_qkv; pr[0].ldb = D; pr[0].rows = act;
     pr[0].N = Dq + 2 * Dkv; pr[0].K = D;
     pr[0].epi = epi_base();
     pr[0].epi.kind = EPI_QKV; pr[0].epi.bias = w.b_qkv; pr[0].epi.out_t = m->q; pr[0].epi.ld_t = Dq;
@@ -665,22 +694,28 @@ static adept_status run_pass(adept_model* m, int n_tok, int batch, int prompt_le
     pr[0].epi.head_dim = m->dh; pr[0].epi.rope = fam == ADEPT_FAMILY_LLAMA; pr[0].epi.rope_table = m->rope_table;
     int np = 1;
     if (!decode && i >= 3) {
-      pr[1] = kv_problem(m, l0, m->xfill, DevRange{nullptr, m->ctr + CTR_EXITED, 0}, m->exit_tok, m->tok_seq,
+      pr[1] = kv_problem(m, l0, m->xfill, m->T_max, DevRange{nullptr, m->ctr + CTR_EXITED, 0}, m->exit_tok, m->tok_seq,
                          m->tok_pos);
       np = 2;
     }
-    gemm(m, st, pr, np, mrs, ADEPT_PROF_GEMM);
+    gemm(m, st, pr, np, mrs, m->gemm_cls);
     // attention over every cached position of layer i
-    launch_attention(st, m->dt, m->q, Dq, m->att, Dq, act, mr, rt, m->tok_seq, m->tok_pos, m->d_seq_len, cv, l0, m->H,
-                     causal);
-    m->launches += 1;
+    {
+      cudaEvent_t b = nullptr;
+      prof_begin(m, ADEPT_PROF_ATTENTION, st, &b);
+      launch_attention(st, m->dt, m->q, Dq, m->att, Dq, act, mr, rt, m->tok_seq, m->tok_pos, m->d_seq_len, cv, l0,
+                       m->H, causal);
+      prof_end(m, ADEPT_PROF_ATTENTION, st, b, 0, 0);
+      m->launches += 1;
+    }
     // O projection + residual
     GemmProblem p;
     memset(&p, 0, sizeof p);
+    p.a_rows = m->T_max;
     p.A = m->att; p.lda = Dq; p.B = w.w_o; p.ldb = Dq; p.rows = act; p.N = D; p.K = Dq;
     p.epi = epi_base(); p.epi.kind = EPI_RESID; p.epi.bias = w.b_o; p.epi.out_f32 = m->X_out; p.epi.ld_f32 = D;
     p.epi.resid = Xi; p.epi.ld_resid = D;
-    gemm(m, st, &p, 1, &mr, ADEPT_PROF_GEMM);
+    gemm(m, st, &p, 1, &mr, m->gemm_cls);
     if (fam == ADEPT_FAMILY_BERT) {
       launch_layernorm_inplace(st, m->X_out, act, mr, D, w.ln1_g, w.ln1_b, eps);
       m->launches += 1;
@@ -697,11 +732,11 @@ static adept_status run_pass(adept_model* m, int n_tok, int batch, int prompt_le
       p.epi.act = fam == ADEPT_FAMILY_GPT2 ? ACT_GELU_TANH : ACT_GELU_ERF;
     }
     p.epi.bias = w.b_up; p.epi.out_t = m->hbuf; p.epi.ld_t = m->F;
-    gemm(m, st, &p, 1, &mr, ADEPT_PROF_GEMM);
+    gemm(m, st, &p, 1, &mr, m->gemm_cls);
     p.A = m->hbuf; p.lda = m->F; p.B = w.w_down; p.ldb = m->F; p.N = D; p.K = m->F;
     p.epi = epi_base(); p.epi.kind = EPI_RESID; p.epi.bias = w.b_down; p.epi.out_f32 = m->X_out; p.epi.ld_f32 = D;
     p.epi.resid = m->X_out; p.epi.ld_resid = D;
-    gemm(m, st, &p, 1, &mr, ADEPT_PROF_GEMM);
+    gemm(m, st, &p, 1, &mr, m->gemm_cls);
     if (fam == ADEPT_FAMILY_BERT) {
       launch_layernorm_inplace(st, m->X_out, act, mr, D, w.ln2_g, w.ln2_b, eps);
       m->launches += 1;
@@ -734,7 +769,7 @@ static adept_status run_pass(adept_model* m, int n_tok, int batch, int prompt_le
     std::vector<GemmProblem> probs;
     std::vector<int> mrs;
     for (int r = 3; r <= N; ++r) {
-      probs.push_back(kv_problem(m, r - 1, m->xfill, DevRange{nullptr, m->ctr + CTR_PREFIX + r - 1, 0}, m->exit_tok,
+      probs.push_back(kv_problem(m, r - 1, m->xfill, m->T_max, DevRange{nullptr, m->ctr + CTR_PREFIX + r - 1, 0}, m->exit_tok,
                                  m->tok_seq, m->tok_pos));
       mrs.push_back(n_tok);
     }
@@ -754,13 +789,14 @@ static adept_status run_head(adept_model* m, int batch, int prompt_len, bool dec
   const DevRange rows{nullptr, nullptr, batch};
   GemmProblem p;
   memset(&p, 0, sizeof p);
+  p.a_rows = c.max_batch;
   if (!enc) {
     launch_standardize(st, m->dt, m->final_, D, m->head_rows, rows, batch, D, attn_norm_mode(m), c.norm_eps, m->xhead,
                        D);
     m->launches += 1;
     p.A = m->xhead; p.lda = D; p.B = m->w_head; p.ldb = D; p.rows = rows; p.N = m->V; p.K = D;
     p.epi = epi_base(); p.epi.kind = EPI_F32; p.epi.bias = m->b_head; p.epi.out_f32 = out; p.epi.ld_f32 = m->V;
-    gemm(m, st, &p, 1, &batch, ADEPT_PROF_GEMM);
+    gemm(m, st, &p, 1, &batch, m->gemm_cls);
     if (next) {
       launch_argmax(st, out, m->V, batch, next);
       m->launches += 1;
@@ -771,10 +807,10 @@ static adept_status run_head(adept_model* m, int batch, int prompt_len, bool dec
     p.A = m->xhead; p.lda = D; p.B = m->w_pool; p.ldb = D; p.rows = rows; p.N = D; p.K = D;
     p.epi = epi_base(); p.epi.kind = EPI_ACT; p.epi.act = ACT_TANH; p.epi.bias = m->b_pool; p.epi.out_t = m->pool_t;
     p.epi.ld_t = D;
-    gemm(m, st, &p, 1, &batch, ADEPT_PROF_GEMM);
+    gemm(m, st, &p, 1, &batch, m->gemm_cls);
     p.A = m->pool_t; p.lda = D; p.B = m->w_cls; p.ldb = D; p.N = c.n_classes; p.K = D;
     p.epi = epi_base(); p.epi.kind = EPI_F32; p.epi.bias = m->b_cls; p.epi.out_f32 = out; p.epi.ld_f32 = c.n_classes;
-    gemm(m, st, &p, 1, &batch, ADEPT_PROF_GEMM);
+    gemm(m, st, &p, 1, &batch, m->gemm_cls);
     if (next) {
       launch_argmax(st, out, c.n_classes, batch, next);
       m->launches += 1;
@@ -823,7 +859,8 @@ adept_status adept_model_load(const adept_config* cfg_in, const adept_tensor_tab
   m->N = cfg.n_layers; m->D = cfg.d_model; m->H = cfg.n_heads; m->Hkv = cfg.n_kv_heads; m->dh = cfg.head_dim;
   m->Dq = m->H * m->dh; m->Dkv = m->Hkv * m->dh; m->F = cfg.d_ffn; m->V = cfg.vocab;
   m->m1 = cfg.hsm_m1; m->m2 = cfg.hsm_m2; m->dt = cfg.dtype; m->esz = cfg.dtype == ADEPT_DTYPE_BF16 ? 2 : 4;
-  m->T_max = cfg.max_batch * cfg.max_seq;
+  m->T_max = cfg.max_pass_tokens > 0 ? cfg.max_pass_tokens : cfg.max_batch * cfg.max_seq;
+  if (m->T_max < cfg.max_batch) m->T_max = cfg.max_batch;
   Loader ld;
   ld.m = m;
   ld.st = (cudaStream_t)stream;
@@ -878,6 +915,9 @@ adept_status adept_prefill(adept_model* m, int batch, int prompt_len, const int3
   if (prompt_len > m->cfg.max_seq)
     return fail(m, ADEPT_ERR_CAPACITY, "prompt_len %d > max_seq %d", prompt_len, m->cfg.max_seq);
   if (std::isnan(delta)) return fail(m, ADEPT_ERR_INVALID_ARG, "delta is NaN");
+  if ((long long)batch * prompt_len > m->T_max)
+    return fail(m, ADEPT_ERR_CAPACITY, "batch * prompt_len %d above the pass workspace (%d rows)", batch * prompt_len,
+                m->T_max);
   cudaStream_t st = (cudaStream_t)stream;
   std::vector<int> lens(batch, prompt_len);
   TRY(reserve_seqs(m, batch, lens.data(), st));
@@ -940,7 +980,7 @@ adept_status adept_skip_kv_fill(adept_model* m, int n_tokens, const void* d_h_ma
   std::vector<GemmProblem> probs;
   std::vector<int> mrs;
   for (int r = 2; r <= m->N; ++r) {
-    probs.push_back(kv_problem(m, r - 1, m->fill_x, DevRange{nullptr, m->fill_start + r, 0}, m->fill_tok, d_seq, d_pos));
+    probs.push_back(kv_problem(m, r - 1, m->fill_x, m->fill_cap, DevRange{nullptr, m->fill_start + r, 0}, m->fill_tok, d_seq, d_pos));
     mrs.push_back(n_tokens);
   }
   // algorithmic work of this launch is only known on the device; the benchmark supplies it

@@ -137,6 +137,7 @@ class ModelConfig:
     max_seq: int = 1024
     n_kv_heads: int = 0        # 0 -> n_heads
     kv_pool_blocks: int = 0    # 0 -> max_batch * ceil(max_seq / kv_block_tokens)
+    max_pass_tokens: int = 0   # rows of per-pass workspaces; 0 -> max_batch * max_seq
     block_shuffle_seed: int = 0  # 0: KV blocks handed out in order; else a seeded permutation
 
     def __post_init__(self):

@@ -165,3 +165,27 @@ def test_synth_generator_cpu_and_cuda_agree():
     a = synth.normal(5, "w", (3, 100003), std=0.02, dtype=torch.bfloat16)
     b = synth.normal(5, "w", (3, 100003), std=0.02, dtype=torch.bfloat16, device="cuda").cpu()
     assert torch.equal(a.view(torch.int16), b.view(torch.int16))
+
+
+def test_tensor_core_gemm_matches_simt_gemm():
+    """The tcgen05 grouped GEMM and the SIMT GEMM give the same pass (bf16 noise level),
+    on a shape with ragged M tiles (130-token prompts) and every epilogue kind."""
+    from parity_utils import row_rel_err
+    for family, kw in ((synth.LLAMA, dict(n_heads=2, head_dim=128)), (synth.GPT2, {}), (synth.BERT, {})):
+        cfg = small(family, n_layers=4, max_seq=256, max_pos=256, **kw)
+        W = synth.make_weights(cfg, seed=0)
+        m = adept.Model(cfg, W)
+        tokens = synth.make_tokens(0, 2, 130, cfg.vocab).cuda()
+        forced = synth.forced_exits_uniform(0, 260, 2, 4).view(2, 130).cuda()
+        out = {}
+        for simt in (1, 0):
+            adept.adept_set_option(m.h, adept.OPT_GEMM_SIMT, simt)
+            ex, lg, nx, sim = m.prefill(tokens, 0.5, forced)
+            m.check()
+            out[simt] = (ex.cpu().numpy(), m.final_states(260).cpu().numpy(), lg.cpu().numpy(),
+                         m.read_kv(1, 1, 0, 130)[0].float().cpu().numpy())
+        np.testing.assert_array_equal(out[0][0], out[1][0])
+        assert row_rel_err(out[0][3], out[1][3]).max() < 2e-3      # first layer's K: one GEMM
+        assert row_rel_err(out[0][1], out[1][1]).max() < 2e-2
+        assert row_rel_err(out[0][2], out[1][2]).max() < 2e-2
+        m.close()
