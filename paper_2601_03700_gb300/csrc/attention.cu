@@ -5,6 +5,8 @@
 #include "common.cuh"
 #include "kernels.h"
 
+#include <algorithm>
+
 namespace adept {
 
 // One warp per (query row, head); lanes own keys for the scores and head dimensions
@@ -65,6 +67,365 @@ __global__ void __launch_bounds__(256) attn_warp_kernel(const T* __restrict__ q,
   for (int j = 0; j < PER; ++j) out[(size_t)ra * ld_out + h * DH + lane + 32 * j] = from_f<T>(acc[j] * inv);
 }
 
+// ---------------------------------------------------------------------------
+// Prompt-pass attention, bf16 tensor cores (mma.sync m16n8k16): a CTA takes 64
+// consecutive active query rows of one head.  Active rows are sorted by (sequence,
+// position), so the tile splits into runs of one sequence; each run streams its keys
+// [0, last position] (causal) or [0, length) from the paged cache in blocks of 64,
+// with an online softmax (exp2 domain) per query row.
+// ---------------------------------------------------------------------------
+__device__ __forceinline__ void ldsm_x4(uint32_t& r0, uint32_t& r1, uint32_t& r2, uint32_t& r3, const void* p) {
+  const uint32_t a = (uint32_t)__cvta_generic_to_shared(p);
+  asm volatile("ldmatrix.sync.aligned.m8n8.x4.shared.b16 {%0, %1, %2, %3}, [%4];"
+               : "=r"(r0), "=r"(r1), "=r"(r2), "=r"(r3)
+               : "r"(a));
+}
+__device__ __forceinline__ void ldsm_x4_t(uint32_t& r0, uint32_t& r1, uint32_t& r2, uint32_t& r3, const void* p) {
+  const uint32_t a = (uint32_t)__cvta_generic_to_shared(p);
+  asm volatile("ldmatrix.sync.aligned.m8n8.x4.trans.shared.b16 {%0, %1, %2, %3}, [%4];"
+               : "=r"(r0), "=r"(r1), "=r"(r2), "=r"(r3)
+               : "r"(a));
+}
+__device__ __forceinline__ void mma_bf16_16816(float (&c)[4], uint32_t a0, uint32_t a1, uint32_t a2, uint32_t a3,
+                                               uint32_t b0, uint32_t b1) {
+  asm volatile(
+      "mma.sync.aligned.m16n8k16.row.col.f32.bf16.bf16.f32 {%0, %1, %2, %3}, {%4, %5, %6, %7}, {%8, %9}, "
+      "{%0, %1, %2, %3};"
+      : "+f"(c[0]), "+f"(c[1]), "+f"(c[2]), "+f"(c[3])
+      : "r"(a0), "r"(a1), "r"(a2), "r"(a3), "r"(b0), "r"(b1));
+}
+__device__ __forceinline__ void cp_async16(void* smem, const void* gmem) {
+  const uint32_t a = (uint32_t)__cvta_generic_to_shared(smem);
+  asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(a), "l"(gmem) : "memory");
+}
+__device__ __forceinline__ void cp_async_wait_all() {
+  asm volatile("cp.async.commit_group;\ncp.async.wait_group 0;" ::: "memory");
+}
+__device__ __forceinline__ uint32_t pack_bf16(float lo, float hi) {
+  __nv_bfloat162 h = __floats2bfloat162_rn(lo, hi);
+  return *reinterpret_cast<uint32_t*>(&h);
+}
+
+// x = hi + lo with hi = bf16(x) and lo = bf16(x - hi), for a pair of values.
+__device__ __forceinline__ void split_bf16(float x0, float x1, uint32_t& hi, uint32_t& lo) {
+  const __nv_bfloat162 h = __floats2bfloat162_rn(x0, x1);
+  const float2 hf = __bfloat1622float2(h);
+  hi = *reinterpret_cast<const uint32_t*>(&h);
+  lo = pack_bf16(x0 - hf.x, x1 - hf.y);
+}
+
+template <int DH>
+__global__ void __launch_bounds__(128) attn_prefill_mma_kernel(const bf16* __restrict__ q, int ld_q,
+                                                               bf16* __restrict__ out, int ld_out, DevRange rows,
+                                                               const int* row_tok, const int* tok_seq,
+                                                               const int* tok_pos, const int* seq_len,
+                                                               KVCacheView cache, int layer0, int n_heads, int causal,
+                                                               float scale_log2) {
+  constexpr int LDS = DH + 8;  // padded rows: conflict-free ldmatrix
+  constexpr int NB = DH / 8;   // 8-column blocks of the output
+  extern __shared__ __align__(16) uint8_t attn_smem[];
+  bf16* sQ = reinterpret_cast<bf16*>(attn_smem);
+  bf16* sK = sQ + 64 * LDS;
+  bf16* sV = sK + 64 * LDS;
+  __shared__ int s_seq[64], s_pos[64];
+
+  const int h = blockIdx.y;
+  const int kvh = h / (n_heads / cache.n_kv_heads);
+  const int r0 = rows.b() + blockIdx.x * 64;
+  const int rend = rows.e();
+  if (r0 >= rend) return;
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const int g = lane >> 2, t4 = lane & 3;
+  if (tid < 64) {
+    const int r = r0 + tid;
+    if (r < rend) {
+      const int tok = row_tok[r];
+      s_seq[tid] = tok_seq[tok];
+      s_pos[tid] = tok_pos[tok];
+    } else {
+      s_seq[tid] = -1;
+      s_pos[tid] = -1;
+    }
+  }
+  // Q tile (rows past the range are zero)
+  for (int c = tid; c < 64 * (DH / 8); c += 128) {
+    const int rr = c / (DH / 8), cc = (c % (DH / 8)) * 8;
+    bf16* dst = sQ + rr * LDS + cc;
+    if (r0 + rr < rend) cp_async16(dst, q + (size_t)(r0 + rr) * ld_q + h * DH + cc);
+    else *reinterpret_cast<uint4*>(dst) = make_uint4(0, 0, 0, 0);
+  }
+  cp_async_wait_all();
+  __syncthreads();
+  const bf16* Kp = (const bf16*)cache.k;
+  const bf16* Vp = (const bf16*)cache.v;
+
+  int a = 0;
+  while (a < 64 && s_seq[a] >= 0) {
+    const int sq = s_seq[a];
+    int b = a;
+    while (b < 64 && s_seq[b] == sq) ++b;
+    const int kend = causal ? s_pos[b - 1] + 1 : seq_len[sq];
+    // this warp's two rows per thread (tile rows 16 warp + g, + 8)
+    const int ra_ = warp * 16 + g, rb_ = ra_ + 8;
+    const bool va = ra_ >= a && ra_ < b, vb = rb_ >= a && rb_ < b;
+    const int pa = va ? s_pos[ra_] : -1, pb = vb ? s_pos[rb_] : -1;
+    const bool warp_active = (warp * 16 < b) && (warp * 16 + 16 > a);
+    // Q fragments of this warp (16 rows x DH)
+    uint32_t qf[DH / 16][4];
+#pragma unroll
+    for (int kk = 0; kk < DH / 16; ++kk) {
+      const int mi = lane >> 3;
+      const int row = warp * 16 + (mi & 1) * 8 + (lane & 7);
+      const int col = kk * 16 + (mi >> 1) * 8;
+      ldsm_x4(qf[kk][0], qf[kk][1], qf[kk][2], qf[kk][3], sQ + row * LDS + col);
+    }
+    float o[NB][4];
+#pragma unroll
+    for (int nb = 0; nb < NB; ++nb) o[nb][0] = o[nb][1] = o[nb][2] = o[nb][3] = 0.f;
+    float m0 = -INFINITY, m1 = -INFINITY, l0 = 0.f, l1 = 0.f;
+
+    for (int kb = 0; kb < kend; kb += 64) {
+      __syncthreads();  // previous K/V tile fully consumed
+      for (int c = tid; c < 64 * (DH / 8); c += 128) {
+        const int j = c / (DH / 8), cc = (c % (DH / 8)) * 8;
+        const int p = kb + j;
+        bf16* dk = sK + j * LDS + cc;
+        bf16* dv = sV + j * LDS + cc;
+        if (p < kend) {
+          const size_t off = cache.offset(layer0, sq, p, kvh) + cc;
+          cp_async16(dk, Kp + off);
+          cp_async16(dv, Vp + off);
+        } else {
+          *reinterpret_cast<uint4*>(dk) = make_uint4(0, 0, 0, 0);
+          *reinterpret_cast<uint4*>(dv) = make_uint4(0, 0, 0, 0);
+        }
+      }
+      cp_async_wait_all();
+      __syncthreads();
+      if (!warp_active) continue;
+      // S = Q K^T for 64 keys (8 blocks of 8)
+      float s[8][4];
+#pragma unroll
+      for (int nb = 0; nb < 8; ++nb) s[nb][0] = s[nb][1] = s[nb][2] = s[nb][3] = 0.f;
+#pragma unroll
+      for (int kk = 0; kk < DH / 16; ++kk) {
+#pragma unroll
+        for (int np = 0; np < 4; ++np) {  // pairs of key blocks (16 keys)
+          const int mi = lane >> 3;
+          const int key = np * 16 + (mi >> 1) * 8 + (lane & 7);
+          const int col = kk * 16 + (mi & 1) * 8;
+          uint32_t b0, b1, b2, b3;
+          ldsm_x4(b0, b1, b2, b3, sK + key * LDS + col);
+          mma_bf16_16816(s[2 * np], qf[kk][0], qf[kk][1], qf[kk][2], qf[kk][3], b0, b1);
+          mma_bf16_16816(s[2 * np + 1], qf[kk][0], qf[kk][1], qf[kk][2], qf[kk][3], b2, b3);
+        }
+      }
+      // mask and online softmax (two rows per thread)
+      float mx0 = -INFINITY, mx1 = -INFINITY;
+#pragma unroll
+      for (int nb = 0; nb < 8; ++nb) {
+#pragma unroll
+        for (int e = 0; e < 2; ++e) {
+          const int key = kb + nb * 8 + 2 * t4 + e;
+          const bool ka = va && key < kend && (!causal || key <= pa);
+          const bool kb_ = vb && key < kend && (!causal || key <= pb);
+          s[nb][e] = ka ? s[nb][e] * scale_log2 : -INFINITY;
+          s[nb][2 + e] = kb_ ? s[nb][2 + e] * scale_log2 : -INFINITY;
+          mx0 = fmaxf(mx0, s[nb][e]);
+          mx1 = fmaxf(mx1, s[nb][2 + e]);
+        }
+      }
+      mx0 = fmaxf(mx0, __shfl_xor_sync(0xffffffffu, mx0, 1));
+      mx0 = fmaxf(mx0, __shfl_xor_sync(0xffffffffu, mx0, 2));
+      mx1 = fmaxf(mx1, __shfl_xor_sync(0xffffffffu, mx1, 1));
+      mx1 = fmaxf(mx1, __shfl_xor_sync(0xffffffffu, mx1, 2));
+      const float mn0 = fmaxf(m0, mx0), mn1 = fmaxf(m1, mx1);
+      const float c0 = (mn0 == -INFINITY) ? 1.f : exp2f(m0 - mn0);
+      const float c1 = (mn1 == -INFINITY) ? 1.f : exp2f(m1 - mn1);
+      float sum0 = 0.f, sum1 = 0.f;
+#pragma unroll
+      for (int nb = 0; nb < 8; ++nb) {
+#pragma unroll
+        for (int e = 0; e < 2; ++e) {
+          const float p0 = (s[nb][e] == -INFINITY) ? 0.f : exp2f(s[nb][e] - mn0);
+          const float p1 = (s[nb][2 + e] == -INFINITY) ? 0.f : exp2f(s[nb][2 + e] - mn1);
+          s[nb][e] = p0;
+          s[nb][2 + e] = p1;
+          sum0 += p0;
+          sum1 += p1;
+        }
+      }
+      sum0 += __shfl_xor_sync(0xffffffffu, sum0, 1);
+      sum0 += __shfl_xor_sync(0xffffffffu, sum0, 2);
+      sum1 += __shfl_xor_sync(0xffffffffu, sum1, 1);
+      sum1 += __shfl_xor_sync(0xffffffffu, sum1, 2);
+      l0 = l0 * c0 + sum0;
+      l1 = l1 * c1 + sum1;
+      m0 = mn0;
+      m1 = mn1;
+#pragma unroll
+      for (int nb = 0; nb < NB; ++nb) {
+        o[nb][0] *= c0;
+        o[nb][1] *= c0;
+        o[nb][2] *= c1;
+        o[nb][3] *= c1;
+      }
+      // O += P V, with P = hi + lo (two bf16 terms) so the probabilities keep ~16 bits
+#pragma unroll
+      for (int kc = 0; kc < 4; ++kc) {  // 16 keys per step
+        uint32_t ah[4], al[4];
+        split_bf16(s[2 * kc][0], s[2 * kc][1], ah[0], al[0]);
+        split_bf16(s[2 * kc][2], s[2 * kc][3], ah[1], al[1]);
+        split_bf16(s[2 * kc + 1][0], s[2 * kc + 1][1], ah[2], al[2]);
+        split_bf16(s[2 * kc + 1][2], s[2 * kc + 1][3], ah[3], al[3]);
+#pragma unroll
+        for (int np = 0; np < NB / 2; ++np) {  // pairs of 8-column output blocks
+          const int mi = lane >> 3;
+          const int key = kc * 16 + (mi & 1) * 8 + (lane & 7);
+          const int col = np * 16 + (mi >> 1) * 8;
+          uint32_t b0, b1, b2, b3;
+          ldsm_x4_t(b0, b1, b2, b3, sV + key * LDS + col);
+          mma_bf16_16816(o[2 * np], ah[0], ah[1], ah[2], ah[3], b0, b1);
+          mma_bf16_16816(o[2 * np + 1], ah[0], ah[1], ah[2], ah[3], b2, b3);
+          mma_bf16_16816(o[2 * np], al[0], al[1], al[2], al[3], b0, b1);
+          mma_bf16_16816(o[2 * np + 1], al[0], al[1], al[2], al[3], b2, b3);
+        }
+      }
+    }
+    // normalise and write this warp's rows of the run
+    const float i0 = l0 > 0.f ? 1.f / l0 : 0.f, i1 = l1 > 0.f ? 1.f / l1 : 0.f;
+#pragma unroll
+    for (int nb = 0; nb < NB; ++nb) {
+      const int col = h * DH + nb * 8 + 2 * t4;
+      if (va) *reinterpret_cast<uint32_t*>(out + (size_t)(r0 + ra_) * ld_out + col) = pack_bf16(o[nb][0] * i0, o[nb][1] * i0);
+      if (vb) *reinterpret_cast<uint32_t*>(out + (size_t)(r0 + rb_) * ld_out + col) = pack_bf16(o[nb][2] * i1, o[nb][3] * i1);
+    }
+    a = b;
+  }
+}
+
+// ---------------------------------------------------------------------------
+// Generation-step attention (one query row per sequence), split over the keys:
+// CTA (row, head, split) covers a key chunk with 4 warps; in a warp, 8 keys at a time,
+// 4 lanes per key each owning DH/4 head dimensions.  Partial (max, sum, output) per
+// split go to a workspace and a second kernel merges them.
+// ---------------------------------------------------------------------------
+template <typename T, int DH>
+__global__ void __launch_bounds__(128) attn_decode_split_kernel(const T* __restrict__ q, int ld_q, DevRange rows,
+                                                                const int* row_tok, const int* tok_seq,
+                                                                const int* tok_pos, const int* seq_len,
+                                                                KVCacheView cache, int layer0, int n_heads, int causal,
+                                                                float scale_log2, int chunk, int n_split,
+                                                                float* ws) {
+  constexpr int PD = DH / 4;   // dimensions per lane
+  __shared__ float sm_m[4], sm_l[4];
+  __shared__ float sm_o[4][DH];
+  const int rh = blockIdx.x, split = blockIdx.y;
+  const int r = rows.b() + rh / n_heads, h = rh % n_heads;
+  if (r >= rows.e()) return;
+  const int kvh = h / (n_heads / cache.n_kv_heads);
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const int gk = lane >> 2, j = lane & 3;
+  const int tok = row_tok[r];
+  const int sq = tok_seq[tok], pos = tok_pos[tok];
+  const int nk = causal ? pos + 1 : seq_len[sq];
+  const int k_lo = split * chunk, k_hi = min(nk, k_lo + chunk);
+  float* w = ws + ((size_t)rh * n_split + split) * (DH + 2);
+  float qv[PD];
+#pragma unroll
+  for (int d = 0; d < PD; ++d) qv[d] = to_f(q[(size_t)r * ld_q + h * DH + j * PD + d]) * scale_log2;
+  const T* Kp = (const T*)cache.k;
+  const T* Vp = (const T*)cache.v;
+  float m = -INFINITY, l = 0.f, o[PD];
+#pragma unroll
+  for (int d = 0; d < PD; ++d) o[d] = 0.f;
+  for (int k0 = k_lo + warp * 8; k0 < k_hi; k0 += 32) {
+    const int key = k0 + gk;
+    const bool valid = key < k_hi;
+    float sc = 0.f;
+    size_t off = 0;
+    if (valid) {
+      off = cache.offset(layer0, sq, key, kvh) + j * PD;
+#pragma unroll
+      for (int d = 0; d < PD; ++d) sc = fmaf(qv[d], to_f(Kp[off + d]), sc);
+    }
+    sc += __shfl_xor_sync(0xffffffffu, sc, 1);
+    sc += __shfl_xor_sync(0xffffffffu, sc, 2);
+    if (!valid) sc = -INFINITY;
+    float mx = sc;
+    mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, 4));
+    mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, 8));
+    mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, 16));
+    const float mn = fmaxf(m, mx);
+    const float corr = (m == -INFINITY) ? 0.f : exp2f(m - mn);
+    const float p = valid ? exp2f(sc - mn) : 0.f;
+    float ps = p;
+    ps += __shfl_xor_sync(0xffffffffu, ps, 4);
+    ps += __shfl_xor_sync(0xffffffffu, ps, 8);
+    ps += __shfl_xor_sync(0xffffffffu, ps, 16);
+    l = l * corr + ps;
+#pragma unroll
+    for (int d = 0; d < PD; ++d) o[d] = o[d] * corr + (valid ? p * to_f(Vp[off + d]) : 0.f);
+    m = mn;
+  }
+  // sum the 8 key groups of the warp
+#pragma unroll
+  for (int d = 0; d < PD; ++d) {
+    o[d] += __shfl_xor_sync(0xffffffffu, o[d], 4);
+    o[d] += __shfl_xor_sync(0xffffffffu, o[d], 8);
+    o[d] += __shfl_xor_sync(0xffffffffu, o[d], 16);
+  }
+  if (lane == 0) {
+    sm_m[warp] = m;
+    sm_l[warp] = l;
+  }
+  if (gk == 0) {
+#pragma unroll
+    for (int d = 0; d < PD; ++d) sm_o[warp][j * PD + d] = o[d];
+  }
+  __syncthreads();
+  float M = fmaxf(fmaxf(sm_m[0], sm_m[1]), fmaxf(sm_m[2], sm_m[3]));
+  for (int d = tid; d < DH; d += 128) {
+    float acc = 0.f;
+#pragma unroll
+    for (int k = 0; k < 4; ++k)
+      if (sm_m[k] != -INFINITY) acc += exp2f(sm_m[k] - M) * sm_o[k][d];
+    w[d] = acc;
+  }
+  if (tid == 0) {
+    float L = 0.f;
+    for (int k = 0; k < 4; ++k)
+      if (sm_m[k] != -INFINITY) L += exp2f(sm_m[k] - M) * sm_l[k];
+    w[DH] = M;
+    w[DH + 1] = L;
+  }
+}
+
+template <typename T, int DH>
+__global__ void attn_decode_combine_kernel(DevRange rows, int n_heads, int n_split, const float* ws, T* out,
+                                           int ld_out) {
+  const int rh = blockIdx.x;
+  const int r = rows.b() + rh / n_heads, h = rh % n_heads;
+  if (r >= rows.e()) return;
+  const float* w = ws + (size_t)rh * n_split * (DH + 2);
+  float M = -INFINITY;
+  for (int s = 0; s < n_split; ++s) M = fmaxf(M, w[s * (DH + 2) + DH]);
+  float L = 0.f;
+  for (int s = 0; s < n_split; ++s) {
+    const float ms = w[s * (DH + 2) + DH];
+    if (ms != -INFINITY) L += exp2f(ms - M) * w[s * (DH + 2) + DH + 1];
+  }
+  const float inv = L > 0.f ? 1.f / L : 0.f;
+  for (int d = threadIdx.x; d < DH; d += blockDim.x) {
+    float acc = 0.f;
+    for (int s = 0; s < n_split; ++s) {
+      const float ms = w[s * (DH + 2) + DH];
+      if (ms != -INFINITY) acc += exp2f(ms - M) * w[s * (DH + 2) + d];
+    }
+    out[(size_t)r * ld_out + h * DH + d] = from_f<T>(acc * inv);
+  }
+}
+
 template <typename T>
 static void attn_dispatch(cudaStream_t st, const void* q, int ld_q, void* out, int ld_out, DevRange rows,
                           int max_rows, const int* row_tok, const int* tok_seq, const int* tok_pos,
@@ -87,10 +448,60 @@ static void attn_dispatch(cudaStream_t st, const void* q, int ld_q, void* out, i
 #undef ATT_CASE
 }
 
+static int g_attn_smem_set[2] = {0, 0};
+
 void launch_attention(cudaStream_t st, int dt, const void* q, int ld_q, void* out, int ld_out, DevRange rows,
                       int max_rows, const int* row_tok, const int* tok_seq, const int* tok_pos, const int* seq_len,
-                      KVCacheView cache, int layer0, int n_heads, int causal) {
+                      KVCacheView cache, int layer0, int n_heads, int causal, int decode_keys, float* ws) {
   if (max_rows <= 0) return;
+  const int dh = cache.head_dim;
+  const float scale_log2 = 1.4426950408889634f / sqrtf((float)dh);
+  if (decode_keys > 0 && ws && (dh == 64 || dh == 128)) {
+    // generation step: split the keys so that rows x heads x splits covers the GPU twice
+    int n_split = (2 * 152 + max_rows * n_heads - 1) / (max_rows * n_heads);
+    n_split = std::max(1, std::min(n_split, ATTN_MAX_SPLIT));
+    int chunk = (decode_keys + n_split - 1) / n_split;
+    chunk = std::max(32, ((chunk + 31) / 32) * 32);
+    n_split = (decode_keys + chunk - 1) / chunk;
+    dim3 grid(max_rows * n_heads, n_split);
+#define DEC_CASE(T, D)                                                                                       \
+  {                                                                                                          \
+    attn_decode_split_kernel<T, D><<<grid, 128, 0, st>>>((const T*)q, ld_q, rows, row_tok, tok_seq, tok_pos, \
+                                                         seq_len, cache, layer0, n_heads, causal, scale_log2, \
+                                                         chunk, n_split, ws);                                \
+    attn_decode_combine_kernel<T, D><<<max_rows * n_heads, 128, 0, st>>>(rows, n_heads, n_split, ws, (T*)out, \
+                                                                         ld_out);                           \
+  }
+    if (dt == 1) {
+      if (dh == 64) DEC_CASE(bf16, 64) else DEC_CASE(bf16, 128)
+    } else {
+      if (dh == 64) DEC_CASE(float, 64) else DEC_CASE(float, 128)
+    }
+#undef DEC_CASE
+    return;
+  }
+  if (dt == 1 && (dh == 64 || dh == 128)) {
+    const int smem = 3 * 64 * (dh + 8) * 2;
+    dim3 grid(cdiv(max_rows, 64), n_heads);
+    if (dh == 64) {
+      if (!g_attn_smem_set[0]) {
+        cudaFuncSetAttribute(attn_prefill_mma_kernel<64>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+        g_attn_smem_set[0] = 1;
+      }
+      attn_prefill_mma_kernel<64><<<grid, 128, smem, st>>>((const bf16*)q, ld_q, (bf16*)out, ld_out, rows, row_tok,
+                                                           tok_seq, tok_pos, seq_len, cache, layer0, n_heads, causal,
+                                                           scale_log2);
+    } else {
+      if (!g_attn_smem_set[1]) {
+        cudaFuncSetAttribute(attn_prefill_mma_kernel<128>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+        g_attn_smem_set[1] = 1;
+      }
+      attn_prefill_mma_kernel<128><<<grid, 128, smem, st>>>((const bf16*)q, ld_q, (bf16*)out, ld_out, rows, row_tok,
+                                                            tok_seq, tok_pos, seq_len, cache, layer0, n_heads, causal,
+                                                            scale_log2);
+    }
+    return;
+  }
   if (dt == 1)
     attn_dispatch<bf16>(st, q, ld_q, out, ld_out, rows, max_rows, row_tok, tok_seq, tok_pos, seq_len, cache, layer0,
                         n_heads, causal);

@@ -52,8 +52,11 @@ void launch_read_kv(cudaStream_t st, int dt, KVCacheView c, int layer0, int seq,
 // GEMMs.  SIMT path: C = A B^T into fp32 scratch, then the epilogue kernel.
 void launch_gemm_simt(cudaStream_t st, int dt, const GemmProblem& p, int max_rows, float* scratch);
 // Attention of the active query rows over the paged cache of one layer.
+// decode_keys > 0 (generation step, one query row per sequence): split-KV kernel over at
+// most decode_keys keys, using ws (>= rows * heads * ATTN_MAX_SPLIT * (head_dim + 2) floats).
+constexpr int ATTN_MAX_SPLIT = 32;
 void launch_attention(cudaStream_t st, int dt, const void* q, int ld_q, void* out, int ld_out, DevRange rows,
                       int max_rows, const int* row_tok, const int* tok_seq, const int* tok_pos, const int* seq_len,
-                      KVCacheView cache, int layer0, int n_heads, int causal);
+                      KVCacheView cache, int layer0, int n_heads, int causal, int decode_keys, float* ws);
 
 }  // namespace adept

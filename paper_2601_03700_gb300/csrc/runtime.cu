@@ -84,6 +84,7 @@ struct adept_model {
   void* xhead = nullptr;
   void* pool_t = nullptr;
   float* logits_ws = nullptr;
+  float* attn_ws = nullptr;
   float* scratch = nullptr;
   size_t scratch_elems = 0;
   // skipped-layer fill workspace (adept_skip_kv_fill)
@@ -548,6 +549,7 @@ static adept_status alloc_runtime(adept_model* m) {
   TRY(dalloc(m, &m->pool_t, (size_t)c.max_batch * D * m->esz));
   const int nout = c.family == ADEPT_FAMILY_BERT ? c.n_classes : m->V;
   TRY(dalloc_t(m, &m->logits_ws, (size_t)c.max_batch * nout));
+  TRY(dalloc_t(m, &m->attn_ws, (size_t)c.max_batch * m->H * ATTN_MAX_SPLIT * (m->dh + 2)));
   // SIMT scratch: the widest GEMM output of any pass step
   size_t w = std::max({(size_t)m->Dq + 2 * m->Dkv, (size_t)m->L[0].up_rows, (size_t)m->m1, (size_t)m->m2, (size_t)D});
   m->scratch_elems = std::max(w * T, (size_t)c.max_batch * nout);
@@ -668,6 +670,9 @@ static adept_status run_pass(adept_model* m, int n_tok, int batch, int prompt_le
   m->launches += 3;
   const KVCacheView cv = cache_view(m);
   const int causal = fam != ADEPT_FAMILY_BERT;
+  int decode_keys = 0;  // generation step: longest key range (the new position included)
+  if (decode)
+    for (int b = 0; b < batch; ++b) decode_keys = std::max(decode_keys, m->h_seq_len[b] + 1);
   int par = 0;
   for (int i = 1; i <= N; ++i) {
     const int l0 = i - 1;
@@ -704,7 +709,7 @@ static adept_status run_pass(adept_model* m, int n_tok, int batch, int prompt_le
       cudaEvent_t b = nullptr;
       prof_begin(m, ADEPT_PROF_ATTENTION, st, &b);
       launch_attention(st, m->dt, m->q, Dq, m->att, Dq, act, mr, rt, m->tok_seq, m->tok_pos, m->d_seq_len, cv, l0,
-                       m->H, causal);
+                       m->H, causal, decode_keys, m->attn_ws);
       prof_end(m, ADEPT_PROF_ATTENTION, st, b, 0, 0);
       m->launches += 1;
     }
