@@ -184,9 +184,15 @@ ADEPT_API adept_status adept_read_final_states(adept_model* m, float* d_out, int
 ADEPT_API adept_status adept_check_device_status(adept_model* m, void* stream);
 
 /* Options (ADEPT_OPT_*).  HSM_IDENTITY=1 replaces the HSM by s~ = s_i* (test switch).
- * PROFILE=1 records CUDA events around every launch of the grouped GEMM so that
- * adept_profile_read can report its launch count and total device time. */
-enum { ADEPT_OPT_HSM_IDENTITY = 1, ADEPT_OPT_PROFILE = 2, ADEPT_OPT_GEMM_SIMT = 3 };
+ * PROFILE=1 records CUDA events around the GEMM, fill and attention launches so that
+ * adept_profile_read can report launch counts and device time per kernel class
+ * (generation steps then run as direct launches).  GEMM_SIMT=1 routes GEMMs to the
+ * SIMT kernels (cross-check).  DECODE_GRAPH (default 1): from its second call with a
+ * given batch size, adept_decode_step replays a CUDA graph of the step captured once;
+ * 0 launches every kernel directly.  SKINNY_GEMM (default 0): GEMMs of at most 32 rows
+ * use the split-K skinny kernel instead of the tcgen05 kernel. */
+enum { ADEPT_OPT_HSM_IDENTITY = 1, ADEPT_OPT_PROFILE = 2, ADEPT_OPT_GEMM_SIMT = 3, ADEPT_OPT_DECODE_GRAPH = 4,
+       ADEPT_OPT_SKINNY_GEMM = 5 };
 ADEPT_API adept_status adept_set_option(adept_model* m, int option, int value);
 
 /* Kernel classes reported by adept_profile_read: the GEMMs of prompt passes (layer

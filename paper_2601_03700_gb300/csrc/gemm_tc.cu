@@ -16,6 +16,7 @@
 #include <cudaTypedefs.h>
 
 #include <mutex>
+#include <unordered_map>
 
 namespace adept {
 
@@ -34,8 +35,9 @@ struct TcGroup {
   Epi epi;
 };
 
+template <int MAXG>
 struct TcParams {
-  TcGroup g[TC_MAXG];
+  TcGroup g[MAXG];
   int n_groups;
   unsigned* err;
 };
@@ -146,8 +148,8 @@ __device__ __forceinline__ constexpr uint32_t idesc_bf16() {
 }
 
 // ---------------------------------------------------------------------------- kernel
-template <int BN, int STAGES>
-__global__ void __launch_bounds__(TC_THREADS, 1) gemm_tc_kernel(const __grid_constant__ TcParams p) {
+template <int BN, int STAGES, int MAXG>
+__global__ void __launch_bounds__(TC_THREADS, 1) gemm_tc_kernel(const __grid_constant__ TcParams<MAXG> p) {
   constexpr int A_BYTES = TC_BM * TC_BK * 2;
   constexpr int B_BYTES = BN * TC_BK * 2;
   constexpr uint32_t TX = A_BYTES + B_BYTES;
@@ -166,8 +168,8 @@ __global__ void __launch_bounds__(TC_THREADS, 1) gemm_tc_kernel(const __grid_con
   uint32_t* tmem_slot = (uint32_t*)(drain + 1);
   volatile int* abort_flag = (volatile int*)(tmem_slot + 1);
 
-  __shared__ int s_tile0[TC_MAXG + 1];
-  __shared__ int s_mbeg[TC_MAXG], s_M[TC_MAXG], s_tn[TC_MAXG];
+  __shared__ int s_tile0[MAXG + 1];
+  __shared__ int s_mbeg[MAXG], s_M[MAXG], s_tn[MAXG];
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int ng = p.n_groups;
@@ -365,40 +367,66 @@ bool tc_gemm_supported() {
   return g_encode != nullptr && g_cc_major == 10;
 }
 
+struct MapKey {
+  const void* base;
+  uint64_t inner, outer, row_bytes;
+  uint32_t box;
+  bool operator==(const MapKey& o) const {
+    return base == o.base && inner == o.inner && outer == o.outer && row_bytes == o.row_bytes && box == o.box;
+  }
+};
+struct MapKeyHash {
+  size_t operator()(const MapKey& k) const {
+    size_t h = std::hash<const void*>()(k.base);
+    h ^= std::hash<uint64_t>()(k.inner * 1315423911u + k.outer) + 0x9e3779b97f4a7c15ULL + (h << 6) + (h >> 2);
+    h ^= std::hash<uint64_t>()(k.row_bytes * 2654435761u + k.box) + (h << 6) + (h >> 2);
+    return h;
+  }
+};
+
+// Tensor maps are encoded once per (address, extent, stride, box) and reused by later
+// launches; a map depends on nothing else, so a reused address with the same extent
+// maps the same way.
 static bool make_map(CUtensorMap* m, const void* base, uint64_t inner, uint64_t outer, uint64_t row_bytes,
                      uint32_t box_outer) {
   if (((uintptr_t)base & 15) || (row_bytes & 15) || outer == 0 || inner == 0) return false;
+  static std::unordered_map<MapKey, CUtensorMap, MapKeyHash> cache;
+  static std::mutex mu;
+  const MapKey key{base, inner, outer, row_bytes, box_outer};
+  std::lock_guard<std::mutex> lock(mu);
+  auto it = cache.find(key);
+  if (it != cache.end()) {
+    *m = it->second;
+    return true;
+  }
   cuuint64_t dims[2] = {inner, outer};
   cuuint64_t strides[1] = {row_bytes};
   cuuint32_t box[2] = {(cuuint32_t)TC_BK, box_outer};
   cuuint32_t estr[2] = {1, 1};
-  return g_encode(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), dims, strides, box, estr,
-                  CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
-                  CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+  if (g_encode(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), dims, strides, box, estr,
+               CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+               CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
+    return false;
+  if (cache.size() > 65536) cache.clear();
+  cache.emplace(key, *m);
+  return true;
 }
 
-template <int BN, int STAGES>
-static int launch_bn(cudaStream_t st, const TcParams& prm, int grid) {
+template <int BN, int STAGES, int MAXG>
+static int launch_bn(cudaStream_t st, const TcParams<MAXG>& prm, int grid) {
   constexpr size_t smem = (size_t)STAGES * (TC_BM + BN) * TC_BK * 2 + 1024 + 256;
   static bool attr = false;
   if (!attr) {
-    cudaFuncSetAttribute(gemm_tc_kernel<BN, STAGES>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    cudaFuncSetAttribute(gemm_tc_kernel<BN, STAGES, MAXG>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     attr = true;
   }
-  gemm_tc_kernel<BN, STAGES><<<grid, TC_THREADS, smem, st>>>(prm);
+  gemm_tc_kernel<BN, STAGES, MAXG><<<grid, TC_THREADS, smem, st>>>(prm);
   return 1;
 }
 
-int tc_gemm_grouped(cudaStream_t st, const GemmProblem* probs, int n_probs, const int* max_rows, unsigned* err_word) {
-  init_once();
-  if (n_probs <= 0) return 0;
-  if (n_probs > TC_MAXG) return -1;
-  // the cache / SwiGLU epilogues work on whole 32-column chunks
-  for (int i = 0; i < n_probs; ++i) {
-    const GemmProblem& q = probs[i];
-    if (q.K % 8 || q.lda % 8 || q.ldb % 8 || q.a_rows <= 0) return -1;
-    if ((q.epi.kind == EPI_QKV || q.epi.kind == EPI_KV || q.epi.kind == EPI_SWIGLU) && (q.N % 32)) return -1;
-  }
+template <int MAXG>
+static int launch_grouped(cudaStream_t st, const GemmProblem* probs, int n_probs, const int* max_rows,
+                          unsigned* err_word) {
   // tile width: the widest that still gives every SM a tile
   long long tiles[4] = {0, 0, 0, 0};
   const int bns[4] = {256, 128, 64, 32};
@@ -413,7 +441,7 @@ int tc_gemm_grouped(cudaStream_t st, const GemmProblem* probs, int n_probs, cons
       break;
     }
   const int BN = bns[pick];
-  static TcParams prm;  // large: keep off the stack (calls on a model are serialised)
+  static TcParams<MAXG> prm;  // kept off the stack; calls on a model are serialised
   memset(&prm, 0, sizeof prm);
   prm.n_groups = n_probs;
   prm.err = err_word;
@@ -430,11 +458,26 @@ int tc_gemm_grouped(cudaStream_t st, const GemmProblem* probs, int n_probs, cons
   const int grid = (int)std::min<long long>(tiles[pick], (long long)g_num_sms);
   if (grid <= 0) return 0;
   switch (BN) {
-    case 256: return launch_bn<256, 4>(st, prm, grid);
-    case 128: return launch_bn<128, 6>(st, prm, grid);
-    case 64: return launch_bn<64, 8>(st, prm, grid);
-    default: return launch_bn<32, 10>(st, prm, grid);
+    case 256: return launch_bn<256, 4, MAXG>(st, prm, grid);
+    case 128: return launch_bn<128, 6, MAXG>(st, prm, grid);
+    case 64: return launch_bn<64, 8, MAXG>(st, prm, grid);
+    default: return launch_bn<32, 10, MAXG>(st, prm, grid);
   }
+}
+
+int tc_gemm_grouped(cudaStream_t st, const GemmProblem* probs, int n_probs, const int* max_rows, unsigned* err_word) {
+  init_once();
+  if (n_probs <= 0) return 0;
+  if (n_probs > TC_MAXG) return -1;
+  // the cache / SwiGLU epilogues work on whole 32-column chunks
+  for (int i = 0; i < n_probs; ++i) {
+    const GemmProblem& q = probs[i];
+    if (q.K % 8 || q.lda % 8 || q.ldb % 8 || q.a_rows <= 0) return -1;
+    if ((q.epi.kind == EPI_QKV || q.epi.kind == EPI_KV || q.epi.kind == EPI_SWIGLU) && (q.N % 32)) return -1;
+  }
+  // small launches carry a small parameter block (cheaper to launch)
+  if (n_probs <= 2) return launch_grouped<2>(st, probs, n_probs, max_rows, err_word);
+  return launch_grouped<TC_MAXG>(st, probs, n_probs, max_rows, err_word);
 }
 
 }  // namespace adept

@@ -22,8 +22,15 @@ void launch_standardize(cudaStream_t st, int dt, const float* X, int ldx, const 
 void launch_layernorm_inplace(cudaStream_t st, float* X, DevRange rows, int max_rows, int D, const float* g,
                               const float* b, float eps);
 void launch_exit_decide(cudaStream_t st, const float* Xout, const float* I, int D, DevRange rows, int max_rows,
-                        const int* row_tok, const int* forced, int layer, int n_layers, float delta, int test,
+                        const int* row_tok, const int* forced, int layer, int n_layers, const float* delta_p, int test,
                         float* sim, int* flag, float* inv_norm, unsigned* err);
+// Test + compaction + moves in one CTA for passes of at most EXIT_SMALL_MAX rows.
+constexpr int EXIT_SMALL_MAX = 256;
+void launch_exit_small(cudaStream_t st, const float* Xin, const float* Xout, const float* I, int first, int D,
+                       int* ctr, int par, const int* row_tok, int* row_tok_next, const int* forced, int layer,
+                       int n_layers, const float* delta_p, int test, float* sim, int* exit_tok, int* exit_layer_out,
+                       float* Xnext, float* Inext, float* hsm_s, float* hsm_prev, float* hsm_I, unsigned* err);
+void launch_set_float(cudaStream_t st, float* p, float v);
 void launch_exit_scan(cudaStream_t st, int* ctr, int in_parity, const int* flag, const int* row_tok,
                       int* row_tok_next, int* exit_tok, int* dst, int* exit_layer_out, int layer);
 void launch_exit_move(cudaStream_t st, const float* Xin, const float* Xout, const float* I, int first, int D,

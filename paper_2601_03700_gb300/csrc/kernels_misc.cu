@@ -123,8 +123,8 @@ __global__ void layernorm_inplace_kernel(float* X, DevRange rows, int D, const f
 // exit test (Sec. 4.1): c = <s_i, I> / (|s_i| |I|) vs delta, or the forced layer
 // ---------------------------------------------------------------------------
 __global__ void exit_decide_kernel(const float* Xout, const float* I, int D, DevRange rows, const int* row_tok,
-                                   const int* forced, int layer, int n_layers, float delta, int test, float* sim,
-                                   int* flag, float* inv_norm, unsigned* err) {
+                                   const int* forced, int layer, int n_layers, const float* delta_p, int test,
+                                   float* sim, int* flag, float* inv_norm, unsigned* err) {
   const int warp = (blockIdx.x * blockDim.x + threadIdx.x) >> 5, lane = threadIdx.x & 31;
   const int r = warp;
   if (r >= rows.e()) return;
@@ -148,7 +148,7 @@ __global__ void exit_decide_kernel(const float* Xout, const float* I, int D, Dev
     if (sim) sim[(size_t)tok * n_layers + (layer - 1)] = c;
     const int f = forced ? forced[tok] : 0;
     if (f != 0 && (f < 2 || f > n_layers)) atomicOr(err, ERRW_FORCED);
-    ex = (f > 0) ? (f == layer) : (c >= delta);
+    ex = (f > 0) ? (f == layer) : (c >= *delta_p);
   }
   flag[r] = ex;
   inv_norm[r] = ns > 0.f ? rsqrtf(ns) : 0.f;
@@ -237,6 +237,106 @@ __global__ void exit_move_kernel(const float* Xin, const float* Xout, const floa
     }
   }
 }
+
+// The three steps above in one CTA, for passes with at most EXIT_SMALL_MAX active rows
+// (generation steps): the similarity test, the stable compaction and the row moves.
+__global__ void __launch_bounds__(256) exit_small_kernel(const float* Xin, const float* Xout, const float* I,
+                                                         int first, int D, int* ctr, int par, const int* row_tok,
+                                                         int* row_tok_next, const int* forced, int layer,
+                                                         int n_layers, const float* delta_p, int test, float* sim,
+                                                         int* exit_tok, int* exit_layer_out, float* Xnext,
+                                                         float* Inext, float* hsm_s, float* hsm_prev, float* hsm_I,
+                                                         unsigned* err) {
+  __shared__ int s_dst[EXIT_SMALL_MAX];
+  __shared__ float s_w[EXIT_SMALL_MAX];
+  const int n = min(ctr[CTR_ACTIVE + par], EXIT_SMALL_MAX);
+  const int base = ctr[CTR_EXITED];
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31, nw = blockDim.x >> 5;
+  const float delta = *delta_p;
+  for (int r = warp; r < n; r += nw) {
+    const float* s = Xout + (size_t)r * D;
+    const float* in = I + (size_t)r * D;
+    float ns = 0.f, ni = 0.f, dot = 0.f;
+    for (int d = lane; d < D; d += 32) {
+      const float a = s[d], c = in[d];
+      ns += a * a;
+      ni += c * c;
+      dot += a * c;
+    }
+    ns = warp_sum(ns);
+    ni = warp_sum(ni);
+    dot = warp_sum(dot);
+    if (lane == 0) {
+      const int tok = row_tok[r];
+      int ex = 0;
+      if (test) {
+        const float c = (ns > 0.f && ni > 0.f) ? dot / sqrtf(ns * ni) : -INFINITY;
+        if (sim) sim[(size_t)tok * n_layers + (layer - 1)] = c;
+        const int f = forced ? forced[tok] : 0;
+        if (f != 0 && (f < 2 || f > n_layers)) atomicOr(err, ERRW_FORCED);
+        ex = (f > 0) ? (f == layer) : (c >= delta);
+      }
+      s_dst[r] = ex;
+      s_w[r] = ns > 0.f ? rsqrtf(ns) : 0.f;
+    }
+  }
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    int e = 0, k = 0;
+    for (int r = 0; r < n; ++r) {
+      const int tok = row_tok[r];
+      if (s_dst[r]) {
+        s_dst[r] = -1 - (base + e);
+        exit_tok[base + e] = tok;
+        if (exit_layer_out) exit_layer_out[tok] = layer;
+        ++e;
+      } else {
+        s_dst[r] = k;
+        row_tok_next[k] = tok;
+        ++k;
+      }
+    }
+    ctr[CTR_ACTIVE + (par ^ 1)] = k;
+    ctr[CTR_EXITED] = base + e;
+    ctr[CTR_PREFIX + layer] = base + e;
+  }
+  __syncthreads();
+  for (int r = warp; r < n; r += nw) {
+    const int d0 = s_dst[r];
+    const float* s = Xout + (size_t)r * D;
+    const float* in = I + (size_t)r * D;
+    if (d0 >= 0) {
+      const float w = s_w[r];
+      float* xn = Xnext + (size_t)d0 * D;
+      float* inn = Inext + (size_t)d0 * D;
+      for (int d = lane; d < D; d += 32) {
+        const float v = s[d];
+        xn[d] = v;
+        inn[d] = (first ? 0.f : in[d]) + v * w;
+      }
+    } else {
+      const size_t kk = (size_t)(-1 - d0);
+      const float* sp = Xin + (size_t)r * D;
+      for (int d = lane; d < D; d += 32) {
+        hsm_s[kk * D + d] = s[d];
+        hsm_prev[kk * D + d] = sp[d];
+        hsm_I[kk * D + d] = in[d];
+      }
+    }
+  }
+}
+
+void launch_exit_small(cudaStream_t st, const float* Xin, const float* Xout, const float* I, int first, int D,
+                       int* ctr, int par, const int* row_tok, int* row_tok_next, const int* forced, int layer,
+                       int n_layers, const float* delta_p, int test, float* sim, int* exit_tok, int* exit_layer_out,
+                       float* Xnext, float* Inext, float* hsm_s, float* hsm_prev, float* hsm_I, unsigned* err) {
+  exit_small_kernel<<<1, 256, 0, st>>>(Xin, Xout, I, first, D, ctr, par, row_tok, row_tok_next, forced, layer,
+                                       n_layers, delta_p, test, sim, exit_tok, exit_layer_out, Xnext, Inext, hsm_s,
+                                       hsm_prev, hsm_I, err);
+}
+
+__global__ void set_float_kernel(float* p, float v) { *p = v; }
+void launch_set_float(cudaStream_t st, float* p, float v) { set_float_kernel<<<1, 1, 0, st>>>(p, v); }
 
 // After layer N: the remaining active rows' s_N are their final states.
 __global__ void final_scatter_kernel(const float* X, int D, const int* n_rows, const int* row_tok, float* final_,
@@ -539,10 +639,10 @@ void launch_layernorm_inplace(cudaStream_t st, float* X, DevRange rows, int max_
 }
 
 void launch_exit_decide(cudaStream_t st, const float* Xout, const float* I, int D, DevRange rows, int max_rows,
-                        const int* row_tok, const int* forced, int layer, int n_layers, float delta, int test,
+                        const int* row_tok, const int* forced, int layer, int n_layers, const float* delta_p, int test,
                         float* sim, int* flag, float* inv_norm, unsigned* err) {
   if (max_rows <= 0) return;
-  exit_decide_kernel<<<cdiv(max_rows, 8), 256, 0, st>>>(Xout, I, D, rows, row_tok, forced, layer, n_layers, delta,
+  exit_decide_kernel<<<cdiv(max_rows, 8), 256, 0, st>>>(Xout, I, D, rows, row_tok, forced, layer, n_layers, delta_p,
                                                        test, sim, flag, inv_norm, err);
 }
 

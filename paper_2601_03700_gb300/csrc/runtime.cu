@@ -5,6 +5,7 @@
 #include "common.cuh"
 #include "kernels.h"
 #include "gemm_tc.h"
+#include "gemm_skinny.h"
 
 #include <algorithm>
 #include <cmath>
@@ -85,17 +86,31 @@ struct adept_model {
   void* pool_t = nullptr;
   float* logits_ws = nullptr;
   float* attn_ws = nullptr;
+  float* sk_ws = nullptr;        // skinny-GEMM partial tiles
+  size_t sk_ws_floats = 0;
+  int* sk_counters = nullptr;    // skinny-GEMM arrival counters (kept zero between launches)
+  int sk_n_counters = 0;
   float* scratch = nullptr;
   size_t scratch_elems = 0;
   // skipped-layer fill workspace (adept_skip_kv_fill)
   int fill_cap = 0;
   void* fill_x = nullptr;
   int *fill_tok = nullptr, *fill_hist = nullptr, *fill_start = nullptr, *fill_cursor = nullptr;
+  // generation-step staging buffers (the captured graph reads and writes only these)
+  float* d_delta = nullptr;
+  int *dec_tok = nullptr, *dec_forced = nullptr, *dec_exit = nullptr, *dec_next = nullptr;
+  float* dec_sim = nullptr;
+  cudaStream_t cap_stream = nullptr;
+  std::vector<cudaGraphExec_t> dec_graph;   // per batch size
+  std::vector<int> dec_warm;                // direct runs done per batch size
   // options / instrumentation
-  int hsm_identity = 0, profile = 0, force_simt = 0;
+  int hsm_identity = 0, profile = 0, force_simt = 0, use_graph = 1, use_skinny = 0;
+  std::vector<cudaEvent_t> ev_pool;
+  size_t ev_used = 0;
   int gemm_cls = ADEPT_PROF_GEMM_PREFILL;
   int last_rows = 0;
   int64_t launches = 0;
+  int64_t graph_launches = 0;   // kernels in one captured generation step
   ProfRec prof[ADEPT_PROF_NCLASS];
 };
 
@@ -143,14 +158,22 @@ static adept_status dalloc_t(adept_model* m, P** p, size_t count, size_t esz = s
     if (s_ != ADEPT_OK) return s_;    \
   } while (0)
 
+static void drop_graphs(adept_model* m) {
+  for (auto& g : m->dec_graph)
+    if (g) cudaGraphExecDestroy(g);
+  for (auto& g : m->dec_graph) g = nullptr;
+  for (auto& w : m->dec_warm) w = 0;
+}
+
 static void free_all(adept_model* m) {
+  drop_graphs(m);
+  if (m->cap_stream) cudaStreamDestroy(m->cap_stream);
+  m->cap_stream = nullptr;
   for (void* p : m->allocs) cudaFree(p);
   m->allocs.clear();
-  for (auto& pr : m->prof)
-    for (auto& e : pr.ev) {
-      cudaEventDestroy(e.first);
-      cudaEventDestroy(e.second);
-    }
+  for (cudaEvent_t e : m->ev_pool) cudaEventDestroy(e);
+  m->ev_pool.clear();
+  for (auto& pr : m->prof) pr.ev.clear();
 }
 
 static int attn_norm_mode(const adept_model* m) {
@@ -180,16 +203,26 @@ static Epi epi_base() {
 // ---------------------------------------------------------------------------
 // GEMM dispatch: tcgen05 grouped GEMM for bf16 models, SIMT otherwise.
 // ---------------------------------------------------------------------------
+// Profiling: CUDA events from a pool, recorded on the launching stream around a launch.
+static cudaEvent_t pool_event(adept_model* m) {
+  if (m->ev_used == m->ev_pool.size()) {
+    cudaEvent_t e;
+    if (cudaEventCreate(&e) != cudaSuccess) return nullptr;
+    m->ev_pool.push_back(e);
+  }
+  return m->ev_pool[m->ev_used++];
+}
 static void prof_begin(adept_model* m, int cls, cudaStream_t st, cudaEvent_t* b) {
+  *b = nullptr;
   if (!m->profile) return;
-  cudaEventCreate(b);
-  cudaEventRecord(*b, st);
+  *b = pool_event(m);
+  if (*b) cudaEventRecord(*b, st);
   (void)cls;
 }
 static void prof_end(adept_model* m, int cls, cudaStream_t st, cudaEvent_t b, double flops, double bytes) {
-  if (!m->profile) return;
-  cudaEvent_t e;
-  cudaEventCreate(&e);
+  if (!m->profile || !b) return;
+  cudaEvent_t e = pool_event(m);
+  if (!e) return;
   cudaEventRecord(e, st);
   m->prof[cls].ev.push_back({b, e});
   m->prof[cls].work.push_back({flops, bytes});
@@ -213,6 +246,17 @@ static void gemm(adept_model* m, cudaStream_t st, const GemmProblem* probs, int 
                  int cls, double flops = 0, double bytes = 0) {
   cudaEvent_t b = nullptr;
   prof_begin(m, cls, st, &b);
+  int small = 1;
+  for (int i = 0; i < n_probs; ++i) small &= max_rows[i] <= SKINNY_MAX_M;
+  if (m->dt == ADEPT_DTYPE_BF16 && !m->force_simt && small && m->sk_ws && m->use_skinny) {
+    const int nl = skinny_gemm_grouped(st, probs, n_probs, max_rows, m->sk_ws, m->sk_ws_floats, m->sk_counters,
+                                       m->sk_n_counters);
+    if (nl >= 0) {
+      m->launches += nl;
+      prof_end(m, cls, st, b, flops, bytes);
+      return;
+    }
+  }
   if (m->dt == ADEPT_DTYPE_BF16 && !m->force_simt && tc_gemm_supported()) {
     const int nl = tc_gemm_grouped(st, probs, n_probs, max_rows, m->err_word);
     if (nl >= 0) {
@@ -550,6 +594,21 @@ static adept_status alloc_runtime(adept_model* m) {
   const int nout = c.family == ADEPT_FAMILY_BERT ? c.n_classes : m->V;
   TRY(dalloc_t(m, &m->logits_ws, (size_t)c.max_batch * nout));
   TRY(dalloc_t(m, &m->attn_ws, (size_t)c.max_batch * m->H * ATTN_MAX_SPLIT * (m->dh + 2)));
+  TRY(dalloc_t(m, &m->d_delta, 1));
+  if (m->dt == ADEPT_DTYPE_BF16) {
+    m->sk_ws_floats = (size_t)16 << 20;   // 64 MiB of partial tiles
+    m->sk_n_counters = 1 << 16;
+    TRY(dalloc_t(m, &m->sk_ws, m->sk_ws_floats));
+    TRY(dalloc_t(m, &m->sk_counters, m->sk_n_counters));
+    CUDA_TRY(m, cudaMemset(m->sk_counters, 0, sizeof(int) * m->sk_n_counters));
+  }
+  TRY(dalloc_t(m, &m->dec_tok, c.max_batch));
+  TRY(dalloc_t(m, &m->dec_forced, c.max_batch));
+  TRY(dalloc_t(m, &m->dec_exit, c.max_batch));
+  TRY(dalloc_t(m, &m->dec_next, c.max_batch));
+  TRY(dalloc_t(m, &m->dec_sim, (size_t)c.max_batch * m->N));
+  m->dec_graph.assign(c.max_batch + 1, nullptr);
+  m->dec_warm.assign(c.max_batch + 1, 0);
   // SIMT scratch: the widest GEMM output of any pass step
   size_t w = std::max({(size_t)m->Dq + 2 * m->Dkv, (size_t)m->L[0].up_rows, (size_t)m->m1, (size_t)m->m2, (size_t)D});
   m->scratch_elems = std::max(w * T, (size_t)c.max_batch * nout);
@@ -650,8 +709,10 @@ static GemmProblem kv_problem(adept_model* m, int layer0, const void* xs, int a_
   return p;
 }
 
+// One early-exit pass over n_tok tokens.  The threshold delta is read from m->d_delta
+// (device memory), so a captured generation step does not depend on it.
 static adept_status run_pass(adept_model* m, int n_tok, int batch, int prompt_len, bool decode, const int32_t* tokens,
-                             float delta, const int32_t* forced, int32_t* exit_out, float* sim_out, cudaStream_t st) {
+                             const int32_t* forced, int32_t* exit_out, float* sim_out, cudaStream_t st) {
   m->gemm_cls = decode ? ADEPT_PROF_GEMM_DECODE : ADEPT_PROF_GEMM_PREFILL;
   const adept_config& c = m->cfg;
   const int N = m->N, D = m->D, Dq = m->Dq, Dkv = m->Dkv;
@@ -670,9 +731,10 @@ static adept_status run_pass(adept_model* m, int n_tok, int batch, int prompt_le
   m->launches += 3;
   const KVCacheView cv = cache_view(m);
   const int causal = fam != ADEPT_FAMILY_BERT;
-  int decode_keys = 0;  // generation step: longest key range (the new position included)
-  if (decode)
-    for (int b = 0; b < batch; ++b) decode_keys = std::max(decode_keys, m->h_seq_len[b] + 1);
+  // generation step: the split-KV attention grid covers the reserved capacity (CTAs past a
+  // sequence's length return at once), which keeps every launch of a step step-invariant
+  const int decode_keys = decode ? std::min(c.max_seq, m->max_blocks_per_seq * c.kv_block_tokens) : 0;
+  (void)batch;
   int par = 0;
   for (int i = 1; i <= N; ++i) {
     const int l0 = i - 1;
@@ -749,12 +811,19 @@ static adept_status run_pass(adept_model* m, int n_tok, int batch, int prompt_le
     if (i < N) {
       // exit test (Sec. 4.1) for 2 <= i <= N-1, inertia update, compaction (App. H)
       const int test = i >= 2;
-      launch_exit_decide(st, m->X_out, Ii, D, act, mr, rt, forced, i, N, delta, test, sim_out, m->flag, m->inv_norm,
-                         m->err_word);
-      launch_exit_scan(st, m->ctr, par, m->flag, rt, m->row_tok[par ^ 1], m->exit_tok, m->dst, exit_out, i);
-      launch_exit_move(st, Xi, m->X_out, Ii, i == 1, D, m->ctr + CTR_ACTIVE + par, mr, m->dst, m->inv_norm, m->X_in[par ^ 1],
-                       m->I[par ^ 1], m->hsm_s, m->hsm_prev, m->hsm_I);
-      m->launches += 3;
+      if (n_tok <= EXIT_SMALL_MAX) {
+        launch_exit_small(st, Xi, m->X_out, Ii, i == 1, D, m->ctr, par, rt, m->row_tok[par ^ 1], forced, i, N,
+                          m->d_delta, test, sim_out, m->exit_tok, exit_out, m->X_in[par ^ 1], m->I[par ^ 1], m->hsm_s,
+                          m->hsm_prev, m->hsm_I, m->err_word);
+        m->launches += 1;
+      } else {
+        launch_exit_decide(st, m->X_out, Ii, D, act, mr, rt, forced, i, N, m->d_delta, test, sim_out, m->flag,
+                           m->inv_norm, m->err_word);
+        launch_exit_scan(st, m->ctr, par, m->flag, rt, m->row_tok[par ^ 1], m->exit_tok, m->dst, exit_out, i);
+        launch_exit_move(st, Xi, m->X_out, Ii, i == 1, D, m->ctr + CTR_ACTIVE + par, mr, m->dst, m->inv_norm,
+                         m->X_in[par ^ 1], m->I[par ^ 1], m->hsm_s, m->hsm_prev, m->hsm_I);
+        m->launches += 3;
+      }
       if (!decode && test) {
         // HSM of the tokens that left at layer i (Sec. 4.2); their s~_N feeds the fills
         run_hsm(m, st, DevRange{m->ctr + CTR_PREFIX + i - 1, m->ctr + CTR_PREFIX + i, 0}, mr);
@@ -926,8 +995,10 @@ adept_status adept_prefill(adept_model* m, int batch, int prompt_len, const int3
   cudaStream_t st = (cudaStream_t)stream;
   std::vector<int> lens(batch, prompt_len);
   TRY(reserve_seqs(m, batch, lens.data(), st));
-  TRY(run_pass(m, batch * prompt_len, batch, prompt_len, false, d_tokens, delta, d_forced_exit, d_exit_layer_out,
-               d_sim_out, st));
+  launch_set_float(st, m->d_delta, delta);
+  m->launches += 1;
+  TRY(run_pass(m, batch * prompt_len, batch, prompt_len, false, d_tokens, d_forced_exit, d_exit_layer_out, d_sim_out,
+               st));
   TRY(run_head(m, batch, prompt_len, false, d_logits_out, d_next_token_out, st));
   return check_launch(m);
 }
@@ -946,9 +1017,60 @@ adept_status adept_decode_step(adept_model* m, int batch, const int32_t* d_token
       return fail(m, ADEPT_ERR_CAPACITY, "sequence %d is full (%d positions)", b, m->h_seq_len[b]);
   }
   cudaStream_t st = (cudaStream_t)stream;
-  TRY(run_pass(m, batch, batch, 1, true, d_tokens, delta, d_forced_exit, d_exit_layer_out, d_sim_out, st));
+  // inputs into the staging buffers; the step itself reads and writes only those
+  launch_set_float(st, m->d_delta, delta);
+  CUDA_TRY(m, cudaMemcpyAsync(m->dec_tok, d_tokens, batch * sizeof(int32_t), cudaMemcpyDeviceToDevice, st));
+  if (d_forced_exit)
+    CUDA_TRY(m, cudaMemcpyAsync(m->dec_forced, d_forced_exit, batch * sizeof(int32_t), cudaMemcpyDeviceToDevice, st));
+  else
+    CUDA_TRY(m, cudaMemsetAsync(m->dec_forced, 0, batch * sizeof(int32_t), st));
+  m->launches += 1;
+  auto body = [&](cudaStream_t s) -> adept_status {
+    TRY(run_pass(m, batch, batch, 1, true, m->dec_tok, m->dec_forced, m->dec_exit, m->dec_sim, s));
+    return run_head(m, batch, 1, true, m->logits_ws, m->dec_next, s);
+  };
+  const bool graph_ok = m->use_graph && !m->profile;
+  if (graph_ok && m->dec_warm[batch] >= 1) {
+    if (!m->dec_graph[batch]) {
+      // capture one generation step on a private stream; later steps replay it
+      if (!m->cap_stream) CUDA_TRY(m, cudaStreamCreateWithFlags(&m->cap_stream, cudaStreamNonBlocking));
+      const int64_t l0 = m->launches;
+      CUDA_TRY(m, cudaStreamBeginCapture(m->cap_stream, cudaStreamCaptureModeThreadLocal));
+      adept_status s = body(m->cap_stream);
+      cudaGraph_t g = nullptr;
+      cudaError_t e = cudaStreamEndCapture(m->cap_stream, &g);
+      if (s != ADEPT_OK) {
+        if (g) cudaGraphDestroy(g);
+        return s;
+      }
+      if (e != cudaSuccess) return fail(m, ADEPT_ERR_CUDA, "graph capture failed: %s", cudaGetErrorString(e));
+      cudaGraphExec_t ex = nullptr;
+      e = cudaGraphInstantiate(&ex, g, 0);
+      cudaGraphDestroy(g);
+      if (e != cudaSuccess) return fail(m, ADEPT_ERR_CUDA, "graph instantiate failed: %s", cudaGetErrorString(e));
+      m->dec_graph[batch] = ex;
+      m->graph_launches = m->launches - l0;
+      m->launches = l0;
+    }
+    CUDA_TRY(m, cudaGraphLaunch(m->dec_graph[batch], st));
+    m->launches += m->graph_launches;
+  } else {
+    TRY(body(st));
+    m->dec_warm[batch] += 1;
+  }
   for (int b = 0; b < batch; ++b) m->h_seq_len[b] += 1;
-  TRY(run_head(m, batch, 1, true, d_logits_out, d_next_token_out, st));
+  // outputs out of the staging buffers
+  const int nout = m->V;
+  if (d_exit_layer_out)
+    CUDA_TRY(m, cudaMemcpyAsync(d_exit_layer_out, m->dec_exit, batch * sizeof(int32_t), cudaMemcpyDeviceToDevice, st));
+  if (d_next_token_out)
+    CUDA_TRY(m, cudaMemcpyAsync(d_next_token_out, m->dec_next, batch * sizeof(int32_t), cudaMemcpyDeviceToDevice, st));
+  if (d_logits_out)
+    CUDA_TRY(m, cudaMemcpyAsync(d_logits_out, m->logits_ws, (size_t)batch * nout * sizeof(float),
+                                cudaMemcpyDeviceToDevice, st));
+  if (d_sim_out)
+    CUDA_TRY(m, cudaMemcpyAsync(d_sim_out, m->dec_sim, (size_t)batch * m->N * sizeof(float), cudaMemcpyDeviceToDevice,
+                                st));
   return check_launch(m);
 }
 
@@ -1039,9 +1161,11 @@ adept_status adept_check_device_status(adept_model* m, void* stream) {
 adept_status adept_set_option(adept_model* m, int option, int value) {
   if (!m) return ADEPT_ERR_INVALID_ARG;
   switch (option) {
-    case ADEPT_OPT_HSM_IDENTITY: m->hsm_identity = value != 0; return ADEPT_OK;
+    case ADEPT_OPT_HSM_IDENTITY: m->hsm_identity = value != 0; drop_graphs(m); return ADEPT_OK;
     case ADEPT_OPT_PROFILE: m->profile = value != 0; return ADEPT_OK;
-    case ADEPT_OPT_GEMM_SIMT: m->force_simt = value != 0; return ADEPT_OK;
+    case ADEPT_OPT_GEMM_SIMT: m->force_simt = value != 0; drop_graphs(m); return ADEPT_OK;
+    case ADEPT_OPT_DECODE_GRAPH: m->use_graph = value != 0; drop_graphs(m); return ADEPT_OK;
+    case ADEPT_OPT_SKINNY_GEMM: m->use_skinny = value != 0; drop_graphs(m); return ADEPT_OK;
   }
   return fail(m, ADEPT_ERR_INVALID_ARG, "unknown option %d", option);
 }
@@ -1058,8 +1182,6 @@ adept_status adept_profile_read(adept_model* m, int cls, int64_t* launches, doub
     ms += t;
     fl += pr.work[i].first;
     by += pr.work[i].second;
-    cudaEventDestroy(pr.ev[i].first);
-    cudaEventDestroy(pr.ev[i].second);
   }
   if (launches) *launches = (int64_t)pr.ev.size();
   if (total_ms) *total_ms = ms;
@@ -1067,6 +1189,9 @@ adept_status adept_profile_read(adept_model* m, int cls, int64_t* launches, doub
   if (bytes) *bytes = by;
   pr.ev.clear();
   pr.work.clear();
+  bool any = false;
+  for (auto& q : m->prof) any |= !q.ev.empty();
+  if (!any) m->ev_used = 0;   // every recorded pair was read: the pool can be reused
   return ADEPT_OK;
 }
 

@@ -189,3 +189,27 @@ def test_tensor_core_gemm_matches_simt_gemm():
         assert row_rel_err(out[0][1], out[1][1]).max() < 2e-2
         assert row_rel_err(out[0][2], out[1][2]).max() < 2e-2
         m.close()
+
+
+def test_decode_graph_replay_equals_direct_launches():
+    """A captured generation step replays to the same bits as direct launches."""
+    cfg = small(synth.GPT2, n_layers=6)
+    W = synth.make_weights(cfg, seed=21)
+    outs = []
+    for graph in (0, 1):
+        m = adept.Model(cfg, W)
+        adept.adept_set_option(m.h, adept.OPT_DECODE_GRAPH, graph)
+        tokens = synth.make_tokens(21, 3, 40, cfg.vocab).cuda()
+        ex, lg, nx, _ = m.prefill(tokens, 0.5, synth.forced_exits_uniform(21, 120, 2, 6).view(3, 40).cuda())
+        steps = []
+        fs = synth.forced_exits_uniform(22, 18, 2, 6).view(6, 3).cuda()
+        for s in range(6):
+            ex, lg, nx, sim = m.decode_step(nx, 0.5, fs[s] if s % 2 == 0 else None)
+            steps.append((ex.cpu(), lg.cpu(), nx.cpu(), sim.cpu()))
+        m.check()
+        outs.append((steps, m.read_kv(6, 1, 0, 46)[0].float().cpu()))
+        m.close()
+    for a, b in zip(outs[0][0], outs[1][0]):
+        for x, y in zip(a, b):
+            assert torch.equal(x.nan_to_num(7.0), y.nan_to_num(7.0))
+    assert torch.equal(outs[0][1], outs[1][1])
