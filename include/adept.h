@@ -155,6 +155,29 @@ ADEPT_API adept_status adept_skip_kv_fill(adept_model* m, int n_tokens, const vo
                                 const int32_t* d_exit_layer, const int32_t* d_seq,
                                 const int32_t* d_pos, void* stream);
 
+/* Allocation-free variant of adept_skip_kv_fill.  The paper has no counterpart: this is
+ * an interface for callers that cannot allocate device memory -- code recording a CUDA
+ * graph (allocation and the synchronisation of cudaFree cannot be captured), serving
+ * loops under a fixed memory budget or their own allocator, and latency-critical paths
+ * that must not synchronise the device.  adept_skip_kv_fill grows a per-model workspace
+ * with cudaMalloc when a call brings more tokens than before; this call keeps the same
+ * working set in a fixed file-scope device array of ADEPT_NOALLOC_SCRATCH_BYTES bytes
+ * (16 MiB, held by every GPU that loads the library until the process exits) and calls
+ * no cudaMalloc, cudaFree or other allocating routine.  Same arguments and results as
+ * adept_skip_kv_fill; bf16 models only.
+ *  - Limit: n_tokens * (d_model * 2 + 4) bytes plus about 3 KiB must fit the array
+ *    (about 2000 tokens at d_model 4096, 10900 at d_model 768); larger calls return
+ *    ADEPT_ERR_CAPACITY with the limit in adept_last_error and enqueue nothing.
+ *  - The first call on a device looks up the array's device address (with that device
+ *    current); make that first call before any stream capture.
+ *  - Every call shares the array and it keeps the last call's contents (each call clears
+ *    the counters it needs zeroed).  Calls that overlap on the GPU -- on different streams
+ *    or for different models on one device -- race on it: serialise them. */
+#define ADEPT_NOALLOC_SCRATCH_BYTES ((size_t)16 << 20)
+ADEPT_API adept_status adept_skip_kv_fill_noalloc(adept_model* m, int n_tokens, const void* d_h_mapped,
+                                                  const int32_t* d_exit_layer, const int32_t* d_seq,
+                                                  const int32_t* d_pos, void* stream);
+
 /* Release everything the model owns (synchronises the device first).  NULL is a no-op. */
 ADEPT_API void adept_free(adept_model* m);
 

@@ -27,7 +27,7 @@ ABI_SYMBOLS = [
     "adept_model_load", "adept_prefill", "adept_decode_step", "adept_skip_kv_fill", "adept_free",
     "adept_last_error", "adept_status_string", "adept_seq_reserve", "adept_read_kv",
     "adept_read_final_states", "adept_check_device_status", "adept_set_option", "adept_profile_read",
-    "adept_launch_count",
+    "adept_launch_count", "adept_skip_kv_fill_noalloc",
 ]
 
 
@@ -76,6 +76,7 @@ def load_library(path: str = LIB_PATH):
     lib.adept_prefill.argtypes = [vp, c_int, c_int, i32p, c_float, i32p, i32p, fp, i32p, fp, st]
     lib.adept_decode_step.argtypes = [vp, c_int, i32p, c_float, i32p, i32p, fp, i32p, fp, st]
     lib.adept_skip_kv_fill.argtypes = [vp, c_int, vp, i32p, i32p, i32p, st]
+    lib.adept_skip_kv_fill_noalloc.argtypes = [vp, c_int, vp, i32p, i32p, i32p, st]
     lib.adept_free.argtypes = [vp]
     lib.adept_free.restype = None
     lib.adept_last_error.argtypes = [vp]
@@ -94,7 +95,8 @@ def load_library(path: str = LIB_PATH):
     for name in ABI_SYMBOLS:
         fn = getattr(lib, name)
         if fn.restype is ctypes.c_int or name in ("adept_model_load", "adept_prefill", "adept_decode_step",
-                                                   "adept_skip_kv_fill", "adept_seq_reserve", "adept_read_kv",
+                                                   "adept_skip_kv_fill", "adept_skip_kv_fill_noalloc",
+                                                   "adept_seq_reserve", "adept_read_kv",
                                                    "adept_read_final_states", "adept_check_device_status",
                                                    "adept_set_option", "adept_profile_read"):
             fn.restype = c_int
@@ -187,6 +189,14 @@ def adept_skip_kv_fill(m, n_tokens: int, h_mapped: torch.Tensor, exit_layer: tor
     lib = load_library()
     _check(lib, m, lib.adept_skip_kv_fill(m, n_tokens, _ptr(h_mapped), _ptr(exit_layer), _ptr(seq), _ptr(pos),
                                            _stream(stream)))
+
+
+def adept_skip_kv_fill_noalloc(m, n_tokens: int, h_mapped: torch.Tensor, exit_layer: torch.Tensor,
+                               seq: torch.Tensor, pos: torch.Tensor, stream=None):
+    """adept_skip_kv_fill with its scratch in a fixed device array (no allocation)."""
+    lib = load_library()
+    _check(lib, m, lib.adept_skip_kv_fill_noalloc(m, n_tokens, _ptr(h_mapped), _ptr(exit_layer), _ptr(seq),
+                                                   _ptr(pos), _stream(stream)))
 
 
 def adept_free(m):

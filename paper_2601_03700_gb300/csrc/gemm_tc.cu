@@ -480,4 +480,62 @@ int tc_gemm_grouped(cudaStream_t st, const GemmProblem* probs, int n_probs, cons
   return launch_grouped<TC_MAXG>(st, probs, n_probs, max_rows, err_word);
 }
 
+// Same launch as tc_gemm_grouped, for callers that must not allocate: the tensor maps are
+// encoded into the launch parameters on every call (no map cache, no host heap use).
+int tc_gemm_grouped_nocache(cudaStream_t st, const GemmProblem* probs, int n_probs, const int* max_rows,
+                            unsigned* err_word) {
+  init_once();
+  if (n_probs <= 0) return 0;
+  if (n_probs > TC_MAXG || !g_encode) return -1;
+  long long tiles[4] = {0, 0, 0, 0};
+  const int bns[4] = {256, 128, 64, 32};
+  for (int i = 0; i < n_probs; ++i) {
+    const GemmProblem& q = probs[i];
+    if (q.K % 8 || q.lda % 8 || q.ldb % 8 || q.a_rows <= 0) return -1;
+    if ((q.epi.kind == EPI_QKV || q.epi.kind == EPI_KV || q.epi.kind == EPI_SWIGLU) && (q.N % 32)) return -1;
+    const long long tm = (max_rows[i] + TC_BM - 1) / TC_BM;
+    for (int k = 0; k < 4; ++k) tiles[k] += tm * ((q.N + bns[k] - 1) / bns[k]);
+  }
+  int pick = 3;
+  for (int k = 0; k < 4; ++k)
+    if (tiles[k] >= g_num_sms) {
+      pick = k;
+      break;
+    }
+  const int BN = bns[pick];
+  static TcParams<TC_MAXG> prm;  // static storage, not heap; callers of this entry point serialise
+  memset(&prm, 0, sizeof prm);
+  prm.n_groups = n_probs;
+  prm.err = err_word;
+  auto encode = [&](CUtensorMap* m, const void* base, uint64_t inner, uint64_t outer, uint64_t row_bytes,
+                    uint32_t box_outer) {
+    if (((uintptr_t)base & 15) || (row_bytes & 15) || outer == 0 || inner == 0) return false;
+    cuuint64_t dims[2] = {inner, outer};
+    cuuint64_t strides[1] = {row_bytes};
+    cuuint32_t box[2] = {(cuuint32_t)TC_BK, box_outer};
+    cuuint32_t estr[2] = {1, 1};
+    return g_encode(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), dims, strides, box, estr,
+                    CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                    CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+  };
+  for (int i = 0; i < n_probs; ++i) {
+    const GemmProblem& q = probs[i];
+    TcGroup& G = prm.g[i];
+    if (!encode(&G.ta, q.A, (uint64_t)q.K, (uint64_t)q.a_rows, (uint64_t)q.lda * 2, TC_BM)) return -1;
+    if (!encode(&G.tb, q.B, (uint64_t)q.K, (uint64_t)q.N, (uint64_t)q.ldb * 2, (uint32_t)BN)) return -1;
+    G.rows = q.rows;
+    G.N = q.N;
+    G.K = q.K;
+    G.epi = q.epi;
+  }
+  const int grid = (int)std::min<long long>(tiles[pick], (long long)g_num_sms);
+  if (grid <= 0) return 0;
+  switch (BN) {
+    case 256: return launch_bn<256, 4, TC_MAXG>(st, prm, grid);
+    case 128: return launch_bn<128, 6, TC_MAXG>(st, prm, grid);
+    case 64: return launch_bn<64, 8, TC_MAXG>(st, prm, grid);
+    default: return launch_bn<32, 10, TC_MAXG>(st, prm, grid);
+  }
+}
+
 }  // namespace adept

@@ -8,4 +8,7 @@ namespace adept {
 bool tc_gemm_supported();
 // Enqueues the problems as one grouped launch; returns the number of kernels launched.
 int tc_gemm_grouped(cudaStream_t st, const GemmProblem* probs, int n_probs, const int* max_rows, unsigned* err_word);
+// As tc_gemm_grouped, without the tensor-map cache (nothing is allocated on any heap).
+int tc_gemm_grouped_nocache(cudaStream_t st, const GemmProblem* probs, int n_probs, const int* max_rows,
+                            unsigned* err_word);
 }  // namespace adept

@@ -6,6 +6,7 @@
 #include "kernels.h"
 #include "gemm_tc.h"
 #include "gemm_skinny.h"
+#include "model_view.h"
 
 #include <algorithm>
 #include <cmath>
@@ -1203,3 +1204,34 @@ int64_t adept_launch_count(adept_model* m) {
 }
 
 }  // extern "C"
+
+// ---------------------------------------------------------------------------
+// Read-only view of a loaded model for the allocation-free fill entry point
+// (fill_noalloc.cu).  Copies pointers and sizes only.
+// ---------------------------------------------------------------------------
+namespace adept {
+bool model_fill_view(adept_model* m, FillView* v) {
+  if (!m || m->N > FILL_VIEW_MAX_LAYERS) return false;
+  v->n_layers = m->N;
+  v->d_model = m->D;
+  v->d_q = m->Dq;
+  v->d_kv = m->Dkv;
+  v->head_dim = m->dh;
+  v->dtype = m->dt;
+  v->norm_mode = attn_norm_mode(m);
+  v->norm_eps = m->cfg.norm_eps;
+  v->rope = m->cfg.family == ADEPT_FAMILY_LLAMA;
+  v->rope_table = m->rope_table;
+  v->cache = cache_view(m);
+  v->err_word = m->err_word;
+  for (int l = 0; l < m->N; ++l) {
+    v->w_kv[l] = (const char*)m->L[l].w_qkv + (size_t)m->Dq * m->D * m->esz;
+    v->b_kv[l] = m->L[l].b_qkv + m->Dq;
+  }
+  return true;
+}
+
+void model_set_error(adept_model* m, const char* msg) {
+  if (m) m->err = msg;
+}
+}  // namespace adept
