@@ -24,6 +24,7 @@ constexpr int TC_MAXG = 32;
 constexpr int TC_BM = 128;
 constexpr int TC_BK = 64;               // one 128-byte swizzle row of bf16
 constexpr int TC_THREADS = 192;
+constexpr int TC_SHORT_ROWS = 32;   // rows of the short-tile variants (3-D k-chunk boxes)
 constexpr long long TC_TIMEOUT_CYCLES = 4000000000LL;   // ~2 s at 2 GHz
 
 struct TcGroup {
@@ -32,6 +33,9 @@ struct TcGroup {
   DevRange rows;
   int N;
   int K;
+  int gm;           // m-tiles per raster super-row (their A rows stay in L2 while n sweeps)
+  int a_box;        // rows of A per TMA box: 128, or fewer when the whole problem is one short tile
+                    // (the MMA still spans 128 rows; rows past the box are never stored)
   Epi epi;
 };
 
@@ -78,12 +82,22 @@ __device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, volati
   }
 }
 
+// No "memory" clobber: the copy lands asynchronously and is ordered by the mbarrier, and
+// a clobber would make the producer reload its loop state every k-block.
 __device__ __forceinline__ void tma_load_2d(const CUtensorMap* tm, uint64_t* bar, void* dst, int x, int y) {
   asm volatile(
       "cp.async.bulk.tensor.2d.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1, {%2, %3}], [%4];" ::"r"(
           smem_u32(dst)),
-      "l"((uint64_t)tm), "r"(x), "r"(y), "r"(smem_u32(bar))
-      : "memory");
+      "l"((uint64_t)tm), "r"(x), "r"(y), "r"(smem_u32(bar)));
+}
+
+// 3-D box {64 k, rows, KC chunks of 64 k}: KC k-chunks of the tile in one instruction,
+// stored chunk after chunk (each chunk a [rows][64] swizzled tile).
+__device__ __forceinline__ void tma_load_3d(const CUtensorMap* tm, uint64_t* bar, void* dst, int y, int z) {
+  asm volatile(
+      "cp.async.bulk.tensor.3d.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1, {%2, %3, %4}], [%5];" ::
+          "r"(smem_u32(dst)),
+      "l"((uint64_t)tm), "r"(0), "r"(y), "r"(z), "r"(smem_u32(bar)));
 }
 
 __device__ __forceinline__ void tmem_alloc(uint32_t* slot, uint32_t ncols) {
@@ -147,12 +161,31 @@ __device__ __forceinline__ constexpr uint32_t idesc_bf16() {
   return (1u << 4) | (1u << 7) | (1u << 10) | ((uint32_t)(BN >> 3) << 17) | ((uint32_t)(TC_BM >> 4) << 24);
 }
 
+#ifdef ADEPT_TC_TRACE
+// Debug builds only (-DADEPT_TC_TRACE): clock64 timestamps of CTA 0's first tile, per
+// launch, in a ring -- entry, TMEM ready, first TMA issued, first stage landed, last
+// commit, accumulator seen by the epilogue, epilogue done, final barrier, TMEM freed.
+__device__ long long g_tc_trace[256][16];
+__device__ unsigned g_tc_launch;
+#define TC_TRACE(k)                                                   \
+  do {                                                                \
+    if (blockIdx.x == 0 && tr_slot >= 0) g_tc_trace[tr_slot][k] = clock64(); \
+  } while (0)
+#else
+#define TC_TRACE(k) \
+  do {              \
+  } while (0)
+#endif
+
 // ---------------------------------------------------------------------------- kernel
-template <int BN, int STAGES, int MAXG>
+// KC > 1 (problems of at most TC_SHORT_ROWS rows, K a multiple of 64): a stage holds KC
+// k-chunks loaded by one 3-D box per operand; the A chunks are packed a_box rows apart
+// and the 128-row MMA of chunk c reads past its own rows into the next chunks (rows
+// that are never stored), so the A region is one 128-row tile plus (KC-1) short tiles.
+template <int BN, int STAGES, int MAXG, int KC>
 __global__ void __launch_bounds__(TC_THREADS, 1) gemm_tc_kernel(const __grid_constant__ TcParams<MAXG> p) {
-  constexpr int A_BYTES = TC_BM * TC_BK * 2;
-  constexpr int B_BYTES = BN * TC_BK * 2;
-  constexpr uint32_t TX = A_BYTES + B_BYTES;
+  constexpr int A_BYTES = TC_BM * TC_BK * 2 + (KC - 1) * TC_SHORT_ROWS * TC_BK * 2;
+  constexpr int B_BYTES = KC * BN * TC_BK * 2;
   constexpr uint32_t TMEM_COLS = 2 * BN;
   constexpr uint32_t IDESC = idesc_bf16<BN>();
 
@@ -169,10 +202,20 @@ __global__ void __launch_bounds__(TC_THREADS, 1) gemm_tc_kernel(const __grid_con
   volatile int* abort_flag = (volatile int*)(tmem_slot + 1);
 
   __shared__ int s_tile0[MAXG + 1];
-  __shared__ int s_mbeg[MAXG], s_M[MAXG], s_tn[MAXG];
+  __shared__ int s_mbeg[MAXG], s_M[MAXG], s_tn[MAXG], s_tm[MAXG], s_gm[MAXG];
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int ng = p.n_groups;
+#ifdef ADEPT_TC_TRACE
+  __shared__ int s_slot;
+  if (threadIdx.x == 0) s_slot = blockIdx.x == 0 ? (int)(atomicAdd(&g_tc_launch, 1u) & 255u) : -1;
+  __syncthreads();
+  const int tr_slot = s_slot;
+  if (threadIdx.x == 0 && blockIdx.x == 0) {
+    g_tc_trace[tr_slot][0] = clock64();
+    g_tc_trace[tr_slot][9] = gridDim.x * 1000 + BN;
+  }
+#endif
   if (threadIdx.x == 0) {
     int acc = 0;
     for (int g = 0; g < ng; ++g) {
@@ -182,8 +225,10 @@ __global__ void __launch_bounds__(TC_THREADS, 1) gemm_tc_kernel(const __grid_con
       s_mbeg[g] = b;
       s_M[g] = M;
       s_tn[g] = tn;
+      s_tm[g] = (M + TC_BM - 1) / TC_BM;
+      s_gm[g] = max(1, p.g[g].gm);
       s_tile0[g] = acc;
-      acc += ((M + TC_BM - 1) / TC_BM) * tn;
+      acc += s_tm[g] * tn;
     }
     s_tile0[ng] = acc;
     for (int s = 0; s < STAGES; ++s) {
@@ -201,6 +246,13 @@ __global__ void __launch_bounds__(TC_THREADS, 1) gemm_tc_kernel(const __grid_con
   __syncthreads();
   const int total = s_tile0[ng];
   if ((int)blockIdx.x >= total) return;  // uniform: nothing allocated yet
+  if (threadIdx.x == 0) {
+    // pull the first tile's tensor maps in while the barriers and TMEM are set up
+    int g0 = 0;
+    while (g0 + 1 < ng && (int)blockIdx.x >= s_tile0[g0 + 1]) ++g0;
+    asm volatile("prefetch.tensormap [%0];" ::"l"((uint64_t)&p.g[g0].ta) : "memory");
+    asm volatile("prefetch.tensormap [%0];" ::"l"((uint64_t)&p.g[g0].tb) : "memory");
+  }
 
   if (warp == 1) {
     tmem_alloc(tmem_slot, TMEM_COLS);
@@ -210,13 +262,21 @@ __global__ void __launch_bounds__(TC_THREADS, 1) gemm_tc_kernel(const __grid_con
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem = *tmem_slot;
+  if (threadIdx.x == 0) TC_TRACE(1);
 
+  // Tile order inside a problem: super-rows of gm m-tiles; within a super-row n is the
+  // outer and m the inner index, so concurrently running CTAs share both the A rows of
+  // the super-row and the weight slab of an n-block through L2.
   auto locate = [&](int t, int& g, int& mb, int& nb) {
     g = 0;
     while (g + 1 < ng && t >= s_tile0[g + 1]) ++g;
     const int local = t - s_tile0[g];
-    nb = local % s_tn[g];
-    mb = local / s_tn[g];
+    const int gm = s_gm[g], tn = s_tn[g];
+    const int sup = local / (gm * tn);
+    const int rem = local - sup * gm * tn;
+    const int rows = min(gm, s_tm[g] - sup * gm);
+    nb = rem / rows;
+    mb = sup * gm + rem % rows;
   };
 
   if (warp == 0) {
@@ -225,17 +285,33 @@ __global__ void __launch_bounds__(TC_THREADS, 1) gemm_tc_kernel(const __grid_con
       int stage = 0;
       uint32_t phase = 0;
       uint32_t issued = 0, last_par = 0;   // per stage: issued at least once / parity of its last issue
+      int n_issued = 0;                    // slots are known free until the ring wraps once
       for (int t = blockIdx.x; t < total && !*abort_flag; t += gridDim.x) {
         int g, mb, nb;
         locate(t, g, mb, nb);
         const TcGroup& G = p.g[g];
-        const int nk = (G.K + TC_BK - 1) / TC_BK;
+        // per-tile values in registers: the asm "memory" clobbers below would otherwise make
+        // every k-block reload them from parameter space
+        const int nk = (G.K + TC_BK * KC - 1) / (TC_BK * KC);   // stages of KC k-chunks
         const int ya = s_mbeg[g] + mb * TC_BM, yb = nb * BN;
+        const uint32_t tx_bytes = (uint32_t)(KC * (G.a_box + BN) * TC_BK * 2);
+        const CUtensorMap* tma_a = &G.ta;
+        const CUtensorMap* tma_b = &G.tb;
         for (int kb = 0; kb < nk; ++kb) {
-          if (!mbar_wait(&empty[stage], phase ^ 1, abort_flag, p.err)) break;
-          mbar_expect_tx(&full[stage], TX);
-          tma_load_2d(&G.ta, &full[stage], sA + stage * A_BYTES, kb * TC_BK, ya);
-          tma_load_2d(&G.tb, &full[stage], sB + stage * B_BYTES, kb * TC_BK, yb);
+          if (n_issued >= STAGES && !mbar_wait(&empty[stage], phase ^ 1, abort_flag, p.err)) break;
+          ++n_issued;
+          mbar_expect_tx(&full[stage], tx_bytes);
+          if (KC == 1) {
+            tma_load_2d(tma_a, &full[stage], sA + stage * A_BYTES, kb * TC_BK, ya);
+          } else {
+            tma_load_3d(tma_a, &full[stage], sA + stage * A_BYTES, ya, kb * KC);
+          }
+          if (KC == 1) {
+            tma_load_2d(tma_b, &full[stage], sB + stage * B_BYTES, kb * TC_BK, yb);
+          } else {
+            tma_load_3d(tma_b, &full[stage], sB + stage * B_BYTES, yb, kb * KC);
+          }
+          if (t == (int)blockIdx.x && kb == 0) TC_TRACE(2);
           issued |= 1u << stage;
           last_par = (last_par & ~(1u << stage)) | (phase << stage);
           if (++stage == STAGES) {
@@ -266,18 +342,24 @@ __global__ void __launch_bounds__(TC_THREADS, 1) gemm_tc_kernel(const __grid_con
       for (int t = blockIdx.x; t < total && ok; t += gridDim.x) {
         int g, mb, nb;
         locate(t, g, mb, nb);
-        const int nk = (p.g[g].K + TC_BK - 1) / TC_BK;
+        const int nk = (p.g[g].K + TC_BK * KC - 1) / (TC_BK * KC);
+        const uint32_t a_chunk = (uint32_t)(p.g[g].a_box * TC_BK * 2);   // bytes between A chunks
         if (!(ok = mbar_wait(&acce[ab], aph ^ 1, abort_flag, p.err))) break;
         tc_fence_after();
         const uint32_t d = tmem + (uint32_t)(ab * BN);
         for (int kb = 0; kb < nk; ++kb) {
           if (!(ok = mbar_wait(&full[stage], phase, abort_flag, p.err))) break;
+          if (t == (int)blockIdx.x && kb == 0) TC_TRACE(3);
+
           tc_fence_after();
-          const uint64_t ad = sdesc_sw128(smem_u32(sA + stage * A_BYTES));
-          const uint64_t bd = sdesc_sw128(smem_u32(sB + stage * B_BYTES));
 #pragma unroll
-          for (int k = 0; k < TC_BK / 16; ++k)
-            umma_bf16(d, ad + (uint64_t)(2 * k), bd + (uint64_t)(2 * k), IDESC, (kb | k) != 0 ? 1u : 0u);
+          for (int c = 0; c < KC; ++c) {
+            const uint64_t ad = sdesc_sw128(smem_u32(sA + stage * A_BYTES) + c * a_chunk);
+            const uint64_t bd = sdesc_sw128(smem_u32(sB + stage * B_BYTES) + c * (BN * TC_BK * 2));
+#pragma unroll
+            for (int k = 0; k < TC_BK / 16; ++k)
+              umma_bf16(d, ad + (uint64_t)(2 * k), bd + (uint64_t)(2 * k), IDESC, (kb | c | k) != 0 ? 1u : 0u);
+          }
           umma_commit(&empty[stage]);
           if (++stage == STAGES) {
             stage = 0;
@@ -286,6 +368,7 @@ __global__ void __launch_bounds__(TC_THREADS, 1) gemm_tc_kernel(const __grid_con
         }
         if (!ok) break;
         umma_commit(&accf[ab]);
+        if (t == (int)blockIdx.x) TC_TRACE(4);
         ab ^= 1;
         if (ab == 0) aph ^= 1;
       }
@@ -309,14 +392,20 @@ __global__ void __launch_bounds__(TC_THREADS, 1) gemm_tc_kernel(const __grid_con
       int g, mb, nb;
       locate(t, g, mb, nb);
       const TcGroup& G = p.g[g];
-      const bool got = mbar_wait(&accf[ab], aph, abort_flag, p.err);
-      if (!__all_sync(0xffffffffu, got)) break;   // warp-uniform: tcgen05.ld below is .sync.aligned
-      tc_fence_after();
+      // the row's cache slot etc. do not depend on the accumulator: look them up first
       const int r = mb * TC_BM + row_in_tile;
       const bool valid = r < s_M[g];
       const int ra = s_mbeg[g] + r;
       EpiRow rr{-1, 0};
       if (valid) rr = epi_row(G.epi, ra);
+      // one lane per warp polls the barrier (128 pollers would crowd the barrier unit the
+      // producer and MMA threads need); the result is broadcast to the warp
+      bool got = true;
+      if (lane == 0) got = mbar_wait(&accf[ab], aph, abort_flag, p.err);
+      got = __shfl_sync(0xffffffffu, got ? 1 : 0, 0) != 0;
+      if (!got) break;   // warp-uniform: tcgen05.ld below is .sync.aligned
+      if (t == (int)blockIdx.x && warp == 2 && lane == 0) TC_TRACE(5);
+      tc_fence_after();
       const uint32_t tb = tmem + ((uint32_t)(q * 32) << 16) + (uint32_t)(ab * BN);
 #pragma unroll 1
       for (int c = 0; c < BN; c += 32) {
@@ -327,17 +416,20 @@ __global__ void __launch_bounds__(TC_THREADS, 1) gemm_tc_kernel(const __grid_con
       }
       tc_fence_before();
       __syncwarp();
+      if (t == (int)blockIdx.x && warp == 2 && lane == 0) TC_TRACE(6);
       if (lane == 0) mbar_arrive(&acce[ab]);
       ab ^= 1;
       if (ab == 0) aph ^= 1;
     }
   }
   __syncthreads();
+  if (threadIdx.x == 0) TC_TRACE(7);
   if (warp == 1) {
     __syncwarp();
     tc_fence_after();
     tmem_dealloc(tmem, TMEM_COLS);
   }
+  if (threadIdx.x == 32) TC_TRACE(8);
 }
 
 // ---------------------------------------------------------------------------- host side
@@ -387,6 +479,22 @@ struct MapKeyHash {
 // Tensor maps are encoded once per (address, extent, stride, box) and reused by later
 // launches; a map depends on nothing else, so a reused address with the same extent
 // maps the same way.
+// Rows per A box: a problem whose rows fit one tile loads only a multiple of 8 rows that
+// covers them (the TMA unit's cost grows with the rows of a box).
+static int a_box_rows(int max_rows) {
+  if (max_rows > 64) return TC_BM;
+  int b = 8;
+  while (b < max_rows) b *= 2;
+  return b;
+}
+
+// m-tiles per raster super-row: their A rows (128 x K bf16 each) should take at most
+// ~48 MiB of the 129 MiB L2, leaving room for the weight slabs and the output stream.
+static int raster_gm(int K) {
+  const long long per = 128LL * K * 2;
+  return (int)std::max(1LL, std::min(64LL, (48LL << 20) / std::max(per, 1LL)));
+}
+
 static bool make_map(CUtensorMap* m, const void* base, uint64_t inner, uint64_t outer, uint64_t row_bytes,
                      uint32_t box_outer) {
   if (((uintptr_t)base & 15) || (row_bytes & 15) || outer == 0 || inner == 0) return false;
@@ -412,16 +520,34 @@ static bool make_map(CUtensorMap* m, const void* base, uint64_t inner, uint64_t 
   return true;
 }
 
-template <int BN, int STAGES, int MAXG>
+template <int BN, int STAGES, int MAXG, int KC = 1>
 static int launch_bn(cudaStream_t st, const TcParams<MAXG>& prm, int grid) {
-  constexpr size_t smem = (size_t)STAGES * (TC_BM + BN) * TC_BK * 2 + 1024 + 256;
+  constexpr size_t a_bytes = (size_t)TC_BM * TC_BK * 2 + (size_t)(KC - 1) * TC_SHORT_ROWS * TC_BK * 2;
+  constexpr size_t b_bytes = (size_t)KC * BN * TC_BK * 2;
+  constexpr size_t smem = (size_t)STAGES * (a_bytes + b_bytes) + 1024 + 256;
+  static_assert(smem <= 232448, "stage ring does not fit shared memory");
   static bool attr = false;
   if (!attr) {
-    cudaFuncSetAttribute(gemm_tc_kernel<BN, STAGES, MAXG>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    cudaFuncSetAttribute(gemm_tc_kernel<BN, STAGES, MAXG, KC>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                         (int)smem);
     attr = true;
   }
-  gemm_tc_kernel<BN, STAGES, MAXG><<<grid, TC_THREADS, smem, st>>>(prm);
+  gemm_tc_kernel<BN, STAGES, MAXG, KC><<<grid, TC_THREADS, smem, st>>>(prm);
   return 1;
+}
+
+// 3-D view {64, rows, K / 64} of a K-major matrix (strides: row, then 128 bytes per
+// k-chunk), box {64, box_rows, kc}.
+static bool encode_3d(CUtensorMap* m, const void* base, uint64_t K, uint64_t rows, uint64_t row_bytes,
+                      uint32_t box_rows, uint32_t kc) {
+  if (((uintptr_t)base & 15) || (row_bytes & 15) || rows == 0 || K == 0 || (K % TC_BK)) return false;
+  cuuint64_t dims[3] = {(cuuint64_t)TC_BK, rows, K / TC_BK};
+  cuuint64_t strides[2] = {row_bytes, (cuuint64_t)TC_BK * 2};
+  cuuint32_t box[3] = {(cuuint32_t)TC_BK, box_rows, kc};
+  cuuint32_t estr[3] = {1, 1, 1};
+  return g_encode(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void*>(base), dims, strides, box, estr,
+                  CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                  CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
 template <int MAXG>
@@ -441,6 +567,12 @@ static int launch_grouped(cudaStream_t st, const GemmProblem* probs, int n_probs
       break;
     }
   const int BN = bns[pick];
+  // short problems (every group one tile of at most TC_SHORT_ROWS rows, K in whole 64-chunks)
+  // take the 3-D box variant: one TMA instruction per operand carries KC k-chunks
+  bool short_rows = true;
+  for (int i = 0; i < n_probs; ++i)
+    short_rows &= max_rows[i] <= TC_SHORT_ROWS && probs[i].K % TC_BK == 0;
+  const int KC = short_rows ? (BN == 256 ? 2 : 4) : 1;
   static TcParams<MAXG> prm;  // kept off the stack; calls on a model are serialised
   memset(&prm, 0, sizeof prm);
   prm.n_groups = n_probs;
@@ -448,15 +580,34 @@ static int launch_grouped(cudaStream_t st, const GemmProblem* probs, int n_probs
   for (int i = 0; i < n_probs; ++i) {
     const GemmProblem& q = probs[i];
     TcGroup& G = prm.g[i];
-    if (!make_map(&G.ta, q.A, (uint64_t)q.K, (uint64_t)q.a_rows, (uint64_t)q.lda * 2, TC_BM)) return -1;
-    if (!make_map(&G.tb, q.B, (uint64_t)q.K, (uint64_t)q.N, (uint64_t)q.ldb * 2, (uint32_t)BN)) return -1;
+    G.a_box = a_box_rows(max_rows[i]);
+    if (KC > 1) {
+      if (!encode_3d(&G.ta, q.A, (uint64_t)q.K, (uint64_t)q.a_rows, (uint64_t)q.lda * 2, (uint32_t)G.a_box,
+                     (uint32_t)KC))
+        return -1;
+      if (!encode_3d(&G.tb, q.B, (uint64_t)q.K, (uint64_t)q.N, (uint64_t)q.ldb * 2, (uint32_t)BN, (uint32_t)KC))
+        return -1;
+    } else {
+      if (!make_map(&G.ta, q.A, (uint64_t)q.K, (uint64_t)q.a_rows, (uint64_t)q.lda * 2, (uint32_t)G.a_box))
+        return -1;
+      if (!make_map(&G.tb, q.B, (uint64_t)q.K, (uint64_t)q.N, (uint64_t)q.ldb * 2, (uint32_t)BN)) return -1;
+    }
     G.rows = q.rows;
     G.N = q.N;
     G.K = q.K;
+    G.gm = raster_gm(q.K);
     G.epi = q.epi;
   }
   const int grid = (int)std::min<long long>(tiles[pick], (long long)g_num_sms);
   if (grid <= 0) return 0;
+  if (KC > 1) {
+    switch (BN) {
+      case 256: return launch_bn<256, 2, MAXG, 2>(st, prm, grid);
+      case 128: return launch_bn<128, 2, MAXG, 4>(st, prm, grid);
+      case 64: return launch_bn<64, 3, MAXG, 4>(st, prm, grid);
+      default: return launch_bn<32, 4, MAXG, 4>(st, prm, grid);
+    }
+  }
   switch (BN) {
     case 256: return launch_bn<256, 4, MAXG>(st, prm, grid);
     case 128: return launch_bn<128, 6, MAXG>(st, prm, grid);
@@ -521,11 +672,13 @@ int tc_gemm_grouped_nocache(cudaStream_t st, const GemmProblem* probs, int n_pro
   for (int i = 0; i < n_probs; ++i) {
     const GemmProblem& q = probs[i];
     TcGroup& G = prm.g[i];
-    if (!encode(&G.ta, q.A, (uint64_t)q.K, (uint64_t)q.a_rows, (uint64_t)q.lda * 2, TC_BM)) return -1;
+    G.a_box = a_box_rows(max_rows[i]);
+    if (!encode(&G.ta, q.A, (uint64_t)q.K, (uint64_t)q.a_rows, (uint64_t)q.lda * 2, (uint32_t)G.a_box)) return -1;
     if (!encode(&G.tb, q.B, (uint64_t)q.K, (uint64_t)q.N, (uint64_t)q.ldb * 2, (uint32_t)BN)) return -1;
     G.rows = q.rows;
     G.N = q.N;
     G.K = q.K;
+    G.gm = raster_gm(q.K);
     G.epi = q.epi;
   }
   const int grid = (int)std::min<long long>(tiles[pick], (long long)g_num_sms);
@@ -539,3 +692,11 @@ int tc_gemm_grouped_nocache(cudaStream_t st, const GemmProblem* probs, int n_pro
 }
 
 }  // namespace adept
+
+#ifdef ADEPT_TC_TRACE
+extern "C" __attribute__((visibility("default"))) int adept_debug_tc_trace(long long* out, unsigned* n_launches) {
+  if (cudaMemcpyFromSymbol(out, adept::g_tc_trace, sizeof(long long) * 256 * 16) != cudaSuccess) return 1;
+  if (cudaMemcpyFromSymbol(n_launches, adept::g_tc_launch, sizeof(unsigned)) != cudaSuccess) return 1;
+  return 0;
+}
+#endif

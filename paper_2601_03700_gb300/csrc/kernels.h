@@ -45,7 +45,8 @@ void launch_hsm_mid(cudaStream_t st, int dt, const float* h3, const float* h1, D
 void launch_hsm_out(cudaStream_t st, int dt, const float* h5, const float* c0f, const float* hs, int identity,
                     DevRange rows, int max_rows, int D, const float* g2, float eps, const int* exit_tok,
                     float* final_, void* xfill, int fill_mode, float norm_eps);
-void launch_argmax(cudaStream_t st, const float* logits, int V, int rows, int* out);
+// Greedy token per row (lowest index on ties); part_v / part_i: rows * 32 partials.
+int launch_argmax(cudaStream_t st, const float* logits, int V, int rows, int* out, float* part_v, int* part_i);
 void launch_head_rows(cudaStream_t st, int batch, int prompt_len, int last, int* rows);
 void launch_fill_sort(cudaStream_t st, int dt, const void* h, int n, int D, const int* exit_layer, int n_layers,
                       int* hist, int* start, int* cursor, int* sorted_tok, void* xs, int mode, float eps,

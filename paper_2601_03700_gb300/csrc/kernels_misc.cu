@@ -694,9 +694,77 @@ void launch_hsm_out(cudaStream_t st, int dt, const float* h5, const float* c0f, 
                                                     (float*)xfill, fill_mode, norm_eps);
 }
 
-void launch_argmax(cudaStream_t st, const float* logits, int V, int rows, int* out) {
-  if (rows <= 0) return;
-  argmax_kernel<<<rows, 256, 0, st>>>(logits, V, rows, out);
+// Two-stage argmax for long rows: ARGMAX_SPLIT blocks per row reduce slices to
+// (value, index) pairs, one thread per row merges them (lowest index on ties).
+constexpr int ARGMAX_SPLIT = 32;
+__global__ void argmax_part_kernel(const float* logits, int V, int rows, float* pv, int* pi) {
+  __shared__ float sv[32];
+  __shared__ int si[32];
+  const int r = blockIdx.x / ARGMAX_SPLIT, part = blockIdx.x % ARGMAX_SPLIT;
+  if (r >= rows) return;
+  const int chunk = (V + ARGMAX_SPLIT - 1) / ARGMAX_SPLIT;
+  const int lo = part * chunk, hi = min(V, lo + chunk);
+  const float* l = logits + (size_t)r * V;
+  float bv = -INFINITY;
+  int bi = 0x7fffffff;
+  for (int v = lo + threadIdx.x; v < hi; v += blockDim.x) {
+    const float x = l[v];
+    if (x > bv || (x == bv && v < bi)) {
+      bv = x;
+      bi = v;
+    }
+  }
+#pragma unroll
+  for (int o = 16; o; o >>= 1) {
+    const float ov = __shfl_xor_sync(0xffffffffu, bv, o);
+    const int oi = __shfl_xor_sync(0xffffffffu, bi, o);
+    if (ov > bv || (ov == bv && oi < bi)) {
+      bv = ov;
+      bi = oi;
+    }
+  }
+  const int lane = threadIdx.x & 31, w = threadIdx.x >> 5;
+  if (lane == 0) {
+    sv[w] = bv;
+    si[w] = bi;
+  }
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    for (int k = 1; k < (int)(blockDim.x >> 5); ++k)
+      if (sv[k] > bv || (sv[k] == bv && si[k] < bi)) {
+        bv = sv[k];
+        bi = si[k];
+      }
+    pv[blockIdx.x] = bv;
+    pi[blockIdx.x] = bi;
+  }
+}
+
+__global__ void argmax_merge_kernel(const float* pv, const int* pi, int rows, int* out) {
+  const int r = blockIdx.x * blockDim.x + threadIdx.x;
+  if (r >= rows) return;
+  float bv = -INFINITY;
+  int bi = 0x7fffffff;
+  for (int k = 0; k < ARGMAX_SPLIT; ++k) {
+    const float x = pv[r * ARGMAX_SPLIT + k];
+    const int i = pi[r * ARGMAX_SPLIT + k];
+    if (x > bv || (x == bv && i < bi)) {
+      bv = x;
+      bi = i;
+    }
+  }
+  out[r] = bi == 0x7fffffff ? 0 : bi;
+}
+
+int launch_argmax(cudaStream_t st, const float* logits, int V, int rows, int* out, float* part_v, int* part_i) {
+  if (rows <= 0) return 0;
+  if (V <= 4096 || !part_v || !part_i) {
+    argmax_kernel<<<rows, 256, 0, st>>>(logits, V, rows, out);
+    return 1;
+  }
+  argmax_part_kernel<<<rows * ARGMAX_SPLIT, 256, 0, st>>>(logits, V, rows, part_v, part_i);
+  argmax_merge_kernel<<<cdiv(rows, 64), 64, 0, st>>>(part_v, part_i, rows, out);
+  return 2;
 }
 
 void launch_head_rows(cudaStream_t st, int batch, int prompt_len, int last, int* rows) {

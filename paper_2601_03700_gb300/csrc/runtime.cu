@@ -87,6 +87,8 @@ struct adept_model {
   void* pool_t = nullptr;
   float* logits_ws = nullptr;
   float* attn_ws = nullptr;
+  float* amax_v = nullptr;       // argmax partials
+  int* amax_i = nullptr;
   float* sk_ws = nullptr;        // skinny-GEMM partial tiles
   size_t sk_ws_floats = 0;
   int* sk_counters = nullptr;    // skinny-GEMM arrival counters (kept zero between launches)
@@ -596,6 +598,8 @@ static adept_status alloc_runtime(adept_model* m) {
   TRY(dalloc_t(m, &m->logits_ws, (size_t)c.max_batch * nout));
   TRY(dalloc_t(m, &m->attn_ws, (size_t)c.max_batch * m->H * ATTN_MAX_SPLIT * (m->dh + 2)));
   TRY(dalloc_t(m, &m->d_delta, 1));
+  TRY(dalloc_t(m, &m->amax_v, (size_t)c.max_batch * 32));
+  TRY(dalloc_t(m, &m->amax_i, (size_t)c.max_batch * 32));
   if (m->dt == ADEPT_DTYPE_BF16) {
     m->sk_ws_floats = (size_t)16 << 20;   // 64 MiB of partial tiles
     m->sk_n_counters = 1 << 16;
@@ -651,7 +655,7 @@ static adept_status reserve_seqs(adept_model* m, int batch, const int* lens, cud
 // ---------------------------------------------------------------------------
 __global__ void set_int_kernel(int* p, int v) { *p = v; }
 
-static void run_hsm(adept_model* m, cudaStream_t st, DevRange rows, int max_rows) {
+static void run_hsm(adept_model* m, cudaStream_t st, DevRange rows, int max_rows, int a_rows) {
   const int D = m->D, m1 = m->m1, m2 = m->m2;
   const float eps = m->cfg.hsm_eps;
   if (m->hsm_identity) {
@@ -666,7 +670,7 @@ static void run_hsm(adept_model* m, cudaStream_t st, DevRange rows, int max_rows
   GemmProblem p;
   memset(&p, 0, sizeof p);
   p.rows = rows;
-  p.a_rows = m->T_max;
+  p.a_rows = a_rows;
   // FC1: h1 = GELU(W1 c0 + b1)
   p.A = m->c0t; p.lda = D; p.B = m->hsm_w1; p.ldb = D; p.N = m1; p.K = D;
   p.epi = epi_base(); p.epi.kind = EPI_ACT; p.epi.act = ACT_GELU_ERF; p.epi.bias = m->hsm_b1;
@@ -753,7 +757,7 @@ static adept_status run_pass(adept_model* m, int n_tok, int batch, int prompt_le
     GemmProblem pr[2];
     int mrs[2] = {mr, mr};
     memset(pr, 0, sizeof pr);
-    pr[0].A = m->xn; pr[0].lda = D; pr[0].a_rows = m->T_max; pr[0].B = w.w_qkv; pr[0].ldb = D; pr[0].rows = act;
+    pr[0].A = m->xn; pr[0].lda = D; pr[0].a_rows = n_tok; pr[0].B = w.w_qkv; pr[0].ldb = D; pr[0].rows = act;
     pr[0].N = Dq + 2 * Dkv; pr[0].K = D;
     pr[0].epi = epi_base();
     pr[0].epi.kind = EPI_QKV; pr[0].epi.bias = w.b_qkv; pr[0].epi.out_t = m->q; pr[0].epi.ld_t = Dq;
@@ -762,7 +766,7 @@ static adept_status run_pass(adept_model* m, int n_tok, int batch, int prompt_le
     pr[0].epi.head_dim = m->dh; pr[0].epi.rope = fam == ADEPT_FAMILY_LLAMA; pr[0].epi.rope_table = m->rope_table;
     int np = 1;
     if (!decode && i >= 3) {
-      pr[1] = kv_problem(m, l0, m->xfill, m->T_max, DevRange{nullptr, m->ctr + CTR_EXITED, 0}, m->exit_tok, m->tok_seq,
+      pr[1] = kv_problem(m, l0, m->xfill, n_tok, DevRange{nullptr, m->ctr + CTR_EXITED, 0}, m->exit_tok, m->tok_seq,
                          m->tok_pos);
       np = 2;
     }
@@ -779,7 +783,7 @@ static adept_status run_pass(adept_model* m, int n_tok, int batch, int prompt_le
     // O projection + residual
     GemmProblem p;
     memset(&p, 0, sizeof p);
-    p.a_rows = m->T_max;
+    p.a_rows = n_tok;   // the TMA view ends at this pass's rows: tiles past them read zeros, not memory
     p.A = m->att; p.lda = Dq; p.B = w.w_o; p.ldb = Dq; p.rows = act; p.N = D; p.K = Dq;
     p.epi = epi_base(); p.epi.kind = EPI_RESID; p.epi.bias = w.b_o; p.epi.out_f32 = m->X_out; p.epi.ld_f32 = D;
     p.epi.resid = Xi; p.epi.ld_resid = D;
@@ -827,7 +831,7 @@ static adept_status run_pass(adept_model* m, int n_tok, int batch, int prompt_le
       }
       if (!decode && test) {
         // HSM of the tokens that left at layer i (Sec. 4.2); their s~_N feeds the fills
-        run_hsm(m, st, DevRange{m->ctr + CTR_PREFIX + i - 1, m->ctr + CTR_PREFIX + i, 0}, mr);
+        run_hsm(m, st, DevRange{m->ctr + CTR_PREFIX + i - 1, m->ctr + CTR_PREFIX + i, 0}, mr, n_tok);
       }
       par ^= 1;
     } else {
@@ -840,11 +844,11 @@ static adept_status run_pass(adept_model* m, int n_tok, int batch, int prompt_le
     // the skipped-layer fills of all exits run once, after the layer loop: one HSM over
     // every exited token, then one grouped launch over (skipped layer r) groups; rows are
     // in exit-layer order, so layer r's rows (i* < r) are a prefix.
-    run_hsm(m, st, DevRange{nullptr, m->ctr + CTR_EXITED, 0}, n_tok);
+    run_hsm(m, st, DevRange{nullptr, m->ctr + CTR_EXITED, 0}, n_tok, n_tok);
     std::vector<GemmProblem> probs;
     std::vector<int> mrs;
     for (int r = 3; r <= N; ++r) {
-      probs.push_back(kv_problem(m, r - 1, m->xfill, m->T_max, DevRange{nullptr, m->ctr + CTR_PREFIX + r - 1, 0}, m->exit_tok,
+      probs.push_back(kv_problem(m, r - 1, m->xfill, n_tok, DevRange{nullptr, m->ctr + CTR_PREFIX + r - 1, 0}, m->exit_tok,
                                  m->tok_seq, m->tok_pos));
       mrs.push_back(n_tok);
     }
@@ -864,7 +868,7 @@ static adept_status run_head(adept_model* m, int batch, int prompt_len, bool dec
   const DevRange rows{nullptr, nullptr, batch};
   GemmProblem p;
   memset(&p, 0, sizeof p);
-  p.a_rows = c.max_batch;
+  p.a_rows = batch;
   if (!enc) {
     launch_standardize(st, m->dt, m->final_, D, m->head_rows, rows, batch, D, attn_norm_mode(m), c.norm_eps, m->xhead,
                        D);
@@ -872,10 +876,7 @@ static adept_status run_head(adept_model* m, int batch, int prompt_len, bool dec
     p.A = m->xhead; p.lda = D; p.B = m->w_head; p.ldb = D; p.rows = rows; p.N = m->V; p.K = D;
     p.epi = epi_base(); p.epi.kind = EPI_F32; p.epi.bias = m->b_head; p.epi.out_f32 = out; p.epi.ld_f32 = m->V;
     gemm(m, st, &p, 1, &batch, m->gemm_cls);
-    if (next) {
-      launch_argmax(st, out, m->V, batch, next);
-      m->launches += 1;
-    }
+    if (next) m->launches += launch_argmax(st, out, m->V, batch, next, m->amax_v, m->amax_i);
   } else {
     launch_standardize(st, m->dt, m->final_, D, m->head_rows, rows, batch, D, NORM_COPY, c.norm_eps, m->xhead, D);
     m->launches += 1;
@@ -886,10 +887,7 @@ static adept_status run_head(adept_model* m, int batch, int prompt_len, bool dec
     p.A = m->pool_t; p.lda = D; p.B = m->w_cls; p.ldb = D; p.N = c.n_classes; p.K = D;
     p.epi = epi_base(); p.epi.kind = EPI_F32; p.epi.bias = m->b_cls; p.epi.out_f32 = out; p.epi.ld_f32 = c.n_classes;
     gemm(m, st, &p, 1, &batch, m->gemm_cls);
-    if (next) {
-      launch_argmax(st, out, c.n_classes, batch, next);
-      m->launches += 1;
-    }
+    if (next) m->launches += launch_argmax(st, out, c.n_classes, batch, next, nullptr, nullptr);
   }
   return ADEPT_OK;
 }
