@@ -436,7 +436,7 @@ def cores():
 
 
 def cpu_baseline(n_tokens: int):
-    n_seq, prompt, steps = 1, n_tokens, 8
+    n_seq, prompt, steps = 4, n_tokens, 8
     tok, dt = oracle_sample(n_seq, prompt, steps)
     return {"value": round(tok / dt, 3), "unit": "tokens/s", "cores": cores(), "kind": "oracle",
             "sample": f"{n_seq} prompt x {prompt} tokens + {steps} decode steps of the same model and exit law "

@@ -114,7 +114,7 @@ ADEPT_API adept_status adept_model_load(const adept_config* cfg, const adept_ten
 
 /* Prompt pass (prefill) of `batch` sequences of `prompt_len` tokens each; resets
  * sequences 0..batch-1 and reserves KV blocks for their whole max_seq.
- * Per layer i (App. H): the still-active tokens run layer i; for 2 <= i <= N-1 each
+ * Per layer i (App. I): the still-active tokens run layer i; for 2 <= i <= N-1 each
  * active token tests <s_hat_i, I_hat> >= delta (Sec. 4.1), or, where
  * d_forced_exit[j] != 0, exits exactly at that layer; exiting tokens are mapped by
  * the HSM (Sec. 4.2) and their K/V for every skipped layer r > i* are produced
@@ -133,7 +133,7 @@ ADEPT_API adept_status adept_prefill(adept_model* m, int batch, int prompt_len, 
                            float* d_logits_out, int32_t* d_next_token_out, float* d_sim_out,
                            void* stream);
 
-/* One generation step (App. H, generation phase): token b of sequence b is appended
+/* One generation step (App. I, generation phase): token b of sequence b is appended
  * at that sequence's next position and exits independently of the others.  Same
  * per-token outputs as adept_prefill with batch rows.  Decoder families only.
  * Errors: INVALID_ARG, CAPACITY (a sequence is full). */
@@ -142,8 +142,8 @@ ADEPT_API adept_status adept_decode_step(adept_model* m, int batch, const int32_
                                float* d_logits_out, int32_t* d_next_token_out, float* d_sim_out,
                                void* stream);
 
-/* Decoupled skipped-layer KV fill (Sec. 4, decoupling equation; Sec. 4.3 KV
- * generation): for every token j and every layer r = i*_j+1..N, writes layer r's
+/* Decoupled skipped-layer KV fill (Eq. 6, the decoupling of Sec. 4; Eq. 9, KV
+ * generation in Sec. 4.3): for every token j and every layer r = i*_j+1..N, writes layer r's
  * K = RoPE(W_K^r norm_r(s~_j) + b_K^r) and V = W_V^r norm_r(s~_j) + b_V^r into the
  * KV cache at (d_seq[j], d_pos[j]); all (token, layer) pairs in one grouped launch.
  *   d_h_mapped  [n_tokens, D] mapped states s~_N in the model dtype

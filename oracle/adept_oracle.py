@@ -15,10 +15,10 @@ What it follows (paper sections / equations / tables):
   RMS-normalised separately, stacked to (3, D_h), a 3x3 convolution with stride 1
   and padding (0, 1) gives one D_h row, then the 4-FC MLP with its normalisations
   and two additions.
-* Skipped-layer K/V (Sec. 4 decoupling equation, Sec. 4.3 KV generation equation):
+* Skipped-layer K/V (Eq. 6, the decoupling of Sec. 4; Eq. 9, KV generation in Sec. 4.3):
   for every r > i*, the K/V of layer r are layer r's K/V projection of the mapped
   state s~_N, computed directly from s~_N (no sequential unfolding).
-* Dynamic shrinkage (App. H): each layer runs only on the still-active tokens.
+* Dynamic shrinkage (App. I): each layer runs only on the still-active tokens.
 
 Readings where the paper is silent (each one is also listed in the design notes):
 
@@ -311,7 +311,7 @@ def layer_body(m: OracleModel, i: int, h: np.ndarray, seq: np.ndarray, pos: np.n
 
 
 # ----------------------------------------------------------------------------
-# the early-exit pass (App. H process, Sec. 4.1-4.3 pieces)
+# the early-exit pass (App. I process, Sec. 4.1-4.3 pieces)
 # ----------------------------------------------------------------------------
 
 @dataclass
@@ -332,7 +332,7 @@ def check_forced(forced: np.ndarray, n_layers: int):
 def early_exit_pass(m: OracleModel, cache: OracleCache, s0: np.ndarray, seq: np.ndarray,
                     pos: np.ndarray, delta: float, forced: Optional[np.ndarray], causal: bool,
                     kv_len: np.ndarray, hsm_mode: str = "hsm") -> PassResult:
-    """Run tokens (all in parallel, App. H) through layers 1..N with token-level exits.
+    """Run tokens (all in parallel, App. I) through layers 1..N with token-level exits.
 
     For each layer i: (a) K/V of the active tokens from their layer input go to the
     cache; (b) the rest of the layer runs for the active tokens; (c) for 2 <= i <= N-1
@@ -417,7 +417,7 @@ def prefill(m: OracleModel, cache: OracleCache, tokens: np.ndarray, delta: float
 
 def decode_step(m: OracleModel, cache: OracleCache, tokens: np.ndarray, delta: float,
                 forced: Optional[np.ndarray] = None, hsm_mode: str = "hsm") -> PassResult:
-    """One generation step: token b of sequence b at position lens[b] (App. H, generation)."""
+    """One generation step: token b of sequence b at position lens[b] (App. I, generation)."""
     c = m.cfg
     if c.family == BERT:
         raise ValueError("decode is defined for decoder models only")

@@ -814,7 +814,7 @@ static adept_status run_pass(adept_model* m, int n_tok, int batch, int prompt_le
       m->launches += 1;
     }
     if (i < N) {
-      // exit test (Sec. 4.1) for 2 <= i <= N-1, inertia update, compaction (App. H)
+      // exit test (Sec. 4.1) for 2 <= i <= N-1, inertia update, compaction (App. I)
       const int test = i >= 2;
       if (n_tok <= EXIT_SMALL_MAX) {
         launch_exit_small(st, Xi, m->X_out, Ii, i == 1, D, m->ctr, par, rt, m->row_tok[par ^ 1], forced, i, N,

@@ -169,7 +169,7 @@ def test_full_depth_decode_matches_recompute(family):
 @pytest.mark.parametrize("hsm_mode", ["hsm", "identity"])
 def test_brute_force_token_major_unfold(hsm_mode):
     """Every forced-exit assignment in {2, 3}^5 on N=3, D=8, 2 heads, 5 tokens: the layer-major
-    parallel pass (App. H) equals a one-token-at-a-time unfold built from library ops,
+    parallel pass (App. I) equals a one-token-at-a-time unfold built from library ops,
     in final states, exit layers and every cached K/V entry of every layer."""
     cfg = small_cfg(synth.LLAMA, n_layers=3, d_model=8, n_heads=2, head_dim=4, d_ffn=16, vocab=11)
     m, ref, _ = model_and_ref(cfg, seed=13, std=0.4)
