@@ -261,6 +261,63 @@ def run_fill_micro(adept, device, peaks, grid_T, grid_i, reps=3):
     return rows
 
 
+def llama_work(cfg, exit_prompt, exit_decode):
+    """Algorithmic flops of a Llama-shaped prompt pass + generation steps (GEMMs, fills, HSM,
+    head) from the exit layers: the cost the early exit saves or adds."""
+    fl = pass_work(cfg, exit_prompt, decode=False)[0]
+    for e in exit_decode:
+        fl += pass_work(cfg, e, decode=True)[0] + decode_fill_work(cfg, e)[0]
+    return fl
+
+
+def run_llama_e2e(adept, device, P=2048, steps=256):
+    """Llama-2-7B shape, batch 1: 2048-token prompt + 256 greedy decode steps, exit layer per
+    token ~ N(24, 4) truncated to [8, 32] -- against the same library forced to full depth."""
+    cfg = synth.llama7b_config(max_batch=1, max_seq=P + steps, max_pass_tokens=P)
+    W = synth.make_weights(cfg, seed=0, device=device)
+    m = adept.Model(cfg, W)
+    del W
+    torch.cuda.empty_cache()
+    tok = synth.make_tokens(0, 1, P, cfg.vocab).to(device)
+    fp = synth.forced_exits_truncnorm(0, P, 24.0, 4.0, 8, 32, name="forced_prompt").view(1, P).to(device)
+    fd = synth.forced_exits_truncnorm(0, steps, 24.0, 4.0, 8, 32, name="forced_decode").view(steps, 1).to(device)
+    full_p = torch.full_like(fp, cfg.n_layers)
+    full_d = torch.full_like(fd, cfg.n_layers)
+    nxt = torch.empty(steps + 1, 1, dtype=torch.int32, device=device)
+    exd = torch.empty(steps, 1, dtype=torch.int32, device=device)
+    exp_ = torch.empty(P, dtype=torch.int32, device=device)
+    st = torch.cuda.current_stream()
+    out = {}
+    for name, a, b in (("early_exit", fp, fd), ("full_depth", full_p, full_d)):
+        for rep in range(2):   # first run warms up (and captures the generation-step graph)
+            e0, e1, e2 = [torch.cuda.Event(enable_timing=True) for _ in range(3)]
+            torch.cuda.synchronize()
+            e0.record(st)
+            adept.adept_prefill(m.h, 1, P, tok.view(-1), 0.9, a.view(-1), exp_, None, nxt[0], None)
+            e1.record(st)
+            for s in range(steps):
+                adept.adept_decode_step(m.h, 1, nxt[s], 0.9, b[s], exd[s], None, nxt[s + 1], None)
+            e2.record(st)
+            torch.cuda.synchronize()
+        adept.adept_check_device_status(m.h)
+        tp, td = e0.elapsed_time(e1) / 1e3, e1.elapsed_time(e2) / 1e3
+        out[name] = {"prefill_tok_s": round(P / tp, 1), "decode_tok_s": round(steps / td, 2),
+                     "tok_s": round((P + steps) / (tp + td), 2), "prefill_ms": round(tp * 1e3, 3),
+                     "decode_ms_per_step": round(td * 1e3 / steps, 4),
+                     "mean_exit_depth": round(float(np.concatenate([exp_.cpu().numpy(),
+                                                                    exd.cpu().numpy().reshape(-1)]).mean()), 3),
+                     "algorithmic_tflop": round(llama_work(cfg, exp_.cpu().numpy(), exd.cpu().numpy()) / 1e12, 3)}
+    m.close()
+    torch.cuda.empty_cache()
+    ee, fd_ = out["early_exit"], out["full_depth"]
+    return {"workload": "Llama-2-7B shape, bf16, random-init; batch 1, 2048-token prompt + 256 greedy decode steps; "
+                        "exit layer per token ~ N(24,4) truncated to [8,32] vs all tokens forced to layer 32",
+            "early_exit": ee, "full_depth": fd_,
+            "speedup": round(ee["tok_s"] / fd_["tok_s"], 4),
+            "algorithmic_ratio": round(fd_["algorithmic_tflop"] / ee["algorithmic_tflop"], 4),
+            "depth_ratio": round(fd_["mean_exit_depth"] / ee["mean_exit_depth"], 4)}
+
+
 def ours(args, rank, world, device):
     import paper_2601_03700_gb300 as adept
     if not os.path.exists(adept.LIB_PATH):
@@ -398,6 +455,8 @@ def ours(args, rank, world, device):
                            "peak": {"tflops": peaks["bf16_tflops"], "gbs": peaks["hbm_gbs"], "source": peaks_src},
                            "grid": rows,
                            "mean_frac": round(float(np.mean([r["frac"] for r in rows])), 4)}
+    if rank == 0 and not args.no_llama:
+        line["llama7b_e2e"] = run_llama_e2e(adept, device)
     if rank == 0 and not args.no_cpu_baseline:
         line["cpu_baseline"] = cpu_baseline(args.cpu_tokens)
     return line
@@ -489,21 +548,46 @@ def kernel_case_fill_small(device):
     m.close()
 
 
+def kernel_case_llama_prefill(device):
+    """Two early-exit prompt passes at the Llama-2-7B shape (2048 tokens, exits ~ N(24,4) on
+    [8, 32]) for launch-list captures: the second pass is the one to capture."""
+    import paper_2601_03700_gb300 as adept
+    adept.load_library()
+    P = 2048
+    cfg = synth.llama7b_config(max_batch=1, max_seq=P, max_pass_tokens=P)
+    W = synth.make_weights(cfg, seed=0, device=device)
+    m = adept.Model(cfg, W)
+    del W
+    tok = synth.make_tokens(0, 1, P, cfg.vocab).to(device)
+    fp = synth.forced_exits_truncnorm(0, P, 24.0, 4.0, 8, 32, name="forced_prompt").to(device)
+    nxt = torch.empty(1, dtype=torch.int32, device=device)
+    for _ in range(2):
+        adept.adept_prefill(m.h, 1, P, tok.view(-1), 0.9, fp, None, None, nxt, None)
+    torch.cuda.synchronize()
+    m.check()
+    print(json.dumps({"kernel_case": "llama_prefill", "prompt": P, "launches_per_pass": adept.adept_launch_count(m.h) // 2}))
+    m.close()
+
+
 def main():
     ap = argparse.ArgumentParser()
-    ap.add_argument("--kernel-case", default=None, choices=["fill_small"])
+    ap.add_argument("--kernel-case", default=None, choices=["fill_small", "llama_prefill"])
     ap.add_argument("--gpus", type=int, default=1)
     ap.add_argument("--steps", type=int, default=5)
     ap.add_argument("--warmup", type=int, default=3)
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--no-kv-fill", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-llama", action="store_true")
     ap.add_argument("--fill-T", default="1,16,256,1024,4096,16384,65536")
     ap.add_argument("--fill-i", default="4,8,16,24")
     ap.add_argument("--cpu-tokens", type=int, default=512)
     args = ap.parse_args()
     if args.kernel_case == "fill_small":
         kernel_case_fill_small(torch.device("cuda", 0))
+        return
+    if args.kernel_case == "llama_prefill":
+        kernel_case_llama_prefill(torch.device("cuda", 0))
         return
     world = int(os.environ.get("WORLD_SIZE", "1"))
     rank = int(os.environ.get("RANK", "0"))
