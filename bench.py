@@ -112,6 +112,19 @@ def decode_fill_work(cfg, exit_layers):
     return fl, by
 
 
+def attention_decode_work(cfg, exit_layers, keys):
+    """Generation-step attention: every token active at layer i reads the K and V of its
+    `keys` cached positions at that layer once.  (flops, bytes)."""
+    N, dq, dkv = cfg.n_layers, cfg.d_q, cfg.d_kv
+    e = np.asarray(exit_layers).reshape(-1)
+    fl = by = 0.0
+    for i in range(1, N + 1):
+        act = int(np.sum(e >= i))
+        fl += act * 4.0 * keys * dq
+        by += act * (keys * 2 * dkv * 2 + 2 * dq * 2)
+    return fl, by
+
+
 def fill_micro_work(T, istar, n_layers=32, d=4096, dkv=4096):
     """Skipped-layer fill of T tokens exiting at i*, all deeper layers: flops and the
     algorithmic bytes (each layer's W_K/W_V once, s~ once, K/V written once)."""
@@ -357,13 +370,13 @@ def ours(args, rank, world, device):
     # CUDA events on the launching stream around every GEMM / fill / attention launch;
     # generation steps run as direct launches while profiling.
     adept.adept_set_option(run.m.h, adept.OPT_PROFILE, 1)
-    for c in range(4):
+    for c in range(adept.PROF_DECODE_STEP + 1):
         adept.adept_profile_read(run.m.h, c)
     flush.zero_()
     torch.cuda.synchronize()
     run.step()
     torch.cuda.synchronize()
-    prof = {c: adept.adept_profile_read(run.m.h, c) for c in range(4)}
+    prof = {c: adept.adept_profile_read(run.m.h, c) for c in range(adept.PROF_DECODE_STEP + 1)}
     adept.adept_set_option(run.m.h, adept.OPT_PROFILE, 0)
     adept.adept_check_device_status(run.m.h)
     t = torch.tensor([total_ms], dtype=torch.float64, device=device)
@@ -402,10 +415,15 @@ def ours(args, rank, world, device):
     wp = pass_work(cfg, e_p, decode=False)
     wd = [pass_work(cfg, e_d[s], decode=True) for s in range(STEPS)]
     wf = [decode_fill_work(cfg, e_d[s]) for s in range(STEPS)]
+    wa = [attention_decode_work(cfg, e_d[s], P + s + 1) for s in range(STEPS)]
     work = {adept.PROF_GEMM_PREFILL: wp, adept.PROF_GEMM_DECODE: (sum(w[0] for w in wd), sum(w[1] for w in wd)),
-            adept.PROF_KV_FILL: (sum(w[0] for w in wf), sum(w[1] for w in wf))}
+            adept.PROF_KV_FILL: (sum(w[0] for w in wf), sum(w[1] for w in wf)),
+            # the persistent generation step: every GEMM of the step, its fills and its attention
+            adept.PROF_DECODE_STEP: (sum(a[0] + b[0] + c[0] for a, b, c in zip(wd, wf, wa)),
+                                     sum(a[1] + b[1] + c[1] for a, b, c in zip(wd, wf, wa)))}
     names = {adept.PROF_GEMM_PREFILL: "gemm_prefill", adept.PROF_GEMM_DECODE: "gemm_decode",
-             adept.PROF_KV_FILL: "kv_fill_decode", adept.PROF_ATTENTION: "attention"}
+             adept.PROF_KV_FILL: "kv_fill_decode", adept.PROF_ATTENTION: "attention",
+             adept.PROF_DECODE_STEP: "decode_step_fused"}
     per_class = {}
     for c, (n, ms, _, _) in prof.items():
         per_class[names[c]] = {"launches": n, "ms_per_step": round(ms, 4)}
@@ -428,6 +446,7 @@ def ours(args, rank, world, device):
     roof["launches"] = n
     roof["peak_source"] = peaks_src + " (MEASURED_PEAKS.json burst)" if peaks_src == "measured" else peaks_src
     roof["timing"] = "CUDA events around each launch of the class, one profiled step after the timed steps"
+    roof["work_per_launch"] = {"flop": round(fl / max(n, 1)), "bytes": round(by / max(n, 1))}
     line = {
         "metric": METRIC, "value": round(value, 2), "unit": "tokens/s", "n_gpus": world, "steps": args.steps,
         "warmup": args.warmup, "ms_per_step": round(total_ms / args.steps, 3), "higher_is_better": True,

@@ -213,22 +213,34 @@ ADEPT_API adept_status adept_check_device_status(adept_model* m, void* stream);
  * SIMT kernels (cross-check).  DECODE_GRAPH (default 1): from its second call with a
  * given batch size, adept_decode_step replays a CUDA graph of the step captured once;
  * 0 launches every kernel directly.  SKINNY_GEMM (default 0): GEMMs of at most 32 rows
- * use the split-K skinny kernel instead of the tcgen05 kernel. */
+ * use the split-K skinny kernel instead of the tcgen05 kernel.  FUSED_DECODE: 1 runs a
+ * generation step of at most adept_fused_decode_batch() sequences of a bf16 decoder as
+ * one persistent cooperative launch (every layer, the HSM, the fills and the head),
+ * reading the caller's inputs and writing its outputs directly; 0 takes the multi-launch
+ * step.  Default: 1 when a layer holds at least 64 MiB of weights (weight streaming
+ * dominates the step), else 0. */
 enum { ADEPT_OPT_HSM_IDENTITY = 1, ADEPT_OPT_PROFILE = 2, ADEPT_OPT_GEMM_SIMT = 3, ADEPT_OPT_DECODE_GRAPH = 4,
-       ADEPT_OPT_SKINNY_GEMM = 5 };
+       ADEPT_OPT_SKINNY_GEMM = 5, ADEPT_OPT_FUSED_DECODE = 6 };
 ADEPT_API adept_status adept_set_option(adept_model* m, int option, int value);
 
 /* Kernel classes reported by adept_profile_read: the GEMMs of prompt passes (layer
  * projections, HSM, head, and the per-layer skipped-layer fills co-launched with
  * layer i's QKV), the GEMMs of generation steps, the grouped skipped-layer fill
- * launches (end of a generation step and adept_skip_kv_fill), and attention. */
+ * launches (end of a generation step and adept_skip_kv_fill), attention, and the
+ * persistent generation-step launch (FUSED_DECODE). */
 enum { ADEPT_PROF_GEMM_PREFILL = 0, ADEPT_PROF_KV_FILL = 1, ADEPT_PROF_ATTENTION = 2,
-       ADEPT_PROF_GEMM_DECODE = 3, ADEPT_PROF_NCLASS = 4 };
+       ADEPT_PROF_GEMM_DECODE = 3, ADEPT_PROF_DECODE_STEP = 4, ADEPT_PROF_NCLASS = 5 };
 /* Synchronise, then return the number of recorded launches of kernel class `cls` and
  * their total device time in ms (CUDA events on the launching stream); resets the
  * record.  flops / bytes are reserved (returned as 0). */
 ADEPT_API adept_status adept_profile_read(adept_model* m, int cls, int64_t* launches, double* total_ms,
                                 double* flops, double* bytes);
+
+/* Largest batch a generation step runs as one persistent launch (0: the model or the
+ * device does not take that path, or FUSED_DECODE is off), and why not (empty if it
+ * does).  The reason string lives as long as the model. */
+ADEPT_API int adept_fused_decode_batch(const adept_model* m);
+ADEPT_API const char* adept_fused_decode_reason(const adept_model* m);
 
 /* Number of kernel launches the library enqueued since the last call (then reset). */
 ADEPT_API int64_t adept_launch_count(adept_model* m);

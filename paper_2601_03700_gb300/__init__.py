@@ -19,15 +19,15 @@ LIB_PATH = os.path.join(_PKG, "libadept.so")
 ADEPT_OK = 0
 STATUS_NAMES = {0: "OK", 1: "INVALID_ARG", 2: "OOM", 3: "CAPACITY", 4: "CUDA", 5: "TIMEOUT", 6: "DEVICE_INPUT"}
 FAMILY = {"llama": 0, "gpt2": 1, "bert": 2}
-OPT_HSM_IDENTITY, OPT_PROFILE, OPT_GEMM_SIMT, OPT_DECODE_GRAPH, OPT_SKINNY_GEMM = 1, 2, 3, 4, 5
-PROF_GEMM_PREFILL, PROF_KV_FILL, PROF_ATTENTION, PROF_GEMM_DECODE = 0, 1, 2, 3
+OPT_HSM_IDENTITY, OPT_PROFILE, OPT_GEMM_SIMT, OPT_DECODE_GRAPH, OPT_SKINNY_GEMM, OPT_FUSED_DECODE = 1, 2, 3, 4, 5, 6
+PROF_GEMM_PREFILL, PROF_KV_FILL, PROF_ATTENTION, PROF_GEMM_DECODE, PROF_DECODE_STEP = 0, 1, 2, 3, 4
 
 # every symbol declared in include/adept.h
 ABI_SYMBOLS = [
     "adept_model_load", "adept_prefill", "adept_decode_step", "adept_skip_kv_fill", "adept_free",
     "adept_last_error", "adept_status_string", "adept_seq_reserve", "adept_read_kv",
     "adept_read_final_states", "adept_check_device_status", "adept_set_option", "adept_profile_read",
-    "adept_launch_count", "adept_skip_kv_fill_noalloc",
+    "adept_launch_count", "adept_skip_kv_fill_noalloc", "adept_fused_decode_batch", "adept_fused_decode_reason",
 ]
 
 
@@ -92,6 +92,10 @@ def load_library(path: str = LIB_PATH):
                                        ctypes.POINTER(ctypes.c_double), ctypes.POINTER(ctypes.c_double)]
     lib.adept_launch_count.argtypes = [vp]
     lib.adept_launch_count.restype = ctypes.c_int64
+    lib.adept_fused_decode_batch.argtypes = [vp]
+    lib.adept_fused_decode_batch.restype = c_int
+    lib.adept_fused_decode_reason.argtypes = [vp]
+    lib.adept_fused_decode_reason.restype = ctypes.c_char_p
     for name in ABI_SYMBOLS:
         fn = getattr(lib, name)
         if fn.restype is ctypes.c_int or name in ("adept_model_load", "adept_prefill", "adept_decode_step",
@@ -304,3 +308,10 @@ class Model:
 
     def check(self):
         adept_check_device_status(self.h)
+
+    def fused_decode_batch(self) -> int:
+        """Largest batch a generation step runs as one persistent launch (0: never)."""
+        return int(load_library().adept_fused_decode_batch(self.h))
+
+    def fused_decode_reason(self) -> str:
+        return load_library().adept_fused_decode_reason(self.h).decode(errors="replace")

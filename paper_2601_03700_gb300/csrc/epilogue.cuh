@@ -42,14 +42,16 @@ __device__ __forceinline__ void store16(T* p, const float* v) {
 }
 
 // Per-row facts the cache epilogues need: the token's position and the cache offset
-// of its slot (-1 if the position has no reserved block).
+// of its slot (-1 if the position has no reserved block); rope (optional): the row's
+// (cos, sin) table row already staged by the caller.
 struct EpiRow {
   long long cbase;
   int pos;
+  const float2* rope;
 };
 
 __device__ __forceinline__ EpiRow epi_row(const Epi& e, int ra) {
-  EpiRow r{-1, 0};
+  EpiRow r{-1, 0, nullptr};
   if (e.kind == EPI_QKV || e.kind == EPI_KV) {
     const int tok = e.row_tok[ra];
     r.pos = e.tok_pos[tok];
@@ -74,10 +76,18 @@ __device__ __forceinline__ void rope_pairs(T* dst, int i0, int half, const float
   store16<T>(dst + i0 + half, b);
 }
 
+// bias32 / resid32 (optional): the chunk's 32 bias values and the row's 32 residual
+// values already staged by the caller (e.g. in shared memory) instead of e.bias[c0..] and
+// e.resid[ra][c0..].
 template <typename T>
-__device__ __forceinline__ void epi_chunk32(const Epi& e, int ra, int c0, int N, float (&v)[32], const EpiRow& rr) {
+__device__ __forceinline__ void epi_chunk32(const Epi& e, int ra, int c0, int N, float (&v)[32], const EpiRow& rr,
+                                            const float* bias32 = nullptr, const float* resid32 = nullptr) {
   const bool full = c0 + 32 <= N;
-  if (e.bias) {
+  if (bias32) {
+#pragma unroll
+    for (int j = 0; j < 32; ++j)
+      if (full || c0 + j < N) v[j] += bias32[j];
+  } else if (e.bias) {
 #pragma unroll
     for (int j = 0; j < 32; ++j)
       if (full || c0 + j < N) v[j] += e.bias[c0 + j];
@@ -118,9 +128,9 @@ __device__ __forceinline__ void epi_chunk32(const Epi& e, int ra, int c0, int N,
       return;
     }
     case EPI_RESID: {
-      const float* r = e.resid + (size_t)ra * e.ld_resid + c0;
+      const float* r = resid32 ? resid32 : e.resid + (size_t)ra * e.ld_resid + c0;
       float* o = e.out_f32 + (size_t)ra * e.ld_f32 + c0;
-      if (full && ((e.ld_f32 & 15) == 0) && ((e.ld_resid & 15) == 0)) {
+      if (full && ((e.ld_f32 & 15) == 0) && (resid32 || (e.ld_resid & 15) == 0)) {
         const float4* r4 = reinterpret_cast<const float4*>(r);
 #pragma unroll
         for (int j = 0; j < 8; ++j) {
@@ -160,7 +170,7 @@ __device__ __forceinline__ void epi_chunk32(const Epi& e, int ra, int c0, int N,
     const int h = c0 / dh, d0 = c0 % dh;
     T* q = (T*)e.out_t + (size_t)ra * e.ld_t + h * dh;
     if (e.rope) {
-      rope_pairs<T>(q, d0 >> 1, half, v, e.rope_table + (size_t)rr.pos * half);
+      rope_pairs<T>(q, d0 >> 1, half, v, rr.rope ? rr.rope : e.rope_table + (size_t)rr.pos * half);
     } else {
       store16<T>(q + d0, v);
       store16<T>(q + d0 + 16, v + 16);
@@ -172,7 +182,7 @@ __device__ __forceinline__ void epi_chunk32(const Epi& e, int ra, int c0, int N,
     const int c = c0 - nq, h = c / dh, d0 = c % dh;
     T* k = (T*)e.cache.k + rr.cbase + (size_t)h * e.cache.head_stride();
     if (e.rope) {
-      rope_pairs<T>(k, d0 >> 1, half, v, e.rope_table + (size_t)rr.pos * half);
+      rope_pairs<T>(k, d0 >> 1, half, v, rr.rope ? rr.rope : e.rope_table + (size_t)rr.pos * half);
     } else {
       store16<T>(k + d0, v);
       store16<T>(k + d0 + 16, v + 16);

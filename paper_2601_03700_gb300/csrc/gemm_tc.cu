@@ -550,6 +550,12 @@ static bool encode_3d(CUtensorMap* m, const void* base, uint64_t K, uint64_t row
                   CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
+bool tc_encode_weight_3d(CUtensorMap* m, const void* base, int K, int rows, size_t row_bytes, int box_rows, int kc) {
+  init_once();
+  if (!g_encode) return false;
+  return encode_3d(m, base, (uint64_t)K, (uint64_t)rows, (uint64_t)row_bytes, (uint32_t)box_rows, (uint32_t)kc);
+}
+
 template <int MAXG>
 static int launch_grouped(cudaStream_t st, const GemmProblem* probs, int n_probs, const int* max_rows,
                           unsigned* err_word) {

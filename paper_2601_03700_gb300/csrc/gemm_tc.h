@@ -3,6 +3,8 @@
 #pragma once
 #include "common.cuh"
 
+#include <cuda.h>
+
 namespace adept {
 // True when the tensor-core path can run (bf16 operands, sm_100-family device).
 bool tc_gemm_supported();
@@ -11,4 +13,7 @@ int tc_gemm_grouped(cudaStream_t st, const GemmProblem* probs, int n_probs, cons
 // As tc_gemm_grouped, without the tensor-map cache (nothing is allocated on any heap).
 int tc_gemm_grouped_nocache(cudaStream_t st, const GemmProblem* probs, int n_probs, const int* max_rows,
                             unsigned* err_word);
+// 3-D view {64, rows, K/64} of a K-major bf16 matrix with box {64, box_rows, kc}, 128-byte
+// swizzle: one copy brings kc 64-wide k chunks of box_rows rows.  False if unsupported.
+bool tc_encode_weight_3d(CUtensorMap* m, const void* base, int K, int rows, size_t row_bytes, int box_rows, int kc);
 }  // namespace adept

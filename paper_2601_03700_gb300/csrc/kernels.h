@@ -10,7 +10,7 @@ enum : int {
   CTR_EXITED = 2,    // exits so far in this pass
   CTR_PREFIX = 3,    // [3 + i]: exits after layer i (i = 0..N)
 };
-static inline int ctr_words(int n_layers) { return CTR_PREFIX + n_layers + 2; }
+__host__ __device__ static inline int ctr_words(int n_layers) { return CTR_PREFIX + n_layers + 2; }
 
 void launch_pass_init(cudaStream_t st, int n_tok, int prompt_len, int decode, int* tok_seq, int* tok_pos,
                       int* row_tok, int* seq_len, int seq_cap, int max_pos, unsigned* err);
