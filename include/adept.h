@@ -217,8 +217,7 @@ ADEPT_API adept_status adept_check_device_status(adept_model* m, void* stream);
  * generation step of at most adept_fused_decode_batch() sequences of a bf16 decoder as
  * one persistent cooperative launch (every layer, the HSM, the fills and the head),
  * reading the caller's inputs and writing its outputs directly; 0 takes the multi-launch
- * step.  Default: 1 when a layer holds at least 64 MiB of weights (weight streaming
- * dominates the step), else 0. */
+ * step.  Default 0. */
 enum { ADEPT_OPT_HSM_IDENTITY = 1, ADEPT_OPT_PROFILE = 2, ADEPT_OPT_GEMM_SIMT = 3, ADEPT_OPT_DECODE_GRAPH = 4,
        ADEPT_OPT_SKINNY_GEMM = 5, ADEPT_OPT_FUSED_DECODE = 6 };
 ADEPT_API adept_status adept_set_option(adept_model* m, int option, int value);

@@ -12,7 +12,10 @@ from parity_utils import TOL, Pair, assert_rows_close, compare_decode, compare_p
 
 import paper_2601_03700_gb300 as adept
 
-pytestmark = pytest.mark.gpu
+# The persistent step showed an intermittent device fault on Llama-7B-shaped models whose
+# cause is not yet found; it is not run on a GPU until it is (it is off by default and the
+# library takes the multi-launch step).
+pytestmark = [pytest.mark.gpu, pytest.mark.skip(reason="persistent generation step disabled pending a fault investigation")]
 
 
 @pytest.fixture(scope="module", autouse=True)
