@@ -17,6 +17,7 @@ __global__ void __launch_bounds__(256) attn_warp_kernel(const T* __restrict__ q,
                                                         const int* tok_seq, const int* tok_pos, const int* seq_len,
                                                         KVCacheView cache, int layer0, int n_heads, int causal,
                                                         float scale) {
+  PDL_ENTRY();
   __shared__ float qs[8][DH];
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int gw = blockIdx.x * 8 + warp;
@@ -121,6 +122,7 @@ __global__ void __launch_bounds__(128) attn_prefill_mma_kernel(const bf16* __res
                                                                const int* tok_pos, const int* seq_len,
                                                                KVCacheView cache, int layer0, int n_heads, int causal,
                                                                float scale_log2) {
+  PDL_ENTRY();
   constexpr int LDS = DH + 8;  // padded rows: conflict-free ldmatrix
   constexpr int NB = DH / 8;   // 8-column blocks of the output
   extern __shared__ __align__(16) uint8_t attn_smem[];
@@ -317,6 +319,7 @@ __global__ void __launch_bounds__(128) attn_decode_split_kernel(const T* __restr
                                                                 KVCacheView cache, int layer0, int n_heads, int causal,
                                                                 float scale_log2, int chunk, int n_split,
                                                                 float* ws) {
+  PDL_ENTRY();
   constexpr int PD = DH / 4;   // dimensions per lane
   __shared__ float sm_m[4], sm_l[4];
   __shared__ float sm_o[4][DH];
@@ -404,6 +407,7 @@ __global__ void __launch_bounds__(128) attn_decode_split_kernel(const T* __restr
 template <typename T, int DH>
 __global__ void attn_decode_combine_kernel(DevRange rows, int n_heads, int n_split, const float* ws, T* out,
                                            int ld_out) {
+  PDL_ENTRY();
   const int rh = blockIdx.x;
   const int r = rows.b() + rh / n_heads, h = rh % n_heads;
   if (r >= rows.e()) return;
@@ -435,7 +439,7 @@ static void attn_dispatch(cudaStream_t st, const void* q, int ld_q, void* out, i
   const int grid = cdiv(max_rows * n_heads, 8);
 #define ATT_CASE(D)                                                                                         \
   case D:                                                                                                   \
-    attn_warp_kernel<T, D><<<grid, 256, 0, st>>>((const T*)q, ld_q, (T*)out, ld_out, rows, row_tok, tok_seq, \
+    launch_k(attn_warp_kernel<T, D>, grid, 256, 0, st, (const T*)q, ld_q, (T*)out, ld_out, rows, row_tok, tok_seq, \
                                                  tok_pos, seq_len, cache, layer0, n_heads, causal, scale);  \
     break;
   switch (dh) {
@@ -466,10 +470,10 @@ void launch_attention(cudaStream_t st, int dt, const void* q, int ld_q, void* ou
     dim3 grid(max_rows * n_heads, n_split);
 #define DEC_CASE(T, D)                                                                                       \
   {                                                                                                          \
-    attn_decode_split_kernel<T, D><<<grid, 128, 0, st>>>((const T*)q, ld_q, rows, row_tok, tok_seq, tok_pos, \
+    launch_k(attn_decode_split_kernel<T, D>, grid, 128, 0, st, (const T*)q, ld_q, rows, row_tok, tok_seq, tok_pos, \
                                                          seq_len, cache, layer0, n_heads, causal, scale_log2, \
                                                          chunk, n_split, ws);                                \
-    attn_decode_combine_kernel<T, D><<<max_rows * n_heads, 128, 0, st>>>(rows, n_heads, n_split, ws, (T*)out, \
+    launch_k(attn_decode_combine_kernel<T, D>, max_rows * n_heads, 128, 0, st, rows, n_heads, n_split, ws, (T*)out, \
                                                                          ld_out);                           \
   }
     if (dt == 1) {
@@ -488,7 +492,7 @@ void launch_attention(cudaStream_t st, int dt, const void* q, int ld_q, void* ou
         cudaFuncSetAttribute(attn_prefill_mma_kernel<64>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
         g_attn_smem_set[0] = 1;
       }
-      attn_prefill_mma_kernel<64><<<grid, 128, smem, st>>>((const bf16*)q, ld_q, (bf16*)out, ld_out, rows, row_tok,
+      launch_k(attn_prefill_mma_kernel<64>, grid, 128, smem, st, (const bf16*)q, ld_q, (bf16*)out, ld_out, rows, row_tok,
                                                            tok_seq, tok_pos, seq_len, cache, layer0, n_heads, causal,
                                                            scale_log2);
     } else {
@@ -496,7 +500,7 @@ void launch_attention(cudaStream_t st, int dt, const void* q, int ld_q, void* ou
         cudaFuncSetAttribute(attn_prefill_mma_kernel<128>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
         g_attn_smem_set[1] = 1;
       }
-      attn_prefill_mma_kernel<128><<<grid, 128, smem, st>>>((const bf16*)q, ld_q, (bf16*)out, ld_out, rows, row_tok,
+      launch_k(attn_prefill_mma_kernel<128>, grid, 128, smem, st, (const bf16*)q, ld_q, (bf16*)out, ld_out, rows, row_tok,
                                                             tok_seq, tok_pos, seq_len, cache, layer0, n_heads, causal,
                                                             scale_log2);
     }

@@ -4,6 +4,8 @@
 #include <cuda_bf16.h>
 #include <stdint.h>
 
+#include <utility>
+
 typedef __nv_bfloat16 bf16;
 
 // Device error word bits (read by adept_check_device_status).
@@ -15,6 +17,41 @@ enum : unsigned {
   ERRW_TIMEOUT = 16u,  // a bounded device-side wait gave up
   ERRW_CONFIG = 32u    // a kernel was launched with a shape it does not support
 };
+
+// Programmatic dependent launch.  Every kernel of the library begins with PDL_ENTRY: it
+// waits until the kernels it depends on have completed and their writes are visible (a no-op
+// when it was launched without the programmatic attribute), then lets the next kernel of the
+// stream be launched, so that kernel's launch and prologue overlap this one.  Work placed
+// before the wait may touch nothing a preceding kernel writes.
+__device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+__device__ __forceinline__ void pdl_launch_dependents() { asm volatile("griddepcontrol.launch_dependents;" ::: "memory"); }
+#define PDL_ENTRY()            \
+  do {                         \
+    pdl_wait();                \
+    pdl_launch_dependents();   \
+  } while (0)
+
+namespace adept {
+// Launches with the programmatic-serialisation attribute while g_pdl is set (each entry
+// point sets it for its calling thread; it is off while per-launch profiling events are
+// recorded, so each timed interval holds one kernel alone).
+extern thread_local bool g_pdl;
+template <typename... KArgs, typename... Args>
+inline cudaError_t launch_k(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t smem, cudaStream_t st,
+                            Args&&... args) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = grid;
+  cfg.blockDim = block;
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = st;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = g_pdl ? 1 : 0;
+  return cudaLaunchKernelEx(&cfg, kernel, std::forward<Args>(args)...);
+}
+}  // namespace adept
 
 template <typename T> __device__ __forceinline__ float to_f(T x);
 template <> __device__ __forceinline__ float to_f<float>(float x) { return x; }

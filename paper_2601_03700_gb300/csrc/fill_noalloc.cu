@@ -59,6 +59,7 @@ extern "C" ADEPT_API adept_status adept_skip_kv_fill_noalloc(adept_model* m, int
                                                              const int32_t* d_exit_layer, const int32_t* d_seq,
                                                              const int32_t* d_pos, void* stream) {
   if (!m) return ADEPT_ERR_INVALID_ARG;
+  g_pdl = true;  // this entry point records no profiling events
   if (n_tokens < 0) {
     model_set_error(m, "n_tokens < 0");
     return ADEPT_ERR_INVALID_ARG;

@@ -11,6 +11,7 @@ namespace adept {
 template <typename T>
 __global__ void __launch_bounds__(256) gemm_simt_kernel(const T* __restrict__ A, int lda, const T* __restrict__ B,
                                                         int ldb, DevRange rows, int N, int K, float* C, int ldc) {
+  PDL_ENTRY();
   __shared__ float As[16][64 + 1];
   __shared__ float Bs[16][64 + 1];
   const int rb = rows.b(), M = rows.e() - rb;
@@ -55,6 +56,7 @@ __global__ void __launch_bounds__(256) gemm_simt_kernel(const T* __restrict__ A,
 // Epilogue of one output row (see EpiKind), one thread per 32-column chunk.
 template <typename T>
 __global__ void epilogue_kernel(Epi e, const float* __restrict__ C, int ldc, DevRange rows, int N) {
+  PDL_ENTRY();
   const int rb = rows.b(), M = rows.e() - rb;
   const int r = blockIdx.x;
   if (r >= M) return;
@@ -74,13 +76,13 @@ void launch_gemm_simt(cudaStream_t st, int dt, const GemmProblem& p, int max_row
   if (max_rows <= 0) return;
   dim3 grid(cdiv(p.N, 64), cdiv(max_rows, 64));
   if (dt == 1) {
-    gemm_simt_kernel<bf16><<<grid, 256, 0, st>>>((const bf16*)p.A, p.lda, (const bf16*)p.B, p.ldb, p.rows, p.N, p.K,
+    launch_k(gemm_simt_kernel<bf16>, grid, 256, 0, st, (const bf16*)p.A, p.lda, (const bf16*)p.B, p.ldb, p.rows, p.N, p.K,
                                                  scratch, p.N);
-    epilogue_kernel<bf16><<<max_rows, 64, 0, st>>>(p.epi, scratch, p.N, p.rows, p.N);
+    launch_k(epilogue_kernel<bf16>, max_rows, 64, 0, st, p.epi, scratch, p.N, p.rows, p.N);
   } else {
-    gemm_simt_kernel<float><<<grid, 256, 0, st>>>((const float*)p.A, p.lda, (const float*)p.B, p.ldb, p.rows, p.N,
+    launch_k(gemm_simt_kernel<float>, grid, 256, 0, st, (const float*)p.A, p.lda, (const float*)p.B, p.ldb, p.rows, p.N,
                                                   p.K, scratch, p.N);
-    epilogue_kernel<float><<<max_rows, 64, 0, st>>>(p.epi, scratch, p.N, p.rows, p.N);
+    launch_k(epilogue_kernel<float>, max_rows, 64, 0, st, p.epi, scratch, p.N, p.rows, p.N);
   }
 }
 

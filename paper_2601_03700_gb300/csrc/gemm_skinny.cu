@@ -68,6 +68,7 @@ __device__ __forceinline__ void sk_mma(float (&c)[4], const uint32_t (&a)[4], ui
 
 template <int MAXG, int MB>   // MB: 8-token blocks (1..4)
 __global__ void __launch_bounds__(SK_THREADS) gemm_skinny_kernel(const __grid_constant__ SkParams<MAXG> p) {
+  PDL_ENTRY();
   extern __shared__ __align__(16) uint8_t sk_smem[];
   bf16* sW = reinterpret_cast<bf16*>(sk_smem);                          // [STAGES][64][LDS]
   bf16* sA = sW + SK_STAGES * SK_BN * SK_LDS;                           // [STAGES][32][LDS]
@@ -204,7 +205,7 @@ static void launch_mb(cudaStream_t st, const SkParams<MAXG>& prm, int grid) {
     cudaFuncSetAttribute(gemm_skinny_kernel<MAXG, MB>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
     attr = true;
   }
-  gemm_skinny_kernel<MAXG, MB><<<grid, SK_THREADS, smem, st>>>(prm);
+  launch_k(gemm_skinny_kernel<MAXG, MB>, grid, SK_THREADS, smem, st, prm);
 }
 
 template <int MAXG>

@@ -216,6 +216,30 @@ __global__ void __launch_bounds__(TC_THREADS, 1) gemm_tc_kernel(const __grid_con
     g_tc_trace[tr_slot][9] = gridDim.x * 1000 + BN;
   }
 #endif
+  // Prologue that touches nothing an earlier kernel writes: barriers, the first group's
+  // tensor maps (kernel parameters), the TMEM allocation.  Then wait for the preceding
+  // kernels (programmatic dependent launch) and build the tile tables, which read row
+  // counts those kernels produced.
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < STAGES; ++s) {
+      mbar_init(&full[s], 1);
+      mbar_init(&empty[s], 1);
+    }
+    for (int b = 0; b < 2; ++b) {
+      mbar_init(&accf[b], 1);
+      mbar_init(&acce[b], 4);
+    }
+    mbar_init(drain, 1);
+    *abort_flag = 0;
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+    asm volatile("prefetch.tensormap [%0];" ::"l"((uint64_t)&p.g[0].ta) : "memory");
+    asm volatile("prefetch.tensormap [%0];" ::"l"((uint64_t)&p.g[0].tb) : "memory");
+  }
+  if (warp == 1) {
+    tmem_alloc(tmem_slot, TMEM_COLS);
+    tmem_relinquish();
+  }
+  pdl_wait();
   if (threadIdx.x == 0) {
     int acc = 0;
     for (int g = 0; g < ng; ++g) {
@@ -231,37 +255,27 @@ __global__ void __launch_bounds__(TC_THREADS, 1) gemm_tc_kernel(const __grid_con
       acc += s_tm[g] * tn;
     }
     s_tile0[ng] = acc;
-    for (int s = 0; s < STAGES; ++s) {
-      mbar_init(&full[s], 1);
-      mbar_init(&empty[s], 1);
-    }
-    for (int b = 0; b < 2; ++b) {
-      mbar_init(&accf[b], 1);
-      mbar_init(&acce[b], 4);
-    }
-    mbar_init(drain, 1);
-    *abort_flag = 0;
-    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
-  }
-  __syncthreads();
-  const int total = s_tile0[ng];
-  if ((int)blockIdx.x >= total) return;  // uniform: nothing allocated yet
-  if (threadIdx.x == 0) {
-    // pull the first tile's tensor maps in while the barriers and TMEM are set up
-    int g0 = 0;
-    while (g0 + 1 < ng && (int)blockIdx.x >= s_tile0[g0 + 1]) ++g0;
-    asm volatile("prefetch.tensormap [%0];" ::"l"((uint64_t)&p.g[g0].ta) : "memory");
-    asm volatile("prefetch.tensormap [%0];" ::"l"((uint64_t)&p.g[g0].tb) : "memory");
-  }
-
-  if (warp == 1) {
-    tmem_alloc(tmem_slot, TMEM_COLS);
-    tmem_relinquish();
   }
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
+  pdl_launch_dependents();   // after the TMEM allocation: a dependent CTA cannot take it first
+  const int total = s_tile0[ng];
   const uint32_t tmem = *tmem_slot;
+  if ((int)blockIdx.x >= total) {
+    // no tile for this CTA (uniform): give the tensor memory back and leave
+    if (warp == 1) tmem_dealloc(tmem, TMEM_COLS);
+    return;
+  }
+  if (threadIdx.x == 0 && ng > 1) {
+    // the first tile's tensor maps, if they are not the first group's
+    int g0 = 0;
+    while (g0 + 1 < ng && (int)blockIdx.x >= s_tile0[g0 + 1]) ++g0;
+    if (g0 > 0) {
+      asm volatile("prefetch.tensormap [%0];" ::"l"((uint64_t)&p.g[g0].ta) : "memory");
+      asm volatile("prefetch.tensormap [%0];" ::"l"((uint64_t)&p.g[g0].tb) : "memory");
+    }
+  }
   if (threadIdx.x == 0) TC_TRACE(1);
 
   // Tile order inside a problem: super-rows of gm m-tiles; within a super-row n is the
@@ -532,7 +546,7 @@ static int launch_bn(cudaStream_t st, const TcParams<MAXG>& prm, int grid) {
                          (int)smem);
     attr = true;
   }
-  gemm_tc_kernel<BN, STAGES, MAXG, KC><<<grid, TC_THREADS, smem, st>>>(prm);
+  launch_k(gemm_tc_kernel<BN, STAGES, MAXG, KC>, grid, TC_THREADS, smem, st, prm);
   return 1;
 }
 

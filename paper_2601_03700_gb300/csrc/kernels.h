@@ -12,8 +12,11 @@ enum : int {
 };
 __host__ __device__ static inline int ctr_words(int n_layers) { return CTR_PREFIX + n_layers + 2; }
 
+// Token -> (sequence, position) maps, identity row map, the pass's counters (all rows
+// active) and, if sim is given, NaN for every (token, layer) similarity.
 void launch_pass_init(cudaStream_t st, int n_tok, int prompt_len, int decode, int* tok_seq, int* tok_pos,
-                      int* row_tok, int* seq_len, int seq_cap, int max_pos, unsigned* err);
+                      int* row_tok, int* seq_len, int seq_cap, int max_pos, unsigned* err, int* ctr, int n_ctr,
+                      float* sim, int n_layers);
 void launch_embed(cudaStream_t st, int dt, const int* tokens, int n_tok, const int* tok_pos, const void* E,
                   const void* P, const float* type_emb, const float* g, const float* b, int family, int D, int V,
                   float eps, float* X, unsigned* err);

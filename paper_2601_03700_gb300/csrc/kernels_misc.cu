@@ -6,15 +6,24 @@
 
 #include <math.h>
 
+#include <algorithm>
+
 namespace adept {
 
 // ---------------------------------------------------------------------------
 // pass set-up: token -> (sequence, position), identity row map, counters
 // ---------------------------------------------------------------------------
 __global__ void pass_init_kernel(int n_tok, int prompt_len, int decode, int* tok_seq, int* tok_pos,
-                                 int* row_tok, int* seq_len, int seq_cap, int max_pos, unsigned* err) {
+                                 int* row_tok, int* seq_len, int seq_cap, int max_pos, unsigned* err, int* ctr,
+                                 int n_ctr, float* sim, int n_layers) {
+  PDL_ENTRY();
   const int t = blockIdx.x * blockDim.x + threadIdx.x;
+  // the pass's counters: all active, nothing exited
+  if (t < n_ctr) ctr[t] = t == CTR_ACTIVE ? n_tok : 0;
   if (t >= n_tok) return;
+  // similarities not tested stay NaN
+  if (sim)
+    for (int l = 0; l < n_layers; ++l) sim[(size_t)t * n_layers + l] = __int_as_float(0x7fffffff);
   int s, p;
   if (decode) {
     s = t;
@@ -41,6 +50,7 @@ template <typename T>
 __global__ void embed_kernel(const int* tokens, int n_tok, const int* tok_pos, const T* E, const T* P,
                              const float* type_emb, const float* g, const float* b, int family, int D, int V,
                              float eps, float* X, unsigned* err) {
+  PDL_ENTRY();
   __shared__ float red[32];
   const int t = blockIdx.x;
   if (t >= n_tok) return;
@@ -76,6 +86,7 @@ __global__ void embed_kernel(const int* tokens, int n_tok, const int* tok_pos, c
 template <typename T>
 __global__ void standardize_kernel(const float* X, int ldx, const int* in_rows, DevRange rows, int D, int mode,
                                    float eps, T* out, int ld_out) {
+  PDL_ENTRY();
   __shared__ float red[32];
   const int r = rows.b() + blockIdx.x;
   if (r >= rows.e()) return;
@@ -103,6 +114,7 @@ __global__ void standardize_kernel(const float* X, int ldx, const int* in_rows, 
 
 // In-place LayerNorm with gain and shift (the post-LN encoder's residual stream).
 __global__ void layernorm_inplace_kernel(float* X, DevRange rows, int D, const float* g, const float* b, float eps) {
+  PDL_ENTRY();
   __shared__ float red[32];
   const int r = rows.b() + blockIdx.x;
   if (r >= rows.e()) return;
@@ -125,6 +137,7 @@ __global__ void layernorm_inplace_kernel(float* X, DevRange rows, int D, const f
 __global__ void exit_decide_kernel(const float* Xout, const float* I, int D, DevRange rows, const int* row_tok,
                                    const int* forced, int layer, int n_layers, const float* delta_p, int test,
                                    float* sim, int* flag, float* inv_norm, unsigned* err) {
+  PDL_ENTRY();
   const int warp = (blockIdx.x * blockDim.x + threadIdx.x) >> 5, lane = threadIdx.x & 31;
   const int r = warp;
   if (r >= rows.e()) return;
@@ -160,6 +173,7 @@ __global__ void exit_decide_kernel(const float* Xout, const float* I, int D, Dev
 // ctr[CTR_PREFIX + i] exits after layer i.
 __global__ void exit_scan_kernel(int* ctr, int in_parity, const int* flag, const int* row_tok, int* row_tok_next,
                                  int* exit_tok, int* dst, int* exit_layer_out, int layer) {
+  PDL_ENTRY();
   __shared__ int s_stay[1024];
   __shared__ int s_exit[1024];
   const int n = ctr[CTR_ACTIVE + in_parity];
@@ -213,6 +227,7 @@ __global__ void exit_scan_kernel(int* ctr, int in_parity, const int* flag, const
 __global__ void exit_move_kernel(const float* Xin, const float* Xout, const float* I, int first, int D,
                                  const int* n_rows, const int* dst, const float* inv_norm, float* Xnext, float* Inext,
                                  float* hsm_s, float* hsm_prev, float* hsm_I) {
+  PDL_ENTRY();
   const int r = blockIdx.x;
   if (r >= *n_rows) return;
   const int d0 = dst[r];
@@ -247,6 +262,7 @@ __global__ void __launch_bounds__(256) exit_small_kernel(const float* Xin, const
                                                          int* exit_tok, int* exit_layer_out, float* Xnext,
                                                          float* Inext, float* hsm_s, float* hsm_prev, float* hsm_I,
                                                          unsigned* err) {
+  PDL_ENTRY();
   __shared__ int s_dst[EXIT_SMALL_MAX];
   __shared__ float s_w[EXIT_SMALL_MAX];
   const int n = min(ctr[CTR_ACTIVE + par], EXIT_SMALL_MAX);
@@ -330,17 +346,19 @@ void launch_exit_small(cudaStream_t st, const float* Xin, const float* Xout, con
                        int* ctr, int par, const int* row_tok, int* row_tok_next, const int* forced, int layer,
                        int n_layers, const float* delta_p, int test, float* sim, int* exit_tok, int* exit_layer_out,
                        float* Xnext, float* Inext, float* hsm_s, float* hsm_prev, float* hsm_I, unsigned* err) {
-  exit_small_kernel<<<1, 256, 0, st>>>(Xin, Xout, I, first, D, ctr, par, row_tok, row_tok_next, forced, layer,
+  launch_k(exit_small_kernel, 1, 256, 0, st, Xin, Xout, I, first, D, ctr, par, row_tok, row_tok_next, forced, layer,
                                        n_layers, delta_p, test, sim, exit_tok, exit_layer_out, Xnext, Inext, hsm_s,
                                        hsm_prev, hsm_I, err);
 }
 
-__global__ void set_float_kernel(float* p, float v) { *p = v; }
-void launch_set_float(cudaStream_t st, float* p, float v) { set_float_kernel<<<1, 1, 0, st>>>(p, v); }
+__global__ void set_float_kernel(float* p, float v) {
+  PDL_ENTRY(); *p = v; }
+void launch_set_float(cudaStream_t st, float* p, float v) { launch_k(set_float_kernel, 1, 1, 0, st, p, v); }
 
 // After layer N: the remaining active rows' s_N are their final states.
 __global__ void final_scatter_kernel(const float* X, int D, const int* n_rows, const int* row_tok, float* final_,
                                      int* exit_layer_out, int n_layers) {
+  PDL_ENTRY();
   const int r = blockIdx.x;
   if (r >= *n_rows) return;
   const int tok = row_tok[r];
@@ -357,6 +375,7 @@ template <typename T>
 __global__ void hsm_prep_kernel(const float* hs, const float* hp, const float* hI, DevRange rows, int D,
                                 const float* g0, const float* conv /* 9 taps + bias */, float eps, float* c0f,
                                 T* c0t) {
+  PDL_ENTRY();
   __shared__ float red[32];
   const int k = rows.b() + blockIdx.x;
   if (k >= rows.e()) return;
@@ -387,6 +406,7 @@ __global__ void hsm_prep_kernel(const float* hs, const float* hp, const float* h
 template <typename T>
 __global__ void hsm_mid_kernel(const float* h3, const float* h1, DevRange rows, int m1, const float* g1, float eps,
                                T* h4) {
+  PDL_ENTRY();
   __shared__ float red[32];
   const int k = rows.b() + blockIdx.x;
   if (k >= rows.e()) return;
@@ -405,6 +425,7 @@ template <typename T>
 __global__ void hsm_out_kernel(const float* h5, const float* c0f, const float* hs, int identity, DevRange rows, int D,
                                const float* g2, float eps, const int* exit_tok, float* final_, T* xfill,
                                int fill_mode, float norm_eps) {
+  PDL_ENTRY();
   __shared__ float red[32];
   const int k = rows.b() + blockIdx.x;
   if (k >= rows.e()) return;
@@ -444,6 +465,7 @@ __global__ void hsm_out_kernel(const float* h5, const float* c0f, const float* h
 // greedy token: argmax with the lowest index on ties
 // ---------------------------------------------------------------------------
 __global__ void argmax_kernel(const float* logits, int V, int rows, int* out) {
+  PDL_ENTRY();
   __shared__ float sv[32];
   __shared__ int si[32];
   const int r = blockIdx.x;
@@ -485,6 +507,7 @@ __global__ void argmax_kernel(const float* logits, int V, int rows, int* out) {
 
 // Rows of the last position of each sequence (decoder head) or of position 0 (encoder).
 __global__ void head_rows_kernel(int batch, int prompt_len, int last, int* rows) {
+  PDL_ENTRY();
   const int b = blockIdx.x * blockDim.x + threadIdx.x;
   if (b < batch) rows[b] = b * prompt_len + (last ? prompt_len - 1 : 0);
 }
@@ -494,6 +517,7 @@ __global__ void head_rows_kernel(int batch, int prompt_len, int last, int* rows)
 // skipped layer r (tokens with i* < r) are a prefix, and standardise s~ once.
 // ---------------------------------------------------------------------------
 __global__ void fill_hist_kernel(const int* exit_layer, int n, int n_layers, int* hist, unsigned* err) {
+  PDL_ENTRY();
   const int j = blockIdx.x * blockDim.x + threadIdx.x;
   if (j >= n) return;
   int l = exit_layer[j];
@@ -506,6 +530,7 @@ __global__ void fill_hist_kernel(const int* exit_layer, int n, int n_layers, int
 
 // hist[1..N] -> start[l] (exclusive prefix) and prefix[r] = #(i* < r) = start[r].
 __global__ void fill_scan_kernel(const int* hist, int n_layers, int* start, int* cursor) {
+  PDL_ENTRY();
   if (threadIdx.x != 0 || blockIdx.x != 0) return;
   int acc = 0;
   for (int l = 0; l <= n_layers + 1; ++l) {
@@ -518,6 +543,7 @@ __global__ void fill_scan_kernel(const int* hist, int n_layers, int* start, int*
 template <typename T>
 __global__ void fill_scatter_kernel(const T* h, int n, int D, const int* exit_layer, int n_layers, const int* start,
                                     int* cursor, int* sorted_tok, T* xs, int mode, float eps) {
+  PDL_ENTRY();
   __shared__ float red[32];
   __shared__ int s_slot;
   const int j = blockIdx.x;
@@ -558,6 +584,7 @@ __global__ void fill_scatter_kernel(const T* h, int n, int D, const int* exit_la
 template <typename T>
 __global__ void fold_rows_kernel(T* dst, int ld_dst, const T* src, int n_rows, int K, const float* gamma,
                                  const float* beta, const float* bias_in, float* bias_out, int row_mode) {
+  PDL_ENTRY();
   const int warp = (blockIdx.x * blockDim.x + threadIdx.x) >> 5, lane = threadIdx.x & 31;
   if (warp >= n_rows) return;
   const int n = warp;
@@ -585,6 +612,7 @@ __global__ void fold_rows_kernel(T* dst, int ld_dst, const T* src, int n_rows, i
 
 template <typename T>
 __global__ void to_f32_kernel(const T* src, float* dst, int n) {
+  PDL_ENTRY();
   const int i = blockIdx.x * blockDim.x + threadIdx.x;
   if (i < n) dst[i] = to_f(src[i]);
 }
@@ -592,6 +620,7 @@ __global__ void to_f32_kernel(const T* src, float* dst, int n) {
 // Copy n_pos positions of one sequence / layer out of the paged cache.
 template <typename T>
 __global__ void read_kv_kernel(KVCacheView c, int layer0, int seq, int pos0, int n_pos, T* ko, T* vo) {
+  PDL_ENTRY();
   const int p = blockIdx.x;
   if (p >= n_pos) return;
   const int per = c.n_kv_heads * c.head_dim;
@@ -607,19 +636,20 @@ __global__ void read_kv_kernel(KVCacheView c, int layer0, int seq, int pos0, int
 // launchers
 // ---------------------------------------------------------------------------
 void launch_pass_init(cudaStream_t st, int n_tok, int prompt_len, int decode, int* tok_seq, int* tok_pos,
-                      int* row_tok, int* seq_len, int seq_cap, int max_pos, unsigned* err) {
-  pass_init_kernel<<<cdiv(n_tok, 256), 256, 0, st>>>(n_tok, prompt_len, decode, tok_seq, tok_pos, row_tok, seq_len,
-                                                    seq_cap, max_pos, err);
+                      int* row_tok, int* seq_len, int seq_cap, int max_pos, unsigned* err, int* ctr, int n_ctr,
+                      float* sim, int n_layers) {
+  launch_k(pass_init_kernel, cdiv(std::max(n_tok, n_ctr), 256), 256, 0, st, n_tok, prompt_len, decode, tok_seq, tok_pos,
+           row_tok, seq_len, seq_cap, max_pos, err, ctr, n_ctr, sim, n_layers);
 }
 
 void launch_embed(cudaStream_t st, int dt, const int* tokens, int n_tok, const int* tok_pos, const void* E,
                   const void* P, const float* type_emb, const float* g, const float* b, int family, int D, int V,
                   float eps, float* X, unsigned* err) {
   if (dt == 1)
-    embed_kernel<bf16><<<n_tok, 256, 0, st>>>(tokens, n_tok, tok_pos, (const bf16*)E, (const bf16*)P, type_emb, g, b,
+    launch_k(embed_kernel<bf16>, n_tok, 256, 0, st, tokens, n_tok, tok_pos, (const bf16*)E, (const bf16*)P, type_emb, g, b,
                                               family, D, V, eps, X, err);
   else
-    embed_kernel<float><<<n_tok, 256, 0, st>>>(tokens, n_tok, tok_pos, (const float*)E, (const float*)P, type_emb, g,
+    launch_k(embed_kernel<float>, n_tok, 256, 0, st, tokens, n_tok, tok_pos, (const float*)E, (const float*)P, type_emb, g,
                                                b, family, D, V, eps, X, err);
 }
 
@@ -627,28 +657,28 @@ void launch_standardize(cudaStream_t st, int dt, const float* X, int ldx, const 
                         int max_rows, int D, int mode, float eps, void* out, int ld_out) {
   if (max_rows <= 0) return;
   if (dt == 1)
-    standardize_kernel<bf16><<<max_rows, 256, 0, st>>>(X, ldx, in_rows, rows, D, mode, eps, (bf16*)out, ld_out);
+    launch_k(standardize_kernel<bf16>, max_rows, 256, 0, st, X, ldx, in_rows, rows, D, mode, eps, (bf16*)out, ld_out);
   else
-    standardize_kernel<float><<<max_rows, 256, 0, st>>>(X, ldx, in_rows, rows, D, mode, eps, (float*)out, ld_out);
+    launch_k(standardize_kernel<float>, max_rows, 256, 0, st, X, ldx, in_rows, rows, D, mode, eps, (float*)out, ld_out);
 }
 
 void launch_layernorm_inplace(cudaStream_t st, float* X, DevRange rows, int max_rows, int D, const float* g,
                               const float* b, float eps) {
   if (max_rows <= 0) return;
-  layernorm_inplace_kernel<<<max_rows, 256, 0, st>>>(X, rows, D, g, b, eps);
+  launch_k(layernorm_inplace_kernel, max_rows, 256, 0, st, X, rows, D, g, b, eps);
 }
 
 void launch_exit_decide(cudaStream_t st, const float* Xout, const float* I, int D, DevRange rows, int max_rows,
                         const int* row_tok, const int* forced, int layer, int n_layers, const float* delta_p, int test,
                         float* sim, int* flag, float* inv_norm, unsigned* err) {
   if (max_rows <= 0) return;
-  exit_decide_kernel<<<cdiv(max_rows, 8), 256, 0, st>>>(Xout, I, D, rows, row_tok, forced, layer, n_layers, delta_p,
+  launch_k(exit_decide_kernel, cdiv(max_rows, 8), 256, 0, st, Xout, I, D, rows, row_tok, forced, layer, n_layers, delta_p,
                                                        test, sim, flag, inv_norm, err);
 }
 
 void launch_exit_scan(cudaStream_t st, int* ctr, int in_parity, const int* flag, const int* row_tok,
                       int* row_tok_next, int* exit_tok, int* dst, int* exit_layer_out, int layer) {
-  exit_scan_kernel<<<1, 1024, 0, st>>>(ctr, in_parity, flag, row_tok, row_tok_next, exit_tok, dst, exit_layer_out,
+  launch_k(exit_scan_kernel, 1, 1024, 0, st, ctr, in_parity, flag, row_tok, row_tok_next, exit_tok, dst, exit_layer_out,
                                        layer);
 }
 
@@ -656,30 +686,30 @@ void launch_exit_move(cudaStream_t st, const float* Xin, const float* Xout, cons
                       const int* n_rows, int max_rows, const int* dst, const float* inv_norm, float* Xnext,
                       float* Inext, float* hsm_s, float* hsm_prev, float* hsm_I) {
   if (max_rows <= 0) return;
-  exit_move_kernel<<<max_rows, 256, 0, st>>>(Xin, Xout, I, first, D, n_rows, dst, inv_norm, Xnext, Inext, hsm_s,
+  launch_k(exit_move_kernel, max_rows, 256, 0, st, Xin, Xout, I, first, D, n_rows, dst, inv_norm, Xnext, Inext, hsm_s,
                                              hsm_prev, hsm_I);
 }
 
 void launch_final_scatter(cudaStream_t st, const float* X, int D, const int* n_rows, int max_rows, const int* row_tok,
                           float* final_, int* exit_layer_out, int n_layers) {
   if (max_rows <= 0) return;
-  final_scatter_kernel<<<max_rows, 256, 0, st>>>(X, D, n_rows, row_tok, final_, exit_layer_out, n_layers);
+  launch_k(final_scatter_kernel, max_rows, 256, 0, st, X, D, n_rows, row_tok, final_, exit_layer_out, n_layers);
 }
 
 void launch_hsm_prep(cudaStream_t st, int dt, const float* hs, const float* hp, const float* hI, DevRange rows,
                      int max_rows, int D, const float* g0, const float* conv, float eps, float* c0f, void* c0t) {
   if (max_rows <= 0) return;
   if (dt == 1)
-    hsm_prep_kernel<bf16><<<max_rows, 256, 0, st>>>(hs, hp, hI, rows, D, g0, conv, eps, c0f, (bf16*)c0t);
+    launch_k(hsm_prep_kernel<bf16>, max_rows, 256, 0, st, hs, hp, hI, rows, D, g0, conv, eps, c0f, (bf16*)c0t);
   else
-    hsm_prep_kernel<float><<<max_rows, 256, 0, st>>>(hs, hp, hI, rows, D, g0, conv, eps, c0f, (float*)c0t);
+    launch_k(hsm_prep_kernel<float>, max_rows, 256, 0, st, hs, hp, hI, rows, D, g0, conv, eps, c0f, (float*)c0t);
 }
 
 void launch_hsm_mid(cudaStream_t st, int dt, const float* h3, const float* h1, DevRange rows, int max_rows, int m1,
                     const float* g1, float eps, void* h4) {
   if (max_rows <= 0) return;
-  if (dt == 1) hsm_mid_kernel<bf16><<<max_rows, 256, 0, st>>>(h3, h1, rows, m1, g1, eps, (bf16*)h4);
-  else hsm_mid_kernel<float><<<max_rows, 256, 0, st>>>(h3, h1, rows, m1, g1, eps, (float*)h4);
+  if (dt == 1) launch_k(hsm_mid_kernel<bf16>, max_rows, 256, 0, st, h3, h1, rows, m1, g1, eps, (bf16*)h4);
+  else launch_k(hsm_mid_kernel<float>, max_rows, 256, 0, st, h3, h1, rows, m1, g1, eps, (float*)h4);
 }
 
 void launch_hsm_out(cudaStream_t st, int dt, const float* h5, const float* c0f, const float* hs, int identity,
@@ -687,10 +717,10 @@ void launch_hsm_out(cudaStream_t st, int dt, const float* h5, const float* c0f, 
                     float* final_, void* xfill, int fill_mode, float norm_eps) {
   if (max_rows <= 0) return;
   if (dt == 1)
-    hsm_out_kernel<bf16><<<max_rows, 256, 0, st>>>(h5, c0f, hs, identity, rows, D, g2, eps, exit_tok, final_,
+    launch_k(hsm_out_kernel<bf16>, max_rows, 256, 0, st, h5, c0f, hs, identity, rows, D, g2, eps, exit_tok, final_,
                                                    (bf16*)xfill, fill_mode, norm_eps);
   else
-    hsm_out_kernel<float><<<max_rows, 256, 0, st>>>(h5, c0f, hs, identity, rows, D, g2, eps, exit_tok, final_,
+    launch_k(hsm_out_kernel<float>, max_rows, 256, 0, st, h5, c0f, hs, identity, rows, D, g2, eps, exit_tok, final_,
                                                     (float*)xfill, fill_mode, norm_eps);
 }
 
@@ -698,6 +728,7 @@ void launch_hsm_out(cudaStream_t st, int dt, const float* h5, const float* c0f, 
 // (value, index) pairs, one thread per row merges them (lowest index on ties).
 constexpr int ARGMAX_SPLIT = 32;
 __global__ void argmax_part_kernel(const float* logits, int V, int rows, float* pv, int* pi) {
+  PDL_ENTRY();
   __shared__ float sv[32];
   __shared__ int si[32];
   const int r = blockIdx.x / ARGMAX_SPLIT, part = blockIdx.x % ARGMAX_SPLIT;
@@ -741,6 +772,7 @@ __global__ void argmax_part_kernel(const float* logits, int V, int rows, float* 
 }
 
 __global__ void argmax_merge_kernel(const float* pv, const int* pi, int rows, int* out) {
+  PDL_ENTRY();
   const int r = blockIdx.x * blockDim.x + threadIdx.x;
   if (r >= rows) return;
   float bv = -INFINITY;
@@ -759,54 +791,54 @@ __global__ void argmax_merge_kernel(const float* pv, const int* pi, int rows, in
 int launch_argmax(cudaStream_t st, const float* logits, int V, int rows, int* out, float* part_v, int* part_i) {
   if (rows <= 0) return 0;
   if (V <= 4096 || !part_v || !part_i) {
-    argmax_kernel<<<rows, 256, 0, st>>>(logits, V, rows, out);
+    launch_k(argmax_kernel, rows, 256, 0, st, logits, V, rows, out);
     return 1;
   }
-  argmax_part_kernel<<<rows * ARGMAX_SPLIT, 256, 0, st>>>(logits, V, rows, part_v, part_i);
-  argmax_merge_kernel<<<cdiv(rows, 64), 64, 0, st>>>(part_v, part_i, rows, out);
+  launch_k(argmax_part_kernel, rows * ARGMAX_SPLIT, 256, 0, st, logits, V, rows, part_v, part_i);
+  launch_k(argmax_merge_kernel, cdiv(rows, 64), 64, 0, st, part_v, part_i, rows, out);
   return 2;
 }
 
 void launch_head_rows(cudaStream_t st, int batch, int prompt_len, int last, int* rows) {
-  head_rows_kernel<<<cdiv(batch, 128), 128, 0, st>>>(batch, prompt_len, last, rows);
+  launch_k(head_rows_kernel, cdiv(batch, 128), 128, 0, st, batch, prompt_len, last, rows);
 }
 
 void launch_fill_sort(cudaStream_t st, int dt, const void* h, int n, int D, const int* exit_layer, int n_layers,
                       int* hist, int* start, int* cursor, int* sorted_tok, void* xs, int mode, float eps,
                       unsigned* err) {
   cudaMemsetAsync(hist, 0, sizeof(int) * (n_layers + 2), st);
-  if (n > 0) fill_hist_kernel<<<cdiv(n, 256), 256, 0, st>>>(exit_layer, n, n_layers, hist, err);
-  fill_scan_kernel<<<1, 32, 0, st>>>(hist, n_layers, start, cursor);
+  if (n > 0) launch_k(fill_hist_kernel, cdiv(n, 256), 256, 0, st, exit_layer, n, n_layers, hist, err);
+  launch_k(fill_scan_kernel, 1, 32, 0, st, hist, n_layers, start, cursor);
   if (n <= 0) return;
   if (dt == 1)
-    fill_scatter_kernel<bf16><<<n, 256, 0, st>>>((const bf16*)h, n, D, exit_layer, n_layers, start, cursor,
+    launch_k(fill_scatter_kernel<bf16>, n, 256, 0, st, (const bf16*)h, n, D, exit_layer, n_layers, start, cursor,
                                                  sorted_tok, (bf16*)xs, mode, eps);
   else
-    fill_scatter_kernel<float><<<n, 256, 0, st>>>((const float*)h, n, D, exit_layer, n_layers, start, cursor,
+    launch_k(fill_scatter_kernel<float>, n, 256, 0, st, (const float*)h, n, D, exit_layer, n_layers, start, cursor,
                                                   sorted_tok, (float*)xs, mode, eps);
 }
 
 void launch_fold_rows(cudaStream_t st, int dt, void* dst, int ld_dst, const void* src, int n_rows, int K,
                       const float* gamma, const float* beta, const float* bias_in, float* bias_out, int row_mode) {
   if (dt == 1)
-    fold_rows_kernel<bf16><<<cdiv(n_rows, 8), 256, 0, st>>>((bf16*)dst, ld_dst, (const bf16*)src, n_rows, K, gamma,
+    launch_k(fold_rows_kernel<bf16>, cdiv(n_rows, 8), 256, 0, st, (bf16*)dst, ld_dst, (const bf16*)src, n_rows, K, gamma,
                                                             beta, bias_in, bias_out, row_mode);
   else
-    fold_rows_kernel<float><<<cdiv(n_rows, 8), 256, 0, st>>>((float*)dst, ld_dst, (const float*)src, n_rows, K,
+    launch_k(fold_rows_kernel<float>, cdiv(n_rows, 8), 256, 0, st, (float*)dst, ld_dst, (const float*)src, n_rows, K,
                                                              gamma, beta, bias_in, bias_out, row_mode);
 }
 
 void launch_to_f32(cudaStream_t st, int dt, const void* src, float* dst, int n) {
   if (n <= 0) return;
-  if (dt == 1) to_f32_kernel<bf16><<<cdiv(n, 256), 256, 0, st>>>((const bf16*)src, dst, n);
-  else to_f32_kernel<float><<<cdiv(n, 256), 256, 0, st>>>((const float*)src, dst, n);
+  if (dt == 1) launch_k(to_f32_kernel<bf16>, cdiv(n, 256), 256, 0, st, (const bf16*)src, dst, n);
+  else launch_k(to_f32_kernel<float>, cdiv(n, 256), 256, 0, st, (const float*)src, dst, n);
 }
 
 void launch_read_kv(cudaStream_t st, int dt, KVCacheView c, int layer0, int seq, int pos0, int n_pos, void* ko,
                     void* vo) {
   if (n_pos <= 0) return;
-  if (dt == 1) read_kv_kernel<bf16><<<n_pos, 256, 0, st>>>(c, layer0, seq, pos0, n_pos, (bf16*)ko, (bf16*)vo);
-  else read_kv_kernel<float><<<n_pos, 256, 0, st>>>(c, layer0, seq, pos0, n_pos, (float*)ko, (float*)vo);
+  if (dt == 1) launch_k(read_kv_kernel<bf16>, n_pos, 256, 0, st, c, layer0, seq, pos0, n_pos, (bf16*)ko, (bf16*)vo);
+  else launch_k(read_kv_kernel<float>, n_pos, 256, 0, st, c, layer0, seq, pos0, n_pos, (float*)ko, (float*)vo);
 }
 
 }  // namespace adept

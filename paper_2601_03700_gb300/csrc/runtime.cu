@@ -21,6 +21,10 @@
 
 using namespace adept;
 
+namespace adept {
+thread_local bool g_pdl = false;
+}
+
 namespace {
 thread_local std::string g_load_error;
 }
@@ -659,7 +663,6 @@ static adept_status reserve_seqs(adept_model* m, int batch, const int* lens, cud
 // ---------------------------------------------------------------------------
 // the early-exit pass
 // ---------------------------------------------------------------------------
-__global__ void set_int_kernel(int* p, int v) { *p = v; }
 
 static void run_hsm(adept_model* m, cudaStream_t st, DevRange rows, int max_rows, int a_rows) {
   const int D = m->D, m1 = m->m1, m2 = m->m2;
@@ -731,15 +734,12 @@ static adept_status run_pass(adept_model* m, int n_tok, int batch, int prompt_le
   const int amode = attn_norm_mode(m);
   const float eps = c.norm_eps;
   m->last_rows = n_tok;
-  if (sim_out) CUDA_TRY(m, cudaMemsetAsync(sim_out, 0xff, (size_t)n_tok * N * sizeof(float), st));  // NaN
-  CUDA_TRY(m, cudaMemsetAsync(m->ctr, 0, ctr_words(N) * sizeof(int), st));
-  set_int_kernel<<<1, 1, 0, st>>>(m->ctr + CTR_ACTIVE, n_tok);
   launch_pass_init(st, n_tok, prompt_len, decode ? 1 : 0, m->tok_seq, m->tok_pos, m->row_tok[0], m->d_seq_len,
                    m->max_blocks_per_seq * c.kv_block_tokens, fam == ADEPT_FAMILY_LLAMA ? 0 : c.max_pos,
-                   m->err_word);
+                   m->err_word, m->ctr, ctr_words(N), sim_out, N);
   launch_embed(st, m->dt, tokens, n_tok, m->tok_pos, m->tok_emb, m->pos_emb, m->type_emb, m->emb_g, m->emb_b, fam, D,
                m->V, eps, m->X_in[0], m->err_word);
-  m->launches += 3;
+  m->launches += 2;
   const KVCacheView cv = cache_view(m);
   const int causal = fam != ADEPT_FAMILY_BERT;
   // generation step: the split-KV attention grid covers the reserved capacity (CTAs past a
@@ -1028,6 +1028,7 @@ adept_status adept_prefill(adept_model* m, int batch, int prompt_len, const int3
                            const int32_t* d_forced_exit, int32_t* d_exit_layer_out, float* d_logits_out,
                            int32_t* d_next_token_out, float* d_sim_out, void* stream) {
   if (!m) return ADEPT_ERR_INVALID_ARG;
+  g_pdl = !m->profile;
   if (!d_tokens) return fail(m, ADEPT_ERR_INVALID_ARG, "d_tokens is NULL");
   if (batch < 1 || prompt_len < 1) return fail(m, ADEPT_ERR_INVALID_ARG, "batch and prompt_len must be positive");
   if (batch > m->cfg.max_batch) return fail(m, ADEPT_ERR_CAPACITY, "batch %d > max_batch %d", batch, m->cfg.max_batch);
@@ -1052,6 +1053,7 @@ adept_status adept_decode_step(adept_model* m, int batch, const int32_t* d_token
                                const int32_t* d_forced_exit, int32_t* d_exit_layer_out, float* d_logits_out,
                                int32_t* d_next_token_out, float* d_sim_out, void* stream) {
   if (!m) return ADEPT_ERR_INVALID_ARG;
+  g_pdl = !m->profile;
   if (m->cfg.family == ADEPT_FAMILY_BERT) return fail(m, ADEPT_ERR_INVALID_ARG, "decode needs a decoder model");
   if (!d_tokens) return fail(m, ADEPT_ERR_INVALID_ARG, "d_tokens is NULL");
   if (batch < 1 || batch > m->cfg.max_batch) return fail(m, ADEPT_ERR_CAPACITY, "batch %d out of range", batch);
@@ -1139,6 +1141,7 @@ adept_status adept_decode_step(adept_model* m, int batch, const int32_t* d_token
 adept_status adept_skip_kv_fill(adept_model* m, int n_tokens, const void* d_h_mapped, const int32_t* d_exit_layer,
                                 const int32_t* d_seq, const int32_t* d_pos, void* stream) {
   if (!m) return ADEPT_ERR_INVALID_ARG;
+  g_pdl = !m->profile;
   if (n_tokens < 0) return fail(m, ADEPT_ERR_INVALID_ARG, "n_tokens < 0");
   if (n_tokens == 0) return ADEPT_OK;
   if (n_tokens > (1 << 20)) return fail(m, ADEPT_ERR_CAPACITY, "n_tokens %d above 1<<20", n_tokens);
