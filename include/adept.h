@@ -212,14 +212,16 @@ ADEPT_API adept_status adept_check_device_status(adept_model* m, void* stream);
  * (generation steps then run as direct launches).  GEMM_SIMT=1 routes GEMMs to the
  * SIMT kernels (cross-check).  DECODE_GRAPH (default 1): from its second call with a
  * given batch size, adept_decode_step replays a CUDA graph of the step captured once;
- * 0 launches every kernel directly.  SKINNY_GEMM (default 0): GEMMs of at most 32 rows
- * use the split-K skinny kernel instead of the tcgen05 kernel.  FUSED_DECODE: 1 runs a
+ * 0 launches every kernel directly.  DECODE_GEMM (default 1): single GEMMs of at most 16
+ * rows (generation steps, output heads) of bf16 models run on the weight-streaming
+ * generation-step kernel, with the input standardisation fused in; 0 routes them to the
+ * tcgen05 kernel after a separate standardisation launch.  FUSED_DECODE: 1 runs a
  * generation step of at most adept_fused_decode_batch() sequences of a bf16 decoder as
  * one persistent cooperative launch (every layer, the HSM, the fills and the head),
  * reading the caller's inputs and writing its outputs directly; 0 takes the multi-launch
  * step.  Default 0. */
 enum { ADEPT_OPT_HSM_IDENTITY = 1, ADEPT_OPT_PROFILE = 2, ADEPT_OPT_GEMM_SIMT = 3, ADEPT_OPT_DECODE_GRAPH = 4,
-       ADEPT_OPT_SKINNY_GEMM = 5, ADEPT_OPT_FUSED_DECODE = 6 };
+       ADEPT_OPT_DECODE_GEMM = 5, ADEPT_OPT_FUSED_DECODE = 6 };
 ADEPT_API adept_status adept_set_option(adept_model* m, int option, int value);
 
 /* Kernel classes reported by adept_profile_read: the GEMMs of prompt passes (layer

@@ -2,6 +2,7 @@
 // of a sequence at layer i are every cached position of that layer -- computed by the
 // token itself if it was active at i, or filled from its mapped state s~_N if it
 // exited earlier -- so attention needs no knowledge of exits.
+#define ADEPT_TU_ID 1
 #include "common.cuh"
 #include "kernels.h"
 
@@ -452,14 +453,257 @@ static void attn_dispatch(cudaStream_t st, const void* q, int ld_q, void* out, i
 #undef ATT_CASE
 }
 
+// ---------------------------------------------------------------------------
+// Generation-step attention (bf16): one query row per sequence, keys split into chunks of
+// AD_CHUNK.  A CTA = (row, kv head, chunk): its K and V cache blocks (16 positions x
+// head_dim, contiguous in the paged pool) are bulk-copied into shared memory on one
+// mbarrier; per query head of the group the chunk's exact softmax partial (max m, sum l,
+// sum p V) is formed in two passes over shared memory.  The last CTA of a (row, head) to
+// finish (arrival counter) merges the chunk partials in chunk order and writes the output,
+// then clears its counter for the next launch.
+// ---------------------------------------------------------------------------
+constexpr int AD_CHUNK = 128;
+constexpr int AD_THREADS = 128;
+constexpr long long AD_TIMEOUT_CYCLES = 4000000000LL;   // ~2 s at 2 GHz
+
+__device__ __forceinline__ uint32_t ad_smem_u32(const void* p) { return (uint32_t)__cvta_generic_to_shared(p); }
+__device__ __forceinline__ bool ad_try_wait(uint64_t* bar, uint32_t parity) {
+  uint32_t ok;
+  asm volatile(
+      "{\n.reg .pred p;\nmbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\nselp.u32 %0, 1, 0, p;\n}\n"
+      : "=r"(ok)
+      : "r"(ad_smem_u32(bar)), "r"(parity)
+      : "memory");
+  return ok != 0;
+}
+__device__ __forceinline__ bool ad_wait(uint64_t* bar, unsigned* err) {
+  if (ad_try_wait(bar, 0)) return true;
+  const long long t0 = clock64();
+  while (!ad_try_wait(bar, 0)) {
+    if (clock64() - t0 > AD_TIMEOUT_CYCLES) {
+      atomicOr(err, ERRW_TIMEOUT);
+      return false;
+    }
+  }
+  return true;
+}
+
+template <int DH>
+__global__ void __launch_bounds__(AD_THREADS)
+    attn_decode_kernel(const bf16* __restrict__ q, int ld_q, DevRange rows, const int* row_tok, const int* tok_seq,
+                       const int* tok_pos, const int* seq_len, KVCacheView cache, int layer0, int n_heads, int causal,
+                       float scale_log2, int n_split, float* __restrict__ ws, int* counters, bf16* __restrict__ out,
+                       int ld_out, unsigned* err) {
+  PDL_ENTRY();
+  constexpr int PARTS = DH / 8;          // 16-byte pieces of a K / V row
+  constexpr int KPI = 32 / PARTS;        // keys per warp instruction
+  extern __shared__ __align__(128) uint8_t ad_smem[];
+  bf16* sK = reinterpret_cast<bf16*>(ad_smem);   // [AD_CHUNK][DH]
+  bf16* sV = sK + AD_CHUNK * DH;                  // [AD_CHUNK][DH]
+  __shared__ __align__(8) uint64_t bar;
+  __shared__ float s_p[AD_CHUNK];
+  __shared__ float s_red[AD_THREADS / 32];
+  __shared__ float s_o[AD_THREADS / 32][DH];
+  __shared__ int s_last;
+
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const int Hkv = cache.n_kv_heads, group = n_heads / Hkv;
+  const int rk = blockIdx.x, split = blockIdx.y;
+  const int rrel = rk / Hkv, kvh = rk - rrel * Hkv;
+  const int r = rows.b() + rrel;
+  if (r >= rows.e()) return;
+  const int tok = row_tok[r];
+  const int sq = tok_seq[tok], pos = tok_pos[tok];
+  const int nk = causal ? pos + 1 : seq_len[sq];
+  const int n_eff = (nk + AD_CHUNK - 1) / AD_CHUNK;   // chunks holding keys of this row
+  if (split >= n_eff) return;
+  const int k_lo = split * AD_CHUNK, nkc = min(nk - k_lo, AD_CHUNK);
+  const int nb = (nkc + 15) >> 4;                      // cache blocks of the chunk
+  constexpr int BLOCK_BYTES = 16 * DH * 2;
+
+  if (tid == 0) {
+    asm volatile("mbarrier.init.shared::cta.b64 [%0], 1;" ::"r"(ad_smem_u32(&bar)) : "memory");
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+  }
+  __syncthreads();
+  if (warp == 0) {
+    if (lane == 0)
+      asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(ad_smem_u32(&bar)),
+                   "r"((uint32_t)(2 * nb * BLOCK_BYTES))
+                   : "memory");
+    __syncwarp();
+    if (lane < nb) {
+      const int bi = (k_lo >> 4) + lane;
+      int blk = (sq >= 0 && sq < cache.max_batch && bi < cache.max_blocks_per_seq)
+                    ? cache.block_table[sq * cache.max_blocks_per_seq + bi]
+                    : -1;
+      if (blk < 0 || blk >= cache.n_blocks) {   // no reserved block: flag, copy block 0 (results unused)
+        atomicOr(err, ERRW_POS);
+        blk = 0;
+      }
+      const size_t off = (((size_t)layer0 * cache.n_blocks + blk) * Hkv + kvh) * (size_t)(16 * DH);
+      asm volatile("cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(
+                       ad_smem_u32(sK + lane * 16 * DH)),
+                   "l"((const bf16*)cache.k + off), "r"((uint32_t)BLOCK_BYTES), "r"(ad_smem_u32(&bar))
+                   : "memory");
+      asm volatile("cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(
+                       ad_smem_u32(sV + lane * 16 * DH)),
+                   "l"((const bf16*)cache.v + off), "r"((uint32_t)BLOCK_BYTES), "r"(ad_smem_u32(&bar))
+                   : "memory");
+    }
+  }
+  const int slot = lane / PARTS, part = lane - slot * PARTS;
+  bool ok = ad_wait(&bar, err);
+  if (!ok) ad_wait(&bar, err);   // second bounded wait for the copies in flight; results flagged
+
+  for (int g = 0; g < group; ++g) {
+    const int h = kvh * group + g;
+    // query piece of this lane (8 dims), scaled into the log2 domain
+    float qv[8];
+    {
+      const uint4 u = *reinterpret_cast<const uint4*>(q + (size_t)r * ld_q + h * DH + part * 8);
+      const __nv_bfloat162* b = reinterpret_cast<const __nv_bfloat162*>(&u);
+#pragma unroll
+      for (int i = 0; i < 4; ++i) {
+        const float2 f = __bfloat1622float2(b[i]);
+        qv[2 * i] = f.x * scale_log2;
+        qv[2 * i + 1] = f.y * scale_log2;
+      }
+    }
+    // pass 1: scores of the chunk's keys
+    for (int k0 = warp * KPI; k0 < AD_CHUNK; k0 += 4 * KPI) {
+      const int key = k0 + slot;
+      float d = 0.f;
+      if (key < nkc) {
+        const uint4 u = *reinterpret_cast<const uint4*>(sK + key * DH + part * 8);
+        const __nv_bfloat162* b = reinterpret_cast<const __nv_bfloat162*>(&u);
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+          const float2 f = __bfloat1622float2(b[i]);
+          d = fmaf(qv[2 * i], f.x, d);
+          d = fmaf(qv[2 * i + 1], f.y, d);
+        }
+      }
+#pragma unroll
+      for (int o = PARTS >> 1; o; o >>= 1) d += __shfl_xor_sync(0xffffffffu, d, o);
+      if (part == 0 && key < AD_CHUNK) s_p[key] = key < nkc ? d : -INFINITY;
+    }
+    __syncthreads();
+    // chunk max, probabilities, chunk sum
+    float mx = -INFINITY;
+    for (int k = tid; k < AD_CHUNK; k += AD_THREADS) mx = fmaxf(mx, s_p[k]);
+    mx = warp_max(mx);
+    if (lane == 0) s_red[warp] = mx;
+    __syncthreads();
+    const float M = fmaxf(fmaxf(s_red[0], s_red[1]), fmaxf(s_red[2], s_red[3]));
+    float ls = 0.f;
+    for (int k = tid; k < AD_CHUNK; k += AD_THREADS) {
+      const float pk = k < nkc ? exp2f(s_p[k] - M) : 0.f;
+      s_p[k] = pk;
+      ls += pk;
+    }
+    ls = warp_sum(ls);
+    __syncthreads();   // every s_red[] read and s_p[] write done
+    if (lane == 0) s_red[warp] = ls;
+    // pass 2: sum p V, lane = (key slot, 8 dims)
+    float o[8];
+#pragma unroll
+    for (int i = 0; i < 8; ++i) o[i] = 0.f;
+    for (int k0 = warp * KPI; k0 < nkc; k0 += 4 * KPI) {
+      const int key = k0 + slot;
+      if (key < nkc) {
+        const float pk = s_p[key];
+        const uint4 u = *reinterpret_cast<const uint4*>(sV + key * DH + part * 8);
+        const __nv_bfloat162* b = reinterpret_cast<const __nv_bfloat162*>(&u);
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+          const float2 f = __bfloat1622float2(b[i]);
+          o[2 * i] = fmaf(pk, f.x, o[2 * i]);
+          o[2 * i + 1] = fmaf(pk, f.y, o[2 * i + 1]);
+        }
+      }
+    }
+#pragma unroll
+    for (int i = 0; i < 8; ++i)
+      for (int sft = PARTS; sft < 32; sft <<= 1) o[i] += __shfl_xor_sync(0xffffffffu, o[i], sft);
+    if (slot == 0) {
+#pragma unroll
+      for (int i = 0; i < 8; ++i) s_o[warp][part * 8 + i] = o[i];
+    }
+    __syncthreads();
+    // chunk partial -> workspace [(row, head), split]: o[DH], m, l
+    const int rh = rrel * n_heads + h;
+    float* w = ws + ((size_t)rh * n_split + split) * (DH + 2);
+    for (int d = tid; d < DH; d += AD_THREADS) w[d] = s_o[0][d] + s_o[1][d] + s_o[2][d] + s_o[3][d];
+    if (tid == 0) {
+      w[DH] = M;
+      w[DH + 1] = s_red[0] + s_red[1] + s_red[2] + s_red[3];
+    }
+    __threadfence();
+    __syncthreads();
+    if (tid == 0) s_last = atomicAdd(&counters[rh], 1) == n_eff - 1;
+    __syncthreads();
+    if (s_last) {
+      // last chunk of (row, head) to finish: merge the chunk partials in chunk order
+      __threadfence();
+      const float* wb = ws + (size_t)rh * n_split * (DH + 2);
+      float Mg = -INFINITY;
+      for (int c = 0; c < n_eff; ++c) Mg = fmaxf(Mg, __ldcg(wb + (size_t)c * (DH + 2) + DH));
+      float L = 0.f;
+      for (int c = 0; c < n_eff; ++c) {
+        const float* wc = wb + (size_t)c * (DH + 2);
+        L += exp2f(__ldcg(wc + DH) - Mg) * __ldcg(wc + DH + 1);
+      }
+      const float inv = L > 0.f ? 1.f / L : 0.f;
+      for (int d = tid; d < DH; d += AD_THREADS) {
+        float acc = 0.f;
+        for (int c = 0; c < n_eff; ++c) {
+          const float* wc = wb + (size_t)c * (DH + 2);
+          acc += exp2f(__ldcg(wc + DH) - Mg) * __ldcg(wc + d);
+        }
+        out[(size_t)r * ld_out + h * DH + d] = __float2bfloat16_rn(acc * inv);
+      }
+      if (tid == 0) counters[rh] = 0;
+    }
+    __syncthreads();   // s_p / s_o / s_red reused by the next head of the group
+  }
+}
+
 static int g_attn_smem_set[2] = {0, 0};
+static int g_ad_smem_set[2] = {0, 0};
 
 void launch_attention(cudaStream_t st, int dt, const void* q, int ld_q, void* out, int ld_out, DevRange rows,
                       int max_rows, const int* row_tok, const int* tok_seq, const int* tok_pos, const int* seq_len,
-                      KVCacheView cache, int layer0, int n_heads, int causal, int decode_keys, float* ws) {
+                      KVCacheView cache, int layer0, int n_heads, int causal, int decode_keys, float* ws,
+                      int* counters, unsigned* err) {
   if (max_rows <= 0) return;
   const int dh = cache.head_dim;
   const float scale_log2 = 1.4426950408889634f / sqrtf((float)dh);
+  if (decode_keys > 0 && ws && counters && dt == 1 && (dh == 64 || dh == 128) && cache.block_tokens == 16 &&
+      (decode_keys + AD_CHUNK - 1) / AD_CHUNK <= ATTN_MAX_SPLIT && n_heads % cache.n_kv_heads == 0 &&
+      ld_q % 8 == 0 && ((uintptr_t)q & 15) == 0) {
+    const int n_split = (decode_keys + AD_CHUNK - 1) / AD_CHUNK;
+    const dim3 grid(max_rows * cache.n_kv_heads, n_split);
+    const int smem = 2 * AD_CHUNK * dh * 2;
+    if (dh == 64) {
+      if (!g_ad_smem_set[0]) {
+        cudaFuncSetAttribute(attn_decode_kernel<64>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+        g_ad_smem_set[0] = 1;
+      }
+      launch_k(attn_decode_kernel<64>, grid, AD_THREADS, smem, st, (const bf16*)q, ld_q, rows, row_tok, tok_seq,
+               tok_pos, seq_len, cache, layer0, n_heads, causal, scale_log2, n_split, ws, counters, (bf16*)out, ld_out,
+               err);
+    } else {
+      if (!g_ad_smem_set[1]) {
+        cudaFuncSetAttribute(attn_decode_kernel<128>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+        g_ad_smem_set[1] = 1;
+      }
+      launch_k(attn_decode_kernel<128>, grid, AD_THREADS, smem, st, (const bf16*)q, ld_q, rows, row_tok, tok_seq,
+               tok_pos, seq_len, cache, layer0, n_heads, causal, scale_log2, n_split, ws, counters, (bf16*)out, ld_out,
+               err);
+    }
+    return;
+  }
   if (decode_keys > 0 && ws && (dh == 64 || dh == 128)) {
     // generation step: split the keys so that rows x heads x splits covers the GPU twice
     int n_split = (2 * 152 + max_rows * n_heads - 1) / (max_rows * n_heads);
@@ -513,5 +757,7 @@ void launch_attention(cudaStream_t st, int dt, const void* q, int ld_q, void* ou
     attn_dispatch<float>(st, q, ld_q, out, ld_out, rows, max_rows, row_tok, tok_seq, tok_pos, seq_len, cache, layer0,
                          n_heads, causal);
 }
+
+ADEPT_KTRACE_ATTACH(attention)
 
 }  // namespace adept

@@ -25,11 +25,91 @@ enum : unsigned {
 // before the wait may touch nothing a preceding kernel writes.
 __device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
 __device__ __forceinline__ void pdl_launch_dependents() { asm volatile("griddepcontrol.launch_dependents;" ::: "memory"); }
-#define PDL_ENTRY()            \
-  do {                         \
-    pdl_wait();                \
-    pdl_launch_dependents();   \
+
+// Debug-only launch timeline (built with -DADEPT_KTRACE): thread 0 of every CTA records
+// its global-timer stamps at entry, after the dependency wait and at exit, with a kernel
+// id (translation unit x 100000 + source line of the entry macro).  Each translation unit
+// holds its own pointer to the host-allocated record buffer (set by kt_attach_<unit>).
+#ifdef ADEPT_KTRACE
+constexpr int KT_MARKS = 8;
+struct KtRec {
+  unsigned long long t0, t1, t2;
+  unsigned long long mk[KT_MARKS];   // optional intermediate stamps (0: not reached)
+  unsigned kid, cta, grid, pad;
+};
+static __device__ KtRec* g_kt_buf = nullptr;
+static __device__ unsigned* g_kt_cnt = nullptr;
+static __device__ unsigned g_kt_cap = 0;
+__device__ __forceinline__ unsigned long long kt_now() {
+  unsigned long long t;
+  asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
+  return t;
+}
+struct KtScope {
+  unsigned long long t0, t1;
+  unsigned long long mk[KT_MARKS];
+  unsigned kid;
+  __device__ explicit KtScope(unsigned k) : t0(kt_now()), t1(0), kid(k) {
+#pragma unroll
+    for (int i = 0; i < KT_MARKS; ++i) mk[i] = 0;
+  }
+  __device__ void waited() { t1 = kt_now(); }
+  __device__ void mark(int i) { mk[i] = kt_now(); }
+  __device__ void add(int i, unsigned long long v) { mk[i] += v; }
+  __device__ ~KtScope() {
+    if (threadIdx.x == 0 && threadIdx.y == 0 && g_kt_buf) {
+      const unsigned i = atomicAdd(g_kt_cnt, 1u);
+      if (i < g_kt_cap) {
+        KtRec r;
+        r.t0 = t0;
+        r.t1 = t1;
+        r.t2 = kt_now();
+#pragma unroll
+        for (int j = 0; j < KT_MARKS; ++j) r.mk[j] = mk[j];
+        r.kid = kid;
+        r.cta = blockIdx.x + blockIdx.y * gridDim.x;
+        r.grid = gridDim.x * gridDim.y;
+        r.pad = 0;
+        g_kt_buf[i] = r;
+      }
+    }
+  }
+};
+#ifndef ADEPT_TU_ID
+#define ADEPT_TU_ID 0
+#endif
+#define KT_BEGIN() KtScope kt_scope_(ADEPT_TU_ID * 100000u + __LINE__)
+#define KT_WAITED() kt_scope_.waited()
+#define KT_MARK(i) kt_scope_.mark(i)
+#define KT_ADD(i, v) kt_scope_.add(i, v)
+#define ADEPT_KTRACE_ATTACH(unit)                                                          \
+  void kt_attach_##unit(void* buf, unsigned* cnt, unsigned cap) {                          \
+    KtRec* b = (KtRec*)buf;                                                                \
+    cudaMemcpyToSymbol(g_kt_buf, &b, sizeof b);                                            \
+    cudaMemcpyToSymbol(g_kt_cnt, &cnt, sizeof cnt);                                        \
+    cudaMemcpyToSymbol(g_kt_cap, &cap, sizeof cap);                                        \
+  }
+#else
+#define KT_BEGIN() \
+  do {             \
   } while (0)
+#define KT_WAITED() \
+  do {              \
+  } while (0)
+#define KT_MARK(i) \
+  do {             \
+  } while (0)
+#define KT_ADD(i, v) \
+  do {               \
+  } while (0)
+#define ADEPT_KTRACE_ATTACH(unit)
+#endif
+
+#define PDL_ENTRY()          \
+  KT_BEGIN();                \
+  pdl_wait();                \
+  KT_WAITED();               \
+  pdl_launch_dependents()
 
 namespace adept {
 // Launches with the programmatic-serialisation attribute while g_pdl is set (each entry

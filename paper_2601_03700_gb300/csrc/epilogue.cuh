@@ -1,6 +1,6 @@
 // GEMM epilogues applied to 32 consecutive output columns of one row.  Shared by the
-// tcgen05 GEMM (a thread owns one accumulator row in tensor memory), the skinny GEMM
-// and the SIMT GEMM, so every path has one definition of each fused epilogue.
+// tcgen05 GEMM (a thread owns one accumulator row in tensor memory), the generation-step
+// GEMM and the SIMT GEMM, so every path has one definition of each fused epilogue.
 //
 // Column layouts the epilogues rely on (fixed by the load-time repacking):
 //  * RoPE families: inside each Q / K head the weight rows are interleaved so that
@@ -78,12 +78,16 @@ __device__ __forceinline__ void rope_pairs(T* dst, int i0, int half, const float
 
 // bias32 / resid32 (optional): the chunk's 32 bias values and the row's 32 residual
 // values already staged by the caller (e.g. in shared memory) instead of e.bias[c0..] and
-// e.resid[ra][c0..].
-template <typename T>
+// e.resid[ra][c0..].  applied: the caller has already added the bias and applied the
+// EPI_ACT activation to v.  KIND >= 0 fixes the epilogue kind at compile time (only its
+// code is generated); -1 switches on e.kind.
+template <typename T, int KIND = -1>
 __device__ __forceinline__ void epi_chunk32(const Epi& e, int ra, int c0, int N, float (&v)[32], const EpiRow& rr,
-                                            const float* bias32 = nullptr, const float* resid32 = nullptr) {
+                                            const float* bias32 = nullptr, const float* resid32 = nullptr,
+                                            bool applied = false) {
   const bool full = c0 + 32 <= N;
-  if (bias32) {
+  if (applied) {
+  } else if (bias32) {
 #pragma unroll
     for (int j = 0; j < 32; ++j)
       if (full || c0 + j < N) v[j] += bias32[j];
@@ -92,7 +96,7 @@ __device__ __forceinline__ void epi_chunk32(const Epi& e, int ra, int c0, int N,
     for (int j = 0; j < 32; ++j)
       if (full || c0 + j < N) v[j] += e.bias[c0 + j];
   }
-  switch (e.kind) {
+  switch (KIND >= 0 ? KIND : e.kind) {
     case EPI_F32: {
       float* o = e.out_f32 + (size_t)ra * e.ld_f32 + c0;
       if (full && ((e.ld_f32 & 15) == 0)) {
@@ -105,8 +109,10 @@ __device__ __forceinline__ void epi_chunk32(const Epi& e, int ra, int c0, int N,
       return;
     }
     case EPI_ACT: {
+      if (!applied) {
 #pragma unroll
-      for (int j = 0; j < 32; ++j) v[j] = apply_act(e.act, v[j]);
+        for (int j = 0; j < 32; ++j) v[j] = apply_act(e.act, v[j]);
+      }
       T* o = (T*)e.out_t + (size_t)ra * e.ld_t + c0;
       if (full && ((e.ld_t & 15) == 0)) {
         store16<T>(o, v);

@@ -1,0 +1,29 @@
+// Generation-step GEMM (gemm_decode.cu): C[M, N] = A[M, K] * W[N, K]^T for passes of at
+// most DG_MAX_M token rows, shaped as a stream over the weights.
+#pragma once
+#include "common.cuh"
+
+namespace adept {
+
+constexpr int DG_MAX_M = 16;
+
+// Optional fused standardisation of the A operand: row r of A is the standardised row
+// in_rows[r] (or r) of the fp32 matrix X (row length K), as the standardisation kernel
+// computes it (LayerNorm without gain / RMS / copy; gains are folded into W at load).
+struct DgNorm {
+  const float* X;
+  int ldx;
+  const int* in_rows;
+  int mode;     // NormMode
+  float eps;
+};
+
+// Enqueues one problem (bf16 operands, fused epilogue).  norm == NULL: A is bf16 at
+// p.A.  Returns the number of launches (1), or -1 when the shape is not taken (the caller
+// runs another path): max_rows > DG_MAX_M, K not a multiple of 64, K above 16384,
+// unaligned operands.
+int decode_gemm(cudaStream_t st, const GemmProblem& p, int max_rows, const DgNorm* norm, unsigned* err);
+// Whether decode_gemm takes the problem (host-side shape and alignment checks only).
+bool decode_gemm_supported(const GemmProblem& p, int max_rows, const DgNorm* norm);
+
+}  // namespace adept

@@ -1,6 +1,7 @@
 // SIMT GEMM (fp32 FMA) with a separate epilogue pass.  This is the path of the fp32
 // models and the cross-check of the tensor-core GEMM; its epilogue semantics are the
 // reference for the fused tcgen05 epilogue.
+#define ADEPT_TU_ID 2
 #include "common.cuh"
 #include "kernels.h"
 #include "epilogue.cuh"
@@ -85,5 +86,7 @@ void launch_gemm_simt(cudaStream_t st, int dt, const GemmProblem& p, int max_row
     launch_k(epilogue_kernel<float>, max_rows, 64, 0, st, p.epi, scratch, p.N, p.rows, p.N);
   }
 }
+
+ADEPT_KTRACE_ATTACH(simt)
 
 }  // namespace adept

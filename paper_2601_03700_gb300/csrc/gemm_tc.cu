@@ -9,6 +9,7 @@
 // accumulator buffers in tensor memory so the epilogue of tile t overlaps the
 // main loop of tile t+1.  Every mbarrier wait is bounded: on time-out the CTA sets
 // ERRW_TIMEOUT in the device error word, stops, drains its MMAs and frees TMEM.
+#define ADEPT_TU_ID 4
 #include "gemm_tc.h"
 #include "epilogue.cuh"
 
@@ -184,6 +185,7 @@ __device__ unsigned g_tc_launch;
 // that are never stored), so the A region is one 128-row tile plus (KC-1) short tiles.
 template <int BN, int STAGES, int MAXG, int KC>
 __global__ void __launch_bounds__(TC_THREADS, 1) gemm_tc_kernel(const __grid_constant__ TcParams<MAXG> p) {
+  KT_BEGIN();
   constexpr int A_BYTES = TC_BM * TC_BK * 2 + (KC - 1) * TC_SHORT_ROWS * TC_BK * 2;
   constexpr int B_BYTES = KC * BN * TC_BK * 2;
   constexpr uint32_t TMEM_COLS = 2 * BN;
@@ -240,6 +242,7 @@ __global__ void __launch_bounds__(TC_THREADS, 1) gemm_tc_kernel(const __grid_con
     tmem_relinquish();
   }
   pdl_wait();
+  KT_WAITED();
   if (threadIdx.x == 0) {
     int acc = 0;
     for (int g = 0; g < ng; ++g) {
@@ -710,6 +713,8 @@ int tc_gemm_grouped_nocache(cudaStream_t st, const GemmProblem* probs, int n_pro
     default: return launch_bn<32, 10, TC_MAXG>(st, prm, grid);
   }
 }
+
+ADEPT_KTRACE_ATTACH(tc)
 
 }  // namespace adept
 

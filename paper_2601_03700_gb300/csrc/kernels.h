@@ -27,12 +27,14 @@ void launch_layernorm_inplace(cudaStream_t st, float* X, DevRange rows, int max_
 void launch_exit_decide(cudaStream_t st, const float* Xout, const float* I, int D, DevRange rows, int max_rows,
                         const int* row_tok, const int* forced, int layer, int n_layers, const float* delta_p, int test,
                         float* sim, int* flag, float* inv_norm, unsigned* err);
-// Test + compaction + moves in one CTA for passes of at most EXIT_SMALL_MAX rows.
+// Test + compaction + moves in one CTA for passes of at most EXIT_SMALL_MAX rows
+// (max_rows: the pass's row bound; at most 16 rows take a register-resident kernel).
 constexpr int EXIT_SMALL_MAX = 256;
 void launch_exit_small(cudaStream_t st, const float* Xin, const float* Xout, const float* I, int first, int D,
                        int* ctr, int par, const int* row_tok, int* row_tok_next, const int* forced, int layer,
                        int n_layers, const float* delta_p, int test, float* sim, int* exit_tok, int* exit_layer_out,
-                       float* Xnext, float* Inext, float* hsm_s, float* hsm_prev, float* hsm_I, unsigned* err);
+                       float* Xnext, float* Inext, float* hsm_s, float* hsm_prev, float* hsm_I, int max_rows,
+                       unsigned* err);
 void launch_set_float(cudaStream_t st, float* p, float v);
 void launch_exit_scan(cudaStream_t st, int* ctr, int in_parity, const int* flag, const int* row_tok,
                       int* row_tok_next, int* exit_tok, int* dst, int* exit_layer_out, int layer);
@@ -64,10 +66,13 @@ void launch_read_kv(cudaStream_t st, int dt, KVCacheView c, int layer0, int seq,
 void launch_gemm_simt(cudaStream_t st, int dt, const GemmProblem& p, int max_rows, float* scratch);
 // Attention of the active query rows over the paged cache of one layer.
 // decode_keys > 0 (generation step, one query row per sequence): split-KV kernel over at
-// most decode_keys keys, using ws (>= rows * heads * ATTN_MAX_SPLIT * (head_dim + 2) floats).
+// most decode_keys keys, using ws (>= rows * heads * ATTN_MAX_SPLIT * (head_dim + 2) floats)
+// and, for bf16, counters (>= rows * heads ints, zero between launches; the kernel leaves
+// them zero).
 constexpr int ATTN_MAX_SPLIT = 32;
 void launch_attention(cudaStream_t st, int dt, const void* q, int ld_q, void* out, int ld_out, DevRange rows,
                       int max_rows, const int* row_tok, const int* tok_seq, const int* tok_pos, const int* seq_len,
-                      KVCacheView cache, int layer0, int n_heads, int causal, int decode_keys, float* ws);
+                      KVCacheView cache, int layer0, int n_heads, int causal, int decode_keys, float* ws,
+                      int* counters, unsigned* err);
 
 }  // namespace adept

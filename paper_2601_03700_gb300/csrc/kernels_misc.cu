@@ -1,6 +1,7 @@
 // Row-wise kernels of the early-exit pass: embedding, norms, the exit test with
 // active-token compaction, the HSM's non-GEMM steps, argmax, skipped-layer-fill
 // bucketing and load-time weight repacking.
+#define ADEPT_TU_ID 3
 #include "common.cuh"
 #include "kernels.h"
 
@@ -297,6 +298,7 @@ __global__ void __launch_bounds__(256) exit_small_kernel(const float* Xin, const
     }
   }
   __syncthreads();
+  KT_MARK(0);
   if (threadIdx.x == 0) {
     int e = 0, k = 0;
     for (int r = 0; r < n; ++r) {
@@ -317,6 +319,7 @@ __global__ void __launch_bounds__(256) exit_small_kernel(const float* Xin, const
     ctr[CTR_PREFIX + layer] = base + e;
   }
   __syncthreads();
+  KT_MARK(1);
   for (int r = warp; r < n; r += nw) {
     const int d0 = s_dst[r];
     const float* s = Xout + (size_t)r * D;
@@ -342,13 +345,155 @@ __global__ void __launch_bounds__(256) exit_small_kernel(const float* Xin, const
   }
 }
 
+// The same test, compaction and moves for a generation step of at most 16 rows, in one
+// pass over memory: each row's s_i, inertia and s_{i-1} are read once into registers (a
+// row per 512 >> rshift threads), the decision and compaction run on the reduced sums,
+// and the moves are written from the registers.
+constexpr int EXD_THREADS = 512;
+constexpr int EXD_V = 4;   // float4 per thread per row vector
+__global__ void __launch_bounds__(EXD_THREADS)
+    exit_decode_kernel(const float* __restrict__ Xin, const float* __restrict__ Xout, const float* __restrict__ I,
+                       int first, int D, int* ctr, int par, const int* row_tok, int* row_tok_next, const int* forced,
+                       int layer, int n_layers, const float* delta_p, int test, float* sim, int* exit_tok,
+                       int* exit_layer_out, float* __restrict__ Xnext, float* __restrict__ Inext,
+                       float* __restrict__ hsm_s, float* __restrict__ hsm_prev, float* __restrict__ hsm_I, int rshift,
+                       unsigned* err) {
+  PDL_ENTRY();
+  __shared__ float s_red[EXD_THREADS / 32][3];
+  __shared__ int s_dst[16], s_tok[16];
+  __shared__ float s_w[16];
+  const int tpr = EXD_THREADS >> rshift;   // threads per row
+  const int row = threadIdx.x >> (9 - rshift), sub = threadIdx.x & (tpr - 1);
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int n = min(ctr[CTR_ACTIVE + par], 1 << rshift);
+  const int D4 = D >> 2;
+  const bool live = row < n;
+  float4 xs[EXD_V], xi[EXD_V], xp[EXD_V];
+  float ns = 0.f, ni = 0.f, dot = 0.f;
+  if (live) {
+    const float4* s4 = reinterpret_cast<const float4*>(Xout + (size_t)row * D);
+    const float4* i4 = reinterpret_cast<const float4*>(I + (size_t)row * D);
+    const float4* p4 = reinterpret_cast<const float4*>(Xin + (size_t)row * D);
+#pragma unroll
+    for (int j = 0; j < EXD_V; ++j) {
+      const int v = sub + j * tpr;
+      if (v < D4) {
+        xs[j] = s4[v];
+        xi[j] = first ? make_float4(0.f, 0.f, 0.f, 0.f) : i4[v];
+        xp[j] = p4[v];
+      }
+    }
+#pragma unroll
+    for (int j = 0; j < EXD_V; ++j) {
+      if (sub + j * tpr < D4) {
+        const float4 a = xs[j], c = xi[j];
+        ns += a.x * a.x + a.y * a.y + a.z * a.z + a.w * a.w;
+        ni += c.x * c.x + c.y * c.y + c.z * c.z + c.w * c.w;
+        dot += a.x * c.x + a.y * c.y + a.z * c.z + a.w * c.w;
+      }
+    }
+  }
+  ns = warp_sum(ns);
+  ni = warp_sum(ni);
+  dot = warp_sum(dot);
+  if (lane == 0) {
+    s_red[warp][0] = ns;
+    s_red[warp][1] = ni;
+    s_red[warp][2] = dot;
+  }
+  __syncthreads();
+  if ((int)threadIdx.x < n) {   // thread r decides row r
+    const int r = threadIdx.x, wpr = tpr >> 5;
+    float a = 0.f, b = 0.f, c = 0.f;
+    for (int w = r * wpr; w < (r + 1) * wpr; ++w) {
+      a += s_red[w][0];
+      b += s_red[w][1];
+      c += s_red[w][2];
+    }
+    const int tok = row_tok[r];
+    int ex = 0;
+    if (test) {
+      const float cs = (a > 0.f && b > 0.f) ? c / sqrtf(a * b) : -INFINITY;
+      if (sim) sim[(size_t)tok * n_layers + (layer - 1)] = cs;
+      const int f = forced ? forced[tok] : 0;
+      if (f != 0 && (f < 2 || f > n_layers)) atomicOr(err, ERRW_FORCED);
+      ex = (f > 0) ? (f == layer) : (cs >= *delta_p);
+    }
+    s_dst[r] = ex;
+    s_tok[r] = tok;
+    s_w[r] = a > 0.f ? rsqrtf(a) : 0.f;
+  }
+  __syncthreads();
+  if (threadIdx.x == 0) {   // stable compaction (n <= 16)
+    const int base = ctr[CTR_EXITED];
+    int e = 0, k = 0;
+    for (int r = 0; r < n; ++r) {
+      const int tok = s_tok[r];
+      if (s_dst[r]) {
+        s_dst[r] = -1 - (base + e);
+        exit_tok[base + e] = tok;
+        if (exit_layer_out) exit_layer_out[tok] = layer;
+        ++e;
+      } else {
+        s_dst[r] = k;
+        row_tok_next[k] = tok;
+        ++k;
+      }
+    }
+    ctr[CTR_ACTIVE + (par ^ 1)] = k;
+    ctr[CTR_EXITED] = base + e;
+    ctr[CTR_PREFIX + layer] = base + e;
+  }
+  __syncthreads();
+  if (!live) return;
+  const int d0 = s_dst[row];
+  if (d0 >= 0) {
+    const float w = s_w[row];
+    float4* xn = reinterpret_cast<float4*>(Xnext + (size_t)d0 * D);
+    float4* inn = reinterpret_cast<float4*>(Inext + (size_t)d0 * D);
+#pragma unroll
+    for (int j = 0; j < EXD_V; ++j) {
+      const int v = sub + j * tpr;
+      if (v < D4) {
+        const float4 a = xs[j], c = xi[j];
+        xn[v] = a;
+        inn[v] = make_float4(c.x + a.x * w, c.y + a.y * w, c.z + a.z * w, c.w + a.w * w);
+      }
+    }
+  } else {
+    const size_t kk = (size_t)(-1 - d0);
+    float4* hs = reinterpret_cast<float4*>(hsm_s + kk * D);
+    float4* hp = reinterpret_cast<float4*>(hsm_prev + kk * D);
+    float4* hi = reinterpret_cast<float4*>(hsm_I + kk * D);
+#pragma unroll
+    for (int j = 0; j < EXD_V; ++j) {
+      const int v = sub + j * tpr;
+      if (v < D4) {
+        hs[v] = xs[j];
+        hp[v] = xp[j];
+        hi[v] = xi[j];
+      }
+    }
+  }
+}
+
 void launch_exit_small(cudaStream_t st, const float* Xin, const float* Xout, const float* I, int first, int D,
                        int* ctr, int par, const int* row_tok, int* row_tok_next, const int* forced, int layer,
                        int n_layers, const float* delta_p, int test, float* sim, int* exit_tok, int* exit_layer_out,
-                       float* Xnext, float* Inext, float* hsm_s, float* hsm_prev, float* hsm_I, unsigned* err) {
+                       float* Xnext, float* Inext, float* hsm_s, float* hsm_prev, float* hsm_I, int max_rows,
+                       unsigned* err) {
+  int rshift = 0;
+  while ((1 << rshift) < max_rows) ++rshift;
+  const bool aligned = ((uintptr_t)Xin | (uintptr_t)Xout | (uintptr_t)I | (uintptr_t)Xnext | (uintptr_t)Inext |
+                        (uintptr_t)hsm_s | (uintptr_t)hsm_prev | (uintptr_t)hsm_I) % 16 == 0;
+  if (max_rows <= 16 && D % 4 == 0 && D / 4 <= EXD_V * (EXD_THREADS >> rshift) && aligned) {
+    launch_k(exit_decode_kernel, 1, EXD_THREADS, 0, st, Xin, Xout, I, first, D, ctr, par, row_tok, row_tok_next, forced,
+             layer, n_layers, delta_p, test, sim, exit_tok, exit_layer_out, Xnext, Inext, hsm_s, hsm_prev, hsm_I,
+             rshift, err);
+    return;
+  }
   launch_k(exit_small_kernel, 1, 256, 0, st, Xin, Xout, I, first, D, ctr, par, row_tok, row_tok_next, forced, layer,
-                                       n_layers, delta_p, test, sim, exit_tok, exit_layer_out, Xnext, Inext, hsm_s,
-                                       hsm_prev, hsm_I, err);
+           n_layers, delta_p, test, sim, exit_tok, exit_layer_out, Xnext, Inext, hsm_s, hsm_prev, hsm_I, err);
 }
 
 __global__ void set_float_kernel(float* p, float v) {
@@ -840,5 +985,7 @@ void launch_read_kv(cudaStream_t st, int dt, KVCacheView c, int layer0, int seq,
   if (dt == 1) launch_k(read_kv_kernel<bf16>, n_pos, 256, 0, st, c, layer0, seq, pos0, n_pos, (bf16*)ko, (bf16*)vo);
   else launch_k(read_kv_kernel<float>, n_pos, 256, 0, st, c, layer0, seq, pos0, n_pos, (float*)ko, (float*)vo);
 }
+
+ADEPT_KTRACE_ATTACH(misc)
 
 }  // namespace adept

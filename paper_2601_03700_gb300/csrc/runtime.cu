@@ -5,7 +5,7 @@
 #include "common.cuh"
 #include "kernels.h"
 #include "gemm_tc.h"
-#include "gemm_skinny.h"
+#include "gemm_decode.h"
 #include "decode_fused.h"
 #include "model_view.h"
 
@@ -92,12 +92,9 @@ struct adept_model {
   void* pool_t = nullptr;
   float* logits_ws = nullptr;
   float* attn_ws = nullptr;
+  int* attn_ctr = nullptr;       // generation-step attention arrival counters (zero between launches)
   float* amax_v = nullptr;       // argmax partials
   int* amax_i = nullptr;
-  float* sk_ws = nullptr;        // skinny-GEMM partial tiles
-  size_t sk_ws_floats = 0;
-  int* sk_counters = nullptr;    // skinny-GEMM arrival counters (kept zero between launches)
-  int sk_n_counters = 0;
   float* scratch = nullptr;
   size_t scratch_elems = 0;
   // skipped-layer fill workspace (adept_skip_kv_fill)
@@ -112,7 +109,7 @@ struct adept_model {
   std::vector<cudaGraphExec_t> dec_graph;   // per batch size
   std::vector<int> dec_warm;                // direct runs done per batch size
   // options / instrumentation
-  int hsm_identity = 0, profile = 0, force_simt = 0, use_graph = 1, use_skinny = 0, use_fused = 1;
+  int hsm_identity = 0, profile = 0, force_simt = 0, use_graph = 1, use_dg = 1, use_fused = 1;
   // persistent generation-step kernel (small batches of bf16 decoders); NULL when not eligible
   DfState* df = nullptr;
   std::string df_why;
@@ -255,20 +252,21 @@ static bool ensure_scratch(adept_model* m, size_t elems) {
   return true;
 }
 
+// The generation-step GEMM (gemm_decode.cu) takes single problems of at most DG_MAX_M rows.
+static bool dg_takes(const adept_model* m, int n_probs, const GemmProblem& p, int max_rows, const DgNorm* norm) {
+  return m->dt == ADEPT_DTYPE_BF16 && !m->force_simt && m->use_dg && n_probs == 1 &&
+         decode_gemm_supported(p, max_rows, norm);
+}
+
 static void gemm(adept_model* m, cudaStream_t st, const GemmProblem* probs, int n_probs, const int* max_rows,
                  int cls, double flops = 0, double bytes = 0) {
   cudaEvent_t b = nullptr;
   prof_begin(m, cls, st, &b);
-  int small = 1;
-  for (int i = 0; i < n_probs; ++i) small &= max_rows[i] <= SKINNY_MAX_M;
-  if (m->dt == ADEPT_DTYPE_BF16 && !m->force_simt && small && m->sk_ws && m->use_skinny) {
-    const int nl = skinny_gemm_grouped(st, probs, n_probs, max_rows, m->sk_ws, m->sk_ws_floats, m->sk_counters,
-                                       m->sk_n_counters);
-    if (nl >= 0) {
-      m->launches += nl;
-      prof_end(m, cls, st, b, flops, bytes);
-      return;
-    }
+  if (dg_takes(m, n_probs, probs[0], max_rows[0], nullptr) &&
+      decode_gemm(st, probs[0], max_rows[0], nullptr, m->err_word) >= 0) {
+    m->launches += 1;
+    prof_end(m, cls, st, b, flops, bytes);
+    return;
   }
   if (m->dt == ADEPT_DTYPE_BF16 && !m->force_simt && tc_gemm_supported()) {
     const int nl = tc_gemm_grouped(st, probs, n_probs, max_rows, m->err_word);
@@ -290,6 +288,27 @@ static void gemm(adept_model* m, cudaStream_t st, const GemmProblem* probs, int 
     }
   }
   prof_end(m, cls, st, b, flops, bytes);
+}
+
+// GEMM whose A operand is the standardised rows of X (rows in_rows[r], or r; row length
+// p.K).  The generation-step GEMM standardises while it stages the operand; otherwise the
+// standardisation runs as its own launch into p.A first.
+static void gemm_std(adept_model* m, cudaStream_t st, const GemmProblem& p, int max_rows, const float* X, int ldx,
+                     const int* in_rows, int mode, float eps, int cls) {
+  const DgNorm nrm{X, ldx, in_rows, mode, eps};
+  if (dg_takes(m, 1, p, max_rows, &nrm)) {
+    cudaEvent_t b = nullptr;
+    prof_begin(m, cls, st, &b);
+    if (decode_gemm(st, p, max_rows, &nrm, m->err_word) >= 0) {
+      m->launches += 1;
+      prof_end(m, cls, st, b, 0, 0);
+      return;
+    }
+    prof_end(m, cls, st, b, 0, 0);   // not launched: an empty interval
+  }
+  launch_standardize(st, m->dt, X, ldx, in_rows, p.rows, max_rows, p.K, mode, eps, const_cast<void*>(p.A), p.lda);
+  m->launches += 1;
+  gemm(m, st, &p, 1, &max_rows, cls);
 }
 
 // ---------------------------------------------------------------------------
@@ -607,16 +626,11 @@ static adept_status alloc_runtime(adept_model* m) {
   const int nout = c.family == ADEPT_FAMILY_BERT ? c.n_classes : m->V;
   TRY(dalloc_t(m, &m->logits_ws, (size_t)c.max_batch * nout));
   TRY(dalloc_t(m, &m->attn_ws, (size_t)c.max_batch * m->H * ATTN_MAX_SPLIT * (m->dh + 2)));
+  TRY(dalloc_t(m, &m->attn_ctr, (size_t)c.max_batch * m->H));
+  CUDA_TRY(m, cudaMemset(m->attn_ctr, 0, sizeof(int) * c.max_batch * m->H));
   TRY(dalloc_t(m, &m->d_delta, 1));
   TRY(dalloc_t(m, &m->amax_v, (size_t)c.max_batch * 32));
   TRY(dalloc_t(m, &m->amax_i, (size_t)c.max_batch * 32));
-  if (m->dt == ADEPT_DTYPE_BF16) {
-    m->sk_ws_floats = (size_t)16 << 20;   // 64 MiB of partial tiles
-    m->sk_n_counters = 1 << 16;
-    TRY(dalloc_t(m, &m->sk_ws, m->sk_ws_floats));
-    TRY(dalloc_t(m, &m->sk_counters, m->sk_n_counters));
-    CUDA_TRY(m, cudaMemset(m->sk_counters, 0, sizeof(int) * m->sk_n_counters));
-  }
   TRY(dalloc_t(m, &m->dec_tok, c.max_batch));
   TRY(dalloc_t(m, &m->dec_forced, c.max_batch));
   TRY(dalloc_t(m, &m->dec_exit, c.max_batch));
@@ -755,9 +769,6 @@ static adept_status run_pass(adept_model* m, int n_tok, int batch, int prompt_le
     float* Ii = m->I[par];
     int* rt = m->row_tok[par];
     const int mr = n_tok;
-    // attention input (standardised; gain folded into W_qkv)
-    launch_standardize(st, m->dt, Xi, D, nullptr, act, mr, D, amode, eps, m->xn, D);
-    m->launches += 1;
     // QKV of the active rows, and (prefill) layer i's K/V of every token that exited
     // before layer i, from its mapped state (Sec. 4.3), in one grouped launch.
     GemmProblem pr[2];
@@ -770,19 +781,22 @@ static adept_status run_pass(adept_model* m, int n_tok, int batch, int prompt_le
     pr[0].epi.row_tok = rt; pr[0].epi.tok_seq = m->tok_seq; pr[0].epi.tok_pos = m->tok_pos;
     pr[0].epi.cache = cv; pr[0].epi.layer0 = l0; pr[0].epi.n_q_cols = Dq; pr[0].epi.n_kv_cols = Dkv;
     pr[0].epi.head_dim = m->dh; pr[0].epi.rope = fam == ADEPT_FAMILY_LLAMA; pr[0].epi.rope_table = m->rope_table;
-    int np = 1;
+    // attention input: standardised (gain folded into W_qkv)
     if (!decode && i >= 3) {
       pr[1] = kv_problem(m, l0, m->xfill, n_tok, DevRange{nullptr, m->ctr + CTR_EXITED, 0}, m->exit_tok, m->tok_seq,
                          m->tok_pos);
-      np = 2;
+      launch_standardize(st, m->dt, Xi, D, nullptr, act, mr, D, amode, eps, m->xn, D);
+      m->launches += 1;
+      gemm(m, st, pr, 2, mrs, m->gemm_cls);
+    } else {
+      gemm_std(m, st, pr[0], mr, Xi, D, nullptr, amode, eps, m->gemm_cls);
     }
-    gemm(m, st, pr, np, mrs, m->gemm_cls);
     // attention over every cached position of layer i
     {
       cudaEvent_t b = nullptr;
       prof_begin(m, ADEPT_PROF_ATTENTION, st, &b);
       launch_attention(st, m->dt, m->q, Dq, m->att, Dq, act, mr, rt, m->tok_seq, m->tok_pos, m->d_seq_len, cv, l0,
-                       m->H, causal, decode_keys, m->attn_ws);
+                       m->H, causal, decode_keys, m->attn_ws, m->attn_ctr, m->err_word);
       prof_end(m, ADEPT_PROF_ATTENTION, st, b, 0, 0);
       m->launches += 1;
     }
@@ -798,9 +812,7 @@ static adept_status run_pass(adept_model* m, int n_tok, int batch, int prompt_le
       launch_layernorm_inplace(st, m->X_out, act, mr, D, w.ln1_g, w.ln1_b, eps);
       m->launches += 1;
     }
-    // FFN
-    launch_standardize(st, m->dt, m->X_out, D, nullptr, act, mr, D, amode, eps, m->xn, D);
-    m->launches += 1;
+    // FFN (input standardised)
     p.A = m->xn; p.lda = D; p.B = w.w_up; p.ldb = D; p.N = w.up_rows; p.K = D;
     p.epi = epi_base();
     if (fam == ADEPT_FAMILY_LLAMA) {
@@ -810,7 +822,7 @@ static adept_status run_pass(adept_model* m, int n_tok, int batch, int prompt_le
       p.epi.act = fam == ADEPT_FAMILY_GPT2 ? ACT_GELU_TANH : ACT_GELU_ERF;
     }
     p.epi.bias = w.b_up; p.epi.out_t = m->hbuf; p.epi.ld_t = m->F;
-    gemm(m, st, &p, 1, &mr, m->gemm_cls);
+    gemm_std(m, st, p, mr, m->X_out, D, nullptr, amode, eps, m->gemm_cls);
     p.A = m->hbuf; p.lda = m->F; p.B = w.w_down; p.ldb = m->F; p.N = D; p.K = m->F;
     p.epi = epi_base(); p.epi.kind = EPI_RESID; p.epi.bias = w.b_down; p.epi.out_f32 = m->X_out; p.epi.ld_f32 = D;
     p.epi.resid = m->X_out; p.epi.ld_resid = D;
@@ -825,7 +837,7 @@ static adept_status run_pass(adept_model* m, int n_tok, int batch, int prompt_le
       if (n_tok <= EXIT_SMALL_MAX) {
         launch_exit_small(st, Xi, m->X_out, Ii, i == 1, D, m->ctr, par, rt, m->row_tok[par ^ 1], forced, i, N,
                           m->d_delta, test, sim_out, m->exit_tok, exit_out, m->X_in[par ^ 1], m->I[par ^ 1], m->hsm_s,
-                          m->hsm_prev, m->hsm_I, m->err_word);
+                          m->hsm_prev, m->hsm_I, mr, m->err_word);
         m->launches += 1;
       } else {
         launch_exit_decide(st, m->X_out, Ii, D, act, mr, rt, forced, i, N, m->d_delta, test, sim_out, m->flag,
@@ -876,20 +888,15 @@ static adept_status run_head(adept_model* m, int batch, int prompt_len, bool dec
   memset(&p, 0, sizeof p);
   p.a_rows = batch;
   if (!enc) {
-    launch_standardize(st, m->dt, m->final_, D, m->head_rows, rows, batch, D, attn_norm_mode(m), c.norm_eps, m->xhead,
-                       D);
-    m->launches += 1;
     p.A = m->xhead; p.lda = D; p.B = m->w_head; p.ldb = D; p.rows = rows; p.N = m->V; p.K = D;
     p.epi = epi_base(); p.epi.kind = EPI_F32; p.epi.bias = m->b_head; p.epi.out_f32 = out; p.epi.ld_f32 = m->V;
-    gemm(m, st, &p, 1, &batch, m->gemm_cls);
+    gemm_std(m, st, p, batch, m->final_, D, m->head_rows, attn_norm_mode(m), c.norm_eps, m->gemm_cls);
     if (next) m->launches += launch_argmax(st, out, m->V, batch, next, m->amax_v, m->amax_i);
   } else {
-    launch_standardize(st, m->dt, m->final_, D, m->head_rows, rows, batch, D, NORM_COPY, c.norm_eps, m->xhead, D);
-    m->launches += 1;
     p.A = m->xhead; p.lda = D; p.B = m->w_pool; p.ldb = D; p.rows = rows; p.N = D; p.K = D;
     p.epi = epi_base(); p.epi.kind = EPI_ACT; p.epi.act = ACT_TANH; p.epi.bias = m->b_pool; p.epi.out_t = m->pool_t;
     p.epi.ld_t = D;
-    gemm(m, st, &p, 1, &batch, m->gemm_cls);
+    gemm_std(m, st, p, batch, m->final_, D, m->head_rows, NORM_COPY, c.norm_eps, m->gemm_cls);
     p.A = m->pool_t; p.lda = D; p.B = m->w_cls; p.ldb = D; p.N = c.n_classes; p.K = D;
     p.epi = epi_base(); p.epi.kind = EPI_F32; p.epi.bias = m->b_cls; p.epi.out_f32 = out; p.epi.ld_f32 = c.n_classes;
     gemm(m, st, &p, 1, &batch, m->gemm_cls);
@@ -1234,7 +1241,7 @@ adept_status adept_set_option(adept_model* m, int option, int value) {
     case ADEPT_OPT_PROFILE: m->profile = value != 0; return ADEPT_OK;
     case ADEPT_OPT_GEMM_SIMT: m->force_simt = value != 0; drop_graphs(m); return ADEPT_OK;
     case ADEPT_OPT_DECODE_GRAPH: m->use_graph = value != 0; drop_graphs(m); return ADEPT_OK;
-    case ADEPT_OPT_SKINNY_GEMM: m->use_skinny = value != 0; drop_graphs(m); return ADEPT_OK;
+    case ADEPT_OPT_DECODE_GEMM: m->use_dg = value != 0; drop_graphs(m); return ADEPT_OK;
     case ADEPT_OPT_FUSED_DECODE: m->use_fused = value != 0; return ADEPT_OK;
   }
   return fail(m, ADEPT_ERR_INVALID_ARG, "unknown option %d", option);
@@ -1283,6 +1290,26 @@ int64_t adept_launch_count(adept_model* m) {
 }
 
 }  // extern "C"
+
+#ifdef ADEPT_KTRACE
+namespace adept {
+void kt_attach_attention(void*, unsigned*, unsigned);
+void kt_attach_simt(void*, unsigned*, unsigned);
+void kt_attach_misc(void*, unsigned*, unsigned);
+void kt_attach_tc(void*, unsigned*, unsigned);
+void kt_attach_dg(void*, unsigned*, unsigned);
+}  // namespace adept
+// Debug build only: points every kernel's timeline records at dev_buf (cap records of 104
+// bytes) and the device counter dev_cnt (NULL buffer: recording off).
+extern "C" ADEPT_API void adept_debug_ktrace(void* dev_buf, unsigned* dev_cnt, unsigned cap) {
+  kt_attach_attention(dev_buf, dev_cnt, cap);
+  kt_attach_simt(dev_buf, dev_cnt, cap);
+  kt_attach_misc(dev_buf, dev_cnt, cap);
+  kt_attach_tc(dev_buf, dev_cnt, cap);
+  kt_attach_dg(dev_buf, dev_cnt, cap);
+}
+#endif
+
 
 // ---------------------------------------------------------------------------
 // Read-only view of a loaded model for the allocation-free fill entry point
