@@ -495,8 +495,9 @@ __global__ void __launch_bounds__(AD_THREADS)
                        float scale_log2, int n_split, float* __restrict__ ws, int* counters, bf16* __restrict__ out,
                        int ld_out, unsigned* err) {
   PDL_ENTRY();
-  constexpr int PARTS = DH / 8;          // 16-byte pieces of a K / V row
-  constexpr int KPI = 32 / PARTS;        // keys per warp instruction
+  constexpr int PARTS = DH / 8;                    // 16-byte pieces of a K / V row
+  constexpr int KPI = 32 / PARTS;                  // keys per warp instruction
+  constexpr int KIT = AD_CHUNK / (4 * KPI);        // key groups per warp
   extern __shared__ __align__(128) uint8_t ad_smem[];
   bf16* sK = reinterpret_cast<bf16*>(ad_smem);   // [AD_CHUNK][DH]
   bf16* sV = sK + AD_CHUNK * DH;                  // [AD_CHUNK][DH]
@@ -520,6 +521,7 @@ __global__ void __launch_bounds__(AD_THREADS)
   const int k_lo = split * AD_CHUNK, nkc = min(nk - k_lo, AD_CHUNK);
   const int nb = (nkc + 15) >> 4;                      // cache blocks of the chunk
   constexpr int BLOCK_BYTES = 16 * DH * 2;
+  KT_MARK(0);
 
   if (tid == 0) {
     asm volatile("mbarrier.init.shared::cta.b64 [%0], 1;" ::"r"(ad_smem_u32(&bar)) : "memory");
@@ -553,15 +555,19 @@ __global__ void __launch_bounds__(AD_THREADS)
     }
   }
   const int slot = lane / PARTS, part = lane - slot * PARTS;
+  // the first query head's piece (8 dims per lane), fetched while the cache blocks are in flight
+  uint4 qraw = *reinterpret_cast<const uint4*>(q + (size_t)r * ld_q + kvh * group * DH + part * 8);
+  KT_MARK(1);
   bool ok = ad_wait(&bar, err);
   if (!ok) ad_wait(&bar, err);   // second bounded wait for the copies in flight; results flagged
+  KT_MARK(2);
 
+#pragma unroll 1
   for (int g = 0; g < group; ++g) {
     const int h = kvh * group + g;
-    // query piece of this lane (8 dims), scaled into the log2 domain
     float qv[8];
     {
-      const uint4 u = *reinterpret_cast<const uint4*>(q + (size_t)r * ld_q + h * DH + part * 8);
+      const uint4 u = g == 0 ? qraw : *reinterpret_cast<const uint4*>(q + (size_t)r * ld_q + h * DH + part * 8);
       const __nv_bfloat162* b = reinterpret_cast<const __nv_bfloat162*>(&u);
 #pragma unroll
       for (int i = 0; i < 4; ++i) {
@@ -570,33 +576,49 @@ __global__ void __launch_bounds__(AD_THREADS)
         qv[2 * i + 1] = f.y * scale_log2;
       }
     }
-    // pass 1: scores of the chunk's keys
-    for (int k0 = warp * KPI; k0 < AD_CHUNK; k0 += 4 * KPI) {
-      const int key = k0 + slot;
-      float d = 0.f;
-      if (key < nkc) {
-        const uint4 u = *reinterpret_cast<const uint4*>(sK + key * DH + part * 8);
-        const __nv_bfloat162* b = reinterpret_cast<const __nv_bfloat162*>(&u);
+    // pass 1: scores of the warp's keys (all loads of the warp issued together)
+    {
+      uint4 kr[KIT];
+#pragma unroll
+      for (int it = 0; it < KIT; ++it)
+        kr[it] = *reinterpret_cast<const uint4*>(sK + (warp * KPI + it * 4 * KPI + slot) * DH + part * 8);
+      float d[KIT];
+#pragma unroll
+      for (int it = 0; it < KIT; ++it) {
+        const __nv_bfloat162* b = reinterpret_cast<const __nv_bfloat162*>(&kr[it]);
+        float a = 0.f;
 #pragma unroll
         for (int i = 0; i < 4; ++i) {
           const float2 f = __bfloat1622float2(b[i]);
-          d = fmaf(qv[2 * i], f.x, d);
-          d = fmaf(qv[2 * i + 1], f.y, d);
+          a = fmaf(qv[2 * i], f.x, a);
+          a = fmaf(qv[2 * i + 1], f.y, a);
         }
+        d[it] = a;
       }
 #pragma unroll
-      for (int o = PARTS >> 1; o; o >>= 1) d += __shfl_xor_sync(0xffffffffu, d, o);
-      if (part == 0 && key < AD_CHUNK) s_p[key] = key < nkc ? d : -INFINITY;
+      for (int o = PARTS >> 1; o; o >>= 1)
+#pragma unroll
+        for (int it = 0; it < KIT; ++it) d[it] += __shfl_xor_sync(0xffffffffu, d[it], o);
+      if (part == 0) {
+#pragma unroll
+        for (int it = 0; it < KIT; ++it) {
+          const int key = warp * KPI + it * 4 * KPI + slot;
+          s_p[key] = key < nkc ? d[it] : -INFINITY;
+        }
+      }
     }
     __syncthreads();
+    KT_MARK(3);
     // chunk max, probabilities, chunk sum
     float mx = -INFINITY;
+#pragma unroll
     for (int k = tid; k < AD_CHUNK; k += AD_THREADS) mx = fmaxf(mx, s_p[k]);
     mx = warp_max(mx);
     if (lane == 0) s_red[warp] = mx;
     __syncthreads();
     const float M = fmaxf(fmaxf(s_red[0], s_red[1]), fmaxf(s_red[2], s_red[3]));
     float ls = 0.f;
+#pragma unroll
     for (int k = tid; k < AD_CHUNK; k += AD_THREADS) {
       const float pk = k < nkc ? exp2f(s_p[k] - M) : 0.f;
       s_p[k] = pk;
@@ -605,26 +627,35 @@ __global__ void __launch_bounds__(AD_THREADS)
     ls = warp_sum(ls);
     __syncthreads();   // every s_red[] read and s_p[] write done
     if (lane == 0) s_red[warp] = ls;
-    // pass 2: sum p V, lane = (key slot, 8 dims)
+    KT_MARK(4);
+    // pass 2: sum p V, lane = (key slot, 8 dims); keys past the chunk carry p = 0
     float o[8];
 #pragma unroll
     for (int i = 0; i < 8; ++i) o[i] = 0.f;
-    for (int k0 = warp * KPI; k0 < nkc; k0 += 4 * KPI) {
-      const int key = k0 + slot;
-      if (key < nkc) {
-        const float pk = s_p[key];
-        const uint4 u = *reinterpret_cast<const uint4*>(sV + key * DH + part * 8);
-        const __nv_bfloat162* b = reinterpret_cast<const __nv_bfloat162*>(&u);
+    {
+      uint4 vr[KIT];
+      float pr[KIT];
+#pragma unroll
+      for (int it = 0; it < KIT; ++it) {
+        const int key = warp * KPI + it * 4 * KPI + slot;
+        vr[it] = *reinterpret_cast<const uint4*>(sV + key * DH + part * 8);
+        pr[it] = s_p[key];
+      }
+#pragma unroll
+      for (int it = 0; it < KIT; ++it) {
+        const __nv_bfloat162* b = reinterpret_cast<const __nv_bfloat162*>(&vr[it]);
 #pragma unroll
         for (int i = 0; i < 4; ++i) {
           const float2 f = __bfloat1622float2(b[i]);
-          o[2 * i] = fmaf(pk, f.x, o[2 * i]);
-          o[2 * i + 1] = fmaf(pk, f.y, o[2 * i + 1]);
+          // p == 0 for keys past the chunk (their V rows may hold anything, NaN included)
+          o[2 * i] += pr[it] != 0.f ? pr[it] * f.x : 0.f;
+          o[2 * i + 1] += pr[it] != 0.f ? pr[it] * f.y : 0.f;
         }
       }
     }
 #pragma unroll
     for (int i = 0; i < 8; ++i)
+#pragma unroll
       for (int sft = PARTS; sft < 32; sft <<= 1) o[i] += __shfl_xor_sync(0xffffffffu, o[i], sft);
     if (slot == 0) {
 #pragma unroll
@@ -641,28 +672,47 @@ __global__ void __launch_bounds__(AD_THREADS)
     }
     __threadfence();
     __syncthreads();
+    KT_MARK(5);
     if (tid == 0) s_last = atomicAdd(&counters[rh], 1) == n_eff - 1;
     __syncthreads();
+    KT_MARK(6);
     if (s_last) {
-      // last chunk of (row, head) to finish: merge the chunk partials in chunk order
+      // last chunk of (row, head) to finish: merge the chunk partials in chunk order, every
+      // load of the merge in flight at once
       __threadfence();
       const float* wb = ws + (size_t)rh * n_split * (DH + 2);
-      float Mg = -INFINITY;
-      for (int c = 0; c < n_eff; ++c) Mg = fmaxf(Mg, __ldcg(wb + (size_t)c * (DH + 2) + DH));
-      float L = 0.f;
-      for (int c = 0; c < n_eff; ++c) {
-        const float* wc = wb + (size_t)c * (DH + 2);
-        L += exp2f(__ldcg(wc + DH) - Mg) * __ldcg(wc + DH + 1);
-      }
-      const float inv = L > 0.f ? 1.f / L : 0.f;
-      for (int d = tid; d < DH; d += AD_THREADS) {
-        float acc = 0.f;
-        for (int c = 0; c < n_eff; ++c) {
-          const float* wc = wb + (size_t)c * (DH + 2);
-          acc += exp2f(__ldcg(wc + DH) - Mg) * __ldcg(wc + d);
+      const int d = tid;   // DH <= AD_THREADS
+      // running merge over groups of 8 chunks (8 chunks' loads in flight at a time)
+      float Mg = -INFINITY, L = 0.f, acc = 0.f;
+      for (int c0 = 0; c0 < n_eff; c0 += 8) {
+        float mc[8], lc[8], oc[8];
+#pragma unroll
+        for (int c = 0; c < 8; ++c) {
+          mc[c] = -INFINITY;
+          lc[c] = oc[c] = 0.f;
+          if (c0 + c < n_eff) {
+            const float* wc = wb + (size_t)(c0 + c) * (DH + 2);
+            mc[c] = __ldcg(wc + DH);
+            lc[c] = __ldcg(wc + DH + 1);
+            oc[c] = d < DH ? __ldcg(wc + d) : 0.f;
+          }
         }
-        out[(size_t)r * ld_out + h * DH + d] = __float2bfloat16_rn(acc * inv);
+        float Mn = Mg;
+#pragma unroll
+        for (int c = 0; c < 8; ++c) Mn = fmaxf(Mn, mc[c]);
+        const float corr = Mg == -INFINITY ? 0.f : exp2f(Mg - Mn);
+        L *= corr;
+        acc *= corr;
+#pragma unroll
+        for (int c = 0; c < 8; ++c)
+          if (c0 + c < n_eff) {
+            const float sc = exp2f(mc[c] - Mn);
+            L += sc * lc[c];
+            acc += sc * oc[c];
+          }
+        Mg = Mn;
       }
+      if (d < DH) out[(size_t)r * ld_out + h * DH + d] = __float2bfloat16_rn(L > 0.f ? acc / L : 0.f);
       if (tid == 0) counters[rh] = 0;
     }
     __syncthreads();   // s_p / s_o / s_red reused by the next head of the group
@@ -681,6 +731,7 @@ void launch_attention(cudaStream_t st, int dt, const void* q, int ld_q, void* ou
   const float scale_log2 = 1.4426950408889634f / sqrtf((float)dh);
   if (decode_keys > 0 && ws && counters && dt == 1 && (dh == 64 || dh == 128) && cache.block_tokens == 16 &&
       (decode_keys + AD_CHUNK - 1) / AD_CHUNK <= ATTN_MAX_SPLIT && n_heads % cache.n_kv_heads == 0 &&
+      n_heads / cache.n_kv_heads <= 8 &&
       ld_q % 8 == 0 && ((uintptr_t)q & 15) == 0) {
     const int n_split = (decode_keys + AD_CHUNK - 1) / AD_CHUNK;
     const dim3 grid(max_rows * cache.n_kv_heads, n_split);

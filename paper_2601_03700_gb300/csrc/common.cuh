@@ -45,16 +45,27 @@ __device__ __forceinline__ unsigned long long kt_now() {
   asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
   return t;
 }
+// Intermediate marks are SM cycles since the dependency wait (clock64: fine-grained, valid
+// within one CTA), stored + 1 so that 0 means "not reached".
+__device__ __forceinline__ long long kt_clk() {
+  long long c;
+  asm volatile("mov.u64 %0, %%clock64;" : "=l"(c));
+  return c;
+}
 struct KtScope {
   unsigned long long t0, t1;
+  long long c1;
   unsigned long long mk[KT_MARKS];
   unsigned kid;
-  __device__ explicit KtScope(unsigned k) : t0(kt_now()), t1(0), kid(k) {
+  __device__ explicit KtScope(unsigned k) : t0(kt_now()), t1(0), c1(kt_clk()), kid(k) {
 #pragma unroll
     for (int i = 0; i < KT_MARKS; ++i) mk[i] = 0;
   }
-  __device__ void waited() { t1 = kt_now(); }
-  __device__ void mark(int i) { mk[i] = kt_now(); }
+  __device__ void waited() {
+    t1 = kt_now();
+    c1 = kt_clk();
+  }
+  __device__ void mark(int i) { mk[i] = (unsigned long long)(kt_clk() - c1) + 1; }
   __device__ void add(int i, unsigned long long v) { mk[i] += v; }
   __device__ ~KtScope() {
     if (threadIdx.x == 0 && threadIdx.y == 0 && g_kt_buf) {
@@ -257,7 +268,13 @@ struct Epi {
   int head_dim;
   int rope;          // apply RoPE to q and k
   const float2* rope_table;   // [max_seq][head_dim/2] (cos, sin)
+  // EPI_RESID, generation-step GEMM only (NULL elsewhere): per output row, the (mean, M2)
+  // of each 32-column tile of the result, [row][N / 32], for the next standardisation
+  float2* tile_stats;
 };
+
+// Bits of epi_chunk32's `applied`: work the caller has already done on v.
+enum : int { EPI_APPLIED_BIAS_ACT = 1, EPI_APPLIED_RESID = 2 };
 
 // One problem of a (grouped) GEMM: C[M, N] = A[M, K] * B[N, K]^T, both K-major.
 struct GemmProblem {

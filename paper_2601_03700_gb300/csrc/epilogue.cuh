@@ -78,15 +78,15 @@ __device__ __forceinline__ void rope_pairs(T* dst, int i0, int half, const float
 
 // bias32 / resid32 (optional): the chunk's 32 bias values and the row's 32 residual
 // values already staged by the caller (e.g. in shared memory) instead of e.bias[c0..] and
-// e.resid[ra][c0..].  applied: the caller has already added the bias and applied the
-// EPI_ACT activation to v.  KIND >= 0 fixes the epilogue kind at compile time (only its
-// code is generated); -1 switches on e.kind.
+// e.resid[ra][c0..].  applied (EPI_APPLIED_* bits): what the caller has already done to v
+// (bias and EPI_ACT activation; EPI_RESID residual).  KIND >= 0 fixes the epilogue kind at
+// compile time (only its code is generated); -1 switches on e.kind.
 template <typename T, int KIND = -1>
 __device__ __forceinline__ void epi_chunk32(const Epi& e, int ra, int c0, int N, float (&v)[32], const EpiRow& rr,
                                             const float* bias32 = nullptr, const float* resid32 = nullptr,
-                                            bool applied = false) {
+                                            int applied = 0) {
   const bool full = c0 + 32 <= N;
-  if (applied) {
+  if (applied & EPI_APPLIED_BIAS_ACT) {
   } else if (bias32) {
 #pragma unroll
     for (int j = 0; j < 32; ++j)
@@ -109,7 +109,7 @@ __device__ __forceinline__ void epi_chunk32(const Epi& e, int ra, int c0, int N,
       return;
     }
     case EPI_ACT: {
-      if (!applied) {
+      if (!(applied & EPI_APPLIED_BIAS_ACT)) {
 #pragma unroll
         for (int j = 0; j < 32; ++j) v[j] = apply_act(e.act, v[j]);
       }
@@ -134,8 +134,18 @@ __device__ __forceinline__ void epi_chunk32(const Epi& e, int ra, int c0, int N,
       return;
     }
     case EPI_RESID: {
-      const float* r = resid32 ? resid32 : e.resid + (size_t)ra * e.ld_resid + c0;
       float* o = e.out_f32 + (size_t)ra * e.ld_f32 + c0;
+      if (applied & EPI_APPLIED_RESID) {
+        if (full && ((e.ld_f32 & 15) == 0)) {
+          store16<float>(o, v);
+          store16<float>(o + 16, v + 16);
+        } else {
+          for (int j = 0; j < 32; ++j)
+            if (c0 + j < N) o[j] = v[j];
+        }
+        return;
+      }
+      const float* r = resid32 ? resid32 : e.resid + (size_t)ra * e.ld_resid + c0;
       if (full && ((e.ld_f32 & 15) == 0) && (resid32 || (e.ld_resid & 15) == 0)) {
         const float4* r4 = reinterpret_cast<const float4*>(r);
 #pragma unroll

@@ -42,6 +42,8 @@ constexpr int DG_MAX_A = 16 * 2048;              // A-slice elements a CTA holds
 constexpr int dg_max_kr(int mb) { return DG_MAX_A / (mb * 8); }   // k per CTA: 4096 (M <= 8), 2048
 constexpr int DG_MAX_SPLITS = 8;                 // portable cluster size
 constexpr int DG_RP = DG_BN + 1;                 // floats per token row of a partial tile
+// Where the fused standardisation takes its row statistics from.
+enum : int { DG_STATS_HERE = 0, DG_STATS_ROWS = 1, DG_STATS_TILES = 2 };
 constexpr int DG_ROPE_HALF = 64;                 // rotary pairs per row staged for the epilogue (head_dim <= 128)
 constexpr int DG_XMAX_BYTES = 64 * 1024;         // fp32 rows staged for the fused standardisation
 constexpr long long DG_TIMEOUT_CYCLES = 4000000000LL;   // ~2 s at 2 GHz
@@ -50,17 +52,20 @@ constexpr long long DG_REDUCE_TIMEOUT_CYCLES = 16 * DG_TIMEOUT_CYCLES;
 
 // Dynamic shared memory: weight ring | A slice | staged fp32 rows | partial tiles.
 struct DgLayout {
-  int off_a, off_x, off_p, total;
+  int off_a, off_x, off_t, off_p, total;
 };
 // Offsets are relative to the ring base (the dynamic shared memory rounded up to 1024
 // bytes, as the 128-byte swizzle pattern repeats every 1024 bytes).
-constexpr DgLayout dg_layout(int stages, int mb, int kr, int xrows, int K, int splits) {
+constexpr DgLayout dg_layout(int stages, int mb, int kr, int xrows, int xk, int tstats, int splits) {
   return DgLayout{stages * DG_STAGE, stages * DG_STAGE + mb * 8 * (kr + 8) * 2,
-                  stages * DG_STAGE + mb * 8 * (kr + 8) * 2 + xrows * K * 4,
-                  stages * DG_STAGE + mb * 8 * (kr + 8) * 2 + xrows * K * 4 + 2 * DG_MAX_M * DG_RP * 4 +
-                      (splits - 1) * DG_MAX_M * DG_BN * 4};
+                  stages * DG_STAGE + mb * 8 * (kr + 8) * 2 + xrows * xk * 4,
+                  stages * DG_STAGE + mb * 8 * (kr + 8) * 2 + xrows * xk * 4 + xrows * tstats * 8,
+                  stages * DG_STAGE + mb * 8 * (kr + 8) * 2 + xrows * xk * 4 + xrows * tstats * 8 +
+                      2 * DG_MAX_M * DG_RP * 4 + (splits - 1) * DG_MAX_M * DG_BN * 4};
 }
+constexpr int DG_MAX_TSTATS = 128;               // 32-column tiles of a row (d_model <= 4096)
 constexpr int DG_MAX_SMEM = 1024 + DG_MAX_STAGES * DG_STAGE + (DG_MAX_A + 16 * 8) * 2 + DG_XMAX_BYTES +
+                            DG_MAX_M * DG_MAX_TSTATS * 8 +
                             2 * DG_MAX_M * DG_RP * 4 + (DG_MAX_SPLITS - 1) * DG_MAX_M * DG_BN * 4;
 constexpr int DG_STATIC_SMEM = 12 * 1024;         // static shared memory of the kernel (bound)
 static_assert(DG_MAX_SMEM + DG_STATIC_SMEM <= 227 * 1024, "shared memory budget");
@@ -86,7 +91,12 @@ struct DgParams {
   int pre;      // stages issued before the grid-dependency wait
   int max_m;    // rows the launch was sized for
   int xrows;    // fp32 rows staged in shared memory for the standardisation (0: streamed)
-  int off_a, off_x, off_p;   // dynamic shared-memory offsets (bytes)
+  int xk;       // staged floats per row: K (statistics computed here) or kr (a k-slice)
+  int stat_mode;   // DG_STATS_*
+  const float2* row_stats;    // DG_STATS_ROWS: (mu, rstd) per row
+  const float2* tile_stats;   // DG_STATS_TILES: [row][n_stiles] (mean, M2) of 32-column tiles
+  int n_stiles;
+  int off_a, off_x, off_t, off_p;   // dynamic shared-memory offsets (bytes)
   int bias_aligned, resid_aligned;
   Epi epi;
   unsigned* err;
@@ -188,7 +198,7 @@ __device__ __forceinline__ void cluster_sync() {
 }
 // MB: 8-token blocks of the A operand (1: M <= 8, 2: M <= 16); KIND: the epilogue kind.
 template <int MB, int KIND>
-__global__ void __launch_bounds__(DG_THREADS) gemm_decode_kernel(const __grid_constant__ DgParams p) {
+__global__ void __launch_bounds__(DG_THREADS, 1) gemm_decode_kernel(const __grid_constant__ DgParams p) {
   KT_BEGIN();
   extern __shared__ __align__(128) uint8_t dg_smem_raw[];
   __shared__ __align__(8) uint64_t full[DG_MAX_STAGES];
@@ -214,7 +224,8 @@ __global__ void __launch_bounds__(DG_THREADS) gemm_decode_kernel(const __grid_co
   uint8_t* dg_smem = dg_smem_raw + ((1024 - (smem_u32(dg_smem_raw) & 1023)) & 1023);
   uint8_t* sW = dg_smem;                                                // [S][2][32 rows][128 B], swizzled
   bf16* sA = reinterpret_cast<bf16*>(dg_smem + p.off_a);                // [MB*8][apitch]
-  float* sX = reinterpret_cast<float*>(dg_smem + p.off_x);              // [xrows][K] (fused standardisation)
+  float* sX = reinterpret_cast<float*>(dg_smem + p.off_x);              // [xrows][xk] (fused standardisation)
+  float2* sT = reinterpret_cast<float2*>(dg_smem + p.off_t);            // [xrows][n_stiles] producer tile stats
   constexpr int SLOT = DG_MAX_M * DG_RP;
   float* sP = reinterpret_cast<float*>(dg_smem + p.off_p);              // [2][DG_MAX_M][DG_RP]: own k halves
   float* sR = sP + 2 * SLOT;                                            // [splits - 1][DG_MAX_M][32]: pushed
@@ -280,16 +291,24 @@ __global__ void __launch_bounds__(DG_THREADS) gemm_decode_kernel(const __grid_co
   if (warp < 3) {
     const int t = tid;   // 0..95
     if (p.fused_norm && p.xrows) {
+      // fp32 rows: whole (statistics computed here) or only the k-slice (statistics from
+      // the producer), and the producer's per-tile statistics
       int src[MB * 8];
 #pragma unroll
       for (int r = 0; r < MB * 8; ++r) src[r] = r < M ? (p.in_rows ? p.in_rows[rb + r] : rb + r) : 0;
-      const int cpr = p.K >> 2;   // 16-byte chunks per fp32 row
+      const int x0 = p.stat_mode == DG_STATS_HERE ? 0 : k_lo;
+      const int cpr = (p.stat_mode == DG_STATS_HERE ? p.K : kr) >> 2;   // 16-byte chunks per row
 #pragma unroll
       for (int r = 0; r < MB * 8; ++r) {
         if (r >= M) break;
-        const float* x = p.X + (size_t)src[r] * p.ldx;
-        for (int c = t; c < cpr; c += 96) cp_async16(sX + (size_t)r * p.K + c * 4, x + c * 4);
+        const float* x = p.X + (size_t)src[r] * p.ldx + x0;
+        for (int c = t; c < cpr; c += 96) cp_async16(sX + (size_t)r * p.xk + c * 4, x + c * 4);
       }
+      if (p.stat_mode == DG_STATS_TILES)
+        for (int c = t; c < M * (p.n_stiles >> 1); c += 96) {
+          const int r = c / (p.n_stiles >> 1), q = c - r * (p.n_stiles >> 1);
+          cp_async16(sT + (size_t)r * p.n_stiles + q * 2, p.tile_stats + (size_t)(rb + r) * p.n_stiles + q * 2);
+        }
     } else if (!p.fused_norm) {
       const int cpr = kr >> 3;   // 16-byte chunks per bf16 row
       for (int r = 0; r < M; ++r) {
@@ -298,6 +317,11 @@ __global__ void __launch_bounds__(DG_THREADS) gemm_decode_kernel(const __grid_co
       }
     }
   } else {
+    if (p.fused_norm && p.stat_mode == DG_STATS_ROWS && lane < M) {
+      const float2 st = p.row_stats[rb + lane];
+      s_mu[lane] = st.x;
+      s_rs[lane] = st.y;
+    }
     if (st_bias && lane < DG_BN / 4) cp_async16(s_bias + lane * 4, e.bias + f_single + lane * 4);
     if (st_res)
       for (int c = lane; c < M * (DG_BN / 4); c += 32) {
@@ -319,7 +343,7 @@ __global__ void __launch_bounds__(DG_THREADS) gemm_decode_kernel(const __grid_co
   __syncthreads();
   KT_MARK(1);
 
-  // ---- fused standardisation of the A operand (full-row statistics; gains live in W)
+  // ---- fused standardisation of the A operand (gains live in W)
   if (p.fused_norm) {
     const int K = p.K;
     if (p.xrows) {
@@ -328,48 +352,86 @@ __global__ void __launch_bounds__(DG_THREADS) gemm_decode_kernel(const __grid_co
       const int tpr = DG_THREADS >> lg;
       const int r = tid >> (7 - lg), sub = tid & (tpr - 1);
       const bool live = r < M;
-      const float4* x4 = reinterpret_cast<const float4*>(sX + (size_t)(live ? r : 0) * K);
-      const int K4 = K >> 2;
-      // sum over the row's tpr threads (shuffles within a warp, shared memory across warps)
-      auto group_sum = [&](float v) {
-        if (tpr <= 32) {
-          for (int o = tpr >> 1; o; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
-          return v;
+      const float4* x4 = reinterpret_cast<const float4*>(sX + (size_t)(live ? r : 0) * p.xk);
+      if (p.stat_mode == DG_STATS_HERE) {
+        const int K4 = K >> 2;
+        // sum over the row's tpr threads (shuffles within a warp, shared memory across warps)
+        auto group_sum = [&](float v) {
+          if (tpr <= 32) {
+            for (int o = tpr >> 1; o; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+            return v;
+          }
+          v = warp_sum(v);
+          if (lane == 0) s_red[warp][0] = v;
+          __syncthreads();
+          const int w0 = (tid / tpr) * (tpr >> 5);
+          float t = 0.f;
+          for (int w = 0; w < (tpr >> 5); ++w) t += s_red[w0 + w][0];
+          __syncthreads();
+          return t;
+        };
+        float mu = 0.f, rs = 1.f;
+        if (p.norm_mode == NORM_LN) {
+          float a0 = 0.f, a1 = 0.f;
+          if (live)
+            for (int v = sub; v < K4; v += tpr) {
+              const float4 t = x4[v];
+              a0 += t.x + t.y;
+              a1 += t.z + t.w;
+            }
+          mu = group_sum(a0 + a1) / K;
         }
-        v = warp_sum(v);
-        if (lane == 0) s_red[warp][0] = v;
-        __syncthreads();
-        const int w0 = (tid / tpr) * (tpr >> 5);
-        float t = 0.f;
-        for (int w = 0; w < (tpr >> 5); ++w) t += s_red[w0 + w][0];
-        __syncthreads();
-        return t;
-      };
-      float mu = 0.f, rs = 1.f;
-      if (p.norm_mode == NORM_LN) {
-        float a0 = 0.f, a1 = 0.f;
-        if (live)
-          for (int v = sub; v < K4; v += tpr) {
-            const float4 t = x4[v];
-            a0 += t.x + t.y;
-            a1 += t.z + t.w;
+        if (p.norm_mode != NORM_COPY) {
+          float a0 = 0.f, a1 = 0.f;
+          if (live)
+            for (int v = sub; v < K4; v += tpr) {
+              const float4 t = x4[v];
+              const float c0 = t.x - mu, c1 = t.y - mu, c2 = t.z - mu, c3 = t.w - mu;
+              a0 += c0 * c0 + c1 * c1;
+              a1 += c2 * c2 + c3 * c3;
+            }
+          rs = rsqrtf(group_sum(a0 + a1) / K + p.eps);
+        }
+        if (live && sub == 0) {
+          s_mu[r] = mu;
+          s_rs[r] = rs;
+        }
+      } else if (p.stat_mode == DG_STATS_TILES) {
+        // the row's moments from the producer's 32-column (mean, M2) tiles, about the first
+        // tile's mean c: S1 = sum 32 (m_t - c), S2 = sum M2_t + 32 (m_t - c)^2; warp w takes
+        // rows w, w + 4, ..., lane l tiles l, l + 32, ...
+        for (int r2 = warp; r2 < M; r2 += 4) {
+          const float2* ts = sT + (size_t)r2 * p.n_stiles;
+          const float c = ts[0].x;
+          float s1 = 0.f, s2 = 0.f;
+          for (int t = lane; t < p.n_stiles; t += 32) {
+            const float2 b = ts[t];
+            const float dm = b.x - c;
+            s1 += 32.f * dm;
+            s2 += b.y + 32.f * dm * dm;
           }
-        mu = group_sum(a0 + a1) / K;
-      }
-      if (p.norm_mode != NORM_COPY) {
-        float a0 = 0.f, a1 = 0.f;
-        if (live)
-          for (int v = sub; v < K4; v += tpr) {
-            const float4 t = x4[v];
-            const float c0 = t.x - mu, c1 = t.y - mu, c2 = t.z - mu, c3 = t.w - mu;
-            a0 += c0 * c0 + c1 * c1;
-            a1 += c2 * c2 + c3 * c3;
+          s1 = warp_sum(s1);
+          s2 = warp_sum(s2);
+          if (lane == 0) {
+            const float dmean = s1 / K, var = fmaxf(s2 / K - dmean * dmean, 0.f), mean = c + dmean;
+            float mu = 0.f, rs = 1.f;
+            if (p.norm_mode == NORM_LN) {
+              mu = mean;
+              rs = rsqrtf(var + p.eps);
+            } else if (p.norm_mode == NORM_RMS) {
+              rs = rsqrtf(var + mean * mean + p.eps);
+            }
+            s_mu[r2] = mu;
+            s_rs[r2] = rs;
           }
-        rs = rsqrtf(group_sum(a0 + a1) / K + p.eps);
+        }
       }
-      if (live)
+      __syncthreads();
+      if (live) {
+        const float mu = s_mu[r], rs = s_rs[r];
+        const int xoff = p.stat_mode == DG_STATS_HERE ? (k_lo >> 2) : 0;
         for (int v = sub; v < (kr >> 2); v += tpr) {
-          const float4 t = x4[(k_lo >> 2) + v];
+          const float4 t = x4[xoff + v];
           const __nv_bfloat162 lo = __floats2bfloat162_rn((t.x - mu) * rs, (t.y - mu) * rs);
           const __nv_bfloat162 hi = __floats2bfloat162_rn((t.z - mu) * rs, (t.w - mu) * rs);
           uint2 u;
@@ -377,6 +439,7 @@ __global__ void __launch_bounds__(DG_THREADS) gemm_decode_kernel(const __grid_co
           u.y = *reinterpret_cast<const uint32_t*>(&hi);
           *reinterpret_cast<uint2*>(sA + r * apitch + v * 4) = u;
         }
+      }
     } else {
       // rows too long to stage: block sums over global memory, all rows at once
       const float* xr[MB * 8];
@@ -530,28 +593,59 @@ __global__ void __launch_bounds__(DG_THREADS) gemm_decode_kernel(const __grid_co
     KT_MARK(4);
     if (dead) return;
 
-    // bias and activation element-wise over the block, then the stores of the fused
-    // epilogue: one thread per token row, 32 features
-    if (e.bias || KIND == EPI_ACT) {
-      for (int e2 = tid; e2 < M * DG_BN; e2 += DG_THREADS) {
-        const int c = e2 & 31, i = (e2 >> 5) * DG_RP + c;
-        float v = sP[i];
-        if (e.bias && f0 + c < p.N) v += st_bias ? s_bias[c] : e.bias[f0 + c];
-        if (KIND == EPI_ACT) v = apply_act(e.act, v);
-        sP[i] = v;
+    // fused epilogue, element-parallel: warp w takes rows w, w + 4, ..., lane = feature
+    KT_MARK(5);
+    for (int row = warp; row < M; row += 4) {
+      const int ra = rb + row, c = f0 + lane;
+      const bool valid = c < p.N;
+      float v = sP[row * DG_RP + lane];
+      if (e.bias && valid) v += st_bias ? s_bias[lane] : e.bias[c];
+      if (KIND == EPI_F32) {
+        if (valid) e.out_f32[(size_t)ra * e.ld_f32 + c] = v;
+      } else if (KIND == EPI_ACT) {
+        v = apply_act(e.act, v);
+        if (valid) {
+          ((bf16*)e.out_t)[(size_t)ra * e.ld_t + c] = __float2bfloat16_rn(v);
+          if (e.out_f32) e.out_f32[(size_t)ra * e.ld_f32 + c] = v;
+        }
+      } else if (KIND == EPI_RESID) {
+        if (valid) v += st_res ? s_res[row][lane] : e.resid[(size_t)ra * e.ld_resid + c];
+        if (valid) e.out_f32[(size_t)ra * e.ld_f32 + c] = v;
+        if (e.tile_stats) {   // (mean, M2) of the row's 32 results (full tiles: N % 32 == 0)
+          const float mean = warp_sum(v) * (1.f / DG_BN);
+          const float m2 = warp_sum((v - mean) * (v - mean));
+          if (lane == 0) e.tile_stats[(size_t)ra * (p.N / DG_BN) + f0 / DG_BN] = make_float2(mean, m2);
+        }
+      } else if (KIND == EPI_SWIGLU) {
+        // features interleaved in blocks of 16: lanes 0-15 gate, 16-31 the matching up
+        const float u = __shfl_down_sync(0xffffffffu, v, 16);
+        if (lane < 16) ((bf16*)e.out_t)[(size_t)ra * e.ld_t + (f0 >> 1) + lane] = __float2bfloat16_rn(silu_f(v) * u);
+      } else {   // EPI_QKV / EPI_KV: q -> out_t, k / v -> the row's cache slot; RoPE pairs adjacent
+        const EpiRow rr = st_rows ? s_rr[row] : epi_row(e, ra);
+        const int dh = e.head_dim, half = dh >> 1, nq = e.n_q_cols, nkv = e.n_kv_cols;
+        const int base = c < nq ? 0 : c < nq + nkv ? nq : nq + nkv;
+        const int hd = (c - base) / dh, d = (c - base) - hd * dh;
+        const float pv = __shfl_xor_sync(0xffffffffu, v, 1);   // the other member of the pair
+        float o = v;
+        int od = d;
+        if (e.rope && base < nq + nkv) {
+          const int ip = d >> 1;
+          const float2 cs = rr.rope ? rr.rope[ip] : e.rope_table[(size_t)rr.pos * half + ip];
+          // (x1, x2) = (even, odd) column of the pair -> x1 c - x2 s at ip, x2 c + x1 s at ip + half
+          o = (d & 1) ? v * cs.x + pv * cs.y : v * cs.x - pv * cs.y;
+          od = (d & 1) ? ip + half : ip;
+        }
+        if (valid) {
+          if (base == 0 && nq > 0) {
+            ((bf16*)e.out_t)[(size_t)ra * e.ld_t + hd * dh + od] = __float2bfloat16_rn(o);
+          } else if (rr.cbase >= 0) {
+            bf16* dst = (bf16*)(base == nq ? e.cache.k : e.cache.v);
+            dst[rr.cbase + (size_t)hd * e.cache.head_stride() + od] = __float2bfloat16_rn(o);
+          }
+        }
       }
-      __syncthreads();
     }
-    if (tid < M) {
-      float v[32];
-#pragma unroll
-      for (int t = 0; t < 32; ++t) v[t] = sP[tid * DG_RP + t];
-      const int ra = rb + tid;
-      const EpiRow rr = st_rows ? s_rr[tid] : epi_row(e, ra);
-      KT_MARK(5);
-      epi_chunk32<bf16, KIND>(e, ra, f0, p.N, v, rr, nullptr, st_res ? s_res[tid] : nullptr, true);
-      KT_MARK(6);
-    }
+    KT_MARK(6);
     __syncthreads();   // slot 0 is rewritten by the next tile
   }
 }
@@ -615,6 +709,8 @@ bool decode_gemm_supported(const GemmProblem& q, int max_rows, const DgNorm* nor
   if ((q.epi.kind == EPI_QKV || q.epi.kind == EPI_KV || q.epi.kind == EPI_SWIGLU) && q.N % 32) return false;
   if (q.epi.rope && (q.epi.head_dim > 2 * DG_ROPE_HALF || q.epi.head_dim % 4)) return false;
   if (q.epi.kind < EPI_F32 || q.epi.kind > EPI_KV) return false;
+  if (q.epi.tile_stats && (q.epi.kind != EPI_RESID || q.N % DG_BN)) return false;
+  if (norm && norm->tile_stats && (q.K % 64 || ((uintptr_t)norm->tile_stats & 15))) return false;
   return true;
 }
 
@@ -658,13 +754,24 @@ int decode_gemm(cudaStream_t st, const GemmProblem& q, int max_rows, const DgNor
   prm.kr = kr;
   prm.stages = stages;
   prm.max_m = max_rows;
-  prm.xrows = norm && (size_t)max_rows * q.K * 4 <= (size_t)DG_XMAX_BYTES && norm->ldx % 4 == 0 &&
-                      ((uintptr_t)norm->X & 15) == 0
-                  ? max_rows
-                  : 0;
-  const DgLayout L = dg_layout(stages, mb, kr, prm.xrows, q.K, splits);
+  // statistics from the producer when given (only the k-slice of each row is staged),
+  // else computed here from whole staged rows (or, rows too long to stage, streamed)
+  prm.stat_mode = !norm                                             ? DG_STATS_HERE
+                  : norm->row_stats                                 ? DG_STATS_ROWS
+                  : norm->tile_stats && q.K / 32 <= DG_MAX_TSTATS ? DG_STATS_TILES
+                                                                    : DG_STATS_HERE;
+  prm.row_stats = norm ? norm->row_stats : nullptr;
+  prm.tile_stats = norm ? norm->tile_stats : nullptr;
+  prm.n_stiles = q.K / 32;
+  prm.xk = prm.stat_mode == DG_STATS_HERE ? q.K : kr;
+  const bool x_ok = norm && norm->ldx % 4 == 0 && ((uintptr_t)norm->X & 15) == 0;
+  prm.xrows = x_ok && (size_t)max_rows * prm.xk * 4 <= (size_t)DG_XMAX_BYTES ? max_rows : 0;
+  if (prm.xrows == 0) prm.stat_mode = DG_STATS_HERE;   // the streamed path computes its own
+  const DgLayout L =
+      dg_layout(stages, mb, kr, prm.xrows, prm.xk, prm.stat_mode == DG_STATS_TILES ? prm.n_stiles : 0, splits);
   prm.off_a = L.off_a;
   prm.off_x = L.off_x;
+  prm.off_t = L.off_t;
   prm.off_p = L.off_p;
   prm.bias_aligned = ((uintptr_t)q.epi.bias & 15) == 0;
   prm.resid_aligned = ((uintptr_t)q.epi.resid & 15) == 0 && q.epi.ld_resid % 4 == 0;

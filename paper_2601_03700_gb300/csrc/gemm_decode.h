@@ -16,6 +16,11 @@ struct DgNorm {
   const int* in_rows;
   int mode;     // NormMode
   float eps;
+  // Row statistics computed by the producer of X (optional; else computed here from the
+  // whole rows): row_stats, (mu, rstd) per row; or tile_stats, [row][K / 32] (mean, M2)
+  // of each 32-column tile, merged here in tile order.
+  const float2* row_stats;
+  const float2* tile_stats;
 };
 
 // Enqueues one problem (bf16 operands, fused epilogue).  norm == NULL: A is bf16 at

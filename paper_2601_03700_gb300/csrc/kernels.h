@@ -17,9 +17,10 @@ __host__ __device__ static inline int ctr_words(int n_layers) { return CTR_PREFI
 void launch_pass_init(cudaStream_t st, int n_tok, int prompt_len, int decode, int* tok_seq, int* tok_pos,
                       int* row_tok, int* seq_len, int seq_cap, int max_pos, unsigned* err, int* ctr, int n_ctr,
                       float* sim, int n_layers);
+// xhat (optional, decoders): the embedded rows standardised (smode, seps) in bf16, [n_tok][D].
 void launch_embed(cudaStream_t st, int dt, const int* tokens, int n_tok, const int* tok_pos, const void* E,
                   const void* P, const float* type_emb, const float* g, const float* b, int family, int D, int V,
-                  float eps, float* X, unsigned* err);
+                  float eps, float* X, unsigned* err, bf16* xhat, int smode, float seps);
 void launch_standardize(cudaStream_t st, int dt, const float* X, int ldx, const int* in_rows, DevRange rows,
                         int max_rows, int D, int mode, float eps, void* out, int ld_out);
 void launch_layernorm_inplace(cudaStream_t st, float* X, DevRange rows, int max_rows, int D, const float* g,
@@ -28,13 +29,16 @@ void launch_exit_decide(cudaStream_t st, const float* Xout, const float* I, int 
                         const int* row_tok, const int* forced, int layer, int n_layers, const float* delta_p, int test,
                         float* sim, int* flag, float* inv_norm, unsigned* err);
 // Test + compaction + moves in one CTA for passes of at most EXIT_SMALL_MAX rows
-// (max_rows: the pass's row bound; at most 16 rows take a register-resident kernel).
+// (max_rows: the pass's row bound; at most 16 rows take a register-resident kernel, which
+// also writes xhat_next (if given): each kept row standardised (smode, seps) for the next
+// layer's attention input, bf16 [new row][D]).  Returns whether the register-resident
+// kernel ran (xhat_next written).
 constexpr int EXIT_SMALL_MAX = 256;
-void launch_exit_small(cudaStream_t st, const float* Xin, const float* Xout, const float* I, int first, int D,
+bool launch_exit_small(cudaStream_t st, const float* Xin, const float* Xout, const float* I, int first, int D,
                        int* ctr, int par, const int* row_tok, int* row_tok_next, const int* forced, int layer,
                        int n_layers, const float* delta_p, int test, float* sim, int* exit_tok, int* exit_layer_out,
                        float* Xnext, float* Inext, float* hsm_s, float* hsm_prev, float* hsm_I, int max_rows,
-                       unsigned* err);
+                       bf16* xhat_next, int smode, float seps, unsigned* err);
 void launch_set_float(cudaStream_t st, float* p, float v);
 void launch_exit_scan(cudaStream_t st, int* ctr, int in_parity, const int* flag, const int* row_tok,
                       int* row_tok_next, int* exit_tok, int* dst, int* exit_layer_out, int layer);

@@ -47,10 +47,12 @@ __global__ void pass_init_kernel(int n_tok, int prompt_len, int decode, int* tok
 // ---------------------------------------------------------------------------
 // embedding (s_0): token embedding (+ learned position) (+ type and LayerNorm for BERT)
 // ---------------------------------------------------------------------------
+// xhat (optional, decoders): each embedded row standardised for the first layer's
+// attention input (smode, seps), as the standardisation kernel computes it, in bf16.
 template <typename T>
 __global__ void embed_kernel(const int* tokens, int n_tok, const int* tok_pos, const T* E, const T* P,
                              const float* type_emb, const float* g, const float* b, int family, int D, int V,
-                             float eps, float* X, unsigned* err) {
+                             float eps, float* X, unsigned* err, bf16* xhat, int smode, float seps) {
   PDL_ENTRY();
   __shared__ float red[32];
   const int t = blockIdx.x;
@@ -70,7 +72,21 @@ __global__ void embed_kernel(const int* tokens, int n_tok, const int* tok_pos, c
     x[d] = v;
     s1 += v;
   }
-  if (family != 2) return;
+  if (family != 2) {
+    if (!xhat) return;
+    // the thread re-reads only the elements it wrote
+    const float mu = smode == NORM_LN ? block_sum(s1, red) / D : 0.f;
+    float s2 = 0.f;
+    for (int d = threadIdx.x; d < D; d += blockDim.x) {
+      const float c = x[d] - mu;
+      s2 += c * c;
+    }
+    const float tot = block_sum(s2, red);
+    const float rs = smode == NORM_COPY ? 1.f : rsqrtf(tot / D + seps);
+    const float m0 = smode == NORM_COPY ? 0.f : mu;
+    for (int d = threadIdx.x; d < D; d += blockDim.x) xhat[(size_t)t * D + d] = __float2bfloat16_rn((x[d] - m0) * rs);
+    return;
+  }
   const float mu = block_sum(s1, red) / D;
   float s2 = 0.f;
   for (int d = threadIdx.x; d < D; d += blockDim.x) {
@@ -357,20 +373,26 @@ __global__ void __launch_bounds__(EXD_THREADS)
                        int layer, int n_layers, const float* delta_p, int test, float* sim, int* exit_tok,
                        int* exit_layer_out, float* __restrict__ Xnext, float* __restrict__ Inext,
                        float* __restrict__ hsm_s, float* __restrict__ hsm_prev, float* __restrict__ hsm_I, int rshift,
-                       unsigned* err) {
+                       int max_rows, bf16* xhat_next, int smode, float seps, unsigned* err) {
   PDL_ENTRY();
-  __shared__ float s_red[EXD_THREADS / 32][3];
+  __shared__ float s_red[EXD_THREADS / 32][4];
+  __shared__ float s_mu[16];
   __shared__ int s_dst[16], s_tok[16];
   __shared__ float s_w[16];
   const int tpr = EXD_THREADS >> rshift;   // threads per row
   const int row = threadIdx.x >> (9 - rshift), sub = threadIdx.x & (tpr - 1);
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int n = min(ctr[CTR_ACTIVE + par], 1 << rshift);
+  // every independent load first: the counters, the decider's token and threshold, and the
+  // row vectors of every row slot below the pass's row bound (slots past the active count
+  // read rows of the pass's buffers whose values go unused)
+  const int n = min(min(ctr[CTR_ACTIVE + par], 1 << rshift), max_rows);
+  const int base = ctr[CTR_EXITED];
+  const int tok_r = (int)threadIdx.x < max_rows ? row_tok[threadIdx.x] : 0;
+  const float delta = *delta_p;
   const int D4 = D >> 2;
-  const bool live = row < n;
   float4 xs[EXD_V], xi[EXD_V], xp[EXD_V];
-  float ns = 0.f, ni = 0.f, dot = 0.f;
-  if (live) {
+  float ns = 0.f, ni = 0.f, dot = 0.f, sx = 0.f;
+  if (row < max_rows) {
     const float4* s4 = reinterpret_cast<const float4*>(Xout + (size_t)row * D);
     const float4* i4 = reinterpret_cast<const float4*>(I + (size_t)row * D);
     const float4* p4 = reinterpret_cast<const float4*>(Xin + (size_t)row * D);
@@ -385,39 +407,45 @@ __global__ void __launch_bounds__(EXD_THREADS)
     }
 #pragma unroll
     for (int j = 0; j < EXD_V; ++j) {
-      if (sub + j * tpr < D4) {
+      if (row < n && sub + j * tpr < D4) {
         const float4 a = xs[j], c = xi[j];
         ns += a.x * a.x + a.y * a.y + a.z * a.z + a.w * a.w;
         ni += c.x * c.x + c.y * c.y + c.z * c.z + c.w * c.w;
         dot += a.x * c.x + a.y * c.y + a.z * c.z + a.w * c.w;
+        sx += a.x + a.y + a.z + a.w;
       }
     }
   }
   ns = warp_sum(ns);
   ni = warp_sum(ni);
   dot = warp_sum(dot);
+  sx = warp_sum(sx);
   if (lane == 0) {
     s_red[warp][0] = ns;
     s_red[warp][1] = ni;
     s_red[warp][2] = dot;
+    s_red[warp][3] = sx;
   }
   __syncthreads();
+  const int wpr = tpr >> 5;   // warps per row
   if ((int)threadIdx.x < n) {   // thread r decides row r
-    const int r = threadIdx.x, wpr = tpr >> 5;
-    float a = 0.f, b = 0.f, c = 0.f;
+    const int r = threadIdx.x;
+    float a = 0.f, b = 0.f, c = 0.f, m = 0.f;
     for (int w = r * wpr; w < (r + 1) * wpr; ++w) {
       a += s_red[w][0];
       b += s_red[w][1];
       c += s_red[w][2];
+      m += s_red[w][3];
     }
-    const int tok = row_tok[r];
+    s_mu[r] = smode == NORM_LN ? m / D : 0.f;
+    const int tok = tok_r;
     int ex = 0;
     if (test) {
       const float cs = (a > 0.f && b > 0.f) ? c / sqrtf(a * b) : -INFINITY;
       if (sim) sim[(size_t)tok * n_layers + (layer - 1)] = cs;
       const int f = forced ? forced[tok] : 0;
       if (f != 0 && (f < 2 || f > n_layers)) atomicOr(err, ERRW_FORCED);
-      ex = (f > 0) ? (f == layer) : (cs >= *delta_p);
+      ex = (f > 0) ? (f == layer) : (cs >= delta);
     }
     s_dst[r] = ex;
     s_tok[r] = tok;
@@ -425,7 +453,6 @@ __global__ void __launch_bounds__(EXD_THREADS)
   }
   __syncthreads();
   if (threadIdx.x == 0) {   // stable compaction (n <= 16)
-    const int base = ctr[CTR_EXITED];
     int e = 0, k = 0;
     for (int r = 0; r < n; ++r) {
       const int tok = s_tok[r];
@@ -445,7 +472,45 @@ __global__ void __launch_bounds__(EXD_THREADS)
     ctr[CTR_PREFIX + layer] = base + e;
   }
   __syncthreads();
-  if (!live) return;
+  if (xhat_next) {
+    // the kept rows standardised for the next layer's attention input, as the
+    // standardisation kernel computes them (two-pass: the centred second moment from the
+    // registers); written to row d0 of xhat_next in bf16
+    const float mu = row < n ? s_mu[row] : 0.f;
+    float c2 = 0.f;
+    if (row < n) {
+#pragma unroll
+      for (int j = 0; j < EXD_V; ++j)
+        if (sub + j * tpr < D4) {
+          const float4 a = xs[j];
+          c2 += (a.x - mu) * (a.x - mu) + (a.y - mu) * (a.y - mu) + (a.z - mu) * (a.z - mu) + (a.w - mu) * (a.w - mu);
+        }
+    }
+    c2 = warp_sum(c2);
+    if (lane == 0) s_red[warp][0] = c2;
+    __syncthreads();
+    if (row < n && s_dst[row] >= 0) {
+      float t = 0.f;
+      for (int w = row * wpr; w < (row + 1) * wpr; ++w) t += s_red[w][0];
+      const float rs = smode == NORM_COPY ? 1.f : rsqrtf(t / D + seps);
+      const float m0 = smode == NORM_COPY ? 0.f : mu;
+      uint2* o = reinterpret_cast<uint2*>(xhat_next + (size_t)s_dst[row] * D);
+#pragma unroll
+      for (int j = 0; j < EXD_V; ++j) {
+        const int v = sub + j * tpr;
+        if (v < D4) {
+          const float4 a = xs[j];
+          const __nv_bfloat162 lo = __floats2bfloat162_rn((a.x - m0) * rs, (a.y - m0) * rs);
+          const __nv_bfloat162 hi = __floats2bfloat162_rn((a.z - m0) * rs, (a.w - m0) * rs);
+          uint2 u;
+          u.x = *reinterpret_cast<const uint32_t*>(&lo);
+          u.y = *reinterpret_cast<const uint32_t*>(&hi);
+          o[v] = u;
+        }
+      }
+    }
+  }
+  if (row >= n) return;
   const int d0 = s_dst[row];
   if (d0 >= 0) {
     const float w = s_w[row];
@@ -477,11 +542,11 @@ __global__ void __launch_bounds__(EXD_THREADS)
   }
 }
 
-void launch_exit_small(cudaStream_t st, const float* Xin, const float* Xout, const float* I, int first, int D,
+bool launch_exit_small(cudaStream_t st, const float* Xin, const float* Xout, const float* I, int first, int D,
                        int* ctr, int par, const int* row_tok, int* row_tok_next, const int* forced, int layer,
                        int n_layers, const float* delta_p, int test, float* sim, int* exit_tok, int* exit_layer_out,
                        float* Xnext, float* Inext, float* hsm_s, float* hsm_prev, float* hsm_I, int max_rows,
-                       unsigned* err) {
+                       bf16* xhat_next, int smode, float seps, unsigned* err) {
   int rshift = 0;
   while ((1 << rshift) < max_rows) ++rshift;
   const bool aligned = ((uintptr_t)Xin | (uintptr_t)Xout | (uintptr_t)I | (uintptr_t)Xnext | (uintptr_t)Inext |
@@ -489,11 +554,12 @@ void launch_exit_small(cudaStream_t st, const float* Xin, const float* Xout, con
   if (max_rows <= 16 && D % 4 == 0 && D / 4 <= EXD_V * (EXD_THREADS >> rshift) && aligned) {
     launch_k(exit_decode_kernel, 1, EXD_THREADS, 0, st, Xin, Xout, I, first, D, ctr, par, row_tok, row_tok_next, forced,
              layer, n_layers, delta_p, test, sim, exit_tok, exit_layer_out, Xnext, Inext, hsm_s, hsm_prev, hsm_I,
-             rshift, err);
-    return;
+             rshift, max_rows, xhat_next, smode, seps, err);
+    return true;
   }
   launch_k(exit_small_kernel, 1, 256, 0, st, Xin, Xout, I, first, D, ctr, par, row_tok, row_tok_next, forced, layer,
            n_layers, delta_p, test, sim, exit_tok, exit_layer_out, Xnext, Inext, hsm_s, hsm_prev, hsm_I, err);
+  return false;
 }
 
 __global__ void set_float_kernel(float* p, float v) {
@@ -789,13 +855,13 @@ void launch_pass_init(cudaStream_t st, int n_tok, int prompt_len, int decode, in
 
 void launch_embed(cudaStream_t st, int dt, const int* tokens, int n_tok, const int* tok_pos, const void* E,
                   const void* P, const float* type_emb, const float* g, const float* b, int family, int D, int V,
-                  float eps, float* X, unsigned* err) {
+                  float eps, float* X, unsigned* err, bf16* xhat, int smode, float seps) {
   if (dt == 1)
-    launch_k(embed_kernel<bf16>, n_tok, 256, 0, st, tokens, n_tok, tok_pos, (const bf16*)E, (const bf16*)P, type_emb, g, b,
-                                              family, D, V, eps, X, err);
+    launch_k(embed_kernel<bf16>, n_tok, 256, 0, st, tokens, n_tok, tok_pos, (const bf16*)E, (const bf16*)P, type_emb, g,
+             b, family, D, V, eps, X, err, xhat, smode, seps);
   else
-    launch_k(embed_kernel<float>, n_tok, 256, 0, st, tokens, n_tok, tok_pos, (const float*)E, (const float*)P, type_emb, g,
-                                               b, family, D, V, eps, X, err);
+    launch_k(embed_kernel<float>, n_tok, 256, 0, st, tokens, n_tok, tok_pos, (const float*)E, (const float*)P, type_emb,
+             g, b, family, D, V, eps, X, err, xhat, smode, seps);
 }
 
 void launch_standardize(cudaStream_t st, int dt, const float* X, int ldx, const int* in_rows, DevRange rows,

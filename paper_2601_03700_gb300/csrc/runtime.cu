@@ -93,6 +93,8 @@ struct adept_model {
   float* logits_ws = nullptr;
   float* attn_ws = nullptr;
   int* attn_ctr = nullptr;       // generation-step attention arrival counters (zero between launches)
+  // standardisation statistics of X_out handed from the O projection to the FFN input
+  float2* tile_stats = nullptr;                // [DG_MAX_M][D / 32] (mean, M2) of X_out tiles
   float* amax_v = nullptr;       // argmax partials
   int* amax_i = nullptr;
   float* scratch = nullptr;
@@ -291,11 +293,13 @@ static void gemm(adept_model* m, cudaStream_t st, const GemmProblem* probs, int 
 }
 
 // GEMM whose A operand is the standardised rows of X (rows in_rows[r], or r; row length
-// p.K).  The generation-step GEMM standardises while it stages the operand; otherwise the
-// standardisation runs as its own launch into p.A first.
+// p.K).  The generation-step GEMM standardises while it stages the operand (with the row
+// statistics its producer computed, when given); otherwise the standardisation runs as its
+// own launch into p.A first.
 static void gemm_std(adept_model* m, cudaStream_t st, const GemmProblem& p, int max_rows, const float* X, int ldx,
-                     const int* in_rows, int mode, float eps, int cls) {
-  const DgNorm nrm{X, ldx, in_rows, mode, eps};
+                     const int* in_rows, int mode, float eps, int cls, const float2* row_stats = nullptr,
+                     const float2* tile_stats = nullptr) {
+  const DgNorm nrm{X, ldx, in_rows, mode, eps, row_stats, tile_stats};
   if (dg_takes(m, 1, p, max_rows, &nrm)) {
     cudaEvent_t b = nullptr;
     prof_begin(m, cls, st, &b);
@@ -627,6 +631,7 @@ static adept_status alloc_runtime(adept_model* m) {
   TRY(dalloc_t(m, &m->logits_ws, (size_t)c.max_batch * nout));
   TRY(dalloc_t(m, &m->attn_ws, (size_t)c.max_batch * m->H * ATTN_MAX_SPLIT * (m->dh + 2)));
   TRY(dalloc_t(m, &m->attn_ctr, (size_t)c.max_batch * m->H));
+  TRY(dalloc_t(m, &m->tile_stats, (size_t)DG_MAX_M * (m->D / 32 + 1)));
   CUDA_TRY(m, cudaMemset(m->attn_ctr, 0, sizeof(int) * c.max_batch * m->H));
   TRY(dalloc_t(m, &m->d_delta, 1));
   TRY(dalloc_t(m, &m->amax_v, (size_t)c.max_batch * 32));
@@ -751,8 +756,14 @@ static adept_status run_pass(adept_model* m, int n_tok, int batch, int prompt_le
   launch_pass_init(st, n_tok, prompt_len, decode ? 1 : 0, m->tok_seq, m->tok_pos, m->row_tok[0], m->d_seq_len,
                    m->max_blocks_per_seq * c.kv_block_tokens, fam == ADEPT_FAMILY_LLAMA ? 0 : c.max_pos,
                    m->err_word, m->ctr, ctr_words(N), sim_out, N);
+  // passes of at most DG_MAX_M rows (bf16 decoders): the producer of each layer's input
+  // (the embedding, then the exit kernel) also writes it standardised into xn, and the O
+  // projection hands the tile statistics of its output to the FFN input's GEMM
+  const bool dgrows = n_tok <= DG_MAX_M && m->dt == ADEPT_DTYPE_BF16 && m->use_dg && !m->force_simt &&
+                      fam != ADEPT_FAMILY_BERT;
   launch_embed(st, m->dt, tokens, n_tok, m->tok_pos, m->tok_emb, m->pos_emb, m->type_emb, m->emb_g, m->emb_b, fam, D,
-               m->V, eps, m->X_in[0], m->err_word);
+               m->V, eps, m->X_in[0], m->err_word, dgrows ? (bf16*)m->xn : nullptr, amode, eps);
+  bool xn_valid = dgrows;   // xn holds X_in[par] standardised
   m->launches += 2;
   const KVCacheView cv = cache_view(m);
   const int causal = fam != ADEPT_FAMILY_BERT;
@@ -789,7 +800,10 @@ static adept_status run_pass(adept_model* m, int n_tok, int batch, int prompt_le
       m->launches += 1;
       gemm(m, st, pr, 2, mrs, m->gemm_cls);
     } else {
-      gemm_std(m, st, pr[0], mr, Xi, D, nullptr, amode, eps, m->gemm_cls);
+      if (xn_valid)
+        gemm(m, st, pr, 1, mrs, m->gemm_cls);
+      else
+        gemm_std(m, st, pr[0], mr, Xi, D, nullptr, amode, eps, m->gemm_cls);
     }
     // attention over every cached position of layer i
     {
@@ -807,6 +821,12 @@ static adept_status run_pass(adept_model* m, int n_tok, int batch, int prompt_le
     p.A = m->att; p.lda = Dq; p.B = w.w_o; p.ldb = Dq; p.rows = act; p.N = D; p.K = Dq;
     p.epi = epi_base(); p.epi.kind = EPI_RESID; p.epi.bias = w.b_o; p.epi.out_f32 = m->X_out; p.epi.ld_f32 = D;
     p.epi.resid = Xi; p.epi.ld_resid = D;
+    bool ts_valid = false;   // the O projection leaves the tile statistics of X_out for the FFN input
+    if (dgrows) {
+      p.epi.tile_stats = m->tile_stats;
+      ts_valid = dg_takes(m, 1, p, mr, nullptr);
+      if (!ts_valid) p.epi.tile_stats = nullptr;
+    }
     gemm(m, st, &p, 1, &mr, m->gemm_cls);
     if (fam == ADEPT_FAMILY_BERT) {
       launch_layernorm_inplace(st, m->X_out, act, mr, D, w.ln1_g, w.ln1_b, eps);
@@ -822,7 +842,7 @@ static adept_status run_pass(adept_model* m, int n_tok, int batch, int prompt_le
       p.epi.act = fam == ADEPT_FAMILY_GPT2 ? ACT_GELU_TANH : ACT_GELU_ERF;
     }
     p.epi.bias = w.b_up; p.epi.out_t = m->hbuf; p.epi.ld_t = m->F;
-    gemm_std(m, st, p, mr, m->X_out, D, nullptr, amode, eps, m->gemm_cls);
+    gemm_std(m, st, p, mr, m->X_out, D, nullptr, amode, eps, m->gemm_cls, nullptr, ts_valid ? m->tile_stats : nullptr);
     p.A = m->hbuf; p.lda = m->F; p.B = w.w_down; p.ldb = m->F; p.N = D; p.K = m->F;
     p.epi = epi_base(); p.epi.kind = EPI_RESID; p.epi.bias = w.b_down; p.epi.out_f32 = m->X_out; p.epi.ld_f32 = D;
     p.epi.resid = m->X_out; p.epi.ld_resid = D;
@@ -835,9 +855,11 @@ static adept_status run_pass(adept_model* m, int n_tok, int batch, int prompt_le
       // exit test (Sec. 4.1) for 2 <= i <= N-1, inertia update, compaction (App. I)
       const int test = i >= 2;
       if (n_tok <= EXIT_SMALL_MAX) {
-        launch_exit_small(st, Xi, m->X_out, Ii, i == 1, D, m->ctr, par, rt, m->row_tok[par ^ 1], forced, i, N,
-                          m->d_delta, test, sim_out, m->exit_tok, exit_out, m->X_in[par ^ 1], m->I[par ^ 1], m->hsm_s,
-                          m->hsm_prev, m->hsm_I, mr, m->err_word);
+        xn_valid = launch_exit_small(st, Xi, m->X_out, Ii, i == 1, D, m->ctr, par, rt, m->row_tok[par ^ 1], forced, i,
+                                     N, m->d_delta, test, sim_out, m->exit_tok, exit_out, m->X_in[par ^ 1],
+                                     m->I[par ^ 1], m->hsm_s, m->hsm_prev, m->hsm_I, mr,
+                                     dgrows ? (bf16*)m->xn : nullptr, amode, eps, m->err_word) &&
+                   dgrows;
         m->launches += 1;
       } else {
         launch_exit_decide(st, m->X_out, Ii, D, act, mr, rt, forced, i, N, m->d_delta, test, sim_out, m->flag,
