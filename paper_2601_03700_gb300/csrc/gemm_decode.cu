@@ -37,7 +37,7 @@ constexpr int DG_BN = 32;                        // output features per tile
 constexpr int DG_KS = 128;                       // k per ring stage
 constexpr int DG_THREADS = 128;
 constexpr int DG_STAGE = DG_BN * DG_KS * 2;      // bytes per stage: two [32 rows][64 k] 128-byte-swizzled chunks
-constexpr int DG_MAX_STAGES = 6;
+constexpr int DG_MAX_STAGES = 12;
 constexpr int DG_MAX_A = 16 * 2048;              // A-slice elements a CTA holds (rows x k)
 constexpr int dg_max_kr(int mb) { return DG_MAX_A / (mb * 8); }   // k per CTA: 4096 (M <= 8), 2048
 constexpr int DG_MAX_SPLITS = 8;                 // portable cluster size
@@ -56,19 +56,16 @@ struct DgLayout {
 };
 // Offsets are relative to the ring base (the dynamic shared memory rounded up to 1024
 // bytes, as the 128-byte swizzle pattern repeats every 1024 bytes).
-constexpr DgLayout dg_layout(int stages, int mb, int kr, int xrows, int xk, int tstats, int splits) {
-  return DgLayout{stages * DG_STAGE, stages * DG_STAGE + mb * 8 * (kr + 8) * 2,
-                  stages * DG_STAGE + mb * 8 * (kr + 8) * 2 + xrows * xk * 4,
-                  stages * DG_STAGE + mb * 8 * (kr + 8) * 2 + xrows * xk * 4 + xrows * tstats * 8,
-                  stages * DG_STAGE + mb * 8 * (kr + 8) * 2 + xrows * xk * 4 + xrows * tstats * 8 +
+constexpr DgLayout dg_layout(int stages, int arows, int kr, int xrows, int xk, int tstats, int splits) {
+  return DgLayout{stages * DG_STAGE, stages * DG_STAGE + arows * (kr + 8) * 2,
+                  stages * DG_STAGE + arows * (kr + 8) * 2 + xrows * xk * 4,
+                  stages * DG_STAGE + arows * (kr + 8) * 2 + xrows * xk * 4 + xrows * tstats * 8,
+                  stages * DG_STAGE + arows * (kr + 8) * 2 + xrows * xk * 4 + xrows * tstats * 8 +
                       2 * DG_MAX_M * DG_RP * 4 + (splits - 1) * DG_MAX_M * DG_BN * 4};
 }
 constexpr int DG_MAX_TSTATS = 128;               // 32-column tiles of a row (d_model <= 4096)
-constexpr int DG_MAX_SMEM = 1024 + DG_MAX_STAGES * DG_STAGE + (DG_MAX_A + 16 * 8) * 2 + DG_XMAX_BYTES +
-                            DG_MAX_M * DG_MAX_TSTATS * 8 +
-                            2 * DG_MAX_M * DG_RP * 4 + (DG_MAX_SPLITS - 1) * DG_MAX_M * DG_BN * 4;
-constexpr int DG_STATIC_SMEM = 12 * 1024;         // static shared memory of the kernel (bound)
-static_assert(DG_MAX_SMEM + DG_STATIC_SMEM <= 227 * 1024, "shared memory budget");
+constexpr int DG_STATIC_SMEM = 12 * 1024;          // static shared memory of the kernel (bound)
+constexpr int DG_SMEM_LIMIT = 227 * 1024 - DG_STATIC_SMEM;   // dynamic shared memory of one CTA
 
 struct DgParams {
   CUtensorMap wmap;     // W as {64, N, K/64}, box {64, 32, 2}, 128-byte swizzle
@@ -178,8 +175,10 @@ __device__ __forceinline__ void ldsm_x4(uint32_t (&r)[4], uint32_t addr) {
                : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3])
                : "r"(addr));
 }
-__device__ __forceinline__ void ldsm_x2(uint32_t (&r)[2], uint32_t addr) {
-  asm volatile("ldmatrix.sync.aligned.m8n8.x2.shared.b16 {%0, %1}, [%2];" : "=r"(r[0]), "=r"(r[1]) : "r"(addr));
+__device__ __forceinline__ uint32_t ld_shared_u32(uint32_t addr) {
+  uint32_t v;
+  asm volatile("ld.shared.u32 %0, [%1];" : "=r"(v) : "r"(addr));
+  return v;
 }
 __device__ __forceinline__ void mma_bf16(float (&c)[4], const uint32_t (&a)[4], uint32_t b0, uint32_t b1) {
   asm volatile(
@@ -223,7 +222,7 @@ __global__ void __launch_bounds__(DG_THREADS, 1) gemm_decode_kernel(const __grid
   const int apitch = p.kr + 8;           // A row pitch in elements (16-byte shift per row)
   uint8_t* dg_smem = dg_smem_raw + ((1024 - (smem_u32(dg_smem_raw) & 1023)) & 1023);
   uint8_t* sW = dg_smem;                                                // [S][2][32 rows][128 B], swizzled
-  bf16* sA = reinterpret_cast<bf16*>(dg_smem + p.off_a);                // [MB*8][apitch]
+  bf16* sA = reinterpret_cast<bf16*>(dg_smem + p.off_a);                // [16 (MB 2) or max_m rows][apitch]
   float* sX = reinterpret_cast<float*>(dg_smem + p.off_x);              // [xrows][xk] (fused standardisation)
   float2* sT = reinterpret_cast<float2*>(dg_smem + p.off_t);            // [xrows][n_stiles] producer tile stats
   constexpr int SLOT = DG_MAX_M * DG_RP;
@@ -501,6 +500,9 @@ __global__ void __launch_bounds__(DG_THREADS, 1) gemm_decode_kernel(const __grid
   const int wx = wrow & 7, wu = (lane >> 4) & 1;
   const uint32_t a_base = smem_u32(sA) + ((lane & 7) + ((lane >> 4) & 1) * 8) * apitch * 2 + ((lane >> 3) & 1) * 16 +
                           kh * 128;
+  // MB == 1: lane (g, t) of the m16n8k16 B fragment reads row g, k 2t (+8) of each k16 step
+  const int bg = lane >> 2;
+  const uint32_t b_base = smem_u32(sA) + (bg * apitch + kh * 64 + (lane & 3) * 2) * 2;
   int dead = 0, g = 0;
   for (int j = 0; j < my_tiles && !dead; ++j) {
     const int f0 = (tile0 + j * tstride) * DG_BN;
@@ -520,6 +522,7 @@ __global__ void __launch_bounds__(DG_THREADS, 1) gemm_decode_kernel(const __grid
       if (ok && kh * 64 < ke) {
         const uint32_t wa = w_base + s * DG_STAGE;
         const uint32_t aa = a_base + kb * DG_KS * 2;
+        const uint32_t ab = b_base + kb * DG_KS * 2;
 #pragma unroll
         for (int kk = 0; kk < 4; ++kk) {
           uint32_t a[4];
@@ -530,9 +533,14 @@ __global__ void __launch_bounds__(DG_THREADS, 1) gemm_decode_kernel(const __grid
             mma_bf16(acc[0], a, b[0], b[1]);
             mma_bf16(acc[MB - 1], a, b[2], b[3]);
           } else {
-            uint32_t b[2];
-            ldsm_x2(b, aa + kk * 32);
-            mma_bf16(acc[0], a, b[0], b[1]);
+            // n8 block of at most 8 rows: fragment words loaded directly, rows >= M zero
+            // (the A slice holds only the launch's rows)
+            uint32_t b0 = 0u, b1 = 0u;
+            if (bg < M) {
+              b0 = ld_shared_u32(ab + kk * 32);
+              b1 = ld_shared_u32(ab + kk * 32 + 16);
+            }
+            mma_bf16(acc[0], a, b0, b1);
           }
         }
       }
@@ -658,7 +666,7 @@ cudaError_t launch_dg(cudaStream_t st, const DgParams& prm, int grid, size_t sme
   static bool attr = false;
   if (!attr) {
     const cudaError_t e = cudaFuncSetAttribute(gemm_decode_kernel<MB, KIND>,
-                                               cudaFuncAttributeMaxDynamicSharedMemorySize, DG_MAX_SMEM);
+                                               cudaFuncAttributeMaxDynamicSharedMemorySize, DG_SMEM_LIMIT);
     if (e != cudaSuccess) return e;
     attr = true;
   }
@@ -733,7 +741,6 @@ int decode_gemm(cudaStream_t st, const GemmProblem& q, int max_rows, const DgNor
   if (kr > kr_max) return -1;
   splits = cdiv(q.K, kr);
   const int nst = kr / DG_KS;
-  const int stages = std::min(DG_MAX_STAGES, nst);
   static DgParams prm;   // 64-byte-aligned tensor map; calls on a model are serialised
   memset(&prm, 0, sizeof prm);
   prm.W = (const bf16*)q.B;
@@ -752,7 +759,6 @@ int decode_gemm(cudaStream_t st, const GemmProblem& q, int max_rows, const DgNor
   prm.tiles = tiles;
   prm.splits = splits;
   prm.kr = kr;
-  prm.stages = stages;
   prm.max_m = max_rows;
   // statistics from the producer when given (only the k-slice of each row is staged),
   // else computed here from whole staged rows (or, rows too long to stage, streamed)
@@ -767,8 +773,25 @@ int decode_gemm(cudaStream_t st, const GemmProblem& q, int max_rows, const DgNor
   const bool x_ok = norm && norm->ldx % 4 == 0 && ((uintptr_t)norm->X & 15) == 0;
   prm.xrows = x_ok && (size_t)max_rows * prm.xk * 4 <= (size_t)DG_XMAX_BYTES ? max_rows : 0;
   if (prm.xrows == 0) prm.stat_mode = DG_STATS_HERE;   // the streamed path computes its own
-  const DgLayout L =
-      dg_layout(stages, mb, kr, prm.xrows, prm.xk, prm.stat_mode == DG_STATS_TILES ? prm.n_stiles : 0, splits);
+  // grid: one K-split -> persistent, two CTAs per SM streaming every tile's weights
+  // through their rings; several splits -> one CTA per (tile, split)
+  const int arows = mb == 2 ? 16 : max_rows;   // A-slice rows held in shared memory
+  const int tst = prm.stat_mode == DG_STATS_TILES ? prm.n_stiles : 0;
+  int grid = tiles * splits, per_sm = std::min(4, cdiv(grid, g_dg_sms));
+  if (splits == 1) {
+    per_sm = 2;
+    grid = std::min(tiles, per_sm * g_dg_sms);
+  }
+  // ring stages: as many as the CTAs resident on an SM leave room for (at most the CTA's
+  // stage count), so that the weight bytes in flight cover the memory latency
+  const int cta_stages = cdiv(tiles, grid / splits) * nst;
+  const int fixed = dg_layout(0, arows, kr, prm.xrows, prm.xk, tst, splits).total + 1024;
+  int stages = (227 * 1024 / per_sm - DG_STATIC_SMEM - fixed) / DG_STAGE;
+  stages = std::max(1, std::min(stages, std::min(DG_MAX_STAGES, cta_stages)));
+  const DgLayout L = dg_layout(stages, arows, kr, prm.xrows, prm.xk, tst, splits);
+  const size_t smem = (size_t)L.total + 1024;   // + slack to align the ring to 1024 bytes
+  if (smem > (size_t)DG_SMEM_LIMIT) return -1;
+  prm.stages = stages;
   prm.off_a = L.off_a;
   prm.off_x = L.off_x;
   prm.off_t = L.off_t;
@@ -777,19 +800,11 @@ int decode_gemm(cudaStream_t st, const GemmProblem& q, int max_rows, const DgNor
   prm.resid_aligned = ((uintptr_t)q.epi.resid & 15) == 0 && q.epi.ld_resid % 4 == 0;
   prm.epi = q.epi;
   prm.err = err;
-  const size_t smem = (size_t)L.total + 1024;   // + slack to align the ring to 1024 bytes
   if (!tc_encode_weight_3d(&prm.wmap, q.B, q.K, q.N, (size_t)q.ldb * 2, DG_BN, DG_KS / 64)) return -1;
-  // one K-split: a persistent grid (as many CTAs as fit on the GPU at once) streams every
-  // tile's weights through each CTA's ring; several splits: one CTA per (tile, split)
-  int grid = tiles * splits;
-  if (splits == 1) {
-    const int per_sm = std::max(1, std::min(4, (227 * 1024) / ((int)smem + DG_STATIC_SMEM + 1024)));
-    grid = std::min(tiles, per_sm * g_dg_sms);
-  }
   // a CTA whose stages fit the ring issues them all before the grid-dependency wait; a
   // longer one (large models) only its first, which bounds the weight traffic of a layer
   // whose rows have all left
-  prm.pre = cdiv(tiles, grid / splits) * nst <= stages ? stages : 1;
+  prm.pre = cta_stages <= stages ? stages : 1;
   const cudaError_t e = mb == 2 ? launch_kind<2>(st, prm, grid, smem) : launch_kind<1>(st, prm, grid, smem);
   return e == cudaSuccess ? 1 : -1;
 }
