@@ -476,6 +476,16 @@ __device__ __forceinline__ bool ad_try_wait(uint64_t* bar, uint32_t parity) {
       : "memory");
   return ok != 0;
 }
+__device__ __forceinline__ bool ad_try_wait_cluster(uint64_t* bar) {
+  uint32_t ok;
+  asm volatile(
+      "{\n.reg .pred p;\nmbarrier.try_wait.parity.acquire.cluster.shared::cta.b64 p, [%1], 0;\nselp.u32 %0, 1, 0, "
+      "p;\n}\n"
+      : "=r"(ok)
+      : "r"(ad_smem_u32(bar))
+      : "memory");
+  return ok != 0;
+}
 __device__ __forceinline__ bool ad_wait(uint64_t* bar, unsigned* err) {
   if (ad_try_wait(bar, 0)) return true;
   const long long t0 = clock64();
@@ -488,7 +498,11 @@ __device__ __forceinline__ bool ad_wait(uint64_t* bar, unsigned* err) {
   return true;
 }
 
-template <int DH>
+// CL: the chunks of a (row, kv head) form one thread-block cluster (n_split <= 8); every
+// CTA pushes its chunk partials into the rank-0 CTA's shared memory (st.async, completing
+// on its mbarrier), which merges them; otherwise partials go through global memory and the
+// last CTA to arrive merges.
+template <int DH, bool CL>
 __global__ void __launch_bounds__(AD_THREADS)
     attn_decode_kernel(const bf16* __restrict__ q, int ld_q, DevRange rows, const int* row_tok, const int* tok_seq,
                        const int* tok_pos, const int* seq_len, KVCacheView cache, int layer0, int n_heads, int causal,
@@ -506,6 +520,8 @@ __global__ void __launch_bounds__(AD_THREADS)
   __shared__ float s_red[AD_THREADS / 32];
   __shared__ float s_o[AD_THREADS / 32][DH];
   __shared__ int s_last;
+  __shared__ __align__(8) uint64_t red_bar;   // CL leader: the other chunks' partials
+  constexpr int PW = DH + 4;                  // floats per pushed partial: o[DH], m, l, pad
 
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int Hkv = cache.n_kv_heads, group = n_heads / Hkv;
@@ -517,15 +533,23 @@ __global__ void __launch_bounds__(AD_THREADS)
   const int sq = tok_seq[tok], pos = tok_pos[tok];
   const int nk = causal ? pos + 1 : seq_len[sq];
   const int n_eff = (nk + AD_CHUNK - 1) / AD_CHUNK;   // chunks holding keys of this row
-  if (split >= n_eff) return;
-  const int k_lo = split * AD_CHUNK, nkc = min(nk - k_lo, AD_CHUNK);
+  if (!CL && split >= n_eff) return;   // (a cluster's CTAs all stay: they push empty partials)
+  const int k_lo = split * AD_CHUNK, nkc = max(0, min(nk - k_lo, AD_CHUNK));
   const int nb = (nkc + 15) >> 4;                      // cache blocks of the chunk
+  float* sPart = reinterpret_cast<float*>(ad_smem + 2 * AD_CHUNK * DH * 2);   // CL: [group][n_split][PW]
   constexpr int BLOCK_BYTES = 16 * DH * 2;
   KT_MARK(0);
 
   if (tid == 0) {
     asm volatile("mbarrier.init.shared::cta.b64 [%0], 1;" ::"r"(ad_smem_u32(&bar)) : "memory");
+    if (CL) {
+      asm volatile("mbarrier.init.shared::cta.b64 [%0], 1;" ::"r"(ad_smem_u32(&red_bar)) : "memory");
+    }
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+    if (CL && split == 0)
+      asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(ad_smem_u32(&red_bar)),
+                   "r"((uint32_t)(group * (n_split - 1) * PW * 4))
+                   : "memory");
   }
   __syncthreads();
   if (warp == 0) {
@@ -557,9 +581,13 @@ __global__ void __launch_bounds__(AD_THREADS)
   const int slot = lane / PARTS, part = lane - slot * PARTS;
   // the first query head's piece (8 dims per lane), fetched while the cache blocks are in flight
   uint4 qraw = *reinterpret_cast<const uint4*>(q + (size_t)r * ld_q + kvh * group * DH + part * 8);
+  // every reduction barrier of the cluster is initialised before any CTA pushes to it
+  if (CL) asm volatile("barrier.cluster.arrive.release.aligned;\nbarrier.cluster.wait.acquire.aligned;" ::: "memory");
   KT_MARK(1);
-  bool ok = ad_wait(&bar, err);
-  if (!ok) ad_wait(&bar, err);   // second bounded wait for the copies in flight; results flagged
+  if (nb > 0) {
+    bool ok = ad_wait(&bar, err);
+    if (!ok) ad_wait(&bar, err);   // second bounded wait for the copies in flight; results flagged
+  }
   KT_MARK(2);
 
 #pragma unroll 1
@@ -662,8 +690,38 @@ __global__ void __launch_bounds__(AD_THREADS)
       for (int i = 0; i < 8; ++i) s_o[warp][part * 8 + i] = o[i];
     }
     __syncthreads();
-    // chunk partial -> workspace [(row, head), split]: o[DH], m, l
     const int rh = rrel * n_heads + h;
+    if (CL) {
+      // chunk partial (empty chunk: m = -inf, l = 0, o = 0) -> slot [g][split] of the leader
+      float* slot = sPart + ((size_t)g * n_split + split) * PW;
+      for (int q4 = tid; q4 < PW / 4; q4 += AD_THREADS) {
+        float4 v;
+        float* vv = reinterpret_cast<float*>(&v);
+#pragma unroll
+        for (int c = 0; c < 4; ++c) {
+          const int d = q4 * 4 + c;
+          vv[c] = nkc == 0 ? (d == DH ? -INFINITY : 0.f)
+                           : d < DH ? s_o[0][d] + s_o[1][d] + s_o[2][d] + s_o[3][d]
+                           : d == DH ? M
+                           : d == DH + 1 ? s_red[0] + s_red[1] + s_red[2] + s_red[3]
+                                         : 0.f;
+        }
+        if (split == 0) {
+          *reinterpret_cast<float4*>(slot + q4 * 4) = v;
+        } else {
+          uint32_t rd, rbar;
+          asm volatile("mapa.shared::cluster.u32 %0, %1, 0;" : "=r"(rd) : "r"(ad_smem_u32(slot + q4 * 4)));
+          asm volatile("mapa.shared::cluster.u32 %0, %1, 0;" : "=r"(rbar) : "r"(ad_smem_u32(&red_bar)));
+          asm volatile(
+              "st.async.shared::cluster.mbarrier::complete_tx::bytes.v4.f32 [%0], {%1, %2, %3, %4}, [%5];" ::"r"(rd),
+              "f"(v.x), "f"(v.y), "f"(v.z), "f"(v.w), "r"(rbar)
+              : "memory");
+        }
+      }
+      __syncthreads();   // s_p / s_o / s_red reused by the next head of the group
+      continue;
+    }
+    // chunk partial -> workspace [(row, head), split]: o[DH], m, l
     float* w = ws + ((size_t)rh * n_split + split) * (DH + 2);
     for (int d = tid; d < DH; d += AD_THREADS) w[d] = s_o[0][d] + s_o[1][d] + s_o[2][d] + s_o[3][d];
     if (tid == 0) {
@@ -717,10 +775,40 @@ __global__ void __launch_bounds__(AD_THREADS)
     }
     __syncthreads();   // s_p / s_o / s_red reused by the next head of the group
   }
+  if (CL && split == 0) {
+    // leader: every chunk's partial is in shared memory -> merge in chunk order per head
+    bool ok = false;
+    {
+      const long long t0 = clock64();
+      while (!(ok = ad_try_wait_cluster(&red_bar))) {
+        if (clock64() - t0 > 16 * AD_TIMEOUT_CYCLES) {
+          atomicOr(err, ERRW_TIMEOUT);
+          break;
+        }
+      }
+    }
+    if (!ok) return;
+    for (int g = 0; g < group; ++g) {
+      const int h = kvh * group + g;
+      const float* sl = sPart + (size_t)g * n_split * PW;
+      float Mg = -INFINITY;
+      for (int c = 0; c < n_split; ++c) Mg = fmaxf(Mg, sl[c * PW + DH]);
+      float L = 0.f, acc = 0.f;
+      const int d = tid;
+      for (int c = 0; c < n_split; ++c) {
+        const float m = sl[c * PW + DH];
+        if (m == -INFINITY) continue;
+        const float sc = exp2f(m - Mg);
+        L += sc * sl[c * PW + DH + 1];
+        if (d < DH) acc += sc * sl[c * PW + d];
+      }
+      if (d < DH) out[(size_t)r * ld_out + h * DH + d] = __float2bfloat16_rn(L > 0.f ? acc / L : 0.f);
+    }
+  }
 }
 
 static int g_attn_smem_set[2] = {0, 0};
-static int g_ad_smem_set[2] = {0, 0};
+static int g_ad_smem_set[4] = {0, 0, 0, 0};
 
 void launch_attention(cudaStream_t st, int dt, const void* q, int ld_q, void* out, int ld_out, DevRange rows,
                       int max_rows, const int* row_tok, const int* tok_seq, const int* tok_pos, const int* seq_len,
@@ -735,24 +823,43 @@ void launch_attention(cudaStream_t st, int dt, const void* q, int ld_q, void* ou
       ld_q % 8 == 0 && ((uintptr_t)q & 15) == 0) {
     const int n_split = (decode_keys + AD_CHUNK - 1) / AD_CHUNK;
     const dim3 grid(max_rows * cache.n_kv_heads, n_split);
-    const int smem = 2 * AD_CHUNK * dh * 2;
-    if (dh == 64) {
-      if (!g_ad_smem_set[0]) {
-        cudaFuncSetAttribute(attn_decode_kernel<64>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
-        g_ad_smem_set[0] = 1;
-      }
-      launch_k(attn_decode_kernel<64>, grid, AD_THREADS, smem, st, (const bf16*)q, ld_q, rows, row_tok, tok_seq,
-               tok_pos, seq_len, cache, layer0, n_heads, causal, scale_log2, n_split, ws, counters, (bf16*)out, ld_out,
-               err);
-    } else {
-      if (!g_ad_smem_set[1]) {
-        cudaFuncSetAttribute(attn_decode_kernel<128>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
-        g_ad_smem_set[1] = 1;
-      }
-      launch_k(attn_decode_kernel<128>, grid, AD_THREADS, smem, st, (const bf16*)q, ld_q, rows, row_tok, tok_seq,
-               tok_pos, seq_len, cache, layer0, n_heads, causal, scale_log2, n_split, ws, counters, (bf16*)out, ld_out,
-               err);
+    const int group = n_heads / cache.n_kv_heads;
+    const bool cl = n_split > 1 && n_split <= 8;   // chunks of a (row, kv head) merged in a cluster
+    const int smem = 2 * AD_CHUNK * dh * 2 + (cl ? group * n_split * (dh + 4) * 4 : 0);
+    const int vi = (dh == 64 ? 0 : 2) + (cl ? 1 : 0);
+    void (*kern)(const bf16*, int, DevRange, const int*, const int*, const int*, const int*, KVCacheView, int, int, int,
+                 float, int, float*, int*, bf16*, int, unsigned*) =
+        vi == 0 ? attn_decode_kernel<64, false>
+        : vi == 1 ? attn_decode_kernel<64, true>
+        : vi == 2 ? attn_decode_kernel<128, false>
+                  : attn_decode_kernel<128, true>;
+    if (g_ad_smem_set[vi] < smem) {
+      cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+      g_ad_smem_set[vi] = smem;
     }
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = grid;
+    cfg.blockDim = dim3(AD_THREADS);
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = st;
+    cudaLaunchAttribute at[2];
+    int na = 0;
+    if (cl) {
+      at[na].id = cudaLaunchAttributeClusterDimension;
+      at[na].val.clusterDim.x = 1;
+      at[na].val.clusterDim.y = n_split;
+      at[na].val.clusterDim.z = 1;
+      ++na;
+    }
+    if (g_pdl) {
+      at[na].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+      at[na].val.programmaticStreamSerializationAllowed = 1;
+      ++na;
+    }
+    cfg.attrs = at;
+    cfg.numAttrs = na;
+    cudaLaunchKernelEx(&cfg, kern, (const bf16*)q, ld_q, rows, row_tok, tok_seq, tok_pos, seq_len, cache, layer0, n_heads,
+                       causal, scale_log2, n_split, ws, counters, (bf16*)out, ld_out, err);
     return;
   }
   if (decode_keys > 0 && ws && (dh == 64 || dh == 128)) {

@@ -75,9 +75,12 @@ def test_tiny_fp32_forced_exits_and_hsm_identity():
 
 # --------------------------------------------------------------------------- bf16 families
 
-@pytest.mark.parametrize("family", [synth.LLAMA, synth.GPT2, synth.BERT])
+@pytest.mark.parametrize("family", [synth.LLAMA, synth.GPT2, synth.BERT, "llama_gqa"])
 def test_bf16_families_forced(family):
-    kw = dict(n_heads=2, head_dim=128) if family == synth.LLAMA else {}
+    if family == "llama_gqa":   # grouped-query attention: 4 query heads share 2 KV heads
+        family, kw = synth.LLAMA, dict(n_heads=4, n_kv_heads=2, head_dim=64)
+    else:
+        kw = dict(n_heads=2, head_dim=128) if family == synth.LLAMA else {}
     cfg = small(family, **kw)
     pair = Pair(cfg, seed=3)
     B, P = 3, 70
