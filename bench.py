@@ -588,9 +588,58 @@ def kernel_case_llama_prefill(device):
     m.close()
 
 
+def kernel_case_gpt2_decode(device):
+    """The benchmark workload's prompt pass (8 x 512) and 8 generation steps (graph replay
+    from the second), for launch-list captures of the generation step: the launches of
+    one step are printed, the last steps are the ones to capture."""
+    import paper_2601_03700_gb300 as adept
+    adept.load_library()
+    cfg = workload_cfg()
+    W = synth.make_weights(cfg, seed=0, device=device)
+    m = adept.Model(cfg, W)
+    del W
+    tok = synth.make_tokens(0, B, P, cfg.vocab).to(device)
+    fp = synth.forced_exits_uniform(0, B * P, LO, HI, name="forced_prompt").view(B, P).to(device)
+    fd = synth.forced_exits_uniform(0, STEPS * B, LO, HI, name="forced_decode").view(STEPS, B).to(device)
+    nxt = torch.empty(9, B, dtype=torch.int32, device=device)
+    adept.adept_prefill(m.h, B, P, tok.view(-1), DELTA, fp.view(-1), None, None, nxt[0], None)
+    adept.adept_launch_count(m.h)
+    for s in range(8):
+        adept.adept_decode_step(m.h, B, nxt[s], DELTA, fd[s], None, None, nxt[s + 1], None)
+    torch.cuda.synchronize()
+    m.check()
+    print(json.dumps({"kernel_case": "gpt2_decode", "steps": 8, "launches_per_step": adept.adept_launch_count(m.h) // 8}))
+    m.close()
+
+
+def kernel_case_llama_decode_small(device):
+    """Generation steps at Llama-2-7B layer shapes (D=4096, 32 heads x 128, SwiGLU 11008) with
+    2 layers, a 1024-token vocabulary and a small HSM, batch 1, 64-token prompt, 4 steps:
+    about 1 GB on the device; each layer's weights (404 MB) exceed L2, so the decode GEMMs'
+    DRAM counters are meaningful in a kernel capture."""
+    import paper_2601_03700_gb300 as adept
+    adept.load_library()
+    cfg = synth.llama7b_config(n_layers=2, vocab=1024, hsm_m1=512, hsm_m2=512, max_batch=1, max_seq=128,
+                               max_pass_tokens=64)
+    W = synth.make_weights(cfg, seed=0, device=device)
+    m = adept.Model(cfg, W)
+    del W
+    tok = synth.make_tokens(0, 1, 64, cfg.vocab).to(device)
+    nxt = torch.empty(5, 1, dtype=torch.int32, device=device)
+    full = torch.full((64,), 2, dtype=torch.int32, device=device)
+    adept.adept_prefill(m.h, 1, 64, tok.view(-1), DELTA, full, None, None, nxt[0], None)
+    for s in range(4):
+        adept.adept_decode_step(m.h, 1, nxt[s], DELTA, full[:1], None, None, nxt[s + 1], None)
+    torch.cuda.synchronize()
+    m.check()
+    print(json.dumps({"kernel_case": "llama_decode_small", "steps": 4, "ok": True}))
+    m.close()
+
+
 def main():
     ap = argparse.ArgumentParser()
-    ap.add_argument("--kernel-case", default=None, choices=["fill_small", "llama_prefill"])
+    ap.add_argument("--kernel-case", default=None,
+                    choices=["fill_small", "llama_prefill", "gpt2_decode", "llama_decode_small"])
     ap.add_argument("--gpus", type=int, default=1)
     ap.add_argument("--steps", type=int, default=5)
     ap.add_argument("--warmup", type=int, default=3)
@@ -607,6 +656,12 @@ def main():
         return
     if args.kernel_case == "llama_prefill":
         kernel_case_llama_prefill(torch.device("cuda", 0))
+        return
+    if args.kernel_case == "gpt2_decode":
+        kernel_case_gpt2_decode(torch.device("cuda", 0))
+        return
+    if args.kernel_case == "llama_decode_small":
+        kernel_case_llama_decode_small(torch.device("cuda", 0))
         return
     world = int(os.environ.get("WORLD_SIZE", "1"))
     rank = int(os.environ.get("RANK", "0"))

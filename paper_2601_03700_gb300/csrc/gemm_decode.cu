@@ -773,20 +773,24 @@ int decode_gemm(cudaStream_t st, const GemmProblem& q, int max_rows, const DgNor
   const bool x_ok = norm && norm->ldx % 4 == 0 && ((uintptr_t)norm->X & 15) == 0;
   prm.xrows = x_ok && (size_t)max_rows * prm.xk * 4 <= (size_t)DG_XMAX_BYTES ? max_rows : 0;
   if (prm.xrows == 0) prm.stat_mode = DG_STATS_HERE;   // the streamed path computes its own
-  // grid: one K-split -> persistent, two CTAs per SM streaming every tile's weights
-  // through their rings; several splits -> one CTA per (tile, split)
+  // grid: one K-split -> persistent CTAs streaming their tiles' weights through their
+  // rings; several splits -> one CTA per (tile, split)
   const int arows = mb == 2 ? 16 : max_rows;   // A-slice rows held in shared memory
   const int tst = prm.stat_mode == DG_STATS_TILES ? prm.n_stiles : 0;
-  int grid = tiles * splits, per_sm = std::min(4, cdiv(grid, g_dg_sms));
+  const int fixed0 = dg_layout(0, arows, kr, prm.xrows, prm.xk, tst, splits).total + 1024;
+  int grid = tiles * splits;
   if (splits == 1) {
-    per_sm = 2;
-    grid = std::min(tiles, per_sm * g_dg_sms);
+    // as many CTAs as can be resident with a ring of at least four stages, each with the
+    // same number of tiles (so that no CTA streams a tile while the others idle)
+    const int cap = std::max(1, std::min(4, (227 * 1024) / (fixed0 + 4 * DG_STAGE + DG_STATIC_SMEM))) * g_dg_sms;
+    const int per_cta = cdiv(tiles, cap);
+    grid = cdiv(tiles, per_cta);
   }
+  const int per_sm = std::min(4, cdiv(grid, g_dg_sms));
   // ring stages: as many as the CTAs resident on an SM leave room for (at most the CTA's
   // stage count), so that the weight bytes in flight cover the memory latency
   const int cta_stages = cdiv(tiles, grid / splits) * nst;
-  const int fixed = dg_layout(0, arows, kr, prm.xrows, prm.xk, tst, splits).total + 1024;
-  int stages = (227 * 1024 / per_sm - DG_STATIC_SMEM - fixed) / DG_STAGE;
+  int stages = (227 * 1024 / per_sm - DG_STATIC_SMEM - fixed0) / DG_STAGE;
   stages = std::max(1, std::min(stages, std::min(DG_MAX_STAGES, cta_stages)));
   const DgLayout L = dg_layout(stages, arows, kr, prm.xrows, prm.xk, tst, splits);
   const size_t smem = (size_t)L.total + 1024;   // + slack to align the ring to 1024 bytes
