@@ -19,6 +19,8 @@ What it follows (paper sections / equations / tables):
   for every r > i*, the K/V of layer r are layer r's K/V projection of the mapped
   state s~_N, computed directly from s~_N (no sequential unfolding).
 * Dynamic shrinkage (App. I): each layer runs only on the still-active tokens.
+* Threshold calibration (Sec. 4.1, Sec. 5.1): bisection on delta to a target reduction
+  in computation (RDC) over a calibration batch.
 
 Readings where the paper is silent (each one is also listed in the design notes):
 
@@ -434,6 +436,45 @@ def decode_step(m: OracleModel, cache: OracleCache, tokens: np.ndarray, delta: f
     res.logits = m.lm_logits(res.final)
     res.next_token = np.argmax(res.logits, axis=-1)
     return res
+
+
+def reduction_in_computation(exit_layer: np.ndarray, n_layers: int) -> float:
+    """RDC, the reduction in computation the paper reports (Sec. 5.1, Tables 3-5): the
+    fraction of the T x N layer evaluations of a pass that early exit skips,
+    1 - (sum_j depth_j) / (T N), where depth_j = i*_j is token j's exit layer."""
+    e = np.asarray(exit_layer, dtype=np.float64).reshape(-1)
+    return 1.0 - float(np.sum(e)) / (len(e) * n_layers)
+
+
+def calibrate_threshold(m: OracleModel, tokens: np.ndarray, target_rdc: float, lo: float = -1.0,
+                        hi: float = 1.0, max_iter: int = 24, tol: float = 0.005, hsm_mode: str = "hsm"):
+    """Threshold calibration (Sec. 4.1: delta is set to meet the computation budget
+    C_threshold; Sec. 5.1): bisection on delta over the prompt pass of a calibration
+    batch until its RDC is within tol of target_rdc.
+
+    A higher delta asks for a closer alignment before a token may leave, so fewer tokens
+    leave and the RDC falls: when the batch's RDC is above the target, the threshold
+    moves up (lo = delta), otherwise down (hi = delta).  The midpoints are dyadic
+    fractions of [lo, hi], exact in float32 for the first 24 steps.  Returns
+    (delta, rdc, [(delta, rdc) of every pass])."""
+    tokens = np.asarray(tokens)
+    B, P = tokens.shape
+    N = m.cfg.n_layers
+    hist = []
+    delta = rdc = None
+    for _ in range(max_iter):
+        delta = 0.5 * (lo + hi)
+        cache = OracleCache(m.cfg, B, P)
+        res = prefill(m, cache, tokens, delta, hsm_mode=hsm_mode)
+        rdc = reduction_in_computation(res.exit_layer, N)
+        hist.append((delta, rdc))
+        if abs(rdc - target_rdc) <= tol:
+            break
+        if rdc > target_rdc:
+            lo = delta
+        else:
+            hi = delta
+    return delta, rdc, hist
 
 
 def skip_kv_fill(m: OracleModel, mapped: np.ndarray, exit_layer: np.ndarray, pos: np.ndarray):

@@ -34,9 +34,9 @@ namespace adept {
 namespace {
 
 constexpr int DG_BN = 32;                        // output features per tile
-constexpr int DG_KS = 128;                       // k per ring stage
+constexpr int DG_KS = 128;                       // k per ring stage of a short k-range (larger: 256)
 constexpr int DG_THREADS = 128;
-constexpr int DG_STAGE = DG_BN * DG_KS * 2;      // bytes per stage: two [32 rows][64 k] 128-byte-swizzled chunks
+constexpr int DG_CHUNK = DG_BN * 128;            // bytes of one [32 rows][64 k] 128-byte-swizzled chunk
 constexpr int DG_MAX_STAGES = 12;
 constexpr int DG_MAX_A = 16 * 2048;              // A-slice elements a CTA holds (rows x k)
 constexpr int dg_max_kr(int mb) { return DG_MAX_A / (mb * 8); }   // k per CTA: 4096 (M <= 8), 2048
@@ -56,12 +56,11 @@ struct DgLayout {
 };
 // Offsets are relative to the ring base (the dynamic shared memory rounded up to 1024
 // bytes, as the 128-byte swizzle pattern repeats every 1024 bytes).
-constexpr DgLayout dg_layout(int stages, int arows, int kr, int xrows, int xk, int tstats, int splits) {
-  return DgLayout{stages * DG_STAGE, stages * DG_STAGE + arows * (kr + 8) * 2,
-                  stages * DG_STAGE + arows * (kr + 8) * 2 + xrows * xk * 4,
-                  stages * DG_STAGE + arows * (kr + 8) * 2 + xrows * xk * 4 + xrows * tstats * 8,
-                  stages * DG_STAGE + arows * (kr + 8) * 2 + xrows * xk * 4 + xrows * tstats * 8 +
-                      2 * DG_MAX_M * DG_RP * 4 + (splits - 1) * DG_MAX_M * DG_BN * 4};
+constexpr DgLayout dg_layout(int ring, int arows, int kr, int xrows, int xk, int tstats, int splits) {
+  return DgLayout{ring, ring + arows * (kr + 8) * 2, ring + arows * (kr + 8) * 2 + xrows * xk * 4,
+                  ring + arows * (kr + 8) * 2 + xrows * xk * 4 + xrows * tstats * 8,
+                  ring + arows * (kr + 8) * 2 + xrows * xk * 4 + xrows * tstats * 8 + 2 * DG_MAX_M * DG_RP * 4 +
+                      (splits - 1) * DG_MAX_M * DG_BN * 4};
 }
 constexpr int DG_MAX_TSTATS = 128;               // 32-column tiles of a row (d_model <= 4096)
 constexpr int DG_STATIC_SMEM = 12 * 1024;          // static shared memory of the kernel (bound)
@@ -83,7 +82,8 @@ struct DgParams {
   int N, K;
   int tiles;    // 32-feature tiles
   int splits;   // CTAs per tile (= cluster size)
-  int kr;       // k per split (a multiple of DG_KS; the last split may be shorter)
+  int kr;       // k per split (a multiple of ks; the last split may be shorter)
+  int ks;       // k per ring stage: 128 or 256 (stage = ks / 64 swizzled chunks)
   int stages;   // ring stages
   int pre;      // stages issued before the grid-dependency wait
   int max_m;    // rows the launch was sized for
@@ -216,7 +216,8 @@ __global__ void __launch_bounds__(DG_THREADS, 1) gemm_decode_kernel(const __grid
   const int my_tiles = (p.tiles - tile0 + tstride - 1) / tstride;
   const int k_lo = split * p.kr;
   const int kr = min(p.K - k_lo, p.kr);
-  const int nst = (kr + DG_KS - 1) / DG_KS;   // stages per tile
+  const int ks = p.ks, stage_bytes = ks * DG_BN * 2;
+  const int nst = (kr + ks - 1) / ks;   // stages per tile
   const int G = my_tiles * nst;               // stages of this CTA
   const int S = p.stages;
   const int apitch = p.kr + 8;           // A row pitch in elements (16-byte shift per row)
@@ -248,8 +249,8 @@ __global__ void __launch_bounds__(DG_THREADS, 1) gemm_decode_kernel(const __grid
     const int j = g / nst, kb = g - j * nst;
     const int f = (tile0 + j * tstride) * DG_BN;
     const int s = g % S;
-    mbar_expect_tx(&full[s], (uint32_t)DG_STAGE);
-    tma_load_3d(&p.wmap, &full[s], sW + (size_t)s * DG_STAGE, f, (k_lo + kb * DG_KS) >> 6);
+    mbar_expect_tx(&full[s], (uint32_t)stage_bytes);
+    tma_load_3d(&p.wmap, &full[s], sW + (size_t)s * stage_bytes, f, (k_lo + kb * ks) >> 6);
   };
   const int first = min(S, G);
   const int pre = min(p.pre, first);
@@ -496,7 +497,7 @@ __global__ void __launch_bounds__(DG_THREADS, 1) gemm_decode_kernel(const __grid
   // weight fragment rows of this lane; k-chunk kh of the stage; 16-byte unit u of a
   // 128-byte row sits at (u ^ (row & 7)) * 16
   const int wrow = mb * 16 + (lane & 7) + ((lane >> 3) & 1) * 8;
-  const uint32_t w_base = smem_u32(sW) + kh * (DG_BN * 128) + wrow * 128;
+  const uint32_t w_base = smem_u32(sW) + kh * DG_CHUNK + wrow * 128;
   const int wx = wrow & 7, wu = (lane >> 4) & 1;
   const uint32_t a_base = smem_u32(sA) + ((lane & 7) + ((lane >> 4) & 1) * 8) * apitch * 2 + ((lane >> 3) & 1) * 16 +
                           kh * 128;
@@ -518,11 +519,12 @@ __global__ void __launch_bounds__(DG_THREADS, 1) gemm_decode_kernel(const __grid
 #ifdef ADEPT_KTRACE
       KT_ADD(7, kt_now() - tw);
 #endif
-      const int ke = min(DG_KS, kr - kb * DG_KS);
-      if (ok && kh * 64 < ke) {
-        const uint32_t wa = w_base + s * DG_STAGE;
-        const uint32_t aa = a_base + kb * DG_KS * 2;
-        const uint32_t ab = b_base + kb * DG_KS * 2;
+      // warp (mb, kh) takes the stage's 64-k chunks kh, kh + 2, ...
+      const int nch = min(ks, kr - kb * ks) >> 6;
+      for (int q = 0; ok && 2 * q + kh < nch; ++q) {
+        const uint32_t wa = w_base + s * stage_bytes + q * (2 * DG_CHUNK);
+        const uint32_t aa = a_base + (kb * ks + q * 128) * 2;
+        const uint32_t ab = b_base + (kb * ks + q * 128) * 2;
 #pragma unroll
         for (int kk = 0; kk < 4; ++kk) {
           uint32_t a[4];
@@ -737,10 +739,13 @@ int decode_gemm(cudaStream_t st, const GemmProblem& q, int max_rows, const DgNor
   // at most kr_max of k
   int splits = std::max(cdiv(2 * g_dg_sms, tiles), cdiv(q.K, kr_max));
   splits = std::min(splits, std::min(DG_MAX_SPLITS, cdiv(q.K, DG_KS)));
-  const int kr = cdiv(cdiv(q.K, splits), DG_KS) * DG_KS;
+  // long k-ranges stage 256 k per row (512 contiguous bytes of each weight row per copy)
+  const int ks = cdiv(q.K, splits) >= 1024 ? 2 * DG_KS : DG_KS;
+  const int kr = cdiv(cdiv(q.K, splits), ks) * ks;
   if (kr > kr_max) return -1;
   splits = cdiv(q.K, kr);
-  const int nst = kr / DG_KS;
+  const int nst = kr / ks;
+  const int stage_bytes = ks * DG_BN * 2;
   static DgParams prm;   // 64-byte-aligned tensor map; calls on a model are serialised
   memset(&prm, 0, sizeof prm);
   prm.W = (const bf16*)q.B;
@@ -759,6 +764,7 @@ int decode_gemm(cudaStream_t st, const GemmProblem& q, int max_rows, const DgNor
   prm.tiles = tiles;
   prm.splits = splits;
   prm.kr = kr;
+  prm.ks = ks;
   prm.max_m = max_rows;
   // statistics from the producer when given (only the k-slice of each row is staged),
   // else computed here from whole staged rows (or, rows too long to stage, streamed)
@@ -782,7 +788,7 @@ int decode_gemm(cudaStream_t st, const GemmProblem& q, int max_rows, const DgNor
   if (splits == 1) {
     // as many CTAs as can be resident with a ring of at least four stages, each with the
     // same number of tiles (so that no CTA streams a tile while the others idle)
-    const int cap = std::max(1, std::min(4, (227 * 1024) / (fixed0 + 4 * DG_STAGE + DG_STATIC_SMEM))) * g_dg_sms;
+    const int cap = std::max(1, std::min(4, (227 * 1024) / (fixed0 + 4 * stage_bytes + DG_STATIC_SMEM))) * g_dg_sms;
     const int per_cta = cdiv(tiles, cap);
     grid = cdiv(tiles, per_cta);
   }
@@ -790,9 +796,9 @@ int decode_gemm(cudaStream_t st, const GemmProblem& q, int max_rows, const DgNor
   // ring stages: as many as the CTAs resident on an SM leave room for (at most the CTA's
   // stage count), so that the weight bytes in flight cover the memory latency
   const int cta_stages = cdiv(tiles, grid / splits) * nst;
-  int stages = (227 * 1024 / per_sm - DG_STATIC_SMEM - fixed0) / DG_STAGE;
+  int stages = (227 * 1024 / per_sm - DG_STATIC_SMEM - fixed0) / stage_bytes;
   stages = std::max(1, std::min(stages, std::min(DG_MAX_STAGES, cta_stages)));
-  const DgLayout L = dg_layout(stages, arows, kr, prm.xrows, prm.xk, tst, splits);
+  const DgLayout L = dg_layout(stages * stage_bytes, arows, kr, prm.xrows, prm.xk, tst, splits);
   const size_t smem = (size_t)L.total + 1024;   // + slack to align the ring to 1024 bytes
   if (smem > (size_t)DG_SMEM_LIMIT) return -1;
   prm.stages = stages;
@@ -804,7 +810,7 @@ int decode_gemm(cudaStream_t st, const GemmProblem& q, int max_rows, const DgNor
   prm.resid_aligned = ((uintptr_t)q.epi.resid & 15) == 0 && q.epi.ld_resid % 4 == 0;
   prm.epi = q.epi;
   prm.err = err;
-  if (!tc_encode_weight_3d(&prm.wmap, q.B, q.K, q.N, (size_t)q.ldb * 2, DG_BN, DG_KS / 64)) return -1;
+  if (!tc_encode_weight_3d(&prm.wmap, q.B, q.K, q.N, (size_t)q.ldb * 2, DG_BN, ks / 64)) return -1;
   // a CTA whose stages fit the ring issues them all before the grid-dependency wait; a
   // longer one (large models) only its first, which bounds the weight traffic of a layer
   // whose rows have all left

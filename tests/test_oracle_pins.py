@@ -306,3 +306,61 @@ def test_synth_generator_is_deterministic_and_normal():
     assert t.min() >= 8 and t.max() <= 32 and abs(t.double().mean().item() - 23.79) < 0.15
     u = synth.forced_exits_uniform(0, 20000, 4, 12)
     assert u.min() == 4 and u.max() == 12
+
+
+# ----------------------------------------------------------------------------- threshold calibration
+
+def test_rdc_closed_forms():
+    """RDC = 1 - sum(depth) / (T N) (Sec. 5.1): every token at layer 2 -> 1 - 2/N, full
+    depth -> 0; a hand example."""
+    cfg = small_cfg(synth.GPT2, n_layers=6)
+    m, _, _ = model_and_ref(cfg, seed=41)
+    tokens = synth.make_tokens(41, 2, 7, cfg.vocab).numpy()
+    lo = O.prefill(m, O.OracleCache(cfg, 2, 8), tokens, -2.0)
+    hi = O.prefill(m, O.OracleCache(cfg, 2, 8), tokens, np.inf)
+    assert O.reduction_in_computation(lo.exit_layer, 6) == pytest.approx(1 - 2 / 6, abs=1e-15)
+    assert O.reduction_in_computation(hi.exit_layer, 6) == 0.0
+    assert O.reduction_in_computation(np.array([2, 6, 4, 4]), 8) == pytest.approx(1 - 16 / 32, abs=1e-15)
+
+
+def test_calibration_bisection_against_brute_force():
+    """Bisection on delta lands on a threshold whose prompt-pass RDC equals an attainable
+    target; the brute-force scan over a delta grid shows the RDC falling with delta (a
+    stricter threshold keeps tokens longer) and gives that target."""
+    cfg = small_cfg(synth.GPT2, n_layers=6)
+    m, _, _ = model_and_ref(cfg, seed=42, std=0.05)
+    tokens = synth.make_tokens(42, 2, 12, cfg.vocab).numpy()
+    grid = np.linspace(-1.0, 1.0, 41)
+    rdc = np.array([O.reduction_in_computation(O.prefill(m, O.OracleCache(cfg, 2, 16), tokens, d).exit_layer, 6)
+                    for d in grid])
+    assert np.all(np.diff(rdc) <= 1e-12)                      # non-increasing in delta
+    assert rdc[0] == pytest.approx(1 - 2 / 6) and rdc[-1] < rdc[0]
+    mids = [r for r in np.unique(rdc) if 0.0 < r < 1 - 2 / 6]
+    assert mids, "the scan should reach intermediate reductions"
+    target = mids[len(mids) // 2]
+    d, r, hist = O.calibrate_threshold(m, tokens, target, tol=1e-12, max_iter=30)
+    assert r == pytest.approx(target, abs=1e-12)
+    # the returned threshold reproduces the reduction in a fresh pass
+    again = O.reduction_in_computation(O.prefill(m, O.OracleCache(cfg, 2, 16), tokens, d).exit_layer, 6)
+    assert again == pytest.approx(target, abs=1e-12)
+    # bisection: each pass halves the bracket, which always holds the result
+    lo, hi = -1.0, 1.0
+    for dd, rr in hist[:-1]:
+        assert dd == pytest.approx(0.5 * (lo + hi), abs=0)
+        if rr > target:
+            lo = dd
+        else:
+            hi = dd
+    assert lo <= d <= hi
+
+
+def test_calibration_unreachable_target_ends_at_the_bound():
+    """A target above the largest attainable reduction (1 - 2/N) drives delta to the lower
+    end of the bracket, with every token leaving at layer 2."""
+    cfg = small_cfg(synth.GPT2, n_layers=6)
+    m, _, _ = model_and_ref(cfg, seed=43)
+    tokens = synth.make_tokens(43, 1, 6, cfg.vocab).numpy()
+    d, r, hist = O.calibrate_threshold(m, tokens, 0.99, lo=-1.0, hi=1.0, max_iter=12)
+    assert len(hist) == 12
+    assert d == pytest.approx(-1.0 + 2.0 ** -11, abs=1e-15)   # passes at 0, -1/2, ..., -1 + 2^-11
+    assert r == pytest.approx(1 - 2 / 6)
