@@ -463,6 +463,15 @@ def ours(args, rank, world, device):
         "exit_depth": {"prompt_mean": round(float(e_p.mean()), 3), "decode_mean": round(float(e_d.mean()), 3)},
         "clocks": clk,
     }
+    # --------------------------------------------------------------- threshold calibration (Sec. 4.1, 5.1)
+    # bisection on delta to a 25% reduction in computation over the workload's prompt batch
+    torch.cuda.synchronize()
+    t0 = time.perf_counter()
+    d_c, r_c, n_c = adept.adept_calibrate_threshold(run.m.h, B, P, run.tokens.view(-1), 0.25, 0.01, 24)
+    t_cal = (time.perf_counter() - t0) * 1e3
+    line["calibration"] = {"target_rdc": 0.25, "tol": 0.01, "delta": round(d_c, 6), "rdc": round(r_c, 4),
+                           "passes": n_c, "ms": round(t_cal, 3), "ms_per_pass": round(t_cal / max(n_c, 1), 3),
+                           "batch": f"{B} x {P} workload prompts, threshold exits"}
     run.m.close()
     del run
     torch.cuda.empty_cache()

@@ -142,6 +142,20 @@ ADEPT_API adept_status adept_decode_step(adept_model* m, int batch, const int32_
                                float* d_logits_out, int32_t* d_next_token_out, float* d_sim_out,
                                void* stream);
 
+/* Threshold calibration (Sec. 4.1: delta is set to meet the computation budget; Sec. 5.1):
+ * bisection on delta in [lo, hi] over prompt passes of the calibration batch d_tokens
+ * [batch, prompt_len] (threshold exits, no forced exits) until the batch's reduction in
+ * computation RDC = 1 - sum(exit layer) / (batch prompt_len N) is within tol of target_rdc,
+ * or max_iter passes have run.  A pass whose RDC is above the target raises the
+ * threshold (lo = delta), otherwise it lowers it (hi = delta).
+ *   delta_out, rdc_out, iters_out: host pointers (the last pass's delta and RDC, passes run)
+ * Synchronous: waits for each pass on `stream`.  Like adept_prefill it resets sequences
+ * 0..batch-1.  Errors: INVALID_ARG (target outside [0, 1), tol < 0, max_iter < 1,
+ * lo >= hi, NULL pointers), and those of adept_prefill. */
+ADEPT_API adept_status adept_calibrate_threshold(adept_model* m, int batch, int prompt_len, const int32_t* d_tokens,
+                                       float target_rdc, float tol, int max_iter, float lo, float hi,
+                                       float* delta_out, float* rdc_out, int* iters_out, void* stream);
+
 /* Decoupled skipped-layer KV fill (Eq. 6, the decoupling of Sec. 4; Eq. 9, KV
  * generation in Sec. 4.3): for every token j and every layer r = i*_j+1..N, writes layer r's
  * K = RoPE(W_K^r norm_r(s~_j) + b_K^r) and V = W_V^r norm_r(s~_j) + b_V^r into the

@@ -28,6 +28,7 @@ ABI_SYMBOLS = [
     "adept_last_error", "adept_status_string", "adept_seq_reserve", "adept_read_kv",
     "adept_read_final_states", "adept_check_device_status", "adept_set_option", "adept_profile_read",
     "adept_launch_count", "adept_skip_kv_fill_noalloc", "adept_fused_decode_batch", "adept_fused_decode_reason",
+    "adept_calibrate_threshold",
 ]
 
 
@@ -96,6 +97,10 @@ def load_library(path: str = LIB_PATH):
     lib.adept_fused_decode_batch.restype = c_int
     lib.adept_fused_decode_reason.argtypes = [vp]
     lib.adept_fused_decode_reason.restype = ctypes.c_char_p
+    lib.adept_calibrate_threshold.argtypes = [vp, c_int, c_int, i32p, c_float, c_float, c_int, c_float, c_float,
+                                              ctypes.POINTER(c_float), ctypes.POINTER(c_float),
+                                              ctypes.POINTER(c_int), st]
+    lib.adept_calibrate_threshold.restype = c_int
     for name in ABI_SYMBOLS:
         fn = getattr(lib, name)
         if fn.restype is ctypes.c_int or name in ("adept_model_load", "adept_prefill", "adept_decode_step",
@@ -201,6 +206,18 @@ def adept_skip_kv_fill_noalloc(m, n_tokens: int, h_mapped: torch.Tensor, exit_la
     lib = load_library()
     _check(lib, m, lib.adept_skip_kv_fill_noalloc(m, n_tokens, _ptr(h_mapped), _ptr(exit_layer), _ptr(seq),
                                                    _ptr(pos), _stream(stream)))
+
+
+def adept_calibrate_threshold(m, batch: int, prompt_len: int, tokens: torch.Tensor, target_rdc: float,
+                              tol: float = 0.005, max_iter: int = 24, lo: float = -1.0, hi: float = 1.0,
+                              stream=None):
+    """Bisection on the exit threshold to a target reduction in computation over the
+    calibration batch (Sec. 4.1, Sec. 5.1).  Returns (delta, rdc, passes)."""
+    lib = load_library()
+    d, r, n = ctypes.c_float(), ctypes.c_float(), ctypes.c_int()
+    _check(lib, m, lib.adept_calibrate_threshold(m, batch, prompt_len, _ptr(tokens), target_rdc, tol, max_iter, lo, hi,
+                                                 ctypes.byref(d), ctypes.byref(r), ctypes.byref(n), _stream(stream)))
+    return d.value, r.value, n.value
 
 
 def adept_free(m):

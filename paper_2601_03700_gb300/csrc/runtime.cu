@@ -93,6 +93,7 @@ struct adept_model {
   float* logits_ws = nullptr;
   float* attn_ws = nullptr;
   int* attn_ctr = nullptr;       // generation-step attention arrival counters (zero between launches)
+  int32_t* calib_exit = nullptr; // threshold calibration: exit layers of a calibration pass
   // standardisation statistics of X_out handed from the O projection to the FFN input
   float2* tile_stats = nullptr;                // [DG_MAX_M][D / 32] (mean, M2) of X_out tiles
   float* amax_v = nullptr;       // argmax partials
@@ -1165,6 +1166,43 @@ adept_status adept_decode_step(adept_model* m, int batch, const int32_t* d_token
     CUDA_TRY(m, cudaMemcpyAsync(d_sim_out, m->dec_sim, (size_t)batch * m->N * sizeof(float), cudaMemcpyDeviceToDevice,
                                 st));
   return check_launch(m);
+}
+
+adept_status adept_calibrate_threshold(adept_model* m, int batch, int prompt_len, const int32_t* d_tokens,
+                                       float target_rdc, float tol, int max_iter, float lo, float hi,
+                                       float* delta_out, float* rdc_out, int* iters_out, void* stream) {
+  if (!m) return ADEPT_ERR_INVALID_ARG;
+  if (!d_tokens || !delta_out || !rdc_out || !iters_out) return fail(m, ADEPT_ERR_INVALID_ARG, "NULL pointer");
+  if (!(target_rdc >= 0.f && target_rdc < 1.f) || !(tol >= 0.f) || max_iter < 1 || !(lo < hi))
+    return fail(m, ADEPT_ERR_INVALID_ARG, "calibration needs target in [0, 1), tol >= 0, max_iter >= 1, lo < hi");
+  if (batch < 1 || prompt_len < 1) return fail(m, ADEPT_ERR_INVALID_ARG, "batch and prompt_len must be positive");
+  const long long T = (long long)batch * prompt_len;
+  if (T > m->T_max) return fail(m, ADEPT_ERR_CAPACITY, "calibration batch above the pass workspace");
+  cudaStream_t st = (cudaStream_t)stream;
+  if (!m->calib_exit) TRY(dalloc_t(m, &m->calib_exit, (size_t)m->T_max));
+  std::vector<int32_t> ex((size_t)T);
+  float delta = lo;
+  double rdc = 0.0;
+  int it = 0;
+  while (it < max_iter) {
+    delta = 0.5f * (lo + hi);
+    TRY(adept_prefill(m, batch, prompt_len, d_tokens, delta, nullptr, m->calib_exit, nullptr, nullptr, nullptr, stream));
+    CUDA_TRY(m, cudaMemcpyAsync(ex.data(), m->calib_exit, (size_t)T * sizeof(int32_t), cudaMemcpyDeviceToHost, st));
+    TRY(adept_check_device_status(m, stream));   // synchronises the stream
+    ++it;
+    long long depth = 0;
+    for (long long j = 0; j < T; ++j) depth += ex[(size_t)j];
+    rdc = 1.0 - (double)depth / ((double)T * m->N);
+    if (std::fabs(rdc - (double)target_rdc) <= (double)tol) break;
+    if (rdc > (double)target_rdc)
+      lo = delta;
+    else
+      hi = delta;
+  }
+  *delta_out = delta;
+  *rdc_out = (float)rdc;
+  *iters_out = it;
+  return ADEPT_OK;
 }
 
 adept_status adept_skip_kv_fill(adept_model* m, int n_tokens, const void* d_h_mapped, const int32_t* d_exit_layer,

@@ -250,3 +250,42 @@ def test_generation_step_gemm_matches_tensor_core_gemm():
                 assert row_rel_err(a[1], b[1]).max() < 2e-2
                 assert row_rel_err(a[2], b[2]).max() < 2e-2
             assert row_rel_err(out[0][1], out[1][1]).max() < 2e-2
+
+
+# --------------------------------------------------------------------------- threshold calibration
+
+@pytest.mark.parametrize("dtype", ["f32", "bf16"])
+def test_threshold_calibration_matches_oracle(dtype):
+    """adept_calibrate_threshold (bisection on delta over device prompt passes) against the
+    oracle's calibration on the same model and batch: the same thresholds pass for pass
+    while no similarity of the batch falls within the +-1e-3 band of the threshold tried,
+    the target reached on both sides, and the oracle's RDC at the device's delta."""
+    from parity_utils import BAND
+    cfg = synth.tiny_config(n_layers=6) if dtype == "f32" else small(synth.GPT2, n_layers=6)
+    pair = Pair(cfg, seed=44, std=0.05)
+    B, P = 2, 24
+    tokens = synth.make_tokens(44, B, P, cfg.vocab)
+    grid = np.linspace(-1.0, 1.0, 21)
+    scan = [O.reduction_in_computation(O.prefill(pair.om, O.OracleCache(cfg, B, P), tokens.numpy(), d).exit_layer,
+                                       cfg.n_layers) for d in grid]
+    mids = sorted({r for r in scan if 0.0 < r < 1 - 2 / cfg.n_layers})
+    assert mids
+    target, tol = mids[len(mids) // 2], 0.02
+    d_o, r_o, hist = O.calibrate_threshold(pair.om, tokens.numpy(), target, tol=tol, max_iter=16)
+    d_g, r_g, n_g = adept.adept_calibrate_threshold(pair.gm.h, B, P, tokens.cuda().view(-1), target, tol, 16)
+    pair.gm.check()
+    assert abs(r_o - target) <= tol and abs(r_g - target) <= tol + 1e-6
+    # pass for pass: identical thresholds unless a similarity sat in the band of one tried
+    banded = False
+    for dd, _ in hist:
+        res = O.prefill(pair.om, O.OracleCache(cfg, B, P), tokens.numpy(), dd)
+        with np.errstate(invalid="ignore"):
+            banded |= bool(np.any(np.abs(res.sim - dd) <= BAND))
+    if not banded:
+        assert n_g == len(hist) and np.float32(d_g) == np.float32(d_o)
+    # the device's threshold gives the oracle the device's reduction (decisions agree)
+    res = O.prefill(pair.om, O.OracleCache(cfg, B, P), tokens.numpy(), d_g)
+    with np.errstate(invalid="ignore"):
+        if not np.any(np.abs(res.sim - d_g) <= BAND):
+            assert O.reduction_in_computation(res.exit_layer, cfg.n_layers) == pytest.approx(r_g, abs=1e-6)
+    pair.close()
