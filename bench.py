@@ -34,6 +34,10 @@ import torch  # noqa: E402
 import synth  # noqa: E402
 
 PEAKS_FALLBACK = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
+# DRAM bytes (read + write) per launch of a kernel class from one ncu capture of the
+# benchmark workload (profiles/launch_list_gpt2_small_generation_step.md); None once the
+# kernel has changed since the capture.
+NCU_TRAFFIC_PER_LAUNCH = {"gemm_decode": 6.38e6}
 METRIC = "early-exit prefill+decode tokens/s at 1 GB300; skipped-layer KV-fill % of roofline"
 B, P, STEPS, LO, HI, DELTA = 8, 512, 128, 4, 12, 0.9
 L2_BYTES = 129 * 2 ** 20
@@ -441,7 +445,8 @@ def ours(args, rank, world, device):
         roof = {"bound": "hbm", "achieved": round(by_s / (ms / 1e3) / 1e9, 2), "peak": peaks["hbm_gbs"],
                 "unit": "GB/s"}
     roof["frac"] = round(roof["achieved"] / roof["peak"], 4)
-    roof["traffic"] = None
+    tr = NCU_TRAFFIC_PER_LAUNCH.get(names[dom])
+    roof["traffic"] = round(tr) if tr else None
     roof["kernel"] = names[dom]
     roof["launches"] = n
     roof["peak_source"] = peaks_src + " (MEASURED_PEAKS.json burst)" if peaks_src == "measured" else peaks_src

@@ -581,8 +581,9 @@ __global__ void __launch_bounds__(AD_THREADS)
   const int slot = lane / PARTS, part = lane - slot * PARTS;
   // the first query head's piece (8 dims per lane), fetched while the cache blocks are in flight
   uint4 qraw = *reinterpret_cast<const uint4*>(q + (size_t)r * ld_q + kvh * group * DH + part * 8);
-  // every reduction barrier of the cluster is initialised before any CTA pushes to it
-  if (CL) asm volatile("barrier.cluster.arrive.release.aligned;\nbarrier.cluster.wait.acquire.aligned;" ::: "memory");
+  // the leader's reduction barrier must be initialised before any CTA pushes to it: every
+  // CTA arrives here (after the initialisation) and waits only just before its first push
+  if (CL) asm volatile("barrier.cluster.arrive.release.aligned;" ::: "memory");
   KT_MARK(1);
   if (nb > 0) {
     bool ok = ad_wait(&bar, err);
@@ -692,6 +693,7 @@ __global__ void __launch_bounds__(AD_THREADS)
     __syncthreads();
     const int rh = rrel * n_heads + h;
     if (CL) {
+      if (g == 0) asm volatile("barrier.cluster.wait.acquire.aligned;" ::: "memory");
       // chunk partial (empty chunk: m = -inf, l = 0, o = 0) -> slot [g][split] of the leader
       float* slot = sPart + ((size_t)g * n_split + split) * PW;
       for (int q4 = tid; q4 < PW / 4; q4 += AD_THREADS) {

@@ -739,8 +739,10 @@ int decode_gemm(cudaStream_t st, const GemmProblem& q, int max_rows, const DgNor
   // at most kr_max of k
   int splits = std::max(cdiv(2 * g_dg_sms, tiles), cdiv(q.K, kr_max));
   splits = std::min(splits, std::min(DG_MAX_SPLITS, cdiv(q.K, DG_KS)));
-  // long k-ranges stage 256 k per row (512 contiguous bytes of each weight row per copy)
-  const int ks = cdiv(q.K, splits) >= 1024 ? 2 * DG_KS : DG_KS;
+  // long k-ranges split over a cluster stage 256 k per row (512 contiguous bytes of each
+  // weight row per copy); a single split keeps 128 k, which leaves room for more resident
+  // CTAs of the persistent grid (measured faster at the Llama-7B QKV shape)
+  const int ks = splits > 1 && cdiv(q.K, splits) >= 1024 ? 2 * DG_KS : DG_KS;
   const int kr = cdiv(cdiv(q.K, splits), ks) * ks;
   if (kr > kr_max) return -1;
   splits = cdiv(q.K, kr);
