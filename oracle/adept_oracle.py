@@ -21,6 +21,8 @@ What it follows (paper sections / equations / tables):
 * Dynamic shrinkage (App. I): each layer runs only on the still-active tokens.
 * Threshold calibration (Sec. 4.1, Sec. 5.1): bisection on delta to a target reduction
   in computation (RDC) over a calibration batch.
+* Exit-rule variants (App. H.2-H.3): the local similarity cos(s_i, s_{i-1}), both
+  similarities, and all-at-once prompt exits decided by each sequence's last token.
 
 Readings where the paper is silent (each one is also listed in the design notes):
 
@@ -333,7 +335,8 @@ def check_forced(forced: np.ndarray, n_layers: int):
 
 def early_exit_pass(m: OracleModel, cache: OracleCache, s0: np.ndarray, seq: np.ndarray,
                     pos: np.ndarray, delta: float, forced: Optional[np.ndarray], causal: bool,
-                    kv_len: np.ndarray, hsm_mode: str = "hsm") -> PassResult:
+                    kv_len: np.ndarray, hsm_mode: str = "hsm", metric: str = "global",
+                    aao_len: int = 0) -> PassResult:
     """Run tokens (all in parallel, App. I) through layers 1..N with token-level exits.
 
     For each layer i: (a) K/V of the active tokens from their layer input go to the
@@ -341,7 +344,15 @@ def early_exit_pass(m: OracleModel, cache: OracleCache, s0: np.ndarray, seq: np.
     the exit test <s_hat_i, I_hat> >= delta (or i == forced exit layer); (d) the
     inertia takes s_hat_i; (e) each exiting token is mapped by the HSM and its K/V of
     every skipped layer r > i are produced from s~_N at once.
+
+    Variants (App. H.3, "Local vs Global Metric"; App. H.2, "All-at-Once Early-Exit"):
+    metric "local" tests cos(s_i, s_{i-1}) (s_{i-1} = the layer's input), "both" requires
+    the global and the local similarity to reach delta (the recorded similarity is then
+    their minimum); aao_len = P > 0 (prompt passes) makes every token take the decision of
+    its sequence's last prompt token (position P - 1), so a sequence leaves at once.
     """
+    if metric not in ("global", "local", "both"):
+        raise ValueError(metric)
     c = m.cfg
     N, T = c.n_layers, len(s0)
     forced = np.zeros(T, dtype=np.int64) if forced is None else np.asarray(forced, dtype=np.int64)
@@ -361,10 +372,15 @@ def early_exit_pass(m: OracleModel, cache: OracleCache, s0: np.ndarray, seq: np.
         s_new = layer_body(m, i, s[A], seq[A], pos[A], cache, causal, kv_len)   # (b)
         exits = np.zeros(len(A), dtype=bool)
         if 2 <= i <= N - 1:                                                # (c)
-            cs = cosine(s_new, inertia[A])
+            cg = cosine(s_new, inertia[A])
+            cl = cosine(s_new, s[A])
+            cs = cg if metric == "global" else cl if metric == "local" else np.minimum(cg, cl)
             sim[A, i - 1] = cs
             f = forced[A]
             exits = np.where(f > 0, f == i, cs >= delta)
+            if aao_len:
+                last = {int(seq[j]): bool(exits[k]) for k, j in enumerate(A) if pos[j] == aao_len - 1}
+                exits = np.array([last[int(seq[j])] for j in A], dtype=bool)
         I_before = inertia[A]
         inertia[A] = I_before + unit(s_new)                                # (d)
         E = A[exits]
@@ -387,7 +403,8 @@ def early_exit_pass(m: OracleModel, cache: OracleCache, s0: np.ndarray, seq: np.
 
 
 def prefill(m: OracleModel, cache: OracleCache, tokens: np.ndarray, delta: float,
-            forced: Optional[np.ndarray] = None, hsm_mode: str = "hsm") -> PassResult:
+            forced: Optional[np.ndarray] = None, hsm_mode: str = "hsm", metric: str = "global",
+            all_at_once: bool = False) -> PassResult:
     """Prompt pass for sequences 0..B-1 (resets them); tokens [B, P].
 
     Decoder: logits [B, V] of each sequence's last position and its greedy token
@@ -407,7 +424,7 @@ def prefill(m: OracleModel, cache: OracleCache, tokens: np.ndarray, delta: float
     kv_len = cache.lens.copy()
     res = early_exit_pass(m, cache, s0, seq, pos, delta,
                           None if forced is None else np.asarray(forced).reshape(-1),
-                          causal, kv_len, hsm_mode)
+                          causal, kv_len, hsm_mode, metric, P if all_at_once else 0)
     fin = res.final.reshape(B, P, -1)
     if c.family == BERT:
         res.logits = m.cls_logits(fin[:, 0])
@@ -418,7 +435,7 @@ def prefill(m: OracleModel, cache: OracleCache, tokens: np.ndarray, delta: float
 
 
 def decode_step(m: OracleModel, cache: OracleCache, tokens: np.ndarray, delta: float,
-                forced: Optional[np.ndarray] = None, hsm_mode: str = "hsm") -> PassResult:
+                forced: Optional[np.ndarray] = None, hsm_mode: str = "hsm", metric: str = "global") -> PassResult:
     """One generation step: token b of sequence b at position lens[b] (App. I, generation)."""
     c = m.cfg
     if c.family == BERT:
@@ -432,7 +449,7 @@ def decode_step(m: OracleModel, cache: OracleCache, tokens: np.ndarray, delta: f
     s0 = m.embed(tokens, pos)
     res = early_exit_pass(m, cache, s0, seq, pos, delta,
                           None if forced is None else np.asarray(forced).reshape(-1),
-                          True, kv_len, hsm_mode)
+                          True, kv_len, hsm_mode, metric)
     res.logits = m.lm_logits(res.final)
     res.next_token = np.argmax(res.logits, axis=-1)
     return res

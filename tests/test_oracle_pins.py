@@ -364,3 +364,98 @@ def test_calibration_unreachable_target_ends_at_the_bound():
     assert len(hist) == 12
     assert d == pytest.approx(-1.0 + 2.0 ** -11, abs=1e-15)   # passes at 0, -1/2, ..., -1 + 2^-11
     assert r == pytest.approx(1 - 2 / 6)
+
+
+# ----------------------------------------------------------------------------- exit-rule variants
+
+def _layer_states(ref, tokens):
+    """Full-depth states s_0..s_N of every token from the independent torch model
+    ([N + 1, B, P, D], float64)."""
+    c = ref.c
+    tokens = torch.as_tensor(tokens)
+    B, P = tokens.shape
+    pos = torch.arange(P).expand(B, P)
+    h = ref.embed(tokens, pos)
+    out = [h]
+    for i in range(1, c.n_layers + 1):
+        q = ref.q(i, h, pos).transpose(1, 2)
+        k, v = ref.kv(i, h, pos)
+        rep = c.n_heads // c.n_kv_heads
+        k = k.repeat_interleave(rep, dim=2).transpose(1, 2)
+        v = v.repeat_interleave(rep, dim=2).transpose(1, 2)
+        a = F.scaled_dot_product_attention(q, k, v, is_causal=True)
+        h = ref.after_attn(i, h, a.transpose(1, 2).flatten(-2))
+        out.append(h)
+    return torch.stack(out).numpy()
+
+
+def _cos(a, b):
+    return np.sum(a * b, -1) / (np.linalg.norm(a, axis=-1) * np.linalg.norm(b, axis=-1))
+
+
+@pytest.mark.parametrize("metric", ["global", "local", "both"])
+def test_recorded_similarities_match_full_depth_states(metric):
+    """At delta = +inf nothing leaves, so the recorded similarity at layer i (2 <= i <= N-1)
+    is the metric on the plain full-depth states: global cos(s_i, sum_{d<i} s_hat_d) (Eq. 7),
+    local cos(s_i, s_{i-1}), both their minimum."""
+    cfg = small_cfg(synth.GPT2, n_layers=6)
+    m, ref, _ = model_and_ref(cfg, seed=51)
+    tokens = synth.make_tokens(51, 2, 7, cfg.vocab).numpy()
+    S = _layer_states(ref, tokens)          # [N+1, B, P, D]
+    r = O.prefill(m, O.OracleCache(cfg, 2, 8), tokens, np.inf, metric=metric)
+    for i in range(2, cfg.n_layers):
+        inertia = sum(S[d] / np.linalg.norm(S[d], axis=-1, keepdims=True) for d in range(1, i))
+        g = _cos(S[i], inertia).reshape(-1)
+        l = _cos(S[i], S[i - 1]).reshape(-1)
+        want = g if metric == "global" else l if metric == "local" else np.minimum(g, l)
+        np.testing.assert_allclose(r.sim[:, i - 1], want, rtol=1e-10, atol=1e-12)
+
+
+@pytest.mark.parametrize("metric", ["global", "local", "both"])
+def test_single_token_sequences_exit_at_the_first_crossing(metric):
+    """A one-token sequence is computed normally until it leaves, so its exit layer is the
+    first i in [2, N-1] where its full-depth metric reaches delta (N if none)."""
+    cfg = small_cfg(synth.GPT2, n_layers=6)
+    m, ref, _ = model_and_ref(cfg, seed=52, std=0.05)
+    tokens = synth.make_tokens(52, 4, 1, cfg.vocab).numpy()
+    S = _layer_states(ref, tokens)[:, :, 0]    # [N+1, B, D]
+    probe = np.unique(O.prefill(m, O.OracleCache(cfg, 4, 2), tokens, np.inf, metric=metric).sim[:, 1:cfg.n_layers - 1])
+    # thresholds half-way between neighbouring similarities: no decision sits on a tie
+    for k in (len(probe) // 4, len(probe) // 2, 3 * len(probe) // 4):
+        delta = 0.5 * (probe[k - 1] + probe[k])
+        r = O.prefill(m, O.OracleCache(cfg, 4, 2), tokens, float(delta), metric=metric)
+        for b in range(4):
+            want = cfg.n_layers
+            for i in range(2, cfg.n_layers):
+                inertia = sum(S[d, b] / np.linalg.norm(S[d, b]) for d in range(1, i))
+                g, l = _cos(S[i, b], inertia), _cos(S[i, b], S[i - 1, b])
+                v = g if metric == "global" else l if metric == "local" else min(g, l)
+                if v >= delta:
+                    want = i
+                    break
+            assert r.exit_layer[b] == want
+
+
+def test_all_at_once_sequences_leave_with_their_last_token():
+    """All-at-once (App. H.2): every token of a sequence leaves at the layer where the
+    sequence's last prompt token first reaches delta on the full-depth states (the
+    sequence is complete until then), N if it never does."""
+    cfg = small_cfg(synth.GPT2, n_layers=6)
+    m, ref, _ = model_and_ref(cfg, seed=53, std=0.05)
+    B, P = 3, 6
+    tokens = synth.make_tokens(53, B, P, cfg.vocab).numpy()
+    S = _layer_states(ref, tokens)[:, :, P - 1]   # last token, [N+1, B, D]
+    probe = np.unique(O.prefill(m, O.OracleCache(cfg, B, P), tokens, np.inf).sim.reshape(B, P, -1)[:, P - 1,
+                                                                                                   1:cfg.n_layers - 1])
+    for k in (len(probe) // 4, 3 * len(probe) // 5):
+        delta = 0.5 * (probe[k - 1] + probe[k])
+        r = O.prefill(m, O.OracleCache(cfg, B, P), tokens, float(delta), all_at_once=True)
+        ex = r.exit_layer.reshape(B, P)
+        for b in range(B):
+            want = cfg.n_layers
+            for i in range(2, cfg.n_layers):
+                inertia = sum(S[d, b] / np.linalg.norm(S[d, b]) for d in range(1, i))
+                if _cos(S[i, b], inertia) >= delta:
+                    want = i
+                    break
+            assert np.all(ex[b] == want)
