@@ -233,9 +233,14 @@ ADEPT_API adept_status adept_check_device_status(adept_model* m, void* stream);
  * generation step of at most adept_fused_decode_batch() sequences of a bf16 decoder as
  * one persistent cooperative launch (every layer, the HSM, the fills and the head),
  * reading the caller's inputs and writing its outputs directly; 0 takes the multi-launch
- * step.  Default 0. */
+ * step.  Default 0.  EXIT_METRIC (App. H.3): 0 (default) the global similarity of Sec. 4.1,
+ * cos(s_i, sum_{d<i} s_hat_d); 1 the local similarity cos(s_i, s_{i-1}); 2 both (a token leaves
+ * when both reach delta; the reported similarity is their minimum).  ALL_AT_ONCE (App. H.2):
+ * 1 makes every token of a prompt take the exit decision of its sequence's last prompt token,
+ * so a sequence leaves at once (generation steps are unaffected: one token per sequence).
+ * Default 0. */
 enum { ADEPT_OPT_HSM_IDENTITY = 1, ADEPT_OPT_PROFILE = 2, ADEPT_OPT_GEMM_SIMT = 3, ADEPT_OPT_DECODE_GRAPH = 4,
-       ADEPT_OPT_DECODE_GEMM = 5, ADEPT_OPT_FUSED_DECODE = 6 };
+       ADEPT_OPT_DECODE_GEMM = 5, ADEPT_OPT_FUSED_DECODE = 6, ADEPT_OPT_EXIT_METRIC = 7, ADEPT_OPT_ALL_AT_ONCE = 8 };
 ADEPT_API adept_status adept_set_option(adept_model* m, int option, int value);
 
 /* Kernel classes reported by adept_profile_read: the GEMMs of prompt passes (layer

@@ -5,6 +5,9 @@
 namespace adept {
 
 // Device counter word layout of one pass.
+// Exit-test similarity (Sec. 4.1 global; App. H.3 local and both).
+enum : int { EXIT_GLOBAL = 0, EXIT_LOCAL = 1, EXIT_BOTH = 2 };
+
 enum : int {
   CTR_ACTIVE = 0,    // [0], [1]: active rows, ping-pong by layer parity
   CTR_EXITED = 2,    // exits so far in this pass
@@ -25,9 +28,14 @@ void launch_standardize(cudaStream_t st, int dt, const float* X, int ldx, const 
                         int max_rows, int D, int mode, float eps, void* out, int ld_out);
 void launch_layernorm_inplace(cudaStream_t st, float* X, DevRange rows, int max_rows, int D, const float* g,
                               const float* b, float eps);
-void launch_exit_decide(cudaStream_t st, const float* Xout, const float* I, int D, DevRange rows, int max_rows,
-                        const int* row_tok, const int* forced, int layer, int n_layers, const float* delta_p, int test,
-                        float* sim, int* flag, float* inv_norm, unsigned* err);
+// Exit decisions of the active rows.  metric: EXIT_*; Xin = the layer's input rows s_{i-1}
+// (local metric).  The exit kernels below take the same metric and aao_len: all-at-once
+// prompt exits (App. H.2) with aao_len = the prompt length (every row takes the decision of
+// its sequence's last prompt token; tok_pos gives a token's position), 0 = token level.
+void launch_exit_decide(cudaStream_t st, const float* Xout, const float* I, const float* Xin, int D, DevRange rows,
+                        int max_rows, const int* row_tok, const int* forced, int layer, int n_layers,
+                        const float* delta_p, int test, int metric, float* sim, int* flag, float* inv_norm,
+                        unsigned* err);
 // Test + compaction + moves in one CTA for passes of at most EXIT_SMALL_MAX rows
 // (max_rows: the pass's row bound; at most 16 rows take a register-resident kernel, which
 // also writes xhat_next (if given): each kept row standardised (smode, seps) for the next
@@ -38,10 +46,12 @@ bool launch_exit_small(cudaStream_t st, const float* Xin, const float* Xout, con
                        int* ctr, int par, const int* row_tok, int* row_tok_next, const int* forced, int layer,
                        int n_layers, const float* delta_p, int test, float* sim, int* exit_tok, int* exit_layer_out,
                        float* Xnext, float* Inext, float* hsm_s, float* hsm_prev, float* hsm_I, int max_rows,
-                       bf16* xhat_next, int smode, float seps, unsigned* err);
+                       bf16* xhat_next, int smode, float seps, int metric, int aao_len, const int* tok_pos,
+                       unsigned* err);
 void launch_set_float(cudaStream_t st, float* p, float v);
 void launch_exit_scan(cudaStream_t st, int* ctr, int in_parity, const int* flag, const int* row_tok,
-                      int* row_tok_next, int* exit_tok, int* dst, int* exit_layer_out, int layer);
+                      int* row_tok_next, int* exit_tok, int* dst, int* exit_layer_out, int layer, int aao_len,
+                      const int* tok_pos);
 void launch_exit_move(cudaStream_t st, const float* Xin, const float* Xout, const float* I, int first, int D,
                       const int* n_rows, int max_rows, const int* dst, const float* inv_norm, float* Xnext,
                       float* Inext, float* hsm_s, float* hsm_prev, float* hsm_I);

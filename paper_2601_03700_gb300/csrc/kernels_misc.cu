@@ -151,30 +151,50 @@ __global__ void layernorm_inplace_kernel(float* X, DevRange rows, int D, const f
 // ---------------------------------------------------------------------------
 // exit test (Sec. 4.1): c = <s_i, I> / (|s_i| |I|) vs delta, or the forced layer
 // ---------------------------------------------------------------------------
-__global__ void exit_decide_kernel(const float* Xout, const float* I, int D, DevRange rows, const int* row_tok,
-                                   const int* forced, int layer, int n_layers, const float* delta_p, int test,
-                                   float* sim, int* flag, float* inv_norm, unsigned* err) {
+// The similarity the exit test compares with delta: global cos(s_i, I) (Eq. 7), local
+// cos(s_i, s_{i-1}) or both (their minimum: both must reach delta), App. H.3; from the sums
+// ns = |s_i|^2, ni = |I|^2, dot = <s_i, I>, np = |s_{i-1}|^2, dp = <s_i, s_{i-1}>.  A zero
+// norm gives -inf (never exits).
+__device__ __forceinline__ float exit_similarity(int metric, float ns, float ni, float dot, float np_, float dp) {
+  const float g = (ns > 0.f && ni > 0.f) ? dot / sqrtf(ns * ni) : -INFINITY;
+  if (metric == EXIT_GLOBAL) return g;
+  const float l = (ns > 0.f && np_ > 0.f) ? dp / sqrtf(ns * np_) : -INFINITY;
+  return metric == EXIT_LOCAL ? l : fminf(g, l);
+}
+
+__global__ void exit_decide_kernel(const float* Xout, const float* I, const float* Xin, int D, DevRange rows,
+                                   const int* row_tok, const int* forced, int layer, int n_layers,
+                                   const float* delta_p, int test, int metric, float* sim, int* flag,
+                                   float* inv_norm, unsigned* err) {
   PDL_ENTRY();
   const int warp = (blockIdx.x * blockDim.x + threadIdx.x) >> 5, lane = threadIdx.x & 31;
   const int r = warp;
   if (r >= rows.e()) return;
   const float* s = Xout + (size_t)r * D;
   const float* in = I + (size_t)r * D;
-  float ns = 0.f, ni = 0.f, dot = 0.f;
+  const float* sp = Xin + (size_t)r * D;
+  float ns = 0.f, ni = 0.f, dot = 0.f, np_ = 0.f, dp = 0.f;
   for (int d = lane; d < D; d += 32) {
     const float a = s[d], c = in[d];
     ns += a * a;
     ni += c * c;
     dot += a * c;
+    if (metric != EXIT_GLOBAL) {
+      const float b = sp[d];
+      np_ += b * b;
+      dp += a * b;
+    }
   }
   ns = warp_sum(ns);
   ni = warp_sum(ni);
   dot = warp_sum(dot);
+  np_ = warp_sum(np_);
+  dp = warp_sum(dp);
   if (lane != 0) return;
   const int tok = row_tok[r];
   int ex = 0;
   if (test) {
-    const float c = (ns > 0.f && ni > 0.f) ? dot / sqrtf(ns * ni) : -INFINITY;
+    const float c = exit_similarity(metric, ns, ni, dot, np_, dp);
     if (sim) sim[(size_t)tok * n_layers + (layer - 1)] = c;
     const int f = forced ? forced[tok] : 0;
     if (f != 0 && (f < 2 || f > n_layers)) atomicOr(err, ERRW_FORCED);
@@ -189,7 +209,8 @@ __global__ void exit_decide_kernel(const float* Xout, const float* I, int D, Dev
 // ctr[CTR_ACTIVE + parity] active counts, ctr[CTR_EXITED] exits so far,
 // ctr[CTR_PREFIX + i] exits after layer i.
 __global__ void exit_scan_kernel(int* ctr, int in_parity, const int* flag, const int* row_tok, int* row_tok_next,
-                                 int* exit_tok, int* dst, int* exit_layer_out, int layer) {
+                                 int* exit_tok, int* dst, int* exit_layer_out, int layer, int aao_len,
+                                 const int* tok_pos) {
   PDL_ENTRY();
   __shared__ int s_stay[1024];
   __shared__ int s_exit[1024];
@@ -198,8 +219,13 @@ __global__ void exit_scan_kernel(int* ctr, int in_parity, const int* flag, const
   const int tid = threadIdx.x, nt = blockDim.x;
   const int per = (n + nt - 1) / nt;
   const int lo = min(n, tid * per), hi = min(n, lo + per);
+  // all-at-once (aao_len = prompt length): a row takes the decision of its sequence's last
+  // prompt token, which is active with it at the same row offset (sequences stay whole)
+  auto fl = [&](int r) {
+    return aao_len ? flag[min(n - 1, r + (aao_len - 1 - tok_pos[row_tok[r]]))] : flag[r];
+  };
   int ce = 0;
-  for (int r = lo; r < hi; ++r) ce += flag[r];
+  for (int r = lo; r < hi; ++r) ce += fl(r);
   s_exit[tid] = ce;
   s_stay[tid] = (hi - lo) - ce;
   __syncthreads();
@@ -218,7 +244,7 @@ __global__ void exit_scan_kernel(int* ctr, int in_parity, const int* flag, const
   int s = s_stay[tid] - ((hi - lo) - ce);
   for (int r = lo; r < hi; ++r) {
     const int tok = row_tok[r];
-    if (flag[r]) {
+    if (fl(r)) {
       dst[r] = -1 - (base + e);
       exit_tok[base + e] = tok;
       if (exit_layer_out) exit_layer_out[tok] = layer;
@@ -278,6 +304,7 @@ __global__ void __launch_bounds__(256) exit_small_kernel(const float* Xin, const
                                                          int n_layers, const float* delta_p, int test, float* sim,
                                                          int* exit_tok, int* exit_layer_out, float* Xnext,
                                                          float* Inext, float* hsm_s, float* hsm_prev, float* hsm_I,
+                                                         int metric, int aao_len, const int* tok_pos,
                                                          unsigned* err) {
   PDL_ENTRY();
   __shared__ int s_dst[EXIT_SMALL_MAX];
@@ -289,21 +316,29 @@ __global__ void __launch_bounds__(256) exit_small_kernel(const float* Xin, const
   for (int r = warp; r < n; r += nw) {
     const float* s = Xout + (size_t)r * D;
     const float* in = I + (size_t)r * D;
-    float ns = 0.f, ni = 0.f, dot = 0.f;
+    const float* sp = Xin + (size_t)r * D;
+    float ns = 0.f, ni = 0.f, dot = 0.f, np_ = 0.f, dp = 0.f;
     for (int d = lane; d < D; d += 32) {
       const float a = s[d], c = in[d];
       ns += a * a;
       ni += c * c;
       dot += a * c;
+      if (metric != EXIT_GLOBAL) {
+        const float b = sp[d];
+        np_ += b * b;
+        dp += a * b;
+      }
     }
     ns = warp_sum(ns);
     ni = warp_sum(ni);
     dot = warp_sum(dot);
+    np_ = warp_sum(np_);
+    dp = warp_sum(dp);
     if (lane == 0) {
       const int tok = row_tok[r];
       int ex = 0;
       if (test) {
-        const float c = (ns > 0.f && ni > 0.f) ? dot / sqrtf(ns * ni) : -INFINITY;
+        const float c = exit_similarity(metric, ns, ni, dot, np_, dp);
         if (sim) sim[(size_t)tok * n_layers + (layer - 1)] = c;
         const int f = forced ? forced[tok] : 0;
         if (f != 0 && (f < 2 || f > n_layers)) atomicOr(err, ERRW_FORCED);
@@ -319,7 +354,10 @@ __global__ void __launch_bounds__(256) exit_small_kernel(const float* Xin, const
     int e = 0, k = 0;
     for (int r = 0; r < n; ++r) {
       const int tok = row_tok[r];
-      if (s_dst[r]) {
+      // all-at-once: the decision of the sequence's last prompt token, a later row not yet
+      // rewritten by this loop
+      const int rl = aao_len ? min(n - 1, r + (aao_len - 1 - tok_pos[tok])) : r;
+      if (s_dst[rl]) {
         s_dst[r] = -1 - (base + e);
         exit_tok[base + e] = tok;
         if (exit_layer_out) exit_layer_out[tok] = layer;
@@ -373,9 +411,10 @@ __global__ void __launch_bounds__(EXD_THREADS)
                        int layer, int n_layers, const float* delta_p, int test, float* sim, int* exit_tok,
                        int* exit_layer_out, float* __restrict__ Xnext, float* __restrict__ Inext,
                        float* __restrict__ hsm_s, float* __restrict__ hsm_prev, float* __restrict__ hsm_I, int rshift,
-                       int max_rows, bf16* xhat_next, int smode, float seps, unsigned* err) {
+                       int max_rows, bf16* xhat_next, int smode, float seps, int metric, int aao_len,
+                       const int* tok_pos, unsigned* err) {
   PDL_ENTRY();
-  __shared__ float s_red[EXD_THREADS / 32][4];
+  __shared__ float s_red[EXD_THREADS / 32][6];
   __shared__ float s_mu[16];
   __shared__ int s_dst[16], s_tok[16];
   __shared__ float s_w[16];
@@ -391,7 +430,7 @@ __global__ void __launch_bounds__(EXD_THREADS)
   const float delta = *delta_p;
   const int D4 = D >> 2;
   float4 xs[EXD_V], xi[EXD_V], xp[EXD_V];
-  float ns = 0.f, ni = 0.f, dot = 0.f, sx = 0.f;
+  float ns = 0.f, ni = 0.f, dot = 0.f, sx = 0.f, np_ = 0.f, dp = 0.f;
   if (row < max_rows) {
     const float4* s4 = reinterpret_cast<const float4*>(Xout + (size_t)row * D);
     const float4* i4 = reinterpret_cast<const float4*>(I + (size_t)row * D);
@@ -413,6 +452,9 @@ __global__ void __launch_bounds__(EXD_THREADS)
         ni += c.x * c.x + c.y * c.y + c.z * c.z + c.w * c.w;
         dot += a.x * c.x + a.y * c.y + a.z * c.z + a.w * c.w;
         sx += a.x + a.y + a.z + a.w;
+        const float4 b = xp[j];
+        np_ += b.x * b.x + b.y * b.y + b.z * b.z + b.w * b.w;
+        dp += a.x * b.x + a.y * b.y + a.z * b.z + a.w * b.w;
       }
     }
   }
@@ -420,28 +462,34 @@ __global__ void __launch_bounds__(EXD_THREADS)
   ni = warp_sum(ni);
   dot = warp_sum(dot);
   sx = warp_sum(sx);
+  np_ = warp_sum(np_);
+  dp = warp_sum(dp);
   if (lane == 0) {
     s_red[warp][0] = ns;
     s_red[warp][1] = ni;
     s_red[warp][2] = dot;
     s_red[warp][3] = sx;
+    s_red[warp][4] = np_;
+    s_red[warp][5] = dp;
   }
   __syncthreads();
   const int wpr = tpr >> 5;   // warps per row
   if ((int)threadIdx.x < n) {   // thread r decides row r
     const int r = threadIdx.x;
-    float a = 0.f, b = 0.f, c = 0.f, m = 0.f;
+    float a = 0.f, b = 0.f, c = 0.f, m = 0.f, pn = 0.f, pd = 0.f;
     for (int w = r * wpr; w < (r + 1) * wpr; ++w) {
       a += s_red[w][0];
       b += s_red[w][1];
       c += s_red[w][2];
       m += s_red[w][3];
+      pn += s_red[w][4];
+      pd += s_red[w][5];
     }
     s_mu[r] = smode == NORM_LN ? m / D : 0.f;
     const int tok = tok_r;
     int ex = 0;
     if (test) {
-      const float cs = (a > 0.f && b > 0.f) ? c / sqrtf(a * b) : -INFINITY;
+      const float cs = exit_similarity(metric, a, b, c, pn, pd);
       if (sim) sim[(size_t)tok * n_layers + (layer - 1)] = cs;
       const int f = forced ? forced[tok] : 0;
       if (f != 0 && (f < 2 || f > n_layers)) atomicOr(err, ERRW_FORCED);
@@ -456,7 +504,9 @@ __global__ void __launch_bounds__(EXD_THREADS)
     int e = 0, k = 0;
     for (int r = 0; r < n; ++r) {
       const int tok = s_tok[r];
-      if (s_dst[r]) {
+      // all-at-once: the decision of the sequence's last prompt token (a later row)
+      const int rl = aao_len ? min(n - 1, r + (aao_len - 1 - tok_pos[tok])) : r;
+      if (s_dst[rl]) {
         s_dst[r] = -1 - (base + e);
         exit_tok[base + e] = tok;
         if (exit_layer_out) exit_layer_out[tok] = layer;
@@ -546,7 +596,8 @@ bool launch_exit_small(cudaStream_t st, const float* Xin, const float* Xout, con
                        int* ctr, int par, const int* row_tok, int* row_tok_next, const int* forced, int layer,
                        int n_layers, const float* delta_p, int test, float* sim, int* exit_tok, int* exit_layer_out,
                        float* Xnext, float* Inext, float* hsm_s, float* hsm_prev, float* hsm_I, int max_rows,
-                       bf16* xhat_next, int smode, float seps, unsigned* err) {
+                       bf16* xhat_next, int smode, float seps, int metric, int aao_len, const int* tok_pos,
+                       unsigned* err) {
   int rshift = 0;
   while ((1 << rshift) < max_rows) ++rshift;
   const bool aligned = ((uintptr_t)Xin | (uintptr_t)Xout | (uintptr_t)I | (uintptr_t)Xnext | (uintptr_t)Inext |
@@ -554,11 +605,12 @@ bool launch_exit_small(cudaStream_t st, const float* Xin, const float* Xout, con
   if (max_rows <= 16 && D % 4 == 0 && D / 4 <= EXD_V * (EXD_THREADS >> rshift) && aligned) {
     launch_k(exit_decode_kernel, 1, EXD_THREADS, 0, st, Xin, Xout, I, first, D, ctr, par, row_tok, row_tok_next, forced,
              layer, n_layers, delta_p, test, sim, exit_tok, exit_layer_out, Xnext, Inext, hsm_s, hsm_prev, hsm_I,
-             rshift, max_rows, xhat_next, smode, seps, err);
+             rshift, max_rows, xhat_next, smode, seps, metric, aao_len, tok_pos, err);
     return true;
   }
   launch_k(exit_small_kernel, 1, 256, 0, st, Xin, Xout, I, first, D, ctr, par, row_tok, row_tok_next, forced, layer,
-           n_layers, delta_p, test, sim, exit_tok, exit_layer_out, Xnext, Inext, hsm_s, hsm_prev, hsm_I, err);
+           n_layers, delta_p, test, sim, exit_tok, exit_layer_out, Xnext, Inext, hsm_s, hsm_prev, hsm_I, metric,
+           aao_len, tok_pos, err);
   return false;
 }
 
@@ -879,18 +931,20 @@ void launch_layernorm_inplace(cudaStream_t st, float* X, DevRange rows, int max_
   launch_k(layernorm_inplace_kernel, max_rows, 256, 0, st, X, rows, D, g, b, eps);
 }
 
-void launch_exit_decide(cudaStream_t st, const float* Xout, const float* I, int D, DevRange rows, int max_rows,
-                        const int* row_tok, const int* forced, int layer, int n_layers, const float* delta_p, int test,
-                        float* sim, int* flag, float* inv_norm, unsigned* err) {
+void launch_exit_decide(cudaStream_t st, const float* Xout, const float* I, const float* Xin, int D, DevRange rows,
+                        int max_rows, const int* row_tok, const int* forced, int layer, int n_layers,
+                        const float* delta_p, int test, int metric, float* sim, int* flag, float* inv_norm,
+                        unsigned* err) {
   if (max_rows <= 0) return;
-  launch_k(exit_decide_kernel, cdiv(max_rows, 8), 256, 0, st, Xout, I, D, rows, row_tok, forced, layer, n_layers, delta_p,
-                                                       test, sim, flag, inv_norm, err);
+  launch_k(exit_decide_kernel, cdiv(max_rows, 8), 256, 0, st, Xout, I, Xin, D, rows, row_tok, forced, layer, n_layers,
+           delta_p, test, metric, sim, flag, inv_norm, err);
 }
 
 void launch_exit_scan(cudaStream_t st, int* ctr, int in_parity, const int* flag, const int* row_tok,
-                      int* row_tok_next, int* exit_tok, int* dst, int* exit_layer_out, int layer) {
+                      int* row_tok_next, int* exit_tok, int* dst, int* exit_layer_out, int layer, int aao_len,
+                      const int* tok_pos) {
   launch_k(exit_scan_kernel, 1, 1024, 0, st, ctr, in_parity, flag, row_tok, row_tok_next, exit_tok, dst, exit_layer_out,
-                                       layer);
+           layer, aao_len, tok_pos);
 }
 
 void launch_exit_move(cudaStream_t st, const float* Xin, const float* Xout, const float* I, int first, int D,

@@ -113,6 +113,8 @@ struct adept_model {
   std::vector<int> dec_warm;                // direct runs done per batch size
   // options / instrumentation
   int hsm_identity = 0, profile = 0, force_simt = 0, use_graph = 1, use_dg = 1, use_fused = 1;
+  int exit_metric = 0;   // EXIT_GLOBAL / EXIT_LOCAL / EXIT_BOTH
+  int all_at_once = 0;   // prompt passes: sequences leave with their last prompt token
   // persistent generation-step kernel (small batches of bf16 decoders); NULL when not eligible
   DfState* df = nullptr;
   std::string df_why;
@@ -771,6 +773,8 @@ static adept_status run_pass(adept_model* m, int n_tok, int batch, int prompt_le
   // generation step: the split-KV attention grid covers the reserved capacity (CTAs past a
   // sequence's length return at once), which keeps every launch of a step step-invariant
   const int decode_keys = decode ? std::min(c.max_seq, m->max_blocks_per_seq * c.kv_block_tokens) : 0;
+  // all-at-once exits apply to prompt passes (a generation step holds one token per sequence)
+  const int aao_len = !decode && m->all_at_once ? prompt_len : 0;
   (void)batch;
   int par = 0;
   for (int i = 1; i <= N; ++i) {
@@ -859,13 +863,15 @@ static adept_status run_pass(adept_model* m, int n_tok, int batch, int prompt_le
         xn_valid = launch_exit_small(st, Xi, m->X_out, Ii, i == 1, D, m->ctr, par, rt, m->row_tok[par ^ 1], forced, i,
                                      N, m->d_delta, test, sim_out, m->exit_tok, exit_out, m->X_in[par ^ 1],
                                      m->I[par ^ 1], m->hsm_s, m->hsm_prev, m->hsm_I, mr,
-                                     dgrows ? (bf16*)m->xn : nullptr, amode, eps, m->err_word) &&
+                                     dgrows ? (bf16*)m->xn : nullptr, amode, eps, m->exit_metric, aao_len,
+                                     m->tok_pos, m->err_word) &&
                    dgrows;
         m->launches += 1;
       } else {
-        launch_exit_decide(st, m->X_out, Ii, D, act, mr, rt, forced, i, N, m->d_delta, test, sim_out, m->flag,
-                           m->inv_norm, m->err_word);
-        launch_exit_scan(st, m->ctr, par, m->flag, rt, m->row_tok[par ^ 1], m->exit_tok, m->dst, exit_out, i);
+        launch_exit_decide(st, m->X_out, Ii, Xi, D, act, mr, rt, forced, i, N, m->d_delta, test, m->exit_metric,
+                           sim_out, m->flag, m->inv_norm, m->err_word);
+        launch_exit_scan(st, m->ctr, par, m->flag, rt, m->row_tok[par ^ 1], m->exit_tok, m->dst, exit_out, i, aao_len,
+                         m->tok_pos);
         launch_exit_move(st, Xi, m->X_out, Ii, i == 1, D, m->ctr + CTR_ACTIVE + par, mr, m->dst, m->inv_norm,
                          m->X_in[par ^ 1], m->I[par ^ 1], m->hsm_s, m->hsm_prev, m->hsm_I);
         m->launches += 3;
@@ -1094,7 +1100,7 @@ adept_status adept_decode_step(adept_model* m, int batch, const int32_t* d_token
       return fail(m, ADEPT_ERR_CAPACITY, "sequence %d is full (%d positions)", b, m->h_seq_len[b]);
   }
   cudaStream_t st = (cudaStream_t)stream;
-  if (m->df && m->use_fused && batch <= df_max_batch(m->df)) {
+  if (m->df && m->use_fused && m->exit_metric == EXIT_GLOBAL && batch <= df_max_batch(m->df)) {
     // one persistent launch for the whole step (decode_fused.cu); it reads the caller's
     // inputs and writes the caller's outputs directly
     cudaEvent_t ev = nullptr;
@@ -1303,6 +1309,12 @@ adept_status adept_set_option(adept_model* m, int option, int value) {
     case ADEPT_OPT_DECODE_GRAPH: m->use_graph = value != 0; drop_graphs(m); return ADEPT_OK;
     case ADEPT_OPT_DECODE_GEMM: m->use_dg = value != 0; drop_graphs(m); return ADEPT_OK;
     case ADEPT_OPT_FUSED_DECODE: m->use_fused = value != 0; return ADEPT_OK;
+    case ADEPT_OPT_EXIT_METRIC:
+      if (value < EXIT_GLOBAL || value > EXIT_BOTH) return fail(m, ADEPT_ERR_INVALID_ARG, "exit metric %d", value);
+      m->exit_metric = value;
+      drop_graphs(m);
+      return ADEPT_OK;
+    case ADEPT_OPT_ALL_AT_ONCE: m->all_at_once = value != 0; return ADEPT_OK;
   }
   return fail(m, ADEPT_ERR_INVALID_ARG, "unknown option %d", option);
 }

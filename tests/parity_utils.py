@@ -76,13 +76,18 @@ def decisions_agree_outside_band(g_sim: np.ndarray, o_sim: np.ndarray, delta: fl
     assert not bad.any(), f"{int(bad.sum())} decisions differ outside the band"
 
 
-def run_prefill(pair: Pair, tokens: np.ndarray, delta: float, forced=None, hsm_identity=False):
+def run_prefill(pair: Pair, tokens: np.ndarray, delta: float, forced=None, hsm_identity=False, metric="global",
+                all_at_once=False):
     """Returns (oracle result, oracle cache, gpu outputs dict); in threshold mode with band
-    tokens, the GPU is re-run with the oracle's exit layers forced."""
+    tokens, the GPU is re-run with the oracle's exit layers forced.  metric / all_at_once:
+    the exit-rule variant (the device options are set here too)."""
     cfg = pair.cfg
     B, P = tokens.shape
     cache = O.OracleCache(cfg, cfg.max_batch, cfg.max_seq)
-    ores = O.prefill(pair.om, cache, tokens, delta, forced, hsm_mode="identity" if hsm_identity else "hsm")
+    ores = O.prefill(pair.om, cache, tokens, delta, forced, hsm_mode="identity" if hsm_identity else "hsm",
+                     metric=metric, all_at_once=all_at_once)
+    adept.adept_set_option(pair.gm.h, adept.OPT_EXIT_METRIC, {"global": 0, "local": 1, "both": 2}[metric])
+    adept.adept_set_option(pair.gm.h, adept.OPT_ALL_AT_ONCE, int(all_at_once))
     adept.adept_set_option(pair.gm.h, adept.OPT_HSM_IDENTITY, int(hsm_identity))
     tk = torch.as_tensor(tokens, dtype=torch.int32, device="cuda")
     fz = None if forced is None else torch.as_tensor(np.asarray(forced).reshape(B, P), dtype=torch.int32, device="cuda")
@@ -109,9 +114,10 @@ def run_prefill(pair: Pair, tokens: np.ndarray, delta: float, forced=None, hsm_i
     return ores, cache, out
 
 
-def compare_prefill(pair: Pair, tokens, delta, forced=None, hsm_identity=False, check_cache=True):
+def compare_prefill(pair: Pair, tokens, delta, forced=None, hsm_identity=False, check_cache=True, metric="global",
+                    all_at_once=False):
     B, P = tokens.shape
-    ores, cache, g = run_prefill(pair, tokens, delta, forced, hsm_identity)
+    ores, cache, g = run_prefill(pair, tokens, delta, forced, hsm_identity, metric, all_at_once)
     assert_rows_close(g["final"], ores.final, pair.tol, "final states")
     assert_rows_close(g["logits"], ores.logits, pair.tol, "logits")
     if pair.cfg.family != synth.BERT:
@@ -136,7 +142,7 @@ def check_greedy(g_next, g_logits, o_logits):
 
 
 def compare_decode(pair: Pair, cache: O.OracleCache, first_tokens, steps: int, delta: float, forced_steps=None,
-                   hsm_identity=False):
+                   hsm_identity=False, metric="global"):
     """Greedy decode for `steps` steps, fed with the oracle's tokens (teacher forcing), so
     both sides stay on one trajectory; per step: exit layers, similarities, final states,
     logits and greedy tokens; at the end every cached position of every layer."""
@@ -144,7 +150,7 @@ def compare_decode(pair: Pair, cache: O.OracleCache, first_tokens, steps: int, d
     tok = np.asarray(first_tokens)
     for s in range(steps):
         f = None if forced_steps is None else np.asarray(forced_steps[s])
-        o = O.decode_step(pair.om, cache, tok, delta, f, hsm_mode="identity" if hsm_identity else "hsm")
+        o = O.decode_step(pair.om, cache, tok, delta, f, hsm_mode="identity" if hsm_identity else "hsm", metric=metric)
         use_forced = f
         if f is None and band_tokens(o.sim, delta).any():
             use_forced = o.exit_layer

@@ -289,3 +289,37 @@ def test_threshold_calibration_matches_oracle(dtype):
         if not np.any(np.abs(res.sim - d_g) <= BAND):
             assert O.reduction_in_computation(res.exit_layer, cfg.n_layers) == pytest.approx(r_g, abs=1e-6)
     pair.close()
+
+
+# --------------------------------------------------------------------------- exit-rule variants
+
+@pytest.mark.parametrize("metric", ["local", "both"])
+@pytest.mark.parametrize("dtype", ["f32", "bf16"])
+def test_exit_metric_variants_match_oracle(metric, dtype):
+    """Local similarity cos(s_i, s_{i-1}) and both similarities (App. H.3): prompt pass and
+    generation steps against the oracle, thresholds that leave some tokens early."""
+    cfg = synth.tiny_config(n_layers=6) if dtype == "f32" else small(synth.LLAMA, n_heads=2, head_dim=128)
+    pair = Pair(cfg, seed=61, std=0.05)
+    tokens = synth.make_tokens(61, 2, 30, cfg.vocab).numpy()
+    probe = O.prefill(pair.om, O.OracleCache(cfg, 2, 32), tokens, np.inf, metric=metric).sim
+    delta = float(np.nanquantile(probe, 0.7))
+    ores, cache, g = compare_prefill(pair, tokens, delta, metric=metric)
+    assert 2 <= ores.exit_layer.min() and ores.exit_layer.min() < cfg.n_layers
+    compare_decode(pair, cache, ores.next_token, 3, delta, metric=metric)
+    pair.close()
+
+
+@pytest.mark.parametrize("dtype", ["f32", "bf16"])
+def test_all_at_once_prompt_exits_match_oracle(dtype):
+    """All-at-once prompt exits (App. H.2): every token of a sequence leaves with its last
+    prompt token; exits, final states, logits and the cache against the oracle."""
+    cfg = synth.tiny_config(n_layers=6) if dtype == "f32" else small(synth.GPT2)
+    pair = Pair(cfg, seed=62, std=0.05)
+    B, P = 3, 20
+    tokens = synth.make_tokens(62, B, P, cfg.vocab).numpy()
+    probe = O.prefill(pair.om, O.OracleCache(cfg, B, P), tokens, np.inf).sim.reshape(B, P, -1)[:, P - 1]
+    delta = float(np.nanquantile(probe, 0.6))
+    ores, cache, g = compare_prefill(pair, tokens, delta, all_at_once=True)
+    ex = g["exit"].reshape(B, P)
+    assert np.all(ex == ex[:, -1:])
+    pair.close()
