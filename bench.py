@@ -477,6 +477,27 @@ def ours(args, rank, world, device):
     line["calibration"] = {"target_rdc": 0.25, "tol": 0.01, "delta": round(d_c, 6), "rdc": round(r_c, 4),
                            "passes": n_c, "ms": round(t_cal, 3), "ms_per_pass": round(t_cal / max(n_c, 1), 3),
                            "batch": f"{B} x {P} workload prompts, threshold exits"}
+    # --------------------------------------------------------------- exit-rule variants (App. H.2-H.3)
+    # the workload's prompt pass at the calibrated threshold: reduction and time per variant
+    variants = {}
+    ex_v = torch.empty(B * P, dtype=torch.int32, device=device)
+    nx_v = torch.empty(B, dtype=torch.int32, device=device)
+    for name, metric, aao in (("global", 0, 0), ("local", 1, 0), ("both", 2, 0), ("all_at_once", 0, 1)):
+        adept.adept_set_option(run.m.h, adept.OPT_EXIT_METRIC, metric)
+        adept.adept_set_option(run.m.h, adept.OPT_ALL_AT_ONCE, aao)
+        adept.adept_prefill(run.m.h, B, P, run.tokens.view(-1), d_c, None, ex_v, None, nx_v, None)
+        torch.cuda.synchronize()
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record(st)
+        adept.adept_prefill(run.m.h, B, P, run.tokens.view(-1), d_c, None, ex_v, None, nx_v, None)
+        e1.record(st)
+        torch.cuda.synchronize()
+        depth = ex_v.double().mean().item()
+        variants[name] = {"rdc": round(1.0 - depth / cfg.n_layers, 4), "prompt_ms": round(e0.elapsed_time(e1), 3)}
+    adept.adept_set_option(run.m.h, adept.OPT_EXIT_METRIC, 0)
+    adept.adept_set_option(run.m.h, adept.OPT_ALL_AT_ONCE, 0)
+    adept.adept_check_device_status(run.m.h)
+    line["exit_variants"] = {"delta": round(d_c, 6), "batch": f"{B} x {P} workload prompts", **variants}
     run.m.close()
     del run
     torch.cuda.empty_cache()
