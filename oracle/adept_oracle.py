@@ -23,6 +23,8 @@ What it follows (paper sections / equations / tables):
   in computation (RDC) over a calibration batch.
 * Exit-rule variants (App. H.2-H.3): the local similarity cos(s_i, s_{i-1}), both
   similarities, and all-at-once prompt exits decided by each sequence's last token.
+* Encoder "stop entirely" (Sec. 4.3, downstream tasks): exited tokens get no deeper K/V
+  and drop out of deeper attention; their s~ feeds the classifier.
 
 Readings where the paper is silent (each one is also listed in the design notes):
 
@@ -265,18 +267,23 @@ class OracleCache:
 
 
 def attend(m: OracleModel, q: np.ndarray, qpos: np.ndarray, K: np.ndarray, V: np.ndarray,
-           causal: bool) -> np.ndarray:
+           causal: bool, key_mask: Optional[np.ndarray] = None) -> np.ndarray:
     """Softmax attention of one sequence's queries q [n, H, dh] over keys K/V [L, Hkv, dh].
 
-    Causal: query at position p sees keys 0..p.  Returns [n, H*dh]."""
+    Causal: query at position p sees keys 0..p.  key_mask [L] (optional): only those keys.
+    Returns [n, H*dh]."""
     c = m.cfg
     rep = c.n_heads // c.n_kv_heads
+    if key_mask is not None:
+        K, V = np.where(key_mask[:, None, None], K, 0.0), np.where(key_mask[:, None, None], V, 0.0)
     Kh = np.repeat(K, rep, axis=1)
     Vh = np.repeat(V, rep, axis=1)
     sc = np.einsum("nhd,lhd->hnl", q, Kh) / math.sqrt(c.head_dim)
     if causal:
         kpos = np.arange(K.shape[0])
         sc = np.where(kpos[None, None, :] <= qpos[None, :, None], sc, -np.inf)
+    if key_mask is not None:
+        sc = np.where(key_mask[None, None, :], sc, -np.inf)
     sc = sc - np.max(sc, axis=-1, keepdims=True)
     p = np.exp(sc)
     p = p / np.sum(p, axis=-1, keepdims=True)
@@ -285,17 +292,21 @@ def attend(m: OracleModel, q: np.ndarray, qpos: np.ndarray, K: np.ndarray, V: np
 
 
 def layer_body(m: OracleModel, i: int, h: np.ndarray, seq: np.ndarray, pos: np.ndarray,
-               cache: OracleCache, causal: bool, kv_len: np.ndarray) -> np.ndarray:
+               cache: OracleCache, causal: bool, kv_len: np.ndarray,
+               key_active: Optional[Dict[int, np.ndarray]] = None) -> np.ndarray:
     """Everything of layer i after its K/V were cached: Q, attention, O, FFN, residuals.
 
-    h: [n, D] layer inputs of the active tokens; returns their layer outputs."""
+    h: [n, D] layer inputs of the active tokens; returns their layer outputs.
+    key_active (optional, "stop entirely"): per sequence, the positions whose K/V layer i
+    holds; attention sees only those keys."""
     c, rb = m.cfg, m.rb
     q = m.q_project(i, h, pos)
     att = np.zeros((len(h), c.n_heads * c.head_dim))
     for b in np.unique(seq):
         sel = np.nonzero(seq == b)[0]
         L = int(kv_len[b])
-        att[sel] = attend(m, q[sel], pos[sel], cache.K[i - 1][b, :L], cache.V[i - 1][b, :L], causal)
+        km = None if key_active is None else key_active[int(b)][:L]
+        att[sel] = attend(m, q[sel], pos[sel], cache.K[i - 1][b, :L], cache.V[i - 1][b, :L], causal, km)
     o = rb(att) @ m.L(i, "wo").T
     if m.has(i, "bo"):
         o = o + m.L(i, "bo")
@@ -336,7 +347,7 @@ def check_forced(forced: np.ndarray, n_layers: int):
 def early_exit_pass(m: OracleModel, cache: OracleCache, s0: np.ndarray, seq: np.ndarray,
                     pos: np.ndarray, delta: float, forced: Optional[np.ndarray], causal: bool,
                     kv_len: np.ndarray, hsm_mode: str = "hsm", metric: str = "global",
-                    aao_len: int = 0) -> PassResult:
+                    aao_len: int = 0, stop_entirely: bool = False) -> PassResult:
     """Run tokens (all in parallel, App. I) through layers 1..N with token-level exits.
 
     For each layer i: (a) K/V of the active tokens from their layer input go to the
@@ -350,6 +361,9 @@ def early_exit_pass(m: OracleModel, cache: OracleCache, s0: np.ndarray, seq: np.
     the global and the local similarity to reach delta (the recorded similarity is then
     their minimum); aao_len = P > 0 (prompt passes) makes every token take the decision of
     its sequence's last prompt token (position P - 1), so a sequence leaves at once.
+    stop_entirely (encoders, Sec. 4.3 on downstream tasks: computation stops beyond the exit
+    layer): an exiting token gets s~ for the classifier but no K/V of deeper layers, and the
+    attention of a deeper layer sees only the tokens still active there.
     """
     if metric not in ("global", "local", "both"):
         raise ValueError(metric)
@@ -369,7 +383,12 @@ def early_exit_pass(m: OracleModel, cache: OracleCache, s0: np.ndarray, seq: np.
             break
         k, v = m.kv_project(i, s[A], pos[A])                              # (a)
         cache.write(i, seq[A], pos[A], k, v)
-        s_new = layer_body(m, i, s[A], seq[A], pos[A], cache, causal, kv_len)   # (b)
+        key_active = None
+        if stop_entirely:
+            key_active = {int(b): np.zeros(int(kv_len[b]), dtype=bool) for b in np.unique(seq)}
+            for j in A:
+                key_active[int(seq[j])][int(pos[j])] = True
+        s_new = layer_body(m, i, s[A], seq[A], pos[A], cache, causal, kv_len, key_active)   # (b)
         exits = np.zeros(len(A), dtype=bool)
         if 2 <= i <= N - 1:                                                # (c)
             cg = cosine(s_new, inertia[A])
@@ -393,7 +412,7 @@ def early_exit_pass(m: OracleModel, cache: OracleCache, s0: np.ndarray, seq: np.
                 raise ValueError(hsm_mode)
             final[E] = st
             exit_layer[E] = i
-            for r in range(i + 1, N + 1):
+            for r in range(i + 1, N + 1) if not stop_entirely else ():
                 kr, vr = m.kv_project(r, st, pos[E])
                 cache.write(r, seq[E], pos[E], kr, vr)
         s[A] = s_new
@@ -404,13 +423,15 @@ def early_exit_pass(m: OracleModel, cache: OracleCache, s0: np.ndarray, seq: np.
 
 def prefill(m: OracleModel, cache: OracleCache, tokens: np.ndarray, delta: float,
             forced: Optional[np.ndarray] = None, hsm_mode: str = "hsm", metric: str = "global",
-            all_at_once: bool = False) -> PassResult:
+            all_at_once: bool = False, stop_entirely: bool = False) -> PassResult:
     """Prompt pass for sequences 0..B-1 (resets them); tokens [B, P].
 
     Decoder: logits [B, V] of each sequence's last position and its greedy token
     (lowest index on ties).  Encoder: bidirectional attention; classifier logits
     [B, C] from position 0's final state."""
     c = m.cfg
+    if stop_entirely and c.family != BERT:
+        raise ValueError("the stop-entirely variant is defined for encoders")
     tokens = np.asarray(tokens)
     B, P = tokens.shape
     seq = np.repeat(np.arange(B), P)
@@ -424,7 +445,7 @@ def prefill(m: OracleModel, cache: OracleCache, tokens: np.ndarray, delta: float
     kv_len = cache.lens.copy()
     res = early_exit_pass(m, cache, s0, seq, pos, delta,
                           None if forced is None else np.asarray(forced).reshape(-1),
-                          causal, kv_len, hsm_mode, metric, P if all_at_once else 0)
+                          causal, kv_len, hsm_mode, metric, P if all_at_once else 0, stop_entirely)
     fin = res.final.reshape(B, P, -1)
     if c.family == BERT:
         res.logits = m.cls_logits(fin[:, 0])

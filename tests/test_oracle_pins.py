@@ -459,3 +459,43 @@ def test_all_at_once_sequences_leave_with_their_last_token():
                     want = i
                     break
             assert np.all(ex[b] == want)
+
+
+def test_encoder_stop_entirely_matches_independent_masked_model():
+    """Encoder "stop entirely" (Sec. 4.3, downstream tasks) with forced exits against a
+    token-subset forward of the independent torch model: at each layer only the tokens
+    still active are computed, and attend to each other only (bidirectional); an exiting
+    token's output is the HSM of (s_i, s_{i-1}, inertia before s_hat_i)."""
+    cfg = small_cfg(synth.BERT, n_layers=5)
+    m, ref, _ = model_and_ref(cfg, seed=54)
+    P = 7
+    tokens = synth.make_tokens(54, 1, P, cfg.vocab).numpy()
+    forced = np.array([2, 5, 3, 4, 2, 5, 3])
+    r = O.prefill(m, O.OracleCache(cfg, 1, 8), tokens, 0.5, forced, stop_entirely=True)
+    np.testing.assert_array_equal(r.exit_layer, forced)
+    # the torch side
+    tk = torch.as_tensor(tokens)
+    pos = torch.arange(P)[None]
+    h = ref.embed(tk, pos)[0]
+    inertia = torch.zeros_like(h)
+    final = torch.zeros_like(h)
+    active = np.ones(P, dtype=bool)
+    for i in range(1, cfg.n_layers + 1):
+        A = np.nonzero(active)[0]
+        hA = h[A][None]
+        q = ref.q(i, hA, pos[:, A]).transpose(1, 2)
+        k, v = ref.kv(i, hA, pos[:, A])
+        a = F.scaled_dot_product_attention(q, k.transpose(1, 2), v.transpose(1, 2))
+        s_new = ref.after_attn(i, hA, a.transpose(1, 2).flatten(-2))[0]
+        ex = (forced[A] == i) if 2 <= i <= cfg.n_layers - 1 else np.zeros(len(A), dtype=bool)
+        I_before = inertia[A].clone()
+        inertia[A] = I_before + s_new / s_new.norm(dim=-1, keepdim=True)
+        for kk in np.nonzero(ex)[0]:
+            j = A[kk]
+            final[j] = ref.hsm(s_new[kk], h[j], I_before[kk])
+        h[A] = s_new
+        active[A[ex]] = False
+    final[active] = h[active]
+    np.testing.assert_allclose(r.final, final.numpy(), rtol=1e-10, atol=1e-10)
+    # the classifier reads position 0's state
+    np.testing.assert_allclose(r.logits[0], ref.head(final[0][None]).numpy()[0], rtol=1e-10, atol=1e-10)
