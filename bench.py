@@ -287,6 +287,44 @@ def llama_work(cfg, exit_prompt, exit_decode):
     return fl
 
 
+def run_encoder(adept, device, B=64, P=128):
+    """BERT-base shape, bf16, random-init: 64 x 128-token classification batch, threshold
+    exits at delta = 0.9, forced exits ~ U{4..12}, and full depth; the default exit (deeper
+    K/V filled from s~) against the encoder's "stop entirely" variant (Sec. 4.3).
+    Throughput in sequences/s and tokens/s including the classifier."""
+    cfg = synth.bert_base_config(max_batch=B, max_seq=P, max_pass_tokens=B * P)
+    W = synth.make_weights(cfg, seed=0, device=device)
+    m = adept.Model(cfg, W)
+    del W
+    tok = synth.make_tokens(0, B, P, cfg.vocab).to(device)
+    fz = synth.forced_exits_uniform(0, B * P, 4, 12, name="forced_encoder").view(-1).to(device)
+    full = torch.full_like(fz, cfg.n_layers)
+    ex = torch.empty(B * P, dtype=torch.int32, device=device)
+    lg = torch.empty(B, cfg.n_classes, device=device)
+    st = torch.cuda.current_stream()
+    out = {}
+    for name, forced, stop in (("threshold_0.9", None, 0), ("forced_U4_12", fz, 0), ("forced_U4_12_stop_entirely", fz, 1),
+                               ("full_depth", full, 0)):
+        adept.adept_set_option(m.h, adept.OPT_STOP_ENTIRELY, stop)
+        ts = []
+        for rep in range(4):
+            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            torch.cuda.synchronize()
+            e0.record(st)
+            adept.adept_prefill(m.h, B, P, tok.view(-1), 0.9, forced, ex, lg, None, None)
+            e1.record(st)
+            torch.cuda.synchronize()
+            ts.append(e0.elapsed_time(e1))
+        t = float(np.median(ts[1:])) / 1e3
+        out[name] = {"ms": round(t * 1e3, 3), "seq_s": round(B / t, 1), "tok_s": round(B * P / t, 1),
+                     "mean_exit_depth": round(float(ex.double().mean().item()), 3)}
+    adept.adept_set_option(m.h, adept.OPT_STOP_ENTIRELY, 0)
+    adept.adept_check_device_status(m.h)
+    m.close()
+    torch.cuda.empty_cache()
+    return {"workload": f"BERT-base shape, bf16, random-init; {B} x {P}-token classification batch", **out}
+
+
 def run_llama_e2e(adept, device, P=2048, steps=256):
     """Llama-2-7B shape, batch 1: 2048-token prompt + 256 greedy decode steps, exit layer per
     token ~ N(24, 4) truncated to [8, 32] -- against the same library forced to full depth."""
@@ -511,6 +549,7 @@ def ours(args, rank, world, device):
                            "mean_frac": round(float(np.mean([r["frac"] for r in rows])), 4)}
     if rank == 0 and not args.no_llama:
         line["llama7b_e2e"] = run_llama_e2e(adept, device)
+        line["encoder"] = run_encoder(adept, device)
     if rank == 0 and not args.no_cpu_baseline:
         line["cpu_baseline"] = cpu_baseline(args.cpu_tokens)
     return line

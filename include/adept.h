@@ -238,9 +238,12 @@ ADEPT_API adept_status adept_check_device_status(adept_model* m, void* stream);
  * when both reach delta; the reported similarity is their minimum).  ALL_AT_ONCE (App. H.2):
  * 1 makes every token of a prompt take the exit decision of its sequence's last prompt token,
  * so a sequence leaves at once (generation steps are unaffected: one token per sequence).
- * Default 0. */
+ * Default 0.  STOP_ENTIRELY (bf16 encoders; Sec. 4.3 on downstream tasks): 1 stops an exited
+ * token's computation entirely — no K/V of deeper layers, and deeper layers' attention sees
+ * only the tokens still active there; its mapped state still feeds the classifier.  Default 0. */
 enum { ADEPT_OPT_HSM_IDENTITY = 1, ADEPT_OPT_PROFILE = 2, ADEPT_OPT_GEMM_SIMT = 3, ADEPT_OPT_DECODE_GRAPH = 4,
-       ADEPT_OPT_DECODE_GEMM = 5, ADEPT_OPT_FUSED_DECODE = 6, ADEPT_OPT_EXIT_METRIC = 7, ADEPT_OPT_ALL_AT_ONCE = 8 };
+       ADEPT_OPT_DECODE_GEMM = 5, ADEPT_OPT_FUSED_DECODE = 6, ADEPT_OPT_EXIT_METRIC = 7, ADEPT_OPT_ALL_AT_ONCE = 8,
+       ADEPT_OPT_STOP_ENTIRELY = 9 };
 ADEPT_API adept_status adept_set_option(adept_model* m, int option, int value);
 
 /* Kernel classes reported by adept_profile_read: the GEMMs of prompt passes (layer

@@ -20,7 +20,7 @@ ADEPT_OK = 0
 STATUS_NAMES = {0: "OK", 1: "INVALID_ARG", 2: "OOM", 3: "CAPACITY", 4: "CUDA", 5: "TIMEOUT", 6: "DEVICE_INPUT"}
 FAMILY = {"llama": 0, "gpt2": 1, "bert": 2}
 OPT_HSM_IDENTITY, OPT_PROFILE, OPT_GEMM_SIMT, OPT_DECODE_GRAPH, OPT_DECODE_GEMM, OPT_FUSED_DECODE = 1, 2, 3, 4, 5, 6
-OPT_EXIT_METRIC, OPT_ALL_AT_ONCE = 7, 8
+OPT_EXIT_METRIC, OPT_ALL_AT_ONCE, OPT_STOP_ENTIRELY = 7, 8, 9
 EXIT_GLOBAL, EXIT_LOCAL, EXIT_BOTH = 0, 1, 2
 PROF_GEMM_PREFILL, PROF_KV_FILL, PROF_ATTENTION, PROF_GEMM_DECODE, PROF_DECODE_STEP = 0, 1, 2, 3, 4
 

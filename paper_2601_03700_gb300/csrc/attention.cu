@@ -122,7 +122,7 @@ __global__ void __launch_bounds__(128) attn_prefill_mma_kernel(const bf16* __res
                                                                const int* row_tok, const int* tok_seq,
                                                                const int* tok_pos, const int* seq_len,
                                                                KVCacheView cache, int layer0, int n_heads, int causal,
-                                                               float scale_log2) {
+                                                               float scale_log2, const int* key_exit, int kp_len) {
   PDL_ENTRY();
   constexpr int LDS = DH + 8;  // padded rows: conflict-free ldmatrix
   constexpr int NB = DH / 8;   // 8-column blocks of the output
@@ -131,6 +131,7 @@ __global__ void __launch_bounds__(128) attn_prefill_mma_kernel(const bf16* __res
   bf16* sK = sQ + 64 * LDS;
   bf16* sV = sK + 64 * LDS;
   __shared__ int s_seq[64], s_pos[64];
+  __shared__ int s_kv[64];   // key of the tile present (in range; with key_exit: still active)
 
   const int h = blockIdx.y;
   const int kvh = h / (n_heads / cache.n_kv_heads);
@@ -194,7 +195,10 @@ __global__ void __launch_bounds__(128) attn_prefill_mma_kernel(const bf16* __res
         const int p = kb + j;
         bf16* dk = sK + j * LDS + cc;
         bf16* dv = sV + j * LDS + cc;
-        if (p < kend) {
+        // "stop entirely": a token that left before this layer has no K/V here
+        const bool present = p < kend && (!key_exit || key_exit[sq * kp_len + p] > layer0);
+        if (cc == 0) s_kv[j] = present;
+        if (present) {
           const size_t off = cache.offset(layer0, sq, p, kvh) + cc;
           cp_async16(dk, Kp + off);
           cp_async16(dv, Vp + off);
@@ -230,8 +234,9 @@ __global__ void __launch_bounds__(128) attn_prefill_mma_kernel(const bf16* __res
 #pragma unroll
         for (int e = 0; e < 2; ++e) {
           const int key = kb + nb * 8 + 2 * t4 + e;
-          const bool ka = va && key < kend && (!causal || key <= pa);
-          const bool kb_ = vb && key < kend && (!causal || key <= pb);
+          const bool kp = s_kv[nb * 8 + 2 * t4 + e];
+          const bool ka = va && kp && (!causal || key <= pa);
+          const bool kb_ = vb && kp && (!causal || key <= pb);
           s[nb][e] = ka ? s[nb][e] * scale_log2 : -INFINITY;
           s[nb][2 + e] = kb_ ? s[nb][2 + e] * scale_log2 : -INFINITY;
           mx0 = fmaxf(mx0, s[nb][e]);
@@ -815,7 +820,7 @@ static int g_ad_smem_set[4] = {0, 0, 0, 0};
 void launch_attention(cudaStream_t st, int dt, const void* q, int ld_q, void* out, int ld_out, DevRange rows,
                       int max_rows, const int* row_tok, const int* tok_seq, const int* tok_pos, const int* seq_len,
                       KVCacheView cache, int layer0, int n_heads, int causal, int decode_keys, float* ws,
-                      int* counters, unsigned* err) {
+                      int* counters, unsigned* err, const int* key_exit, int kp_len) {
   if (max_rows <= 0) return;
   const int dh = cache.head_dim;
   const float scale_log2 = 1.4426950408889634f / sqrtf((float)dh);
@@ -898,7 +903,7 @@ void launch_attention(cudaStream_t st, int dt, const void* q, int ld_q, void* ou
       }
       launch_k(attn_prefill_mma_kernel<64>, grid, 128, smem, st, (const bf16*)q, ld_q, (bf16*)out, ld_out, rows, row_tok,
                                                            tok_seq, tok_pos, seq_len, cache, layer0, n_heads, causal,
-                                                           scale_log2);
+                                                           scale_log2, key_exit, kp_len);
     } else {
       if (!g_attn_smem_set[1]) {
         cudaFuncSetAttribute(attn_prefill_mma_kernel<128>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
@@ -906,7 +911,7 @@ void launch_attention(cudaStream_t st, int dt, const void* q, int ld_q, void* ou
       }
       launch_k(attn_prefill_mma_kernel<128>, grid, 128, smem, st, (const bf16*)q, ld_q, (bf16*)out, ld_out, rows, row_tok,
                                                             tok_seq, tok_pos, seq_len, cache, layer0, n_heads, causal,
-                                                            scale_log2);
+                                                            scale_log2, key_exit, kp_len);
     }
     return;
   }

@@ -16,10 +16,11 @@ enum : int {
 __host__ __device__ static inline int ctr_words(int n_layers) { return CTR_PREFIX + n_layers + 2; }
 
 // Token -> (sequence, position) maps, identity row map, the pass's counters (all rows
-// active) and, if sim is given, NaN for every (token, layer) similarity.
+// active), if sim is given NaN for every (token, layer) similarity, and if tok_exit is
+// given N as every token's exit layer so far.
 void launch_pass_init(cudaStream_t st, int n_tok, int prompt_len, int decode, int* tok_seq, int* tok_pos,
                       int* row_tok, int* seq_len, int seq_cap, int max_pos, unsigned* err, int* ctr, int n_ctr,
-                      float* sim, int n_layers);
+                      float* sim, int n_layers, int* tok_exit);
 // xhat (optional, decoders): the embedded rows standardised (smode, seps) in bf16, [n_tok][D].
 void launch_embed(cudaStream_t st, int dt, const int* tokens, int n_tok, const int* tok_pos, const void* E,
                   const void* P, const float* type_emb, const float* g, const float* b, int family, int D, int V,
@@ -82,11 +83,13 @@ void launch_gemm_simt(cudaStream_t st, int dt, const GemmProblem& p, int max_row
 // decode_keys > 0 (generation step, one query row per sequence): split-KV kernel over at
 // most decode_keys keys, using ws (>= rows * heads * ATTN_MAX_SPLIT * (head_dim + 2) floats)
 // and, for bf16, counters (>= rows * heads ints, zero between launches; the kernel leaves
-// them zero).
+// them zero).  key_exit (prompt passes, bf16; the encoder's "stop entirely" variant): the
+// exit layer so far of each token of the pass (token = sequence * kp_len + position); a key
+// whose token left before this layer is left out.
 constexpr int ATTN_MAX_SPLIT = 32;
 void launch_attention(cudaStream_t st, int dt, const void* q, int ld_q, void* out, int ld_out, DevRange rows,
                       int max_rows, const int* row_tok, const int* tok_seq, const int* tok_pos, const int* seq_len,
                       KVCacheView cache, int layer0, int n_heads, int causal, int decode_keys, float* ws,
-                      int* counters, unsigned* err);
+                      int* counters, unsigned* err, const int* key_exit = nullptr, int kp_len = 0);
 
 }  // namespace adept

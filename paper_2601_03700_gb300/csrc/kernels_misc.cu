@@ -16,12 +16,14 @@ namespace adept {
 // ---------------------------------------------------------------------------
 __global__ void pass_init_kernel(int n_tok, int prompt_len, int decode, int* tok_seq, int* tok_pos,
                                  int* row_tok, int* seq_len, int seq_cap, int max_pos, unsigned* err, int* ctr,
-                                 int n_ctr, float* sim, int n_layers) {
+                                 int n_ctr, float* sim, int n_layers, int* tok_exit) {
   PDL_ENTRY();
   const int t = blockIdx.x * blockDim.x + threadIdx.x;
   // the pass's counters: all active, nothing exited
   if (t < n_ctr) ctr[t] = t == CTR_ACTIVE ? n_tok : 0;
   if (t >= n_tok) return;
+  // every token active: its exit layer so far is N
+  if (tok_exit) tok_exit[t] = n_layers;
   // similarities not tested stay NaN
   if (sim)
     for (int l = 0; l < n_layers; ++l) sim[(size_t)t * n_layers + l] = __int_as_float(0x7fffffff);
@@ -900,9 +902,9 @@ __global__ void read_kv_kernel(KVCacheView c, int layer0, int seq, int pos0, int
 // ---------------------------------------------------------------------------
 void launch_pass_init(cudaStream_t st, int n_tok, int prompt_len, int decode, int* tok_seq, int* tok_pos,
                       int* row_tok, int* seq_len, int seq_cap, int max_pos, unsigned* err, int* ctr, int n_ctr,
-                      float* sim, int n_layers) {
+                      float* sim, int n_layers, int* tok_exit) {
   launch_k(pass_init_kernel, cdiv(std::max(n_tok, n_ctr), 256), 256, 0, st, n_tok, prompt_len, decode, tok_seq, tok_pos,
-           row_tok, seq_len, seq_cap, max_pos, err, ctr, n_ctr, sim, n_layers);
+           row_tok, seq_len, seq_cap, max_pos, err, ctr, n_ctr, sim, n_layers, tok_exit);
 }
 
 void launch_embed(cudaStream_t st, int dt, const int* tokens, int n_tok, const int* tok_pos, const void* E,

@@ -115,6 +115,8 @@ struct adept_model {
   int hsm_identity = 0, profile = 0, force_simt = 0, use_graph = 1, use_dg = 1, use_fused = 1;
   int exit_metric = 0;   // EXIT_GLOBAL / EXIT_LOCAL / EXIT_BOTH
   int all_at_once = 0;   // prompt passes: sequences leave with their last prompt token
+  int stop_entirely = 0; // encoders: exited tokens get no deeper K/V and leave deeper attention
+  int32_t* tok_exit = nullptr;   // stop-entirely passes: each token's exit layer so far
   // persistent generation-step kernel (small batches of bf16 decoders); NULL when not eligible
   DfState* df = nullptr;
   std::string df_why;
@@ -756,9 +758,13 @@ static adept_status run_pass(adept_model* m, int n_tok, int batch, int prompt_le
   const int amode = attn_norm_mode(m);
   const float eps = c.norm_eps;
   m->last_rows = n_tok;
+  // encoder "stop entirely" (Sec. 4.3, downstream tasks): exits are recorded in tok_exit
+  // (the attention leaves out keys of tokens gone before its layer) and get no fills
+  const bool stop = fam == ADEPT_FAMILY_BERT && m->stop_entirely && !decode;
+  int32_t* exit_w = stop ? m->tok_exit : exit_out;
   launch_pass_init(st, n_tok, prompt_len, decode ? 1 : 0, m->tok_seq, m->tok_pos, m->row_tok[0], m->d_seq_len,
                    m->max_blocks_per_seq * c.kv_block_tokens, fam == ADEPT_FAMILY_LLAMA ? 0 : c.max_pos,
-                   m->err_word, m->ctr, ctr_words(N), sim_out, N);
+                   m->err_word, m->ctr, ctr_words(N), sim_out, N, stop ? m->tok_exit : nullptr);
   // passes of at most DG_MAX_M rows (bf16 decoders): the producer of each layer's input
   // (the embedding, then the exit kernel) also writes it standardised into xn, and the O
   // projection hands the tile statistics of its output to the FFN input's GEMM
@@ -798,7 +804,7 @@ static adept_status run_pass(adept_model* m, int n_tok, int batch, int prompt_le
     pr[0].epi.cache = cv; pr[0].epi.layer0 = l0; pr[0].epi.n_q_cols = Dq; pr[0].epi.n_kv_cols = Dkv;
     pr[0].epi.head_dim = m->dh; pr[0].epi.rope = fam == ADEPT_FAMILY_LLAMA; pr[0].epi.rope_table = m->rope_table;
     // attention input: standardised (gain folded into W_qkv)
-    if (!decode && i >= 3) {
+    if (!decode && i >= 3 && !stop) {
       pr[1] = kv_problem(m, l0, m->xfill, n_tok, DevRange{nullptr, m->ctr + CTR_EXITED, 0}, m->exit_tok, m->tok_seq,
                          m->tok_pos);
       launch_standardize(st, m->dt, Xi, D, nullptr, act, mr, D, amode, eps, m->xn, D);
@@ -815,7 +821,8 @@ static adept_status run_pass(adept_model* m, int n_tok, int batch, int prompt_le
       cudaEvent_t b = nullptr;
       prof_begin(m, ADEPT_PROF_ATTENTION, st, &b);
       launch_attention(st, m->dt, m->q, Dq, m->att, Dq, act, mr, rt, m->tok_seq, m->tok_pos, m->d_seq_len, cv, l0,
-                       m->H, causal, decode_keys, m->attn_ws, m->attn_ctr, m->err_word);
+                       m->H, causal, decode_keys, m->attn_ws, m->attn_ctr, m->err_word, stop ? m->tok_exit : nullptr,
+                       prompt_len);
       prof_end(m, ADEPT_PROF_ATTENTION, st, b, 0, 0);
       m->launches += 1;
     }
@@ -861,7 +868,7 @@ static adept_status run_pass(adept_model* m, int n_tok, int batch, int prompt_le
       const int test = i >= 2;
       if (n_tok <= EXIT_SMALL_MAX) {
         xn_valid = launch_exit_small(st, Xi, m->X_out, Ii, i == 1, D, m->ctr, par, rt, m->row_tok[par ^ 1], forced, i,
-                                     N, m->d_delta, test, sim_out, m->exit_tok, exit_out, m->X_in[par ^ 1],
+                                     N, m->d_delta, test, sim_out, m->exit_tok, exit_w, m->X_in[par ^ 1],
                                      m->I[par ^ 1], m->hsm_s, m->hsm_prev, m->hsm_I, mr,
                                      dgrows ? (bf16*)m->xn : nullptr, amode, eps, m->exit_metric, aao_len,
                                      m->tok_pos, m->err_word) &&
@@ -870,7 +877,7 @@ static adept_status run_pass(adept_model* m, int n_tok, int batch, int prompt_le
       } else {
         launch_exit_decide(st, m->X_out, Ii, Xi, D, act, mr, rt, forced, i, N, m->d_delta, test, m->exit_metric,
                            sim_out, m->flag, m->inv_norm, m->err_word);
-        launch_exit_scan(st, m->ctr, par, m->flag, rt, m->row_tok[par ^ 1], m->exit_tok, m->dst, exit_out, i, aao_len,
+        launch_exit_scan(st, m->ctr, par, m->flag, rt, m->row_tok[par ^ 1], m->exit_tok, m->dst, exit_w, i, aao_len,
                          m->tok_pos);
         launch_exit_move(st, Xi, m->X_out, Ii, i == 1, D, m->ctr + CTR_ACTIVE + par, mr, m->dst, m->inv_norm,
                          m->X_in[par ^ 1], m->I[par ^ 1], m->hsm_s, m->hsm_prev, m->hsm_I);
@@ -882,10 +889,12 @@ static adept_status run_pass(adept_model* m, int n_tok, int batch, int prompt_le
       }
       par ^= 1;
     } else {
-      launch_final_scatter(st, m->X_out, D, m->ctr + CTR_ACTIVE + par, mr, rt, m->final_, exit_out, N);
+      launch_final_scatter(st, m->X_out, D, m->ctr + CTR_ACTIVE + par, mr, rt, m->final_, exit_w, N);
       m->launches += 1;
     }
   }
+  if (stop && exit_out)
+    CUDA_TRY(m, cudaMemcpyAsync(exit_out, m->tok_exit, (size_t)n_tok * sizeof(int32_t), cudaMemcpyDeviceToDevice, st));
   if (decode && N >= 3) {
     // Generation step: the step's tokens belong to different sequences, so the HSM and
     // the skipped-layer fills of all exits run once, after the layer loop: one HSM over
@@ -1315,6 +1324,12 @@ adept_status adept_set_option(adept_model* m, int option, int value) {
       drop_graphs(m);
       return ADEPT_OK;
     case ADEPT_OPT_ALL_AT_ONCE: m->all_at_once = value != 0; return ADEPT_OK;
+    case ADEPT_OPT_STOP_ENTIRELY:
+      if (value && (m->cfg.family != ADEPT_FAMILY_BERT || m->dt != ADEPT_DTYPE_BF16))
+        return fail(m, ADEPT_ERR_INVALID_ARG, "stop-entirely is defined for bf16 encoder models");
+      if (value && !m->tok_exit) TRY(dalloc_t(m, &m->tok_exit, (size_t)m->T_max));
+      m->stop_entirely = value != 0;
+      return ADEPT_OK;
   }
   return fail(m, ADEPT_ERR_INVALID_ARG, "unknown option %d", option);
 }

@@ -77,7 +77,7 @@ def decisions_agree_outside_band(g_sim: np.ndarray, o_sim: np.ndarray, delta: fl
 
 
 def run_prefill(pair: Pair, tokens: np.ndarray, delta: float, forced=None, hsm_identity=False, metric="global",
-                all_at_once=False):
+                all_at_once=False, stop_entirely=False):
     """Returns (oracle result, oracle cache, gpu outputs dict); in threshold mode with band
     tokens, the GPU is re-run with the oracle's exit layers forced.  metric / all_at_once:
     the exit-rule variant (the device options are set here too)."""
@@ -85,7 +85,9 @@ def run_prefill(pair: Pair, tokens: np.ndarray, delta: float, forced=None, hsm_i
     B, P = tokens.shape
     cache = O.OracleCache(cfg, cfg.max_batch, cfg.max_seq)
     ores = O.prefill(pair.om, cache, tokens, delta, forced, hsm_mode="identity" if hsm_identity else "hsm",
-                     metric=metric, all_at_once=all_at_once)
+                     metric=metric, all_at_once=all_at_once, stop_entirely=stop_entirely)
+    if cfg.family == synth.BERT:
+        adept.adept_set_option(pair.gm.h, adept.OPT_STOP_ENTIRELY, int(stop_entirely))
     adept.adept_set_option(pair.gm.h, adept.OPT_EXIT_METRIC, {"global": 0, "local": 1, "both": 2}[metric])
     adept.adept_set_option(pair.gm.h, adept.OPT_ALL_AT_ONCE, int(all_at_once))
     adept.adept_set_option(pair.gm.h, adept.OPT_HSM_IDENTITY, int(hsm_identity))
@@ -115,9 +117,9 @@ def run_prefill(pair: Pair, tokens: np.ndarray, delta: float, forced=None, hsm_i
 
 
 def compare_prefill(pair: Pair, tokens, delta, forced=None, hsm_identity=False, check_cache=True, metric="global",
-                    all_at_once=False):
+                    all_at_once=False, stop_entirely=False):
     B, P = tokens.shape
-    ores, cache, g = run_prefill(pair, tokens, delta, forced, hsm_identity, metric, all_at_once)
+    ores, cache, g = run_prefill(pair, tokens, delta, forced, hsm_identity, metric, all_at_once, stop_entirely)
     assert_rows_close(g["final"], ores.final, pair.tol, "final states")
     assert_rows_close(g["logits"], ores.logits, pair.tol, "logits")
     if pair.cfg.family != synth.BERT:

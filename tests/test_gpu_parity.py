@@ -323,3 +323,29 @@ def test_all_at_once_prompt_exits_match_oracle(dtype):
     ex = g["exit"].reshape(B, P)
     assert np.all(ex == ex[:, -1:])
     pair.close()
+
+
+def test_encoder_stop_entirely_matches_oracle():
+    """Encoder "stop entirely" (Sec. 4.3, downstream tasks): forced and threshold exits,
+    exited tokens left out of deeper attention and given no deeper K/V; final states,
+    classifier logits and every K/V the oracle wrote, against the oracle."""
+    from parity_utils import assert_rows_close
+    cfg = small(synth.BERT)
+    pair = Pair(cfg, seed=63)
+    B, P = 3, 40
+    tokens = synth.make_tokens(63, B, P, cfg.vocab).numpy()
+    forced = synth.forced_exits_uniform(63, B * P, 2, cfg.n_layers).numpy().reshape(B, P)
+    for fz, delta in ((forced, 0.9), (None, 0.6)):
+        ores, cache, g = compare_prefill(pair, tokens, delta, fz, check_cache=False, stop_entirely=True)
+        for l in range(1, cfg.n_layers + 1):
+            for b in range(B):
+                k, v = pair.gpu_kv(l, b, P)
+                ok = ~np.isnan(cache.K[l - 1][b, :P, 0, 0])   # written by the oracle: tokens active at l
+                if l == 1:
+                    assert ok.all()
+                if not ok.any():
+                    continue
+                assert_rows_close(k[ok], cache.K[l - 1][b, :P][ok], pair.tol, f"K layer {l} seq {b}")
+                assert_rows_close(v[ok], cache.V[l - 1][b, :P][ok], pair.tol, f"V layer {l} seq {b}")
+    adept.adept_set_option(pair.gm.h, adept.OPT_STOP_ENTIRELY, 0)
+    pair.close()
