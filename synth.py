@@ -339,3 +339,24 @@ def make_mapped_states(seed: int, n: int, d: int, dtype=torch.bfloat16, device="
                        name: str = "mapped") -> torch.Tensor:
     """Exit-state rows s~ ~ N(0, 1) for the skipped-layer KV-fill microbenchmark."""
     return normal(seed, name, (n, d), std=1.0, dtype=dtype, device=device)
+
+
+# ----------------------------------------------------------------------------
+# HSM training batches
+# ----------------------------------------------------------------------------
+
+def hsm_train_batch(cfg: ModelConfig, n: int, seed: int = 0, std: float = 1.0):
+    """n synthetic training examples of the Hidden State Mapper: (s_i, s_{i-1}, I, target).
+
+    Recipe: s_{i-1} ~ N(0, std^2) per element; s_i = s_{i-1} + N(0, (0.3 std)^2) (a layer's
+    residual update); I = (k - 1) unit(s_{i-1}) + N(0, 0.1^2) with the exit layer k uniform on
+    [2, N - 1] (the inertia sums k - 1 unit vectors of similar direction); the target is a
+    uniform token id on [0, vocab).  Returned as float32 [n, D] tensors and int32 [n]."""
+    D = cfg.d_model
+    s_prev = normal(seed, "hsm-train-s-prev", (n, D), std=std)
+    s_i = s_prev + normal(seed, "hsm-train-delta", (n, D), std=0.3 * std)
+    k = randint(seed, "hsm-train-layer", n, 2, max(2, cfg.n_layers - 1)).to(torch.float32)
+    u = s_prev / s_prev.norm(dim=1, keepdim=True).clamp_min(1e-30)
+    inertia = (k - 1)[:, None] * u + normal(seed, "hsm-train-inertia", (n, D), std=0.1)
+    target = randint(seed, "hsm-train-target", n, 0, cfg.vocab - 1)
+    return s_i.contiguous(), s_prev.contiguous(), inertia.contiguous(), target
