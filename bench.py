@@ -325,6 +325,65 @@ def run_encoder(adept, device, B=64, P=128):
     return {"workload": f"BERT-base shape, bf16, random-init; {B} x {P}-token classification batch", **out}
 
 
+def hsm_train_flops(cfg, n):
+    """GEMM FLOPs of one HSM training step on n examples: the four FC products forward, their
+    input and weight gradients (3 x 2 x FC weights per example), the head forward and its input
+    gradient (2 x 2 D V per example)."""
+    D, m1, m2 = cfg.d_model, cfg.hsm_m1, cfg.hsm_m2
+    fc = D * m1 + m1 * m2 + m2 * m1 + m1 * D
+    return n * (6.0 * fc + 4.0 * D * cfg.vocab)
+
+
+def run_hsm_train(adept, device, peaks, n=8192, reps=5):
+    """HSM training step (Sec. 4.2; App. D): GPT-2-small shape (D 768, HSM widths 3072 / 6144,
+    vocabulary 50257, bf16 GEMM operands, fp32 master weights and AdamW state), n synthetic
+    examples per step (128 sequences x 64 tokens).  Step time with CUDA events; the GEMMs'
+    share and TFLOP/s from per-GEMM events in a separate profiled step."""
+    cfg = synth.gpt2_small_config(n_layers=2, max_batch=1, max_seq=16)
+    W = synth.make_weights(cfg, seed=0, device=device)
+    m = adept.Model(cfg, W)
+    del W
+    s_i, s_prev, inertia, tgt = [x.to(device) for x in synth.hsm_train_batch(cfg, n, seed=1)]
+    adept.adept_hsm_train_init(m.h, n)
+    loss = torch.zeros(1, device=device)
+    st = torch.cuda.current_stream()
+    step = lambda: adept.adept_hsm_train_step(m.h, n, s_i, s_prev, inertia, tgt, 1e-4, 0.9, 0.999, 1e-8, 0.0,  # noqa
+                                              loss_out=loss)
+    step()
+    adept.adept_check_device_status(m.h)
+    first_loss = float(loss.item())
+    adept.adept_launch_count(m.h)
+    ts = []
+    for _ in range(reps):
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        torch.cuda.synchronize()
+        e0.record(st)
+        step()
+        e1.record(st)
+        torch.cuda.synchronize()
+        ts.append(e0.elapsed_time(e1))
+    launches = adept.adept_launch_count(m.h) // reps
+    t = float(np.median(ts)) / 1e3
+    fl = hsm_train_flops(cfg, n)
+    adept.adept_set_option(m.h, adept.OPT_PROFILE, 1)
+    step()
+    ng, gms, _, _ = adept.adept_profile_read(m.h, adept.PROF_GEMM_TRAIN)
+    adept.adept_set_option(m.h, adept.OPT_PROFILE, 0)
+    adept.adept_check_device_status(m.h)
+    last_loss = float(loss.item())
+    m.close()
+    torch.cuda.empty_cache()
+    peak = peaks["bf16_tflops_sustained"]
+    return {"workload": f"GPT-2-small shape HSM (768 -> 3072 -> 6144 -> 3072 -> 768) + frozen 50257-token head, "
+                        f"{n} examples/step, bf16 GEMM operands, fp32 AdamW",
+            "ms_per_step": round(t * 1e3, 3), "examples_s": round(n / t, 1), "gpu_launches": int(launches),
+            "gemm_tflop_per_step": round(fl / 1e12, 4), "tflops_step": round(fl / t / 1e12, 1),
+            "gemm_launches": int(ng), "gemm_ms_profiled": round(gms, 3),
+            "gemm_tflops_profiled": round(fl / (gms / 1e3) / 1e12, 1) if gms > 0 else None,
+            "gemm_frac_of_measured_sustained_bf16": round(fl / (gms / 1e3) / 1e12 / peak, 4) if gms > 0 else None,
+            "loss_first": round(first_loss, 5), "loss_after": round(last_loss, 5)}
+
+
 def run_llama_e2e(adept, device, P=2048, steps=256):
     """Llama-2-7B shape, batch 1: 2048-token prompt + 256 greedy decode steps, exit layer per
     token ~ N(24, 4) truncated to [8, 32] -- against the same library forced to full depth."""
@@ -550,6 +609,7 @@ def ours(args, rank, world, device):
     if rank == 0 and not args.no_llama:
         line["llama7b_e2e"] = run_llama_e2e(adept, device)
         line["encoder"] = run_encoder(adept, device)
+        line["hsm_train"] = run_hsm_train(adept, device, peaks)
     if rank == 0 and not args.no_cpu_baseline:
         line["cpu_baseline"] = cpu_baseline(args.cpu_tokens)
     return line

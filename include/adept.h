@@ -250,9 +250,9 @@ ADEPT_API adept_status adept_set_option(adept_model* m, int option, int value);
  * projections, HSM, head, and the per-layer skipped-layer fills co-launched with
  * layer i's QKV), the GEMMs of generation steps, the grouped skipped-layer fill
  * launches (end of a generation step and adept_skip_kv_fill), attention, and the
- * persistent generation-step launch (FUSED_DECODE). */
+ * persistent generation-step launch (FUSED_DECODE), and the GEMMs of HSM training steps. */
 enum { ADEPT_PROF_GEMM_PREFILL = 0, ADEPT_PROF_KV_FILL = 1, ADEPT_PROF_ATTENTION = 2,
-       ADEPT_PROF_GEMM_DECODE = 3, ADEPT_PROF_DECODE_STEP = 4, ADEPT_PROF_NCLASS = 5 };
+       ADEPT_PROF_GEMM_DECODE = 3, ADEPT_PROF_DECODE_STEP = 4, ADEPT_PROF_GEMM_TRAIN = 5, ADEPT_PROF_NCLASS = 6 };
 /* Synchronise, then return the number of recorded launches of kernel class `cls` and
  * their total device time in ms (CUDA events on the launching stream); resets the
  * record.  flops / bytes are reserved (returned as 0). */
@@ -264,6 +264,55 @@ ADEPT_API adept_status adept_profile_read(adept_model* m, int cls, int64_t* laun
  * does).  The reason string lives as long as the model. */
 ADEPT_API int adept_fused_decode_batch(const adept_model* m);
 ADEPT_API const char* adept_fused_decode_reason(const adept_model* m);
+
+/* ---- HSM training (Sec. 4.2; Sec. 5.1 "Training"; App. D) ----------------------------
+ * The Hidden State Mapper is trained with the base model frozen: its mapped state s~ of an
+ * example (s_i, s_{i-1}, I) goes through the frozen final norm and LM head, and the mean
+ * cross-entropy against the example's target token (the next input token) is minimised with
+ * AdamW (decoupled weight decay, bias-corrected moments).  Decoders only (the classification
+ * loss of encoders is not provided).
+ *
+ * Parameters, in this order (Table S1): 0 g0 [D], 1 conv_w [3][3], 2 conv_b [1], 3 fc1_w
+ * [m1][D], 4 fc1_b [m1], 5 fc2_w [m2][m1], 6 fc2_b [m2], 7 fc3_w [m1][m2], 8 fc3_b [m1], 9 g1
+ * [m1], 10 fc4_w [D][m1], 11 fc4_b [D], 12 g2 [D].  The library keeps fp32 master copies and
+ * the two AdamW moments of each; the products run on the model dtype's GEMMs (bf16 models:
+ * bf16 operands, fp32 accumulation), everything else in fp32.  After every step the model's
+ * own HSM weights (used by adept_prefill / adept_decode_step) hold the updated values. */
+typedef struct {
+  float lr, beta1, beta2, eps, weight_decay;
+} adept_adamw;
+
+/* Starts HSM training: master parameters from the model's current HSM weights, zero moments,
+ * step count 0, and device workspaces for up to max_rows examples per step (a second call
+ * frees the previous ones and starts over).  Synchronous on `stream`.
+ * Errors: INVALID_ARG (max_rows < 1, an encoder model, a bf16 model whose D, m1 or m2 is not
+ * a multiple of 8), OOM. */
+ADEPT_API adept_status adept_hsm_train_init(adept_model* m, int max_rows, void* stream);
+
+/* One training step on n examples, enqueued on `stream`: forward (Table S1) with the
+ * activations kept, frozen head, cross-entropy, backward, AdamW with step number t = (steps
+ * so far) + 1, write-back of the model's HSM weights.
+ *   d_s_i, d_s_prev, d_inertia  [n, D] fp32 device rows: s_i, s_{i-1} and I of each example
+ *   d_target                    [n] int32 device token ids in [0, vocab) (a bad id flags
+ *                               DEVICE_INPUT at adept_check_device_status; its row adds
+ *                               nothing to the loss or the gradients)
+ *   hp                          host pointer to the hyperparameters
+ *   d_loss_out                  device float: the mean loss before the update (NULL: not written)
+ * Errors: INVALID_ARG (no adept_hsm_train_init, n outside [1, max_rows], NULL pointers,
+ * lr < 0, beta outside [0, 1), eps <= 0, weight_decay < 0). */
+ADEPT_API adept_status adept_hsm_train_step(adept_model* m, int n, const float* d_s_i, const float* d_s_prev,
+                                  const float* d_inertia, const int32_t* d_target, const adept_adamw* hp,
+                                  float* d_loss_out, void* stream);
+
+/* Copies one parameter's fp32 training values to device memory d_out (count = its element
+ * count, adept_hsm_param_numel): what = ADEPT_HSM_PARAMS (master values), ADEPT_HSM_GRADS
+ * (gradients of the last step), ADEPT_HSM_MOMENT1 / ADEPT_HSM_MOMENT2 (AdamW moments).
+ * Enqueued on `stream`.  Errors: INVALID_ARG (no training state, bad what / param / count). */
+enum { ADEPT_HSM_PARAMS = 0, ADEPT_HSM_GRADS = 1, ADEPT_HSM_MOMENT1 = 2, ADEPT_HSM_MOMENT2 = 3 };
+ADEPT_API adept_status adept_hsm_train_read(adept_model* m, int what, int param, float* d_out, int64_t count,
+                                  void* stream);
+/* Element count of HSM parameter `param` (0..12), or -1. */
+ADEPT_API int64_t adept_hsm_param_numel(const adept_model* m, int param);
 
 /* Number of kernel launches the library enqueued since the last call (then reset). */
 ADEPT_API int64_t adept_launch_count(adept_model* m);

@@ -22,7 +22,11 @@ FAMILY = {"llama": 0, "gpt2": 1, "bert": 2}
 OPT_HSM_IDENTITY, OPT_PROFILE, OPT_GEMM_SIMT, OPT_DECODE_GRAPH, OPT_DECODE_GEMM, OPT_FUSED_DECODE = 1, 2, 3, 4, 5, 6
 OPT_EXIT_METRIC, OPT_ALL_AT_ONCE, OPT_STOP_ENTIRELY = 7, 8, 9
 EXIT_GLOBAL, EXIT_LOCAL, EXIT_BOTH = 0, 1, 2
-PROF_GEMM_PREFILL, PROF_KV_FILL, PROF_ATTENTION, PROF_GEMM_DECODE, PROF_DECODE_STEP = 0, 1, 2, 3, 4
+PROF_GEMM_PREFILL, PROF_KV_FILL, PROF_ATTENTION, PROF_GEMM_DECODE, PROF_DECODE_STEP, PROF_GEMM_TRAIN = 0, 1, 2, 3, 4, 5
+HSM_PARAMS, HSM_GRADS, HSM_MOMENT1, HSM_MOMENT2 = 0, 1, 2, 3
+# HSM parameters in the order of adept_hsm_train_read's `param` (Table S1)
+HSM_PARAM_NAMES = ["hsm.g0", "hsm.conv_w", "hsm.conv_b", "hsm.fc1_w", "hsm.fc1_b", "hsm.fc2_w", "hsm.fc2_b",
+                   "hsm.fc3_w", "hsm.fc3_b", "hsm.g1", "hsm.fc4_w", "hsm.fc4_b", "hsm.g2"]
 
 # every symbol declared in include/adept.h
 ABI_SYMBOLS = [
@@ -30,7 +34,8 @@ ABI_SYMBOLS = [
     "adept_last_error", "adept_status_string", "adept_seq_reserve", "adept_read_kv",
     "adept_read_final_states", "adept_check_device_status", "adept_set_option", "adept_profile_read",
     "adept_launch_count", "adept_skip_kv_fill_noalloc", "adept_fused_decode_batch", "adept_fused_decode_reason",
-    "adept_calibrate_threshold",
+    "adept_calibrate_threshold", "adept_hsm_train_init", "adept_hsm_train_step", "adept_hsm_train_read",
+    "adept_hsm_param_numel",
 ]
 
 
@@ -55,6 +60,11 @@ class AdeptConfig(ctypes.Structure):
 
 class AdeptTensor(ctypes.Structure):
     _fields_ = [("name", ctypes.c_char_p), ("data", ctypes.c_void_p), ("numel", ctypes.c_int64)]
+
+
+class AdeptAdamW(ctypes.Structure):
+    _fields_ = [("lr", ctypes.c_float), ("beta1", ctypes.c_float), ("beta2", ctypes.c_float),
+                ("eps", ctypes.c_float), ("weight_decay", ctypes.c_float)]
 
 
 class AdeptTensorTable(ctypes.Structure):
@@ -103,6 +113,14 @@ def load_library(path: str = LIB_PATH):
                                               ctypes.POINTER(c_float), ctypes.POINTER(c_float),
                                               ctypes.POINTER(c_int), st]
     lib.adept_calibrate_threshold.restype = c_int
+    lib.adept_hsm_train_init.argtypes = [vp, c_int, st]
+    lib.adept_hsm_train_init.restype = c_int
+    lib.adept_hsm_train_step.argtypes = [vp, c_int, fp, fp, fp, i32p, ctypes.POINTER(AdeptAdamW), fp, st]
+    lib.adept_hsm_train_step.restype = c_int
+    lib.adept_hsm_train_read.argtypes = [vp, c_int, c_int, fp, ctypes.c_int64, st]
+    lib.adept_hsm_train_read.restype = c_int
+    lib.adept_hsm_param_numel.argtypes = [vp, c_int]
+    lib.adept_hsm_param_numel.restype = ctypes.c_int64
     for name in ABI_SYMBOLS:
         fn = getattr(lib, name)
         if fn.restype is ctypes.c_int or name in ("adept_model_load", "adept_prefill", "adept_decode_step",
@@ -222,6 +240,34 @@ def adept_calibrate_threshold(m, batch: int, prompt_len: int, tokens: torch.Tens
     return d.value, r.value, n.value
 
 
+def adept_hsm_train_init(m, max_rows: int, stream=None):
+    """Master parameters from the model's HSM weights, zero AdamW moments, workspaces for
+    max_rows examples per step (Sec. 4.2; App. D)."""
+    lib = load_library()
+    _check(lib, m, lib.adept_hsm_train_init(m, int(max_rows), _stream(stream)))
+
+
+def adept_hsm_train_step(m, n: int, s_i: torch.Tensor, s_prev: torch.Tensor, inertia: torch.Tensor,
+                         target: torch.Tensor, lr: float, beta1: float = 0.9, beta2: float = 0.999,
+                         eps: float = 1e-8, weight_decay: float = 0.0, loss_out: Optional[torch.Tensor] = None,
+                         stream=None):
+    """One HSM training step: cross-entropy of the mapped state through the frozen head
+    against the target tokens, backward, AdamW."""
+    lib = load_library()
+    hp = AdeptAdamW(lr, beta1, beta2, eps, weight_decay)
+    _check(lib, m, lib.adept_hsm_train_step(m, int(n), _ptr(s_i), _ptr(s_prev), _ptr(inertia), _ptr(target),
+                                             ctypes.byref(hp), _ptr(loss_out), _stream(stream)))
+
+
+def adept_hsm_train_read(m, what: int, param: int, out: torch.Tensor, stream=None):
+    lib = load_library()
+    _check(lib, m, lib.adept_hsm_train_read(m, int(what), int(param), _ptr(out), out.numel(), _stream(stream)))
+
+
+def adept_hsm_param_numel(m, param: int) -> int:
+    return int(load_library().adept_hsm_param_numel(m, int(param)))
+
+
 def adept_free(m):
     if m:
         load_library().adept_free(m)
@@ -327,6 +373,11 @@ class Model:
 
     def check(self):
         adept_check_device_status(self.h)
+
+    def hsm_train_read(self, what: int, param: int) -> torch.Tensor:
+        out = torch.empty(adept_hsm_param_numel(self.h, param), dtype=torch.float32, device="cuda")
+        adept_hsm_train_read(self.h, what, param, out)
+        return out
 
     def fused_decode_batch(self) -> int:
         """Largest batch a generation step runs as one persistent launch (0: never)."""

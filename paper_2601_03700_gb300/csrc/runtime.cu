@@ -8,6 +8,7 @@
 #include "gemm_decode.h"
 #include "decode_fused.h"
 #include "model_view.h"
+#include "hsm_train.h"
 
 #include <algorithm>
 #include <cmath>
@@ -45,6 +46,30 @@ struct LayerW {
 struct ProfRec {
   std::vector<std::pair<cudaEvent_t, cudaEvent_t>> ev;
   std::vector<std::pair<double, double>> work;  // (flops, bytes) per recorded launch
+};
+
+// HSM training state (adept_hsm_train_*): fp32 master parameters, gradients and AdamW
+// moments in flat buffers (parameter i at off[i], each start 64-byte aligned except conv_b,
+// which follows conv_w so that the 10 convolution values stay contiguous), transposed weight
+// copies for the input-gradient products, and the per-step workspaces.
+enum { HT_G0, HT_CONV_W, HT_CONV_B, HT_FC1_W, HT_FC1_B, HT_FC2_W, HT_FC2_B, HT_FC3_W, HT_FC3_B, HT_G1, HT_FC4_W,
+       HT_FC4_B, HT_G2, HT_NPARAM };
+struct HsmTrain {
+  int cap = 0, ldTc = 0, Vp = 0, part_cols = 0;
+  long long step = 0;
+  long long off[HT_NPARAM + 1] = {};
+  long long numel[HT_NPARAM] = {};
+  std::vector<void*> mine;   // this state's allocations (also listed in the model's)
+  float *theta = nullptr, *grad = nullptr, *mom1 = nullptr, *mom2 = nullptr;
+  void *w1T = nullptr, *w2T = nullptr, *w3T = nullptr, *w4T = nullptr, *headT = nullptr;
+  int* iota = nullptr;
+  float *c0f = nullptr, *z1f = nullptr, *h1f = nullptr, *z2f = nullptr, *h3f = nullptr, *h5f = nullptr,
+        *stf = nullptr, *logits = nullptr, *lossr = nullptr, *dxh = nullptr, *dc0f = nullptr, *dh5f = nullptr,
+        *dh4f = nullptr, *dh3f = nullptr, *dh2f = nullptr, *r1 = nullptr, *r2 = nullptr, *cw = nullptr,
+        *part = nullptr;
+  void *c0t = nullptr, *c0T = nullptr, *h1t = nullptr, *h1T = nullptr, *h2t = nullptr, *h2T = nullptr,
+       *h4t = nullptr, *h4T = nullptr, *xht = nullptr, *dlt = nullptr, *dh5t = nullptr, *dh5T = nullptr,
+       *dh3t = nullptr, *dh3T = nullptr, *dz2t = nullptr, *dz2T = nullptr;
 };
 
 struct adept_model {
@@ -120,6 +145,7 @@ struct adept_model {
   // persistent generation-step kernel (small batches of bf16 decoders); NULL when not eligible
   DfState* df = nullptr;
   std::string df_why;
+  HsmTrain* ht = nullptr;   // HSM training state (adept_hsm_train_init)
   std::vector<cudaEvent_t> ev_pool;
   size_t ev_used = 0;
   int gemm_cls = ADEPT_PROF_GEMM_PREFILL;
@@ -182,6 +208,8 @@ static void drop_graphs(adept_model* m) {
 
 static void free_all(adept_model* m) {
   drop_graphs(m);
+  delete m->ht;
+  m->ht = nullptr;
   df_destroy(m->df);
   m->df = nullptr;
   if (m->cap_stream) cudaStreamDestroy(m->cap_stream);
@@ -943,6 +971,229 @@ static adept_status run_head(adept_model* m, int batch, int prompt_len, bool dec
   return ADEPT_OK;
 }
 
+static adept_status check_launch(adept_model* m) {
+  cudaError_t e = cudaGetLastError();
+  if (e != cudaSuccess) return fail(m, ADEPT_ERR_CUDA, "kernel launch failed: %s", cudaGetErrorString(e));
+  return ADEPT_OK;
+}
+
+// ---------------------------------------------------------------------------
+// HSM training step (Sec. 4.2; Sec. 5.1 "Training"; App. D)
+// ---------------------------------------------------------------------------
+
+static void ht_free(adept_model* m) {
+  if (!m->ht) return;
+  for (void* p : m->ht->mine) {
+    cudaFree(p);
+    m->allocs.erase(std::remove(m->allocs.begin(), m->allocs.end(), p), m->allocs.end());
+  }
+  delete m->ht;
+  m->ht = nullptr;
+}
+
+// C[M, N] (+)= A[M, K] B[N, K]^T (+ bias) into fp32 `out` (ld ldo); acc adds into out in place.
+static void ht_gemm(adept_model* m, cudaStream_t st, const void* A, int lda, int a_rows, const void* B, int ldb, int M,
+                    int N, int K, float* out, int ldo, const float* bias, bool acc) {
+  GemmProblem p;
+  memset(&p, 0, sizeof p);
+  p.A = A; p.lda = lda; p.a_rows = a_rows; p.B = B; p.ldb = ldb;
+  p.rows = DevRange{nullptr, nullptr, M}; p.N = N; p.K = K;
+  p.epi = epi_base(); p.epi.kind = acc ? EPI_RESID : EPI_F32; p.epi.bias = bias;
+  p.epi.out_f32 = out; p.epi.ld_f32 = ldo;
+  if (acc) { p.epi.resid = out; p.epi.ld_resid = ldo; }
+  gemm(m, st, &p, 1, &M, ADEPT_PROF_GEMM_TRAIN, 2.0 * M * N * K, 0);
+}
+
+static adept_status ht_init(adept_model* m, int cap, cudaStream_t st) {
+  const adept_config& c = m->cfg;
+  const int D = m->D, m1 = m->m1, m2 = m->m2, V = m->V, dt = m->dt;
+  const size_t es = m->esz;
+  ht_free(m);
+  m->ht = new HsmTrain();
+  HsmTrain& t = *m->ht;
+  t.cap = cap;
+  t.ldTc = (cap + 7) / 8 * 8;
+  t.Vp = (V + 7) / 8 * 8;
+  const long long n_el[HT_NPARAM] = {D, 9, 1, (long long)m1 * D, m1, (long long)m2 * m1, m2, (long long)m1 * m2,
+                                     m1, m1, (long long)D * m1, D, D};
+  long long o = 0;
+  for (int i = 0; i < HT_NPARAM; ++i) {
+    if (i != HT_CONV_B) o = (o + 15) / 16 * 16;
+    t.off[i] = o;
+    t.numel[i] = n_el[i];
+    o += n_el[i];
+  }
+  t.off[HT_NPARAM] = (o + 15) / 16 * 16;
+  const size_t P = (size_t)t.off[HT_NPARAM];
+  auto A = [&](auto** p, size_t bytes) -> adept_status {
+    TRY(dalloc(m, (void**)p, bytes));
+    t.mine.push_back((void*)*p);
+    return ADEPT_OK;
+  };
+  const size_t n = cap, L = t.ldTc;
+  TRY(A(&t.theta, P * 4)); TRY(A(&t.grad, P * 4)); TRY(A(&t.mom1, P * 4)); TRY(A(&t.mom2, P * 4));
+  TRY(A(&t.w1T, (size_t)m1 * D * es)); TRY(A(&t.w2T, (size_t)m2 * m1 * es));
+  TRY(A(&t.w3T, (size_t)m1 * m2 * es)); TRY(A(&t.w4T, (size_t)D * m1 * es));
+  TRY(A(&t.headT, (size_t)D * t.Vp * es));
+  TRY(A(&t.iota, n * 4));
+  TRY(A(&t.c0f, n * D * 4)); TRY(A(&t.z1f, n * m1 * 4)); TRY(A(&t.h1f, n * m1 * 4)); TRY(A(&t.z2f, n * m2 * 4));
+  TRY(A(&t.h3f, n * m1 * 4)); TRY(A(&t.h5f, n * D * 4)); TRY(A(&t.stf, n * D * 4)); TRY(A(&t.logits, n * V * 4));
+  TRY(A(&t.lossr, n * 4)); TRY(A(&t.dxh, n * D * 4)); TRY(A(&t.dc0f, n * D * 4)); TRY(A(&t.dh5f, n * D * 4));
+  TRY(A(&t.dh4f, n * m1 * 4)); TRY(A(&t.dh3f, n * m1 * 4)); TRY(A(&t.dh2f, n * m2 * 4));
+  TRY(A(&t.r1, n * 4)); TRY(A(&t.r2, n * 4)); TRY(A(&t.cw, n * 10 * 4));
+  t.part_cols = std::max({2 * D, 2 * m1, m2, D + 10});
+  TRY(A(&t.part, (size_t)ht_colsum_chunks(cap) * t.part_cols * 4));
+  TRY(A(&t.c0t, n * D * es)); TRY(A(&t.c0T, (size_t)D * L * es));
+  TRY(A(&t.h1t, n * m1 * es)); TRY(A(&t.h1T, (size_t)m1 * L * es));
+  TRY(A(&t.h2t, n * m2 * es)); TRY(A(&t.h2T, (size_t)m2 * L * es));
+  TRY(A(&t.h4t, n * m1 * es)); TRY(A(&t.h4T, (size_t)m1 * L * es));
+  TRY(A(&t.xht, n * D * es)); TRY(A(&t.dlt, n * t.Vp * es));
+  TRY(A(&t.dh5t, n * D * es)); TRY(A(&t.dh5T, (size_t)D * L * es));
+  TRY(A(&t.dh3t, n * m1 * es)); TRY(A(&t.dh3T, (size_t)m1 * L * es));
+  TRY(A(&t.dz2t, n * m2 * es)); TRY(A(&t.dz2T, (size_t)m2 * L * es));
+  if (dt != ADEPT_DTYPE_BF16 || m->force_simt) {
+    // SIMT GEMMs stage C in the model's scratch: size it for the largest training product now
+    const size_t big = std::max({n * (size_t)std::max({V, m2, m1, D}), (size_t)m1 * m2, (size_t)m1 * D});
+    if (!ensure_scratch(m, big)) return ADEPT_ERR_OOM;
+  }
+  // master parameters = the model's HSM weights; zero gradients and moments
+  CUDA_TRY(m, cudaMemsetAsync(t.theta, 0, P * 4, st));
+  CUDA_TRY(m, cudaMemsetAsync(t.grad, 0, P * 4, st));
+  CUDA_TRY(m, cudaMemsetAsync(t.mom1, 0, P * 4, st));
+  CUDA_TRY(m, cudaMemsetAsync(t.mom2, 0, P * 4, st));
+  const std::pair<int, const float*> vecs[] = {{HT_G0, m->hsm_g0}, {HT_FC1_B, m->hsm_b1}, {HT_FC2_B, m->hsm_b2},
+                                               {HT_FC3_B, m->hsm_b3}, {HT_G1, m->hsm_g1}, {HT_FC4_B, m->hsm_b4},
+                                               {HT_G2, m->hsm_g2}};
+  for (const auto& v : vecs)
+    CUDA_TRY(m, cudaMemcpyAsync(t.theta + t.off[v.first], v.second, t.numel[v.first] * 4, cudaMemcpyDeviceToDevice, st));
+  CUDA_TRY(m, cudaMemcpyAsync(t.theta + t.off[HT_CONV_W], m->hsm_conv, 10 * 4, cudaMemcpyDeviceToDevice, st));
+  launch_to_f32(st, dt, m->hsm_w1, t.theta + t.off[HT_FC1_W], (int)t.numel[HT_FC1_W]);
+  launch_to_f32(st, dt, m->hsm_w2, t.theta + t.off[HT_FC2_W], (int)t.numel[HT_FC2_W]);
+  launch_to_f32(st, dt, m->hsm_w3, t.theta + t.off[HT_FC3_W], (int)t.numel[HT_FC3_W]);
+  launch_to_f32(st, dt, m->hsm_w4, t.theta + t.off[HT_FC4_W], (int)t.numel[HT_FC4_W]);
+  // transposed copies: W1^T [D][m1], W2^T [m1][m2], W3^T [m2][m1], W4^T [m1][D], head^T [D][Vp]
+  ht_launch_transpose(st, dt, m->hsm_w1, m1, D, t.w1T, m1);
+  ht_launch_transpose(st, dt, m->hsm_w2, m2, m1, t.w2T, m2);
+  ht_launch_transpose(st, dt, m->hsm_w3, m1, m2, t.w3T, m1);
+  ht_launch_transpose(st, dt, m->hsm_w4, D, m1, t.w4T, D);
+  ht_launch_transpose(st, dt, m->w_head, V, D, t.headT, t.Vp);
+  std::vector<int> io(cap);
+  for (int i = 0; i < cap; ++i) io[i] = i;
+  CUDA_TRY(m, cudaMemcpyAsync(t.iota, io.data(), (size_t)cap * 4, cudaMemcpyHostToDevice, st));
+  CUDA_TRY(m, cudaStreamSynchronize(st));
+  (void)c;
+  return check_launch(m);
+}
+
+static adept_status ht_step(adept_model* m, int n, const float* s_i, const float* s_prev, const float* inertia,
+                            const int32_t* target, const adept_adamw& hp, float* loss, cudaStream_t st) {
+  HsmTrain& t = *m->ht;
+  const int D = m->D, m1 = m->m1, m2 = m->m2, V = m->V, Vp = t.Vp, dt = m->dt;
+  const int ldT = (n + 7) / 8 * 8;
+  const float eps = m->cfg.hsm_eps, neps = m->cfg.norm_eps;
+  const int hmode = attn_norm_mode(m);
+  const DevRange rows{nullptr, nullptr, n};
+  auto P = [&](int i) { return t.theta + t.off[i]; };
+  auto G = [&](int i) { return t.grad + t.off[i]; };
+  // forward (Table S1), keeping what the backward reads
+  launch_hsm_prep(st, dt, s_i, s_prev, inertia, rows, n, D, P(HT_G0), P(HT_CONV_W), eps, t.c0f, t.c0t);
+  ht_gemm(m, st, t.c0t, D, n, m->hsm_w1, D, n, m1, D, t.z1f, m1, P(HT_FC1_B), false);
+  ht_launch_act(st, dt, t.z1f, (long long)n * m1, t.h1f, t.h1t);
+  ht_gemm(m, st, t.h1t, m1, n, m->hsm_w2, m1, n, m2, m1, t.z2f, m2, P(HT_FC2_B), false);
+  ht_launch_act(st, dt, t.z2f, (long long)n * m2, nullptr, t.h2t);
+  ht_gemm(m, st, t.h2t, m2, n, m->hsm_w3, m2, n, m1, m2, t.h3f, m1, P(HT_FC3_B), false);
+  launch_hsm_mid(st, dt, t.h3f, t.h1f, rows, n, m1, P(HT_G1), eps, t.h4t);
+  ht_gemm(m, st, t.h4t, m1, n, m->hsm_w4, m1, n, D, m1, t.h5f, D, P(HT_FC4_B), false);
+  launch_hsm_out(st, dt, t.h5f, t.c0f, nullptr, 0, rows, n, D, P(HT_G2), eps, t.iota, t.stf, t.xht, hmode, neps);
+  // the frozen head (final-norm gain and shift folded into its weights) and the loss
+  ht_gemm(m, st, t.xht, D, n, m->w_head, D, n, V, D, t.logits, V, m->b_head, false);
+  ht_launch_ce(st, dt, t.logits, n, V, Vp, target, t.lossr, t.dlt, loss, m->err_word);
+  // backward
+  ht_gemm(m, st, t.dlt, Vp, n, t.headT, Vp, n, D, Vp, t.dxh, D, nullptr, false);
+  ht_launch_out_bwd(st, dt, t.dxh, t.stf, t.h5f, n, D, P(HT_G2), eps, hmode, neps, t.dc0f, t.dh5f, t.dh5t, t.r2);
+  int cl = 0;
+  {
+    ColJobs J{};
+    J.n = n; J.nj = 2;
+    J.j[0] = ColJob{t.dh5f, nullptr, nullptr, D, G(HT_FC4_B)};
+    J.j[1] = ColJob{t.dc0f, t.h5f, t.r2, D, G(HT_G2)};
+    cl += ht_launch_colsum(st, J, t.part);
+  }
+  ht_launch_transpose(st, dt, t.dh5t, n, D, t.dh5T, ldT);
+  ht_launch_transpose(st, dt, t.h4t, n, m1, t.h4T, ldT);
+  ht_gemm(m, st, t.dh5T, ldT, D, t.h4T, ldT, D, m1, ldT, G(HT_FC4_W), m1, nullptr, false);
+  ht_gemm(m, st, t.dh5t, D, n, t.w4T, D, n, m1, D, t.dh4f, m1, nullptr, false);
+  ht_launch_mid_bwd(st, dt, t.dh4f, t.h3f, n, m1, P(HT_G1), eps, t.dh3f, t.dh3t, t.r1);
+  {
+    ColJobs J{};
+    J.n = n; J.nj = 2;
+    J.j[0] = ColJob{t.dh4f, t.h3f, t.r1, m1, G(HT_G1)};
+    J.j[1] = ColJob{t.dh3f, nullptr, nullptr, m1, G(HT_FC3_B)};
+    cl += ht_launch_colsum(st, J, t.part);
+  }
+  ht_launch_transpose(st, dt, t.dh3t, n, m1, t.dh3T, ldT);
+  ht_launch_transpose(st, dt, t.h2t, n, m2, t.h2T, ldT);
+  ht_gemm(m, st, t.dh3T, ldT, m1, t.h2T, ldT, m1, m2, ldT, G(HT_FC3_W), m2, nullptr, false);
+  ht_gemm(m, st, t.dh3t, m1, n, t.w3T, m1, n, m2, m1, t.dh2f, m2, nullptr, false);
+  ht_launch_gelu_bwd(st, dt, t.dh2f, t.z2f, (long long)n * m2, t.dz2t);
+  {
+    ColJobs J{};
+    J.n = n; J.nj = 1;
+    J.j[0] = ColJob{t.dh2f, nullptr, nullptr, m2, G(HT_FC2_B)};
+    cl += ht_launch_colsum(st, J, t.part);
+  }
+  ht_launch_transpose(st, dt, t.dz2t, n, m2, t.dz2T, ldT);
+  ht_launch_transpose(st, dt, t.h1t, n, m1, t.h1T, ldT);
+  ht_gemm(m, st, t.dz2T, ldT, m2, t.h1T, ldT, m2, m1, ldT, G(HT_FC2_W), m1, nullptr, false);
+  ht_gemm(m, st, t.dz2t, m2, n, t.w2T, m2, n, m1, m2, t.dh4f, m1, nullptr, true);   // dh1 = dh4 + dz2 W2
+  ht_launch_gelu_bwd(st, dt, t.dh4f, t.z1f, (long long)n * m1, t.dh3t);            // dz1 (dh3's buffers are free)
+  {
+    ColJobs J{};
+    J.n = n; J.nj = 1;
+    J.j[0] = ColJob{t.dh4f, nullptr, nullptr, m1, G(HT_FC1_B)};
+    cl += ht_launch_colsum(st, J, t.part);
+  }
+  ht_launch_transpose(st, dt, t.dh3t, n, m1, t.dh3T, ldT);
+  ht_launch_transpose(st, dt, t.c0t, n, D, t.c0T, ldT);
+  ht_gemm(m, st, t.dh3T, ldT, m1, t.c0T, ldT, m1, D, ldT, G(HT_FC1_W), D, nullptr, false);
+  ht_gemm(m, st, t.dh3t, m1, n, t.w1T, m1, n, D, m1, t.dc0f, D, nullptr, true);     // dc0 += dz1 W1
+  ht_launch_prep_bwd(st, s_i, s_prev, inertia, t.dc0f, n, D, P(HT_G0), P(HT_CONV_W), eps, t.dh5f, t.cw);
+  {
+    ColJobs J{};
+    J.n = n; J.nj = 2;
+    J.j[0] = ColJob{t.dh5f, nullptr, nullptr, D, G(HT_G0)};
+    J.j[1] = ColJob{t.cw, nullptr, nullptr, 10, G(HT_CONV_W)};
+    cl += ht_launch_colsum(st, J, t.part);
+  }
+  // AdamW, writing the updated values back into the model's HSM weights
+  t.step += 1;
+  AdamArgs a{};
+  a.theta = t.theta; a.grad = t.grad; a.m = t.mom1; a.v = t.mom2;
+  a.lr = hp.lr; a.b1 = hp.beta1; a.b2 = hp.beta2; a.eps = hp.eps; a.wd = hp.weight_decay;
+  a.ibc1 = (float)(1.0 / (1.0 - std::pow((double)hp.beta1, (double)t.step)));
+  a.ibc2 = (float)(1.0 / (1.0 - std::pow((double)hp.beta2, (double)t.step)));
+  const AdamSeg segs[] = {
+      {t.off[HT_G0], 1, D, m->hsm_g0, nullptr, nullptr, 0, 0},
+      {t.off[HT_CONV_W], 1, 10, m->hsm_conv, nullptr, nullptr, 0, 0},
+      {t.off[HT_FC1_W], m1, D, nullptr, m->hsm_w1, t.w1T, 0, 0},
+      {t.off[HT_FC1_B], 1, m1, m->hsm_b1, nullptr, nullptr, 0, 0},
+      {t.off[HT_FC2_W], m2, m1, nullptr, m->hsm_w2, t.w2T, 0, 0},
+      {t.off[HT_FC2_B], 1, m2, m->hsm_b2, nullptr, nullptr, 0, 0},
+      {t.off[HT_FC3_W], m1, m2, nullptr, m->hsm_w3, t.w3T, 0, 0},
+      {t.off[HT_FC3_B], 1, m1, m->hsm_b3, nullptr, nullptr, 0, 0},
+      {t.off[HT_G1], 1, m1, m->hsm_g1, nullptr, nullptr, 0, 0},
+      {t.off[HT_FC4_W], D, m1, nullptr, m->hsm_w4, t.w4T, 0, 0},
+      {t.off[HT_FC4_B], 1, D, m->hsm_b4, nullptr, nullptr, 0, 0},
+      {t.off[HT_G2], 1, D, m->hsm_g2, nullptr, nullptr, 0, 0}};
+  a.nseg = (int)(sizeof segs / sizeof segs[0]);
+  for (int i = 0; i < a.nseg; ++i) a.seg[i] = segs[i];
+  ht_launch_adamw(st, dt, a);
+  // launches outside ht_gemm: prep, 2 act, mid, out, ce (+ loss), out_bwd, mid_bwd, 2 gelu_bwd, prep_bwd,
+  // 8 transposes, the column sums and AdamW
+  m->launches += 20 + (loss ? 1 : 0) + cl;
+  return check_launch(m);
+}
+
 // Plan of the persistent generation-step kernel (bf16 decoders; see decode_fused.cu).
 static void build_fused(adept_model* m) {
   const adept_config& c = m->cfg;
@@ -982,11 +1233,6 @@ static void build_fused(adept_model* m) {
   m->use_fused = 0;
 }
 
-static adept_status check_launch(adept_model* m) {
-  cudaError_t e = cudaGetLastError();
-  if (e != cudaSuccess) return fail(m, ADEPT_ERR_CUDA, "kernel launch failed: %s", cudaGetErrorString(e));
-  return ADEPT_OK;
-}
 
 // ---------------------------------------------------------------------------
 // C ABI
@@ -1369,6 +1615,56 @@ const char* adept_fused_decode_reason(const adept_model* m) {
   return m->df ? "" : m->df_why.c_str();
 }
 
+adept_status adept_hsm_train_init(adept_model* m, int max_rows, void* stream) {
+  if (!m) return ADEPT_ERR_INVALID_ARG;
+  g_pdl = !m->profile;
+  if (max_rows < 1) return fail(m, ADEPT_ERR_INVALID_ARG, "max_rows %d < 1", max_rows);
+  if (m->cfg.family == ADEPT_FAMILY_BERT)
+    return fail(m, ADEPT_ERR_INVALID_ARG, "HSM training takes decoders (next-token cross-entropy)");
+  if (m->dt == ADEPT_DTYPE_BF16 && ((m->D | m->m1 | m->m2) & 7))
+    return fail(m, ADEPT_ERR_INVALID_ARG, "bf16 HSM training needs D, m1, m2 multiples of 8");
+  const adept_status s = ht_init(m, max_rows, (cudaStream_t)stream);
+  if (s != ADEPT_OK) ht_free(m);
+  return s;
+}
+
+adept_status adept_hsm_train_step(adept_model* m, int n, const float* d_s_i, const float* d_s_prev,
+                                  const float* d_inertia, const int32_t* d_target, const adept_adamw* hp,
+                                  float* d_loss_out, void* stream) {
+  if (!m) return ADEPT_ERR_INVALID_ARG;
+  g_pdl = !m->profile;
+  if (!m->ht) return fail(m, ADEPT_ERR_INVALID_ARG, "adept_hsm_train_init has not run");
+  if (n < 1 || n > m->ht->cap) return fail(m, ADEPT_ERR_INVALID_ARG, "n %d outside [1, %d]", n, m->ht->cap);
+  if (!d_s_i || !d_s_prev || !d_inertia || !d_target || !hp) return fail(m, ADEPT_ERR_INVALID_ARG, "NULL pointer");
+  if (!(hp->lr >= 0.f) || !(hp->beta1 >= 0.f && hp->beta1 < 1.f) || !(hp->beta2 >= 0.f && hp->beta2 < 1.f) ||
+      !(hp->eps > 0.f) || !(hp->weight_decay >= 0.f))
+    return fail(m, ADEPT_ERR_INVALID_ARG, "AdamW hyperparameters out of range");
+  return ht_step(m, n, d_s_i, d_s_prev, d_inertia, d_target, *hp, d_loss_out, (cudaStream_t)stream);
+}
+
+adept_status adept_hsm_train_read(adept_model* m, int what, int param, float* d_out, int64_t count, void* stream) {
+  if (!m) return ADEPT_ERR_INVALID_ARG;
+  if (!m->ht) return fail(m, ADEPT_ERR_INVALID_ARG, "adept_hsm_train_init has not run");
+  if (param < 0 || param >= HT_NPARAM) return fail(m, ADEPT_ERR_INVALID_ARG, "param %d outside [0, 12]", param);
+  const HsmTrain& t = *m->ht;
+  const float* base = what == ADEPT_HSM_PARAMS ? t.theta : what == ADEPT_HSM_GRADS ? t.grad
+                      : what == ADEPT_HSM_MOMENT1 ? t.mom1 : what == ADEPT_HSM_MOMENT2 ? t.mom2 : nullptr;
+  if (!base) return fail(m, ADEPT_ERR_INVALID_ARG, "what %d unknown", what);
+  if (!d_out || count != t.numel[param])
+    return fail(m, ADEPT_ERR_INVALID_ARG, "count %lld != %lld", (long long)count, t.numel[param]);
+  CUDA_TRY(m, cudaMemcpyAsync(d_out, base + t.off[param], (size_t)count * 4, cudaMemcpyDeviceToDevice,
+                              (cudaStream_t)stream));
+  return ADEPT_OK;
+}
+
+int64_t adept_hsm_param_numel(const adept_model* m, int param) {
+  if (!m || param < 0 || param >= HT_NPARAM) return -1;
+  const int D = m->D, m1 = m->m1, m2 = m->m2;
+  const int64_t n[HT_NPARAM] = {D, 9, 1, (int64_t)m1 * D, m1, (int64_t)m2 * m1, m2, (int64_t)m1 * m2, m1, m1,
+                                (int64_t)D * m1, D, D};
+  return n[param];
+}
+
 int64_t adept_launch_count(adept_model* m) {
   if (!m) return 0;
   const int64_t n = m->launches;
@@ -1385,6 +1681,7 @@ void kt_attach_simt(void*, unsigned*, unsigned);
 void kt_attach_misc(void*, unsigned*, unsigned);
 void kt_attach_tc(void*, unsigned*, unsigned);
 void kt_attach_dg(void*, unsigned*, unsigned);
+void kt_attach_hsm_train(void*, unsigned*, unsigned);
 }  // namespace adept
 // Debug build only: points every kernel's timeline records at dev_buf (cap records of 104
 // bytes) and the device counter dev_cnt (NULL buffer: recording off).
@@ -1394,6 +1691,7 @@ extern "C" ADEPT_API void adept_debug_ktrace(void* dev_buf, unsigned* dev_cnt, u
   kt_attach_misc(dev_buf, dev_cnt, cap);
   kt_attach_tc(dev_buf, dev_cnt, cap);
   kt_attach_dg(dev_buf, dev_cnt, cap);
+  kt_attach_hsm_train(dev_buf, dev_cnt, cap);
 }
 #endif
 

@@ -54,3 +54,7 @@ def test_status_strings_and_load_validation_without_gpu(lib):
     assert lib.adept_prefill(None, 1, 1, None, ctypes.c_float(0.5), None, None, None, None, None, None) == 1
     assert lib.adept_set_option(None, 1, 1) == 1
     assert lib.adept_launch_count(None) == 0
+    assert lib.adept_hsm_train_init(None, 8, None) == 1
+    assert lib.adept_hsm_train_step(None, 1, None, None, None, None, None, None, None) == 1
+    assert lib.adept_hsm_train_read(None, 0, 0, None, 0, None) == 1
+    assert lib.adept_hsm_param_numel(None, 0) == -1
