@@ -770,10 +770,29 @@ def kernel_case_llama_decode_small(device):
     m.close()
 
 
+def kernel_case_hsm_train(device, n=8192, steps=2):
+    """HSM training steps at GPT-2-small shapes (the bench section's workload): n examples,
+    two steps after one warm-up step; about 5 GB on the device."""
+    import paper_2601_03700_gb300 as adept
+    adept.load_library()
+    cfg = synth.gpt2_small_config(n_layers=2, max_batch=1, max_seq=16)
+    W = synth.make_weights(cfg, seed=0)   # on the host: the launch list then holds the library's kernels only
+    m = adept.Model(cfg, W)
+    del W
+    s_i, s_prev, inertia, tgt = [x.to(device) for x in synth.hsm_train_batch(cfg, n, seed=1)]
+    adept.adept_hsm_train_init(m.h, n)
+    for _ in range(steps + 1):
+        adept.adept_hsm_train_step(m.h, n, s_i, s_prev, inertia, tgt, 1e-4)
+    torch.cuda.synchronize()
+    m.check()
+    print(json.dumps({"kernel_case": "hsm_train", "n": n, "steps": steps + 1, "ok": True}))
+    m.close()
+
+
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--kernel-case", default=None,
-                    choices=["fill_small", "llama_prefill", "gpt2_decode", "llama_decode_small"])
+                    choices=["fill_small", "llama_prefill", "gpt2_decode", "llama_decode_small", "hsm_train"])
     ap.add_argument("--gpus", type=int, default=1)
     ap.add_argument("--steps", type=int, default=5)
     ap.add_argument("--warmup", type=int, default=3)
@@ -784,6 +803,7 @@ def main():
     ap.add_argument("--fill-T", default="1,16,256,1024,4096,16384,65536")
     ap.add_argument("--fill-i", default="4,8,16,24")
     ap.add_argument("--cpu-tokens", type=int, default=512)
+    ap.add_argument("--hsm-n", type=int, default=8192, help="examples per step of --kernel-case hsm_train")
     args = ap.parse_args()
     if args.kernel_case == "fill_small":
         kernel_case_fill_small(torch.device("cuda", 0))
@@ -796,6 +816,9 @@ def main():
         return
     if args.kernel_case == "llama_decode_small":
         kernel_case_llama_decode_small(torch.device("cuda", 0))
+        return
+    if args.kernel_case == "hsm_train":
+        kernel_case_hsm_train(torch.device("cuda", 0), n=args.hsm_n)
         return
     world = int(os.environ.get("WORLD_SIZE", "1"))
     rank = int(os.environ.get("RANK", "0"))

@@ -205,6 +205,7 @@ __global__ void __launch_bounds__(TC_THREADS, 1) gemm_tc_kernel(const __grid_con
 
   __shared__ int s_tile0[MAXG + 1];
   __shared__ int s_mbeg[MAXG], s_M[MAXG], s_tn[MAXG], s_tm[MAXG], s_gm[MAXG];
+  __shared__ float s_bias[4][BN];   // epilogue: each warp's copy of the tile's bias columns
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int ng = p.n_groups;
@@ -415,6 +416,16 @@ __global__ void __launch_bounds__(TC_THREADS, 1) gemm_tc_kernel(const __grid_con
       const int ra = s_mbeg[g] + r;
       EpiRow rr{-1, 0};
       if (valid) rr = epi_row(G.epi, ra);
+      // the tile's bias columns, loaded once per warp (coalesced) while the accumulator fills,
+      // instead of 32 broadcast loads per row chunk after it
+      const float* bias = G.epi.bias;
+      if (bias) {
+        for (int c = lane; c < BN; c += 32) {
+          const int col = nb * BN + c;
+          s_bias[q][c] = col < G.N ? bias[col] : 0.f;
+        }
+        __syncwarp();
+      }
       // one lane per warp polls the barrier (128 pollers would crowd the barrier unit the
       // producer and MMA threads need); the result is broadcast to the warp
       bool got = true;
@@ -429,7 +440,7 @@ __global__ void __launch_bounds__(TC_THREADS, 1) gemm_tc_kernel(const __grid_con
         float v[32];
         tmem_ld32(tb + (uint32_t)c, v);
         const int c0 = nb * BN + c;
-        if (valid && c0 < G.N) epi_chunk32<bf16>(G.epi, ra, c0, G.N, v, rr);
+        if (valid && c0 < G.N) epi_chunk32<bf16>(G.epi, ra, c0, G.N, v, rr, bias ? &s_bias[q][c] : nullptr);
       }
       tc_fence_before();
       __syncwarp();

@@ -21,49 +21,66 @@ namespace {
 // forward
 // ---------------------------------------------------------------------------
 
-// h = GELU_erf(z) elementwise over count values; hf (optional) keeps it in fp32.
-template <typename T>
-__global__ void ht_act_kernel(const float* __restrict__ z, long long count, float* hf, T* ht) {
-  PDL_ENTRY();
-  for (long long i = (long long)blockIdx.x * blockDim.x + threadIdx.x; i < count; i += (long long)gridDim.x * blockDim.x) {
-    const float h = gelu_erf_f(z[i]);
-    if (hf) hf[i] = h;
-    ht[i] = from_f<T>(h);
-  }
+template <typename T> __device__ __forceinline__ void store4(T* p, float a, float b, float c, float d);
+template <> __device__ __forceinline__ void store4<float>(float* p, float a, float b, float c, float d) {
+  *reinterpret_cast<float4*>(p) = make_float4(a, b, c, d);
+}
+template <> __device__ __forceinline__ void store4<bf16>(bf16* p, float a, float b, float c, float d) {
+  __nv_bfloat162 lo = __floats2bfloat162_rn(a, b), hi = __floats2bfloat162_rn(c, d);
+  uint2 u;
+  u.x = *reinterpret_cast<unsigned*>(&lo);
+  u.y = *reinterpret_cast<unsigned*>(&hi);
+  *reinterpret_cast<uint2*>(p) = u;
 }
 
 // Softmax cross-entropy of one row of logits against its target (one CTA per row):
 // lossr[r] = logsumexp(l) - l[target]; dl[r][v] = (softmax(l)_v - [v == target]) / n for
 // v < V and 0 for the padding columns V..Vp-1.  A target outside [0, V) flags ERRW_TOKEN and
-// leaves a zero loss and gradient for the row.
+// leaves a zero loss and gradient for the row.  Rows are read as float4 groups (ldl and Vp
+// multiples of 4; columns at or past V are masked), four groups in flight per thread; the
+// second pass finds the row in L2.
 template <typename T>
-__global__ void __launch_bounds__(512) ht_ce_kernel(const float* __restrict__ logits, int V, int Vp,
+__global__ void __launch_bounds__(512) ht_ce_kernel(const float* __restrict__ logits, int ldl, int V, int Vp,
                                                     const int* __restrict__ target, float inv_n, float* lossr, T* dl,
                                                     unsigned* err) {
   PDL_ENTRY();
   __shared__ float red[32];
   __shared__ float rmax[32];
   const int r = blockIdx.x;
-  const float* l = logits + (size_t)r * V;
+  const float4* l4 = reinterpret_cast<const float4*>(logits + (size_t)r * ldl);
   T* g = dl + (size_t)r * Vp;
+  const int n4 = Vp >> 2;
   const int tg = target[r];
   if (tg < 0 || tg >= V) {
     if (threadIdx.x == 0) {
       atomicOr(err, ERRW_TOKEN);
       lossr[r] = 0.f;
     }
-    for (int v = threadIdx.x; v < Vp; v += blockDim.x) g[v] = from_f<T>(0.f);
+    for (int j = threadIdx.x; j < n4; j += blockDim.x) store4<T>(g + 4 * j, 0.f, 0.f, 0.f, 0.f);
     return;
   }
   // online (max, sum of exp) per thread, then across the block
   float mx = -INFINITY, s = 0.f;
-  for (int v = threadIdx.x; v < V; v += blockDim.x) {
-    const float x = l[v];
-    if (x > mx) {
-      s = s * expf(mx - x) + 1.f;
-      mx = x;
-    } else {
-      s += expf(x - mx);
+  constexpr int U = 4;
+  for (int j0 = threadIdx.x; j0 < n4; j0 += U * blockDim.x) {
+    float4 x[U];
+#pragma unroll
+    for (int u = 0; u < U; ++u) {
+      const int j = j0 + u * blockDim.x;
+      x[u] = j < n4 ? l4[j] : make_float4(-INFINITY, -INFINITY, -INFINITY, -INFINITY);
+    }
+#pragma unroll
+    for (int u = 0; u < U; ++u) {
+      const int v = 4 * (j0 + u * blockDim.x);
+      const float a0 = v < V ? x[u].x : -INFINITY, a1 = v + 1 < V ? x[u].y : -INFINITY;
+      const float a2 = v + 2 < V ? x[u].z : -INFINITY, a3 = v + 3 < V ? x[u].w : -INFINITY;
+      const float m4 = fmaxf(fmaxf(a0, a1), fmaxf(a2, a3));
+      if (m4 == -INFINITY) continue;
+      if (m4 > mx) {
+        s *= expf(mx - m4);
+        mx = m4;
+      }
+      s += expf(a0 - mx) + expf(a1 - mx) + expf(a2 - mx) + expf(a3 - mx);
     }
   }
   const int lane = threadIdx.x & 31, w = threadIdx.x >> 5, nw = blockDim.x >> 5;
@@ -74,11 +91,16 @@ __global__ void __launch_bounds__(512) ht_ce_kernel(const float* __restrict__ lo
   for (int i = 0; i < nw; ++i) bm = fmaxf(bm, rmax[i]);
   const float S = block_sum(mx == -INFINITY ? 0.f : s * expf(mx - bm), red);
   const float inv_s = 1.f / S;
-  if (threadIdx.x == 0) lossr[r] = logf(S) + bm - l[tg];
-  for (int v = threadIdx.x; v < Vp; v += blockDim.x) {
-    float d = 0.f;
-    if (v < V) d = (expf(l[v] - bm) * inv_s - (v == tg ? 1.f : 0.f)) * inv_n;
-    g[v] = from_f<T>(d);
+  if (threadIdx.x == 0) lossr[r] = logf(S) + bm - reinterpret_cast<const float*>(l4)[tg];
+  for (int j = threadIdx.x; j < n4; j += blockDim.x) {
+    const float4 x = l4[j];
+    const int v = 4 * j;
+    const float xv[4] = {x.x, x.y, x.z, x.w};
+    float d[4];
+#pragma unroll
+    for (int q = 0; q < 4; ++q)
+      d[q] = v + q < V ? (expf(xv[q] - bm) * inv_s - (v + q == tg ? 1.f : 0.f)) * inv_n : 0.f;
+    store4<T>(g + v, d[0], d[1], d[2], d[3]);
   }
 }
 
@@ -102,14 +124,22 @@ __global__ void ht_loss_kernel(const float* lossr, int n, float scale, float* lo
 //   dst = rstd (dxh - mean(dxh) - xh mean(dxh xh))          (LN; RMS drops mean(dxh))
 //   dc0 = dst;  dr = dst g2;  dh5 = r2 (dr - rh mean(dr rh)),  rh = h5 r2
 // Writes dc0 (fp32), dh5 (fp32 and T) and r2 (for the g2 column sum).
+// dxh arrives as nsplit partial sums (K-split parts of the head's input-gradient product),
+// split_stride floats apart.
 template <typename T>
-__global__ void ht_out_bwd_kernel(const float* __restrict__ dxh, const float* __restrict__ st,
-                                  const float* __restrict__ h5, int D, const float* __restrict__ g2, float eps,
-                                  int mode, float norm_eps, float* dc0, float* dh5f, T* dh5t, float* r2_out) {
+__global__ void ht_out_bwd_kernel(const float* __restrict__ dxh, int nsplit, size_t split_stride,
+                                  const float* __restrict__ st, const float* __restrict__ h5, int D,
+                                  const float* __restrict__ g2, float eps, int mode, float norm_eps, float* dc0,
+                                  float* dh5f, T* dh5t, float* r2_out) {
   PDL_ENTRY();
   __shared__ float red[32];
   const size_t o = (size_t)blockIdx.x * D;
-  const float *x = dxh + o, *f = st + o, *h = h5 + o;
+  const float *f = st + o, *h = h5 + o;
+  auto X = [&](int d) {
+    float v = dxh[o + d];
+    for (int s = 1; s < nsplit; ++s) v += dxh[s * split_stride + o + d];
+    return v;
+  };
   float mu = 0.f;
   if (mode == NORM_LN) {
     float s = 0.f;
@@ -124,14 +154,15 @@ __global__ void ht_out_bwd_kernel(const float* __restrict__ dxh, const float* __
   const float rs = rsqrtf(block_sum(s2, red) / D + norm_eps);
   float sa = 0.f, sb = 0.f;
   for (int d = threadIdx.x; d < D; d += blockDim.x) {
-    sa += x[d];
-    sb += x[d] * (f[d] - mu) * rs;
+    const float xd = X(d);
+    sa += xd;
+    sb += xd * (f[d] - mu) * rs;
   }
   const float ma = mode == NORM_LN ? block_sum(sa, red) / D : 0.f;
   const float mb = block_sum(sb, red) / D;
   float q2 = 0.f;
   for (int d = threadIdx.x; d < D; d += blockDim.x) {
-    const float v = rs * (x[d] - ma - (f[d] - mu) * rs * mb);
+    const float v = rs * (X(d) - ma - (f[d] - mu) * rs * mb);
     dc0[o + d] = v;
     q2 += h[d] * h[d];
   }
@@ -168,19 +199,6 @@ __global__ void ht_mid_bwd_kernel(const float* __restrict__ dh4, const float* __
     dh3t[o + d] = from_f<T>(v);
   }
   if (threadIdx.x == 0) r1_out[blockIdx.x] = r1;
-}
-
-// dz = dh * GELU_erf'(z) in place over count values (GELU'(z) = Phi(z) + z phi(z)), and its T copy.
-template <typename T>
-__global__ void ht_gelu_bwd_kernel(float* dh, const float* __restrict__ z, long long count, T* dzt) {
-  PDL_ENTRY();
-  for (long long i = (long long)blockIdx.x * blockDim.x + threadIdx.x; i < count; i += (long long)gridDim.x * blockDim.x) {
-    const float x = z[i];
-    const float gp = 0.5f * (1.f + erff(x * 0.70710678118654752f)) + x * 0.39894228040143268f * expf(-0.5f * x * x);
-    const float v = dh[i] * gp;
-    dh[i] = v;
-    dzt[i] = from_f<T>(v);
-  }
 }
 
 // Through the convolution and the input RMSNorms (one CTA per row).  With Xn_a = xh_a g0,
@@ -254,15 +272,62 @@ __global__ void ht_colsum_kernel(ColJobs J, float* part, int ctot) {
   part[(size_t)blockIdx.y * ctot + J.pc[j] + c] = s;
 }
 
+// Sum of the chunk partials per column: a block of 32 columns x 8 warps, warp w adding the
+// chunks w, w + 8, ..., then the 8 warp sums in a fixed order.
 __global__ void ht_colsum_finish_kernel(ColJobs J, const float* part, int ctot, int chunks) {
   PDL_ENTRY();
-  const int i = blockIdx.x * blockDim.x + threadIdx.x;
-  if (i >= ctot) return;
+  __shared__ float acc[8][33];
+  const int tx = threadIdx.x & 31, ty = threadIdx.x >> 5;
+  const int i = blockIdx.x * 32 + tx;
+  float s = 0.f;
+  if (i < ctot)
+    for (int y = ty; y < chunks; y += 8) s += part[(size_t)y * ctot + i];
+  acc[ty][tx] = s;
+  __syncthreads();
+  if (ty != 0 || i >= ctot) return;
+  float t = 0.f;
+#pragma unroll
+  for (int w = 0; w < 8; ++w) t += acc[w][tx];
   int j = 0;
   while (j + 1 < J.nj && i >= J.pc[j + 1]) ++j;
-  float s = 0.f;
-  for (int y = 0; y < chunks; ++y) s += part[(size_t)y * ctot + i];
-  J.j[j].out[i - J.pc[j]] = s;
+  J.j[j].out[i - J.pc[j]] = t;
+}
+
+// Elementwise GELU steps that also write their result transposed (32 x 32 tiles through shared
+// memory), for the weight-gradient products that read it as their K-major operand:
+//   BWD = 0 (forward):  h = GELU_erf(z)            -> hf (optional, fp32), ht [n][C], hT [C][ldT]
+//   BWD = 1 (backward): dz = dh GELU_erf'(z)      -> dh (in place, fp32), ht [n][C], hT [C][ldT]
+// Rows n..ldT-1 of the tile grid only write zeros into hT's padding columns.
+template <typename T, int BWD>
+__global__ void ht_gelu_tile_kernel(const float* __restrict__ z, float* hf, int n, int C, T* ht, T* hT, int ldT) {
+  PDL_ENTRY();
+  __shared__ float tile[32][33];
+  const int c0 = blockIdx.x * 32, r0 = blockIdx.y * 32;
+  const int tx = threadIdx.x & 31, ty = threadIdx.x >> 5;
+  for (int i = ty; i < 32; i += blockDim.x >> 5) {
+    const int r = r0 + i, c = c0 + tx;
+    float v = 0.f;
+    if (r < n && c < C) {
+      const size_t e = (size_t)r * C + c;
+      const float x = z[e];
+      if (BWD) {
+        const float gp =
+            0.5f * (1.f + erff(x * 0.70710678118654752f)) + x * 0.39894228040143268f * expf(-0.5f * x * x);
+        v = hf[e] * gp;
+        hf[e] = v;
+      } else {
+        v = gelu_erf_f(x);
+        if (hf) hf[e] = v;
+      }
+      ht[e] = from_f<T>(v);
+    }
+    tile[i][tx] = v;
+  }
+  __syncthreads();
+  for (int i = ty; i < 32; i += blockDim.x >> 5) {
+    const int c = c0 + i, r = r0 + tx;
+    if (c < C && r < ldT) hT[(size_t)c * ldT + r] = from_f<T>(tile[tx][i]);
+  }
 }
 
 // ---------------------------------------------------------------------------
@@ -326,37 +391,29 @@ __global__ void ht_adamw_kernel(AdamArgs A) {
   }
 }
 
-inline int ew_grid(long long count) { return (int)std::min<long long>((count + 255) / 256, 152LL * 8); }
-
 }  // namespace
 
 // ---------------------------------------------------------------------------
 // launchers
 // ---------------------------------------------------------------------------
 
-void ht_launch_act(cudaStream_t st, int dt, const float* z, long long count, float* hf, void* ht) {
-  if (count <= 0) return;
-  if (dt == 1) launch_k(ht_act_kernel<bf16>, ew_grid(count), 256, 0, st, z, count, hf, (bf16*)ht);
-  else launch_k(ht_act_kernel<float>, ew_grid(count), 256, 0, st, z, count, hf, (float*)ht);
-}
-
-void ht_launch_ce(cudaStream_t st, int dt, const float* logits, int n, int V, int Vp, const int* target, float* lossr,
-                  void* dl, float* loss, unsigned* err) {
+void ht_launch_ce(cudaStream_t st, int dt, const float* logits, int ldl, int n, int V, int Vp, const int* target,
+                  float* lossr, void* dl, float* loss, unsigned* err) {
   const float inv_n = 1.f / (float)n;
-  if (dt == 1) launch_k(ht_ce_kernel<bf16>, n, 512, 0, st, logits, V, Vp, target, inv_n, lossr, (bf16*)dl, err);
-  else launch_k(ht_ce_kernel<float>, n, 512, 0, st, logits, V, Vp, target, inv_n, lossr, (float*)dl, err);
+  if (dt == 1) launch_k(ht_ce_kernel<bf16>, n, 512, 0, st, logits, ldl, V, Vp, target, inv_n, lossr, (bf16*)dl, err);
+  else launch_k(ht_ce_kernel<float>, n, 512, 0, st, logits, ldl, V, Vp, target, inv_n, lossr, (float*)dl, err);
   if (loss) launch_k(ht_loss_kernel, 1, 1024, 0, st, (const float*)lossr, n, inv_n, loss);
 }
 
-void ht_launch_out_bwd(cudaStream_t st, int dt, const float* dxh, const float* stv, const float* h5, int n, int D,
-                       const float* g2, float eps, int mode, float norm_eps, float* dc0, float* dh5f, void* dh5t,
-                       float* r2) {
+void ht_launch_out_bwd(cudaStream_t st, int dt, const float* dxh, int nsplit, size_t split_stride, const float* stv,
+                       const float* h5, int n, int D, const float* g2, float eps, int mode, float norm_eps, float* dc0,
+                       float* dh5f, void* dh5t, float* r2) {
   if (dt == 1)
-    launch_k(ht_out_bwd_kernel<bf16>, n, 256, 0, st, dxh, stv, h5, D, g2, eps, mode, norm_eps, dc0, dh5f, (bf16*)dh5t,
-             r2);
+    launch_k(ht_out_bwd_kernel<bf16>, n, 256, 0, st, dxh, nsplit, split_stride, stv, h5, D, g2, eps, mode, norm_eps,
+             dc0, dh5f, (bf16*)dh5t, r2);
   else
-    launch_k(ht_out_bwd_kernel<float>, n, 256, 0, st, dxh, stv, h5, D, g2, eps, mode, norm_eps, dc0, dh5f,
-             (float*)dh5t, r2);
+    launch_k(ht_out_bwd_kernel<float>, n, 256, 0, st, dxh, nsplit, split_stride, stv, h5, D, g2, eps, mode, norm_eps,
+             dc0, dh5f, (float*)dh5t, r2);
 }
 
 void ht_launch_mid_bwd(cudaStream_t st, int dt, const float* dh4, const float* h3, int n, int m1, const float* g1,
@@ -365,10 +422,16 @@ void ht_launch_mid_bwd(cudaStream_t st, int dt, const float* dh4, const float* h
   else launch_k(ht_mid_bwd_kernel<float>, n, 256, 0, st, dh4, h3, m1, g1, eps, dh3f, (float*)dh3t, r1);
 }
 
-void ht_launch_gelu_bwd(cudaStream_t st, int dt, float* dh, const float* z, long long count, void* dzt) {
-  if (count <= 0) return;
-  if (dt == 1) launch_k(ht_gelu_bwd_kernel<bf16>, ew_grid(count), 256, 0, st, dh, z, count, (bf16*)dzt);
-  else launch_k(ht_gelu_bwd_kernel<float>, ew_grid(count), 256, 0, st, dh, z, count, (float*)dzt);
+void ht_launch_gelu_tile(cudaStream_t st, int dt, int bwd, const float* z, float* hf, int n, int C, void* ht, void* hT,
+                         int ldT) {
+  const dim3 grid((C + 31) / 32, (ldT + 31) / 32);
+  if (dt == 1) {
+    if (bwd) launch_k(ht_gelu_tile_kernel<bf16, 1>, grid, 256, 0, st, z, hf, n, C, (bf16*)ht, (bf16*)hT, ldT);
+    else launch_k(ht_gelu_tile_kernel<bf16, 0>, grid, 256, 0, st, z, hf, n, C, (bf16*)ht, (bf16*)hT, ldT);
+  } else {
+    if (bwd) launch_k(ht_gelu_tile_kernel<float, 1>, grid, 256, 0, st, z, hf, n, C, (float*)ht, (float*)hT, ldT);
+    else launch_k(ht_gelu_tile_kernel<float, 0>, grid, 256, 0, st, z, hf, n, C, (float*)ht, (float*)hT, ldT);
+  }
 }
 
 void ht_launch_prep_bwd(cudaStream_t st, const float* hs, const float* hp, const float* hI, const float* dc0, int n,
@@ -391,7 +454,7 @@ int ht_launch_colsum(cudaStream_t st, ColJobs J, float* part) {
   J.rows_per = HT_COLSUM_ROWS;
   const int chunks = ht_colsum_chunks(J.n);
   launch_k(ht_colsum_kernel, dim3(nb, chunks), 256, 0, st, J, part, ctot);
-  launch_k(ht_colsum_finish_kernel, (ctot + 255) / 256, 256, 0, st, J, (const float*)part, ctot, chunks);
+  launch_k(ht_colsum_finish_kernel, (ctot + 31) / 32, 256, 0, st, J, (const float*)part, ctot, chunks);
   return 2;
 }
 

@@ -48,17 +48,21 @@ struct AdamArgs {
   AdamSeg seg[HT_MAX_SEGS];
 };
 
-void ht_launch_act(cudaStream_t st, int dt, const float* z, long long count, float* hf, void* ht);
-// Cross-entropy rows (logits [n][V]) -> lossr[n], gradient dl [n][Vp] (T); loss (optional,
-// device scalar) = mean of lossr.
-void ht_launch_ce(cudaStream_t st, int dt, const float* logits, int n, int V, int Vp, const int* target, float* lossr,
-                  void* dl, float* loss, unsigned* err);
-void ht_launch_out_bwd(cudaStream_t st, int dt, const float* dxh, const float* stv, const float* h5, int n, int D,
-                       const float* g2, float eps, int mode, float norm_eps, float* dc0, float* dh5f, void* dh5t,
-                       float* r2);
+// Cross-entropy rows (logits [n][ldl], V used) -> lossr[n], gradient dl [n][Vp] (T); loss
+// (optional, device scalar) = mean of lossr.
+void ht_launch_ce(cudaStream_t st, int dt, const float* logits, int ldl, int n, int V, int Vp, const int* target,
+                  float* lossr, void* dl, float* loss, unsigned* err);
+// dxh: nsplit partial sums [n][D], split_stride floats apart.
+void ht_launch_out_bwd(cudaStream_t st, int dt, const float* dxh, int nsplit, size_t split_stride, const float* stv,
+                       const float* h5, int n, int D, const float* g2, float eps, int mode, float norm_eps, float* dc0,
+                       float* dh5f, void* dh5t, float* r2);
 void ht_launch_mid_bwd(cudaStream_t st, int dt, const float* dh4, const float* h3, int n, int m1, const float* g1,
                        float eps, float* dh3f, void* dh3t, float* r1);
-void ht_launch_gelu_bwd(cudaStream_t st, int dt, float* dh, const float* z, long long count, void* dzt);
+// GELU (bwd = 0: h = GELU(z) into hf (optional), ht, hT) or its derivative (bwd = 1: dz = hf *
+// GELU'(z) in place in hf, and into ht, hT), with the transposed copy hT [C][ldT] (zero columns
+// n..ldT-1) written by the same launch.
+void ht_launch_gelu_tile(cudaStream_t st, int dt, int bwd, const float* z, float* hf, int n, int C, void* ht, void* hT,
+                         int ldT);
 void ht_launch_prep_bwd(cudaStream_t st, const float* hs, const float* hp, const float* hI, const float* dc0, int n,
                         int D, const float* g0, const float* conv, float eps, float* pg0, float* cw);
 // Two launches; part holds chunks(J.n) * sum(C) floats.  Returns the launch count.

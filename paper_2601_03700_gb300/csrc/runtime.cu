@@ -55,7 +55,7 @@ struct ProfRec {
 enum { HT_G0, HT_CONV_W, HT_CONV_B, HT_FC1_W, HT_FC1_B, HT_FC2_W, HT_FC2_B, HT_FC3_W, HT_FC3_B, HT_G1, HT_FC4_W,
        HT_FC4_B, HT_G2, HT_NPARAM };
 struct HsmTrain {
-  int cap = 0, ldTc = 0, Vp = 0, part_cols = 0;
+  int cap = 0, ldTc = 0, Vp = 0, Vl = 0, part_cols = 0, sms = 1;
   long long step = 0;
   long long off[HT_NPARAM + 1] = {};
   long long numel[HT_NPARAM] = {};
@@ -992,8 +992,8 @@ static void ht_free(adept_model* m) {
 }
 
 // C[M, N] (+)= A[M, K] B[N, K]^T (+ bias) into fp32 `out` (ld ldo); acc adds into out in place.
-static void ht_gemm(adept_model* m, cudaStream_t st, const void* A, int lda, int a_rows, const void* B, int ldb, int M,
-                    int N, int K, float* out, int ldo, const float* bias, bool acc) {
+static GemmProblem ht_prob(const void* A, int lda, int a_rows, const void* B, int ldb, int M, int N, int K, float* out,
+                           int ldo, const float* bias, bool acc) {
   GemmProblem p;
   memset(&p, 0, sizeof p);
   p.A = A; p.lda = lda; p.a_rows = a_rows; p.B = B; p.ldb = ldb;
@@ -1001,7 +1001,44 @@ static void ht_gemm(adept_model* m, cudaStream_t st, const void* A, int lda, int
   p.epi = epi_base(); p.epi.kind = acc ? EPI_RESID : EPI_F32; p.epi.bias = bias;
   p.epi.out_f32 = out; p.epi.ld_f32 = ldo;
   if (acc) { p.epi.resid = out; p.epi.ld_resid = ldo; }
-  gemm(m, st, &p, 1, &M, ADEPT_PROF_GEMM_TRAIN, 2.0 * M * N * K, 0);
+  return p;
+}
+
+// One launch over independent problems (a weight gradient and the matching input gradient
+// share the launch, so that the small one does not leave SMs idle; K-split parts of one
+// product likewise).
+static void ht_gemm_n(adept_model* m, cudaStream_t st, const GemmProblem* ps, int n) {
+  int mr[8];
+  double fl = 0;
+  for (int i = 0; i < n; ++i) {
+    mr[i] = ps[i].rows.count;
+    fl += 2.0 * ps[i].rows.count * ps[i].N * ps[i].K;
+  }
+  gemm(m, st, ps, n, mr, ADEPT_PROF_GEMM_TRAIN, fl, 0);
+}
+
+static void ht_gemm(adept_model* m, cudaStream_t st, std::initializer_list<GemmProblem> ps) {
+  ht_gemm_n(m, st, ps.begin(), (int)ps.size());
+}
+
+constexpr int HT_DXH_SPLITS = 4;   // most K-splits of the head's input-gradient product
+
+// K-splits of the head's input-gradient product (M = n, N = D, K = Vp): the count in 1..4 whose
+// tiles (128 x 256) fill the SMs' last wave best, each split at least 512 of K.
+static int ht_dxh_splits(int n, int D, int Vp, int sms) {
+  const long long tiles = (long long)cdiv(n, 128) * cdiv(D, 256);
+  int best = 1;
+  double best_eff = 0;
+  for (int s = 1; s <= HT_DXH_SPLITS; ++s) {
+    if (s > 1 && Vp / s < 512) break;
+    const double waves = (double)(tiles * s) / sms;
+    const double eff = waves / std::ceil(waves);
+    if (eff > best_eff + 1e-9) {
+      best_eff = eff;
+      best = s;
+    }
+  }
+  return best;
 }
 
 static adept_status ht_init(adept_model* m, int cap, cudaStream_t st) {
@@ -1014,6 +1051,13 @@ static adept_status ht_init(adept_model* m, int cap, cudaStream_t st) {
   t.cap = cap;
   t.ldTc = (cap + 7) / 8 * 8;
   t.Vp = (V + 7) / 8 * 8;
+  t.Vl = (V + 15) / 16 * 16;   // logits rows 64-byte aligned: the GEMM epilogue stores whole 16-float runs
+  {
+    int dev = 0;
+    cudaGetDevice(&dev);
+    cudaDeviceGetAttribute(&t.sms, cudaDevAttrMultiProcessorCount, dev);
+    t.sms = std::max(1, t.sms);
+  }
   const long long n_el[HT_NPARAM] = {D, 9, 1, (long long)m1 * D, m1, (long long)m2 * m1, m2, (long long)m1 * m2,
                                      m1, m1, (long long)D * m1, D, D};
   long long o = 0;
@@ -1037,8 +1081,8 @@ static adept_status ht_init(adept_model* m, int cap, cudaStream_t st) {
   TRY(A(&t.headT, (size_t)D * t.Vp * es));
   TRY(A(&t.iota, n * 4));
   TRY(A(&t.c0f, n * D * 4)); TRY(A(&t.z1f, n * m1 * 4)); TRY(A(&t.h1f, n * m1 * 4)); TRY(A(&t.z2f, n * m2 * 4));
-  TRY(A(&t.h3f, n * m1 * 4)); TRY(A(&t.h5f, n * D * 4)); TRY(A(&t.stf, n * D * 4)); TRY(A(&t.logits, n * V * 4));
-  TRY(A(&t.lossr, n * 4)); TRY(A(&t.dxh, n * D * 4)); TRY(A(&t.dc0f, n * D * 4)); TRY(A(&t.dh5f, n * D * 4));
+  TRY(A(&t.h3f, n * m1 * 4)); TRY(A(&t.h5f, n * D * 4)); TRY(A(&t.stf, n * D * 4)); TRY(A(&t.logits, n * t.Vl * 4));
+  TRY(A(&t.lossr, n * 4)); TRY(A(&t.dxh, (size_t)HT_DXH_SPLITS * n * D * 4)); TRY(A(&t.dc0f, n * D * 4)); TRY(A(&t.dh5f, n * D * 4));
   TRY(A(&t.dh4f, n * m1 * 4)); TRY(A(&t.dh3f, n * m1 * 4)); TRY(A(&t.dh2f, n * m2 * 4));
   TRY(A(&t.r1, n * 4)); TRY(A(&t.r2, n * 4)); TRY(A(&t.cw, n * 10 * 4));
   t.part_cols = std::max({2 * D, 2 * m1, m2, D + 10});
@@ -1097,20 +1141,31 @@ static adept_status ht_step(adept_model* m, int n, const float* s_i, const float
   auto G = [&](int i) { return t.grad + t.off[i]; };
   // forward (Table S1), keeping what the backward reads
   launch_hsm_prep(st, dt, s_i, s_prev, inertia, rows, n, D, P(HT_G0), P(HT_CONV_W), eps, t.c0f, t.c0t);
-  ht_gemm(m, st, t.c0t, D, n, m->hsm_w1, D, n, m1, D, t.z1f, m1, P(HT_FC1_B), false);
-  ht_launch_act(st, dt, t.z1f, (long long)n * m1, t.h1f, t.h1t);
-  ht_gemm(m, st, t.h1t, m1, n, m->hsm_w2, m1, n, m2, m1, t.z2f, m2, P(HT_FC2_B), false);
-  ht_launch_act(st, dt, t.z2f, (long long)n * m2, nullptr, t.h2t);
-  ht_gemm(m, st, t.h2t, m2, n, m->hsm_w3, m2, n, m1, m2, t.h3f, m1, P(HT_FC3_B), false);
+  ht_gemm(m, st, {ht_prob(t.c0t, D, n, m->hsm_w1, D, n, m1, D, t.z1f, m1, P(HT_FC1_B), false)});
+  ht_launch_gelu_tile(st, dt, 0, t.z1f, t.h1f, n, m1, t.h1t, t.h1T, ldT);
+  ht_gemm(m, st, {ht_prob(t.h1t, m1, n, m->hsm_w2, m1, n, m2, m1, t.z2f, m2, P(HT_FC2_B), false)});
+  ht_launch_gelu_tile(st, dt, 0, t.z2f, nullptr, n, m2, t.h2t, t.h2T, ldT);
+  ht_gemm(m, st, {ht_prob(t.h2t, m2, n, m->hsm_w3, m2, n, m1, m2, t.h3f, m1, P(HT_FC3_B), false)});
   launch_hsm_mid(st, dt, t.h3f, t.h1f, rows, n, m1, P(HT_G1), eps, t.h4t);
-  ht_gemm(m, st, t.h4t, m1, n, m->hsm_w4, m1, n, D, m1, t.h5f, D, P(HT_FC4_B), false);
+  ht_gemm(m, st, {ht_prob(t.h4t, m1, n, m->hsm_w4, m1, n, D, m1, t.h5f, D, P(HT_FC4_B), false)});
   launch_hsm_out(st, dt, t.h5f, t.c0f, nullptr, 0, rows, n, D, P(HT_G2), eps, t.iota, t.stf, t.xht, hmode, neps);
   // the frozen head (final-norm gain and shift folded into its weights) and the loss
-  ht_gemm(m, st, t.xht, D, n, m->w_head, D, n, V, D, t.logits, V, m->b_head, false);
-  ht_launch_ce(st, dt, t.logits, n, V, Vp, target, t.lossr, t.dlt, loss, m->err_word);
+  ht_gemm(m, st, {ht_prob(t.xht, D, n, m->w_head, D, n, V, D, t.logits, t.Vl, m->b_head, false)});
+  ht_launch_ce(st, dt, t.logits, t.Vl, n, V, Vp, target, t.lossr, t.dlt, loss, m->err_word);
   // backward
-  ht_gemm(m, st, t.dlt, Vp, n, t.headT, Vp, n, D, Vp, t.dxh, D, nullptr, false);
-  ht_launch_out_bwd(st, dt, t.dxh, t.stf, t.h5f, n, D, P(HT_G2), eps, hmode, neps, t.dc0f, t.dh5f, t.dh5t, t.r2);
+  // dxh = dlogits W_head, K = Vp split into parts summed by the next kernel
+  {
+    const int S0 = ht_dxh_splits(n, D, Vp, t.sms);
+    const int kc = (cdiv(Vp, S0) + 63) / 64 * 64;
+    GemmProblem ps[HT_DXH_SPLITS];
+    int S = 0;
+    for (int k0 = 0; k0 < Vp; k0 += kc, ++S)
+      ps[S] = ht_prob((const char*)t.dlt + (size_t)k0 * m->esz, Vp, n, (const char*)t.headT + (size_t)k0 * m->esz, Vp,
+                      n, D, std::min(kc, Vp - k0), t.dxh + (size_t)S * n * D, D, nullptr, false);
+    ht_gemm_n(m, st, ps, S);
+    ht_launch_out_bwd(st, dt, t.dxh, S, (size_t)n * D, t.stf, t.h5f, n, D, P(HT_G2), eps, hmode, neps, t.dc0f,
+                      t.dh5f, t.dh5t, t.r2);
+  }
   int cl = 0;
   {
     ColJobs J{};
@@ -1121,8 +1176,8 @@ static adept_status ht_step(adept_model* m, int n, const float* s_i, const float
   }
   ht_launch_transpose(st, dt, t.dh5t, n, D, t.dh5T, ldT);
   ht_launch_transpose(st, dt, t.h4t, n, m1, t.h4T, ldT);
-  ht_gemm(m, st, t.dh5T, ldT, D, t.h4T, ldT, D, m1, ldT, G(HT_FC4_W), m1, nullptr, false);
-  ht_gemm(m, st, t.dh5t, D, n, t.w4T, D, n, m1, D, t.dh4f, m1, nullptr, false);
+  ht_gemm(m, st, {ht_prob(t.dh5T, ldT, D, t.h4T, ldT, D, m1, ldT, G(HT_FC4_W), m1, nullptr, false),    // dW4
+                   ht_prob(t.dh5t, D, n, t.w4T, D, n, m1, D, t.dh4f, m1, nullptr, false)});            // dh4
   ht_launch_mid_bwd(st, dt, t.dh4f, t.h3f, n, m1, P(HT_G1), eps, t.dh3f, t.dh3t, t.r1);
   {
     ColJobs J{};
@@ -1132,31 +1187,27 @@ static adept_status ht_step(adept_model* m, int n, const float* s_i, const float
     cl += ht_launch_colsum(st, J, t.part);
   }
   ht_launch_transpose(st, dt, t.dh3t, n, m1, t.dh3T, ldT);
-  ht_launch_transpose(st, dt, t.h2t, n, m2, t.h2T, ldT);
-  ht_gemm(m, st, t.dh3T, ldT, m1, t.h2T, ldT, m1, m2, ldT, G(HT_FC3_W), m2, nullptr, false);
-  ht_gemm(m, st, t.dh3t, m1, n, t.w3T, m1, n, m2, m1, t.dh2f, m2, nullptr, false);
-  ht_launch_gelu_bwd(st, dt, t.dh2f, t.z2f, (long long)n * m2, t.dz2t);
+  ht_gemm(m, st, {ht_prob(t.dh3T, ldT, m1, t.h2T, ldT, m1, m2, ldT, G(HT_FC3_W), m2, nullptr, false),   // dW3
+                   ht_prob(t.dh3t, m1, n, t.w3T, m1, n, m2, m1, t.dh2f, m2, nullptr, false)});          // dh2
+  ht_launch_gelu_tile(st, dt, 1, t.z2f, t.dh2f, n, m2, t.dz2t, t.dz2T, ldT);
   {
     ColJobs J{};
     J.n = n; J.nj = 1;
     J.j[0] = ColJob{t.dh2f, nullptr, nullptr, m2, G(HT_FC2_B)};
     cl += ht_launch_colsum(st, J, t.part);
   }
-  ht_launch_transpose(st, dt, t.dz2t, n, m2, t.dz2T, ldT);
-  ht_launch_transpose(st, dt, t.h1t, n, m1, t.h1T, ldT);
-  ht_gemm(m, st, t.dz2T, ldT, m2, t.h1T, ldT, m2, m1, ldT, G(HT_FC2_W), m1, nullptr, false);
-  ht_gemm(m, st, t.dz2t, m2, n, t.w2T, m2, n, m1, m2, t.dh4f, m1, nullptr, true);   // dh1 = dh4 + dz2 W2
-  ht_launch_gelu_bwd(st, dt, t.dh4f, t.z1f, (long long)n * m1, t.dh3t);            // dz1 (dh3's buffers are free)
+  ht_gemm(m, st, {ht_prob(t.dz2T, ldT, m2, t.h1T, ldT, m2, m1, ldT, G(HT_FC2_W), m1, nullptr, false),   // dW2
+                   ht_prob(t.dz2t, m2, n, t.w2T, m2, n, m1, m2, t.dh4f, m1, nullptr, true)});           // dh1 = dh4 + dz2 W2
+  ht_launch_gelu_tile(st, dt, 1, t.z1f, t.dh4f, n, m1, t.dh3t, t.dh3T, ldT);        // dz1 (dh3's buffers are free)
   {
     ColJobs J{};
     J.n = n; J.nj = 1;
     J.j[0] = ColJob{t.dh4f, nullptr, nullptr, m1, G(HT_FC1_B)};
     cl += ht_launch_colsum(st, J, t.part);
   }
-  ht_launch_transpose(st, dt, t.dh3t, n, m1, t.dh3T, ldT);
   ht_launch_transpose(st, dt, t.c0t, n, D, t.c0T, ldT);
-  ht_gemm(m, st, t.dh3T, ldT, m1, t.c0T, ldT, m1, D, ldT, G(HT_FC1_W), D, nullptr, false);
-  ht_gemm(m, st, t.dh3t, m1, n, t.w1T, m1, n, D, m1, t.dc0f, D, nullptr, true);     // dc0 += dz1 W1
+  ht_gemm(m, st, {ht_prob(t.dh3T, ldT, m1, t.c0T, ldT, m1, D, ldT, G(HT_FC1_W), D, nullptr, false),    // dW1
+                   ht_prob(t.dh3t, m1, n, t.w1T, m1, n, D, m1, t.dc0f, D, nullptr, true)});             // dc0 += dz1 W1
   ht_launch_prep_bwd(st, s_i, s_prev, inertia, t.dc0f, n, D, P(HT_G0), P(HT_CONV_W), eps, t.dh5f, t.cw);
   {
     ColJobs J{};
@@ -1188,9 +1239,9 @@ static adept_status ht_step(adept_model* m, int n, const float* s_i, const float
   a.nseg = (int)(sizeof segs / sizeof segs[0]);
   for (int i = 0; i < a.nseg; ++i) a.seg[i] = segs[i];
   ht_launch_adamw(st, dt, a);
-  // launches outside ht_gemm: prep, 2 act, mid, out, ce (+ loss), out_bwd, mid_bwd, 2 gelu_bwd, prep_bwd,
-  // 8 transposes, the column sums and AdamW
-  m->launches += 20 + (loss ? 1 : 0) + cl;
+  // launches outside ht_gemm: prep, 2 GELU, mid, out, ce (+ loss), out_bwd, mid_bwd, 2 GELU', prep_bwd,
+  // 4 transposes, the column sums and AdamW
+  m->launches += 16 + (loss ? 1 : 0) + cl;
   return check_launch(m);
 }
 

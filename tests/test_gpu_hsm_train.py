@@ -91,13 +91,14 @@ def check_step(cfg, W, o, g, theta0_o, tol, what):
         assert e <= tol, f"{what}: update of {k}: {e:.3e}"
 
 
-@pytest.mark.parametrize("family,dtype,n", [(synth.LLAMA, "f32", 13), (synth.GPT2, "f32", 8),
-                                            (synth.LLAMA, "bf16", 13), (synth.GPT2, "bf16", 37),
-                                            (synth.GPT2, "bf16", 1)])
-def test_one_step_matches_oracle(family, dtype, n):
+@pytest.mark.parametrize("family,dtype,n,vocab", [(synth.LLAMA, "f32", 13, 1000), (synth.GPT2, "f32", 8, 1000),
+                                                  (synth.LLAMA, "bf16", 13, 1000), (synth.GPT2, "bf16", 37, 1000),
+                                                  (synth.GPT2, "bf16", 1, 1000), (synth.LLAMA, "bf16", 45, 4099)])
+def test_one_step_matches_oracle(family, dtype, n, vocab):
     """Loss, gradients, moments and update of one step (n examples; ragged n exercises the
-    padded transposes; n <= 16 takes the generation-step GEMM for the n-row products)."""
-    cfg = cfg_of(family, dtype)
+    padded transposes; n <= 16 takes the generation-step GEMM for the n-row products; a
+    4099-token vocabulary splits the head's input-gradient product over K and pads its rows)."""
+    cfg = cfg_of(family, dtype, vocab=vocab)
     W = synth.make_weights(cfg, seed=3, std=0.05, gain_std=0.1 if dtype == "f32" else None)
     batch = synth.hsm_train_batch(cfg, n, seed=5)
     eps = adam_eps_for(W, cfg, batch)
