@@ -38,11 +38,12 @@ template <> __device__ __forceinline__ void store4<bf16>(bf16* p, float a, float
 // v < V and 0 for the padding columns V..Vp-1.  A target outside [0, V) flags ERRW_TOKEN and
 // leaves a zero loss and gradient for the row.  Rows are read as float4 groups (ldl and Vp
 // multiples of 4; columns at or past V are masked), four groups in flight per thread; the
-// second pass finds the row in L2.
+// second pass finds the row in L2 (1024-thread CTAs keep at most 2 rows per SM in flight, a
+// working set well inside L2 for rows of up to ~100 K logits).
 template <typename T>
-__global__ void __launch_bounds__(512) ht_ce_kernel(const float* __restrict__ logits, int ldl, int V, int Vp,
-                                                    const int* __restrict__ target, float inv_n, float* lossr, T* dl,
-                                                    unsigned* err) {
+__global__ void __launch_bounds__(1024) ht_ce_kernel(const float* __restrict__ logits, int ldl, int V, int Vp,
+                                                     const int* __restrict__ target, float inv_n, float* lossr, T* dl,
+                                                     unsigned* err) {
   PDL_ENTRY();
   __shared__ float red[32];
   __shared__ float rmax[32];
@@ -71,7 +72,8 @@ __global__ void __launch_bounds__(512) ht_ce_kernel(const float* __restrict__ lo
     }
 #pragma unroll
     for (int u = 0; u < U; ++u) {
-      const int v = 4 * (j0 + u * blockDim.x);
+      const int j = j0 + u * blockDim.x;
+      const int v = 4 * j;
       const float a0 = v < V ? x[u].x : -INFINITY, a1 = v + 1 < V ? x[u].y : -INFINITY;
       const float a2 = v + 2 < V ? x[u].z : -INFINITY, a3 = v + 3 < V ? x[u].w : -INFINITY;
       const float m4 = fmaxf(fmaxf(a0, a1), fmaxf(a2, a3));
@@ -298,8 +300,11 @@ __global__ void ht_colsum_finish_kernel(ColJobs J, const float* part, int ctot, 
 //   BWD = 0 (forward):  h = GELU_erf(z)            -> hf (optional, fp32), ht [n][C], hT [C][ldT]
 //   BWD = 1 (backward): dz = dh GELU_erf'(z)      -> dh (in place, fp32), ht [n][C], hT [C][ldT]
 // Rows n..ldT-1 of the tile grid only write zeros into hT's padding columns.
+// BWD = 1 also writes the tile's column sums over its 32 rows into part[blockIdx.y][C] (the
+// chunk partials of the bias gradient, HT_COLSUM_ROWS = 32).
 template <typename T, int BWD>
-__global__ void ht_gelu_tile_kernel(const float* __restrict__ z, float* hf, int n, int C, T* ht, T* hT, int ldT) {
+__global__ void ht_gelu_tile_kernel(const float* __restrict__ z, float* hf, int n, int C, T* ht, T* hT, int ldT,
+                                    float* part) {
   PDL_ENTRY();
   __shared__ float tile[32][33];
   const int c0 = blockIdx.x * 32, r0 = blockIdx.y * 32;
@@ -327,6 +332,11 @@ __global__ void ht_gelu_tile_kernel(const float* __restrict__ z, float* hf, int 
   for (int i = ty; i < 32; i += blockDim.x >> 5) {
     const int c = c0 + i, r = r0 + tx;
     if (c < C && r < ldT) hT[(size_t)c * ldT + r] = from_f<T>(tile[tx][i]);
+  }
+  if (BWD && ty == 0 && c0 + tx < C) {
+    float cs = 0.f;
+    for (int i = 0; i < 32; ++i) cs += tile[i][tx];
+    part[(size_t)blockIdx.y * C + c0 + tx] = cs;
   }
 }
 
@@ -400,8 +410,8 @@ __global__ void ht_adamw_kernel(AdamArgs A) {
 void ht_launch_ce(cudaStream_t st, int dt, const float* logits, int ldl, int n, int V, int Vp, const int* target,
                   float* lossr, void* dl, float* loss, unsigned* err) {
   const float inv_n = 1.f / (float)n;
-  if (dt == 1) launch_k(ht_ce_kernel<bf16>, n, 512, 0, st, logits, ldl, V, Vp, target, inv_n, lossr, (bf16*)dl, err);
-  else launch_k(ht_ce_kernel<float>, n, 512, 0, st, logits, ldl, V, Vp, target, inv_n, lossr, (float*)dl, err);
+  if (dt == 1) launch_k(ht_ce_kernel<bf16>, n, 1024, 0, st, logits, ldl, V, Vp, target, inv_n, lossr, (bf16*)dl, err);
+  else launch_k(ht_ce_kernel<float>, n, 1024, 0, st, logits, ldl, V, Vp, target, inv_n, lossr, (float*)dl, err);
   if (loss) launch_k(ht_loss_kernel, 1, 1024, 0, st, (const float*)lossr, n, inv_n, loss);
 }
 
@@ -423,14 +433,14 @@ void ht_launch_mid_bwd(cudaStream_t st, int dt, const float* dh4, const float* h
 }
 
 void ht_launch_gelu_tile(cudaStream_t st, int dt, int bwd, const float* z, float* hf, int n, int C, void* ht, void* hT,
-                         int ldT) {
+                         int ldT, float* part) {
   const dim3 grid((C + 31) / 32, (ldT + 31) / 32);
   if (dt == 1) {
-    if (bwd) launch_k(ht_gelu_tile_kernel<bf16, 1>, grid, 256, 0, st, z, hf, n, C, (bf16*)ht, (bf16*)hT, ldT);
-    else launch_k(ht_gelu_tile_kernel<bf16, 0>, grid, 256, 0, st, z, hf, n, C, (bf16*)ht, (bf16*)hT, ldT);
+    if (bwd) launch_k(ht_gelu_tile_kernel<bf16, 1>, grid, 256, 0, st, z, hf, n, C, (bf16*)ht, (bf16*)hT, ldT, part);
+    else launch_k(ht_gelu_tile_kernel<bf16, 0>, grid, 256, 0, st, z, hf, n, C, (bf16*)ht, (bf16*)hT, ldT, part);
   } else {
-    if (bwd) launch_k(ht_gelu_tile_kernel<float, 1>, grid, 256, 0, st, z, hf, n, C, (float*)ht, (float*)hT, ldT);
-    else launch_k(ht_gelu_tile_kernel<float, 0>, grid, 256, 0, st, z, hf, n, C, (float*)ht, (float*)hT, ldT);
+    if (bwd) launch_k(ht_gelu_tile_kernel<float, 1>, grid, 256, 0, st, z, hf, n, C, (float*)ht, (float*)hT, ldT, part);
+    else launch_k(ht_gelu_tile_kernel<float, 0>, grid, 256, 0, st, z, hf, n, C, (float*)ht, (float*)hT, ldT, part);
   }
 }
 
@@ -441,21 +451,34 @@ void ht_launch_prep_bwd(cudaStream_t st, const float* hs, const float* hp, const
 
 int ht_colsum_chunks(int n) { return (n + HT_COLSUM_ROWS - 1) / HT_COLSUM_ROWS; }
 
+static void colsum_layout(ColJobs& J, int* nb, int* ctot) {
+  *ctot = 0;
+  *nb = 0;
+  for (int j = 0; j < J.nj; ++j) {
+    J.cb[j] = *nb;
+    J.pc[j] = *ctot;
+    *nb += (J.j[j].C + 255) / 256;
+    *ctot += J.j[j].C;
+  }
+  J.cb[J.nj] = *nb;
+  J.pc[J.nj] = *ctot;
+  J.rows_per = HT_COLSUM_ROWS;
+}
+
 int ht_launch_colsum(cudaStream_t st, ColJobs J, float* part) {
   int ctot = 0, nb = 0;
-  for (int j = 0; j < J.nj; ++j) {
-    J.cb[j] = nb;
-    J.pc[j] = ctot;
-    nb += (J.j[j].C + 255) / 256;
-    ctot += J.j[j].C;
-  }
-  J.cb[J.nj] = nb;
-  J.pc[J.nj] = ctot;
-  J.rows_per = HT_COLSUM_ROWS;
+  colsum_layout(J, &nb, &ctot);
   const int chunks = ht_colsum_chunks(J.n);
   launch_k(ht_colsum_kernel, dim3(nb, chunks), 256, 0, st, J, part, ctot);
   launch_k(ht_colsum_finish_kernel, (ctot + 31) / 32, 256, 0, st, J, (const float*)part, ctot, chunks);
   return 2;
+}
+
+int ht_launch_colsum_finish(cudaStream_t st, ColJobs J, const float* part) {
+  int ctot = 0, nb = 0;
+  colsum_layout(J, &nb, &ctot);
+  launch_k(ht_colsum_finish_kernel, (ctot + 31) / 32, 256, 0, st, J, part, ctot, ht_colsum_chunks(J.n));
+  return 1;
 }
 
 void ht_launch_transpose(cudaStream_t st, int dt, const void* src, int n, int C, void* dst, int ldT) {

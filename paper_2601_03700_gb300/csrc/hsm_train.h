@@ -61,12 +61,16 @@ void ht_launch_mid_bwd(cudaStream_t st, int dt, const float* dh4, const float* h
 // GELU (bwd = 0: h = GELU(z) into hf (optional), ht, hT) or its derivative (bwd = 1: dz = hf *
 // GELU'(z) in place in hf, and into ht, hT), with the transposed copy hT [C][ldT] (zero columns
 // n..ldT-1) written by the same launch.
+// bwd = 1 also leaves the chunk partials of the column sums of dz in part ([chunks(n)][C], for
+// ht_launch_colsum_finish).
 void ht_launch_gelu_tile(cudaStream_t st, int dt, int bwd, const float* z, float* hf, int n, int C, void* ht, void* hT,
-                         int ldT);
+                         int ldT, float* part);
 void ht_launch_prep_bwd(cudaStream_t st, const float* hs, const float* hp, const float* hI, const float* dc0, int n,
                         int D, const float* g0, const float* conv, float eps, float* pg0, float* cw);
 // Two launches; part holds chunks(J.n) * sum(C) floats.  Returns the launch count.
 int ht_launch_colsum(cudaStream_t st, ColJobs J, float* part);
+// The second half of ht_launch_colsum, for partials a producer already wrote ([chunks(J.n)][sum C]).
+int ht_launch_colsum_finish(cudaStream_t st, ColJobs J, const float* part);
 // dst [C][ldT] = src [n][C] transposed, zero columns n..ldT-1.
 void ht_launch_transpose(cudaStream_t st, int dt, const void* src, int n, int C, void* dst, int ldT);
 void ht_launch_adamw(cudaStream_t st, int dt, AdamArgs A);

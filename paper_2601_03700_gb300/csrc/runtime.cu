@@ -1142,9 +1142,9 @@ static adept_status ht_step(adept_model* m, int n, const float* s_i, const float
   // forward (Table S1), keeping what the backward reads
   launch_hsm_prep(st, dt, s_i, s_prev, inertia, rows, n, D, P(HT_G0), P(HT_CONV_W), eps, t.c0f, t.c0t);
   ht_gemm(m, st, {ht_prob(t.c0t, D, n, m->hsm_w1, D, n, m1, D, t.z1f, m1, P(HT_FC1_B), false)});
-  ht_launch_gelu_tile(st, dt, 0, t.z1f, t.h1f, n, m1, t.h1t, t.h1T, ldT);
+  ht_launch_gelu_tile(st, dt, 0, t.z1f, t.h1f, n, m1, t.h1t, t.h1T, ldT, nullptr);
   ht_gemm(m, st, {ht_prob(t.h1t, m1, n, m->hsm_w2, m1, n, m2, m1, t.z2f, m2, P(HT_FC2_B), false)});
-  ht_launch_gelu_tile(st, dt, 0, t.z2f, nullptr, n, m2, t.h2t, t.h2T, ldT);
+  ht_launch_gelu_tile(st, dt, 0, t.z2f, nullptr, n, m2, t.h2t, t.h2T, ldT, nullptr);
   ht_gemm(m, st, {ht_prob(t.h2t, m2, n, m->hsm_w3, m2, n, m1, m2, t.h3f, m1, P(HT_FC3_B), false)});
   launch_hsm_mid(st, dt, t.h3f, t.h1f, rows, n, m1, P(HT_G1), eps, t.h4t);
   ht_gemm(m, st, {ht_prob(t.h4t, m1, n, m->hsm_w4, m1, n, D, m1, t.h5f, D, P(HT_FC4_B), false)});
@@ -1189,21 +1189,21 @@ static adept_status ht_step(adept_model* m, int n, const float* s_i, const float
   ht_launch_transpose(st, dt, t.dh3t, n, m1, t.dh3T, ldT);
   ht_gemm(m, st, {ht_prob(t.dh3T, ldT, m1, t.h2T, ldT, m1, m2, ldT, G(HT_FC3_W), m2, nullptr, false),   // dW3
                    ht_prob(t.dh3t, m1, n, t.w3T, m1, n, m2, m1, t.dh2f, m2, nullptr, false)});          // dh2
-  ht_launch_gelu_tile(st, dt, 1, t.z2f, t.dh2f, n, m2, t.dz2t, t.dz2T, ldT);
+  ht_launch_gelu_tile(st, dt, 1, t.z2f, t.dh2f, n, m2, t.dz2t, t.dz2T, ldT, t.part);
   {
     ColJobs J{};
     J.n = n; J.nj = 1;
-    J.j[0] = ColJob{t.dh2f, nullptr, nullptr, m2, G(HT_FC2_B)};
-    cl += ht_launch_colsum(st, J, t.part);
+    J.j[0] = ColJob{nullptr, nullptr, nullptr, m2, G(HT_FC2_B)};
+    cl += ht_launch_colsum_finish(st, J, t.part);
   }
   ht_gemm(m, st, {ht_prob(t.dz2T, ldT, m2, t.h1T, ldT, m2, m1, ldT, G(HT_FC2_W), m1, nullptr, false),   // dW2
                    ht_prob(t.dz2t, m2, n, t.w2T, m2, n, m1, m2, t.dh4f, m1, nullptr, true)});           // dh1 = dh4 + dz2 W2
-  ht_launch_gelu_tile(st, dt, 1, t.z1f, t.dh4f, n, m1, t.dh3t, t.dh3T, ldT);        // dz1 (dh3's buffers are free)
+  ht_launch_gelu_tile(st, dt, 1, t.z1f, t.dh4f, n, m1, t.dh3t, t.dh3T, ldT, t.part);  // dz1 (dh3's buffers are free)
   {
     ColJobs J{};
     J.n = n; J.nj = 1;
-    J.j[0] = ColJob{t.dh4f, nullptr, nullptr, m1, G(HT_FC1_B)};
-    cl += ht_launch_colsum(st, J, t.part);
+    J.j[0] = ColJob{nullptr, nullptr, nullptr, m1, G(HT_FC1_B)};
+    cl += ht_launch_colsum_finish(st, J, t.part);
   }
   ht_launch_transpose(st, dt, t.c0t, n, D, t.c0T, ldT);
   ht_gemm(m, st, {ht_prob(t.dh3T, ldT, m1, t.c0T, ldT, m1, D, ldT, G(HT_FC1_W), D, nullptr, false),    // dW1
