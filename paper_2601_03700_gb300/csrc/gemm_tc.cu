@@ -26,11 +26,14 @@ constexpr int TC_BM = 128;
 constexpr int TC_BK = 64;               // one 128-byte swizzle row of bf16
 constexpr int TC_THREADS = 192;
 constexpr int TC_SHORT_ROWS = 32;   // rows of the short-tile variants (3-D k-chunk boxes)
+constexpr int TC_OUT_STAGE_BYTES = 4 * 32 * 32 * 4;   // epilogue TMA-store staging, one 32 x 32 fp32 chunk per warp
 constexpr long long TC_TIMEOUT_CYCLES = 4000000000LL;   // ~2 s at 2 GHz
 
 struct TcGroup {
   CUtensorMap ta;   // A: [rows, K] bf16, box 64 x 128
   CUtensorMap tb;   // B: [N, K] bf16, box 64 x BN
+  CUtensorMap tout; // EPI_F32 output [rows, N] fp32, box 32 x 32, 128-byte swizzle (when tma_out)
+  int tma_out;      // the epilogue stores 32 x 32 fp32 chunks by TMA instead of per-row stores
   DevRange rows;
   int N;
   int K;
@@ -100,6 +103,20 @@ __device__ __forceinline__ void tma_load_3d(const CUtensorMap* tm, uint64_t* bar
           "r"(smem_u32(dst)),
       "l"((uint64_t)tm), "r"(0), "r"(y), "r"(z), "r"(smem_u32(bar)));
 }
+
+// Bulk tensor store of a 32 x 32 fp32 chunk staged in shared memory (128-byte swizzle) at
+// column x, row y of the output; out-of-range rows and columns are not written.
+__device__ __forceinline__ void tma_store_2d(const CUtensorMap* tm, const void* src, int x, int y) {
+  asm volatile("cp.async.bulk.tensor.2d.global.shared::cta.bulk_group [%0, {%2, %3}], [%1];" ::"l"((uint64_t)tm),
+               "r"(smem_u32(src)), "r"(x), "r"(y)
+               : "memory");
+  asm volatile("cp.async.bulk.commit_group;" ::: "memory");
+}
+// Wait until the bulk stores issued by this thread have read their shared-memory source.
+__device__ __forceinline__ void bulk_wait_read() { asm volatile("cp.async.bulk.wait_group.read 0;" ::: "memory"); }
+// Wait until the bulk stores issued by this thread are complete.
+__device__ __forceinline__ void bulk_wait_all() { asm volatile("cp.async.bulk.wait_group 0;" ::: "memory"); }
+__device__ __forceinline__ void fence_async_shared() { asm volatile("fence.proxy.async.shared::cta;" ::: "memory"); }
 
 __device__ __forceinline__ void tmem_alloc(uint32_t* slot, uint32_t ncols) {
   asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(smem_u32(slot)), "r"(ncols)
@@ -195,7 +212,8 @@ __global__ void __launch_bounds__(TC_THREADS, 1) gemm_tc_kernel(const __grid_con
   uint8_t* smem = (uint8_t*)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
   uint8_t* sA = smem;
   uint8_t* sB = smem + STAGES * A_BYTES;
-  uint64_t* full = (uint64_t*)(smem + STAGES * (A_BYTES + B_BYTES));
+  uint8_t* sOut = smem + STAGES * (A_BYTES + B_BYTES);   // 4 x 4 KB: each epilogue warp's store chunk
+  uint64_t* full = (uint64_t*)(sOut + TC_OUT_STAGE_BYTES);
   uint64_t* empty = full + STAGES;
   uint64_t* accf = empty + STAGES;
   uint64_t* acce = accf + 2;
@@ -435,12 +453,39 @@ __global__ void __launch_bounds__(TC_THREADS, 1) gemm_tc_kernel(const __grid_con
       if (t == (int)blockIdx.x && warp == 2 && lane == 0) TC_TRACE(5);
       tc_fence_after();
       const uint32_t tb = tmem + ((uint32_t)(q * 32) << 16) + (uint32_t)(ab * BN);
+      if (G.tma_out) {
+        // plain fp32 output: each 32 x 32 chunk goes to shared memory (row = lane, 16-byte
+        // pieces in the 128-byte swizzle order) and leaves as one bulk tensor store, instead of
+        // 32 row-strided 128-byte stores per warp instruction
+        uint8_t* stg = sOut + q * 4096;
+        const int y = s_mbeg[g] + mb * TC_BM + q * 32;
 #pragma unroll 1
-      for (int c = 0; c < BN; c += 32) {
-        float v[32];
-        tmem_ld32(tb + (uint32_t)c, v);
-        const int c0 = nb * BN + c;
-        if (valid && c0 < G.N) epi_chunk32<bf16>(G.epi, ra, c0, G.N, v, rr, bias ? &s_bias[q][c] : nullptr);
+        for (int c = 0; c < BN; c += 32) {
+          float v[32];
+          tmem_ld32(tb + (uint32_t)c, v);
+          const int c0 = nb * BN + c;
+          if (c0 >= G.N) continue;   // warp-uniform
+          if (bias) {
+#pragma unroll
+            for (int j = 0; j < 32; ++j) v[j] += s_bias[q][c + j];
+          }
+          if (lane == 0) bulk_wait_read();   // the previous chunk's store has read the buffer
+          __syncwarp();
+          float4* row = reinterpret_cast<float4*>(stg + lane * 128);
+#pragma unroll
+          for (int k = 0; k < 8; ++k) row[k ^ (lane & 7)] = make_float4(v[4 * k], v[4 * k + 1], v[4 * k + 2], v[4 * k + 3]);
+          fence_async_shared();
+          __syncwarp();
+          if (lane == 0) tma_store_2d(&G.tout, stg, c0, y);
+        }
+      } else {
+#pragma unroll 1
+        for (int c = 0; c < BN; c += 32) {
+          float v[32];
+          tmem_ld32(tb + (uint32_t)c, v);
+          const int c0 = nb * BN + c;
+          if (valid && c0 < G.N) epi_chunk32<bf16>(G.epi, ra, c0, G.N, v, rr, bias ? &s_bias[q][c] : nullptr);
+        }
       }
       tc_fence_before();
       __syncwarp();
@@ -449,6 +494,7 @@ __global__ void __launch_bounds__(TC_THREADS, 1) gemm_tc_kernel(const __grid_con
       ab ^= 1;
       if (ab == 0) aph ^= 1;
     }
+    if (lane == 0) bulk_wait_all();   // this warp's bulk stores are complete before the CTA ends
   }
   __syncthreads();
   if (threadIdx.x == 0) TC_TRACE(7);
@@ -548,11 +594,39 @@ static bool make_map(CUtensorMap* m, const void* base, uint64_t inner, uint64_t 
   return true;
 }
 
+// fp32 output map of an EPI_F32 problem with a fixed row range: dims {N, rows}, box 32 x 32,
+// 128-byte swizzle (the epilogue's staging order).  False when the output does not qualify.
+static bool make_out_map(CUtensorMap* m, const GemmProblem& q) {
+  if (q.epi.kind != EPI_F32 || q.rows.begin || q.rows.end || q.rows.count <= 0 || !q.epi.out_f32) return false;
+  if (((uintptr_t)q.epi.out_f32 & 15) || (q.epi.ld_f32 & 3) || q.N <= 0) return false;
+  static std::unordered_map<MapKey, CUtensorMap, MapKeyHash> cache;
+  static std::mutex mu;
+  const uint64_t row_bytes = (uint64_t)q.epi.ld_f32 * 4;
+  const MapKey key{q.epi.out_f32, (uint64_t)q.N, (uint64_t)q.rows.count, row_bytes, 32};
+  std::lock_guard<std::mutex> lock(mu);
+  auto it = cache.find(key);
+  if (it != cache.end()) {
+    *m = it->second;
+    return true;
+  }
+  cuuint64_t dims[2] = {(cuuint64_t)q.N, (cuuint64_t)q.rows.count};
+  cuuint64_t strides[1] = {row_bytes};
+  cuuint32_t box[2] = {32, 32};
+  cuuint32_t estr[2] = {1, 1};
+  if (g_encode(m, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 2, q.epi.out_f32, dims, strides, box, estr,
+               CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_NONE,
+               CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
+    return false;
+  if (cache.size() > 65536) cache.clear();
+  cache.emplace(key, *m);
+  return true;
+}
+
 template <int BN, int STAGES, int MAXG, int KC = 1>
 static int launch_bn(cudaStream_t st, const TcParams<MAXG>& prm, int grid) {
   constexpr size_t a_bytes = (size_t)TC_BM * TC_BK * 2 + (size_t)(KC - 1) * TC_SHORT_ROWS * TC_BK * 2;
   constexpr size_t b_bytes = (size_t)KC * BN * TC_BK * 2;
-  constexpr size_t smem = (size_t)STAGES * (a_bytes + b_bytes) + 1024 + 256;
+  constexpr size_t smem = (size_t)STAGES * (a_bytes + b_bytes) + TC_OUT_STAGE_BYTES + 1024 + 256;
   static_assert(smem <= 232448, "stage ring does not fit shared memory");
   static bool attr = false;
   if (!attr) {
@@ -631,6 +705,7 @@ static int launch_grouped(cudaStream_t st, const GemmProblem* probs, int n_probs
     G.K = q.K;
     G.gm = raster_gm(q.K);
     G.epi = q.epi;
+    G.tma_out = make_out_map(&G.tout, q) ? 1 : 0;
   }
   const int grid = (int)std::min<long long>(tiles[pick], (long long)g_num_sms);
   if (grid <= 0) return 0;

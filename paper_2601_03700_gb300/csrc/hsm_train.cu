@@ -38,10 +38,10 @@ template <> __device__ __forceinline__ void store4<bf16>(bf16* p, float a, float
 // v < V and 0 for the padding columns V..Vp-1.  A target outside [0, V) flags ERRW_TOKEN and
 // leaves a zero loss and gradient for the row.  Rows are read as float4 groups (ldl and Vp
 // multiples of 4; columns at or past V are masked), four groups in flight per thread; the
-// second pass finds the row in L2 (1024-thread CTAs keep at most 2 rows per SM in flight, a
-// working set well inside L2 for rows of up to ~100 K logits).
+// second pass finds the row in L2 (512-thread CTAs, two per SM: one CTA's reductions overlap
+// the other's loads, and ~300 rows in flight stay well inside L2 for vocabularies of ~50 K).
 template <typename T>
-__global__ void __launch_bounds__(1024) ht_ce_kernel(const float* __restrict__ logits, int ldl, int V, int Vp,
+__global__ void __launch_bounds__(512, 2) ht_ce_kernel(const float* __restrict__ logits, int ldl, int V, int Vp,
                                                      const int* __restrict__ target, float inv_n, float* lossr, T* dl,
                                                      unsigned* err) {
   PDL_ENTRY();
@@ -410,8 +410,8 @@ __global__ void ht_adamw_kernel(AdamArgs A) {
 void ht_launch_ce(cudaStream_t st, int dt, const float* logits, int ldl, int n, int V, int Vp, const int* target,
                   float* lossr, void* dl, float* loss, unsigned* err) {
   const float inv_n = 1.f / (float)n;
-  if (dt == 1) launch_k(ht_ce_kernel<bf16>, n, 1024, 0, st, logits, ldl, V, Vp, target, inv_n, lossr, (bf16*)dl, err);
-  else launch_k(ht_ce_kernel<float>, n, 1024, 0, st, logits, ldl, V, Vp, target, inv_n, lossr, (float*)dl, err);
+  if (dt == 1) launch_k(ht_ce_kernel<bf16>, n, 512, 0, st, logits, ldl, V, Vp, target, inv_n, lossr, (bf16*)dl, err);
+  else launch_k(ht_ce_kernel<float>, n, 512, 0, st, logits, ldl, V, Vp, target, inv_n, lossr, (float*)dl, err);
   if (loss) launch_k(ht_loss_kernel, 1, 1024, 0, st, (const float*)lossr, n, inv_n, loss);
 }
 
