@@ -334,12 +334,19 @@ def hsm_train_flops(cfg, n):
     return n * (6.0 * fc + 4.0 * D * cfg.vocab)
 
 
-def run_hsm_train(adept, device, peaks, n=8192, reps=5):
-    """HSM training step (Sec. 4.2; App. D): GPT-2-small shape (D 768, HSM widths 3072 / 6144,
-    vocabulary 50257, bf16 GEMM operands, fp32 master weights and AdamW state), n synthetic
-    examples per step (128 sequences x 64 tokens).  Step time with CUDA events; the GEMMs'
-    share and TFLOP/s from per-GEMM events in a separate profiled step."""
-    cfg = synth.gpt2_small_config(n_layers=2, max_batch=1, max_seq=16)
+def run_hsm_train(adept, device, peaks, n=8192, reps=5, shape="gpt2"):
+    """HSM training step (Sec. 4.2; App. D), n synthetic examples per step, bf16 GEMM operands,
+    fp32 master weights and AdamW state.  shape "gpt2": GPT-2-small (D 768, HSM widths 3072 /
+    6144, vocabulary 50257; 8192 examples = 128 sequences x 64 tokens); "llama7b": Llama-2-7B
+    (D 4096, HSM widths 8192 / 32768, vocabulary 32000; 8192 examples = 8 sequences x 1024
+    tokens).  Only the frozen head and the HSM take part, so the models carry 2 layers.  Step
+    time with CUDA events; the GEMMs' TFLOP/s from per-GEMM events in a separate profiled step."""
+    if shape == "llama7b":
+        cfg = synth.llama7b_config(n_layers=2, max_batch=1, max_seq=16)
+        desc = "Llama-2-7B shape HSM (4096 -> 8192 -> 32768 -> 8192 -> 4096) + frozen 32000-token head"
+    else:
+        cfg = synth.gpt2_small_config(n_layers=2, max_batch=1, max_seq=16)
+        desc = "GPT-2-small shape HSM (768 -> 3072 -> 6144 -> 3072 -> 768) + frozen 50257-token head"
     W = synth.make_weights(cfg, seed=0, device=device)
     m = adept.Model(cfg, W)
     del W
@@ -374,8 +381,7 @@ def run_hsm_train(adept, device, peaks, n=8192, reps=5):
     m.close()
     torch.cuda.empty_cache()
     peak = peaks["bf16_tflops_sustained"]
-    return {"workload": f"GPT-2-small shape HSM (768 -> 3072 -> 6144 -> 3072 -> 768) + frozen 50257-token head, "
-                        f"{n} examples/step, bf16 GEMM operands, fp32 AdamW",
+    return {"workload": f"{desc}, {n} examples/step, bf16 GEMM operands, fp32 AdamW",
             "ms_per_step": round(t * 1e3, 3), "examples_s": round(n / t, 1), "gpu_launches": int(launches),
             "gemm_tflop_per_step": round(fl / 1e12, 4), "tflops_step": round(fl / t / 1e12, 1),
             "gemm_launches": int(ng), "gemm_ms_profiled": round(gms, 3),
@@ -432,6 +438,21 @@ def run_llama_e2e(adept, device, P=2048, steps=256):
             "depth_ratio": round(fd_["mean_exit_depth"] / ee["mean_exit_depth"], 4)}
 
 
+def max_over_ranks(x: float, world: int, device) -> float:
+    """The slowest rank's value (replicas: the job ends when the last rank does)."""
+    if world <= 1:
+        return float(x)
+    t = torch.tensor([float(x)], dtype=torch.float64, device=device)
+    torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
+    return float(t.item())
+
+
+def replica_throughput(units_per_rank_step: float, steps: int, world: int, seconds: float) -> float:
+    """Whole-job throughput of `world` independent replicas: every rank's units over the
+    slowest rank's time."""
+    return world * units_per_rank_step * steps / seconds
+
+
 def ours(args, rank, world, device):
     import paper_2601_03700_gb300 as adept
     if not os.path.exists(adept.LIB_PATH):
@@ -480,12 +501,9 @@ def ours(args, rank, world, device):
     prof = {c: adept.adept_profile_read(run.m.h, c) for c in range(adept.PROF_DECODE_STEP + 1)}
     adept.adept_set_option(run.m.h, adept.OPT_PROFILE, 0)
     adept.adept_check_device_status(run.m.h)
-    t = torch.tensor([total_ms], dtype=torch.float64, device=device)
-    if world > 1:
-        torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
-    total_ms = float(t.item())
+    total_ms = max_over_ranks(total_ms, world, device)
     tok_per_step = B * P + B * STEPS
-    value = world * tok_per_step * args.steps / (total_ms / 1e3)
+    value = replica_throughput(tok_per_step, args.steps, world, total_ms / 1e3)
     # --------------------------------------------------------------- end-to-end through the API with host buffers
     tok_h = run.tokens.cpu().pin_memory()
     fp_h = run.fp.cpu().pin_memory()
@@ -507,7 +525,8 @@ def ours(args, rank, world, device):
         ex_h[B * P:].copy_(run.exit_d.view(-1), non_blocking=True)
         torch.cuda.synchronize()
         e2e_t += time.perf_counter() - t0
-    e2e = world * tok_per_step * max(1, args.steps) / e2e_t
+    e2e_t = max_over_ranks(e2e_t, world, device)
+    e2e = replica_throughput(tok_per_step, max(1, args.steps), world, e2e_t)
     h2d = (tok_h.numel() + fp_h.numel() + fd_h.numel()) * 4
     d2h = (out_h.numel() + ex_h.numel()) * 4
     # --------------------------------------------------------------- dominant kernel roofline
@@ -610,6 +629,7 @@ def ours(args, rank, world, device):
         line["llama7b_e2e"] = run_llama_e2e(adept, device)
         line["encoder"] = run_encoder(adept, device)
         line["hsm_train"] = run_hsm_train(adept, device, peaks)
+        line["hsm_train_llama7b"] = run_hsm_train(adept, device, peaks, shape="llama7b", reps=3)
     if rank == 0 and not args.no_cpu_baseline:
         line["cpu_baseline"] = cpu_baseline(args.cpu_tokens)
     return line
