@@ -634,10 +634,199 @@ __global__ void final_scatter_kernel(const float* X, int D, const int* n_rows, c
 // ---------------------------------------------------------------------------
 // Hidden State Mapper, non-GEMM steps (Sec. 4.2, App. B Table S1)
 // ---------------------------------------------------------------------------
+// Hidden State Mapper row steps (Table S1).  One CTA per row.  The register-resident
+// kernels hold a row as EPT elements per thread (d = threadIdx.x + j * blockDim.x), issue
+// every load of the row before the first reduction and compute from registers, so a row
+// costs one round of memory latency instead of one per strided loop iteration (these
+// kernels run on a handful of rows in a generation step, where latency is the cost).  Longer
+// rows (above 4096 elements for the convolution step, 8192 for the others) take the
+// strided-loop kernels further below.
+// ---------------------------------------------------------------------------
+
+template <int EPT>
+__device__ __forceinline__ void hsm_load_row(const float* __restrict__ p, int n, float (&v)[EPT]) {
+#pragma unroll
+  for (int j = 0; j < EPT; ++j) {
+    const int d = threadIdx.x + j * blockDim.x;
+    v[j] = d < n ? p[d] : 0.f;
+  }
+}
+
+// Block-wide sums of NV values in a fixed order (blockDim.x a multiple of 32); red holds
+// 32 * NV floats.  Every thread gets the sums.
+template <int NV>
+__device__ __forceinline__ void block_sum_n(float (&v)[NV], float* red) {
+  const int lane = threadIdx.x & 31, w = threadIdx.x >> 5, nw = blockDim.x >> 5;
+#pragma unroll
+  for (int i = 0; i < NV; ++i) v[i] = warp_sum(v[i]);
+  __syncthreads();
+  if (lane == 0) {
+#pragma unroll
+    for (int i = 0; i < NV; ++i) red[w * NV + i] = v[i];
+  }
+  __syncthreads();
+#pragma unroll
+  for (int i = 0; i < NV; ++i) {
+    float t = 0.f;
+    for (int k = 0; k < nw; ++k) t += red[k * NV + i];
+    v[i] = t;
+  }
+}
+
+// Three separately RMS-normalised rows (shared gain g0), then the 3x3 convolution with
+// padding (0, 1): c0[t] = b + sum_a sum_u w[a][u] Xn_a[t + u - 1], Xn_a = x_a rstd_a g0.
+// Dynamic shared memory: the three normalised rows, 3 * D floats.
+template <typename T, int EPT>
+__global__ void __launch_bounds__(256) hsm_prep_kernel(const float* hs, const float* hp, const float* hI, DevRange rows, int D,
+                                const float* g0, const float* conv /* 9 taps + bias */, float eps, float* c0f,
+                                T* c0t) {
+  PDL_ENTRY();
+  extern __shared__ float s_xn[];
+  __shared__ float red[32 * 3];
+  const int k = rows.b() + blockIdx.x;
+  if (k >= rows.e()) return;
+  float xa[EPT], xb[EPT], xc[EPT], g[EPT];
+  hsm_load_row(hs + (size_t)k * D, D, xa);
+  hsm_load_row(hp + (size_t)k * D, D, xb);
+  hsm_load_row(hI + (size_t)k * D, D, xc);
+  hsm_load_row(g0, D, g);
+  float w[10];
+#pragma unroll
+  for (int i = 0; i < 10; ++i) w[i] = conv[i];
+  float ss[3] = {0.f, 0.f, 0.f};
+#pragma unroll
+  for (int j = 0; j < EPT; ++j) {
+    ss[0] += xa[j] * xa[j];
+    ss[1] += xb[j] * xb[j];
+    ss[2] += xc[j] * xc[j];
+  }
+  block_sum_n<3>(ss, red);
+  const float sa = rsqrtf(ss[0] / D + eps), sb = rsqrtf(ss[1] / D + eps), sc = rsqrtf(ss[2] / D + eps);
+#pragma unroll
+  for (int j = 0; j < EPT; ++j) {
+    const int d = threadIdx.x + j * blockDim.x;
+    if (d < D) {
+      s_xn[d] = xa[j] * sa * g[j];
+      s_xn[D + d] = xb[j] * sb * g[j];
+      s_xn[2 * D + d] = xc[j] * sc * g[j];
+    }
+  }
+  __syncthreads();
+#pragma unroll
+  for (int j = 0; j < EPT; ++j) {
+    const int t = threadIdx.x + j * blockDim.x;
+    if (t >= D) continue;
+    float acc = w[9];
+#pragma unroll
+    for (int a = 0; a < 3; ++a) {
+#pragma unroll
+      for (int u = 0; u < 3; ++u) {
+        const int tt = t + u - 1;
+        if (tt >= 0 && tt < D) acc += w[a * 3 + u] * s_xn[a * D + tt];
+      }
+    }
+    c0f[(size_t)k * D + t] = acc;
+    c0t[(size_t)k * D + t] = from_f<T>(acc);
+  }
+}
+
+// h4 = RMSNorm_g1(h3) + h1 (the MLP's addition), rounded for FC4.
+template <typename T, int EPT>
+__global__ void __launch_bounds__(1024) hsm_mid_kernel(const float* h3, const float* h1, DevRange rows, int m1, const float* g1, float eps,
+                               T* h4) {
+  PDL_ENTRY();
+  __shared__ float red[32];
+  const int k = rows.b() + blockIdx.x;
+  if (k >= rows.e()) return;
+  float a[EPT], b[EPT];
+  hsm_load_row(h3 + (size_t)k * m1, m1, a);
+  hsm_load_row(h1 + (size_t)k * m1, m1, b);
+  float s2[1] = {0.f};
+#pragma unroll
+  for (int j = 0; j < EPT; ++j) s2[0] += a[j] * a[j];
+  block_sum_n<1>(s2, red);
+  const float sc = rsqrtf(s2[0] / m1 + eps);
+#pragma unroll
+  for (int j = 0; j < EPT; ++j) {
+    const int d = threadIdx.x + j * blockDim.x;
+    if (d < m1) h4[(size_t)k * m1 + d] = from_f<T>(a[j] * sc * g1[d] + b[j]);
+  }
+}
+
+// s~ = RMSNorm_g2(h5) + c0 (the final addition); written to the token's final state,
+// and standardised (the attention-input normalisation of the family) for the fills.
+// identity != 0: s~ = s_i* (test switch replacing the HSM).
+template <typename T, int EPT>
+__global__ void __launch_bounds__(1024) hsm_out_kernel(const float* h5, const float* c0f, const float* hs, int identity, DevRange rows, int D,
+                               const float* g2, float eps, const int* exit_tok, float* final_, T* xfill,
+                               int fill_mode, float norm_eps) {
+  PDL_ENTRY();
+  __shared__ float red[32];
+  const int k = rows.b() + blockIdx.x;
+  if (k >= rows.e()) return;
+  const int tok = exit_tok[k];
+  float f[EPT];
+  if (identity) {
+    hsm_load_row(hs + (size_t)k * D, D, f);
+  } else {
+    float c[EPT];
+    hsm_load_row(h5 + (size_t)k * D, D, f);
+    hsm_load_row(c0f + (size_t)k * D, D, c);
+    float s2[1] = {0.f};
+#pragma unroll
+    for (int j = 0; j < EPT; ++j) s2[0] += f[j] * f[j];
+    block_sum_n<1>(s2, red);
+    const float sc = rsqrtf(s2[0] / D + eps);
+#pragma unroll
+    for (int j = 0; j < EPT; ++j) {
+      const int d = threadIdx.x + j * blockDim.x;
+      f[j] = d < D ? f[j] * sc * g2[d] + c[j] : 0.f;
+    }
+  }
+  float* fo = final_ + (size_t)tok * D;
+  T* o = xfill + (size_t)k * D;
+#pragma unroll
+  for (int j = 0; j < EPT; ++j) {
+    const int d = threadIdx.x + j * blockDim.x;
+    if (d < D) fo[d] = f[j];
+  }
+  if (fill_mode == NORM_COPY) {
+#pragma unroll
+    for (int j = 0; j < EPT; ++j) {
+      const int d = threadIdx.x + j * blockDim.x;
+      if (d < D) o[d] = from_f<T>(f[j]);
+    }
+    return;
+  }
+  float mu = 0.f;
+  if (fill_mode == NORM_LN) {
+    float s[1] = {0.f};
+#pragma unroll
+    for (int j = 0; j < EPT; ++j) s[0] += f[j];
+    block_sum_n<1>(s, red);
+    mu = s[0] / D;
+  }
+  float v[1] = {0.f};
+#pragma unroll
+  for (int j = 0; j < EPT; ++j) {
+    const int d = threadIdx.x + j * blockDim.x;
+    const float c = d < D ? f[j] - mu : 0.f;
+    v[0] += c * c;
+  }
+  block_sum_n<1>(v, red);
+  const float rstd = rsqrtf(v[0] / D + norm_eps);
+#pragma unroll
+  for (int j = 0; j < EPT; ++j) {
+    const int d = threadIdx.x + j * blockDim.x;
+    if (d < D) o[d] = from_f<T>((f[j] - mu) * rstd);
+  }
+}
+
+// Strided-loop forms of the three kernels above, for the longer rows.
 // Three separately RMS-normalised rows (shared gain g0), then the 3x3 convolution with
 // padding (0, 1): c0[t] = b + sum_a sum_u w[a][u] x_a[t + u - 1].
 template <typename T>
-__global__ void hsm_prep_kernel(const float* hs, const float* hp, const float* hI, DevRange rows, int D,
+__global__ void hsm_prep_loop_kernel(const float* hs, const float* hp, const float* hI, DevRange rows, int D,
                                 const float* g0, const float* conv /* 9 taps + bias */, float eps, float* c0f,
                                 T* c0t) {
   PDL_ENTRY();
@@ -669,7 +858,7 @@ __global__ void hsm_prep_kernel(const float* hs, const float* hp, const float* h
 
 // h4 = RMSNorm_g1(h3) + h1 (the MLP's addition), rounded for FC4.
 template <typename T>
-__global__ void hsm_mid_kernel(const float* h3, const float* h1, DevRange rows, int m1, const float* g1, float eps,
+__global__ void hsm_mid_loop_kernel(const float* h3, const float* h1, DevRange rows, int m1, const float* g1, float eps,
                                T* h4) {
   PDL_ENTRY();
   __shared__ float red[32];
@@ -687,7 +876,7 @@ __global__ void hsm_mid_kernel(const float* h3, const float* h1, DevRange rows, 
 // and standardised (the attention-input normalisation of the family) for the fills.
 // identity != 0: s~ = s_i* (test switch replacing the HSM).
 template <typename T>
-__global__ void hsm_out_kernel(const float* h5, const float* c0f, const float* hs, int identity, DevRange rows, int D,
+__global__ void hsm_out_loop_kernel(const float* h5, const float* c0f, const float* hs, int identity, DevRange rows, int D,
                                const float* g2, float eps, const int* exit_tok, float* final_, T* xfill,
                                int fill_mode, float norm_eps) {
   PDL_ENTRY();
@@ -963,32 +1152,94 @@ void launch_final_scatter(cudaStream_t st, const float* X, int D, const int* n_r
   launch_k(final_scatter_kernel, max_rows, 256, 0, st, X, D, n_rows, row_tok, final_, exit_layer_out, n_layers);
 }
 
+// Threads per CTA of the register-resident mid / out kernels for a row of n elements (4
+// elements per thread up to 1024, else 8), or 0 when the row needs the strided-loop kernel.
+static int hsm_row_threads(int n) {
+  if (n <= 4 * 256) return 256;
+  if (n <= 8 * 512) return 512;
+  if (n <= 8 * 1024) return 1024;
+  return 0;
+}
+
+template <typename T, int EPT>
+static void hsm_prep_go(cudaStream_t st, int thr, const float* hs, const float* hp, const float* hI, DevRange rows,
+                        int max_rows, int D, const float* g0, const float* conv, float eps, float* c0f, void* c0t) {
+  const size_t smem = (size_t)3 * D * sizeof(float);   // D <= 4096: at most 48 KB (+ static) -> opt in
+  static bool attr = false;
+  if (!attr) {
+    cudaFuncSetAttribute(hsm_prep_kernel<T, EPT>, cudaFuncAttributeMaxDynamicSharedMemorySize, 3 * 16 * 256 * 4);
+    attr = true;
+  }
+  launch_k(hsm_prep_kernel<T, EPT>, max_rows, thr, smem, st, hs, hp, hI, rows, D, g0, conv, eps, c0f, (T*)c0t);
+}
+
 void launch_hsm_prep(cudaStream_t st, int dt, const float* hs, const float* hp, const float* hI, DevRange rows,
                      int max_rows, int D, const float* g0, const float* conv, float eps, float* c0f, void* c0t) {
   if (max_rows <= 0) return;
-  if (dt == 1)
-    launch_k(hsm_prep_kernel<bf16>, max_rows, 256, 0, st, hs, hp, hI, rows, D, g0, conv, eps, c0f, (bf16*)c0t);
-  else
-    launch_k(hsm_prep_kernel<float>, max_rows, 256, 0, st, hs, hp, hI, rows, D, g0, conv, eps, c0f, (float*)c0t);
+  const int thr = D <= 16 * 256 ? 256 : 0;   // four row arrays in registers: 256 threads, 16 elements each
+  if (thr == 0) {
+    if (dt == 1)
+      launch_k(hsm_prep_loop_kernel<bf16>, max_rows, 256, 0, st, hs, hp, hI, rows, D, g0, conv, eps, c0f, (bf16*)c0t);
+    else
+      launch_k(hsm_prep_loop_kernel<float>, max_rows, 256, 0, st, hs, hp, hI, rows, D, g0, conv, eps, c0f,
+               (float*)c0t);
+    return;
+  }
+  const bool small = D <= 4 * 256;
+  if (dt == 1) {
+    if (small) hsm_prep_go<bf16, 4>(st, thr, hs, hp, hI, rows, max_rows, D, g0, conv, eps, c0f, c0t);
+    else hsm_prep_go<bf16, 16>(st, thr, hs, hp, hI, rows, max_rows, D, g0, conv, eps, c0f, c0t);
+  } else {
+    if (small) hsm_prep_go<float, 4>(st, thr, hs, hp, hI, rows, max_rows, D, g0, conv, eps, c0f, c0t);
+    else hsm_prep_go<float, 16>(st, thr, hs, hp, hI, rows, max_rows, D, g0, conv, eps, c0f, c0t);
+  }
 }
 
 void launch_hsm_mid(cudaStream_t st, int dt, const float* h3, const float* h1, DevRange rows, int max_rows, int m1,
                     const float* g1, float eps, void* h4) {
   if (max_rows <= 0) return;
-  if (dt == 1) launch_k(hsm_mid_kernel<bf16>, max_rows, 256, 0, st, h3, h1, rows, m1, g1, eps, (bf16*)h4);
-  else launch_k(hsm_mid_kernel<float>, max_rows, 256, 0, st, h3, h1, rows, m1, g1, eps, (float*)h4);
+  const int thr = hsm_row_threads(m1);
+  if (thr == 0) {
+    if (dt == 1) launch_k(hsm_mid_loop_kernel<bf16>, max_rows, 256, 0, st, h3, h1, rows, m1, g1, eps, (bf16*)h4);
+    else launch_k(hsm_mid_loop_kernel<float>, max_rows, 256, 0, st, h3, h1, rows, m1, g1, eps, (float*)h4);
+    return;
+  }
+  const bool small = m1 <= 4 * 256;
+  if (dt == 1) {
+    if (small) launch_k(hsm_mid_kernel<bf16, 4>, max_rows, thr, 0, st, h3, h1, rows, m1, g1, eps, (bf16*)h4);
+    else launch_k(hsm_mid_kernel<bf16, 8>, max_rows, thr, 0, st, h3, h1, rows, m1, g1, eps, (bf16*)h4);
+  } else {
+    if (small) launch_k(hsm_mid_kernel<float, 4>, max_rows, thr, 0, st, h3, h1, rows, m1, g1, eps, (float*)h4);
+    else launch_k(hsm_mid_kernel<float, 8>, max_rows, thr, 0, st, h3, h1, rows, m1, g1, eps, (float*)h4);
+  }
 }
 
 void launch_hsm_out(cudaStream_t st, int dt, const float* h5, const float* c0f, const float* hs, int identity,
                     DevRange rows, int max_rows, int D, const float* g2, float eps, const int* exit_tok,
                     float* final_, void* xfill, int fill_mode, float norm_eps) {
   if (max_rows <= 0) return;
-  if (dt == 1)
-    launch_k(hsm_out_kernel<bf16>, max_rows, 256, 0, st, h5, c0f, hs, identity, rows, D, g2, eps, exit_tok, final_,
-                                                   (bf16*)xfill, fill_mode, norm_eps);
-  else
-    launch_k(hsm_out_kernel<float>, max_rows, 256, 0, st, h5, c0f, hs, identity, rows, D, g2, eps, exit_tok, final_,
-                                                    (float*)xfill, fill_mode, norm_eps);
+  const int thr = hsm_row_threads(D);
+  if (thr == 0) {
+    if (dt == 1)
+      launch_k(hsm_out_loop_kernel<bf16>, max_rows, 256, 0, st, h5, c0f, hs, identity, rows, D, g2, eps, exit_tok,
+               final_, (bf16*)xfill, fill_mode, norm_eps);
+    else
+      launch_k(hsm_out_loop_kernel<float>, max_rows, 256, 0, st, h5, c0f, hs, identity, rows, D, g2, eps, exit_tok,
+               final_, (float*)xfill, fill_mode, norm_eps);
+    return;
+  }
+  const bool small = D <= 4 * 256;
+#define HSM_OUT(T, E)                                                                                              \
+  launch_k(hsm_out_kernel<T, E>, max_rows, thr, 0, st, h5, c0f, hs, identity, rows, D, g2, eps, exit_tok, final_, \
+           (T*)xfill, fill_mode, norm_eps)
+  if (dt == 1) {
+    if (small) HSM_OUT(bf16, 4);
+    else HSM_OUT(bf16, 8);
+  } else {
+    if (small) HSM_OUT(float, 4);
+    else HSM_OUT(float, 8);
+  }
+#undef HSM_OUT
 }
 
 // Two-stage argmax for long rows: ARGMAX_SPLIT blocks per row reduce slices to
