@@ -58,13 +58,20 @@ void launch_exit_move(cudaStream_t st, const float* Xin, const float* Xout, cons
                       float* Inext, float* hsm_s, float* hsm_prev, float* hsm_I);
 void launch_final_scatter(cudaStream_t st, const float* X, int D, const int* n_rows, int max_rows, const int* row_tok,
                           float* final_, int* exit_layer_out, int n_layers);
+// launch_final_scatter that also writes each row standardised for the output head (hmode, heps)
+// in bf16 at xhead[token] (generation steps); rows of up to 8192 elements (head_rows_supported).
+bool head_rows_supported(int D);
+void launch_final_scatter_head(cudaStream_t st, const float* X, int D, const int* n_rows, int max_rows,
+                               const int* row_tok, float* final_, int* exit_layer_out, int n_layers, bf16* xhead,
+                               int hmode, float heps);
 void launch_hsm_prep(cudaStream_t st, int dt, const float* hs, const float* hp, const float* hI, DevRange rows,
                      int max_rows, int D, const float* g0, const float* conv, float eps, float* c0f, void* c0t);
 void launch_hsm_mid(cudaStream_t st, int dt, const float* h3, const float* h1, DevRange rows, int max_rows, int m1,
                     const float* g1, float eps, void* h4);
+// xhead (optional): each row's standardised s~ also at xhead[token] (generation steps' head input).
 void launch_hsm_out(cudaStream_t st, int dt, const float* h5, const float* c0f, const float* hs, int identity,
                     DevRange rows, int max_rows, int D, const float* g2, float eps, const int* exit_tok,
-                    float* final_, void* xfill, int fill_mode, float norm_eps);
+                    float* final_, void* xfill, int fill_mode, float norm_eps, void* xhead = nullptr);
 // Greedy token per row (lowest index on ties); part_v / part_i: rows * 32 partials.
 int launch_argmax(cudaStream_t st, const float* logits, int V, int rows, int* out, float* part_v, int* part_i);
 void launch_head_rows(cudaStream_t st, int batch, int prompt_len, int last, int* rows);

@@ -631,6 +631,16 @@ __global__ void final_scatter_kernel(const float* X, int D, const int* n_rows, c
   if (threadIdx.x == 0 && exit_layer_out) exit_layer_out[tok] = n_layers;
 }
 
+// final_scatter_kernel that also writes the row standardised for the output head (hmode
+// NORM_RMS / NORM_LN, the head's gain and shift folded into its weights) at the token's head
+// row of xhead (generation steps: token = sequence); the row is held in registers.
+template <int EPT>
+__global__ void __launch_bounds__(1024) final_scatter_head_kernel(const float* X, int D, const int* n_rows,
+                                                                  const int* row_tok, float* final_,
+                                                                  int* exit_layer_out, int n_layers, bf16* xhead,
+                                                                  int hmode, float heps);
+
+
 // ---------------------------------------------------------------------------
 // Hidden State Mapper, non-GEMM steps (Sec. 4.2, App. B Table S1)
 // ---------------------------------------------------------------------------
@@ -756,10 +766,11 @@ __global__ void __launch_bounds__(1024) hsm_mid_kernel(const float* h3, const fl
 // s~ = RMSNorm_g2(h5) + c0 (the final addition); written to the token's final state,
 // and standardised (the attention-input normalisation of the family) for the fills.
 // identity != 0: s~ = s_i* (test switch replacing the HSM).
+// xhead (optional, generation steps): the same standardised row also at the token's head row.
 template <typename T, int EPT>
 __global__ void __launch_bounds__(1024) hsm_out_kernel(const float* h5, const float* c0f, const float* hs, int identity, DevRange rows, int D,
                                const float* g2, float eps, const int* exit_tok, float* final_, T* xfill,
-                               int fill_mode, float norm_eps) {
+                               int fill_mode, float norm_eps, T* xhead) {
   PDL_ENTRY();
   __shared__ float red[32];
   const int k = rows.b() + blockIdx.x;
@@ -815,10 +826,59 @@ __global__ void __launch_bounds__(1024) hsm_out_kernel(const float* h5, const fl
   }
   block_sum_n<1>(v, red);
   const float rstd = rsqrtf(v[0] / D + norm_eps);
+  T* oh = xhead ? xhead + (size_t)tok * D : nullptr;
 #pragma unroll
   for (int j = 0; j < EPT; ++j) {
     const int d = threadIdx.x + j * blockDim.x;
-    if (d < D) o[d] = from_f<T>((f[j] - mu) * rstd);
+    if (d < D) {
+      const T x = from_f<T>((f[j] - mu) * rstd);
+      o[d] = x;
+      if (oh) oh[d] = x;
+    }
+  }
+}
+
+template <int EPT>
+__global__ void __launch_bounds__(1024) final_scatter_head_kernel(const float* X, int D, const int* n_rows,
+                                                                  const int* row_tok, float* final_,
+                                                                  int* exit_layer_out, int n_layers, bf16* xhead,
+                                                                  int hmode, float heps) {
+  PDL_ENTRY();
+  __shared__ float red[32];
+  const int r = blockIdx.x;
+  if (r >= *n_rows) return;
+  const int tok = row_tok[r];
+  float f[EPT];
+  hsm_load_row(X + (size_t)r * D, D, f);
+  float* fo = final_ + (size_t)tok * D;
+#pragma unroll
+  for (int j = 0; j < EPT; ++j) {
+    const int d = threadIdx.x + j * blockDim.x;
+    if (d < D) fo[d] = f[j];
+  }
+  if (threadIdx.x == 0 && exit_layer_out) exit_layer_out[tok] = n_layers;
+  float mu = 0.f;
+  if (hmode == NORM_LN) {
+    float s[1] = {0.f};
+#pragma unroll
+    for (int j = 0; j < EPT; ++j) s[0] += f[j];
+    block_sum_n<1>(s, red);
+    mu = s[0] / D;
+  }
+  float v[1] = {0.f};
+#pragma unroll
+  for (int j = 0; j < EPT; ++j) {
+    const int d = threadIdx.x + j * blockDim.x;
+    const float c = d < D ? f[j] - mu : 0.f;
+    v[0] += c * c;
+  }
+  block_sum_n<1>(v, red);
+  const float rstd = rsqrtf(v[0] / D + heps);
+  bf16* oh = xhead + (size_t)tok * D;
+#pragma unroll
+  for (int j = 0; j < EPT; ++j) {
+    const int d = threadIdx.x + j * blockDim.x;
+    if (d < D) oh[d] = __float2bfloat16_rn((f[j] - mu) * rstd);
   }
 }
 
@@ -878,7 +938,7 @@ __global__ void hsm_mid_loop_kernel(const float* h3, const float* h1, DevRange r
 template <typename T>
 __global__ void hsm_out_loop_kernel(const float* h5, const float* c0f, const float* hs, int identity, DevRange rows, int D,
                                const float* g2, float eps, const int* exit_tok, float* final_, T* xfill,
-                               int fill_mode, float norm_eps) {
+                               int fill_mode, float norm_eps, T* xhead) {
   PDL_ENTRY();
   __shared__ float red[32];
   const int k = rows.b() + blockIdx.x;
@@ -912,7 +972,12 @@ __global__ void hsm_out_loop_kernel(const float* h5, const float* c0f, const flo
     s2 += c * c;
   }
   const float rstd = rsqrtf(block_sum(s2, red) / D + norm_eps);
-  for (int d = threadIdx.x; d < D; d += blockDim.x) o[d] = from_f<T>((f[d] - mu) * rstd);
+  T* oh = xhead ? xhead + (size_t)tok * D : nullptr;
+  for (int d = threadIdx.x; d < D; d += blockDim.x) {
+    const T x = from_f<T>((f[d] - mu) * rstd);
+    o[d] = x;
+    if (oh) oh[d] = x;
+  }
 }
 
 // ---------------------------------------------------------------------------
@@ -1152,6 +1217,7 @@ void launch_final_scatter(cudaStream_t st, const float* X, int D, const int* n_r
   launch_k(final_scatter_kernel, max_rows, 256, 0, st, X, D, n_rows, row_tok, final_, exit_layer_out, n_layers);
 }
 
+
 // Threads per CTA of the register-resident mid / out kernels for a row of n elements (4
 // elements per thread up to 1024, else 8), or 0 when the row needs the strided-loop kernel.
 static int hsm_row_threads(int n) {
@@ -1216,22 +1282,22 @@ void launch_hsm_mid(cudaStream_t st, int dt, const float* h3, const float* h1, D
 
 void launch_hsm_out(cudaStream_t st, int dt, const float* h5, const float* c0f, const float* hs, int identity,
                     DevRange rows, int max_rows, int D, const float* g2, float eps, const int* exit_tok,
-                    float* final_, void* xfill, int fill_mode, float norm_eps) {
+                    float* final_, void* xfill, int fill_mode, float norm_eps, void* xhead) {
   if (max_rows <= 0) return;
   const int thr = hsm_row_threads(D);
   if (thr == 0) {
     if (dt == 1)
       launch_k(hsm_out_loop_kernel<bf16>, max_rows, 256, 0, st, h5, c0f, hs, identity, rows, D, g2, eps, exit_tok,
-               final_, (bf16*)xfill, fill_mode, norm_eps);
+               final_, (bf16*)xfill, fill_mode, norm_eps, (bf16*)xhead);
     else
       launch_k(hsm_out_loop_kernel<float>, max_rows, 256, 0, st, h5, c0f, hs, identity, rows, D, g2, eps, exit_tok,
-               final_, (float*)xfill, fill_mode, norm_eps);
+               final_, (float*)xfill, fill_mode, norm_eps, (float*)xhead);
     return;
   }
   const bool small = D <= 4 * 256;
 #define HSM_OUT(T, E)                                                                                              \
   launch_k(hsm_out_kernel<T, E>, max_rows, thr, 0, st, h5, c0f, hs, identity, rows, D, g2, eps, exit_tok, final_, \
-           (T*)xfill, fill_mode, norm_eps)
+           (T*)xfill, fill_mode, norm_eps, (T*)xhead)
   if (dt == 1) {
     if (small) HSM_OUT(bf16, 4);
     else HSM_OUT(bf16, 8);
@@ -1240,6 +1306,21 @@ void launch_hsm_out(cudaStream_t st, int dt, const float* h5, const float* c0f, 
     else HSM_OUT(float, 8);
   }
 #undef HSM_OUT
+}
+
+bool head_rows_supported(int D) { return hsm_row_threads(D) > 0; }
+
+void launch_final_scatter_head(cudaStream_t st, const float* X, int D, const int* n_rows, int max_rows,
+                               const int* row_tok, float* final_, int* exit_layer_out, int n_layers, bf16* xhead,
+                               int hmode, float heps) {
+  if (max_rows <= 0) return;
+  const int thr = hsm_row_threads(D);
+  if (D <= 4 * 256)
+    launch_k(final_scatter_head_kernel<4>, max_rows, thr, 0, st, X, D, n_rows, row_tok, final_, exit_layer_out,
+             n_layers, xhead, hmode, heps);
+  else
+    launch_k(final_scatter_head_kernel<8>, max_rows, thr, 0, st, X, D, n_rows, row_tok, final_, exit_layer_out,
+             n_layers, xhead, hmode, heps);
 }
 
 // Two-stage argmax for long rows: ARGMAX_SPLIT blocks per row reduce slices to

@@ -146,6 +146,7 @@ struct adept_model {
   DfState* df = nullptr;
   std::string df_why;
   HsmTrain* ht = nullptr;   // HSM training state (adept_hsm_train_init)
+  bool xhead_ready = false; // the last generation step left its head input rows in xhead
   std::vector<cudaEvent_t> ev_pool;
   size_t ev_used = 0;
   int gemm_cls = ADEPT_PROF_GEMM_PREFILL;
@@ -716,12 +717,13 @@ static adept_status reserve_seqs(adept_model* m, int batch, const int* lens, cud
 // the early-exit pass
 // ---------------------------------------------------------------------------
 
-static void run_hsm(adept_model* m, cudaStream_t st, DevRange rows, int max_rows, int a_rows) {
+// xhead (generation steps): each exit's standardised s~ also becomes its head input row.
+static void run_hsm(adept_model* m, cudaStream_t st, DevRange rows, int max_rows, int a_rows, void* xhead = nullptr) {
   const int D = m->D, m1 = m->m1, m2 = m->m2;
   const float eps = m->cfg.hsm_eps;
   if (m->hsm_identity) {
     launch_hsm_out(st, m->dt, nullptr, nullptr, m->hsm_s, 1, rows, max_rows, D, m->hsm_g2, eps, m->exit_tok,
-                   m->final_, m->xfill, attn_norm_mode(m), m->cfg.norm_eps);
+                   m->final_, m->xfill, attn_norm_mode(m), m->cfg.norm_eps, xhead);
     m->launches += 1;
     return;
   }
@@ -753,7 +755,7 @@ static void run_hsm(adept_model* m, cudaStream_t st, DevRange rows, int max_rows
   p.epi = epi_base(); p.epi.kind = EPI_F32; p.epi.bias = m->hsm_b4; p.epi.out_f32 = m->h5f; p.epi.ld_f32 = D;
   gemm(m, st, &p, 1, &max_rows, m->gemm_cls);
   launch_hsm_out(st, m->dt, m->h5f, m->c0f, m->hsm_s, 0, rows, max_rows, D, m->hsm_g2, eps, m->exit_tok, m->final_,
-                 m->xfill, attn_norm_mode(m), m->cfg.norm_eps);
+                 m->xfill, attn_norm_mode(m), m->cfg.norm_eps, xhead);
   m->launches += 1;
 }
 
@@ -789,6 +791,11 @@ static adept_status run_pass(adept_model* m, int n_tok, int batch, int prompt_le
   // encoder "stop entirely" (Sec. 4.3, downstream tasks): exits are recorded in tok_exit
   // (the attention leaves out keys of tokens gone before its layer) and get no fills
   const bool stop = fam == ADEPT_FAMILY_BERT && m->stop_entirely && !decode;
+  // generation steps of bf16 decoders: the producers of the final states (the last layer's
+  // row scatter, the HSM's output step) also write them standardised for the head, so the
+  // head GEMM streams its weights against ready bf16 rows
+  const bool head_x = decode && fam != ADEPT_FAMILY_BERT && m->dt == ADEPT_DTYPE_BF16 && head_rows_supported(D);
+  m->xhead_ready = head_x;
   int32_t* exit_w = stop ? m->tok_exit : exit_out;
   launch_pass_init(st, n_tok, prompt_len, decode ? 1 : 0, m->tok_seq, m->tok_pos, m->row_tok[0], m->d_seq_len,
                    m->max_blocks_per_seq * c.kv_block_tokens, fam == ADEPT_FAMILY_LLAMA ? 0 : c.max_pos,
@@ -917,7 +924,11 @@ static adept_status run_pass(adept_model* m, int n_tok, int batch, int prompt_le
       }
       par ^= 1;
     } else {
-      launch_final_scatter(st, m->X_out, D, m->ctr + CTR_ACTIVE + par, mr, rt, m->final_, exit_w, N);
+      if (head_x)
+        launch_final_scatter_head(st, m->X_out, D, m->ctr + CTR_ACTIVE + par, mr, rt, m->final_, exit_w, N,
+                                  (bf16*)m->xhead, attn_norm_mode(m), m->cfg.norm_eps);
+      else
+        launch_final_scatter(st, m->X_out, D, m->ctr + CTR_ACTIVE + par, mr, rt, m->final_, exit_w, N);
       m->launches += 1;
     }
   }
@@ -928,7 +939,7 @@ static adept_status run_pass(adept_model* m, int n_tok, int batch, int prompt_le
     // the skipped-layer fills of all exits run once, after the layer loop: one HSM over
     // every exited token, then one grouped launch over (skipped layer r) groups; rows are
     // in exit-layer order, so layer r's rows (i* < r) are a prefix.
-    run_hsm(m, st, DevRange{nullptr, m->ctr + CTR_EXITED, 0}, n_tok, n_tok);
+    run_hsm(m, st, DevRange{nullptr, m->ctr + CTR_EXITED, 0}, n_tok, n_tok, head_x ? m->xhead : nullptr);
     std::vector<GemmProblem> probs;
     std::vector<int> mrs;
     for (int r = 3; r <= N; ++r) {
@@ -947,8 +958,11 @@ static adept_status run_head(adept_model* m, int batch, int prompt_len, bool dec
   const int D = m->D;
   const bool enc = c.family == ADEPT_FAMILY_BERT;
   float* out = logits ? logits : m->logits_ws;
-  launch_head_rows(st, batch, decode ? 1 : prompt_len, enc ? 0 : 1, m->head_rows);
-  m->launches += 1;
+  const bool rows_ready = !enc && decode && m->xhead_ready;   // head input already in xhead
+  if (!rows_ready) {
+    launch_head_rows(st, batch, decode ? 1 : prompt_len, enc ? 0 : 1, m->head_rows);
+    m->launches += 1;
+  }
   const DevRange rows{nullptr, nullptr, batch};
   GemmProblem p;
   memset(&p, 0, sizeof p);
@@ -956,7 +970,10 @@ static adept_status run_head(adept_model* m, int batch, int prompt_len, bool dec
   if (!enc) {
     p.A = m->xhead; p.lda = D; p.B = m->w_head; p.ldb = D; p.rows = rows; p.N = m->V; p.K = D;
     p.epi = epi_base(); p.epi.kind = EPI_F32; p.epi.bias = m->b_head; p.epi.out_f32 = out; p.epi.ld_f32 = m->V;
-    gemm_std(m, st, p, batch, m->final_, D, m->head_rows, attn_norm_mode(m), c.norm_eps, m->gemm_cls);
+    if (rows_ready)
+      gemm(m, st, &p, 1, &batch, m->gemm_cls);   // rows standardised by their producers
+    else
+      gemm_std(m, st, p, batch, m->final_, D, m->head_rows, attn_norm_mode(m), c.norm_eps, m->gemm_cls);
     if (next) m->launches += launch_argmax(st, out, m->V, batch, next, m->amax_v, m->amax_i);
   } else {
     p.A = m->xhead; p.lda = D; p.B = m->w_pool; p.ldb = D; p.rows = rows; p.N = D; p.K = D;
