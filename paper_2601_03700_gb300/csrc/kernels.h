@@ -50,6 +50,13 @@ bool launch_exit_small(cudaStream_t st, const float* Xin, const float* Xout, con
                        bf16* xhat_next, int smode, float seps, int metric, int aao_len, const int* tok_pos,
                        unsigned* err);
 void launch_set_float(cudaStream_t st, float* p, float v);
+// Generation-step staging of the caller's inputs (forced NULL -> zeros) and outputs (each
+// output optional).
+void launch_stage_in(cudaStream_t st, float* d_delta, float delta, const int* tokens, int* dec_tok, const int* forced,
+                     int* dec_forced, int batch);
+void launch_stage_out(cudaStream_t st, int batch, const int* dec_exit, int* exit_out, const int* dec_next,
+                      int* next_out, const float* logits, float* logits_out, long long n_logits, const float* sim,
+                      float* sim_out, int n_sim);
 void launch_exit_scan(cudaStream_t st, int* ctr, int in_parity, const int* flag, const int* row_tok,
                       int* row_tok_next, int* exit_tok, int* dst, int* exit_layer_out, int layer, int aao_len,
                       const int* tok_pos);

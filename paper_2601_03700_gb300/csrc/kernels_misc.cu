@@ -620,6 +620,45 @@ __global__ void set_float_kernel(float* p, float v) {
   PDL_ENTRY(); *p = v; }
 void launch_set_float(cudaStream_t st, float* p, float v) { launch_k(set_float_kernel, 1, 1, 0, st, p, v); }
 
+// Generation-step staging: the caller's inputs into the library's fixed buffers (the captured
+// step reads only those), in one launch instead of a kernel and two copies.
+__global__ void stage_in_kernel(float* d_delta, float delta, const int* tokens, int* dec_tok, const int* forced,
+                                int* dec_forced, int batch) {
+  PDL_ENTRY();
+  if (threadIdx.x == 0) *d_delta = delta;
+  for (int b = threadIdx.x; b < batch; b += blockDim.x) {
+    dec_tok[b] = tokens[b];
+    dec_forced[b] = forced ? forced[b] : 0;
+  }
+}
+void launch_stage_in(cudaStream_t st, float* d_delta, float delta, const int* tokens, int* dec_tok, const int* forced,
+                     int* dec_forced, int batch) {
+  launch_k(stage_in_kernel, 1, 32, 0, st, d_delta, delta, tokens, dec_tok, forced, dec_forced, batch);
+}
+
+// ... and the step's outputs out of them into the caller's buffers (each optional).
+__global__ void stage_out_kernel(int batch, const int* dec_exit, int* exit_out, const int* dec_next, int* next_out,
+                                 const float* logits, float* logits_out, long long n_logits, const float* sim,
+                                 float* sim_out, int n_sim) {
+  PDL_ENTRY();
+  const long long i0 = (long long)blockIdx.x * blockDim.x + threadIdx.x, step = (long long)gridDim.x * blockDim.x;
+  for (long long i = i0; i < batch; i += step) {
+    if (exit_out) exit_out[i] = dec_exit[i];
+    if (next_out) next_out[i] = dec_next[i];
+  }
+  if (sim_out)
+    for (long long i = i0; i < n_sim; i += step) sim_out[i] = sim[i];
+  if (logits_out)
+    for (long long i = i0; i < n_logits; i += step) logits_out[i] = logits[i];
+}
+void launch_stage_out(cudaStream_t st, int batch, const int* dec_exit, int* exit_out, const int* dec_next,
+                      int* next_out, const float* logits, float* logits_out, long long n_logits, const float* sim,
+                      float* sim_out, int n_sim) {
+  const int grid = logits_out ? (int)std::min<long long>(304, (n_logits + 255) / 256) : 1;
+  launch_k(stage_out_kernel, std::max(grid, 1), 256, 0, st, batch, dec_exit, exit_out, dec_next, next_out, logits,
+           logits_out, n_logits, sim, sim_out, n_sim);
+}
+
 // After layer N: the remaining active rows' s_N are their final states.
 __global__ void final_scatter_kernel(const float* X, int D, const int* n_rows, const int* row_tok, float* final_,
                                      int* exit_layer_out, int n_layers) {

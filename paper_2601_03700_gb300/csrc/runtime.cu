@@ -1441,12 +1441,7 @@ adept_status adept_decode_step(adept_model* m, int batch, const int32_t* d_token
     return check_launch(m);
   }
   // inputs into the staging buffers; the step itself reads and writes only those
-  launch_set_float(st, m->d_delta, delta);
-  CUDA_TRY(m, cudaMemcpyAsync(m->dec_tok, d_tokens, batch * sizeof(int32_t), cudaMemcpyDeviceToDevice, st));
-  if (d_forced_exit)
-    CUDA_TRY(m, cudaMemcpyAsync(m->dec_forced, d_forced_exit, batch * sizeof(int32_t), cudaMemcpyDeviceToDevice, st));
-  else
-    CUDA_TRY(m, cudaMemsetAsync(m->dec_forced, 0, batch * sizeof(int32_t), st));
+  launch_stage_in(st, m->d_delta, delta, d_tokens, m->dec_tok, d_forced_exit, m->dec_forced, batch);
   m->launches += 1;
   auto body = [&](cudaStream_t s) -> adept_status {
     TRY(run_pass(m, batch, batch, 1, true, m->dec_tok, m->dec_forced, m->dec_exit, m->dec_sim, s));
@@ -1482,18 +1477,12 @@ adept_status adept_decode_step(adept_model* m, int batch, const int32_t* d_token
     m->dec_warm[batch] += 1;
   }
   for (int b = 0; b < batch; ++b) m->h_seq_len[b] += 1;
-  // outputs out of the staging buffers
-  const int nout = m->V;
-  if (d_exit_layer_out)
-    CUDA_TRY(m, cudaMemcpyAsync(d_exit_layer_out, m->dec_exit, batch * sizeof(int32_t), cudaMemcpyDeviceToDevice, st));
-  if (d_next_token_out)
-    CUDA_TRY(m, cudaMemcpyAsync(d_next_token_out, m->dec_next, batch * sizeof(int32_t), cudaMemcpyDeviceToDevice, st));
-  if (d_logits_out)
-    CUDA_TRY(m, cudaMemcpyAsync(d_logits_out, m->logits_ws, (size_t)batch * nout * sizeof(float),
-                                cudaMemcpyDeviceToDevice, st));
-  if (d_sim_out)
-    CUDA_TRY(m, cudaMemcpyAsync(d_sim_out, m->dec_sim, (size_t)batch * m->N * sizeof(float), cudaMemcpyDeviceToDevice,
-                                st));
+  // outputs out of the staging buffers, one launch
+  if (d_exit_layer_out || d_next_token_out || d_logits_out || d_sim_out) {
+    launch_stage_out(st, batch, m->dec_exit, d_exit_layer_out, m->dec_next, d_next_token_out, m->logits_ws,
+                     d_logits_out, (long long)batch * m->V, m->dec_sim, d_sim_out, batch * m->N);
+    m->launches += 1;
+  }
   return check_launch(m);
 }
 
