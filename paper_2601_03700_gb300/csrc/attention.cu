@@ -503,17 +503,25 @@ __device__ __forceinline__ bool ad_wait(uint64_t* bar, unsigned* err) {
   return true;
 }
 
-// CL: the chunks of a (row, kv head) form one thread-block cluster (n_split <= 8); every
+// CL: the chunks of a (token, kv head) form one thread-block cluster (n_split <= 8); every
 // CTA pushes its chunk partials into the rank-0 CTA's shared memory (st.async, completing
 // on its mbarrier), which merges them; otherwise partials go through global memory and the
 // last CTA to arrive merges.
+//
+// CTAs are indexed by the step's token (not by its compacted row), so each CTA knows before
+// the grid-dependency wait which cache blocks it reads: the blocks below the block of the
+// token's own position were written by earlier steps (or the prompt pass) and are copied
+// before the wait, overlapping the preceding kernels; the block holding the new key is
+// copied after it.  The token's row among this layer's active rows is found after the wait;
+// a token that left at an earlier layer lets its copies land and leaves.  The copy barrier
+// takes two arrivals (before and after the wait), so it cannot complete between them.
 template <int DH, bool CL>
 __global__ void __launch_bounds__(AD_THREADS)
     attn_decode_kernel(const bf16* __restrict__ q, int ld_q, DevRange rows, const int* row_tok, const int* tok_seq,
                        const int* tok_pos, const int* seq_len, KVCacheView cache, int layer0, int n_heads, int causal,
                        float scale_log2, int n_split, float* __restrict__ ws, int* counters, bf16* __restrict__ out,
                        int ld_out, unsigned* err) {
-  PDL_ENTRY();
+  KT_BEGIN();
   constexpr int PARTS = DH / 8;                    // 16-byte pieces of a K / V row
   constexpr int KPI = 32 / PARTS;                  // keys per warp instruction
   constexpr int KIT = AD_CHUNK / (4 * KPI);        // key groups per warp
@@ -525,28 +533,29 @@ __global__ void __launch_bounds__(AD_THREADS)
   __shared__ float s_red[AD_THREADS / 32];
   __shared__ float s_o[AD_THREADS / 32][DH];
   __shared__ int s_last;
+  __shared__ int s_row;
   __shared__ __align__(8) uint64_t red_bar;   // CL leader: the other chunks' partials
   constexpr int PW = DH + 4;                  // floats per pushed partial: o[DH], m, l, pad
 
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int Hkv = cache.n_kv_heads, group = n_heads / Hkv;
   const int rk = blockIdx.x, split = blockIdx.y;
-  const int rrel = rk / Hkv, kvh = rk - rrel * Hkv;
-  const int r = rows.b() + rrel;
-  if (r >= rows.e()) return;
-  const int tok = row_tok[r];
-  const int sq = tok_seq[tok], pos = tok_pos[tok];
+  const int t = rk / Hkv, kvh = rk - t * Hkv;   // the step's token t (its sequence and position
+                                                // come from the pass's first kernel)
+  const int sq = tok_seq[t], pos = tok_pos[t];
   const int nk = causal ? pos + 1 : seq_len[sq];
-  const int n_eff = (nk + AD_CHUNK - 1) / AD_CHUNK;   // chunks holding keys of this row
+  const int n_eff = (nk + AD_CHUNK - 1) / AD_CHUNK;   // chunks holding keys of this token
   if (!CL && split >= n_eff) return;   // (a cluster's CTAs all stay: they push empty partials)
   const int k_lo = split * AD_CHUNK, nkc = max(0, min(nk - k_lo, AD_CHUNK));
   const int nb = (nkc + 15) >> 4;                      // cache blocks of the chunk
+  // blocks of the chunk below the block of the token's own position: written before this step
+  const int n_pre = max(0, min(nb, (pos >> 4) - (k_lo >> 4)));
   float* sPart = reinterpret_cast<float*>(ad_smem + 2 * AD_CHUNK * DH * 2);   // CL: [group][n_split][PW]
   constexpr int BLOCK_BYTES = 16 * DH * 2;
   KT_MARK(0);
 
   if (tid == 0) {
-    asm volatile("mbarrier.init.shared::cta.b64 [%0], 1;" ::"r"(ad_smem_u32(&bar)) : "memory");
+    asm volatile("mbarrier.init.shared::cta.b64 [%0], 2;" ::"r"(ad_smem_u32(&bar)) : "memory");
     if (CL) {
       asm volatile("mbarrier.init.shared::cta.b64 [%0], 1;" ::"r"(ad_smem_u32(&red_bar)) : "memory");
     }
@@ -557,31 +566,71 @@ __global__ void __launch_bounds__(AD_THREADS)
                    : "memory");
   }
   __syncthreads();
+  // copy of block lane of the chunk (lane < nb) into its K / V slots
+  auto copy_block = [&](int b) {
+    const int bi = (k_lo >> 4) + b;
+    int blk = (sq >= 0 && sq < cache.max_batch && bi < cache.max_blocks_per_seq)
+                  ? cache.block_table[sq * cache.max_blocks_per_seq + bi]
+                  : -1;
+    if (blk < 0 || blk >= cache.n_blocks) {   // no reserved block: flag, copy block 0 (results unused)
+      atomicOr(err, ERRW_POS);
+      blk = 0;
+    }
+    const size_t off = (((size_t)layer0 * cache.n_blocks + blk) * Hkv + kvh) * (size_t)(16 * DH);
+    asm volatile("cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(
+                     ad_smem_u32(sK + b * 16 * DH)),
+                 "l"((const bf16*)cache.k + off), "r"((uint32_t)BLOCK_BYTES), "r"(ad_smem_u32(&bar))
+                 : "memory");
+    asm volatile("cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(
+                     ad_smem_u32(sV + b * 16 * DH)),
+                 "l"((const bf16*)cache.v + off), "r"((uint32_t)BLOCK_BYTES), "r"(ad_smem_u32(&bar))
+                 : "memory");
+  };
   if (warp == 0) {
     if (lane == 0)
       asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(ad_smem_u32(&bar)),
-                   "r"((uint32_t)(2 * nb * BLOCK_BYTES))
+                   "r"((uint32_t)(2 * n_pre * BLOCK_BYTES))
                    : "memory");
     __syncwarp();
-    if (lane < nb) {
-      const int bi = (k_lo >> 4) + lane;
-      int blk = (sq >= 0 && sq < cache.max_batch && bi < cache.max_blocks_per_seq)
-                    ? cache.block_table[sq * cache.max_blocks_per_seq + bi]
-                    : -1;
-      if (blk < 0 || blk >= cache.n_blocks) {   // no reserved block: flag, copy block 0 (results unused)
-        atomicOr(err, ERRW_POS);
-        blk = 0;
-      }
-      const size_t off = (((size_t)layer0 * cache.n_blocks + blk) * Hkv + kvh) * (size_t)(16 * DH);
-      asm volatile("cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(
-                       ad_smem_u32(sK + lane * 16 * DH)),
-                   "l"((const bf16*)cache.k + off), "r"((uint32_t)BLOCK_BYTES), "r"(ad_smem_u32(&bar))
-                   : "memory");
-      asm volatile("cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(
-                       ad_smem_u32(sV + lane * 16 * DH)),
-                   "l"((const bf16*)cache.v + off), "r"((uint32_t)BLOCK_BYTES), "r"(ad_smem_u32(&bar))
-                   : "memory");
+    if (lane < n_pre) copy_block(lane);
+  }
+  pdl_wait();
+  KT_WAITED();
+  pdl_launch_dependents();
+  // this token's row among the layer's active rows (rows keep token order), or -1
+  if (warp == 0) {
+    const int rb = rows.b(), M = rows.e() - rb;
+    int found = -1;
+    for (int j0 = 0; j0 < M && found < 0; j0 += 32) {
+      const int j = j0 + lane;
+      const unsigned hit = __ballot_sync(0xffffffffu, j < M && row_tok[rb + j] == t);
+      if (hit) found = rb + j0 + __ffs(hit) - 1;
     }
+    if (lane == 0) s_row = found;
+  }
+  __syncthreads();
+  const int r = s_row;
+  if (warp == 0) {
+    // second arrival: the block holding the new key (active tokens), or none
+    if (lane == 0) {
+      if (r >= 0)
+        asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(ad_smem_u32(&bar)),
+                     "r"((uint32_t)(2 * (nb - n_pre) * BLOCK_BYTES))
+                     : "memory");
+      else
+        asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(ad_smem_u32(&bar)) : "memory");
+    }
+    __syncwarp();
+    if (r >= 0 && lane >= n_pre && lane < nb) copy_block(lane);
+  }
+  if (r < 0) {
+    // the token left at an earlier layer (uniform over the cluster): let the copies land, leave
+    if (warp == 0 && lane == 0) {
+      bool ok = ad_wait(&bar, err);
+      if (!ok) ad_wait(&bar, err);
+    }
+    __syncthreads();
+    return;
   }
   const int slot = lane / PARTS, part = lane - slot * PARTS;
   // the first query head's piece (8 dims per lane), fetched while the cache blocks are in flight
@@ -590,7 +639,7 @@ __global__ void __launch_bounds__(AD_THREADS)
   // CTA arrives here (after the initialisation) and waits only just before its first push
   if (CL) asm volatile("barrier.cluster.arrive.release.aligned;" ::: "memory");
   KT_MARK(1);
-  if (nb > 0) {
+  {
     bool ok = ad_wait(&bar, err);
     if (!ok) ad_wait(&bar, err);   // second bounded wait for the copies in flight; results flagged
   }
@@ -696,7 +745,7 @@ __global__ void __launch_bounds__(AD_THREADS)
       for (int i = 0; i < 8; ++i) s_o[warp][part * 8 + i] = o[i];
     }
     __syncthreads();
-    const int rh = rrel * n_heads + h;
+    const int rh = t * n_heads + h;
     if (CL) {
       if (g == 0) asm volatile("barrier.cluster.wait.acquire.aligned;" ::: "memory");
       // chunk partial (empty chunk: m = -inf, l = 0, o = 0) -> slot [g][split] of the leader
