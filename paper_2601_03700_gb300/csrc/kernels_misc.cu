@@ -722,6 +722,79 @@ __device__ __forceinline__ void block_sum_n(float (&v)[NV], float* red) {
   }
 }
 
+// embed_kernel with the row held in registers (EPT elements per thread, all loads issued
+// before the first reduction): rows of up to 16 x blockDim.x elements.
+template <typename T, int EPT>
+__global__ void __launch_bounds__(256) embed_reg_kernel(const int* tokens, int n_tok, const int* tok_pos, const T* E,
+                                                        const T* P, const float* type_emb, const float* g,
+                                                        const float* b, int family, int D, int V, float eps, float* X,
+                                                        unsigned* err, bf16* xhat, int smode, float seps) {
+  PDL_ENTRY();
+  __shared__ float red[32];
+  const int t = blockIdx.x;
+  if (t >= n_tok) return;
+  int tok = tokens[t];
+  if (tok < 0 || tok >= V) {
+    if (threadIdx.x == 0) atomicOr(err, ERRW_TOKEN);
+    tok = 0;
+  }
+  const int pos = tok_pos[t];
+  float v[EPT];
+#pragma unroll
+  for (int j = 0; j < EPT; ++j) {
+    const int d = threadIdx.x + j * blockDim.x;
+    float x = 0.f;
+    if (d < D) {
+      x = to_f(E[(size_t)tok * D + d]);
+      if (P) x += to_f(P[(size_t)pos * D + d]);
+      if (type_emb) x += type_emb[d];
+    }
+    v[j] = x;
+  }
+  float* x = X + (size_t)t * D;
+  float s1[1] = {0.f};
+#pragma unroll
+  for (int j = 0; j < EPT; ++j) s1[0] += v[j];
+  const bool ln = family == 2 || smode == NORM_LN;
+  if (family != 2) {
+#pragma unroll
+    for (int j = 0; j < EPT; ++j) {
+      const int d = threadIdx.x + j * blockDim.x;
+      if (d < D) x[d] = v[j];
+    }
+    if (!xhat) return;
+  }
+  float mu = 0.f;
+  if (ln) {
+    block_sum_n<1>(s1, red);
+    mu = s1[0] / D;
+  }
+  float s2[1] = {0.f};
+#pragma unroll
+  for (int j = 0; j < EPT; ++j) {
+    const int d = threadIdx.x + j * blockDim.x;
+    const float c = d < D ? v[j] - mu : 0.f;
+    s2[0] += c * c;
+  }
+  block_sum_n<1>(s2, red);
+  if (family != 2) {
+    const float rs = smode == NORM_COPY ? 1.f : rsqrtf(s2[0] / D + seps);
+    const float m0 = smode == NORM_COPY ? 0.f : mu;
+#pragma unroll
+    for (int j = 0; j < EPT; ++j) {
+      const int d = threadIdx.x + j * blockDim.x;
+      if (d < D) xhat[(size_t)t * D + d] = __float2bfloat16_rn((v[j] - m0) * rs);
+    }
+    return;
+  }
+  const float rstd = rsqrtf(s2[0] / D + eps);
+#pragma unroll
+  for (int j = 0; j < EPT; ++j) {
+    const int d = threadIdx.x + j * blockDim.x;
+    if (d < D) x[d] = (v[j] - mu) * rstd * g[d] + b[d];
+  }
+}
+
 // Three separately RMS-normalised rows (shared gain g0), then the 3x3 convolution with
 // padding (0, 1): c0[t] = b + sum_a sum_u w[a][u] Xn_a[t + u - 1], Xn_a = x_a rstd_a g0.
 // Dynamic shared memory: the three normalised rows, 3 * D floats.
@@ -1203,6 +1276,20 @@ void launch_pass_init(cudaStream_t st, int n_tok, int prompt_len, int decode, in
 void launch_embed(cudaStream_t st, int dt, const int* tokens, int n_tok, const int* tok_pos, const void* E,
                   const void* P, const float* type_emb, const float* g, const float* b, int family, int D, int V,
                   float eps, float* X, unsigned* err, bf16* xhat, int smode, float seps) {
+  if (D <= 16 * 256) {
+#define EMB(T, EPT)                                                                                                  \
+  launch_k(embed_reg_kernel<T, EPT>, n_tok, 256, 0, st, tokens, n_tok, tok_pos, (const T*)E, (const T*)P, type_emb, g, \
+           b, family, D, V, eps, X, err, xhat, smode, seps)
+    if (dt == 1) {
+      if (D <= 4 * 256) EMB(bf16, 4);
+      else EMB(bf16, 16);
+    } else {
+      if (D <= 4 * 256) EMB(float, 4);
+      else EMB(float, 16);
+    }
+#undef EMB
+    return;
+  }
   if (dt == 1)
     launch_k(embed_kernel<bf16>, n_tok, 256, 0, st, tokens, n_tok, tok_pos, (const bf16*)E, (const bf16*)P, type_emb, g,
              b, family, D, V, eps, X, err, xhat, smode, seps);
@@ -1376,11 +1463,21 @@ __global__ void argmax_part_kernel(const float* logits, int V, int rows, float* 
   const float* l = logits + (size_t)r * V;
   float bv = -INFINITY;
   int bi = 0x7fffffff;
-  for (int v = lo + threadIdx.x; v < hi; v += blockDim.x) {
-    const float x = l[v];
-    if (x > bv || (x == bv && v < bi)) {
-      bv = x;
-      bi = v;
+  // the thread's values in groups of 8 loads in flight (ties: the lowest index wins in any order)
+  for (int v0 = lo + threadIdx.x; v0 < hi; v0 += 8 * blockDim.x) {
+    float x[8];
+#pragma unroll
+    for (int u = 0; u < 8; ++u) {
+      const int v = v0 + u * blockDim.x;
+      x[u] = v < hi ? l[v] : -INFINITY;
+    }
+#pragma unroll
+    for (int u = 0; u < 8; ++u) {
+      const int v = v0 + u * blockDim.x;
+      if (v < hi && (x[u] > bv || (x[u] == bv && v < bi))) {
+        bv = x[u];
+        bi = v;
+      }
     }
   }
 #pragma unroll
