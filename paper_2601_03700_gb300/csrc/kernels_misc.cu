@@ -415,7 +415,11 @@ __global__ void __launch_bounds__(EXD_THREADS)
                        float* __restrict__ hsm_s, float* __restrict__ hsm_prev, float* __restrict__ hsm_I, int rshift,
                        int max_rows, bf16* xhat_next, int smode, float seps, int metric, int aao_len,
                        const int* tok_pos, unsigned* err) {
-  PDL_ENTRY();
+  // Before the grid-dependency wait: everything the previous layer's exit kernel wrote (the
+  // counters, the row map, the inertia and the layer input s_{i-1}), which has completed by the
+  // time this kernel starts (the attention kernel between them releases its dependents only
+  // after its own wait); after it: the layer output s_i.
+  KT_BEGIN();
   __shared__ float s_red[EXD_THREADS / 32][6];
   __shared__ float s_mu[16];
   __shared__ int s_dst[16], s_tok[16];
@@ -434,17 +438,26 @@ __global__ void __launch_bounds__(EXD_THREADS)
   float4 xs[EXD_V], xi[EXD_V], xp[EXD_V];
   float ns = 0.f, ni = 0.f, dot = 0.f, sx = 0.f, np_ = 0.f, dp = 0.f;
   if (row < max_rows) {
-    const float4* s4 = reinterpret_cast<const float4*>(Xout + (size_t)row * D);
     const float4* i4 = reinterpret_cast<const float4*>(I + (size_t)row * D);
     const float4* p4 = reinterpret_cast<const float4*>(Xin + (size_t)row * D);
 #pragma unroll
     for (int j = 0; j < EXD_V; ++j) {
       const int v = sub + j * tpr;
       if (v < D4) {
-        xs[j] = s4[v];
         xi[j] = first ? make_float4(0.f, 0.f, 0.f, 0.f) : i4[v];
         xp[j] = p4[v];
       }
+    }
+  }
+  pdl_wait();
+  KT_WAITED();
+  pdl_launch_dependents();
+  if (row < max_rows) {
+    const float4* s4 = reinterpret_cast<const float4*>(Xout + (size_t)row * D);
+#pragma unroll
+    for (int j = 0; j < EXD_V; ++j) {
+      const int v = sub + j * tpr;
+      if (v < D4) xs[j] = s4[v];
     }
 #pragma unroll
     for (int j = 0; j < EXD_V; ++j) {
