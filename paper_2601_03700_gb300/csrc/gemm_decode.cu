@@ -99,6 +99,21 @@ struct DgParams {
   unsigned* err;
 };
 
+// Several problems of one launch that differ only in the weights, the row range and the
+// epilogue (the grouped skipped-layer fill: one problem per layer), blockIdx.y = problem.
+constexpr int DG_MAX_GROUPS = 32;
+struct DgParamsG : DgParams {
+  CUtensorMap gmap[DG_MAX_GROUPS];
+  DevRange grows[DG_MAX_GROUPS];
+  Epi gepi[DG_MAX_GROUPS];
+};
+__device__ __forceinline__ const CUtensorMap* dg_wmap(const DgParams& p) { return &p.wmap; }
+__device__ __forceinline__ const CUtensorMap* dg_wmap(const DgParamsG& p) { return &p.gmap[blockIdx.y]; }
+__device__ __forceinline__ DevRange dg_rows(const DgParams& p) { return p.rows; }
+__device__ __forceinline__ DevRange dg_rows(const DgParamsG& p) { return p.grows[blockIdx.y]; }
+__device__ __forceinline__ const Epi& dg_epi(const DgParams& p) { return p.epi; }
+__device__ __forceinline__ const Epi& dg_epi(const DgParamsG& p) { return p.gepi[blockIdx.y]; }
+
 __device__ __forceinline__ uint32_t smem_u32(const void* p) { return (uint32_t)__cvta_generic_to_shared(p); }
 __device__ __forceinline__ void mbar_init(uint64_t* bar, uint32_t count) {
   asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(smem_u32(bar)), "r"(count) : "memory");
@@ -196,8 +211,8 @@ __device__ __forceinline__ void cluster_sync() {
   asm volatile("barrier.cluster.arrive.release.aligned;\nbarrier.cluster.wait.acquire.aligned;" ::: "memory");
 }
 // MB: 8-token blocks of the A operand (1: M <= 8, 2: M <= 16); KIND: the epilogue kind.
-template <int MB, int KIND>
-__global__ void __launch_bounds__(DG_THREADS, 1) gemm_decode_kernel(const __grid_constant__ DgParams p) {
+template <int MB, int KIND, class P = DgParams>
+__global__ void __launch_bounds__(DG_THREADS, 1) gemm_decode_kernel(const __grid_constant__ P p) {
   KT_BEGIN();
   extern __shared__ __align__(128) uint8_t dg_smem_raw[];
   __shared__ __align__(8) uint64_t full[DG_MAX_STAGES];
@@ -250,7 +265,7 @@ __global__ void __launch_bounds__(DG_THREADS, 1) gemm_decode_kernel(const __grid
     const int f = (tile0 + j * tstride) * DG_BN;
     const int s = g % S;
     mbar_expect_tx(&full[s], (uint32_t)stage_bytes);
-    tma_load_3d(&p.wmap, &full[s], sW + (size_t)s * stage_bytes, f, (k_lo + kb * ks) >> 6);
+    tma_load_3d(dg_wmap(p), &full[s], sW + (size_t)s * stage_bytes, f, (k_lo + kb * ks) >> 6);
   };
   const int first = min(S, G);
   const int pre = min(p.pre, first);
@@ -262,8 +277,9 @@ __global__ void __launch_bounds__(DG_THREADS, 1) gemm_decode_kernel(const __grid
   pdl_wait();   // from here on, the preceding kernels' writes are visible
   KT_WAITED();
 
-  const int rb = p.rows.b();
-  int M = p.rows.e() - rb;
+  const DevRange prow = dg_rows(p);
+  const int rb = prow.b();
+  int M = prow.e() - rb;
   if (M > p.max_m) {   // more rows than the launch was sized for
     if (tid == 0) atomicOr(p.err, ERRW_CONFIG);
     M = p.max_m;
@@ -280,7 +296,7 @@ __global__ void __launch_bounds__(DG_THREADS, 1) gemm_decode_kernel(const __grid
   KT_MARK(0);
 
   // ---- one round trip: operand rows (warps 0-2) and the epilogue's inputs (warp 3)
-  const Epi& e = p.epi;
+  const Epi& e = dg_epi(p);
   const bool leader = rank == 0;
   // bias and residual columns are staged for a CTA with a single full tile
   const bool single = my_tiles == 1 && (tile0 + 1) * DG_BN <= p.N;
@@ -696,6 +712,40 @@ cudaError_t launch_dg(cudaStream_t st, const DgParams& prm, int grid, size_t sme
   return cudaLaunchKernelEx(&cfg, gemm_decode_kernel<MB, KIND>, prm);
 }
 
+// Grouped launch (EPI_KV problems): grid (gx, groups), clusters along x.
+template <int MB>
+cudaError_t launch_dg_grouped(cudaStream_t st, const DgParamsG& prm, int gx, int groups, size_t smem) {
+  static bool attr = false;
+  if (!attr) {
+    const cudaError_t e = cudaFuncSetAttribute(gemm_decode_kernel<MB, EPI_KV, DgParamsG>,
+                                               cudaFuncAttributeMaxDynamicSharedMemorySize, DG_SMEM_LIMIT);
+    if (e != cudaSuccess) return e;
+    attr = true;
+  }
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(gx, groups);
+  cfg.blockDim = dim3(DG_THREADS);
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = st;
+  cudaLaunchAttribute at[2];
+  int na = 0;
+  if (prm.splits > 1) {
+    at[na].id = cudaLaunchAttributeClusterDimension;
+    at[na].val.clusterDim.x = prm.splits;
+    at[na].val.clusterDim.y = 1;
+    at[na].val.clusterDim.z = 1;
+    ++na;
+  }
+  if (g_pdl) {
+    at[na].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    at[na].val.programmaticStreamSerializationAllowed = 1;
+    ++na;
+  }
+  cfg.attrs = at;
+  cfg.numAttrs = na;
+  return cudaLaunchKernelEx(&cfg, gemm_decode_kernel<MB, EPI_KV, DgParamsG>, prm);
+}
+
 template <int MB>
 cudaError_t launch_kind(cudaStream_t st, const DgParams& prm, int grid, size_t smem) {
   switch (prm.epi.kind) {
@@ -724,8 +774,11 @@ bool decode_gemm_supported(const GemmProblem& q, int max_rows, const DgNorm* nor
   return true;
 }
 
-int decode_gemm(cudaStream_t st, const GemmProblem& q, int max_rows, const DgNorm* norm, unsigned* err) {
-  if (!decode_gemm_supported(q, max_rows, norm)) return -1;
+// Launch plan of one problem (or of `groups` problems of the same shape, one per gridDim.y):
+// fills prm (except the tensor map) and the x-grid, dynamic shared memory and row blocks.
+static bool dg_plan(const GemmProblem& q, int max_rows, const DgNorm* norm, int groups, unsigned* err, DgParams& prm,
+                    int& grid_out, size_t& smem_out, int& mb_out) {
+  if (!decode_gemm_supported(q, max_rows, norm)) return false;
   if (!g_dg_sms) {
     int dev = 0;
     cudaGetDevice(&dev);
@@ -737,19 +790,17 @@ int decode_gemm(cudaStream_t st, const GemmProblem& q, int max_rows, const DgNor
   const int kr_max = dg_max_kr(mb);
   // K-splits: enough CTAs to cover the GPU about twice, each split at least one stage and
   // at most kr_max of k
-  int splits = std::max(cdiv(2 * g_dg_sms, tiles), cdiv(q.K, kr_max));
+  int splits = std::max(cdiv(2 * g_dg_sms, tiles * groups), cdiv(q.K, kr_max));
   splits = std::min(splits, std::min(DG_MAX_SPLITS, cdiv(q.K, DG_KS)));
   // long k-ranges split over a cluster stage 256 k per row (512 contiguous bytes of each
   // weight row per copy); a single split keeps 128 k, which leaves room for more resident
   // CTAs of the persistent grid (measured faster at the Llama-7B QKV shape)
   const int ks = splits > 1 && cdiv(q.K, splits) >= 1024 ? 2 * DG_KS : DG_KS;
   const int kr = cdiv(cdiv(q.K, splits), ks) * ks;
-  if (kr > kr_max) return -1;
+  if (kr > kr_max) return false;
   splits = cdiv(q.K, kr);
   const int nst = kr / ks;
   const int stage_bytes = ks * DG_BN * 2;
-  static DgParams prm;   // 64-byte-aligned tensor map; calls on a model are serialised
-  memset(&prm, 0, sizeof prm);
   prm.W = (const bf16*)q.B;
   prm.ldw = q.ldb;
   prm.A = (const bf16*)q.A;
@@ -787,14 +838,14 @@ int decode_gemm(cudaStream_t st, const GemmProblem& q, int max_rows, const DgNor
   const int tst = prm.stat_mode == DG_STATS_TILES ? prm.n_stiles : 0;
   const int fixed0 = dg_layout(0, arows, kr, prm.xrows, prm.xk, tst, splits).total + 1024;
   int grid = tiles * splits;
-  if (splits == 1) {
+  if (splits == 1 && groups == 1) {
     // as many CTAs as can be resident with a ring of at least four stages, each with the
     // same number of tiles (so that no CTA streams a tile while the others idle)
     const int cap = std::max(1, std::min(4, (227 * 1024) / (fixed0 + 4 * stage_bytes + DG_STATIC_SMEM))) * g_dg_sms;
     const int per_cta = cdiv(tiles, cap);
     grid = cdiv(tiles, per_cta);
   }
-  const int per_sm = std::min(4, cdiv(grid, g_dg_sms));
+  const int per_sm = std::min(4, cdiv(grid * groups, g_dg_sms));
   // ring stages: as many as the CTAs resident on an SM leave room for (at most the CTA's
   // stage count), so that the weight bytes in flight cover the memory latency
   const int cta_stages = cdiv(tiles, grid / splits) * nst;
@@ -802,7 +853,7 @@ int decode_gemm(cudaStream_t st, const GemmProblem& q, int max_rows, const DgNor
   stages = std::max(1, std::min(stages, std::min(DG_MAX_STAGES, cta_stages)));
   const DgLayout L = dg_layout(stages * stage_bytes, arows, kr, prm.xrows, prm.xk, tst, splits);
   const size_t smem = (size_t)L.total + 1024;   // + slack to align the ring to 1024 bytes
-  if (smem > (size_t)DG_SMEM_LIMIT) return -1;
+  if (smem > (size_t)DG_SMEM_LIMIT) return false;
   prm.stages = stages;
   prm.off_a = L.off_a;
   prm.off_x = L.off_x;
@@ -812,12 +863,50 @@ int decode_gemm(cudaStream_t st, const GemmProblem& q, int max_rows, const DgNor
   prm.resid_aligned = ((uintptr_t)q.epi.resid & 15) == 0 && q.epi.ld_resid % 4 == 0;
   prm.epi = q.epi;
   prm.err = err;
-  if (!tc_encode_weight_3d(&prm.wmap, q.B, q.K, q.N, (size_t)q.ldb * 2, DG_BN, ks / 64)) return -1;
   // a CTA whose stages fit the ring issues them all before the grid-dependency wait; a
   // longer one (large models) only its first, which bounds the weight traffic of a layer
   // whose rows have all left
   prm.pre = cta_stages <= stages ? stages : 1;
+  grid_out = grid;
+  smem_out = smem;
+  mb_out = mb;
+  return true;
+}
+
+int decode_gemm(cudaStream_t st, const GemmProblem& q, int max_rows, const DgNorm* norm, unsigned* err) {
+  static DgParams prm;   // 64-byte-aligned tensor map; calls on a model are serialised
+  memset(&prm, 0, sizeof prm);
+  int grid = 0, mb = 1;
+  size_t smem = 0;
+  if (!dg_plan(q, max_rows, norm, 1, err, prm, grid, smem, mb)) return -1;
+  if (!tc_encode_weight_3d(&prm.wmap, q.B, q.K, q.N, (size_t)q.ldb * 2, DG_BN, prm.ks / 64)) return -1;
   const cudaError_t e = mb == 2 ? launch_kind<2>(st, prm, grid, smem) : launch_kind<1>(st, prm, grid, smem);
+  return e == cudaSuccess ? 1 : -1;
+}
+
+int decode_gemm_grouped(cudaStream_t st, const GemmProblem* probs, int n, int max_rows, unsigned* err) {
+  if (n < 1 || n > DG_MAX_GROUPS) return -1;
+  const GemmProblem& q0 = probs[0];
+  for (int i = 0; i < n; ++i) {
+    const GemmProblem& q = probs[i];
+    if (q.epi.kind != EPI_KV || q.A != q0.A || q.lda != q0.lda || q.N != q0.N || q.K != q0.K || q.ldb != q0.ldb ||
+        q.rows.begin != nullptr || !decode_gemm_supported(q, max_rows, nullptr))
+      return -1;
+  }
+  static DgParamsG prm;   // calls on a model are serialised
+  memset(&prm, 0, sizeof prm);
+  int grid = 0, mb = 1;
+  size_t smem = 0;
+  if (!dg_plan(q0, max_rows, nullptr, n, err, prm, grid, smem, mb)) return -1;
+  for (int i = 0; i < n; ++i) {
+    if (!tc_encode_weight_3d(&prm.gmap[i], probs[i].B, q0.K, q0.N, (size_t)q0.ldb * 2, DG_BN, prm.ks / 64)) return -1;
+    prm.grows[i] = probs[i].rows;
+    prm.gepi[i] = probs[i].epi;
+    prm.gepi[i].tile_stats = nullptr;
+  }
+  prm.bias_aligned = 1;
+  for (int i = 0; i < n; ++i) prm.bias_aligned &= ((uintptr_t)probs[i].epi.bias & 15) == 0;
+  const cudaError_t e = mb == 2 ? launch_dg_grouped<2>(st, prm, grid, n, smem) : launch_dg_grouped<1>(st, prm, grid, n, smem);
   return e == cudaSuccess ? 1 : -1;
 }
 

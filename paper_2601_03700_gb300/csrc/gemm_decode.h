@@ -30,5 +30,9 @@ struct DgNorm {
 int decode_gemm(cudaStream_t st, const GemmProblem& p, int max_rows, const DgNorm* norm, unsigned* err);
 // Whether decode_gemm takes the problem (host-side shape and alignment checks only).
 bool decode_gemm_supported(const GemmProblem& p, int max_rows, const DgNorm* norm);
+// n (<= 32) cache-fill problems (EPI_KV) of one shape that differ only in their weights, row
+// range (rows [0, end)) and epilogue (layer, bias), as one launch (blockIdx.y = problem).
+// Returns 1, or -1 when not taken (the caller runs another path).
+int decode_gemm_grouped(cudaStream_t st, const GemmProblem* probs, int n, int max_rows, unsigned* err);
 
 }  // namespace adept

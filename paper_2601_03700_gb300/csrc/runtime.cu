@@ -947,7 +947,17 @@ static adept_status run_pass(adept_model* m, int n_tok, int batch, int prompt_le
                                  m->tok_seq, m->tok_pos));
       mrs.push_back(n_tok);
     }
-    gemm(m, st, probs.data(), (int)probs.size(), mrs.data(), ADEPT_PROF_KV_FILL);
+    // one weight-streaming launch over the skipped layers when the rows fit it, else the
+    // grouped tcgen05 GEMM
+    bool done = false;
+    if (m->dt == ADEPT_DTYPE_BF16 && m->use_dg && !m->force_simt && n_tok <= DG_MAX_M) {
+      cudaEvent_t b = nullptr;
+      prof_begin(m, ADEPT_PROF_KV_FILL, st, &b);
+      done = decode_gemm_grouped(st, probs.data(), (int)probs.size(), n_tok, m->err_word) >= 0;
+      prof_end(m, ADEPT_PROF_KV_FILL, st, b, 0, 0);
+      if (done) m->launches += 1;
+    }
+    if (!done) gemm(m, st, probs.data(), (int)probs.size(), mrs.data(), ADEPT_PROF_KV_FILL);
   }
   return ADEPT_OK;
 }
