@@ -790,12 +790,15 @@ def kernel_case_llama_decode_small(device):
     m.close()
 
 
-def kernel_case_hsm_train(device, n=8192, steps=2):
-    """HSM training steps at GPT-2-small shapes (the bench section's workload): n examples,
-    two steps after one warm-up step; about 5 GB on the device."""
+def kernel_case_hsm_train(device, n=8192, steps=2, shape="gpt2"):
+    """HSM training steps at GPT-2-small shapes (the bench section's workload; about 5 GB on
+    the device) or Llama-2-7B shapes (about 25 GB): n examples, two steps after one warm-up."""
     import paper_2601_03700_gb300 as adept
     adept.load_library()
-    cfg = synth.gpt2_small_config(n_layers=2, max_batch=1, max_seq=16)
+    if shape == "llama7b":
+        cfg = synth.llama7b_config(n_layers=2, max_batch=1, max_seq=16)
+    else:
+        cfg = synth.gpt2_small_config(n_layers=2, max_batch=1, max_seq=16)
     W = synth.make_weights(cfg, seed=0)   # on the host: the launch list then holds the library's kernels only
     m = adept.Model(cfg, W)
     del W
@@ -824,6 +827,7 @@ def main():
     ap.add_argument("--fill-i", default="4,8,16,24")
     ap.add_argument("--cpu-tokens", type=int, default=512)
     ap.add_argument("--hsm-n", type=int, default=8192, help="examples per step of --kernel-case hsm_train")
+    ap.add_argument("--hsm-shape", default="gpt2", choices=["gpt2", "llama7b"], help="model shape of --kernel-case hsm_train")
     args = ap.parse_args()
     if args.kernel_case == "fill_small":
         kernel_case_fill_small(torch.device("cuda", 0))
@@ -838,7 +842,7 @@ def main():
         kernel_case_llama_decode_small(torch.device("cuda", 0))
         return
     if args.kernel_case == "hsm_train":
-        kernel_case_hsm_train(torch.device("cuda", 0), n=args.hsm_n)
+        kernel_case_hsm_train(torch.device("cuda", 0), n=args.hsm_n, shape=args.hsm_shape)
         return
     world = int(os.environ.get("WORLD_SIZE", "1"))
     rank = int(os.environ.get("RANK", "0"))

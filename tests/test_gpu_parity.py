@@ -108,12 +108,12 @@ def test_bf16_families_threshold(family):
 
 # --------------------------------------------------------------------------- skipped-layer fill ABI
 
-@pytest.mark.parametrize("dtype", ["f32", "bf16"])
-def test_skip_kv_fill_matches_oracle(dtype):
-    """adept_skip_kv_fill: every (token, r > i*) entry equals layer r's K/V projection of s~."""
+@pytest.mark.parametrize("dtype,n", [("f32", 150), ("bf16", 150), ("bf16", 7)])
+def test_skip_kv_fill_matches_oracle(dtype, n):
+    """adept_skip_kv_fill: every (token, r > i*) entry equals layer r's K/V projection of s~
+    (7 bf16 tokens take the grouped weight-streaming launch, 150 the grouped tcgen05 GEMM)."""
     cfg = small(synth.LLAMA, dtype=dtype, n_layers=8, n_heads=2, head_dim=128, block_shuffle_seed=7)
     pair = Pair(cfg, seed=8)
-    n = 150
     lens = [cfg.max_seq] * cfg.max_batch
     adept.adept_seq_reserve(pair.gm.h, lens)
     h = synth.make_mapped_states(9, n, cfg.d_model, dtype=cfg.torch_dtype)
@@ -138,7 +138,7 @@ def test_skip_kv_fill_matches_oracle(dtype):
             assert_rows_close(gk[pos[rows]], k[np.searchsorted(sel, rows)], pair.tol, f"K r={r}")
             assert_rows_close(gv[pos[rows]], v[np.searchsorted(sel, rows)], pair.tol, f"V r={r}")
             checked += len(rows)
-    assert checked > n
+    assert checked >= n - int(np.sum(el == cfg.n_layers))
     pair.close()
 
 
