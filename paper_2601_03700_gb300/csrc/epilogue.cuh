@@ -76,6 +76,37 @@ __device__ __forceinline__ void rope_pairs(T* dst, int i0, int half, const float
   store16<T>(dst + i0 + half, b);
 }
 
+// A short tanh for the tanh form of GELU with bf16 results (its error stays far below the bf16
+// rounding of the output): the hardware approximation tanh.approx.f32, relative error about
+// 2^-11.
+__device__ __forceinline__ float tanh_approx(float x) {
+  float y;
+  asm("tanh.approx.f32 %0, %1;" : "=f"(y) : "f"(x));
+  return y;
+}
+
+// The activation of a 32-value chunk, switched once per chunk: a per-element switch in the
+// unrolled loop would lay out 32 copies of every activation's code (for the epilogue warps of
+// the tcgen05 GEMM, instruction fetch then dominated: GELU epilogues ran 5x slower than the
+// others).  The tanh form of GELU with bf16 results uses tanh_approx; the rest keep tanhf / erff.
+template <typename T>
+__device__ __forceinline__ void act_chunk32(int act, float (&v)[32]) {
+  constexpr bool fast = sizeof(T) == 2;
+  if (act == ACT_GELU_TANH) {
+#pragma unroll
+    for (int j = 0; j < 32; ++j) {
+      const float x = v[j], u = 0.79788456080286536f * (x + 0.044715f * x * x * x);
+      v[j] = 0.5f * x * (1.f + (fast ? tanh_approx(u) : tanhf(u)));
+    }
+  } else if (act == ACT_GELU_ERF) {
+#pragma unroll
+    for (int j = 0; j < 32; ++j) v[j] = gelu_erf_f(v[j]);
+  } else if (act == ACT_TANH) {   // the encoder's pooler (one row per sequence): kept exact
+#pragma unroll
+    for (int j = 0; j < 32; ++j) v[j] = tanhf(v[j]);
+  }
+}
+
 // bias32 / resid32 (optional): the chunk's 32 bias values and the row's 32 residual
 // values already staged by the caller (e.g. in shared memory) instead of e.bias[c0..] and
 // e.resid[ra][c0..].  applied (EPI_APPLIED_* bits): what the caller has already done to v
@@ -109,10 +140,7 @@ __device__ __forceinline__ void epi_chunk32(const Epi& e, int ra, int c0, int N,
       return;
     }
     case EPI_ACT: {
-      if (!(applied & EPI_APPLIED_BIAS_ACT)) {
-#pragma unroll
-        for (int j = 0; j < 32; ++j) v[j] = apply_act(e.act, v[j]);
-      }
+      if (!(applied & EPI_APPLIED_BIAS_ACT)) act_chunk32<T>(e.act, v);
       T* o = (T*)e.out_t + (size_t)ra * e.ld_t + c0;
       if (full && ((e.ld_t & 15) == 0)) {
         store16<T>(o, v);
