@@ -433,6 +433,7 @@ __global__ void __launch_bounds__(EXD_THREADS)
   const int n = min(min(ctr[CTR_ACTIVE + par], 1 << rshift), max_rows);
   const int base = ctr[CTR_EXITED];
   const int tok_r = (int)threadIdx.x < max_rows ? row_tok[threadIdx.x] : 0;
+  const int forced_r = forced && (int)threadIdx.x < max_rows ? forced[tok_r] : 0;   // the decider's forced layer
   const float delta = *delta_p;
   const int D4 = D >> 2;
   float4 xs[EXD_V], xi[EXD_V], xp[EXD_V];
@@ -506,7 +507,7 @@ __global__ void __launch_bounds__(EXD_THREADS)
     if (test) {
       const float cs = exit_similarity(metric, a, b, c, pn, pd);
       if (sim) sim[(size_t)tok * n_layers + (layer - 1)] = cs;
-      const int f = forced ? forced[tok] : 0;
+      const int f = forced_r;
       if (f != 0 && (f < 2 || f > n_layers)) atomicOr(err, ERRW_FORCED);
       ex = (f > 0) ? (f == layer) : (cs >= delta);
     }
