@@ -14,11 +14,19 @@ the next input token (labels = one-position-shifted input tokens) is minimised w
   gain g0), a 3x3 convolution with padding (0, 1), FC1 and FC2 with erf-GELU, FC3, RMSNorm
   with gain g1 plus FC1's output, FC4, RMSNorm with gain g2 plus the convolution output.
 * The loss is the mean over the n examples of -log softmax(logits)[target].
+* Classification (encoders, Sec. 4.3): with no next token to predict, the mapped state is
+  pulled toward the original final hidden state s_N of the same token by a similarity loss,
+  and the task loss of the frozen pooler and classifier is added.  Read here as: similarity
+  loss = mean over the n examples of 1 - cos(s~, s_N) (cos taken as 0 where a norm is 0);
+  task loss = softmax cross-entropy of the classifier's logits on the pooled mapped state of
+  the first n_cls examples (the [CLS] rows that carry a label; with two classes this is the
+  binary cross-entropy of the class-1 probability), averaged over those rows and weighted by
+  cls_weight (1 by default: the paper adds the two).
 * AdamW is the decoupled-weight-decay Adam of Loshchilov & Hutter, written out: m = b1 m +
   (1 - b1) g, v = b2 v + (1 - b2) g^2, theta -= lr (m / (1 - b1^t)) / (sqrt(v / (1 - b2^t)) +
   eps) + lr wd theta (the decay applied to the parameter before this step's update).
-* Precision: float64 throughout.  With ``bf16=True`` every linear layer (the four FCs and the
-  head) rounds its inputs to bfloat16 the way the library's bf16 models feed their tensor cores:
+* Precision: float64 throughout.  With ``bf16=True`` every linear layer (the four FCs, the
+  LM head, the pooler and the classifier) rounds its inputs to bfloat16 the way the library's bf16 models feed their tensor cores:
   the forward product takes round(x) and round(W); the input gradient takes round(g) and
   round(W); the weight gradient takes round(g) and round(x).  Bias gradients, norms,
   activations, the loss and the optimiser stay unrounded.  (The paper fixes no training
@@ -104,6 +112,30 @@ def hsm_loss(p: Dict[str, torch.Tensor], W, cfg, s_i, s_prev, inertia, targets, 
     return F.cross_entropy(logits, torch.as_tensor(np.asarray(targets), dtype=torch.long))
 
 
+def cls_head_logits(W: Dict[str, object], cfg, x: torch.Tensor, bf16: bool = False) -> torch.Tensor:
+    """The frozen pooler (dense + tanh) and classifier of an encoder, applied to final states."""
+    pooled = torch.tanh(linear(x, _t(W["pool.w"]), _t(W["pool.b"]), bf16))
+    return linear(pooled, _t(W["cls.w"]), _t(W["cls.b"]), bf16)
+
+
+def cosine_rows(a: torch.Tensor, b: torch.Tensor) -> torch.Tensor:
+    """cos of each row pair, a.b / (|a| |b|), and 0 where |a| |b| = 0."""
+    den = torch.sqrt(torch.clamp_min((a * a).sum(-1) * (b * b).sum(-1), 1e-300))
+    return (a * b).sum(-1) / den
+
+
+def hsm_cls_loss(p: Dict[str, torch.Tensor], W, cfg, s_i, s_prev, inertia, s_final, labels, cls_weight: float = 1.0,
+                 bf16: bool = False) -> torch.Tensor:
+    """Similarity loss against the original final states plus the weighted task loss of the
+    first len(labels) rows (Sec. 4.3)."""
+    st = hsm_forward(p, cfg, s_i, s_prev, inertia, bf16)
+    loss = torch.mean(1.0 - cosine_rows(st, _t(s_final)))
+    lab = torch.as_tensor(np.asarray(labels), dtype=torch.long).reshape(-1)
+    if lab.numel():
+        loss = loss + cls_weight * F.cross_entropy(cls_head_logits(W, cfg, st[:lab.numel()], bf16), lab)
+    return loss
+
+
 def adamw_update(theta: np.ndarray, g: np.ndarray, m: np.ndarray, v: np.ndarray, t: int, lr: float, b1: float,
                  b2: float, eps: float, wd: float) -> Tuple[np.ndarray, np.ndarray, np.ndarray]:
     """One AdamW step (decoupled weight decay, bias-corrected moments) of one parameter."""
@@ -122,12 +154,27 @@ def hsm_train_step(W: Dict[str, object], cfg, s_i, s_prev, inertia, targets, lr:
 
     params / state: the HSM parameters and (m, v) moments of the previous step (default:
     the model's HSM weights, zero moments); t: this step's number (1 for the first)."""
+    return _step(lambda p: hsm_loss(p, W, cfg, s_i, s_prev, inertia, targets, bf16), W, lr, b1, b2, eps, wd, t,
+                 params, state)
+
+
+def hsm_cls_train_step(W: Dict[str, object], cfg, s_i, s_prev, inertia, s_final, labels, cls_weight: float, lr: float,
+                       b1: float, b2: float, eps: float, wd: float, t: int,
+                       params: Optional[Dict[str, np.ndarray]] = None,
+                       state: Optional[Dict[str, Tuple[np.ndarray, np.ndarray]]] = None, bf16: bool = False):
+    """The encoder (classification) training step of Sec. 4.3: as hsm_train_step with
+    hsm_cls_loss; labels belong to the first len(labels) examples."""
+    return _step(lambda p: hsm_cls_loss(p, W, cfg, s_i, s_prev, inertia, s_final, labels, cls_weight, bf16), W, lr, b1,
+                 b2, eps, wd, t, params, state)
+
+
+def _step(loss_fn, W, lr, b1, b2, eps, wd, t, params, state):
     if params is None:
         params = {k: np.asarray(_t(W[k])) for k in HSM_PARAMS}
     if state is None:
         state = {k: (np.zeros_like(params[k]), np.zeros_like(params[k])) for k in HSM_PARAMS}
     p = {k: torch.tensor(params[k], dtype=torch.float64, requires_grad=True) for k in HSM_PARAMS}
-    loss = hsm_loss(p, W, cfg, s_i, s_prev, inertia, targets, bf16)
+    loss = loss_fn(p)
     loss.backward()
     grads = {k: p[k].grad.numpy().copy() for k in HSM_PARAMS}
     new_params, new_state = {}, {}

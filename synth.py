@@ -360,3 +360,17 @@ def hsm_train_batch(cfg: ModelConfig, n: int, seed: int = 0, std: float = 1.0):
     inertia = (k - 1)[:, None] * u + normal(seed, "hsm-train-inertia", (n, D), std=0.1)
     target = randint(seed, "hsm-train-target", n, 0, cfg.vocab - 1)
     return s_i.contiguous(), s_prev.contiguous(), inertia.contiguous(), target
+
+
+def hsm_cls_batch(cfg: ModelConfig, n: int, n_cls: int, seed: int = 0, std: float = 1.0):
+    """n synthetic encoder training examples of the Hidden State Mapper for classification:
+    (s_i, s_{i-1}, I, s_N, labels).
+
+    Recipe: s_i, s_{i-1} and I as in hsm_train_batch; the original final state s_N =
+    s_i + N(0, (0.5 std)^2) (the remaining layers' residual updates); the first n_cls rows are
+    the labelled [CLS] rows, labels uniform on [0, n_classes).  Returned as float32 [n, D]
+    tensors and int32 [n_cls]."""
+    s_i, s_prev, inertia, _ = hsm_train_batch(cfg, n, seed=seed, std=std)
+    s_final = s_i + normal(seed, "hsm-cls-final", (n, cfg.d_model), std=0.5 * std)
+    labels = randint(seed, "hsm-cls-label", n_cls, 0, max(0, cfg.n_classes - 1))
+    return s_i, s_prev, inertia, s_final.contiguous(), labels

@@ -143,3 +143,140 @@ def test_steps_reduce_the_loss_on_a_fixed_batch():
                                                    params=params, state=state)
         losses.append(loss)
     assert losses[-1] < losses[0] - 1e-3, losses
+
+
+# ---------------------------------------------------------------------------
+# encoders: similarity loss + task loss (Sec. 4.3)
+# ---------------------------------------------------------------------------
+
+def tiny_bert(dtype="f32", **kw):
+    base = dict(max_pos=32, n_classes=3, norm_eps=1e-12)
+    base.update(kw)
+    return tiny(synth.BERT, dtype, **base)
+
+
+def setup_cls(cfg, n=6, n_cls=3, seed=0, std=0.2):
+    W = synth.make_weights(cfg, seed=seed, std=std, gain_std=0.1 if cfg.dtype == "f32" else None)
+    s_i, s_prev, inertia, s_fin, lab = synth.hsm_cls_batch(cfg, n, n_cls, seed=seed + 1)
+    return W, s_i.double(), s_prev.double(), inertia.double(), s_fin.double(), lab.long()
+
+
+@pytest.mark.parametrize("dtype", ["f32", "bf16"])
+def test_cls_head_matches_inference_oracle(dtype):
+    """The pooler + classifier written with torch ops against the inference oracle's numpy
+    restatement of the encoder's classification head."""
+    cfg = tiny_bert(dtype)
+    W, s_i, s_prev, inertia, _, _ = setup_cls(cfg)
+    om = O.OracleModel(cfg, W)
+    st = om.hsm(s_i.numpy(), s_prev.numpy(), inertia.numpy())
+    with torch.no_grad():
+        got = HT.cls_head_logits(W, cfg, torch.from_numpy(st), bf16=dtype == "bf16").numpy()
+    np.testing.assert_allclose(got, om.cls_logits(st), rtol=1e-10, atol=1e-10)
+
+
+def test_similarity_loss_is_mean_cosine_distance():
+    """With no labelled rows the loss is the mean cosine distance (scipy) between the
+    inference oracle's mapped states and the final states."""
+    from scipy.spatial.distance import cosine
+    cfg = tiny_bert()
+    W, s_i, s_prev, inertia, s_fin, _ = setup_cls(cfg, n=7)
+    om = O.OracleModel(cfg, W)
+    st = om.hsm(s_i.numpy(), s_prev.numpy(), inertia.numpy())
+    want = np.mean([cosine(st[i], s_fin[i].numpy()) for i in range(7)])
+    with torch.no_grad():
+        got = float(HT.hsm_cls_loss(params_of(W), W, cfg, s_i, s_prev, inertia, s_fin, []))
+    assert abs(got - want) < 1e-12
+
+
+@pytest.mark.parametrize("sign", [1.0, -1.0])
+def test_aligned_targets_are_stationary(sign):
+    """Targets along (+) or against (-) the mapped states: loss 0 or 2, and the gradient of
+    1 - cos vanishes at both extremes."""
+    cfg = tiny_bert()
+    W, s_i, s_prev, inertia, _, _ = setup_cls(cfg, n=5)
+    om = O.OracleModel(cfg, W)
+    st = om.hsm(s_i.numpy(), s_prev.numpy(), inertia.numpy())
+    scale = sign * (0.5 + np.arange(5))[:, None]
+    loss, grads, _, _ = HT.hsm_cls_train_step(W, cfg, s_i, s_prev, inertia, torch.from_numpy(st * scale), [], 1.0,
+                                              1e-3, 0.9, 0.999, 1e-8, 0.0, 1)
+    assert abs(loss - (1.0 - sign)) < 1e-12
+    for k in HT.HSM_PARAMS:
+        assert np.abs(grads[k]).max() < 1e-9, k
+
+
+def test_zero_target_row_adds_one_and_no_gradient():
+    """A zero final state has no direction: its cosine is taken as 0 (term 1), with no gradient."""
+    cfg = tiny_bert()
+    W, s_i, s_prev, inertia, s_fin, _ = setup_cls(cfg, n=4)
+    z = s_fin.clone()
+    z[2] = 0.0
+    l_all, g_all, _, _ = HT.hsm_cls_train_step(W, cfg, s_i, s_prev, inertia, z, [], 1.0, 1e-3, 0.9, 0.999, 1e-8, 0.0, 1)
+    keep = [0, 1, 3]
+    l3, g3, _, _ = HT.hsm_cls_train_step(W, cfg, s_i[keep], s_prev[keep], inertia[keep], z[keep], [], 1.0, 1e-3, 0.9,
+                                         0.999, 1e-8, 0.0, 1)
+    assert abs(l_all - (3 * l3 + 1.0) / 4) < 1e-12
+    for k in HT.HSM_PARAMS:
+        np.testing.assert_allclose(g_all[k], 0.75 * g3[k], rtol=1e-9, atol=1e-15)
+
+
+def test_two_class_task_loss_is_binary_cross_entropy():
+    """Two classes: the task term is torch's binary cross-entropy with logits on z1 - z0 of the
+    inference oracle's classifier logits, times cls_weight."""
+    cfg = tiny_bert(n_classes=2)
+    W, s_i, s_prev, inertia, s_fin, lab = setup_cls(cfg, n=6, n_cls=4)
+    om = O.OracleModel(cfg, W)
+    st = om.hsm(s_i.numpy(), s_prev.numpy(), inertia.numpy())
+    z = torch.from_numpy(om.cls_logits(st[:4]))
+    bce = F_bce(z[:, 1] - z[:, 0], lab.double())
+    p = params_of(W)
+    with torch.no_grad():
+        l0 = float(HT.hsm_cls_loss(p, W, cfg, s_i, s_prev, inertia, s_fin, lab, cls_weight=0.0))
+        l1 = float(HT.hsm_cls_loss(p, W, cfg, s_i, s_prev, inertia, s_fin, lab, cls_weight=0.6))
+    assert abs((l1 - l0) - 0.6 * bce) < 1e-12
+
+
+def F_bce(x, y):
+    return float(torch.nn.functional.binary_cross_entropy_with_logits(x, y))
+
+
+@pytest.mark.parametrize("n_cls", [0, 3, 5])
+def test_cls_gradients_match_central_differences(n_cls):
+    """Every HSM parameter's gradient of similarity + weighted task loss against central
+    differences (no labelled rows, some, all)."""
+    cfg = tiny_bert(hsm_eps=1e-6)
+    W, s_i, s_prev, inertia, s_fin, lab = setup_cls(cfg, n=5, n_cls=n_cls)
+    p0 = {k: v.numpy() for k, v in params_of(W).items()}
+    loss, grads, _, _ = HT.hsm_cls_train_step(W, cfg, s_i, s_prev, inertia, s_fin, lab, 0.7, 1e-3, 0.9, 0.999, 1e-8,
+                                              0.0, 1, params=p0)
+    rng = np.random.default_rng(11)
+
+    def L(p):
+        with torch.no_grad():
+            return float(HT.hsm_cls_loss({k: torch.from_numpy(v) for k, v in p.items()}, W, cfg, s_i, s_prev, inertia,
+                                         s_fin, lab, 0.7))
+
+    assert abs(L(p0) - loss) < 1e-13
+    h = 1e-6
+    for k in HT.HSM_PARAMS:
+        flat = p0[k].reshape(-1)
+        for i in rng.choice(flat.size, size=min(5, flat.size), replace=False):
+            pp = {kk: vv.copy() for kk, vv in p0.items()}
+            pm = {kk: vv.copy() for kk, vv in p0.items()}
+            pp[k].reshape(-1)[i] += h
+            pm[k].reshape(-1)[i] -= h
+            fd = (L(pp) - L(pm)) / (2 * h)
+            g = grads[k].reshape(-1)[i]
+            assert abs(fd - g) <= 1e-6 * max(1.0, abs(g)) + 1e-8, (k, int(i), fd, g)
+        assert np.abs(grads[k]).max() > 0, k
+
+
+def test_cls_bf16_mode_stays_within_rounding_of_exact():
+    cfg = tiny_bert("bf16", d_model=64, head_dim=32, hsm_m1=96, hsm_m2=160)
+    W, s_i, s_prev, inertia, s_fin, lab = setup_cls(cfg, n=12, n_cls=4, std=0.05)
+    l64, g64, _, _ = HT.hsm_cls_train_step(W, cfg, s_i, s_prev, inertia, s_fin, lab, 1.0, 1e-3, 0.9, 0.999, 1e-8, 0.0, 1)
+    l16, g16, _, _ = HT.hsm_cls_train_step(W, cfg, s_i, s_prev, inertia, s_fin, lab, 1.0, 1e-3, 0.9, 0.999, 1e-8, 0.0, 1,
+                                           bf16=True)
+    assert abs(l16 - l64) <= 1e-2 * abs(l64)
+    for k in HT.HSM_PARAMS:
+        e = np.linalg.norm(g16[k] - g64[k]) / np.linalg.norm(g64[k])
+        assert e < 3e-2, (k, e)
