@@ -325,12 +325,15 @@ def run_encoder(adept, device, B=64, P=128):
     return {"workload": f"BERT-base shape, bf16, random-init; {B} x {P}-token classification batch", **out}
 
 
-def hsm_train_flops(cfg, n):
+def hsm_train_flops(cfg, n, n_cls=0):
     """GEMM FLOPs of one HSM training step on n examples: the four FC products forward, their
-    input and weight gradients (3 x 2 x FC weights per example), the head forward and its input
-    gradient (2 x 2 D V per example)."""
+    input and weight gradients (3 x 2 x FC weights per example), then for decoders the head
+    forward and its input gradient (2 x 2 D V per example), for encoders the pooler forward
+    and its input gradient on the n_cls labelled rows (2 x 2 D^2 per row)."""
     D, m1, m2 = cfg.d_model, cfg.hsm_m1, cfg.hsm_m2
     fc = D * m1 + m1 * m2 + m2 * m1 + m1 * D
+    if cfg.family == synth.BERT:
+        return n * 6.0 * fc + n_cls * 4.0 * D * D
     return n * (6.0 * fc + 4.0 * D * cfg.vocab)
 
 
@@ -339,9 +342,17 @@ def run_hsm_train(adept, device, peaks, n=8192, reps=5, shape="gpt2"):
     fp32 master weights and AdamW state.  shape "gpt2": GPT-2-small (D 768, HSM widths 3072 /
     6144, vocabulary 50257; 8192 examples = 128 sequences x 64 tokens); "llama7b": Llama-2-7B
     (D 4096, HSM widths 8192 / 32768, vocabulary 32000; 8192 examples = 8 sequences x 1024
-    tokens).  Only the frozen head and the HSM take part, so the models carry 2 layers.  Step
-    time with CUDA events; the GEMMs' TFLOP/s from per-GEMM events in a separate profiled step."""
-    if shape == "llama7b":
+    tokens); "bert": BERT-base encoder (D 768, HSM widths 3072 / 6144, two classes; 8192
+    examples = 64 sequences x 128 tokens, the 64 [CLS] rows labelled) with the similarity +
+    classification loss of Sec. 4.3.  Only the frozen head and the HSM take part, so the models
+    carry 2 layers.  Step time with CUDA events; the GEMMs' TFLOP/s from per-GEMM events in a
+    separate profiled step."""
+    n_cls = 0
+    if shape == "bert":
+        cfg = synth.bert_base_config(n_layers=2, max_batch=1, max_seq=16)
+        desc = "BERT-base shape HSM (768 -> 3072 -> 6144 -> 3072 -> 768) + frozen pooler / 2-class classifier"
+        n_cls = n // 128
+    elif shape == "llama7b":
         cfg = synth.llama7b_config(n_layers=2, max_batch=1, max_seq=16)
         desc = "Llama-2-7B shape HSM (4096 -> 8192 -> 32768 -> 8192 -> 4096) + frozen 32000-token head"
     else:
@@ -350,12 +361,17 @@ def run_hsm_train(adept, device, peaks, n=8192, reps=5, shape="gpt2"):
     W = synth.make_weights(cfg, seed=0, device=device)
     m = adept.Model(cfg, W)
     del W
-    s_i, s_prev, inertia, tgt = [x.to(device) for x in synth.hsm_train_batch(cfg, n, seed=1)]
     adept.adept_hsm_train_init(m.h, n)
     loss = torch.zeros(1, device=device)
     st = torch.cuda.current_stream()
-    step = lambda: adept.adept_hsm_train_step(m.h, n, s_i, s_prev, inertia, tgt, 1e-4, 0.9, 0.999, 1e-8, 0.0,  # noqa
-                                              loss_out=loss)
+    if shape == "bert":
+        s_i, s_prev, inertia, s_fin, lab = [x.to(device) for x in synth.hsm_cls_batch(cfg, n, n_cls, seed=1)]
+        step = lambda: adept.adept_hsm_train_step_cls(m.h, n, s_i, s_prev, inertia, s_fin, lab, 1e-4,  # noqa
+                                                      loss_out=loss)
+    else:
+        s_i, s_prev, inertia, tgt = [x.to(device) for x in synth.hsm_train_batch(cfg, n, seed=1)]
+        step = lambda: adept.adept_hsm_train_step(m.h, n, s_i, s_prev, inertia, tgt, 1e-4, 0.9, 0.999, 1e-8,  # noqa
+                                                  0.0, loss_out=loss)
     step()
     adept.adept_check_device_status(m.h)
     first_loss = float(loss.item())
@@ -371,7 +387,7 @@ def run_hsm_train(adept, device, peaks, n=8192, reps=5, shape="gpt2"):
         ts.append(e0.elapsed_time(e1))
     launches = adept.adept_launch_count(m.h) // reps
     t = float(np.median(ts)) / 1e3
-    fl = hsm_train_flops(cfg, n)
+    fl = hsm_train_flops(cfg, n, n_cls)
     adept.adept_set_option(m.h, adept.OPT_PROFILE, 1)
     step()
     ng, gms, _, _ = adept.adept_profile_read(m.h, adept.PROF_GEMM_TRAIN)
@@ -630,6 +646,7 @@ def ours(args, rank, world, device):
         line["encoder"] = run_encoder(adept, device)
         line["hsm_train"] = run_hsm_train(adept, device, peaks)
         line["hsm_train_llama7b"] = run_hsm_train(adept, device, peaks, shape="llama7b", reps=3)
+        line["hsm_train_bert"] = run_hsm_train(adept, device, peaks, shape="bert")
     if rank == 0 and not args.no_cpu_baseline:
         line["cpu_baseline"] = cpu_baseline(args.cpu_tokens)
     return line

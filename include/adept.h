@@ -285,8 +285,8 @@ typedef struct {
 /* Starts HSM training: master parameters from the model's current HSM weights, zero moments,
  * step count 0, and device workspaces for up to max_rows examples per step (a second call
  * frees the previous ones and starts over).  Synchronous on `stream`.
- * Errors: INVALID_ARG (max_rows < 1, an encoder model, a bf16 model whose D, m1 or m2 is not
- * a multiple of 8), OOM. */
+ * Errors: INVALID_ARG (max_rows < 1, an encoder whose n_classes is outside [1, 64], a bf16
+ * model whose D, m1 or m2 is not a multiple of 8), OOM. */
 ADEPT_API adept_status adept_hsm_train_init(adept_model* m, int max_rows, void* stream);
 
 /* One training step on n examples, enqueued on `stream`: forward (Table S1) with the
@@ -298,11 +298,32 @@ ADEPT_API adept_status adept_hsm_train_init(adept_model* m, int max_rows, void* 
  *                               nothing to the loss or the gradients)
  *   hp                          host pointer to the hyperparameters
  *   d_loss_out                  device float: the mean loss before the update (NULL: not written)
- * Errors: INVALID_ARG (no adept_hsm_train_init, n outside [1, max_rows], NULL pointers,
- * lr < 0, beta outside [0, 1), eps <= 0, weight_decay < 0). */
+ * Errors: INVALID_ARG (no adept_hsm_train_init, an encoder model, n outside [1, max_rows],
+ * NULL pointers, lr < 0, beta outside [0, 1), eps <= 0, weight_decay < 0). */
 ADEPT_API adept_status adept_hsm_train_step(adept_model* m, int n, const float* d_s_i, const float* d_s_prev,
                                   const float* d_inertia, const int32_t* d_target, const adept_adamw* hp,
                                   float* d_loss_out, void* stream);
+
+/* One training step of an encoder's HSM for classification (Sec. 4.3), enqueued on `stream`:
+ * with no next token to predict, the loss is the similarity loss against the original final
+ * hidden states, mean over the n examples of 1 - cos(s~, s_N) (cos = 0 where a norm is 0),
+ * plus cls_weight times the frozen pooler + classifier's softmax cross-entropy (for two
+ * classes, the binary cross-entropy) on the first n_cls examples, the labelled [CLS] rows,
+ * averaged over them.  Then backward, AdamW and the weight write-back as adept_hsm_train_step.
+ *   d_s_i, d_s_prev, d_inertia  [n, D] fp32 device rows as in adept_hsm_train_step
+ *   d_s_final                   [n, D] fp32 device rows: the original final hidden states
+ *   n_cls, d_label              labelled rows 0..n_cls-1 (0 <= n_cls <= n) and their int32 class
+ *                               ids in [0, n_classes) on the device (NULL allowed when n_cls = 0;
+ *                               a bad id flags DEVICE_INPUT at adept_check_device_status and its
+ *                               row adds no task loss or gradient)
+ *   cls_weight                  weight of the task loss (>= 0; the paper adds the two: 1)
+ *   hp, d_loss_out              as in adept_hsm_train_step
+ * Errors: INVALID_ARG (no adept_hsm_train_init, a decoder model, n or n_cls out of range, NULL
+ * pointers, cls_weight < 0 or not finite, AdamW hyperparameters as above). */
+ADEPT_API adept_status adept_hsm_train_step_cls(adept_model* m, int n, const float* d_s_i, const float* d_s_prev,
+                                      const float* d_inertia, const float* d_s_final, int n_cls,
+                                      const int32_t* d_label, float cls_weight, const adept_adamw* hp,
+                                      float* d_loss_out, void* stream);
 
 /* Copies one parameter's fp32 training values to device memory d_out (count = its element
  * count, adept_hsm_param_numel): what = ADEPT_HSM_PARAMS (master values), ADEPT_HSM_GRADS

@@ -35,7 +35,7 @@ ABI_SYMBOLS = [
     "adept_read_final_states", "adept_check_device_status", "adept_set_option", "adept_profile_read",
     "adept_launch_count", "adept_skip_kv_fill_noalloc", "adept_fused_decode_batch", "adept_fused_decode_reason",
     "adept_calibrate_threshold", "adept_hsm_train_init", "adept_hsm_train_step", "adept_hsm_train_read",
-    "adept_hsm_param_numel",
+    "adept_hsm_param_numel", "adept_hsm_train_step_cls",
 ]
 
 
@@ -117,6 +117,9 @@ def load_library(path: str = LIB_PATH):
     lib.adept_hsm_train_init.restype = c_int
     lib.adept_hsm_train_step.argtypes = [vp, c_int, fp, fp, fp, i32p, ctypes.POINTER(AdeptAdamW), fp, st]
     lib.adept_hsm_train_step.restype = c_int
+    lib.adept_hsm_train_step_cls.argtypes = [vp, c_int, fp, fp, fp, fp, c_int, i32p, ctypes.c_float,
+                                             ctypes.POINTER(AdeptAdamW), fp, st]
+    lib.adept_hsm_train_step_cls.restype = c_int
     lib.adept_hsm_train_read.argtypes = [vp, c_int, c_int, fp, ctypes.c_int64, st]
     lib.adept_hsm_train_read.restype = c_int
     lib.adept_hsm_param_numel.argtypes = [vp, c_int]
@@ -257,6 +260,21 @@ def adept_hsm_train_step(m, n: int, s_i: torch.Tensor, s_prev: torch.Tensor, ine
     hp = AdeptAdamW(lr, beta1, beta2, eps, weight_decay)
     _check(lib, m, lib.adept_hsm_train_step(m, int(n), _ptr(s_i), _ptr(s_prev), _ptr(inertia), _ptr(target),
                                              ctypes.byref(hp), _ptr(loss_out), _stream(stream)))
+
+
+def adept_hsm_train_step_cls(m, n: int, s_i: torch.Tensor, s_prev: torch.Tensor, inertia: torch.Tensor,
+                             s_final: torch.Tensor, labels: Optional[torch.Tensor], lr: float, cls_weight: float = 1.0,
+                             beta1: float = 0.9, beta2: float = 0.999, eps: float = 1e-8, weight_decay: float = 0.0,
+                             loss_out: Optional[torch.Tensor] = None, stream=None):
+    """One encoder HSM training step (Sec. 4.3): similarity loss against the original final
+    states plus cls_weight times the classifier's cross-entropy on the first len(labels)
+    rows, backward, AdamW."""
+    lib = load_library()
+    hp = AdeptAdamW(lr, beta1, beta2, eps, weight_decay)
+    n_cls = 0 if labels is None else labels.numel()
+    _check(lib, m, lib.adept_hsm_train_step_cls(m, int(n), _ptr(s_i), _ptr(s_prev), _ptr(inertia), _ptr(s_final),
+                                                 int(n_cls), _ptr(labels), float(cls_weight), ctypes.byref(hp),
+                                                 _ptr(loss_out), _stream(stream)))
 
 
 def adept_hsm_train_read(m, what: int, param: int, out: torch.Tensor, stream=None):

@@ -15,7 +15,8 @@ enum : unsigned {
   ERRW_POS = 4u,       // position outside the sequence's reserved blocks / max_pos
   ERRW_EXIT_LAYER = 8u,// exit layer outside [1, N] (skipped-layer fill input)
   ERRW_TIMEOUT = 16u,  // a bounded device-side wait gave up
-  ERRW_CONFIG = 32u    // a kernel was launched with a shape it does not support
+  ERRW_CONFIG = 32u,   // a kernel was launched with a shape it does not support
+  ERRW_LABEL = 64u     // class label outside [0, n_classes)
 };
 
 // Programmatic dependent launch.  Every kernel of the library begins with PDL_ENTRY: it

@@ -1,12 +1,15 @@
 // Kernels of the HSM training step (Sec. 4.2; Sec. 5.1 "Training"; App. D): the Hidden State
 // Mapper is trained with the base model frozen, by cross-entropy of its mapped state, read
-// through the frozen final norm and LM head, against the next token, and AdamW.
+// through the frozen final norm and LM head, against the next token, and AdamW.  Encoders
+// (Sec. 4.3) train it by the cosine similarity of the mapped state to the original final
+// state plus the frozen pooler + classifier's cross-entropy on the labelled [CLS] rows.
 //
 // The products (the four FC layers of Table S1, their input and weight gradients, the head
 // and its input gradient) run on the library's GEMMs; these kernels are the elementwise and
-// row-wise steps between them (GELU and its derivative, the softmax cross-entropy, the RMSNorm
-// / LayerNorm backward, the convolution backward), the deterministic column sums that give
-// bias, gain and convolution gradients, operand transposes, and the AdamW update.
+// row-wise steps between them (GELU and its derivative, the softmax cross-entropy, the
+// similarity and classifier rows, the RMSNorm / LayerNorm backward, the convolution
+// backward), the deterministic column sums that give bias, gain and convolution gradients,
+// operand transposes, and the AdamW update.
 #define ADEPT_TU_ID 9
 #include "common.cuh"
 #include "hsm_train.h"
@@ -106,14 +109,97 @@ __global__ void __launch_bounds__(512, 2) ht_ce_kernel(const float* __restrict__
   }
 }
 
-// loss = scale * sum_r lossr[r] in a fixed order (one CTA).
-__global__ void ht_loss_kernel(const float* lossr, int n, float scale, float* loss) {
+// loss = scale * sum_r lossr[r] (+ scale_b * sum_r lossb[r]) in a fixed order (one CTA).
+__global__ void ht_loss_kernel(const float* lossr, int n, float scale, const float* lossb, int nb, float scale_b,
+                               float* loss) {
   PDL_ENTRY();
   __shared__ float red[32];
   float s = 0.f;
   for (int i = threadIdx.x; i < n; i += blockDim.x) s += lossr[i];
   s = block_sum(s, red);
-  if (threadIdx.x == 0) *loss = s * scale;
+  float sb = 0.f;
+  for (int i = threadIdx.x; i < nb; i += blockDim.x) sb += lossb[i];
+  sb = block_sum(sb, red);
+  if (threadIdx.x == 0) *loss = s * scale + (nb ? sb * scale_b : 0.f);
+}
+
+// Similarity loss rows of the encoder step (Sec. 4.3; one CTA per row): with s = s~_r and
+// t = s_N,r, lossr[r] = 1 - cos, cos = s.t / (|s| |t|), and the row's gradient
+//   dxh[r] = -inv_n (t / (|s| |t|) - cos s / |s|^2)
+// (cos = 0 and no gradient where |s| |t| = 0).
+__global__ void ht_cos_kernel(const float* __restrict__ st, const float* __restrict__ tg, int D, float inv_n,
+                              float* lossr, float* dxh) {
+  PDL_ENTRY();
+  __shared__ float red[32];
+  const size_t o = (size_t)blockIdx.x * D;
+  float a = 0.f, ss = 0.f, tt = 0.f;
+  for (int d = threadIdx.x; d < D; d += blockDim.x) {
+    const float s = st[o + d], t = tg[o + d];
+    a += s * t;
+    ss += s * s;
+    tt += t * t;
+  }
+  a = block_sum(a, red);
+  ss = block_sum(ss, red);
+  tt = block_sum(tt, red);
+  float cs = 0.f, ct = 0.f, cosv = 0.f;
+  if (ss > 0.f && tt > 0.f) {
+    const float den = sqrtf(ss) * sqrtf(tt);
+    cosv = a / den;
+    ct = -inv_n / den;
+    cs = inv_n * cosv / ss;
+  }
+  for (int d = threadIdx.x; d < D; d += blockDim.x) dxh[o + d] = ct * tg[o + d] + cs * st[o + d];
+  if (threadIdx.x == 0) lossr[blockIdx.x] = 1.f - cosv;
+}
+
+template <typename T> __device__ __forceinline__ float round_to(float x) { return to_f<T>(from_f<T>(x)); }
+
+// Task loss of the encoder step (Sec. 4.3) on the labelled rows (one CTA per row): pooled =
+// tanh(zp) (zp: the pooler's pre-activation, bias included), logits z_c = round(pooled) . Wc[c]
+// + bc[c], lossc[r] = logsumexp(z) - z[label]; with dz_c = scale (softmax(z)_c - [c = label])
+// rounded like a GEMM input, dpt[r][d] = (sum_c dz_c Wc[c][d]) (1 - pooled[d]^2), the gradient
+// into the pooler's pre-activation (T, the next product's input).  A label outside [0, C)
+// flags ERRW_LABEL and leaves a zero loss and gradient for the row.
+template <typename T>
+__global__ void ht_cls_kernel(const float* __restrict__ zp, int D, const T* __restrict__ wc,
+                              const float* __restrict__ bc, int C, const int* __restrict__ label, float scale,
+                              float* lossc, T* dpt, unsigned* err) {
+  PDL_ENTRY();
+  __shared__ float red[32];
+  __shared__ float dz[HT_MAX_CLASSES];
+  const size_t o = (size_t)blockIdx.x * D;
+  const int y = label[blockIdx.x];
+  if (y < 0 || y >= C) {
+    if (threadIdx.x == 0) {
+      atomicOr(err, ERRW_LABEL);
+      lossc[blockIdx.x] = 0.f;
+    }
+    for (int d = threadIdx.x; d < D; d += blockDim.x) dpt[o + d] = from_f<T>(0.f);
+    return;
+  }
+  for (int c = 0; c < C; ++c) {
+    float s = 0.f;
+    for (int d = threadIdx.x; d < D; d += blockDim.x) s += round_to<T>(tanhf(zp[o + d])) * to_f(wc[(size_t)c * D + d]);
+    s = block_sum(s, red);
+    if (threadIdx.x == 0) dz[c] = s + bc[c];
+  }
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    float mx = -INFINITY;
+    for (int c = 0; c < C; ++c) mx = fmaxf(mx, dz[c]);
+    float S = 0.f;
+    for (int c = 0; c < C; ++c) S += expf(dz[c] - mx);
+    lossc[blockIdx.x] = logf(S) + mx - dz[y];
+    for (int c = 0; c < C; ++c) dz[c] = round_to<T>(scale * (expf(dz[c] - mx) / S - (c == y ? 1.f : 0.f)));
+  }
+  __syncthreads();
+  for (int d = threadIdx.x; d < D; d += blockDim.x) {
+    float g = 0.f;
+    for (int c = 0; c < C; ++c) g += dz[c] * to_f(wc[(size_t)c * D + d]);
+    const float p = tanhf(zp[o + d]);
+    dpt[o + d] = from_f<T>(g * (1.f - p * p));
+  }
 }
 
 // ---------------------------------------------------------------------------
@@ -122,7 +208,8 @@ __global__ void ht_loss_kernel(const float* lossr, int n, float scale, float* lo
 
 // Through the frozen head's standardisation and the HSM's last block (one CTA per row).
 // st = s~ = RMSNorm_g2(h5) + c0; xh = standardise(st) (LayerNorm without affine for mode LN,
-// RMS scaling for mode RMS; the head's gain and bias are folded into its weights).
+// RMS scaling for mode RMS; the head's gain and bias are folded into its weights; mode COPY,
+// the encoder's post-LN final state, reads s~ itself: dst = dxh).
 //   dst = rstd (dxh - mean(dxh) - xh mean(dxh xh))          (LN; RMS drops mean(dxh))
 //   dc0 = dst;  dr = dst g2;  dh5 = r2 (dr - rh mean(dr rh)),  rh = h5 r2
 // Writes dc0 (fp32), dh5 (fp32 and T) and r2 (for the g2 column sum).
@@ -142,31 +229,38 @@ __global__ void ht_out_bwd_kernel(const float* __restrict__ dxh, int nsplit, siz
     for (int s = 1; s < nsplit; ++s) v += dxh[s * split_stride + o + d];
     return v;
   };
-  float mu = 0.f;
-  if (mode == NORM_LN) {
-    float s = 0.f;
-    for (int d = threadIdx.x; d < D; d += blockDim.x) s += f[d];
-    mu = block_sum(s, red) / D;
-  }
-  float s2 = 0.f;
-  for (int d = threadIdx.x; d < D; d += blockDim.x) {
-    const float c = f[d] - mu;
-    s2 += c * c;
-  }
-  const float rs = rsqrtf(block_sum(s2, red) / D + norm_eps);
-  float sa = 0.f, sb = 0.f;
-  for (int d = threadIdx.x; d < D; d += blockDim.x) {
-    const float xd = X(d);
-    sa += xd;
-    sb += xd * (f[d] - mu) * rs;
-  }
-  const float ma = mode == NORM_LN ? block_sum(sa, red) / D : 0.f;
-  const float mb = block_sum(sb, red) / D;
   float q2 = 0.f;
-  for (int d = threadIdx.x; d < D; d += blockDim.x) {
-    const float v = rs * (X(d) - ma - (f[d] - mu) * rs * mb);
-    dc0[o + d] = v;
-    q2 += h[d] * h[d];
+  if (mode == NORM_COPY) {
+    for (int d = threadIdx.x; d < D; d += blockDim.x) {
+      dc0[o + d] = X(d);
+      q2 += h[d] * h[d];
+    }
+  } else {
+    float mu = 0.f;
+    if (mode == NORM_LN) {
+      float s = 0.f;
+      for (int d = threadIdx.x; d < D; d += blockDim.x) s += f[d];
+      mu = block_sum(s, red) / D;
+    }
+    float s2 = 0.f;
+    for (int d = threadIdx.x; d < D; d += blockDim.x) {
+      const float c = f[d] - mu;
+      s2 += c * c;
+    }
+    const float rs = rsqrtf(block_sum(s2, red) / D + norm_eps);
+    float sa = 0.f, sb = 0.f;
+    for (int d = threadIdx.x; d < D; d += blockDim.x) {
+      const float xd = X(d);
+      sa += xd;
+      sb += xd * (f[d] - mu) * rs;
+    }
+    const float ma = mode == NORM_LN ? block_sum(sa, red) / D : 0.f;
+    const float mb = block_sum(sb, red) / D;
+    for (int d = threadIdx.x; d < D; d += blockDim.x) {
+      const float v = rs * (X(d) - ma - (f[d] - mu) * rs * mb);
+      dc0[o + d] = v;
+      q2 += h[d] * h[d];
+    }
   }
   const float r2 = rsqrtf(block_sum(q2, red) / D + eps);
   float sc = 0.f;
@@ -412,7 +506,26 @@ void ht_launch_ce(cudaStream_t st, int dt, const float* logits, int ldl, int n, 
   const float inv_n = 1.f / (float)n;
   if (dt == 1) launch_k(ht_ce_kernel<bf16>, n, 512, 0, st, logits, ldl, V, Vp, target, inv_n, lossr, (bf16*)dl, err);
   else launch_k(ht_ce_kernel<float>, n, 512, 0, st, logits, ldl, V, Vp, target, inv_n, lossr, (float*)dl, err);
-  if (loss) launch_k(ht_loss_kernel, 1, 1024, 0, st, (const float*)lossr, n, inv_n, loss);
+  if (loss) launch_k(ht_loss_kernel, 1, 1024, 0, st, (const float*)lossr, n, inv_n, (const float*)nullptr, 0, 0.f, loss);
+}
+
+void ht_launch_cos(cudaStream_t st, const float* stv, const float* tgt, int n, int D, float* lossr, float* dxh) {
+  launch_k(ht_cos_kernel, n, 256, 0, st, stv, tgt, D, 1.f / (float)n, lossr, dxh);
+}
+
+void ht_launch_cls(cudaStream_t st, int dt, const float* zp, int n_cls, int D, const void* wc, const float* bc, int C,
+                   const int* label, float scale, float* lossc, void* dpt, unsigned* err) {
+  if (dt == 1)
+    launch_k(ht_cls_kernel<bf16>, n_cls, 256, 0, st, zp, D, (const bf16*)wc, bc, C, label, scale, lossc, (bf16*)dpt,
+             err);
+  else
+    launch_k(ht_cls_kernel<float>, n_cls, 256, 0, st, zp, D, (const float*)wc, bc, C, label, scale, lossc,
+             (float*)dpt, err);
+}
+
+void ht_launch_loss(cudaStream_t st, const float* la, int na, float sa, const float* lb, int nb, float sb,
+                    float* loss) {
+  launch_k(ht_loss_kernel, 1, 1024, 0, st, la, na, sa, lb, nb, sb, loss);
 }
 
 void ht_launch_out_bwd(cudaStream_t st, int dt, const float* dxh, int nsplit, size_t split_stride, const float* stv,

@@ -52,6 +52,15 @@ struct AdamArgs {
 // (optional, device scalar) = mean of lossr.
 void ht_launch_ce(cudaStream_t st, int dt, const float* logits, int ldl, int n, int V, int Vp, const int* target,
                   float* lossr, void* dl, float* loss, unsigned* err);
+// Encoder step (Sec. 4.3): similarity rows (lossr[n] = 1 - cos, dxh [n][D] overwritten),
+// classifier rows (zp [n_cls][D] pooler pre-activations -> lossc[n_cls], dpt [n_cls][D] T;
+// C <= HT_MAX_CLASSES), and loss = sa * sum(la) + sb * sum(lb) (fixed order).
+constexpr int HT_MAX_CLASSES = 64;
+void ht_launch_cos(cudaStream_t st, const float* stv, const float* tgt, int n, int D, float* lossr, float* dxh);
+void ht_launch_cls(cudaStream_t st, int dt, const float* zp, int n_cls, int D, const void* wc, const float* bc, int C,
+                   const int* label, float scale, float* lossc, void* dpt, unsigned* err);
+void ht_launch_loss(cudaStream_t st, const float* la, int na, float sa, const float* lb, int nb, float sb,
+                    float* loss);
 // dxh: nsplit partial sums [n][D], split_stride floats apart.
 void ht_launch_out_bwd(cudaStream_t st, int dt, const float* dxh, int nsplit, size_t split_stride, const float* stv,
                        const float* h5, int n, int D, const float* g2, float eps, int mode, float norm_eps, float* dc0,

@@ -70,6 +70,10 @@ struct HsmTrain {
   void *c0t = nullptr, *c0T = nullptr, *h1t = nullptr, *h1T = nullptr, *h2t = nullptr, *h2T = nullptr,
        *h4t = nullptr, *h4T = nullptr, *xht = nullptr, *dlt = nullptr, *dh5t = nullptr, *dh5T = nullptr,
        *dh3t = nullptr, *dh3T = nullptr, *dz2t = nullptr, *dz2T = nullptr;
+  // encoders (classification): pooler weight transposed, pooler pre-activations, their
+  // gradient, the classifier rows' losses
+  void *poolT = nullptr, *dpt = nullptr;
+  float *zp = nullptr, *lossc = nullptr;
 };
 
 struct adept_model {
@@ -1107,13 +1111,20 @@ static adept_status ht_init(adept_model* m, int cap, cudaStream_t st) {
     return ADEPT_OK;
   };
   const size_t n = cap, L = t.ldTc;
+  const bool enc = c.family == ADEPT_FAMILY_BERT;
   TRY(A(&t.theta, P * 4)); TRY(A(&t.grad, P * 4)); TRY(A(&t.mom1, P * 4)); TRY(A(&t.mom2, P * 4));
   TRY(A(&t.w1T, (size_t)m1 * D * es)); TRY(A(&t.w2T, (size_t)m2 * m1 * es));
   TRY(A(&t.w3T, (size_t)m1 * m2 * es)); TRY(A(&t.w4T, (size_t)D * m1 * es));
-  TRY(A(&t.headT, (size_t)D * t.Vp * es));
+  if (enc) {
+    TRY(A(&t.poolT, (size_t)D * D * es)); TRY(A(&t.zp, n * D * 4)); TRY(A(&t.dpt, n * D * es));
+    TRY(A(&t.lossc, n * 4));
+  } else {
+    TRY(A(&t.headT, (size_t)D * t.Vp * es));
+  }
   TRY(A(&t.iota, n * 4));
   TRY(A(&t.c0f, n * D * 4)); TRY(A(&t.z1f, n * m1 * 4)); TRY(A(&t.h1f, n * m1 * 4)); TRY(A(&t.z2f, n * m2 * 4));
-  TRY(A(&t.h3f, n * m1 * 4)); TRY(A(&t.h5f, n * D * 4)); TRY(A(&t.stf, n * D * 4)); TRY(A(&t.logits, n * t.Vl * 4));
+  TRY(A(&t.h3f, n * m1 * 4)); TRY(A(&t.h5f, n * D * 4)); TRY(A(&t.stf, n * D * 4));
+  if (!enc) TRY(A(&t.logits, n * t.Vl * 4));
   TRY(A(&t.lossr, n * 4)); TRY(A(&t.dxh, (size_t)HT_DXH_SPLITS * n * D * 4)); TRY(A(&t.dc0f, n * D * 4)); TRY(A(&t.dh5f, n * D * 4));
   TRY(A(&t.dh4f, n * m1 * 4)); TRY(A(&t.dh3f, n * m1 * 4)); TRY(A(&t.dh2f, n * m2 * 4));
   TRY(A(&t.r1, n * 4)); TRY(A(&t.r2, n * 4)); TRY(A(&t.cw, n * 10 * 4));
@@ -1123,13 +1134,14 @@ static adept_status ht_init(adept_model* m, int cap, cudaStream_t st) {
   TRY(A(&t.h1t, n * m1 * es)); TRY(A(&t.h1T, (size_t)m1 * L * es));
   TRY(A(&t.h2t, n * m2 * es)); TRY(A(&t.h2T, (size_t)m2 * L * es));
   TRY(A(&t.h4t, n * m1 * es)); TRY(A(&t.h4T, (size_t)m1 * L * es));
-  TRY(A(&t.xht, n * D * es)); TRY(A(&t.dlt, n * t.Vp * es));
+  TRY(A(&t.xht, n * D * es));
+  if (!enc) TRY(A(&t.dlt, n * t.Vp * es));
   TRY(A(&t.dh5t, n * D * es)); TRY(A(&t.dh5T, (size_t)D * L * es));
   TRY(A(&t.dh3t, n * m1 * es)); TRY(A(&t.dh3T, (size_t)m1 * L * es));
   TRY(A(&t.dz2t, n * m2 * es)); TRY(A(&t.dz2T, (size_t)m2 * L * es));
   if (dt != ADEPT_DTYPE_BF16 || m->force_simt) {
     // SIMT GEMMs stage C in the model's scratch: size it for the largest training product now
-    const size_t big = std::max({n * (size_t)std::max({V, m2, m1, D}), (size_t)m1 * m2, (size_t)m1 * D});
+    const size_t big = std::max({n * (size_t)std::max({enc ? D : V, m2, m1, D}), (size_t)m1 * m2, (size_t)m1 * D});
     if (!ensure_scratch(m, big)) return ADEPT_ERR_OOM;
   }
   // master parameters = the model's HSM weights; zero gradients and moments
@@ -1152,26 +1164,26 @@ static adept_status ht_init(adept_model* m, int cap, cudaStream_t st) {
   ht_launch_transpose(st, dt, m->hsm_w2, m2, m1, t.w2T, m2);
   ht_launch_transpose(st, dt, m->hsm_w3, m1, m2, t.w3T, m1);
   ht_launch_transpose(st, dt, m->hsm_w4, D, m1, t.w4T, D);
-  ht_launch_transpose(st, dt, m->w_head, V, D, t.headT, t.Vp);
+  if (enc) ht_launch_transpose(st, dt, m->w_pool, D, D, t.poolT, D);
+  else ht_launch_transpose(st, dt, m->w_head, V, D, t.headT, t.Vp);
   std::vector<int> io(cap);
   for (int i = 0; i < cap; ++i) io[i] = i;
   CUDA_TRY(m, cudaMemcpyAsync(t.iota, io.data(), (size_t)cap * 4, cudaMemcpyHostToDevice, st));
   CUDA_TRY(m, cudaStreamSynchronize(st));
-  (void)c;
   return check_launch(m);
 }
 
-static adept_status ht_step(adept_model* m, int n, const float* s_i, const float* s_prev, const float* inertia,
-                            const int32_t* target, const adept_adamw& hp, float* loss, cudaStream_t st) {
+// Table S1 forward on n rows, keeping what the backward reads; the mapped state s~ lands in
+// stf (fp32) and, standardised for the head (decoders) or as it is (encoders), in xht (T).
+static void ht_forward(adept_model* m, cudaStream_t st, int n, const float* s_i, const float* s_prev,
+                       const float* inertia) {
   HsmTrain& t = *m->ht;
-  const int D = m->D, m1 = m->m1, m2 = m->m2, V = m->V, Vp = t.Vp, dt = m->dt;
+  const int D = m->D, m1 = m->m1, m2 = m->m2, dt = m->dt;
   const int ldT = (n + 7) / 8 * 8;
   const float eps = m->cfg.hsm_eps, neps = m->cfg.norm_eps;
   const int hmode = attn_norm_mode(m);
   const DevRange rows{nullptr, nullptr, n};
   auto P = [&](int i) { return t.theta + t.off[i]; };
-  auto G = [&](int i) { return t.grad + t.off[i]; };
-  // forward (Table S1), keeping what the backward reads
   launch_hsm_prep(st, dt, s_i, s_prev, inertia, rows, n, D, P(HT_G0), P(HT_CONV_W), eps, t.c0f, t.c0t);
   ht_gemm(m, st, {ht_prob(t.c0t, D, n, m->hsm_w1, D, n, m1, D, t.z1f, m1, P(HT_FC1_B), false)});
   ht_launch_gelu_tile(st, dt, 0, t.z1f, t.h1f, n, m1, t.h1t, t.h1T, ldT, nullptr);
@@ -1181,23 +1193,22 @@ static adept_status ht_step(adept_model* m, int n, const float* s_i, const float
   launch_hsm_mid(st, dt, t.h3f, t.h1f, rows, n, m1, P(HT_G1), eps, t.h4t);
   ht_gemm(m, st, {ht_prob(t.h4t, m1, n, m->hsm_w4, m1, n, D, m1, t.h5f, D, P(HT_FC4_B), false)});
   launch_hsm_out(st, dt, t.h5f, t.c0f, nullptr, 0, rows, n, D, P(HT_G2), eps, t.iota, t.stf, t.xht, hmode, neps);
-  // the frozen head (final-norm gain and shift folded into its weights) and the loss
-  ht_gemm(m, st, {ht_prob(t.xht, D, n, m->w_head, D, n, V, D, t.logits, t.Vl, m->b_head, false)});
-  ht_launch_ce(st, dt, t.logits, t.Vl, n, V, Vp, target, t.lossr, t.dlt, loss, m->err_word);
-  // backward
-  // dxh = dlogits W_head, K = Vp split into parts summed by the next kernel
-  {
-    const int S0 = ht_dxh_splits(n, D, Vp, t.sms);
-    const int kc = (cdiv(Vp, S0) + 63) / 64 * 64;
-    GemmProblem ps[HT_DXH_SPLITS];
-    int S = 0;
-    for (int k0 = 0; k0 < Vp; k0 += kc, ++S)
-      ps[S] = ht_prob((const char*)t.dlt + (size_t)k0 * m->esz, Vp, n, (const char*)t.headT + (size_t)k0 * m->esz, Vp,
-                      n, D, std::min(kc, Vp - k0), t.dxh + (size_t)S * n * D, D, nullptr, false);
-    ht_gemm_n(m, st, ps, S);
-    ht_launch_out_bwd(st, dt, t.dxh, S, (size_t)n * D, t.stf, t.h5f, n, D, P(HT_G2), eps, hmode, neps, t.dc0f,
-                      t.dh5f, t.dh5t, t.r2);
-  }
+}
+
+// Backward of Table S1 from dxh (nsplit partial sums [n][D] of the gradient with respect to
+// the head's input), then AdamW and the write-back of the model's HSM weights.  `launches`:
+// the caller's own non-GEMM launches, added to the count.
+static adept_status ht_backward(adept_model* m, cudaStream_t st, int n, int nsplit, const float* s_i,
+                                const float* s_prev, const float* inertia, const adept_adamw& hp, int launches) {
+  HsmTrain& t = *m->ht;
+  const int D = m->D, m1 = m->m1, m2 = m->m2, dt = m->dt;
+  const int ldT = (n + 7) / 8 * 8;
+  const float eps = m->cfg.hsm_eps, neps = m->cfg.norm_eps;
+  const int hmode = attn_norm_mode(m);
+  auto P = [&](int i) { return t.theta + t.off[i]; };
+  auto G = [&](int i) { return t.grad + t.off[i]; };
+  ht_launch_out_bwd(st, dt, t.dxh, nsplit, (size_t)n * D, t.stf, t.h5f, n, D, P(HT_G2), eps, hmode, neps, t.dc0f,
+                    t.dh5f, t.dh5t, t.r2);
   int cl = 0;
   {
     ColJobs J{};
@@ -1271,10 +1282,61 @@ static adept_status ht_step(adept_model* m, int n, const float* s_i, const float
   a.nseg = (int)(sizeof segs / sizeof segs[0]);
   for (int i = 0; i < a.nseg; ++i) a.seg[i] = segs[i];
   ht_launch_adamw(st, dt, a);
-  // launches outside ht_gemm: prep, 2 GELU, mid, out, ce (+ loss), out_bwd, mid_bwd, 2 GELU', prep_bwd,
-  // 4 transposes, the column sums and AdamW
-  m->launches += 16 + (loss ? 1 : 0) + cl;
+  // launches outside ht_gemm: prep, 2 GELU, mid, out (forward), out_bwd, mid_bwd, 2 GELU', prep_bwd,
+  // 4 transposes, the column sums and AdamW, and the caller's loss launches
+  m->launches += 15 + launches + cl;
   return check_launch(m);
+}
+
+// Decoder step (Sec. 4.2): the frozen head (final-norm gain and shift folded into its
+// weights), next-token cross-entropy, and the head's input gradient dxh = dlogits W_head with
+// K = Vp split into parts that the backward's first kernel sums.
+static adept_status ht_step(adept_model* m, int n, const float* s_i, const float* s_prev, const float* inertia,
+                            const int32_t* target, const adept_adamw& hp, float* loss, cudaStream_t st) {
+  HsmTrain& t = *m->ht;
+  const int D = m->D, V = m->V, Vp = t.Vp, dt = m->dt;
+  ht_forward(m, st, n, s_i, s_prev, inertia);
+  ht_gemm(m, st, {ht_prob(t.xht, D, n, m->w_head, D, n, V, D, t.logits, t.Vl, m->b_head, false)});
+  ht_launch_ce(st, dt, t.logits, t.Vl, n, V, Vp, target, t.lossr, t.dlt, loss, m->err_word);
+  const int S0 = ht_dxh_splits(n, D, Vp, t.sms);
+  const int kc = (cdiv(Vp, S0) + 63) / 64 * 64;
+  GemmProblem ps[HT_DXH_SPLITS];
+  int S = 0;
+  for (int k0 = 0; k0 < Vp; k0 += kc, ++S)
+    ps[S] = ht_prob((const char*)t.dlt + (size_t)k0 * m->esz, Vp, n, (const char*)t.headT + (size_t)k0 * m->esz, Vp, n,
+                    D, std::min(kc, Vp - k0), t.dxh + (size_t)S * n * D, D, nullptr, false);
+  ht_gemm_n(m, st, ps, S);
+  return ht_backward(m, st, n, S, s_i, s_prev, inertia, hp, 1 + (loss ? 1 : 0));
+}
+
+// Encoder step (Sec. 4.3): similarity rows against the original final states, then, on the
+// first n_cls rows, the frozen pooler (dense + tanh) and classifier with their cross-entropy;
+// the pooler's input gradient adds into those rows of dxh.
+static adept_status ht_step_cls(adept_model* m, int n, const float* s_i, const float* s_prev, const float* inertia,
+                                const float* s_final, int n_cls, const int32_t* label, float cls_weight,
+                                const adept_adamw& hp, float* loss, cudaStream_t st) {
+  HsmTrain& t = *m->ht;
+  const int D = m->D, dt = m->dt;
+  ht_forward(m, st, n, s_i, s_prev, inertia);
+  ht_launch_cos(st, t.stf, s_final, n, D, t.lossr, t.dxh);
+  int own = 1;
+  const float wc = n_cls > 0 ? cls_weight / (float)n_cls : 0.f;
+  if (n_cls > 0) {
+    ht_gemm(m, st, {ht_prob(t.xht, D, n_cls, m->w_pool, D, n_cls, D, D, t.zp, D, m->b_pool, false)});
+    ht_launch_cls(st, dt, t.zp, n_cls, D, m->w_cls, m->b_cls, m->cfg.n_classes, label, wc, t.lossc, t.dpt, m->err_word);
+    ht_gemm(m, st, {ht_prob(t.dpt, D, n_cls, t.poolT, D, n_cls, D, D, t.dxh, D, nullptr, true)});
+    ++own;
+  }
+  if (loss) {
+    ht_launch_loss(st, t.lossr, n, 1.f / (float)n, t.lossc, n_cls, wc, loss);
+    ++own;
+  }
+  return ht_backward(m, st, n, 1, s_i, s_prev, inertia, hp, own);
+}
+
+static bool adamw_ok(const adept_adamw* hp) {
+  return hp->lr >= 0.f && hp->beta1 >= 0.f && hp->beta1 < 1.f && hp->beta2 >= 0.f && hp->beta2 < 1.f && hp->eps > 0.f &&
+         hp->weight_decay >= 0.f;
 }
 
 // Plan of the persistent generation-step kernel (bf16 decoders; see decode_fused.cu).
@@ -1700,8 +1762,8 @@ adept_status adept_hsm_train_init(adept_model* m, int max_rows, void* stream) {
   if (!m) return ADEPT_ERR_INVALID_ARG;
   g_pdl = !m->profile;
   if (max_rows < 1) return fail(m, ADEPT_ERR_INVALID_ARG, "max_rows %d < 1", max_rows);
-  if (m->cfg.family == ADEPT_FAMILY_BERT)
-    return fail(m, ADEPT_ERR_INVALID_ARG, "HSM training takes decoders (next-token cross-entropy)");
+  if (m->cfg.family == ADEPT_FAMILY_BERT && (m->cfg.n_classes < 1 || m->cfg.n_classes > HT_MAX_CLASSES))
+    return fail(m, ADEPT_ERR_INVALID_ARG, "encoder HSM training needs n_classes in [1, %d]", HT_MAX_CLASSES);
   if (m->dt == ADEPT_DTYPE_BF16 && ((m->D | m->m1 | m->m2) & 7))
     return fail(m, ADEPT_ERR_INVALID_ARG, "bf16 HSM training needs D, m1, m2 multiples of 8");
   const adept_status s = ht_init(m, max_rows, (cudaStream_t)stream);
@@ -1715,12 +1777,31 @@ adept_status adept_hsm_train_step(adept_model* m, int n, const float* d_s_i, con
   if (!m) return ADEPT_ERR_INVALID_ARG;
   g_pdl = !m->profile;
   if (!m->ht) return fail(m, ADEPT_ERR_INVALID_ARG, "adept_hsm_train_init has not run");
+  if (m->cfg.family == ADEPT_FAMILY_BERT)
+    return fail(m, ADEPT_ERR_INVALID_ARG, "encoders train with adept_hsm_train_step_cls");
   if (n < 1 || n > m->ht->cap) return fail(m, ADEPT_ERR_INVALID_ARG, "n %d outside [1, %d]", n, m->ht->cap);
   if (!d_s_i || !d_s_prev || !d_inertia || !d_target || !hp) return fail(m, ADEPT_ERR_INVALID_ARG, "NULL pointer");
-  if (!(hp->lr >= 0.f) || !(hp->beta1 >= 0.f && hp->beta1 < 1.f) || !(hp->beta2 >= 0.f && hp->beta2 < 1.f) ||
-      !(hp->eps > 0.f) || !(hp->weight_decay >= 0.f))
-    return fail(m, ADEPT_ERR_INVALID_ARG, "AdamW hyperparameters out of range");
+  if (!adamw_ok(hp)) return fail(m, ADEPT_ERR_INVALID_ARG, "AdamW hyperparameters out of range");
   return ht_step(m, n, d_s_i, d_s_prev, d_inertia, d_target, *hp, d_loss_out, (cudaStream_t)stream);
+}
+
+adept_status adept_hsm_train_step_cls(adept_model* m, int n, const float* d_s_i, const float* d_s_prev,
+                                      const float* d_inertia, const float* d_s_final, int n_cls,
+                                      const int32_t* d_label, float cls_weight, const adept_adamw* hp,
+                                      float* d_loss_out, void* stream) {
+  if (!m) return ADEPT_ERR_INVALID_ARG;
+  g_pdl = !m->profile;
+  if (!m->ht) return fail(m, ADEPT_ERR_INVALID_ARG, "adept_hsm_train_init has not run");
+  if (m->cfg.family != ADEPT_FAMILY_BERT)
+    return fail(m, ADEPT_ERR_INVALID_ARG, "decoders train with adept_hsm_train_step");
+  if (n < 1 || n > m->ht->cap) return fail(m, ADEPT_ERR_INVALID_ARG, "n %d outside [1, %d]", n, m->ht->cap);
+  if (n_cls < 0 || n_cls > n) return fail(m, ADEPT_ERR_INVALID_ARG, "n_cls %d outside [0, %d]", n_cls, n);
+  if (!d_s_i || !d_s_prev || !d_inertia || !d_s_final || (n_cls > 0 && !d_label) || !hp)
+    return fail(m, ADEPT_ERR_INVALID_ARG, "NULL pointer");
+  if (!(cls_weight >= 0.f && cls_weight < INFINITY)) return fail(m, ADEPT_ERR_INVALID_ARG, "cls_weight out of range");
+  if (!adamw_ok(hp)) return fail(m, ADEPT_ERR_INVALID_ARG, "AdamW hyperparameters out of range");
+  return ht_step_cls(m, n, d_s_i, d_s_prev, d_inertia, d_s_final, n_cls, d_label, cls_weight, *hp, d_loss_out,
+                     (cudaStream_t)stream);
 }
 
 adept_status adept_hsm_train_read(adept_model* m, int what, int param, float* d_out, int64_t count, void* stream) {
