@@ -809,20 +809,28 @@ def kernel_case_llama_decode_small(device):
 
 def kernel_case_hsm_train(device, n=8192, steps=2, shape="gpt2"):
     """HSM training steps at GPT-2-small shapes (the bench section's workload; about 5 GB on
-    the device) or Llama-2-7B shapes (about 25 GB): n examples, two steps after one warm-up."""
+    the device), Llama-2-7B shapes (about 25 GB) or BERT-base shapes (the encoder step, n / 128
+    labelled rows): n examples, two steps after one warm-up."""
     import paper_2601_03700_gb300 as adept
     adept.load_library()
     if shape == "llama7b":
         cfg = synth.llama7b_config(n_layers=2, max_batch=1, max_seq=16)
+    elif shape == "bert":
+        cfg = synth.bert_base_config(n_layers=2, max_batch=1, max_seq=16)
     else:
         cfg = synth.gpt2_small_config(n_layers=2, max_batch=1, max_seq=16)
     W = synth.make_weights(cfg, seed=0)   # on the host: the launch list then holds the library's kernels only
     m = adept.Model(cfg, W)
     del W
-    s_i, s_prev, inertia, tgt = [x.to(device) for x in synth.hsm_train_batch(cfg, n, seed=1)]
     adept.adept_hsm_train_init(m.h, n)
+    if shape == "bert":
+        s_i, s_prev, inertia, s_fin, lab = [x.to(device) for x in synth.hsm_cls_batch(cfg, n, n // 128, seed=1)]
+        step = lambda: adept.adept_hsm_train_step_cls(m.h, n, s_i, s_prev, inertia, s_fin, lab, 1e-4)  # noqa
+    else:
+        s_i, s_prev, inertia, tgt = [x.to(device) for x in synth.hsm_train_batch(cfg, n, seed=1)]
+        step = lambda: adept.adept_hsm_train_step(m.h, n, s_i, s_prev, inertia, tgt, 1e-4)  # noqa
     for _ in range(steps + 1):
-        adept.adept_hsm_train_step(m.h, n, s_i, s_prev, inertia, tgt, 1e-4)
+        step()
     torch.cuda.synchronize()
     m.check()
     print(json.dumps({"kernel_case": "hsm_train", "n": n, "steps": steps + 1, "ok": True}))
@@ -844,7 +852,8 @@ def main():
     ap.add_argument("--fill-i", default="4,8,16,24")
     ap.add_argument("--cpu-tokens", type=int, default=512)
     ap.add_argument("--hsm-n", type=int, default=8192, help="examples per step of --kernel-case hsm_train")
-    ap.add_argument("--hsm-shape", default="gpt2", choices=["gpt2", "llama7b"], help="model shape of --kernel-case hsm_train")
+    ap.add_argument("--hsm-shape", default="gpt2", choices=["gpt2", "llama7b", "bert"],
+                    help="model shape of --kernel-case hsm_train")
     args = ap.parse_args()
     if args.kernel_case == "fill_small":
         kernel_case_fill_small(torch.device("cuda", 0))
