@@ -65,12 +65,13 @@ def gemm_work(M, N, K, esz=2, extra_out_bytes=0, extra_in_bytes=0):
     return 2.0 * M * N * K, float(N * K * esz + M * K * esz + extra_out_bytes + extra_in_bytes)
 
 
-def pass_work(cfg, exit_layers, decode: bool):
+def pass_work(cfg, exit_layers, decode: bool, n_seq: int = B, hsm: bool = True):
     """Algorithmic (flops, bytes) of the GEMMs of one pass given each token's exit layer.
 
     Counts what the method needs: layer i's projections for the tokens active at i,
     layer i's K/V of the tokens that left before i (prompt pass), the HSM of the
-    exiting tokens, and the head; weights are read once per launch."""
+    exiting tokens (hsm=False: the identity mapper, no HSM work), and the head (one row per
+    sequence in a prompt pass of n_seq sequences); weights are read once per launch."""
     N, D, F = cfg.n_layers, cfg.d_model, cfg.d_ffn
     dq, dkv, m1, m2 = cfg.d_q, cfg.d_kv, cfg.hsm_m1, cfg.hsm_m2
     up = 2 * F if cfg.family == synth.LLAMA else F
@@ -88,17 +89,17 @@ def pass_work(cfg, exit_layers, decode: bool):
         if not decode and ex > 0 and i >= 3:
             fl += 2.0 * ex * 2 * dkv * D
             by += ex * D * 2 + ex * 2 * dkv * 2
-        E = int(np.sum(e == i)) if i < N else 0
+        E = int(np.sum(e == i)) if i < N and hsm else 0
         if not decode and E > 0:
             for w in (gemm_work(E, m1, D), gemm_work(E, m2, m1), gemm_work(E, m1, m2), gemm_work(E, D, m1)):
                 fl += w[0]
                 by += w[1]
-    if decode:
+    if decode and hsm:
         E = int(np.sum(e < N))
         for w in (gemm_work(E, m1, D), gemm_work(E, m2, m1), gemm_work(E, m1, m2), gemm_work(E, D, m1)):
             fl += w[0]
             by += w[1]
-    rows = len(e) if decode else B
+    rows = len(e) if decode else n_seq
     w = gemm_work(rows, cfg.vocab, D, extra_out_bytes=rows * cfg.vocab * 4)
     return fl + w[0], by + w[1]
 
@@ -278,12 +279,13 @@ def run_fill_micro(adept, device, peaks, grid_T, grid_i, reps=3):
     return rows
 
 
-def llama_work(cfg, exit_prompt, exit_decode):
-    """Algorithmic flops of a Llama-shaped prompt pass + generation steps (GEMMs, fills, HSM,
-    head) from the exit layers: the cost the early exit saves or adds."""
-    fl = pass_work(cfg, exit_prompt, decode=False)[0]
+def llama_work(cfg, exit_prompt, exit_decode, hsm: bool = True):
+    """Algorithmic flops of a one-sequence Llama-shaped prompt pass + generation steps (GEMMs,
+    fills, HSM unless hsm=False, head) from the exit layers: the cost the early exit saves or
+    adds."""
+    fl = pass_work(cfg, exit_prompt, decode=False, n_seq=1, hsm=hsm)[0]
     for e in exit_decode:
-        fl += pass_work(cfg, e, decode=True)[0] + decode_fill_work(cfg, e)[0]
+        fl += pass_work(cfg, e, decode=True, hsm=hsm)[0] + decode_fill_work(cfg, e)[0]
     return fl
 
 
@@ -408,7 +410,9 @@ def run_hsm_train(adept, device, peaks, n=8192, reps=5, shape="gpt2"):
 
 def run_llama_e2e(adept, device, P=2048, steps=256):
     """Llama-2-7B shape, batch 1: 2048-token prompt + 256 greedy decode steps, exit layer per
-    token ~ N(24, 4) truncated to [8, 32] -- against the same library forced to full depth."""
+    token ~ N(24, 4) truncated to [8, 32] -- against the same library forced to full depth, and
+    the same exits with the identity mapper in place of the HSM (s~ = s_i*: the speed-up the
+    exits and fills alone allow)."""
     cfg = synth.llama7b_config(max_batch=1, max_seq=P + steps, max_pass_tokens=P)
     W = synth.make_weights(cfg, seed=0, device=device)
     m = adept.Model(cfg, W)
@@ -424,7 +428,8 @@ def run_llama_e2e(adept, device, P=2048, steps=256):
     exp_ = torch.empty(P, dtype=torch.int32, device=device)
     st = torch.cuda.current_stream()
     out = {}
-    for name, a, b in (("early_exit", fp, fd), ("full_depth", full_p, full_d)):
+    for name, a, b in (("early_exit", fp, fd), ("full_depth", full_p, full_d), ("hsm_identity", fp, fd)):
+        adept.adept_set_option(m.h, adept.OPT_HSM_IDENTITY, int(name == "hsm_identity"))
         for rep in range(2):   # first run warms up (and captures the generation-step graph)
             e0, e1, e2 = [torch.cuda.Event(enable_timing=True) for _ in range(3)]
             torch.cuda.synchronize()
@@ -442,16 +447,21 @@ def run_llama_e2e(adept, device, P=2048, steps=256):
                      "decode_ms_per_step": round(td * 1e3 / steps, 4),
                      "mean_exit_depth": round(float(np.concatenate([exp_.cpu().numpy(),
                                                                     exd.cpu().numpy().reshape(-1)]).mean()), 3),
-                     "algorithmic_tflop": round(llama_work(cfg, exp_.cpu().numpy(), exd.cpu().numpy()) / 1e12, 3)}
+                     "algorithmic_tflop": round(llama_work(cfg, exp_.cpu().numpy(), exd.cpu().numpy(),
+                                                           hsm=name != "hsm_identity") / 1e12, 3)}
+    adept.adept_set_option(m.h, adept.OPT_HSM_IDENTITY, 0)
     m.close()
     torch.cuda.empty_cache()
-    ee, fd_ = out["early_exit"], out["full_depth"]
+    ee, fd_, hi = out["early_exit"], out["full_depth"], out["hsm_identity"]
     return {"workload": "Llama-2-7B shape, bf16, random-init; batch 1, 2048-token prompt + 256 greedy decode steps; "
-                        "exit layer per token ~ N(24,4) truncated to [8,32] vs all tokens forced to layer 32",
-            "early_exit": ee, "full_depth": fd_,
+                        "exit layer per token ~ N(24,4) truncated to [8,32] vs all tokens forced to layer 32; "
+                        "the same exits with the identity mapper",
+            "early_exit": ee, "full_depth": fd_, "hsm_identity": hi,
             "speedup": round(ee["tok_s"] / fd_["tok_s"], 4),
             "algorithmic_ratio": round(fd_["algorithmic_tflop"] / ee["algorithmic_tflop"], 4),
-            "depth_ratio": round(fd_["mean_exit_depth"] / ee["mean_exit_depth"], 4)}
+            "depth_ratio": round(fd_["mean_exit_depth"] / ee["mean_exit_depth"], 4),
+            "speedup_hsm_identity": round(hi["tok_s"] / fd_["tok_s"], 4),
+            "algorithmic_ratio_hsm_identity": round(fd_["algorithmic_tflop"] / hi["algorithmic_tflop"], 4)}
 
 
 def max_over_ranks(x: float, world: int, device) -> float:
@@ -687,9 +697,28 @@ def cores():
 def cpu_baseline(n_tokens: int):
     n_seq, prompt, steps = 4, n_tokens, 8
     tok, dt = oracle_sample(n_seq, prompt, steps)
-    return {"value": round(tok / dt, 3), "unit": "tokens/s", "cores": cores(), "kind": "oracle",
-            "sample": f"{n_seq} prompt x {prompt} tokens + {steps} decode steps of the same model and exit law "
-                      f"(fp64 NumPy oracle, {dt:.1f} s)"}
+    out = {"value": round(tok / dt, 3), "unit": "tokens/s", "cores": cores(), "kind": "oracle",
+           "sample": f"{n_seq} prompt x {prompt} tokens + {steps} decode steps of the same model and exit law "
+                     f"(fp64 NumPy oracle, {dt:.1f} s)"}
+    out["single_core"] = oracle_single_core(1, 128, 8)
+    return out
+
+
+def oracle_single_core(n_seq: int, prompt: int, steps: int):
+    """The same oracle on one host core: a fresh interpreter with every BLAS / OpenMP pool
+    limited to one thread, on a smaller bounded sample."""
+    env = dict(os.environ)
+    for k in ("OMP_NUM_THREADS", "OPENBLAS_NUM_THREADS", "MKL_NUM_THREADS", "BLIS_NUM_THREADS"):
+        env[k] = "1"
+    env["CUDA_VISIBLE_DEVICES"] = ""
+    try:
+        r = subprocess.run([sys.executable, os.path.abspath(__file__), "--oracle-sample", f"{n_seq},{prompt},{steps}"],
+                           env=env, capture_output=True, text=True, timeout=600)
+        d = json.loads([x for x in r.stdout.splitlines() if x.startswith("{")][-1])
+    except Exception as e:   # reported, not fatal: the all-core figure stands
+        return {"unavailable": f"{type(e).__name__}: {e}"[:200]}
+    return {"value": round(d["tokens"] / d["seconds"], 3), "unit": "tokens/s", "cores": 1,
+            "sample": f"{n_seq} prompt x {prompt} tokens + {steps} decode steps ({d['seconds']:.1f} s)"}
 
 
 def reference_arm(args, rank, world):
@@ -854,7 +883,13 @@ def main():
     ap.add_argument("--hsm-n", type=int, default=8192, help="examples per step of --kernel-case hsm_train")
     ap.add_argument("--hsm-shape", default="gpt2", choices=["gpt2", "llama7b", "bert"],
                     help="model shape of --kernel-case hsm_train")
+    ap.add_argument("--oracle-sample", default=None, help="n_seq,prompt,steps: time the oracle alone (CPU)")
     args = ap.parse_args()
+    if args.oracle_sample:
+        n_seq, prompt, steps = (int(x) for x in args.oracle_sample.split(","))
+        tok, dt = oracle_sample(n_seq, prompt, steps)
+        print(json.dumps({"tokens": tok, "seconds": dt}), flush=True)
+        return
     if args.kernel_case == "fill_small":
         kernel_case_fill_small(torch.device("cuda", 0))
         return
