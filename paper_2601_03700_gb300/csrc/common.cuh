@@ -288,6 +288,9 @@ struct GemmProblem {
   int N;
   int K;
   Epi epi;
+  // rows on the device that are usually far below their bound (the prompt pass's exiting
+  // rows): the tensor-core launcher may split the problem by the live count
+  int split_live = 0;
 };
 
 static inline int cdiv(int a, int b) { return (a + b - 1) / b; }

@@ -40,6 +40,7 @@ struct TcGroup {
   int gm;           // m-tiles per raster super-row (their A rows stay in L2 while n sweeps)
   int a_box;        // rows of A per TMA box: 128, or fewer when the whole problem is one short tile
                     // (the MMA still spans 128 rows; rows past the box are never stored)
+  int m_lo, m_hi;   // live row-count gate: no tiles unless m_lo <= M and (m_hi == 0 or M <= m_hi)
   Epi epi;
 };
 
@@ -266,7 +267,8 @@ __global__ void __launch_bounds__(TC_THREADS, 1) gemm_tc_kernel(const __grid_con
     int acc = 0;
     for (int g = 0; g < ng; ++g) {
       const int b = p.g[g].rows.b();
-      const int M = max(0, p.g[g].rows.e() - b);
+      int M = max(0, p.g[g].rows.e() - b);
+      if (M < p.g[g].m_lo || (p.g[g].m_hi > 0 && M > p.g[g].m_hi)) M = 0;
       const int tn = (p.g[g].N + BN - 1) / BN;
       s_mbeg[g] = b;
       s_M[g] = M;
@@ -658,10 +660,9 @@ bool tc_encode_weight_3d(CUtensorMap* m, const void* base, int K, int rows, size
   return encode_3d(m, base, (uint64_t)K, (uint64_t)rows, (uint64_t)row_bytes, (uint32_t)box_rows, (uint32_t)kc);
 }
 
-template <int MAXG>
-static int launch_grouped(cudaStream_t st, const GemmProblem* probs, int n_probs, const int* max_rows,
-                          unsigned* err_word) {
-  // tile width: the widest that still gives every SM a tile
+// Tile width for row bounds max_rows: the widest that still gives every SM a tile; *tiles
+// the tile count at that width.
+static int pick_bn(const GemmProblem* probs, int n_probs, const int* max_rows, long long* tiles_out) {
   long long tiles[4] = {0, 0, 0, 0};
   const int bns[4] = {256, 128, 64, 32};
   for (int i = 0; i < n_probs; ++i) {
@@ -674,20 +675,46 @@ static int launch_grouped(cudaStream_t st, const GemmProblem* probs, int n_probs
       pick = k;
       break;
     }
-  const int BN = bns[pick];
+  *tiles_out = tiles[pick];
+  return bns[pick];
+}
+
+// A prepared launch: parameters (tensor maps encoded), tile width, k-chunks per stage, grid.
+template <int MAXG>
+struct TcPrepared {
+  TcParams<MAXG> prm;
+  int BN, KC, grid;
+};
+
+// Fills `L` for problems with row bounds max_rows and the live row-count gate [m_lo, m_hi]
+// (m_hi = 0: none); tile width force_bn, or (0) pick_bn's.  -1 when a tensor map cannot be
+// encoded (nothing launched).
+template <int MAXG>
+static int prepare_grouped(TcPrepared<MAXG>& L, const GemmProblem* probs, int n_probs, const int* max_rows,
+                           unsigned* err_word, int m_lo, int m_hi, int force_bn = 0) {
+  long long n_tiles = 0;
+  int BN = pick_bn(probs, n_probs, max_rows, &n_tiles);
+  if (force_bn) {
+    BN = force_bn;
+    n_tiles = 0;
+    for (int i = 0; i < n_probs; ++i)
+      n_tiles += (long long)((max_rows[i] + TC_BM - 1) / TC_BM) * ((probs[i].N + BN - 1) / BN);
+  }
   // short problems (every group one tile of at most TC_SHORT_ROWS rows, K in whole 64-chunks)
   // take the 3-D box variant: one TMA instruction per operand carries KC k-chunks
   bool short_rows = true;
   for (int i = 0; i < n_probs; ++i)
     short_rows &= max_rows[i] <= TC_SHORT_ROWS && probs[i].K % TC_BK == 0;
   const int KC = short_rows ? (BN == 256 ? 2 : 4) : 1;
-  static TcParams<MAXG> prm;  // kept off the stack; calls on a model are serialised
+  TcParams<MAXG>& prm = L.prm;
   memset(&prm, 0, sizeof prm);
   prm.n_groups = n_probs;
   prm.err = err_word;
   for (int i = 0; i < n_probs; ++i) {
     const GemmProblem& q = probs[i];
     TcGroup& G = prm.g[i];
+    G.m_lo = m_lo;
+    G.m_hi = m_hi;
     G.a_box = a_box_rows(max_rows[i]);
     if (KC > 1) {
       if (!encode_3d(&G.ta, q.A, (uint64_t)q.K, (uint64_t)q.a_rows, (uint64_t)q.lda * 2, (uint32_t)G.a_box,
@@ -707,22 +734,62 @@ static int launch_grouped(cudaStream_t st, const GemmProblem* probs, int n_probs
     G.epi = q.epi;
     G.tma_out = make_out_map(&G.tout, q) ? 1 : 0;
   }
-  const int grid = (int)std::min<long long>(tiles[pick], (long long)g_num_sms);
+  L.BN = BN;
+  L.KC = KC;
+  L.grid = (int)std::min<long long>(n_tiles, (long long)g_num_sms);
+  return 0;
+}
+
+template <int MAXG>
+static int launch_prepared(cudaStream_t st, const TcPrepared<MAXG>& L) {
+  const int grid = L.grid;
   if (grid <= 0) return 0;
-  if (KC > 1) {
-    switch (BN) {
-      case 256: return launch_bn<256, 2, MAXG, 2>(st, prm, grid);
-      case 128: return launch_bn<128, 2, MAXG, 4>(st, prm, grid);
-      case 64: return launch_bn<64, 3, MAXG, 4>(st, prm, grid);
-      default: return launch_bn<32, 4, MAXG, 4>(st, prm, grid);
+  if (L.KC > 1) {
+    switch (L.BN) {
+      case 256: return launch_bn<256, 2, MAXG, 2>(st, L.prm, grid);
+      case 128: return launch_bn<128, 2, MAXG, 4>(st, L.prm, grid);
+      case 64: return launch_bn<64, 3, MAXG, 4>(st, L.prm, grid);
+      default: return launch_bn<32, 4, MAXG, 4>(st, L.prm, grid);
     }
   }
-  switch (BN) {
-    case 256: return launch_bn<256, 4, MAXG>(st, prm, grid);
-    case 128: return launch_bn<128, 6, MAXG>(st, prm, grid);
-    case 64: return launch_bn<64, 8, MAXG>(st, prm, grid);
-    default: return launch_bn<32, 10, MAXG>(st, prm, grid);
+  switch (L.BN) {
+    case 256: return launch_bn<256, 4, MAXG>(st, L.prm, grid);
+    case 128: return launch_bn<128, 6, MAXG>(st, L.prm, grid);
+    case 64: return launch_bn<64, 8, MAXG>(st, L.prm, grid);
+    default: return launch_bn<32, 10, MAXG>(st, L.prm, grid);
   }
+}
+
+template <int MAXG>
+static int launch_grouped(cudaStream_t st, const GemmProblem* probs, int n_probs, const int* max_rows,
+                          unsigned* err_word) {
+  static TcPrepared<MAXG> L;  // kept off the stack; calls on a model are serialised
+  if (prepare_grouped(L, probs, n_probs, max_rows, err_word, 0, 0) < 0) return -1;
+  return launch_prepared(st, L);
+}
+
+// One problem whose live row count is on the device and usually far below its bound (the
+// prompt pass's exiting rows, flagged split_live): the host knows only the bound, whose tile
+// width can leave most SMs idle for the live count.  Two launches then share the problem: one
+// with the next narrower tiles for live counts up to m_split rows, the most row tiles that
+// width still fits in one wave (there each CTA loads (128 + BN) x K per tile instead of
+// (128 + 2 BN) x K, and twice the SMs pull), and the bound's launch for larger counts.  Each
+// finds no tiles when the count is outside its range, so exactly one of them runs the
+// product.  Both are prepared before either is launched.  Returns the launch count, or -1 when
+// the split does not apply.
+static int launch_split_live_rows(cudaStream_t st, const GemmProblem& q, int max_rows, unsigned* err_word) {
+  if (!q.split_live || !(q.rows.begin || q.rows.end) || max_rows <= TC_BM) return -1;
+  long long tiles = 0;
+  const int bn_wide = pick_bn(&q, 1, &max_rows, &tiles);
+  if (bn_wide <= 32) return -1;
+  const int bn_narrow = bn_wide / 2;
+  const long long row_tiles = g_num_sms / ((q.N + bn_narrow - 1) / bn_narrow);
+  if (row_tiles < 1) return -1;
+  const int m_split = (int)std::min<long long>(row_tiles * TC_BM, (long long)max_rows - 1);
+  static TcPrepared<2> narrow, wide;
+  if (prepare_grouped(narrow, &q, 1, &m_split, err_word, 0, m_split, bn_narrow) < 0) return -1;
+  if (prepare_grouped(wide, &q, 1, &max_rows, err_word, m_split + 1, 0) < 0) return -1;
+  return launch_prepared(st, narrow) + launch_prepared(st, wide);
 }
 
 int tc_gemm_grouped(cudaStream_t st, const GemmProblem* probs, int n_probs, const int* max_rows, unsigned* err_word) {
@@ -734,6 +801,10 @@ int tc_gemm_grouped(cudaStream_t st, const GemmProblem* probs, int n_probs, cons
     const GemmProblem& q = probs[i];
     if (q.K % 8 || q.lda % 8 || q.ldb % 8 || q.a_rows <= 0) return -1;
     if ((q.epi.kind == EPI_QKV || q.epi.kind == EPI_KV || q.epi.kind == EPI_SWIGLU) && (q.N % 32)) return -1;
+  }
+  if (n_probs == 1) {
+    const int nl = launch_split_live_rows(st, probs[0], max_rows[0], err_word);
+    if (nl >= 0) return nl;
   }
   // small launches carry a small parameter block (cheaper to launch)
   if (n_probs <= 2) return launch_grouped<2>(st, probs, n_probs, max_rows, err_word);

@@ -743,6 +743,7 @@ static void run_hsm(adept_model* m, cudaStream_t st, DevRange rows, int max_rows
   memset(&p, 0, sizeof p);
   p.rows = rows;
   p.a_rows = a_rows;
+  p.split_live = 1;   // the exiting rows of one layer: usually a small part of the pass
   // FC1: h1 = GELU(W1 c0 + b1)
   p.A = m->c0t; p.lda = D; p.B = m->hsm_w1; p.ldb = D; p.N = m1; p.K = D;
   p.epi = epi_base(); p.epi.kind = EPI_ACT; p.epi.act = ACT_GELU_ERF; p.epi.bias = m->hsm_b1;

@@ -170,6 +170,23 @@ def test_synth_generator_cpu_and_cuda_agree():
     assert torch.equal(a.view(torch.int16), b.view(torch.int16))
 
 
+def test_prompt_pass_mapper_split_by_live_rows():
+    """The prompt pass's mapper products split by the device-side exit count (narrow tiles up
+    to the split bound, the bound's tiles above it): 600 tokens with 300 leaving at layer 2 and
+    100 at layers 3 and 4 take both launches of each split product (a D = 512 model with
+    mapper widths 2048 / 4096 so that the bound's tiles are wide enough to split)."""
+    cfg = small(synth.GPT2, n_layers=6, d_model=512, n_heads=8, head_dim=64, d_ffn=1024, hsm_m1=2048, hsm_m2=4096,
+                max_seq=160, max_pos=160)
+    pair = Pair(cfg, seed=12, std=0.04)
+    B, P = 4, 150
+    tokens = synth.make_tokens(12, B, P, cfg.vocab).numpy()
+    law = np.array([2] * 300 + [3] * 100 + [4] * 100 + [6] * 100)
+    rng = np.random.default_rng(12)
+    forced = rng.permutation(law).reshape(B, P)
+    compare_prefill(pair, tokens, 0.9, forced)
+    pair.close()
+
+
 def test_tensor_core_gemm_matches_simt_gemm():
     """The tcgen05 grouped GEMM and the SIMT GEMM give the same pass (bf16 noise level),
     on a shape with ragged M tiles (130-token prompts) and every epilogue kind."""
