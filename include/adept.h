@@ -265,12 +265,14 @@ ADEPT_API adept_status adept_profile_read(adept_model* m, int cls, int64_t* laun
 ADEPT_API int adept_fused_decode_batch(const adept_model* m);
 ADEPT_API const char* adept_fused_decode_reason(const adept_model* m);
 
-/* ---- HSM training (Sec. 4.2; Sec. 5.1 "Training"; App. D) ----------------------------
- * The Hidden State Mapper is trained with the base model frozen: its mapped state s~ of an
- * example (s_i, s_{i-1}, I) goes through the frozen final norm and LM head, and the mean
- * cross-entropy against the example's target token (the next input token) is minimised with
- * AdamW (decoupled weight decay, bias-corrected moments).  Decoders only (the classification
- * loss of encoders is not provided).
+/* ---- HSM training (Sec. 4.2; Sec. 4.3; Sec. 5.1 "Training"; App. D) -------------------
+ * The Hidden State Mapper is trained with the base model frozen.  Decoders: its mapped state
+ * s~ of an example (s_i, s_{i-1}, I) goes through the frozen final norm and LM head, and the
+ * mean cross-entropy against the example's target token (the next input token) is minimised
+ * (adept_hsm_train_step).  Encoders: a similarity loss against the original final hidden
+ * states plus the frozen classifier's cross-entropy on the labelled rows
+ * (adept_hsm_train_step_cls).  Both with AdamW (decoupled weight decay, bias-corrected
+ * moments).
  *
  * Parameters, in this order (Table S1): 0 g0 [D], 1 conv_w [3][3], 2 conv_b [1], 3 fc1_w
  * [m1][D], 4 fc1_b [m1], 5 fc2_w [m2][m1], 6 fc2_b [m2], 7 fc3_w [m1][m2], 8 fc3_b [m1], 9 g1
