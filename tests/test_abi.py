@@ -57,4 +57,5 @@ def test_status_strings_and_load_validation_without_gpu(lib):
     assert lib.adept_hsm_train_init(None, 8, None) == 1
     assert lib.adept_hsm_train_step(None, 1, None, None, None, None, None, None, None) == 1
     assert lib.adept_hsm_train_read(None, 0, 0, None, 0, None) == 1
+    assert lib.adept_hsm_train_step_cls(None, 1, None, None, None, None, 0, None, 1.0, None, None, None) == 1
     assert lib.adept_hsm_param_numel(None, 0) == -1
