@@ -777,15 +777,34 @@ static int launch_grouped(cudaStream_t st, const GemmProblem* probs, int n_probs
 // finds no tiles when the count is outside its range, so exactly one of them runs the
 // product.  Both are prepared before either is launched.  Returns the launch count, or -1 when
 // the split does not apply.
+// The plan of that split for N columns and the row bound max_rows on `sms` SMs: the bound's
+// tile width (pick_bn's choice for one problem), the next narrower width, and m_split; false
+// when the split does not apply (one row tile, the narrowest width already, or one row tile of
+// the narrower width does not fit in one wave).
+static bool split_plan(int N, int max_rows, int sms, int* bn_wide, int* bn_narrow, int* m_split) {
+  if (max_rows <= TC_BM || N <= 0 || sms <= 0) return false;
+  const long long tm = (max_rows + TC_BM - 1) / TC_BM;
+  const int bns[4] = {256, 128, 64, 32};
+  int w = 32;
+  for (int k = 0; k < 4; ++k)
+    if (tm * ((N + bns[k] - 1) / bns[k]) >= sms) {
+      w = bns[k];
+      break;
+    }
+  if (w <= 32) return false;
+  const int nb = w / 2;
+  const long long row_tiles = sms / ((N + nb - 1) / nb);
+  if (row_tiles < 1) return false;
+  *bn_wide = w;
+  *bn_narrow = nb;
+  *m_split = (int)std::min<long long>(row_tiles * TC_BM, (long long)max_rows - 1);
+  return true;
+}
+
 static int launch_split_live_rows(cudaStream_t st, const GemmProblem& q, int max_rows, unsigned* err_word) {
-  if (!q.split_live || !(q.rows.begin || q.rows.end) || max_rows <= TC_BM) return -1;
-  long long tiles = 0;
-  const int bn_wide = pick_bn(&q, 1, &max_rows, &tiles);
-  if (bn_wide <= 32) return -1;
-  const int bn_narrow = bn_wide / 2;
-  const long long row_tiles = g_num_sms / ((q.N + bn_narrow - 1) / bn_narrow);
-  if (row_tiles < 1) return -1;
-  const int m_split = (int)std::min<long long>(row_tiles * TC_BM, (long long)max_rows - 1);
+  if (!q.split_live || !(q.rows.begin || q.rows.end)) return -1;
+  int bn_wide = 0, bn_narrow = 0, m_split = 0;
+  if (!split_plan(q.N, max_rows, g_num_sms, &bn_wide, &bn_narrow, &m_split)) return -1;
   static TcPrepared<2> narrow, wide;
   if (prepare_grouped(narrow, &q, 1, &m_split, err_word, 0, m_split, bn_narrow) < 0) return -1;
   if (prepare_grouped(wide, &q, 1, &max_rows, err_word, m_split + 1, 0) < 0) return -1;
@@ -874,6 +893,18 @@ int tc_gemm_grouped_nocache(cudaStream_t st, const GemmProblem* probs, int n_pro
 ADEPT_KTRACE_ATTACH(tc)
 
 }  // namespace adept
+
+// Host-side check of the live-row split plan (no device work): returns 1 and {bound's tile
+// width, narrower width, m_split} in out3, or 0 when the split does not apply.
+extern "C" __attribute__((visibility("default"))) int adept_debug_tc_split_plan(int N, int max_rows, int sms,
+                                                                                 int* out3) {
+  int a = 0, b = 0, c = 0;
+  if (!adept::split_plan(N, max_rows, sms, &a, &b, &c)) return 0;
+  out3[0] = a;
+  out3[1] = b;
+  out3[2] = c;
+  return 1;
+}
 
 #ifdef ADEPT_TC_TRACE
 extern "C" __attribute__((visibility("default"))) int adept_debug_tc_trace(long long* out, unsigned* n_launches) {
