@@ -308,6 +308,25 @@ def test_synth_generator_is_deterministic_and_normal():
     assert u.min() == 4 and u.max() == 12
 
 
+def test_synth_training_batches_follow_their_recipe():
+    """HSM training examples: s_i - s_{i-1} ~ N(0, (0.3 std)^2); I = (k - 1) unit(s_{i-1}) + noise
+    with k in [2, N - 1]; targets in [0, V); encoder examples add s_N - s_i ~ N(0, (0.5 std)^2) and
+    labels in [0, n_classes) for the first n_cls rows."""
+    cfg = synth.bert_base_config(n_layers=12)
+    s_i, s_prev, inertia, tgt = synth.hsm_train_batch(cfg, 4000, seed=3, std=0.5)
+    assert abs(s_prev.std().item() / 0.5 - 1) < 0.01
+    assert abs((s_i - s_prev).std().item() / 0.15 - 1) < 0.01
+    u = s_prev / s_prev.norm(dim=1, keepdim=True)
+    k1 = (inertia * u).sum(1)   # (k - 1) + the noise's projection
+    assert k1.min().item() > 1 - 0.6 and k1.max().item() < cfg.n_layers - 2 + 0.6
+    assert int(tgt.min()) >= 0 and int(tgt.max()) < cfg.vocab
+    a, b, c, s_fin, lab = synth.hsm_cls_batch(cfg, 4000, 64, seed=3, std=0.5)
+    assert torch.equal(a, s_i) and torch.equal(b, s_prev) and torch.equal(c, inertia)
+    assert abs((s_fin - s_i).std().item() / 0.25 - 1) < 0.01
+    assert lab.shape == (64,) and lab.dtype == torch.int32
+    assert int(lab.min()) == 0 and int(lab.max()) == cfg.n_classes - 1
+
+
 # ----------------------------------------------------------------------------- threshold calibration
 
 def test_rdc_closed_forms():
