@@ -280,3 +280,16 @@ def test_cls_bf16_mode_stays_within_rounding_of_exact():
     for k in HT.HSM_PARAMS:
         e = np.linalg.norm(g16[k] - g64[k]) / np.linalg.norm(g64[k])
         assert e < 3e-2, (k, e)
+
+
+def test_one_class_task_term_vanishes():
+    """With a single class the softmax is 1 whatever the logits: the task term and its gradient
+    are exactly zero, so the step equals the similarity-only step."""
+    cfg = tiny_bert(n_classes=1)
+    W, s_i, s_prev, inertia, s_fin, _ = setup_cls(cfg, n=5, n_cls=3)
+    lab = torch.zeros(3, dtype=torch.long)
+    l1, g1, _, _ = HT.hsm_cls_train_step(W, cfg, s_i, s_prev, inertia, s_fin, lab, 2.0, 1e-3, 0.9, 0.999, 1e-8, 0.0, 1)
+    l0, g0, _, _ = HT.hsm_cls_train_step(W, cfg, s_i, s_prev, inertia, s_fin, [], 2.0, 1e-3, 0.9, 0.999, 1e-8, 0.0, 1)
+    assert l1 == l0
+    for k in HT.HSM_PARAMS:
+        np.testing.assert_array_equal(g1[k], g0[k])
