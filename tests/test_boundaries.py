@@ -44,3 +44,14 @@ def test_library_imports_with_the_oracle_unavailable():
             "print(len(a.ABI_SYMBOLS))")
     r = subprocess.run([sys.executable, "-c", code], cwd=ROOT, capture_output=True, text=True, timeout=300)
     assert r.returncode == 0, r.stderr[-2000:]
+
+
+def test_missing_library_fails_loudly():
+    """No CPU fallback: loading a library that is not built raises."""
+    code = ("import paper_2601_03700_gb300 as a\n"
+            "try:\n"
+            "    a.load_library('/nonexistent/libadept.so')\n"
+            "except RuntimeError as e:\n"
+            "    print('raised', 'not built' in str(e))\n")
+    r = subprocess.run([sys.executable, "-c", code], cwd=ROOT, capture_output=True, text=True, timeout=300)
+    assert r.returncode == 0 and "raised True" in r.stdout, (r.stdout, r.stderr[-2000:])
