@@ -186,7 +186,11 @@ ADEPT_API adept_status adept_skip_kv_fill(adept_model* m, int n_tokens, const vo
  *    current); make that first call before any stream capture.
  *  - Every call shares the array and it keeps the last call's contents (each call clears
  *    the counters it needs zeroed).  Calls that overlap on the GPU -- on different streams
- *    or for different models on one device -- race on it: serialise them. */
+ *    or for different models on one device -- race on it: serialise them.
+ *  - On the host the call keeps its launch description on the calling thread's stack and
+ *    in thread-local storage: host threads that drive different models (on different
+ *    devices, or one after the other on the GPU of one device) do not share host state.
+ *    The calling thread's programmatic-dependent-launch setting is restored on return. */
 #define ADEPT_NOALLOC_SCRATCH_BYTES ((size_t)16 << 20)
 ADEPT_API adept_status adept_skip_kv_fill_noalloc(adept_model* m, int n_tokens, const void* d_h_mapped,
                                                   const int32_t* d_exit_layer, const int32_t* d_seq,
@@ -229,11 +233,7 @@ ADEPT_API adept_status adept_check_device_status(adept_model* m, void* stream);
  * 0 launches every kernel directly.  DECODE_GEMM (default 1): single GEMMs of at most 16
  * rows (generation steps, output heads) of bf16 models run on the weight-streaming
  * generation-step kernel, with the input standardisation fused in; 0 routes them to the
- * tcgen05 kernel after a separate standardisation launch.  FUSED_DECODE: 1 runs a
- * generation step of at most adept_fused_decode_batch() sequences of a bf16 decoder as
- * one persistent cooperative launch (every layer, the HSM, the fills and the head),
- * reading the caller's inputs and writing its outputs directly; 0 takes the multi-launch
- * step.  Default 0.  EXIT_METRIC (App. H.3): 0 (default) the global similarity of Sec. 4.1,
+ * tcgen05 kernel after a separate standardisation launch.  EXIT_METRIC (App. H.3): 0 (default) the global similarity of Sec. 4.1,
  * cos(s_i, sum_{d<i} s_hat_d); 1 the local similarity cos(s_i, s_{i-1}); 2 both (a token leaves
  * when both reach delta; the reported similarity is their minimum).  ALL_AT_ONCE (App. H.2):
  * 1 makes every token of a prompt take the exit decision of its sequence's last prompt token,
@@ -242,28 +242,22 @@ ADEPT_API adept_status adept_check_device_status(adept_model* m, void* stream);
  * token's computation entirely — no K/V of deeper layers, and deeper layers' attention sees
  * only the tokens still active there; its mapped state still feeds the classifier.  Default 0. */
 enum { ADEPT_OPT_HSM_IDENTITY = 1, ADEPT_OPT_PROFILE = 2, ADEPT_OPT_GEMM_SIMT = 3, ADEPT_OPT_DECODE_GRAPH = 4,
-       ADEPT_OPT_DECODE_GEMM = 5, ADEPT_OPT_FUSED_DECODE = 6, ADEPT_OPT_EXIT_METRIC = 7, ADEPT_OPT_ALL_AT_ONCE = 8,
+       ADEPT_OPT_DECODE_GEMM = 5, ADEPT_OPT_EXIT_METRIC = 7, ADEPT_OPT_ALL_AT_ONCE = 8,
        ADEPT_OPT_STOP_ENTIRELY = 9 };
 ADEPT_API adept_status adept_set_option(adept_model* m, int option, int value);
 
 /* Kernel classes reported by adept_profile_read: the GEMMs of prompt passes (layer
  * projections, HSM, head, and the per-layer skipped-layer fills co-launched with
  * layer i's QKV), the GEMMs of generation steps, the grouped skipped-layer fill
- * launches (end of a generation step and adept_skip_kv_fill), attention, and the
- * persistent generation-step launch (FUSED_DECODE), and the GEMMs of HSM training steps. */
+ * launches (end of a generation step and adept_skip_kv_fill), attention, and the GEMMs
+ * of HSM training steps. */
 enum { ADEPT_PROF_GEMM_PREFILL = 0, ADEPT_PROF_KV_FILL = 1, ADEPT_PROF_ATTENTION = 2,
-       ADEPT_PROF_GEMM_DECODE = 3, ADEPT_PROF_DECODE_STEP = 4, ADEPT_PROF_GEMM_TRAIN = 5, ADEPT_PROF_NCLASS = 6 };
+       ADEPT_PROF_GEMM_DECODE = 3, ADEPT_PROF_GEMM_TRAIN = 4, ADEPT_PROF_NCLASS = 5 };
 /* Synchronise, then return the number of recorded launches of kernel class `cls` and
  * their total device time in ms (CUDA events on the launching stream); resets the
  * record.  flops / bytes are reserved (returned as 0). */
 ADEPT_API adept_status adept_profile_read(adept_model* m, int cls, int64_t* launches, double* total_ms,
                                 double* flops, double* bytes);
-
-/* Largest batch a generation step runs as one persistent launch (0: the model or the
- * device does not take that path, or FUSED_DECODE is off), and why not (empty if it
- * does).  The reason string lives as long as the model. */
-ADEPT_API int adept_fused_decode_batch(const adept_model* m);
-ADEPT_API const char* adept_fused_decode_reason(const adept_model* m);
 
 /* ---- HSM training (Sec. 4.2; Sec. 4.3; Sec. 5.1 "Training"; App. D) -------------------
  * The Hidden State Mapper is trained with the base model frozen.  Decoders: its mapped state

@@ -19,10 +19,10 @@ LIB_PATH = os.path.join(_PKG, "libadept.so")
 ADEPT_OK = 0
 STATUS_NAMES = {0: "OK", 1: "INVALID_ARG", 2: "OOM", 3: "CAPACITY", 4: "CUDA", 5: "TIMEOUT", 6: "DEVICE_INPUT"}
 FAMILY = {"llama": 0, "gpt2": 1, "bert": 2}
-OPT_HSM_IDENTITY, OPT_PROFILE, OPT_GEMM_SIMT, OPT_DECODE_GRAPH, OPT_DECODE_GEMM, OPT_FUSED_DECODE = 1, 2, 3, 4, 5, 6
+OPT_HSM_IDENTITY, OPT_PROFILE, OPT_GEMM_SIMT, OPT_DECODE_GRAPH, OPT_DECODE_GEMM = 1, 2, 3, 4, 5
 OPT_EXIT_METRIC, OPT_ALL_AT_ONCE, OPT_STOP_ENTIRELY = 7, 8, 9
 EXIT_GLOBAL, EXIT_LOCAL, EXIT_BOTH = 0, 1, 2
-PROF_GEMM_PREFILL, PROF_KV_FILL, PROF_ATTENTION, PROF_GEMM_DECODE, PROF_DECODE_STEP, PROF_GEMM_TRAIN = 0, 1, 2, 3, 4, 5
+PROF_GEMM_PREFILL, PROF_KV_FILL, PROF_ATTENTION, PROF_GEMM_DECODE, PROF_GEMM_TRAIN = 0, 1, 2, 3, 4
 HSM_PARAMS, HSM_GRADS, HSM_MOMENT1, HSM_MOMENT2 = 0, 1, 2, 3
 # HSM parameters in the order of adept_hsm_train_read's `param` (Table S1)
 HSM_PARAM_NAMES = ["hsm.g0", "hsm.conv_w", "hsm.conv_b", "hsm.fc1_w", "hsm.fc1_b", "hsm.fc2_w", "hsm.fc2_b",
@@ -33,7 +33,7 @@ ABI_SYMBOLS = [
     "adept_model_load", "adept_prefill", "adept_decode_step", "adept_skip_kv_fill", "adept_free",
     "adept_last_error", "adept_status_string", "adept_seq_reserve", "adept_read_kv",
     "adept_read_final_states", "adept_check_device_status", "adept_set_option", "adept_profile_read",
-    "adept_launch_count", "adept_skip_kv_fill_noalloc", "adept_fused_decode_batch", "adept_fused_decode_reason",
+    "adept_launch_count", "adept_skip_kv_fill_noalloc",
     "adept_calibrate_threshold", "adept_hsm_train_init", "adept_hsm_train_step", "adept_hsm_train_read",
     "adept_hsm_param_numel", "adept_hsm_train_step_cls",
 ]
@@ -105,10 +105,6 @@ def load_library(path: str = LIB_PATH):
                                        ctypes.POINTER(ctypes.c_double), ctypes.POINTER(ctypes.c_double)]
     lib.adept_launch_count.argtypes = [vp]
     lib.adept_launch_count.restype = ctypes.c_int64
-    lib.adept_fused_decode_batch.argtypes = [vp]
-    lib.adept_fused_decode_batch.restype = c_int
-    lib.adept_fused_decode_reason.argtypes = [vp]
-    lib.adept_fused_decode_reason.restype = ctypes.c_char_p
     lib.adept_calibrate_threshold.argtypes = [vp, c_int, c_int, i32p, c_float, c_float, c_int, c_float, c_float,
                                               ctypes.POINTER(c_float), ctypes.POINTER(c_float),
                                               ctypes.POINTER(c_int), st]
@@ -396,10 +392,3 @@ class Model:
         out = torch.empty(adept_hsm_param_numel(self.h, param), dtype=torch.float32, device="cuda")
         adept_hsm_train_read(self.h, what, param, out)
         return out
-
-    def fused_decode_batch(self) -> int:
-        """Largest batch a generation step runs as one persistent launch (0: never)."""
-        return int(load_library().adept_fused_decode_batch(self.h))
-
-    def fused_decode_reason(self) -> str:
-        return load_library().adept_fused_decode_reason(self.h).decode(errors="replace")

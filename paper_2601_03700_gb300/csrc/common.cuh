@@ -128,6 +128,14 @@ namespace adept {
 // point sets it for its calling thread; it is off while per-launch profiling events are
 // recorded, so each timed interval holds one kernel alone).
 extern thread_local bool g_pdl;
+// Sets g_pdl for the calling thread for one scope and restores the previous value on exit.
+struct PdlScope {
+  bool prev;
+  explicit PdlScope(bool on) : prev(g_pdl) { g_pdl = on; }
+  ~PdlScope() { g_pdl = prev; }
+  PdlScope(const PdlScope&) = delete;
+  PdlScope& operator=(const PdlScope&) = delete;
+};
 template <typename... KArgs, typename... Args>
 inline cudaError_t launch_k(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t smem, cudaStream_t st,
                             Args&&... args) {

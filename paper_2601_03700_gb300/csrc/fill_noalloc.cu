@@ -59,7 +59,9 @@ extern "C" ADEPT_API adept_status adept_skip_kv_fill_noalloc(adept_model* m, int
                                                              const int32_t* d_exit_layer, const int32_t* d_seq,
                                                              const int32_t* d_pos, void* stream) {
   if (!m) return ADEPT_ERR_INVALID_ARG;
-  g_pdl = true;  // this entry point records no profiling events
+  // launches chain by programmatic dependent launch (this entry point records no profiling
+  // events); the calling thread's setting is restored on return
+  PdlScope pdl_scope(true);
   if (n_tokens < 0) {
     model_set_error(m, "n_tokens < 0");
     return ADEPT_ERR_INVALID_ARG;
@@ -69,7 +71,7 @@ extern "C" ADEPT_API adept_status adept_skip_kv_fill_noalloc(adept_model* m, int
     model_set_error(m, "NULL device pointer");
     return ADEPT_ERR_INVALID_ARG;
   }
-  static FillView v;  // static storage: nothing on the heap
+  FillView v;  // on the stack (about 4 KB): nothing on the heap, nothing shared between threads
   if (!model_fill_view(m, &v)) {
     model_set_error(m, "adept_skip_kv_fill_noalloc: model has more layers than the fixed view holds");
     return ADEPT_ERR_INVALID_ARG;
@@ -82,7 +84,7 @@ extern "C" ADEPT_API adept_status adept_skip_kv_fill_noalloc(adept_model* m, int
   const size_t tok_bytes = align256((size_t)n_tokens * sizeof(int));
   const size_t bucket_bytes = align256(3 * (size_t)(FILL_VIEW_MAX_LAYERS + 2) * sizeof(int));
   if (x_bytes + tok_bytes + bucket_bytes > NOALLOC_SCRATCH_BYTES) {
-    static char msg[200];
+    char msg[200];
     snprintf(msg, sizeof msg,
              "adept_skip_kv_fill_noalloc: %d tokens need %zu bytes of scratch, above the fixed %zu bytes "
              "(at most %zu tokens of d_model %d)",
@@ -111,6 +113,7 @@ extern "C" ADEPT_API adept_status adept_skip_kv_fill_noalloc(adept_model* m, int
   // bucket by exit layer (the histogram is cleared here), standardise s~ once
   launch_fill_sort(st, v.dtype, d_h_mapped, n_tokens, v.d_model, d_exit_layer, v.n_layers, hist, start, cursor,
                    sorted_tok, xs, v.norm_mode, v.norm_eps, v.err_word);
+  model_add_launches(m, 4);
   // layer r's rows are the sorted prefix with i* < r; groups of at most 32 layers per launch
   GemmProblem probs[32];
   int max_rows[32];
@@ -141,10 +144,12 @@ extern "C" ADEPT_API adept_status adept_skip_kv_fill_noalloc(adept_model* m, int
     max_rows[np] = n_tokens;
     ++np;
     if (np == 32 || r == v.n_layers) {
-      if (tc_gemm_grouped_nocache(st, probs, np, max_rows, v.err_word) < 0) {
+      const int nl = tc_gemm_grouped_nocache(st, probs, np, max_rows, v.err_word);
+      if (nl < 0) {
         model_set_error(m, "adept_skip_kv_fill_noalloc: tensor-core launch rejected the shapes");
         return ADEPT_ERR_INVALID_ARG;
       }
+      model_add_launches(m, nl);
       np = 0;
     }
   }

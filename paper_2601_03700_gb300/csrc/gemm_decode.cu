@@ -874,7 +874,7 @@ static bool dg_plan(const GemmProblem& q, int max_rows, const DgNorm* norm, int 
 }
 
 int decode_gemm(cudaStream_t st, const GemmProblem& q, int max_rows, const DgNorm* norm, unsigned* err) {
-  static DgParams prm;   // 64-byte-aligned tensor map; calls on a model are serialised
+  thread_local DgParams prm;   // 64-byte-aligned tensor map; one per host thread
   memset(&prm, 0, sizeof prm);
   int grid = 0, mb = 1;
   size_t smem = 0;
@@ -893,7 +893,7 @@ int decode_gemm_grouped(cudaStream_t st, const GemmProblem* probs, int n, int ma
         q.rows.begin != nullptr || !decode_gemm_supported(q, max_rows, nullptr))
       return -1;
   }
-  static DgParamsG prm;   // calls on a model are serialised
+  thread_local DgParamsG prm;   // one per host thread
   memset(&prm, 0, sizeof prm);
   int grid = 0, mb = 1;
   size_t smem = 0;

@@ -763,7 +763,8 @@ static int launch_prepared(cudaStream_t st, const TcPrepared<MAXG>& L) {
 template <int MAXG>
 static int launch_grouped(cudaStream_t st, const GemmProblem* probs, int n_probs, const int* max_rows,
                           unsigned* err_word) {
-  static TcPrepared<MAXG> L;  // kept off the stack; calls on a model are serialised
+  // kept off the stack; one per host thread, so threads driving different models do not share it
+  thread_local TcPrepared<MAXG> L;
   if (prepare_grouped(L, probs, n_probs, max_rows, err_word, 0, 0) < 0) return -1;
   return launch_prepared(st, L);
 }
@@ -805,7 +806,7 @@ static int launch_split_live_rows(cudaStream_t st, const GemmProblem& q, int max
   if (!q.split_live || !(q.rows.begin || q.rows.end)) return -1;
   int bn_wide = 0, bn_narrow = 0, m_split = 0;
   if (!split_plan(q.N, max_rows, g_num_sms, &bn_wide, &bn_narrow, &m_split)) return -1;
-  static TcPrepared<2> narrow, wide;
+  thread_local TcPrepared<2> narrow, wide;
   if (prepare_grouped(narrow, &q, 1, &m_split, err_word, 0, m_split, bn_narrow) < 0) return -1;
   if (prepare_grouped(wide, &q, 1, &max_rows, err_word, m_split + 1, 0) < 0) return -1;
   return launch_prepared(st, narrow) + launch_prepared(st, wide);
@@ -853,7 +854,7 @@ int tc_gemm_grouped_nocache(cudaStream_t st, const GemmProblem* probs, int n_pro
       break;
     }
   const int BN = bns[pick];
-  static TcParams<TC_MAXG> prm;  // static storage, not heap; callers of this entry point serialise
+  thread_local TcParams<TC_MAXG> prm;  // per host thread, not on the heap
   memset(&prm, 0, sizeof prm);
   prm.n_groups = n_probs;
   prm.err = err_word;

@@ -19,4 +19,6 @@ struct FillView {
 
 bool model_fill_view(adept_model* m, FillView* v);
 void model_set_error(adept_model* m, const char* msg);
+// Adds n kernel launches to the model's count (adept_launch_count).
+void model_add_launches(adept_model* m, int n);
 }  // namespace adept

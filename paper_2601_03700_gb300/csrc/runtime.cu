@@ -6,7 +6,6 @@
 #include "kernels.h"
 #include "gemm_tc.h"
 #include "gemm_decode.h"
-#include "decode_fused.h"
 #include "model_view.h"
 #include "hsm_train.h"
 
@@ -141,14 +140,11 @@ struct adept_model {
   std::vector<cudaGraphExec_t> dec_graph;   // per batch size
   std::vector<int> dec_warm;                // direct runs done per batch size
   // options / instrumentation
-  int hsm_identity = 0, profile = 0, force_simt = 0, use_graph = 1, use_dg = 1, use_fused = 1;
+  int hsm_identity = 0, profile = 0, force_simt = 0, use_graph = 1, use_dg = 1;
   int exit_metric = 0;   // EXIT_GLOBAL / EXIT_LOCAL / EXIT_BOTH
   int all_at_once = 0;   // prompt passes: sequences leave with their last prompt token
   int stop_entirely = 0; // encoders: exited tokens get no deeper K/V and leave deeper attention
   int32_t* tok_exit = nullptr;   // stop-entirely passes: each token's exit layer so far
-  // persistent generation-step kernel (small batches of bf16 decoders); NULL when not eligible
-  DfState* df = nullptr;
-  std::string df_why;
   HsmTrain* ht = nullptr;   // HSM training state (adept_hsm_train_init)
   bool xhead_ready = false; // the last generation step left its head input rows in xhead
   std::vector<cudaEvent_t> ev_pool;
@@ -215,8 +211,6 @@ static void free_all(adept_model* m) {
   drop_graphs(m);
   delete m->ht;
   m->ht = nullptr;
-  df_destroy(m->df);
-  m->df = nullptr;
   if (m->cap_stream) cudaStreamDestroy(m->cap_stream);
   m->cap_stream = nullptr;
   for (void* p : m->allocs) cudaFree(p);
@@ -1340,45 +1334,6 @@ static bool adamw_ok(const adept_adamw* hp) {
          hp->weight_decay >= 0.f;
 }
 
-// Plan of the persistent generation-step kernel (bf16 decoders; see decode_fused.cu).
-static void build_fused(adept_model* m) {
-  const adept_config& c = m->cfg;
-  if (m->dt != ADEPT_DTYPE_BF16 || c.family == ADEPT_FAMILY_BERT) {
-    m->df_why = "fp32 models and encoders take the multi-launch step";
-    return;
-  }
-  std::vector<DfLayerSrc> L(m->N);
-  for (int l = 0; l < m->N; ++l) {
-    const LayerW& w = m->L[l];
-    L[l] = DfLayerSrc{w.w_qkv, w.b_qkv, w.w_o, w.b_o, w.w_up, w.b_up, w.up_rows, w.w_down, w.b_down};
-  }
-  DfModelSrc s;
-  memset(&s, 0, sizeof s);
-  s.N = m->N; s.D = m->D; s.H = m->H; s.Hkv = m->Hkv; s.dh = m->dh; s.Dq = m->Dq; s.Dkv = m->Dkv; s.F = m->F;
-  s.V = m->V; s.m1 = m->m1; s.m2 = m->m2; s.family = c.family; s.norm_mode = attn_norm_mode(m);
-  s.eps = c.norm_eps; s.hsm_eps = c.hsm_eps; s.max_batch = c.max_batch;
-  s.seq_cap = m->max_blocks_per_seq * c.kv_block_tokens;
-  s.max_pos = c.family == ADEPT_FAMILY_LLAMA ? 0 : c.max_pos;
-  s.tok_emb = m->tok_emb; s.pos_emb = m->pos_emb; s.L = L.data(); s.w_head = m->w_head; s.b_head = m->b_head;
-  s.hsm_w1 = m->hsm_w1; s.hsm_w2 = m->hsm_w2; s.hsm_w3 = m->hsm_w3; s.hsm_w4 = m->hsm_w4;
-  s.hsm_b1 = m->hsm_b1; s.hsm_b2 = m->hsm_b2; s.hsm_b3 = m->hsm_b3; s.hsm_b4 = m->hsm_b4;
-  s.hsm_g0 = m->hsm_g0; s.hsm_conv = m->hsm_conv; s.hsm_g1 = m->hsm_g1; s.hsm_g2 = m->hsm_g2;
-  s.rope_table = m->rope_table; s.cache = cache_view(m);
-  for (int k = 0; k < 2; ++k) {
-    s.X_in[k] = m->X_in[k];
-    s.I[k] = m->I[k];
-    s.row_tok[k] = m->row_tok[k];
-  }
-  s.X_out = m->X_out; s.tok_seq = m->tok_seq; s.tok_pos = m->tok_pos; s.seq_len = m->d_seq_len; s.ctr = m->ctr;
-  s.err = m->err_word; s.q = m->q; s.att = m->att; s.hbuf = m->hbuf; s.xfill = m->xfill; s.h1t = m->h1t;
-  s.h2t = m->h2t; s.hsm_s = m->hsm_s; s.hsm_prev = m->hsm_prev; s.hsm_I = m->hsm_I; s.final_ = m->final_;
-  s.c0f = m->c0f; s.h1f = m->h1f; s.h3f = m->h3f; s.h5f = m->h5f; s.logits = m->logits_ws; s.exit_tok = m->exit_tok;
-  m->df = df_create(s, &m->df_why);
-  // Off unless requested: the persistent step is under investigation for an intermittent
-  // device fault on large (Llama-7B-shaped) models; the multi-launch step is the default.
-  m->use_fused = 0;
-}
-
 
 // ---------------------------------------------------------------------------
 // C ABI
@@ -1430,7 +1385,6 @@ adept_status adept_model_load(const adept_config* cfg_in, const adept_tensor_tab
   }
   adept_status s = load_weights(m, ld);
   if (s == ADEPT_OK) s = alloc_runtime(m);
-  if (s == ADEPT_OK) build_fused(m);
   if (s == ADEPT_OK) {
     cudaError_t e = cudaStreamSynchronize(ld.st);
     if (e != cudaSuccess) s = fail(m, ADEPT_ERR_CUDA, "load: %s", cudaGetErrorString(e));
@@ -1501,23 +1455,6 @@ adept_status adept_decode_step(adept_model* m, int batch, const int32_t* d_token
       return fail(m, ADEPT_ERR_CAPACITY, "sequence %d is full (%d positions)", b, m->h_seq_len[b]);
   }
   cudaStream_t st = (cudaStream_t)stream;
-  if (m->df && m->use_fused && m->exit_metric == EXIT_GLOBAL && batch <= df_max_batch(m->df)) {
-    // one persistent launch for the whole step (decode_fused.cu); it reads the caller's
-    // inputs and writes the caller's outputs directly
-    cudaEvent_t ev = nullptr;
-    prof_begin(m, ADEPT_PROF_DECODE_STEP, st, &ev);
-    const cudaError_t e = df_step(m->df, st, batch, d_tokens, d_forced_exit, delta, m->hsm_identity, m->h_seq_len.data(),
-                                  d_exit_layer_out, d_sim_out, d_next_token_out ? d_next_token_out : m->dec_next);
-    prof_end(m, ADEPT_PROF_DECODE_STEP, st, ev, 0, 0);
-    if (e != cudaSuccess) return fail(m, ADEPT_ERR_CUDA, "fused generation step: %s", cudaGetErrorString(e));
-    m->launches += 1;
-    m->last_rows = batch;
-    for (int b = 0; b < batch; ++b) m->h_seq_len[b] += 1;
-    if (d_logits_out)
-      CUDA_TRY(m, cudaMemcpyAsync(d_logits_out, m->logits_ws, (size_t)batch * m->V * sizeof(float),
-                                  cudaMemcpyDeviceToDevice, st));
-    return check_launch(m);
-  }
   // inputs into the staging buffers; the step itself reads and writes only those
   launch_stage_in(st, m->d_delta, delta, d_tokens, m->dec_tok, d_forced_exit, m->dec_forced, batch);
   m->launches += 1;
@@ -1691,8 +1628,6 @@ adept_status adept_check_device_status(adept_model* m, void* stream) {
   CUDA_TRY(m, cudaMemcpy(&w, m->err_word, sizeof w, cudaMemcpyDeviceToHost));
   CUDA_TRY(m, cudaMemset(m->err_word, 0, sizeof(unsigned)));
   if (w & ERRW_TIMEOUT) {
-    df_reset(m->df, st);
-    CUDA_TRY(m, cudaStreamSynchronize(st));
     return fail(m, ADEPT_ERR_TIMEOUT, "a device-side wait timed out (word 0x%x)", w);
   }
   if (w) return fail(m, ADEPT_ERR_DEVICE_INPUT, "device-side input check failed (word 0x%x)", w);
@@ -1707,7 +1642,6 @@ adept_status adept_set_option(adept_model* m, int option, int value) {
     case ADEPT_OPT_GEMM_SIMT: m->force_simt = value != 0; drop_graphs(m); return ADEPT_OK;
     case ADEPT_OPT_DECODE_GRAPH: m->use_graph = value != 0; drop_graphs(m); return ADEPT_OK;
     case ADEPT_OPT_DECODE_GEMM: m->use_dg = value != 0; drop_graphs(m); return ADEPT_OK;
-    case ADEPT_OPT_FUSED_DECODE: m->use_fused = value != 0; return ADEPT_OK;
     case ADEPT_OPT_EXIT_METRIC:
       if (value < EXIT_GLOBAL || value > EXIT_BOTH) return fail(m, ADEPT_ERR_INVALID_ARG, "exit metric %d", value);
       m->exit_metric = value;
@@ -1747,16 +1681,6 @@ adept_status adept_profile_read(adept_model* m, int cls, int64_t* launches, doub
   for (auto& q : m->prof) any |= !q.ev.empty();
   if (!any) m->ev_used = 0;   // every recorded pair was read: the pool can be reused
   return ADEPT_OK;
-}
-
-int adept_fused_decode_batch(const adept_model* m) {
-  if (!m || !m->df || !m->use_fused) return 0;
-  return df_max_batch(m->df);
-}
-
-const char* adept_fused_decode_reason(const adept_model* m) {
-  if (!m) return "no model";
-  return m->df ? "" : m->df_why.c_str();
 }
 
 adept_status adept_hsm_train_init(adept_model* m, int max_rows, void* stream) {
@@ -1887,5 +1811,9 @@ bool model_fill_view(adept_model* m, FillView* v) {
 
 void model_set_error(adept_model* m, const char* msg) {
   if (m) m->err = msg;
+}
+
+void model_add_launches(adept_model* m, int n) {
+  if (m) m->launches += n;
 }
 }  // namespace adept

@@ -518,3 +518,111 @@ def test_encoder_stop_entirely_matches_independent_masked_model():
     np.testing.assert_allclose(r.final, final.numpy(), rtol=1e-10, atol=1e-10)
     # the classifier reads position 0's state
     np.testing.assert_allclose(r.logits[0], ref.head(final[0][None]).numpy()[0], rtol=1e-10, atol=1e-10)
+
+
+# ----------------------------------------------------------------------------- skipped-layer fill rows
+
+def test_skip_kv_fill_rows_are_exactly_the_skipped_layers():
+    """O.skip_kv_fill (Sec. 4.3 KV generation): token j is filled at exactly the layers
+    r = i*_j + 1 .. N (never at its exit layer i*_j itself, nothing for i*_j = N), and each
+    entry equals layer r's K/V projection of s~ evaluated with library ops (TorchRef.kv)."""
+    for family in (synth.LLAMA, synth.GPT2, synth.BERT):
+        cfg = small_cfg(family, n_layers=5)
+        m, ref, _ = model_and_ref(cfg, seed=22)
+        n = 12
+        mapped = synth.normal(22, "mapped", (n, cfg.d_model), std=1.0, dtype=torch.float64).numpy()
+        exit_layer = np.array([1, 2, 3, 4, 5, 5, 2, 3, 1, 4, 5, 2])
+        pos = np.array([0, 3, 1, 7, 2, 5, 4, 6, 9, 8, 11, 10])
+        out = O.skip_kv_fill(m, mapped, exit_layer, pos)
+        filled = {j: set() for j in range(n)}
+        for r, (k, v, sel) in out.items():
+            assert 2 <= r <= cfg.n_layers
+            for a, j in enumerate(sel):
+                filled[int(j)].add(r)
+                kw, vw = ref.kv(r, torch.as_tensor(mapped[j]), torch.tensor(int(pos[j])))
+                np.testing.assert_allclose(k[a], kw.numpy(), rtol=1e-11, atol=1e-12)
+                np.testing.assert_allclose(v[a], vw.numpy(), rtol=1e-11, atol=1e-12)
+        for j in range(n):
+            assert filled[j] == set(range(int(exit_layer[j]) + 1, cfg.n_layers + 1)), (family, j)
+
+
+# ----------------------------------------------------------------------------- bf16 contract
+
+def _bf16_pair(family):
+    cfg = small_cfg(family, n_layers=4, dtype="bf16")
+    W = synth.make_weights(cfg, seed=21, std=0.2, gain_std=0.1)
+    return cfg, O.OracleModel(cfg, W), TorchRef(cfg, W, bf16=True)
+
+
+def _bf16_gap(cfg, m, ref, tokens, forced):
+    """Largest relative gap between the oracle's bf16 pass and the reference's bf16 statement
+    of the contract, over final states, logits and every cached K/V entry."""
+    gaps = []
+    rel = lambda a, b: float(np.max(np.abs(a - b)) / max(np.max(np.abs(b)), 1e-30))  # noqa: E731
+    if cfg.family == synth.BERT:
+        cache = O.OracleCache(cfg, 1, 8)
+        r = O.prefill(m, cache, tokens, np.inf)
+        want = ref.full_forward(torch.as_tensor(tokens))[0]
+        gaps.append(rel(r.final, want.numpy()))
+        gaps.append(rel(r.logits, ref.head(want[0:1]).numpy()))
+        pos = torch.arange(tokens.shape[1])
+        h = ref.embed(torch.as_tensor(tokens[0]), pos)
+        for i in range(1, cfg.n_layers + 1):     # layer inputs again, for the cached K/V
+            k, v = ref.kv(i, h, pos)
+            gaps.append(rel(cache.K[i - 1][0, :tokens.shape[1]], k.numpy()))
+            gaps.append(rel(cache.V[i - 1][0, :tokens.shape[1]], v.numpy()))
+            q = ref.q(i, h, pos).transpose(0, 1)
+            a = F.scaled_dot_product_attention(q, k.transpose(0, 1), v.transpose(0, 1))
+            h = ref.after_attn(i, h, a.transpose(0, 1).flatten(-2))
+        return max(gaps)
+    cache = O.OracleCache(cfg, 1, 8)
+    r = O.prefill(m, cache, tokens, 0.5, forced)
+    fin, el, K, V = ref.token_major(tokens[0], forced)
+    np.testing.assert_array_equal(r.exit_layer, el.numpy())
+    gaps.append(rel(r.final, fin.numpy()))
+    gaps.append(rel(r.logits, ref.head(fin[-1:]).numpy()))
+    for i in range(1, cfg.n_layers + 1):
+        for j in range(tokens.shape[1]):
+            gaps.append(rel(cache.K[i - 1][0, j], K[i][j].numpy()))
+            gaps.append(rel(cache.V[i - 1][0, j], V[i][j].numpy()))
+    return max(gaps)
+
+
+@pytest.mark.parametrize("family", [synth.LLAMA, synth.GPT2, synth.BERT])
+def test_bf16_contract_matches_independent_statement(family):
+    """bf16 models: the oracle's pass (decoders: forced exits through the mapper and the fills;
+    the encoder: full depth) equals the torch reference with the contract's rounding points
+    applied by torch's own bf16 cast, to ~1e-12, in final states, logits and every cached K/V
+    entry."""
+    cfg, m, ref = _bf16_pair(family)
+    tokens = synth.make_tokens(21, 1, 6, cfg.vocab).numpy()
+    forced = np.array([2, 4, 3, 2, 4, 3])
+    assert _bf16_gap(cfg, m, ref, tokens, forced) < 1e-12
+
+
+@pytest.mark.parametrize("family", [synth.LLAMA, synth.GPT2, synth.BERT])
+def test_bf16_contract_pin_fails_on_a_missing_or_extra_rounding_point(family, monkeypatch):
+    """The agreement above has teeth: dropping any single rounding point the oracle takes
+    during the pass (each call of OracleModel.rb in turn), or adding one on the residual
+    stream, moves the oracle away from the reference by far more than 1e-12."""
+    cfg, m, ref = _bf16_pair(family)
+    tokens = synth.make_tokens(21, 1, 6, cfg.vocab).numpy()
+    forced = np.array([2, 4, 3, 2, 4, 3])
+    rb = O.OracleModel.rb
+    calls = {"n": 0, "skip": -1}
+
+    def counting_rb(self, x):
+        calls["n"] += 1
+        return x if calls["n"] - 1 == calls["skip"] else rb(self, x)
+
+    monkeypatch.setattr(O.OracleModel, "rb", counting_rb)
+    _bf16_gap(cfg, m, ref, tokens, forced)
+    total = calls["n"]
+    assert total >= 8 * cfg.n_layers
+    for k in range(total):
+        calls["n"], calls["skip"] = 0, k
+        assert _bf16_gap(cfg, m, ref, tokens, forced) > 1e-6, f"rounding point {k} of {total} has no effect"
+    monkeypatch.setattr(O.OracleModel, "rb", rb)
+    body = O.layer_body
+    monkeypatch.setattr(O, "layer_body", lambda mm, *a, **kw: O.round_bf16(body(mm, *a, **kw)))
+    assert _bf16_gap(cfg, m, ref, tokens, forced) > 1e-6

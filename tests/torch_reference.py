@@ -5,6 +5,12 @@ Used only to pin the oracle: it evaluates the same definitions in a different or
 "sequential unfold"), with library kernels (F.linear, F.rms_norm, F.layer_norm,
 F.conv2d, F.scaled_dot_product_attention, complex-number RoPE) instead of the
 oracle's NumPy expressions.  Layers are 1-based as in the paper.
+
+bf16=True states the bf16 precision contract on its own: weights are bf16 values, and
+torch's own float -> bfloat16 cast (round to nearest even) is applied to every GEMM input
+(the normalised layer and head inputs, the attention output, the FFN's activated hidden
+rows, the mapper's FC inputs, the pooler's input and output), to Q and to the cached K
+and V; everything else stays float64.
 """
 from __future__ import annotations
 
@@ -17,9 +23,14 @@ LLAMA, GPT2, BERT = 0, 1, 2
 
 
 class TorchRef:
-    def __init__(self, cfg, W):
+    def __init__(self, cfg, W, bf16: bool = False):
         self.c = cfg
         self.W = {k: (v if torch.is_tensor(v) else torch.as_tensor(v)).double() for k, v in W.items()}
+        self.bf16 = bf16
+
+    def r(self, x):
+        """A contract rounding point: bf16 round trip in bf16 mode, identity otherwise."""
+        return x.to(torch.bfloat16).double() if self.bf16 else x
 
     def lw(self, i, n):
         return self.W.get(f"layers.{i - 1}.{n}")
@@ -45,37 +56,37 @@ class TorchRef:
 
     def kv(self, i, h, pos):
         c = self.c
-        x = self.pre_attn(i, h)
+        x = self.r(self.pre_attn(i, h))
         k = F.linear(x, self.lw(i, "wk"), self.lw(i, "bk")).unflatten(-1, (c.n_kv_heads, c.head_dim))
         v = F.linear(x, self.lw(i, "wv"), self.lw(i, "bv")).unflatten(-1, (c.n_kv_heads, c.head_dim))
         if c.family == LLAMA:
             k = self.rope(k, pos)
-        return k, v
+        return self.r(k), self.r(v)
 
     def q(self, i, h, pos):
         c = self.c
-        x = self.pre_attn(i, h)
+        x = self.r(self.pre_attn(i, h))
         q = F.linear(x, self.lw(i, "wq"), self.lw(i, "bq")).unflatten(-1, (c.n_heads, c.head_dim))
         if c.family == LLAMA:
             q = self.rope(q, pos)
-        return q
+        return self.r(q)
 
     def after_attn(self, i, h, a):
         """Residual / FFN part of layer i given the attention output a [..., H*dh]."""
-        c = self.c
-        o = F.linear(a, self.lw(i, "wo"), self.lw(i, "bo"))
+        c, r = self.c, self.r
+        o = F.linear(r(a), self.lw(i, "wo"), self.lw(i, "bo"))
         if c.family == BERT:
             h1 = F.layer_norm(h + o, (c.d_model,), self.lw(i, "attn_norm.g"), self.lw(i, "attn_norm.b"), c.norm_eps)
-            f = F.linear(F.gelu(F.linear(h1, self.lw(i, "w_fc"), self.lw(i, "b_fc"))),
+            f = F.linear(r(F.gelu(F.linear(r(h1), self.lw(i, "w_fc"), self.lw(i, "b_fc")))),
                          self.lw(i, "w_proj"), self.lw(i, "b_proj"))
             return F.layer_norm(h1 + f, (c.d_model,), self.lw(i, "ffn_norm.g"), self.lw(i, "ffn_norm.b"), c.norm_eps)
         h1 = h + o
         if c.family == GPT2:
-            x = F.layer_norm(h1, (c.d_model,), self.lw(i, "ffn_norm.g"), self.lw(i, "ffn_norm.b"), c.norm_eps)
-            f = F.gelu(F.linear(x, self.lw(i, "w_fc"), self.lw(i, "b_fc")), approximate="tanh")
+            x = r(F.layer_norm(h1, (c.d_model,), self.lw(i, "ffn_norm.g"), self.lw(i, "ffn_norm.b"), c.norm_eps))
+            f = r(F.gelu(F.linear(x, self.lw(i, "w_fc"), self.lw(i, "b_fc")), approximate="tanh"))
             return h1 + F.linear(f, self.lw(i, "w_proj"), self.lw(i, "b_proj"))
-        x = F.rms_norm(h1, (c.d_model,), self.lw(i, "ffn_norm.g"), c.norm_eps)
-        f = F.silu(F.linear(x, self.lw(i, "w_gate"))) * F.linear(x, self.lw(i, "w_up"))
+        x = r(F.rms_norm(h1, (c.d_model,), self.lw(i, "ffn_norm.g"), c.norm_eps))
+        f = r(F.silu(F.linear(x, self.lw(i, "w_gate"))) * F.linear(x, self.lw(i, "w_up")))
         return h1 + F.linear(f, self.lw(i, "w_down"))
 
     def embed(self, tok, pos):
@@ -92,24 +103,25 @@ class TorchRef:
         c, W = self.c, self.W
         D, eps = c.d_model, c.hsm_eps
         X = torch.stack([F.rms_norm(t, (D,), W["hsm.g0"], eps) for t in (s_i, s_prev, inertia)], 0)
+        r = self.r
         c0 = F.conv2d(X[None, None], W["hsm.conv_w"][None, None], W["hsm.conv_b"], stride=1,
                       padding=(0, 1))[0, 0, 0]
-        h1 = F.gelu(F.linear(c0, W["hsm.fc1_w"], W["hsm.fc1_b"]))
-        h2 = F.gelu(F.linear(h1, W["hsm.fc2_w"], W["hsm.fc2_b"]))
-        h3 = F.linear(h2, W["hsm.fc3_w"], W["hsm.fc3_b"])
+        h1 = F.gelu(F.linear(r(c0), W["hsm.fc1_w"], W["hsm.fc1_b"]))
+        h2 = F.gelu(F.linear(r(h1), W["hsm.fc2_w"], W["hsm.fc2_b"]))
+        h3 = F.linear(r(h2), W["hsm.fc3_w"], W["hsm.fc3_b"])
         h4 = F.rms_norm(h3, (c.hsm_m1,), W["hsm.g1"], eps) + h1
-        h5 = F.linear(h4, W["hsm.fc4_w"], W["hsm.fc4_b"])
+        h5 = F.linear(r(h4), W["hsm.fc4_w"], W["hsm.fc4_b"])
         return F.rms_norm(h5, (D,), W["hsm.g2"], eps) + c0
 
     def head(self, x):
-        c, W = self.c, self.W
+        c, W, r = self.c, self.W, self.r
         if c.family == LLAMA:
-            return F.linear(F.rms_norm(x, (c.d_model,), W["final_norm.g"], c.norm_eps), W["lm_head"])
+            return F.linear(r(F.rms_norm(x, (c.d_model,), W["final_norm.g"], c.norm_eps)), W["lm_head"])
         if c.family == GPT2:
-            return F.linear(F.layer_norm(x, (c.d_model,), W["final_norm.g"], W["final_norm.b"], c.norm_eps),
+            return F.linear(r(F.layer_norm(x, (c.d_model,), W["final_norm.g"], W["final_norm.b"], c.norm_eps)),
                             W["tok_emb"])
-        pooled = torch.tanh(F.linear(x, W["pool.w"], W["pool.b"]))
-        return F.linear(pooled, W["cls.w"], W["cls.b"])
+        pooled = torch.tanh(F.linear(r(x), W["pool.w"], W["pool.b"]))
+        return F.linear(r(pooled), W["cls.w"], W["cls.b"])
 
     # ---------------------------------------------------------------- full depth, batched
     def full_forward(self, tokens):
