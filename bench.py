@@ -1,15 +1,21 @@
 #!/usr/bin/env python
 """Benchmark of the early-exit forward pass on one GB300 (N GPUs: independent replicas).
 
-Workload (one step): a GPT-2-small-shaped decoder in bf16 (12 layers, D=768, 12 heads,
-FFN 3072, vocab 50257, random-init N(0, 0.02)); a prompt pass over 8 x 512 uniform
-random token ids, then 128 greedy generation steps; each token's exit layer is forced
-from the integer-uniform law on [4, 12] (12 = full depth).  value = (prompt + generated
-tokens) / s over the timed steps, inputs resident in HBM, L2 flushed between steps.
+Workload (one step): a Llama-2-7B-shaped decoder in bf16 (32 layers, D=4096, 32 heads x 128,
+SwiGLU 11008, vocabulary 32000, the 36 D^2 mapper, random-init N(0, 0.02)); a prompt pass over
+one 2048-token prompt of uniform random ids, then 256 greedy generation steps; each token's
+exit layer is forced from a normal law N(24, 4) truncated to [8, 32] (32 = full depth), paged
+KV cache in 16-token blocks.  value = (prompt + generated tokens) / s over the timed steps,
+inputs resident in HBM, L2 flushed between steps (every step also streams ~13 GB of weights,
+far above L2).  e2e: the same steps through the C ABI with the inputs copied from pinned host
+memory and the exit layers and greedy tokens copied back inside the timed region.
 
-Also reported: the skipped-layer KV fill at Llama-7B layer shapes (32 layers,
-D=4096, 32 KV heads x 128) on a grid of exited-token counts and exit layers, against
-its roofline; and the CPU oracle on a bounded sample of the same workload.
+Also reported: the same library forced to full depth and with the identity mapper (the
+speed-up the exits buy against the algorithmic ratio); the skipped-layer KV fill at Llama-7B
+layer shapes on a grid of exited-token counts and exit layers, against its roofline; the
+GPT-2-small workload (8 x 512-token prompts + 128 steps, exits ~ U{4..12}), threshold
+calibration and the exit-rule variants on it; the BERT-base classification batch; the mapper
+training steps; and the CPU oracle on a bounded sample of the Llama workload.
 
 --impl reference times that oracle (the slow plain statement of the method) as the
 reference arm.
@@ -34,11 +40,14 @@ import torch  # noqa: E402
 import synth  # noqa: E402
 
 PEAKS_FALLBACK = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
-# DRAM bytes (read + write) per launch of a kernel class from one ncu capture of the
-# benchmark workload (profiles/launch_list_gpt2_small_generation_step.md); None once the
-# kernel has changed since the capture.
-NCU_TRAFFIC_PER_LAUNCH = {"gemm_decode": 6.38e6}
+# DRAM bytes (read + write) per launch of a kernel class from one ncu capture at the
+# workload's shapes, scaled to a launch of the workload (profiles/); None until a capture of
+# the current kernel exists.
+NCU_TRAFFIC_PER_LAUNCH = {}
 METRIC = "early-exit prefill+decode tokens/s at 1 GB300; skipped-layer KV-fill % of roofline"
+# Llama-7B headline workload: one prompt of LP tokens, LSTEPS greedy steps, exits ~ N(24, 4) on [8, 32]
+LP, LSTEPS, LMEAN, LSD, LLO, LHI = 2048, 256, 24.0, 4.0, 8, 32
+# GPT-2-small extra: B x P prompts, STEPS steps, exits ~ U{LO..HI}
 B, P, STEPS, LO, HI, DELTA = 8, 512, 128, 4, 12, 0.9
 L2_BYTES = 129 * 2 ** 20
 
@@ -196,17 +205,32 @@ class Clocks:
 # ----------------------------------------------------------------------------- our arm
 
 def make_inputs(cfg, device):
+    """GPT-2-small workload inputs: B x P prompt ids, prompt and generation-step exit layers."""
     tokens = synth.make_tokens(0, B, P, cfg.vocab).to(device)
     fp = synth.forced_exits_uniform(0, B * P, LO, HI, name="forced_prompt").view(B, P).to(device)
     fd = synth.forced_exits_uniform(0, STEPS * B, LO, HI, name="forced_decode").view(STEPS, B).to(device)
     return tokens, fp, fd
 
 
+def llama_cfg():
+    return synth.llama7b_config(max_batch=1, max_seq=LP + LSTEPS, max_pass_tokens=LP)
+
+
+def llama_inputs(cfg, device):
+    """Llama workload inputs: LP prompt ids, LP prompt and LSTEPS generation-step exit layers
+    ~ N(LMEAN, LSD) truncated to [LLO, LHI]."""
+    tok = synth.make_tokens(0, 1, LP, cfg.vocab).to(device)
+    fp = synth.forced_exits_truncnorm(0, LP, LMEAN, LSD, LLO, LHI, name="forced_prompt").view(1, LP).to(device)
+    fd = synth.forced_exits_truncnorm(0, LSTEPS, LMEAN, LSD, LLO, LHI, name="forced_decode").view(LSTEPS, 1).to(device)
+    return tok, fp, fd
+
+
 class Runner:
+    """The GPT-2-small workload: B x P prompt pass, then STEPS generation steps."""
+
     def __init__(self, adept, cfg, device):
         self.a = adept
         self.cfg = cfg
-        torch.manual_seed(0)
         W = synth.make_weights(cfg, seed=0, device=device)
         self.m = adept.Model(cfg, W)
         del W
@@ -217,14 +241,44 @@ class Runner:
         self.logits = torch.empty(B, cfg.vocab, dtype=torch.float32, device=device)
         self.nxt = torch.empty(STEPS + 1, B, dtype=torch.int32, device=device)
 
-    def step(self, tokens=None, fp=None, fd=None):
+    def step(self, delta=DELTA, threshold=False):
         a, h = self.a, self.m.h
-        tokens = self.tokens if tokens is None else tokens
-        fp = self.fp if fp is None else fp
-        fd = self.fd if fd is None else fd
-        a.adept_prefill(h, B, P, tokens.view(-1), DELTA, fp.view(-1), self.exit_p, self.logits, self.nxt[0], None)
+        a.adept_prefill(h, B, P, self.tokens.view(-1), delta, None if threshold else self.fp.view(-1), self.exit_p,
+                        self.logits, self.nxt[0], None)
         for s in range(STEPS):
-            a.adept_decode_step(h, B, self.nxt[s], DELTA, fd[s], self.exit_d[s], self.logits, self.nxt[s + 1], None)
+            a.adept_decode_step(h, B, self.nxt[s], delta, None if threshold else self.fd[s], self.exit_d[s],
+                                self.logits, self.nxt[s + 1], None)
+
+
+class LlamaRunner:
+    """The headline step at the Llama-2-7B shape: one LP-token prompt pass and LSTEPS greedy
+    generation steps through the C ABI."""
+
+    def __init__(self, adept, device):
+        self.a = adept
+        self.cfg = cfg = llama_cfg()
+        W = synth.make_weights(cfg, seed=0, device=device)
+        self.m = adept.Model(cfg, W)
+        del W
+        torch.cuda.empty_cache()
+        self.tok, self.fp, self.fd = llama_inputs(cfg, device)
+        self.exit_p = torch.empty(LP, dtype=torch.int32, device=device)
+        self.exit_d = torch.empty(LSTEPS, 1, dtype=torch.int32, device=device)
+        self.nxt = torch.empty(LSTEPS + 1, 1, dtype=torch.int32, device=device)
+
+    def prefill(self, tok=None, fp=None):
+        self.a.adept_prefill(self.m.h, 1, LP, (self.tok if tok is None else tok).view(-1), DELTA,
+                             (self.fp if fp is None else fp).view(-1), self.exit_p, None, self.nxt[0], None)
+
+    def decode(self, fd=None):
+        fd = self.fd if fd is None else fd
+        for s in range(LSTEPS):
+            self.a.adept_decode_step(self.m.h, 1, self.nxt[s], DELTA, fd[s], self.exit_d[s], None, self.nxt[s + 1],
+                                     None)
+
+    def step(self, tok=None, fp=None, fd=None):
+        self.prefill(tok, fp)
+        self.decode(fd)
 
 
 def run_fill_micro(adept, device, peaks, grid_T, grid_i, reps=3):
@@ -268,11 +322,16 @@ def run_fill_micro(adept, device, peaks, grid_T, grid_i, reps=3):
             fl, by = fill_micro_work(T, istar)
             t = float(np.median(ts)) / 1e3
             tk = kms / max(n, 1) / 1e3
-            roof = max(fl / (peaks["bf16_tflops"] * 1e12), by / (peaks["hbm_gbs"] * 1e9))
-            rows.append({"T": T, "exit_layer": istar, "ms": round(t * 1e3, 4), "gemm_ms": round(tk * 1e3, 4),
-                         "tflops": round(fl / t / 1e12, 2), "gbs": round(by / t / 1e9, 1),
-                         "roofline_ms": round(roof * 1e3, 4), "frac": round(roof / t, 4),
-                         "bound": "tensor" if fl / (peaks["bf16_tflops"] * 1e12) > by / (peaks["hbm_gbs"] * 1e9) else "hbm"})
+            t_f, t_b = fl / (peaks["bf16_tflops"] * 1e12), by / (peaks["hbm_gbs"] * 1e9)
+            roof = max(t_f, t_b)
+            row = {"T": T, "exit_layer": istar, "ms": round(t * 1e3, 4), "gemm_ms": round(tk * 1e3, 4),
+                   "tflops": round(fl / t / 1e12, 2), "gbs": round(by / t / 1e9, 1),
+                   "roofline_ms": round(roof * 1e3, 4), "frac": round(roof / t, 4),
+                   "bound": "tensor" if t_f > t_b else "hbm"}
+            if t_f > t_b:   # a long tensor-bound launch also against the sustained bf16 peak
+                roof_s = max(fl / (peaks["bf16_tflops_sustained"] * 1e12), t_b)
+                row["frac_of_sustained"] = round(roof_s / t, 4)
+            rows.append(row)
     m.close()
     del h_all
     torch.cuda.empty_cache()
@@ -290,10 +349,12 @@ def llama_work(cfg, exit_prompt, exit_decode, hsm: bool = True):
 
 
 def run_encoder(adept, device, B=64, P=128):
-    """BERT-base shape, bf16, random-init: 64 x 128-token classification batch, threshold
-    exits at delta = 0.9, forced exits ~ U{4..12}, and full depth; the default exit (deeper
-    K/V filled from s~) against the encoder's "stop entirely" variant (Sec. 4.3).
-    Throughput in sequences/s and tokens/s including the classifier."""
+    """BERT-base shape, bf16, random-init: 64 x 128-token classification batch.  Threshold
+    exits at delta = 0.9 (the configuration's threshold; with random-init weights every token
+    leaves at the first eligible layer there), at the delta that threshold calibration finds
+    for a 25 % reduction in computation on this batch, forced exits ~ U{4..12}, and full depth;
+    the default exit (deeper K/V filled from s~) against the encoder's "stop entirely" variant
+    (Sec. 4.3).  Throughput in sequences/s and tokens/s including the classifier."""
     cfg = synth.bert_base_config(max_batch=B, max_seq=P, max_pass_tokens=B * P)
     W = synth.make_weights(cfg, seed=0, device=device)
     m = adept.Model(cfg, W)
@@ -304,22 +365,26 @@ def run_encoder(adept, device, B=64, P=128):
     ex = torch.empty(B * P, dtype=torch.int32, device=device)
     lg = torch.empty(B, cfg.n_classes, device=device)
     st = torch.cuda.current_stream()
+    d_c, r_c, n_c = adept.adept_calibrate_threshold(m.h, B, P, tok.view(-1), 0.25, 0.01, 24)
     out = {}
-    for name, forced, stop in (("threshold_0.9", None, 0), ("forced_U4_12", fz, 0), ("forced_U4_12_stop_entirely", fz, 1),
-                               ("full_depth", full, 0)):
+    for name, forced, stop, delta in (("threshold_0.9", None, 0, 0.9), ("threshold_calibrated", None, 0, d_c),
+                                      ("forced_U4_12", fz, 0, 0.9), ("forced_U4_12_stop_entirely", fz, 1, 0.9),
+                                      ("full_depth", full, 0, 0.9)):
         adept.adept_set_option(m.h, adept.OPT_STOP_ENTIRELY, stop)
         ts = []
         for rep in range(4):
             e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
             torch.cuda.synchronize()
             e0.record(st)
-            adept.adept_prefill(m.h, B, P, tok.view(-1), 0.9, forced, ex, lg, None, None)
+            adept.adept_prefill(m.h, B, P, tok.view(-1), delta, forced, ex, lg, None, None)
             e1.record(st)
             torch.cuda.synchronize()
             ts.append(e0.elapsed_time(e1))
         t = float(np.median(ts[1:])) / 1e3
         out[name] = {"ms": round(t * 1e3, 3), "seq_s": round(B / t, 1), "tok_s": round(B * P / t, 1),
                      "mean_exit_depth": round(float(ex.double().mean().item()), 3)}
+        if name == "threshold_calibrated":
+            out[name].update(delta=round(d_c, 6), rdc=round(r_c, 4), calibration_passes=n_c)
     adept.adept_set_option(m.h, adept.OPT_STOP_ENTIRELY, 0)
     adept.adept_check_device_status(m.h)
     m.close()
@@ -408,60 +473,108 @@ def run_hsm_train(adept, device, peaks, n=8192, reps=5, shape="gpt2"):
             "loss_first": round(first_loss, 5), "loss_after": round(last_loss, 5)}
 
 
-def run_llama_e2e(adept, device, P=2048, steps=256):
-    """Llama-2-7B shape, batch 1: 2048-token prompt + 256 greedy decode steps, exit layer per
-    token ~ N(24, 4) truncated to [8, 32] -- against the same library forced to full depth, and
-    the same exits with the identity mapper in place of the HSM (s~ = s_i*: the speed-up the
-    exits and fills alone allow)."""
-    cfg = synth.llama7b_config(max_batch=1, max_seq=P + steps, max_pass_tokens=P)
-    W = synth.make_weights(cfg, seed=0, device=device)
-    m = adept.Model(cfg, W)
-    del W
-    torch.cuda.empty_cache()
-    tok = synth.make_tokens(0, 1, P, cfg.vocab).to(device)
-    fp = synth.forced_exits_truncnorm(0, P, 24.0, 4.0, 8, 32, name="forced_prompt").view(1, P).to(device)
-    fd = synth.forced_exits_truncnorm(0, steps, 24.0, 4.0, 8, 32, name="forced_decode").view(steps, 1).to(device)
-    full_p = torch.full_like(fp, cfg.n_layers)
-    full_d = torch.full_like(fd, cfg.n_layers)
-    nxt = torch.empty(steps + 1, 1, dtype=torch.int32, device=device)
-    exd = torch.empty(steps, 1, dtype=torch.int32, device=device)
-    exp_ = torch.empty(P, dtype=torch.int32, device=device)
-    st = torch.cuda.current_stream()
+def timed_prefill_decode(run, st, tok=None, fp=None, fd=None, reps=2):
+    """(prompt-pass ms, generation ms per step) of the last of `reps` runs of the Llama step
+    (the first warms up and captures the generation-step graph)."""
+    for _ in range(reps):
+        e0, e1, e2 = [torch.cuda.Event(enable_timing=True) for _ in range(3)]
+        torch.cuda.synchronize()
+        e0.record(st)
+        run.prefill(tok, fp)
+        e1.record(st)
+        run.decode(fd)
+        e2.record(st)
+        torch.cuda.synchronize()
+    return e0.elapsed_time(e1), e1.elapsed_time(e2) / LSTEPS
+
+
+def llama_arms(adept, run, st):
+    """The headline model against itself forced to full depth, and with the identity mapper in
+    place of the HSM (s~ = s_i*: the speed-up the exits and fills alone allow)."""
+    cfg = run.cfg
+    full_p = torch.full_like(run.fp, cfg.n_layers)
+    full_d = torch.full_like(run.fd, cfg.n_layers)
     out = {}
-    for name, a, b in (("early_exit", fp, fd), ("full_depth", full_p, full_d), ("hsm_identity", fp, fd)):
-        adept.adept_set_option(m.h, adept.OPT_HSM_IDENTITY, int(name == "hsm_identity"))
-        for rep in range(2):   # first run warms up (and captures the generation-step graph)
-            e0, e1, e2 = [torch.cuda.Event(enable_timing=True) for _ in range(3)]
-            torch.cuda.synchronize()
-            e0.record(st)
-            adept.adept_prefill(m.h, 1, P, tok.view(-1), 0.9, a.view(-1), exp_, None, nxt[0], None)
-            e1.record(st)
-            for s in range(steps):
-                adept.adept_decode_step(m.h, 1, nxt[s], 0.9, b[s], exd[s], None, nxt[s + 1], None)
-            e2.record(st)
-            torch.cuda.synchronize()
-        adept.adept_check_device_status(m.h)
-        tp, td = e0.elapsed_time(e1) / 1e3, e1.elapsed_time(e2) / 1e3
-        out[name] = {"prefill_tok_s": round(P / tp, 1), "decode_tok_s": round(steps / td, 2),
-                     "tok_s": round((P + steps) / (tp + td), 2), "prefill_ms": round(tp * 1e3, 3),
-                     "decode_ms_per_step": round(td * 1e3 / steps, 4),
-                     "mean_exit_depth": round(float(np.concatenate([exp_.cpu().numpy(),
-                                                                    exd.cpu().numpy().reshape(-1)]).mean()), 3),
-                     "algorithmic_tflop": round(llama_work(cfg, exp_.cpu().numpy(), exd.cpu().numpy(),
-                                                           hsm=name != "hsm_identity") / 1e12, 3)}
-    adept.adept_set_option(m.h, adept.OPT_HSM_IDENTITY, 0)
-    m.close()
-    torch.cuda.empty_cache()
+    for name, fp, fd in (("early_exit", run.fp, run.fd), ("full_depth", full_p, full_d), ("hsm_identity", run.fp, run.fd)):
+        adept.adept_set_option(run.m.h, adept.OPT_HSM_IDENTITY, int(name == "hsm_identity"))
+        tp, td = timed_prefill_decode(run, st, None, fp, fd)
+        adept.adept_check_device_status(run.m.h)
+        ep, ed = run.exit_p.cpu().numpy(), run.exit_d.cpu().numpy()
+        out[name] = {"prefill_tok_s": round(LP / tp * 1e3, 1), "decode_tok_s": round(1e3 / td, 2),
+                     "tok_s": round((LP + LSTEPS) / (tp + td * LSTEPS) * 1e3, 2), "prefill_ms": round(tp, 3),
+                     "decode_ms_per_step": round(td, 4),
+                     "mean_exit_depth": round(float(np.concatenate([ep, ed.reshape(-1)]).mean()), 3),
+                     "algorithmic_tflop": round(llama_work(cfg, ep, ed, hsm=name != "hsm_identity") / 1e12, 3)}
+    adept.adept_set_option(run.m.h, adept.OPT_HSM_IDENTITY, 0)
     ee, fd_, hi = out["early_exit"], out["full_depth"], out["hsm_identity"]
-    return {"workload": "Llama-2-7B shape, bf16, random-init; batch 1, 2048-token prompt + 256 greedy decode steps; "
-                        "exit layer per token ~ N(24,4) truncated to [8,32] vs all tokens forced to layer 32; "
-                        "the same exits with the identity mapper",
-            "early_exit": ee, "full_depth": fd_, "hsm_identity": hi,
+    return {"workload": "the headline workload vs all tokens forced to layer 32, and the same exits with the "
+                        "identity mapper",
+            **out,
             "speedup": round(ee["tok_s"] / fd_["tok_s"], 4),
+            "prefill_speedup": round(fd_["prefill_ms"] / ee["prefill_ms"], 4),
+            "decode_speedup": round(fd_["decode_ms_per_step"] / ee["decode_ms_per_step"], 4),
             "algorithmic_ratio": round(fd_["algorithmic_tflop"] / ee["algorithmic_tflop"], 4),
             "depth_ratio": round(fd_["mean_exit_depth"] / ee["mean_exit_depth"], 4),
             "speedup_hsm_identity": round(hi["tok_s"] / fd_["tok_s"], 4),
             "algorithmic_ratio_hsm_identity": round(fd_["algorithmic_tflop"] / hi["algorithmic_tflop"], 4)}
+
+
+def run_gpt2(adept, device, reps=3):
+    """GPT-2-small workload (B x P prompts + STEPS greedy steps) with forced exits ~ U{4..12}
+    and in threshold mode at delta 0.9, then threshold calibration to a 25 % reduction in
+    computation and the exit-rule variants at the calibrated delta (prompt passes)."""
+    cfg = workload_cfg()
+    run = Runner(adept, cfg, device)
+    st = torch.cuda.current_stream()
+    out = {"workload": "gpt2-small-shaped decoder, bf16, random-init N(0,0.02); batch 8 x 512-token uniform random "
+                       "prompts + 128 greedy decode steps"}
+    for name, thr in (("forced_U4_12", False), ("threshold_0.9", True)):
+        ts = []
+        for _ in range(reps):
+            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            torch.cuda.synchronize()
+            e0.record(st)
+            run.step(DELTA, thr)
+            e1.record(st)
+            torch.cuda.synchronize()
+            ts.append(e0.elapsed_time(e1))
+        adept.adept_check_device_status(run.m.h)
+        t = float(np.median(ts[1:])) / 1e3
+        out[name] = {"ms_per_step": round(t * 1e3, 3), "tok_s": round((B * P + B * STEPS) / t, 1),
+                     "prompt_mean_exit": round(float(run.exit_p.double().mean().item()), 3),
+                     "decode_mean_exit": round(float(run.exit_d.double().mean().item()), 3)}
+    # threshold calibration (Sec. 4.1, 5.1): bisection on delta to a 25 % reduction in computation
+    torch.cuda.synchronize()
+    t0 = time.perf_counter()
+    d_c, r_c, n_c = adept.adept_calibrate_threshold(run.m.h, B, P, run.tokens.view(-1), 0.25, 0.01, 24)
+    t_cal = (time.perf_counter() - t0) * 1e3
+    out["calibration"] = {"target_rdc": 0.25, "tol": 0.01, "delta": round(d_c, 6), "rdc": round(r_c, 4),
+                          "passes": n_c, "ms": round(t_cal, 3), "ms_per_pass": round(t_cal / max(n_c, 1), 3),
+                          "batch": f"{B} x {P} workload prompts, threshold exits"}
+    # exit-rule variants (App. H.2-H.3) at the calibrated threshold
+    variants = {}
+    ex_v = torch.empty(B * P, dtype=torch.int32, device=device)
+    nx_v = torch.empty(B, dtype=torch.int32, device=device)
+    for name, metric, aao in (("global", 0, 0), ("local", 1, 0), ("both", 2, 0), ("all_at_once", 0, 1)):
+        adept.adept_set_option(run.m.h, adept.OPT_EXIT_METRIC, metric)
+        adept.adept_set_option(run.m.h, adept.OPT_ALL_AT_ONCE, aao)
+        adept.adept_prefill(run.m.h, B, P, run.tokens.view(-1), d_c, None, ex_v, None, nx_v, None)
+        torch.cuda.synchronize()
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record(st)
+        adept.adept_prefill(run.m.h, B, P, run.tokens.view(-1), d_c, None, ex_v, None, nx_v, None)
+        e1.record(st)
+        torch.cuda.synchronize()
+        depth = ex_v.double().mean().item()
+        variants[name] = {"rdc": round(1.0 - depth / cfg.n_layers, 4), "prompt_ms": round(e0.elapsed_time(e1), 3)}
+    adept.adept_set_option(run.m.h, adept.OPT_EXIT_METRIC, 0)
+    adept.adept_set_option(run.m.h, adept.OPT_ALL_AT_ONCE, 0)
+    adept.adept_check_device_status(run.m.h)
+    out["exit_variants"] = {"delta": round(d_c, 6), "batch": f"{B} x {P} workload prompts", **variants}
+    run.m.close()
+    del run
+    torch.cuda.empty_cache()
+    return out
 
 
 def max_over_ranks(x: float, world: int, device) -> float:
@@ -479,6 +592,17 @@ def replica_throughput(units_per_rank_step: float, steps: int, world: int, secon
     return world * units_per_rank_step * steps / seconds
 
 
+def class_work(cfg, e_p, e_d):
+    """Algorithmic (flops, bytes) of one headline step per kernel class: the prompt pass's
+    GEMMs (one sequence), the generation steps' GEMMs (layers on the active token, mapper,
+    head) and their grouped skipped-layer fills."""
+    wd = [pass_work(cfg, e_d[s], decode=True) for s in range(len(e_d))]
+    wf = [decode_fill_work(cfg, e_d[s]) for s in range(len(e_d))]
+    return {"gemm_prefill": pass_work(cfg, e_p, decode=False, n_seq=1),
+            "gemm_decode": (sum(w[0] for w in wd), sum(w[1] for w in wd)),
+            "kv_fill_decode": (sum(w[0] for w in wf), sum(w[1] for w in wf))}
+
+
 def ours(args, rank, world, device):
     import paper_2601_03700_gb300 as adept
     if not os.path.exists(adept.LIB_PATH):
@@ -486,8 +610,8 @@ def ours(args, rank, world, device):
         _b.build()
     adept.load_library()
     peaks, peaks_src = load_peaks()
-    cfg = workload_cfg()
-    run = Runner(adept, cfg, device)
+    run = LlamaRunner(adept, device)
+    cfg = run.cfg
     flush = torch.empty(2 * L2_BYTES // 4, dtype=torch.float32, device=device)
     st = torch.cuda.current_stream()
     for _ in range(args.warmup):
@@ -514,31 +638,18 @@ def ours(args, rank, world, device):
     clk = clocks.stop() if clocks else None
     launches = adept.adept_launch_count(run.m.h)
     adept.adept_check_device_status(run.m.h)
-    # --------------------------------------------------------------- one profiled step (per-class device time)
-    # CUDA events on the launching stream around every GEMM / fill / attention launch;
-    # generation steps run as direct launches while profiling.
-    adept.adept_set_option(run.m.h, adept.OPT_PROFILE, 1)
-    for c in range(adept.PROF_DECODE_STEP + 1):
-        adept.adept_profile_read(run.m.h, c)
-    flush.zero_()
-    torch.cuda.synchronize()
-    run.step()
-    torch.cuda.synchronize()
-    prof = {c: adept.adept_profile_read(run.m.h, c) for c in range(adept.PROF_DECODE_STEP + 1)}
-    adept.adept_set_option(run.m.h, adept.OPT_PROFILE, 0)
-    adept.adept_check_device_status(run.m.h)
     total_ms = max_over_ranks(total_ms, world, device)
-    tok_per_step = B * P + B * STEPS
+    tok_per_step = LP + LSTEPS
     value = replica_throughput(tok_per_step, args.steps, world, total_ms / 1e3)
+    ms_per_step = total_ms / args.steps
     # --------------------------------------------------------------- end-to-end through the API with host buffers
-    tok_h = run.tokens.cpu().pin_memory()
-    fp_h = run.fp.cpu().pin_memory()
-    fd_h = run.fd.cpu().pin_memory()
-    out_h = torch.empty(STEPS + 1, B, dtype=torch.int32).pin_memory()
-    ex_h = torch.empty(B * P + STEPS * B, dtype=torch.int32).pin_memory()
-    tok_d, fp_d, fd_d = torch.empty_like(run.tokens), torch.empty_like(run.fp), torch.empty_like(run.fd)
+    tok_h, fp_h, fd_h = run.tok.cpu().pin_memory(), run.fp.cpu().pin_memory(), run.fd.cpu().pin_memory()
+    nxt_h = torch.empty(LSTEPS + 1, 1, dtype=torch.int32).pin_memory()
+    ex_h = torch.empty(LP + LSTEPS, dtype=torch.int32).pin_memory()
+    tok_d, fp_d, fd_d = torch.empty_like(run.tok), torch.empty_like(run.fp), torch.empty_like(run.fd)
     e2e_t = 0.0
-    for _ in range(max(1, args.steps)):
+    n_e2e = max(1, args.steps)
+    for _ in range(n_e2e):
         flush.zero_()
         torch.cuda.synchronize()
         t0 = time.perf_counter()
@@ -546,63 +657,74 @@ def ours(args, rank, world, device):
         fp_d.copy_(fp_h, non_blocking=True)
         fd_d.copy_(fd_h, non_blocking=True)
         run.step(tok_d, fp_d, fd_d)
-        out_h.copy_(run.nxt, non_blocking=True)
-        ex_h[:B * P].copy_(run.exit_p, non_blocking=True)
-        ex_h[B * P:].copy_(run.exit_d.view(-1), non_blocking=True)
+        nxt_h.copy_(run.nxt, non_blocking=True)
+        ex_h[:LP].copy_(run.exit_p, non_blocking=True)
+        ex_h[LP:].copy_(run.exit_d.view(-1), non_blocking=True)
         torch.cuda.synchronize()
         e2e_t += time.perf_counter() - t0
     e2e_t = max_over_ranks(e2e_t, world, device)
-    e2e = replica_throughput(tok_per_step, max(1, args.steps), world, e2e_t)
+    e2e = replica_throughput(tok_per_step, n_e2e, world, e2e_t)
     h2d = (tok_h.numel() + fp_h.numel() + fd_h.numel()) * 4
-    d2h = (out_h.numel() + ex_h.numel()) * 4
+    d2h = (nxt_h.numel() + ex_h.numel()) * 4
+    # --------------------------------------------------------------- one profiled step (per-class device time)
+    # CUDA events on the launching stream bracket every GEMM / fill / attention launch, so each
+    # bracketed kernel runs alone (it cannot overlap its neighbours as it does under
+    # programmatic dependent launch in the timed steps); generation steps run as direct
+    # launches while profiling.  Per-launch times are therefore a little pessimistic.
+    adept.adept_set_option(run.m.h, adept.OPT_PROFILE, 1)
+    for c in range(adept.PROF_GEMM_TRAIN + 1):
+        adept.adept_profile_read(run.m.h, c)
+    flush.zero_()
+    torch.cuda.synchronize()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record(st)
+    run.step()
+    e1.record(st)
+    torch.cuda.synchronize()
+    prof_step_ms = e0.elapsed_time(e1)
+    prof = {c: adept.adept_profile_read(run.m.h, c) for c in range(adept.PROF_GEMM_TRAIN + 1)}
+    adept.adept_set_option(run.m.h, adept.OPT_PROFILE, 0)
+    adept.adept_check_device_status(run.m.h)
     # --------------------------------------------------------------- dominant kernel roofline
     e_p = run.exit_p.cpu().numpy()
     e_d = run.exit_d.cpu().numpy()
-    wp = pass_work(cfg, e_p, decode=False)
-    wd = [pass_work(cfg, e_d[s], decode=True) for s in range(STEPS)]
-    wf = [decode_fill_work(cfg, e_d[s]) for s in range(STEPS)]
-    wa = [attention_decode_work(cfg, e_d[s], P + s + 1) for s in range(STEPS)]
-    work = {adept.PROF_GEMM_PREFILL: wp, adept.PROF_GEMM_DECODE: (sum(w[0] for w in wd), sum(w[1] for w in wd)),
-            adept.PROF_KV_FILL: (sum(w[0] for w in wf), sum(w[1] for w in wf)),
-            # the persistent generation step: every GEMM of the step, its fills and its attention
-            adept.PROF_DECODE_STEP: (sum(a[0] + b[0] + c[0] for a, b, c in zip(wd, wf, wa)),
-                                     sum(a[1] + b[1] + c[1] for a, b, c in zip(wd, wf, wa)))}
+    work = class_work(cfg, e_p, e_d)
     names = {adept.PROF_GEMM_PREFILL: "gemm_prefill", adept.PROF_GEMM_DECODE: "gemm_decode",
-             adept.PROF_KV_FILL: "kv_fill_decode", adept.PROF_ATTENTION: "attention",
-             adept.PROF_DECODE_STEP: "decode_step_fused"}
-    per_class = {}
-    for c, (n, ms, _, _) in prof.items():
-        per_class[names[c]] = {"launches": n, "ms_per_step": round(ms, 4)}
-    dom = max((c for c in work), key=lambda c: prof[c][1])
-    n, ms, _, _ = prof[dom]
+             adept.PROF_KV_FILL: "kv_fill_decode", adept.PROF_ATTENTION: "attention"}
+    per_class = {names[c]: {"launches": prof[c][0], "ms_per_step": round(prof[c][1], 4)} for c in names}
+    dom_c = max((c for c in names if names[c] in work), key=lambda c: prof[c][1])
+    dom = names[dom_c]
+    n, ms = prof[dom_c][0], prof[dom_c][1]
     fl, by = work[dom]
-    fl_s = fl
-    by_s = by
-    t_f = fl_s / (peaks["bf16_tflops"] * 1e12)
-    t_b = by_s / (peaks["hbm_gbs"] * 1e9)
+    t_f = fl / (peaks["bf16_tflops"] * 1e12)
+    t_b = by / (peaks["hbm_gbs"] * 1e9)
     if t_f >= t_b:
-        roof = {"bound": "tensor", "achieved": round(fl_s / (ms / 1e3) / 1e12, 3), "peak": peaks["bf16_tflops"],
+        roof = {"bound": "tensor", "achieved": round(fl / (ms / 1e3) / 1e12, 3), "peak": peaks["bf16_tflops"],
                 "unit": "TFLOP/s"}
     else:
-        roof = {"bound": "hbm", "achieved": round(by_s / (ms / 1e3) / 1e9, 2), "peak": peaks["hbm_gbs"],
-                "unit": "GB/s"}
+        roof = {"bound": "hbm", "achieved": round(by / (ms / 1e3) / 1e9, 2), "peak": peaks["hbm_gbs"], "unit": "GB/s"}
     roof["frac"] = round(roof["achieved"] / roof["peak"], 4)
-    tr = NCU_TRAFFIC_PER_LAUNCH.get(names[dom])
+    tr = NCU_TRAFFIC_PER_LAUNCH.get(dom)
     roof["traffic"] = round(tr) if tr else None
-    roof["kernel"] = names[dom]
+    roof["kernel"] = dom
     roof["launches"] = n
-    roof["peak_source"] = peaks_src + " (MEASURED_PEAKS.json burst)" if peaks_src == "measured" else peaks_src
-    roof["timing"] = "CUDA events around each launch of the class, one profiled step after the timed steps"
+    roof["peak_source"] = (peaks_src + " (MEASURED_PEAKS.json)") if peaks_src == "measured" else peaks_src
+    roof["timing"] = ("CUDA events bracketing each launch of the class in one profiled step after the timed steps "
+                      "(each bracketed launch runs alone)")
+    roof["class_ms_per_step"] = round(ms, 3)
+    roof["class_share_of_step"] = round(ms / ms_per_step, 4)
+    roof["profiled_step_ms"] = round(prof_step_ms, 3)
     roof["work_per_launch"] = {"flop": round(fl / max(n, 1)), "bytes": round(by / max(n, 1))}
     line = {
         "metric": METRIC, "value": round(value, 2), "unit": "tokens/s", "n_gpus": world, "steps": args.steps,
-        "warmup": args.warmup, "ms_per_step": round(total_ms / args.steps, 3), "higher_is_better": True,
+        "warmup": args.warmup, "ms_per_step": round(ms_per_step, 3), "higher_is_better": True,
         "scaling": "weak", "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
-        "config": {"workload": "gpt2-small-shaped decoder, bf16, random-init N(0,0.02); batch 8 x 512-token "
-                               "uniform random prompts + 128 greedy decode steps; forced exit layer per token "
-                               "~ U{4..12}", "model": "gpt2-small-shape", "global_batch": B * world,
-                   "seq_len": P, "decode_steps": STEPS, "parallelism": f"replicas{world}" if world > 1 else "single",
-                   "l2": "flushed between timed steps (256 MiB write)"},
+        "config": {"workload": "Llama-2-7B-shaped decoder, bf16, random-init N(0,0.02); batch 1, 2048-token uniform "
+                               "random prompt + 256 greedy decode steps; forced exit layer per token ~ N(24,4) "
+                               "truncated to [8,32]; paged KV cache, 16-token blocks",
+                   "model": "llama2-7b-shape", "global_batch": world, "seq_len": LP, "decode_steps": LSTEPS,
+                   "parallelism": f"replicas{world}" if world > 1 else "single",
+                   "l2": "flushed between timed steps (256 MiB write); each step streams ~13 GB of weights"},
         "e2e": {"value": round(e2e, 2), "unit": "tokens/s", "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h},
         "gpu_launches": int(launches),
         "roofline": roof,
@@ -610,36 +732,8 @@ def ours(args, rank, world, device):
         "exit_depth": {"prompt_mean": round(float(e_p.mean()), 3), "decode_mean": round(float(e_d.mean()), 3)},
         "clocks": clk,
     }
-    # --------------------------------------------------------------- threshold calibration (Sec. 4.1, 5.1)
-    # bisection on delta to a 25% reduction in computation over the workload's prompt batch
-    torch.cuda.synchronize()
-    t0 = time.perf_counter()
-    d_c, r_c, n_c = adept.adept_calibrate_threshold(run.m.h, B, P, run.tokens.view(-1), 0.25, 0.01, 24)
-    t_cal = (time.perf_counter() - t0) * 1e3
-    line["calibration"] = {"target_rdc": 0.25, "tol": 0.01, "delta": round(d_c, 6), "rdc": round(r_c, 4),
-                           "passes": n_c, "ms": round(t_cal, 3), "ms_per_pass": round(t_cal / max(n_c, 1), 3),
-                           "batch": f"{B} x {P} workload prompts, threshold exits"}
-    # --------------------------------------------------------------- exit-rule variants (App. H.2-H.3)
-    # the workload's prompt pass at the calibrated threshold: reduction and time per variant
-    variants = {}
-    ex_v = torch.empty(B * P, dtype=torch.int32, device=device)
-    nx_v = torch.empty(B, dtype=torch.int32, device=device)
-    for name, metric, aao in (("global", 0, 0), ("local", 1, 0), ("both", 2, 0), ("all_at_once", 0, 1)):
-        adept.adept_set_option(run.m.h, adept.OPT_EXIT_METRIC, metric)
-        adept.adept_set_option(run.m.h, adept.OPT_ALL_AT_ONCE, aao)
-        adept.adept_prefill(run.m.h, B, P, run.tokens.view(-1), d_c, None, ex_v, None, nx_v, None)
-        torch.cuda.synchronize()
-        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-        e0.record(st)
-        adept.adept_prefill(run.m.h, B, P, run.tokens.view(-1), d_c, None, ex_v, None, nx_v, None)
-        e1.record(st)
-        torch.cuda.synchronize()
-        depth = ex_v.double().mean().item()
-        variants[name] = {"rdc": round(1.0 - depth / cfg.n_layers, 4), "prompt_ms": round(e0.elapsed_time(e1), 3)}
-    adept.adept_set_option(run.m.h, adept.OPT_EXIT_METRIC, 0)
-    adept.adept_set_option(run.m.h, adept.OPT_ALL_AT_ONCE, 0)
-    adept.adept_check_device_status(run.m.h)
-    line["exit_variants"] = {"delta": round(d_c, 6), "batch": f"{B} x {P} workload prompts", **variants}
+    if rank == 0 and not args.no_llama:
+        line["llama7b_arms"] = llama_arms(adept, run, st)
     run.m.close()
     del run
     torch.cuda.empty_cache()
@@ -647,33 +741,82 @@ def ours(args, rank, world, device):
         grid_T = [int(x) for x in args.fill_T.split(",")]
         grid_i = [int(x) for x in args.fill_i.split(",")]
         rows = run_fill_micro(adept, device, peaks, grid_T, grid_i)
+        fr = [r["frac"] for r in rows]
         line["kv_fill"] = {"shape": "Llama-7B layers: 32 x (D=4096 -> K,V 2x4096), bf16, paged 16-token blocks",
-                           "peak": {"tflops": peaks["bf16_tflops"], "gbs": peaks["hbm_gbs"], "source": peaks_src},
-                           "grid": rows,
-                           "mean_frac": round(float(np.mean([r["frac"] for r in rows])), 4)}
+                           "peak": {"tflops": peaks["bf16_tflops"], "tflops_sustained": peaks["bf16_tflops_sustained"],
+                                    "gbs": peaks["hbm_gbs"], "source": peaks_src},
+                           "mean_frac": round(float(np.mean(fr)), 4), "min_frac": round(float(np.min(fr)), 4),
+                           "cells_below_0.6": int(sum(f < 0.6 for f in fr)), "grid": rows}
+        line["kv_fill_frac"] = {"mean": line["kv_fill"]["mean_frac"], "min": line["kv_fill"]["min_frac"],
+                                "cells": len(rows)}
     if rank == 0 and not args.no_llama:
-        line["llama7b_e2e"] = run_llama_e2e(adept, device)
+        line["gpt2_small"] = run_gpt2(adept, device)
         line["encoder"] = run_encoder(adept, device)
         line["hsm_train"] = run_hsm_train(adept, device, peaks)
         line["hsm_train_llama7b"] = run_hsm_train(adept, device, peaks, shape="llama7b", reps=3)
         line["hsm_train_bert"] = run_hsm_train(adept, device, peaks, shape="bert")
     if rank == 0 and not args.no_cpu_baseline:
-        line["cpu_baseline"] = cpu_baseline(args.cpu_tokens)
+        line["cpu_baseline"] = cpu_baseline(args.cpu_tokens, args.cpu_steps)
     return line
 
 
 # ----------------------------------------------------------------------------- oracle (CPU) arms
 
-def oracle_sample(n_seq: int, prompt: int, steps: int):
-    """Runs the oracle on a bounded sample of the workload: n_seq prompts of `prompt`
-    tokens and `steps` generation steps, same model, same exit law.  Returns
-    (tokens processed, seconds)."""
+def host_mem_available() -> int:
+    """MemAvailable of the host in bytes (0 when unknown)."""
+    try:
+        with open("/proc/meminfo") as f:
+            for ln in f:
+                if ln.startswith("MemAvailable:"):
+                    return int(ln.split()[1]) * 1024
+    except Exception:
+        pass
+    return 0
+
+
+# fp64 oracle copy of the Llama-7B-shaped model: 7.3e9 weights x 8 B
+ORACLE_LLAMA_BYTES = 59 * 2 ** 30
+
+
+class _WeightStream:
+    """The workload's weights as a mapping whose items() generates one tensor at a time (on
+    the GPU when there is one: the same values bit for bit), so the oracle's fp64 copy is the
+    only full copy of the model in host memory."""
+
+    def __init__(self, cfg):
+        self.cfg = cfg
+        self.dev = "cuda" if torch.cuda.is_available() else "cpu"
+
+    def items(self):
+        for name, shape in synth.weight_shapes(self.cfg).items():
+            yield name, synth.make_weight(self.cfg, name, shape, seed=0, device=self.dev).cpu()
+
+
+def oracle_llama_model():
+    """(cfg, oracle model) of the headline workload."""
     from oracle import adept_oracle as O
-    cfg = workload_cfg()
-    W = synth.make_weights(cfg, seed=0)
-    om = O.OracleModel(cfg, W)
-    del W
-    tokens, fp, fd = make_inputs(cfg, "cpu")
+    cfg = llama_cfg()
+    om = O.OracleModel(cfg, _WeightStream(cfg))
+    if torch.cuda.is_available():
+        torch.cuda.empty_cache()
+    return cfg, om
+
+
+def oracle_sample(n_seq: int, prompt: int, steps: int, model=None):
+    """Runs the oracle on a bounded sample of a workload: n_seq prompts of `prompt` tokens and
+    `steps` generation steps, same model, same exit law.  model = (cfg, oracle model) of the
+    Llama workload (prompt ids and exit layers are the workload's leading ones); None: the
+    GPT-2-small workload.  Returns (tokens processed, seconds)."""
+    from oracle import adept_oracle as O
+    if model is None:
+        cfg = workload_cfg()
+        W = synth.make_weights(cfg, seed=0)
+        om = O.OracleModel(cfg, W)
+        del W
+        tokens, fp, fd = make_inputs(cfg, "cpu")
+    else:
+        cfg, om = model
+        tokens, fp, fd = llama_inputs(cfg, "cpu")
     tk = tokens[:n_seq, :prompt].numpy()
     f = fp[:n_seq, :prompt].numpy()
     cache = O.OracleCache(cfg, n_seq, prompt + steps + 1)
@@ -694,19 +837,37 @@ def cores():
         return os.cpu_count() or 1
 
 
-def cpu_baseline(n_tokens: int):
-    n_seq, prompt, steps = 4, n_tokens, 8
-    tok, dt = oracle_sample(n_seq, prompt, steps)
-    out = {"value": round(tok / dt, 3), "unit": "tokens/s", "cores": cores(), "kind": "oracle",
-           "sample": f"{n_seq} prompt x {prompt} tokens + {steps} decode steps of the same model and exit law "
-                     f"(fp64 NumPy oracle, {dt:.1f} s)"}
+def llama_oracle_fits() -> bool:
+    return host_mem_available() >= 1.4 * ORACLE_LLAMA_BYTES
+
+
+def cpu_baseline(prompt: int, steps: int):
+    """The oracle on the host cores, on a bounded sample of the headline workload (the Llama
+    model with the workload's first `prompt` prompt tokens and `steps` generation steps).  Where
+    the host cannot hold the oracle's fp64 copy of that model, the GPT-2-small workload stands in
+    (said in `sample`)."""
+    if llama_oracle_fits():
+        t0 = time.perf_counter()
+        model = oracle_llama_model()
+        t_build = time.perf_counter() - t0
+        tok, dt = oracle_sample(1, prompt, steps, model)
+        out = {"value": round(tok / dt, 3), "unit": "tokens/s", "cores": cores(), "kind": "oracle",
+               "sample": f"Llama-2-7B-shaped model of the workload, its first {prompt} prompt tokens + {steps} "
+                         f"generation steps, same exit law (fp64 NumPy oracle, {dt:.1f} s; model build "
+                         f"{t_build:.0f} s untimed)"}
+        del model
+    else:
+        tok, dt = oracle_sample(4, 512, 8)
+        out = {"value": round(tok / dt, 3), "unit": "tokens/s", "cores": cores(), "kind": "oracle",
+               "sample": f"host memory below the fp64 Llama-7B oracle's ~75 GB: GPT-2-small workload instead, "
+                         f"4 prompts x 512 tokens + 8 generation steps ({dt:.1f} s)"}
     out["single_core"] = oracle_single_core(1, 128, 8)
     return out
 
 
 def oracle_single_core(n_seq: int, prompt: int, steps: int):
-    """The same oracle on one host core: a fresh interpreter with every BLAS / OpenMP pool
-    limited to one thread, on a smaller bounded sample."""
+    """The oracle on one host core (GPT-2-small workload): a fresh interpreter with every BLAS /
+    OpenMP pool limited to one thread, on a smaller bounded sample."""
     env = dict(os.environ)
     for k in ("OMP_NUM_THREADS", "OPENBLAS_NUM_THREADS", "MKL_NUM_THREADS", "BLIS_NUM_THREADS"):
         env[k] = "1"
@@ -718,27 +879,37 @@ def oracle_single_core(n_seq: int, prompt: int, steps: int):
     except Exception as e:   # reported, not fatal: the all-core figure stands
         return {"unavailable": f"{type(e).__name__}: {e}"[:200]}
     return {"value": round(d["tokens"] / d["seconds"], 3), "unit": "tokens/s", "cores": 1,
-            "sample": f"{n_seq} prompt x {prompt} tokens + {steps} decode steps ({d['seconds']:.1f} s)"}
+            "sample": f"GPT-2-small workload, {n_seq} prompt x {prompt} tokens + {steps} decode steps "
+                      f"({d['seconds']:.1f} s)"}
 
 
 def reference_arm(args, rank, world):
+    """The oracle as the reference arm: each step a bounded sample of the headline workload
+    (its first --ref-prompt prompt tokens and --ref-steps generation steps on the Llama model;
+    the GPT-2-small workload where the host cannot hold the fp64 Llama model)."""
     if rank != 0:
         return None
-    tot_tok, tot_s = 0, 0.0
+    llama = llama_oracle_fits()
+    model = oracle_llama_model() if llama else None
+    prompt, steps = (args.ref_prompt, args.ref_steps) if llama else (args.cpu_tokens, 8)
     for _ in range(args.warmup):
-        oracle_sample(1, 32, 1)
+        oracle_sample(1, 16, 1, model)
+    tot_tok, tot_s = 0, 0.0
     for _ in range(args.steps):
-        tok, dt = oracle_sample(1, args.cpu_tokens, 8)
+        tok, dt = oracle_sample(1, prompt, steps, model)
         tot_tok += tok
         tot_s += dt
     v = tot_tok / tot_s
+    what = (f"Llama-2-7B-shaped workload (same model and exit law), bounded sample: its first {prompt} prompt tokens "
+            f"+ {steps} generation steps per step") if llama else \
+        (f"host memory below the fp64 Llama oracle's need: GPT-2-small workload, 1 prompt x {prompt} tokens + "
+         f"{steps} generation steps per step")
     return {"metric": METRIC, "value": round(v, 3), "unit": "tokens/s", "n_gpus": world, "steps": args.steps,
             "warmup": args.warmup, "ms_per_step": round(tot_s / args.steps * 1e3, 3), "higher_is_better": True,
             "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic", "impl": "reference",
-            "config": {"workload": "gpt2-small-shaped decoder (same model and exit law), bounded sample: "
-                                   f"1 prompt x {args.cpu_tokens} tokens + 8 decode steps per step"},
+            "config": {"workload": what},
             "cpu_baseline": {"value": round(v, 3), "unit": "tokens/s", "cores": cores(), "kind": "oracle",
-                             "sample": f"1 prompt x {args.cpu_tokens} + 8 decode steps per step"},
+                             "sample": what},
             "e2e": {"value": round(v, 3), "unit": "tokens/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
 
 
@@ -877,9 +1048,12 @@ def main():
     ap.add_argument("--no-kv-fill", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-llama", action="store_true")
-    ap.add_argument("--fill-T", default="1,16,256,1024,4096,16384,65536")
+    ap.add_argument("--fill-T", default="1,4,16,64,256,1024,4096,16384,65536")
     ap.add_argument("--fill-i", default="4,8,16,24")
-    ap.add_argument("--cpu-tokens", type=int, default=512)
+    ap.add_argument("--cpu-tokens", type=int, default=256, help="prompt tokens of the CPU-baseline oracle sample")
+    ap.add_argument("--cpu-steps", type=int, default=8, help="generation steps of the CPU-baseline oracle sample")
+    ap.add_argument("--ref-prompt", type=int, default=64, help="prompt tokens per step of --impl reference")
+    ap.add_argument("--ref-steps", type=int, default=2, help="generation steps per step of --impl reference")
     ap.add_argument("--hsm-n", type=int, default=8192, help="examples per step of --kernel-case hsm_train")
     ap.add_argument("--hsm-shape", default="gpt2", choices=["gpt2", "llama7b", "bert"],
                     help="model shape of --kernel-case hsm_train")
