@@ -6,6 +6,7 @@
 #include "kernels.h"
 #include "gemm_tc.h"
 #include "gemm_decode.h"
+#include "gemm_stream.h"
 #include "model_view.h"
 #include "hsm_train.h"
 
@@ -124,6 +125,10 @@ struct adept_model {
   int32_t* calib_exit = nullptr; // threshold calibration: exit layers of a calibration pass
   // standardisation statistics of X_out handed from the O projection to the FFN input
   float2* tile_stats = nullptr;                // [DG_MAX_M][D / 32] (mean, M2) of X_out tiles
+  // stream-K weight-streaming GEMM workspace (bf16 models): partial tiles and arrival counters
+  float* ds_part = nullptr;
+  int* ds_cnt = nullptr;
+  int ds_ctas = 0;
   float* amax_v = nullptr;       // argmax partials
   int* amax_i = nullptr;
   float* scratch = nullptr;
@@ -140,7 +145,7 @@ struct adept_model {
   std::vector<cudaGraphExec_t> dec_graph;   // per batch size
   std::vector<int> dec_warm;                // direct runs done per batch size
   // options / instrumentation
-  int hsm_identity = 0, profile = 0, force_simt = 0, use_graph = 1, use_dg = 1;
+  int hsm_identity = 0, profile = 0, force_simt = 0, use_graph = 1, use_dg = 1, use_stream = 1;
   int exit_metric = 0;   // EXIT_GLOBAL / EXIT_LOCAL / EXIT_BOTH
   int all_at_once = 0;   // prompt passes: sequences leave with their last prompt token
   int stop_entirely = 0; // encoders: exited tokens get no deeper K/V and leave deeper attention
@@ -297,12 +302,34 @@ static bool dg_takes(const adept_model* m, int n_probs, const GemmProblem& p, in
          decode_gemm_supported(p, max_rows, norm);
 }
 
+static DsWork ds_work(const adept_model* m) {
+  DsWork w;
+  w.part = m->use_stream ? m->ds_part : nullptr;
+  w.part_ctas = m->ds_ctas;
+  w.cnt = m->ds_cnt;
+  w.cnt_cap = DS_CNT_CAP;
+  return w;
+}
+
+// A weight-streaming problem of at most DG_MAX_M rows: the stream-K kernel where it takes the
+// shape (weights large enough to stream, A rows fitting in shared memory), else the cluster
+// K-split kernel.  Returns the launches, or -1 when neither takes it.
+static int streaming_gemm(adept_model* m, cudaStream_t st, const GemmProblem& p, int max_rows, const DgNorm* norm) {
+  if (stream_gemm(st, p, max_rows, norm, ds_work(m), m->err_word) >= 0) return 1;
+  return decode_gemm(st, p, max_rows, norm, m->err_word);
+}
+
+// The grouped skipped-layer fill of a few tokens on the weight-streaming kernels.
+static int streaming_gemm_grouped(adept_model* m, cudaStream_t st, const GemmProblem* probs, int n, int max_rows) {
+  if (stream_gemm_grouped(st, probs, n, max_rows, ds_work(m), m->err_word) >= 0) return 1;
+  return max_rows <= DG_FILL_MAX_ROWS ? decode_gemm_grouped(st, probs, n, max_rows, m->err_word) : -1;
+}
+
 static void gemm(adept_model* m, cudaStream_t st, const GemmProblem* probs, int n_probs, const int* max_rows,
                  int cls, double flops = 0, double bytes = 0) {
   cudaEvent_t b = nullptr;
   prof_begin(m, cls, st, &b);
-  if (dg_takes(m, n_probs, probs[0], max_rows[0], nullptr) &&
-      decode_gemm(st, probs[0], max_rows[0], nullptr, m->err_word) >= 0) {
+  if (dg_takes(m, n_probs, probs[0], max_rows[0], nullptr) && streaming_gemm(m, st, probs[0], max_rows[0], nullptr) >= 0) {
     m->launches += 1;
     prof_end(m, cls, st, b, flops, bytes);
     return;
@@ -340,7 +367,7 @@ static void gemm_std(adept_model* m, cudaStream_t st, const GemmProblem& p, int 
   if (dg_takes(m, 1, p, max_rows, &nrm)) {
     cudaEvent_t b = nullptr;
     prof_begin(m, cls, st, &b);
-    if (decode_gemm(st, p, max_rows, &nrm, m->err_word) >= 0) {
+    if (streaming_gemm(m, st, p, max_rows, &nrm) >= 0) {
       m->launches += 1;
       prof_end(m, cls, st, b, 0, 0);
       return;
@@ -669,6 +696,15 @@ static adept_status alloc_runtime(adept_model* m) {
   TRY(dalloc_t(m, &m->attn_ws, (size_t)c.max_batch * m->H * ATTN_MAX_SPLIT * (m->dh + 2)));
   TRY(dalloc_t(m, &m->attn_ctr, (size_t)c.max_batch * m->H));
   TRY(dalloc_t(m, &m->tile_stats, (size_t)DG_MAX_M * (m->D / 32 + 1)));
+  if (m->dt == ADEPT_DTYPE_BF16) {
+    int dev = 0, sms = 0;
+    CUDA_TRY(m, cudaGetDevice(&dev));
+    CUDA_TRY(m, cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev));
+    m->ds_ctas = std::max(sms, 1);
+    TRY(dalloc(m, (void**)&m->ds_part, stream_gemm_part_bytes(m->ds_ctas)));
+    TRY(dalloc_t(m, &m->ds_cnt, DS_CNT_CAP));
+    CUDA_TRY(m, cudaMemset(m->ds_cnt, 0, sizeof(int) * DS_CNT_CAP));
+  }
   CUDA_TRY(m, cudaMemset(m->attn_ctr, 0, sizeof(int) * c.max_batch * m->H));
   TRY(dalloc_t(m, &m->d_delta, 1));
   TRY(dalloc_t(m, &m->amax_v, (size_t)c.max_batch * 32));
@@ -954,10 +990,10 @@ static adept_status run_pass(adept_model* m, int n_tok, int batch, int prompt_le
     // one weight-streaming launch over the skipped layers when the rows fit it, else the
     // grouped tcgen05 GEMM
     bool done = false;
-    if (m->dt == ADEPT_DTYPE_BF16 && m->use_dg && !m->force_simt && n_tok <= DG_FILL_MAX_ROWS) {
+    if (m->dt == ADEPT_DTYPE_BF16 && m->use_dg && !m->force_simt && n_tok <= DG_MAX_M) {
       cudaEvent_t b = nullptr;
       prof_begin(m, ADEPT_PROF_KV_FILL, st, &b);
-      done = decode_gemm_grouped(st, probs.data(), (int)probs.size(), n_tok, m->err_word) >= 0;
+      done = streaming_gemm_grouped(m, st, probs.data(), (int)probs.size(), n_tok) >= 0;
       prof_end(m, ADEPT_PROF_KV_FILL, st, b, 0, 0);
       if (done) m->launches += 1;
     }
@@ -1578,10 +1614,10 @@ adept_status adept_skip_kv_fill(adept_model* m, int n_tokens, const void* d_h_ma
   // algorithmic work of this launch is only known on the device; the benchmark supplies it.
   // A few tokens: one weight-streaming launch over the layers; else the grouped tcgen05 GEMM.
   bool done = false;
-  if (m->dt == ADEPT_DTYPE_BF16 && m->use_dg && !m->force_simt && n_tokens <= DG_FILL_MAX_ROWS) {
+  if (m->dt == ADEPT_DTYPE_BF16 && m->use_dg && !m->force_simt && n_tokens <= DG_MAX_M) {
     cudaEvent_t b = nullptr;
     prof_begin(m, ADEPT_PROF_KV_FILL, st, &b);
-    done = decode_gemm_grouped(st, probs.data(), (int)probs.size(), n_tokens, m->err_word) >= 0;
+    done = streaming_gemm_grouped(m, st, probs.data(), (int)probs.size(), n_tokens) >= 0;
     prof_end(m, ADEPT_PROF_KV_FILL, st, b, 0, 0);
     if (done) m->launches += 1;
   }
@@ -1628,6 +1664,8 @@ adept_status adept_check_device_status(adept_model* m, void* stream) {
   CUDA_TRY(m, cudaMemcpy(&w, m->err_word, sizeof w, cudaMemcpyDeviceToHost));
   CUDA_TRY(m, cudaMemset(m->err_word, 0, sizeof(unsigned)));
   if (w & ERRW_TIMEOUT) {
+    // a launch that gave up may have left arrival counters of the stream-K GEMM counted
+    if (m->ds_cnt) CUDA_TRY(m, cudaMemset(m->ds_cnt, 0, sizeof(int) * DS_CNT_CAP));
     return fail(m, ADEPT_ERR_TIMEOUT, "a device-side wait timed out (word 0x%x)", w);
   }
   if (w) return fail(m, ADEPT_ERR_DEVICE_INPUT, "device-side input check failed (word 0x%x)", w);
@@ -1642,6 +1680,7 @@ adept_status adept_set_option(adept_model* m, int option, int value) {
     case ADEPT_OPT_GEMM_SIMT: m->force_simt = value != 0; drop_graphs(m); return ADEPT_OK;
     case ADEPT_OPT_DECODE_GRAPH: m->use_graph = value != 0; drop_graphs(m); return ADEPT_OK;
     case ADEPT_OPT_DECODE_GEMM: m->use_dg = value != 0; drop_graphs(m); return ADEPT_OK;
+    case ADEPT_OPT_DECODE_STREAM: m->use_stream = value != 0; drop_graphs(m); return ADEPT_OK;
     case ADEPT_OPT_EXIT_METRIC:
       if (value < EXIT_GLOBAL || value > EXIT_BOTH) return fail(m, ADEPT_ERR_INVALID_ARG, "exit metric %d", value);
       m->exit_metric = value;

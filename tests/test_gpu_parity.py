@@ -218,7 +218,6 @@ def test_decode_graph_replay_equals_direct_launches():
     outs = []
     for graph in (0, 1):
         m = adept.Model(cfg, W)
-        adept.adept_set_option(m.h, adept.OPT_FUSED_DECODE, 0)   # the multi-launch step is the one captured
         adept.adept_set_option(m.h, adept.OPT_DECODE_GRAPH, graph)
         tokens = synth.make_tokens(21, 3, 40, cfg.vocab).cuda()
         ex, lg, nx, _ = m.prefill(tokens, 0.5, synth.forced_exits_uniform(21, 120, 2, 6).view(3, 40).cuda())
