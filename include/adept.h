@@ -335,6 +335,22 @@ ADEPT_API adept_status adept_hsm_train_read(adept_model* m, int what, int param,
 /* Element count of HSM parameter `param` (0..12), or -1. */
 ADEPT_API int64_t adept_hsm_param_numel(const adept_model* m, int param);
 
+/* ---- failure injection (tests of the error paths; no GPU fault is involved) ------------
+ * adept_set_wait_limit: limit, in SM cycles, of the kernels' bounded waits on pipeline
+ * progress (a ring slot being filled or released, an accumulator becoming ready) in the
+ * tensor-core, weight-streaming and stream-K GEMMs; 0 restores the default (4e9 cycles, about
+ * 2 s).  A wait that runs out sets the device error word, its CTA stops, lets the copies it
+ * has in flight land (those waits, and the waits of cross-CTA reductions, keep their own long
+ * limits), frees its tensor memory and exits, and adept_check_device_status then returns
+ * ADEPT_ERR_TIMEOUT; the outputs of that call are undefined and the model stays usable.
+ * Applies to every model of the process on the current device.  Errors: INVALID_ARG
+ * (cycles < 0), CUDA.
+ * adept_set_alloc_fail_after: after n more device allocations by the library, every further
+ * allocation fails as if the device were out of memory (n < 0: off, the default); calls that
+ * need memory then return ADEPT_ERR_OOM with everything they allocated released. */
+ADEPT_API adept_status adept_set_wait_limit(int64_t cycles);
+ADEPT_API void adept_set_alloc_fail_after(int64_t n);
+
 /* Number of kernel launches the library enqueued since the last call (then reset). */
 ADEPT_API int64_t adept_launch_count(adept_model* m);
 

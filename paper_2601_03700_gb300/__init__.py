@@ -35,7 +35,7 @@ ABI_SYMBOLS = [
     "adept_read_final_states", "adept_check_device_status", "adept_set_option", "adept_profile_read",
     "adept_launch_count", "adept_skip_kv_fill_noalloc",
     "adept_calibrate_threshold", "adept_hsm_train_init", "adept_hsm_train_step", "adept_hsm_train_read",
-    "adept_hsm_param_numel", "adept_hsm_train_step_cls",
+    "adept_hsm_param_numel", "adept_hsm_train_step_cls", "adept_set_wait_limit", "adept_set_alloc_fail_after",
 ]
 
 
@@ -118,6 +118,10 @@ def load_library(path: str = LIB_PATH):
     lib.adept_hsm_train_step_cls.restype = c_int
     lib.adept_hsm_train_read.argtypes = [vp, c_int, c_int, fp, ctypes.c_int64, st]
     lib.adept_hsm_train_read.restype = c_int
+    lib.adept_set_wait_limit.argtypes = [ctypes.c_int64]
+    lib.adept_set_wait_limit.restype = c_int
+    lib.adept_set_alloc_fail_after.argtypes = [ctypes.c_int64]
+    lib.adept_set_alloc_fail_after.restype = None
     lib.adept_hsm_param_numel.argtypes = [vp, c_int]
     lib.adept_hsm_param_numel.restype = ctypes.c_int64
     for name in ABI_SYMBOLS:
@@ -325,6 +329,15 @@ def adept_profile_read(m, cls: int):
 
 def adept_launch_count(m) -> int:
     return int(load_library().adept_launch_count(m))
+
+
+def adept_set_wait_limit(cycles: int):
+    lib = load_library()
+    _check(lib, None, lib.adept_set_wait_limit(int(cycles)))
+
+
+def adept_set_alloc_fail_after(n: int):
+    load_library().adept_set_alloc_fail_after(int(n))
 
 
 # ---------------------------------------------------------------------------

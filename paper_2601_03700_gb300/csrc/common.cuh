@@ -123,7 +123,24 @@ struct KtScope {
   KT_WAITED();               \
   pdl_launch_dependents()
 
+// Limit of the library's bounded waits on pipeline progress (a ring slot filling or being
+// released, an accumulator becoming ready), in SM cycles; adept_set_wait_limit changes it.
+// Each translation unit holds its own copy, set through its set_wait_limit_* function.  The
+// waits that let a CTA's copies in flight land before it exits, and the waits of a cluster's
+// reduction, keep fixed limits: they must outlast any peer's shortened wait.
+constexpr long long WAIT_LIMIT_DEFAULT = 4000000000LL;   // ~2 s at 2 GHz
+static __device__ long long g_wait_limit = WAIT_LIMIT_DEFAULT;
+__device__ __forceinline__ long long wait_limit() { return *(volatile const long long*)&g_wait_limit; }
+#define ADEPT_WAIT_LIMIT_SETTER(unit)                                               \
+  cudaError_t set_wait_limit_##unit(long long cycles) {                              \
+    return cudaMemcpyToSymbol(g_wait_limit, &cycles, sizeof cycles);                \
+  }
+
 namespace adept {
+cudaError_t set_wait_limit_tc(long long cycles);
+cudaError_t set_wait_limit_dg(long long cycles);
+cudaError_t set_wait_limit_ds(long long cycles);
+
 // Launches with the programmatic-serialisation attribute while g_pdl is set (each entry
 // point sets it for its calling thread; it is off while per-launch profiling events are
 // recorded, so each timed interval holds one kernel alone).

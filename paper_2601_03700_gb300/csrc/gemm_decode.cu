@@ -17,9 +17,10 @@
 //    statistics of all rows are reduced in one pass of the block over the full rows.
 //  * MMA: mma.sync m16n8k16 bf16 with the weight features as the m16 operand and the
 //    tokens as the n8 operand, so a generation step of 8 sequences fills it unpadded.
-//  * Every mbarrier wait is bounded; on time-out the CTA records ERRW_TIMEOUT, stops
-//    issuing, waits (bounded) for its copies in flight and still takes part in the
-//    cluster barriers, so its cluster always completes.
+//  * Every mbarrier wait is bounded (the ring wait by the runtime wait limit, the drain of
+//    copies in flight and the cluster reduction by fixed, longer limits); on time-out the CTA
+//    records ERRW_TIMEOUT, stops issuing, waits for its copies in flight and still takes part
+//    in the cluster barriers, so its cluster always completes.
 #define ADEPT_TU_ID 5
 #include "gemm_decode.h"
 #include "epilogue.cuh"
@@ -531,7 +532,7 @@ __global__ void __launch_bounds__(DG_THREADS, 1) gemm_decode_kernel(const __grid
 #ifdef ADEPT_KTRACE
       const unsigned long long tw = kt_now();
 #endif
-      const bool ok = dg_wait(&full[s], (uint32_t)((g / S) & 1), p.err, DG_TIMEOUT_CYCLES);
+      const bool ok = dg_wait(&full[s], (uint32_t)((g / S) & 1), p.err, wait_limit());
 #ifdef ADEPT_KTRACE
       KT_ADD(7, kt_now() - tw);
 #endif
@@ -911,5 +912,7 @@ int decode_gemm_grouped(cudaStream_t st, const GemmProblem* probs, int n, int ma
 }
 
 ADEPT_KTRACE_ATTACH(dg)
+
+ADEPT_WAIT_LIMIT_SETTER(dg)
 
 }  // namespace adept

@@ -26,8 +26,9 @@
 //    counter; the CTA that sees the final count sums the partials in contributor order (the
 //    same sum every run), applies the fused epilogue and resets the counter.  No CTA waits for
 //    another.
-//  * Every mbarrier wait is bounded; on time-out the CTA records ERRW_TIMEOUT, stops, and
-//    waits (bounded) for its copies in flight before it exits.
+//  * Every mbarrier wait is bounded (ring waits by the runtime wait limit, the drain of copies
+//    in flight by a fixed, longer one); on time-out the CTA records ERRW_TIMEOUT, stops, and
+//    waits for its copies in flight before it exits.
 #define ADEPT_TU_ID 8
 #include "gemm_stream.h"
 #include "epilogue.cuh"
@@ -51,7 +52,7 @@ constexpr int DS_MAX_STAGES = 12;
 constexpr int DS_PRE = 3;                         // units issued before the dependency wait
 constexpr int DS_RP = DS_BN + 1;                  // floats per token row of a partial tile
 constexpr int DS_MAXG = 32;
-constexpr int DS_COHOST_SMEM = 112 * 1024;        // two launches' CTAs fit on one SM
+constexpr int DS_COHOST_SMEM = 113 * 1024;        // two launches' CTAs fit on one SM (228 KB, 1 KB each reserved)
 constexpr int DS_SMEM_LIMIT = 200 * 1024;
 constexpr long long DS_TIMEOUT_CYCLES = 4000000000LL;   // ~2 s at 2 GHz
 constexpr long long DS_MIN_STREAM_BYTES = 8ll << 20;    // below: the cluster K-split kernel
@@ -106,11 +107,13 @@ __device__ __forceinline__ bool mbar_try_wait(uint64_t* bar, uint32_t parity) {
       : "memory");
   return ok != 0;
 }
-__device__ __forceinline__ bool ds_wait(uint64_t* bar, uint32_t parity, unsigned* err) {
+// Bounded wait: `limit` is the runtime wait limit for pipeline progress, DS_TIMEOUT_CYCLES for
+// the drain of copies in flight.
+__device__ __forceinline__ bool ds_wait(uint64_t* bar, uint32_t parity, unsigned* err, long long limit) {
   if (mbar_try_wait(bar, parity)) return true;
   const long long t0 = clock64();
   while (!mbar_try_wait(bar, parity)) {
-    if (clock64() - t0 > DS_TIMEOUT_CYCLES) {
+    if (clock64() - t0 > limit) {
       atomicOr(err, ERRW_TIMEOUT);
       return false;
     }
@@ -161,7 +164,7 @@ __device__ __forceinline__ long long ds_owner(long long u, long long U, long lon
 // cw, cw + DS_NC, ..., lane = feature.
 template <int KIND>
 __device__ __forceinline__ void ds_epilogue(const Epi& e, const float* sS, int M, int rb, int f0, int N, int cw,
-                                            int lane) {
+                                            int lane, const int* s_pos, const int* s_blk) {
   for (int row = cw; row < M; row += DS_NC) {
     const int ra = rb + row, c = f0 + lane;
     const bool valid = c < N;
@@ -188,7 +191,14 @@ __device__ __forceinline__ void ds_epilogue(const Epi& e, const float* sS, int M
       const float u = __shfl_down_sync(0xffffffffu, v, 16);
       if (lane < 16) ((bf16*)e.out_t)[(size_t)ra * e.ld_t + (f0 >> 1) + lane] = __float2bfloat16_rn(silu_f(v) * u);
     } else {   // EPI_QKV / EPI_KV: q -> out_t, k / v -> the row's cache slot; RoPE pairs adjacent
-      const EpiRow rr = epi_row(e, ra);
+      const KVCacheView& cv = e.cache;
+      const int pos = s_pos[row], blk = s_blk[row];
+      EpiRow rr;
+      rr.pos = blk < 0 ? 0 : pos;   // an invalid position (flagged by the pass) reads a valid table row
+      rr.cbase = blk < 0 ? -1
+                         : (long long)((((size_t)e.layer0 * cv.n_blocks + blk) * cv.n_kv_heads) * cv.block_tokens +
+                                       (pos % cv.block_tokens)) *
+                               cv.head_dim;
       const int dh = e.head_dim, half = dh >> 1, nq = e.n_q_cols, nkv = e.n_kv_cols;
       const int base = c < nq ? 0 : c < nq + nkv ? nq : nq + nkv;
       const int hd = (c - base) / dh, d = (c - base) - hd * dh;
@@ -336,6 +346,7 @@ __global__ void __launch_bounds__(DS_THREADS, 1) gemm_stream_kernel(const __grid
   __shared__ int s_live[MAXG];     // problems with rows, in order
   __shared__ int s_M[MAXG], s_rb[MAXG];
   __shared__ int s_nlive, s_last;
+  __shared__ int s_pos[16], s_blk[16];   // cache epilogues: each row's position and cache block
 
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   uint8_t* smem = ds_smem_raw + ((1024 - (smem_u32(ds_smem_raw) & 1023)) & 1023);
@@ -360,13 +371,31 @@ __global__ void __launch_bounds__(DS_THREADS, 1) gemm_stream_kernel(const __grid
   __syncthreads();
   pdl_launch_dependents();
 
-  // unit u -> (problem slot li in the live list, tile t, k-block kb)
-  auto issue = [&](long long u, int g, int q) {
-    const long long li = u / per_prob, rem = u - li * per_prob;
-    const int t = (int)(rem / p.nkb), kb = (int)(rem - (long long)t * p.nkb);
-    const int s = g % S;
+  // Unit cursor: (live-problem slot li, tile t, k-block kb) of a unit, advanced one unit at a
+  // time, so that the loops carry no integer divisions.
+  struct Cur {
+    int li, t, kb;
+  };
+  auto cur_at = [&](long long u) {
+    Cur r;
+    r.li = (int)(u / per_prob);
+    const long long rem = u - (long long)r.li * per_prob;
+    r.t = (int)(rem / p.nkb);
+    r.kb = (int)(rem - (long long)r.t * p.nkb);
+    return r;
+  };
+  auto advance = [&](Cur& r) {
+    if (++r.kb == p.nkb) {
+      r.kb = 0;
+      if (++r.t == p.tiles) {
+        r.t = 0;
+        ++r.li;
+      }
+    }
+  };
+  auto issue = [&](const Cur& r, int q, int s) {
     mbar_expect_tx(&full[s], (uint32_t)DS_STAGE);
-    tma_load_3d(&p.wmap[q], &full[s], sW + (size_t)s * DS_STAGE, t * DS_BN, kb * (DS_KB / 64));
+    tma_load_3d(&p.wmap[q], &full[s], sW + (size_t)s * DS_STAGE, r.t * DS_BN, r.kb * (DS_KB / 64));
   };
 
   // single problem: the partition is known before the wait; its first units are issued
@@ -379,7 +408,11 @@ __global__ void __launch_bounds__(DS_THREADS, 1) gemm_stream_kernel(const __grid
     const long long avail = u1 - u0;
     pre = S < DS_PRE ? S : DS_PRE;
     if ((long long)pre > avail) pre = (int)avail;
-    for (int g = 0; g < pre; ++g) issue(u0 + g, g, 0);
+    Cur r = cur_at(u0);
+    for (int g = 0; g < pre; ++g) {
+      issue(r, 0, g);
+      advance(r);
+    }
   }
 
   pdl_wait();   // from here on, the preceding kernels' writes are visible
@@ -412,7 +445,7 @@ __global__ void __launch_bounds__(DS_THREADS, 1) gemm_stream_kernel(const __grid
     // no rows (every token of the step has left), or no units for this CTA: let the copies
     // in flight land, leave
     if (warp == 0 && lane == 0)
-      for (int g = 0; g < pre; ++g) ds_wait(&full[g], 0, p.err);
+      for (int g = 0; g < pre; ++g) ds_wait(&full[g], 0, p.err, DS_TIMEOUT_CYCLES);
     return;
   }
   const int n_units = (int)(u1 - u0);
@@ -422,6 +455,23 @@ __global__ void __launch_bounds__(DS_THREADS, 1) gemm_stream_kernel(const __grid
   int Ms = 0;
   for (int k = 0; k < nlive; ++k) Ms = max(Ms, s_M[s_live[k]]);
   const int rb0 = s_rb[s_live[0]];
+  if (KIND == EPI_QKV || KIND == EPI_KV) {
+    // each row's position and cache block, looked up once (every problem of the launch holds
+    // the same tokens in the same rows)
+    const Epi& e0 = p.epi[s_live[0]];
+    if (tid < Ms) {
+      const int tok = e0.row_tok[rb0 + tid];
+      const int pos = e0.tok_pos[tok], seq = e0.tok_seq[tok];
+      const KVCacheView& cv = e0.cache;
+      int blk = -1;
+      if (seq >= 0 && seq < cv.max_batch && pos >= 0 && pos < cv.max_blocks_per_seq * cv.block_tokens) {
+        blk = cv.block_table[seq * cv.max_blocks_per_seq + pos / cv.block_tokens];
+        if (blk < 0 || blk >= cv.n_blocks) blk = -1;
+      }
+      s_pos[tid] = pos;
+      s_blk[tid] = blk;
+    }
+  }
   ds_stage_a(p, sA, rb0, Ms, s_mu, s_rs, s_red);
   KT_MARK(1);
 
@@ -430,18 +480,28 @@ __global__ void __launch_bounds__(DS_THREADS, 1) gemm_stream_kernel(const __grid
     if (lane == 0) {
       bool ok = true;
       int issued = pre;
+      Cur r = cur_at(u0 + pre);
+      int s = pre, n = 0;   // slot and use number of unit g
+      if (s == S) {
+        s = 0;
+        n = 1;
+      }
       for (int g = pre; g < n_units && ok; ++g) {
-        const int s = g % S;
-        if (g >= S) ok = ds_wait(&empty[s], (uint32_t)(((g / S) - 1) & 1), p.err);
+        if (n >= 1) ok = ds_wait(&empty[s], (uint32_t)((n - 1) & 1), p.err, wait_limit());
         if (ok) {
-          const long long u = u0 + g;
-          issue(u, g, s_live[u / per_prob]);
+          issue(r, s_live[r.li], s);
           issued = g + 1;
+          advance(r);
+          if (++s == S) {
+            s = 0;
+            ++n;
+          }
         }
       }
       // before leaving, every copy this CTA issued has landed (bounded waits; immediate when
       // the consumers have taken them)
-      for (int h = max(0, issued - S); h < issued; ++h) ds_wait(&full[h % S], (uint32_t)((h / S) & 1), p.err);
+      for (int h = max(0, issued - S); h < issued; ++h)
+        ds_wait(&full[h % S], (uint32_t)((h / S) & 1), p.err, DS_TIMEOUT_CYCLES);
     }
     return;
   }
@@ -456,6 +516,7 @@ __global__ void __launch_bounds__(DS_THREADS, 1) gemm_stream_kernel(const __grid
                           kh * 128;
   const int bg = lane >> 2;
   const uint32_t b_base = smem_u32(sA) + (bg * ap + kh * 64 + (lane & 3) * 2) * 2;
+  const int ct = tid - 32;   // 0..127 among the consumers
 
   float acc[MB][4];
   auto zero_acc = [&]() {
@@ -463,12 +524,12 @@ __global__ void __launch_bounds__(DS_THREADS, 1) gemm_stream_kernel(const __grid
     for (int t = 0; t < MB; ++t) acc[t][0] = acc[t][1] = acc[t][2] = acc[t][3] = 0.f;
   };
   zero_acc();
-  const long long first_gt = u0 / p.nkb;   // this CTA's first (live-enumerated) tile
+  Cur r = cur_at(u0);
+  const long long gt_first = (long long)r.li * p.tiles + r.t;   // this CTA's first (live-enumerated) tile
 
-  // the tile that ends at unit u (inclusive) of a segment that began at unit useg
-  auto finish_tile = [&](long long useg, long long u) -> bool {
-    const long long gt = u / p.nkb;                 // live-enumerated global tile
-    const int li = (int)(gt / p.tiles), t = (int)(gt - (long long)li * p.tiles);
+  // the tile (li, t) ends here; whole: this CTA covered all of its k-blocks
+  auto finish_tile = [&](int li, int t, bool whole) {
+    const long long gt = (long long)li * p.tiles + t;
     const int q = s_live[li];
     const int M = s_M[q], rb = s_rb[q];
     const Epi& e = p.epi[q];
@@ -487,58 +548,58 @@ __global__ void __launch_bounds__(DS_THREADS, 1) gemm_stream_kernel(const __grid
     }
     zero_acc();
     consumers_sync();
-    const int ct = tid - 32;   // 0..127
     for (int i = ct; i < M * DS_BN; i += DS_NC * 32) {
       const int j = (i >> 5) * DS_RP + (i & 31);
       sS[j] = sP[j] + sP[16 * DS_RP + j];
     }
     consumers_sync();
-    const bool whole = useg == gt * p.nkb && u == gt * p.nkb + p.nkb - 1;
     if (!whole) {
       // shared tile: publish this CTA's partial, count the arrival; the last one finishes it
-      const long long slot = 2 * c + (gt == first_gt ? 0 : 1);
+      const long long slot = 2 * c + (gt == gt_first ? 0 : 1);
       float* mine = p.part + slot * (16 * DS_BN);
       for (int i = ct; i < M * DS_BN; i += DS_NC * 32) mine[i] = sS[(i >> 5) * DS_RP + (i & 31)];
       __threadfence();
       consumers_sync();
+      const long long c_first = ds_owner(gt * p.nkb, U, G), c_last = ds_owner(gt * p.nkb + p.nkb - 1, U, G);
       if (ct == 0) {
-        const long long c_first = ds_owner(gt * p.nkb, U, G), c_last = ds_owner(gt * p.nkb + p.nkb - 1, U, G);
-        const int n_contrib = (int)(c_last - c_first + 1);
         const int old = atomicAdd(&p.cnt[(long long)q * p.tiles + t], 1);
-        s_last = old == n_contrib - 1;
+        s_last = old == (int)(c_last - c_first);
       }
       consumers_sync();
-      if (!s_last) return true;
+      if (!s_last) return;
       __threadfence();
-      // sum the contributors' partials in contributor order
-      const long long c_first = ds_owner(gt * p.nkb, U, G), c_last = ds_owner(gt * p.nkb + p.nkb - 1, U, G);
-      for (int i = ct; i < M * DS_BN; i += DS_NC * 32) {
-        float v = 0.f;
-        for (long long cc = c_first; cc <= c_last; ++cc) {
-          const long long sl = 2 * cc + (gt == ds_start(cc, U, G) / p.nkb ? 0 : 1);
-          v += __ldcg(p.part + sl * (16 * DS_BN) + i);
+      // the contributors' partials summed in contributor order (each thread at most 4 values)
+      float v[4] = {0.f, 0.f, 0.f, 0.f};
+      for (long long cc = c_first; cc <= c_last; ++cc) {
+        const long long sl = 2 * cc + (gt == ds_start(cc, U, G) / p.nkb ? 0 : 1);
+        const float* src = p.part + sl * (16 * DS_BN);
+#pragma unroll
+        for (int k = 0; k < 4; ++k) {
+          const int i = ct + k * DS_NC * 32;
+          if (i < M * DS_BN) v[k] += __ldcg(src + i);
         }
-        sS[(i >> 5) * DS_RP + (i & 31)] = v;
+      }
+#pragma unroll
+      for (int k = 0; k < 4; ++k) {
+        const int i = ct + k * DS_NC * 32;
+        if (i < M * DS_BN) sS[(i >> 5) * DS_RP + (i & 31)] = v[k];
       }
       if (ct == 0) p.cnt[(long long)q * p.tiles + t] = 0;
       consumers_sync();
     }
-    ds_epilogue<KIND>(e, sS, M, rb, t * DS_BN, p.N, cw, lane);
+    ds_epilogue<KIND>(e, sS, M, rb, t * DS_BN, p.N, cw, lane, s_pos, s_blk);
     consumers_sync();   // sP / sS are rewritten by the next tile
-    return true;
   };
 
   // A warp whose wait gives up stops waiting and computing but still releases its slots and
   // takes part in every consumer barrier, so the CTA always completes (the error word is set).
-  long long useg = u0;
   bool ok = true;
+  bool seg_whole_start = r.kb == 0;   // the current tile's segment began at its first k-block
+  int Mq = s_M[s_live[r.li]];
+  int s = 0, n = 0;                   // slot and use number of unit g
   for (int g = 0; g < n_units; ++g) {
-    const long long u = u0 + g;
-    const int s = g % S;
-    const long long rem = u % per_prob;
-    const int kb = (int)(rem % p.nkb);
-    const int Mq = s_M[s_live[u / per_prob]];
-    if (ok) ok = ds_wait(&full[s], (uint32_t)((g / S) & 1), p.err);
+    if (ok) ok = ds_wait(&full[s], (uint32_t)(n & 1), p.err, wait_limit());
+    const int kb = r.kb;
     const int nch = ok ? min(DS_KB, p.K - kb * DS_KB) >> 6 : 0;
     const uint32_t sbase = w_base + s * DS_STAGE;
     for (int q = 0; 2 * q + kh < nch; ++q) {
@@ -567,11 +628,18 @@ __global__ void __launch_bounds__(DS_THREADS, 1) gemm_stream_kernel(const __grid
     }
     __syncwarp();
     if (lane == 0) mbar_arrive(&empty[s]);
+    const bool last = g == n_units - 1;
     // tile boundary or the end of the range: finish the tile
-    if (kb == p.nkb - 1 || g == n_units - 1) {
-      finish_tile(useg, u);
-      useg = u + 1;
+    if (kb == p.nkb - 1 || last) {
+      finish_tile(r.li, r.t, seg_whole_start && kb == p.nkb - 1);
+      seg_whole_start = true;
     }
+    advance(r);
+    if (++s == S) {
+      s = 0;
+      ++n;
+    }
+    if (r.kb == 0 && !last) Mq = s_M[s_live[r.li]];
   }
   KT_MARK(6);
 }
@@ -642,7 +710,7 @@ bool ds_plan(const GemmProblem& q, int n_probs, int max_rows, const DgNorm* norm
   const int a_bytes = ((arows * apitch * 2) + 127) & ~127;
   const int p_bytes = 3 * 16 * DS_RP * 4;
   const int fixed = 1024 + a_bytes + p_bytes;
-  const int STATIC = 2 * DS_MAX_STAGES * 8 + 64 * 4 + (DS_NC + 1) * 64 + 3 * MAXG * 4 + 64;
+  const int STATIC = 2 * DS_MAX_STAGES * 8 + 64 * 4 + (DS_NC + 1) * 64 + 3 * MAXG * 4 + 64 + 128;
   int stages = (DS_COHOST_SMEM - STATIC - fixed) / DS_STAGE;
   if (stages < 4) stages = (DS_SMEM_LIMIT - STATIC - fixed) / DS_STAGE;
   if (stages < 2) return false;
@@ -725,5 +793,7 @@ int stream_gemm_grouped(cudaStream_t st, const GemmProblem* probs, int n, int ma
                                 : ds_launch<1, EPI_KV, DS_MAXG>(st, prm, grid, smem);
   return e == cudaSuccess ? 1 : -1;
 }
+
+ADEPT_WAIT_LIMIT_SETTER(ds)
 
 }  // namespace adept

@@ -72,14 +72,15 @@ __device__ __forceinline__ bool mbar_try_wait(uint64_t* bar, uint32_t parity) {
       : "memory");
   return ok != 0;
 }
-// Bounded wait for the phase of `parity`; false on time-out or when another role aborted.
+// Bounded wait (the runtime wait limit) for the phase of `parity`; false on time-out or when
+// another role aborted.  The drains below keep the fixed TC_TIMEOUT_CYCLES.
 __device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, volatile int* abort_flag, unsigned* err) {
   if (mbar_try_wait(bar, parity)) return true;
-  const long long t0 = clock64();
+  const long long t0 = clock64(), lim = wait_limit();
   while (true) {
     if (mbar_try_wait(bar, parity)) return true;
     if (*abort_flag) return false;
-    if (clock64() - t0 > TC_TIMEOUT_CYCLES) {
+    if (clock64() - t0 > lim) {
       atomicOr(err, ERRW_TIMEOUT);
       *abort_flag = 1;
       return false;
@@ -892,6 +893,8 @@ int tc_gemm_grouped_nocache(cudaStream_t st, const GemmProblem* probs, int n_pro
 }
 
 ADEPT_KTRACE_ATTACH(tc)
+
+ADEPT_WAIT_LIMIT_SETTER(tc)
 
 }  // namespace adept
 

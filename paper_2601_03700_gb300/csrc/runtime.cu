@@ -11,6 +11,7 @@
 #include "hsm_train.h"
 
 #include <algorithm>
+#include <atomic>
 #include <cmath>
 #include <cstdarg>
 #include <cstdio>
@@ -157,6 +158,7 @@ struct adept_model {
   int gemm_cls = ADEPT_PROF_GEMM_PREFILL;
   int last_rows = 0;
   int64_t launches = 0;
+  adept_status deferred = ADEPT_OK;   // an error met inside a launch sequence, reported by check_launch
   int64_t graph_launches = 0;   // kernels in one captured generation step
   ProfRec prof[ADEPT_PROF_NCLASS];
 };
@@ -181,9 +183,17 @@ static adept_status fail(adept_model* m, adept_status s, const char* fmt, ...) {
     if (e_ != cudaSuccess) return fail(m, ADEPT_ERR_CUDA, "%s failed: %s", #call, cudaGetErrorString(e_)); \
   } while (0)
 
+// Allocation-failure hook (adept_set_alloc_fail_after): allocations left before every device
+// allocation of the library fails; negative: off.
+static std::atomic<long long> g_alloc_budget{-1};
+
 static adept_status dalloc(adept_model* m, void** p, size_t bytes) {
   *p = nullptr;
   if (bytes == 0) return ADEPT_OK;
+  for (long long b = g_alloc_budget.load(); b >= 0;) {
+    if (b == 0) return fail(m, ADEPT_ERR_OOM, "cudaMalloc(%zu) refused by the allocation-failure hook", bytes);
+    if (g_alloc_budget.compare_exchange_weak(b, b - 1)) break;
+  }
   cudaError_t e = cudaMalloc(p, bytes);
   if (e != cudaSuccess) {
     cudaGetLastError();
@@ -347,7 +357,10 @@ static void gemm(adept_model* m, cudaStream_t st, const GemmProblem* probs, int 
     for (int i = 0; i < n_probs; ++i) {
       if (!ensure_scratch(m, (size_t)max_rows[i] * probs[i].N)) {
         cudaStreamSynchronize(st);
-        if (!ensure_scratch(m, (size_t)max_rows[i] * probs[i].N)) continue;  // error already recorded
+        if (!ensure_scratch(m, (size_t)max_rows[i] * probs[i].N)) {   // the call returns OOM
+          m->deferred = ADEPT_ERR_OOM;
+          continue;
+        }
       }
       launch_gemm_simt(st, m->dt, probs[i], max_rows[i], m->scratch);
       m->launches += 2;
@@ -624,8 +637,10 @@ static adept_status alloc_runtime(adept_model* m) {
   // RoPE table (cos, sin) per position and pair, evaluated in double once.
   if (c.family == ADEPT_FAMILY_LLAMA) {
     const int half = m->dh / 2;
-    std::vector<float2> tab((size_t)c.max_seq * half);
-    for (int p = 0; p < c.max_seq; ++p)
+    // every position a reserved KV block can hold (max_seq rounded up to whole blocks)
+    const int rope_rows = cdiv(c.max_seq, c.kv_block_tokens) * c.kv_block_tokens;
+    std::vector<float2> tab((size_t)rope_rows * half);
+    for (int p = 0; p < rope_rows; ++p)
       for (int i = 0; i < half; ++i) {
         const double inv = std::pow((double)c.rope_theta, -2.0 * i / m->dh);
         const double a = p * inv;
@@ -1041,7 +1056,9 @@ static adept_status run_head(adept_model* m, int batch, int prompt_len, bool dec
 static adept_status check_launch(adept_model* m) {
   cudaError_t e = cudaGetLastError();
   if (e != cudaSuccess) return fail(m, ADEPT_ERR_CUDA, "kernel launch failed: %s", cudaGetErrorString(e));
-  return ADEPT_OK;
+  const adept_status d = m->deferred;
+  m->deferred = ADEPT_OK;
+  return d;   // the message was recorded where the error was met
 }
 
 // ---------------------------------------------------------------------------
@@ -1592,6 +1609,7 @@ adept_status adept_skip_kv_fill(adept_model* m, int n_tokens, const void* d_h_ma
     }
     m->fill_x = nullptr;
     m->fill_tok = nullptr;
+    m->fill_cap = 0;   // until both buffers of the new capacity exist
     int cap = std::max(n_tokens, 1024);
     TRY(dalloc(m, &m->fill_x, (size_t)cap * m->D * m->esz));
     TRY(dalloc_t(m, &m->fill_tok, cap));
@@ -1671,6 +1689,16 @@ adept_status adept_check_device_status(adept_model* m, void* stream) {
   if (w) return fail(m, ADEPT_ERR_DEVICE_INPUT, "device-side input check failed (word 0x%x)", w);
   return ADEPT_OK;
 }
+
+adept_status adept_set_wait_limit(int64_t cycles) {
+  if (cycles < 0) return fail(nullptr, ADEPT_ERR_INVALID_ARG, "wait limit %lld < 0", (long long)cycles);
+  const long long v = cycles == 0 ? WAIT_LIMIT_DEFAULT : (long long)cycles;
+  for (cudaError_t e : {set_wait_limit_tc(v), set_wait_limit_dg(v), set_wait_limit_ds(v)})
+    if (e != cudaSuccess) return fail(nullptr, ADEPT_ERR_CUDA, "setting the wait limit: %s", cudaGetErrorString(e));
+  return ADEPT_OK;
+}
+
+void adept_set_alloc_fail_after(int64_t n) { g_alloc_budget.store(n < 0 ? -1 : (long long)n); }
 
 adept_status adept_set_option(adept_model* m, int option, int value) {
   if (!m) return ADEPT_ERR_INVALID_ARG;
