@@ -130,7 +130,8 @@ struct KtScope {
 // reduction, keep fixed limits: they must outlast any peer's shortened wait.
 constexpr long long WAIT_LIMIT_DEFAULT = 4000000000LL;   // ~2 s at 2 GHz
 static __device__ long long g_wait_limit = WAIT_LIMIT_DEFAULT;
-__device__ __forceinline__ long long wait_limit() { return *(volatile const long long*)&g_wait_limit; }
+// Read once per CTA at kernel entry (a global load; the waits then compare against a register).
+__device__ __forceinline__ long long wait_limit() { return g_wait_limit; }
 #define ADEPT_WAIT_LIMIT_SETTER(unit)                                               \
   cudaError_t set_wait_limit_##unit(long long cycles) {                              \
     return cudaMemcpyToSymbol(g_wait_limit, &cycles, sizeof cycles);                \

@@ -225,6 +225,7 @@ __global__ void __launch_bounds__(DG_THREADS, 1) gemm_decode_kernel(const __grid
   __shared__ float s_red[DG_THREADS / 32][MB * 8];
   __shared__ float s_mu[MB * 8], s_rs[MB * 8];
 
+  const long long wlim = wait_limit();   // the runtime wait limit, read once
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   // tiles tile0, tile0 + tstride, ... of one K-split (several only when splits == 1)
   const int tile0 = blockIdx.x / p.splits, split = blockIdx.x - tile0 * p.splits;
@@ -532,7 +533,11 @@ __global__ void __launch_bounds__(DG_THREADS, 1) gemm_decode_kernel(const __grid
 #ifdef ADEPT_KTRACE
       const unsigned long long tw = kt_now();
 #endif
-      const bool ok = dg_wait(&full[s], (uint32_t)((g / S) & 1), p.err, wait_limit());
+      // lane 0 waits and broadcasts: the MMAs below are .aligned, so the warp decides as one
+      bool ok = true;
+      if (lane == 0) ok = dg_wait(&full[s], (uint32_t)((g / S) & 1), p.err, wlim);
+      ok = __shfl_sync(0xffffffffu, ok ? 1 : 0, 0) != 0;
+      __syncwarp();
 #ifdef ADEPT_KTRACE
       KT_ADD(7, kt_now() - tw);
 #endif

@@ -46,16 +46,18 @@ constexpr int DS_BN = 32;                         // output features per tile
 constexpr int DS_KB = 256;                        // k per unit
 constexpr int DS_CHUNK = DS_BN * 128;             // one [32 rows][64 k] 128-byte-swizzled chunk
 constexpr int DS_STAGE = DS_BN * DS_KB * 2;       // 16 KB per unit
-constexpr int DS_NC = 4;                          // consumer warps
-constexpr int DS_THREADS = 32 * (DS_NC + 1);      // + the producer warp
+constexpr int DS_NC = 4;                          // MMA (consumer) warps
+constexpr int DS_NE = 2;                          // epilogue warps
+constexpr int DS_WARPS = 1 + DS_NC + DS_NE;       // + the producer warp
+constexpr int DS_THREADS = 32 * DS_WARPS;
 constexpr int DS_MAX_STAGES = 12;
-constexpr int DS_PRE = 3;                         // units issued before the dependency wait
 constexpr int DS_RP = DS_BN + 1;                  // floats per token row of a partial tile
 constexpr int DS_MAXG = 32;
 constexpr int DS_COHOST_SMEM = 113 * 1024;        // two launches' CTAs fit on one SM (228 KB, 1 KB each reserved)
 constexpr int DS_SMEM_LIMIT = 200 * 1024;
 constexpr long long DS_TIMEOUT_CYCLES = 4000000000LL;   // ~2 s at 2 GHz
 constexpr long long DS_MIN_STREAM_BYTES = 8ll << 20;    // below: the cluster K-split kernel
+constexpr int DS_MIN_N = 8192;                           // single problems narrower: the cluster kernel
 enum : int { DS_STATS_HERE = 0, DS_STATS_ROWS = 1, DS_STATS_TILES = 2 };
 
 template <int MAXG>
@@ -150,8 +152,8 @@ __device__ __forceinline__ void mma_bf16(float (&c)[4], const uint32_t (&a)[4], 
       : "+f"(c[0]), "+f"(c[1]), "+f"(c[2]), "+f"(c[3])
       : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(b0), "r"(b1));
 }
-// Barrier of the consumer warps only (the producer keeps streaming meanwhile).
-__device__ __forceinline__ void consumers_sync() { asm volatile("bar.sync 1, %0;" ::"n"(DS_NC * 32) : "memory"); }
+// Barrier of the epilogue warps only (producer and MMA warps keep streaming meanwhile).
+__device__ __forceinline__ void epilogue_sync() { asm volatile("bar.sync 1, %0;" ::"n"(DS_NE * 32) : "memory"); }
 
 // Stream-K partition of U units over G CTAs: CTA c takes [start(c), start(c + 1)).
 __device__ __forceinline__ long long ds_start(long long c, long long U, long long G) { return c * U / G; }
@@ -160,12 +162,12 @@ __device__ __forceinline__ long long ds_owner(long long u, long long U, long lon
   return ((u + 1) * G + U - 1) / U - 1;
 }
 
-// Fused epilogue of one tile, element-parallel over the consumer warps: warp cw takes rows
-// cw, cw + DS_NC, ..., lane = feature.
+// Fused epilogue of one tile, element-parallel over the epilogue warps: warp ew takes rows
+// ew, ew + DS_NE, ..., lane = feature.
 template <int KIND>
-__device__ __forceinline__ void ds_epilogue(const Epi& e, const float* sS, int M, int rb, int f0, int N, int cw,
+__device__ __forceinline__ void ds_epilogue(const Epi& e, const float* sS, int M, int rb, int f0, int N, int ew,
                                             int lane, const int* s_pos, const int* s_blk) {
-  for (int row = cw; row < M; row += DS_NC) {
+  for (int row = ew; row < M; row += DS_NE) {
     const int ra = rb + row, c = f0 + lane;
     const bool valid = c < N;
     float v = sS[row * DS_RP + lane];
@@ -223,151 +225,196 @@ __device__ __forceinline__ void ds_epilogue(const Epi& e, const float* sS, int M
   }
 }
 
-// Stages rows [rb, rb + M) of the A operand into sA (bf16, pitch apitch; all K), rows
-// M..arows-1 zero.  All threads of the CTA take part.
+// Stages rows 0..Ms-1 of the A operand into sA (bf16, pitch apitch; all K), rows
+// Ms..arows-1 zero.  All threads of the CTA take part; one round trip to memory: a plain bf16
+// operand is copied with cp.async; a standardised one is read into registers (two rows at a
+// time, DS_XV float4 per thread and row) while its row statistics are loaded (or reduced from
+// those registers), then written standardised.
+constexpr int DS_XV = 5;    // float4 per thread and row: rows up to DS_XV * 4 * DS_THREADS floats
 template <int MAXG>
-__device__ void ds_stage_a(const DsParams<MAXG>& p, bf16* sA, int rb, int M, float* s_mu, float* s_rs,
-                           float (*s_red)[16]) {
+__device__ void ds_stage_a(const DsParams<MAXG>& p, bf16* sA, int Ms, float* s_mu, float* s_rs,
+                           float (*s_red)[16]) {   // s_red: [DS_WARPS][16]
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5, K = p.K, ap = p.apitch;
-  for (int i = tid; i < (p.arows - M) * (ap >> 3); i += DS_THREADS) {   // zero rows past M
-    const int r = M + i / (ap >> 3), c = i % (ap >> 3);
+  for (int i = tid; i < (p.arows - Ms) * (ap >> 3); i += DS_THREADS) {   // zero rows past Ms
+    const int r = Ms + i / (ap >> 3), c = i % (ap >> 3);
     *reinterpret_cast<uint4*>(sA + (size_t)r * ap + c * 8) = make_uint4(0, 0, 0, 0);
   }
   if (!p.fused_norm) {
     const int cpr = K >> 3;
-    for (int i = tid; i < M * cpr; i += DS_THREADS) {
+    for (int i = tid; i < Ms * cpr; i += DS_THREADS) {
       const int r = i / cpr, c = i - r * cpr;
-      cp_async16(sA + (size_t)r * ap + c * 8, p.A + (size_t)(rb + r) * p.lda + c * 8);
+      cp_async16(sA + (size_t)r * ap + c * 8, p.A + (size_t)r * p.lda + c * 8);
     }
     cp_async_wait_all();
     __syncthreads();
     return;
   }
-  // row statistics (mu, rstd) of the fp32 source rows
-  const float* xr[16];
+  const int K4 = K >> 2;
+  for (int r0 = 0; r0 < Ms; r0 += 2) {
+    const int nr = min(2, Ms - r0);
+    float4 xv[2][DS_XV];
+    const float* xr[2];
 #pragma unroll
-  for (int r = 0; r < 16; ++r) xr[r] = p.X + (size_t)(r < M ? (p.in_rows ? p.in_rows[rb + r] : rb + r) : 0) * p.ldx;
-  if (p.stat_mode == DS_STATS_ROWS) {
-    if (tid < M) {
-      const float2 s = p.row_stats[rb + tid];
-      s_mu[tid] = s.x;
-      s_rs[tid] = s.y;
+    for (int k = 0; k < 2; ++k) {
+      const int r = k < nr ? r0 + k : r0;
+      xr[k] = p.X + (size_t)(p.in_rows ? p.in_rows[r] : r) * p.ldx;
     }
-  } else if (p.stat_mode == DS_STATS_TILES) {
-    // the row's moments from the producer's 32-column (mean, M2) tiles, about the first
-    // tile's mean c: S1 = sum 32 (m_t - c), S2 = sum M2_t + 32 (m_t - c)^2
-    for (int r = warp; r < M; r += DS_NC + 1) {
-      const float2* ts = p.tile_stats + (size_t)(rb + r) * p.n_stiles;
-      const float c = ts[0].x;
-      float s1 = 0.f, s2 = 0.f;
-      for (int t = lane; t < p.n_stiles; t += 32) {
-        const float2 b = ts[t];
-        const float dm = b.x - c;
-        s1 += 32.f * dm;
-        s2 += b.y + 32.f * dm * dm;
+    // the rows' values: every load issued before any is used
+#pragma unroll
+    for (int k = 0; k < 2; ++k)
+#pragma unroll
+      for (int j = 0; j < DS_XV; ++j) {
+        const int v = tid + j * DS_THREADS;
+        xv[k][j] = (k < nr && v < K4) ? *reinterpret_cast<const float4*>(xr[k] + v * 4) : make_float4(0.f, 0.f, 0.f, 0.f);
       }
-      s1 = warp_sum(s1);
-      s2 = warp_sum(s2);
-      if (lane == 0) {
-        const float dmean = s1 / K, var = fmaxf(s2 / K - dmean * dmean, 0.f), mean = c + dmean;
-        float mu = 0.f, rs = 1.f;
-        if (p.norm_mode == NORM_LN) {
-          mu = mean;
-          rs = rsqrtf(var + p.eps);
-        } else if (p.norm_mode == NORM_RMS) {
-          rs = rsqrtf(var + mean * mean + p.eps);
+    if (p.stat_mode == DS_STATS_ROWS) {
+      if (tid < nr) {
+        const float2 st = p.row_stats[r0 + tid];
+        s_mu[r0 + tid] = st.x;
+        s_rs[r0 + tid] = st.y;
+      }
+    } else if (p.stat_mode == DS_STATS_TILES) {
+      // the row's moments from the producer's 32-column (mean, M2) tiles, about the first
+      // tile's mean c: S1 = sum 32 (m_t - c), S2 = sum M2_t + 32 (m_t - c)^2 (warp k: row r0 + k)
+      if (warp < nr) {
+        const int r = r0 + warp;
+        const float2* ts = p.tile_stats + (size_t)r * p.n_stiles;
+        const float c = ts[0].x;
+        float s1 = 0.f, s2 = 0.f;
+        for (int t = lane; t < p.n_stiles; t += 32) {
+          const float2 b = ts[t];
+          const float dm = b.x - c;
+          s1 += 32.f * dm;
+          s2 += b.y + 32.f * dm * dm;
         }
-        s_mu[r] = mu;
-        s_rs[r] = rs;
-      }
-    }
-  } else {
-    // two passes over the rows (L2-resident): mean, then the centred second moment
-    auto row_sums = [&](auto term, float* out) {
-      float part[16];
-#pragma unroll
-      for (int r = 0; r < 16; ++r) part[r] = 0.f;
-      for (int d = tid * 4; d < K; d += DS_THREADS * 4) {
-#pragma unroll
-        for (int r = 0; r < 16; ++r)
-          if (r < M) {
-            const float4 x = *reinterpret_cast<const float4*>(xr[r] + d);
-            part[r] += term(r, x.x) + term(r, x.y) + term(r, x.z) + term(r, x.w);
+        s1 = warp_sum(s1);
+        s2 = warp_sum(s2);
+        if (lane == 0) {
+          const float dmean = s1 / K, var = fmaxf(s2 / K - dmean * dmean, 0.f), mean = c + dmean;
+          float mu = 0.f, rs = 1.f;
+          if (p.norm_mode == NORM_LN) {
+            mu = mean;
+            rs = rsqrtf(var + p.eps);
+          } else if (p.norm_mode == NORM_RMS) {
+            rs = rsqrtf(var + mean * mean + p.eps);
           }
+          s_mu[r] = mu;
+          s_rs[r] = rs;
+        }
       }
+    } else {
+      // statistics of the rows in registers: mean (LayerNorm), then the centred second moment
+      float mu[2] = {0.f, 0.f};
+      if (p.norm_mode == NORM_LN) {
 #pragma unroll
-      for (int r = 0; r < 16; ++r) {
-        const float v = warp_sum(part[r]);
-        if (lane == 0) s_red[warp][r] = v;
+        for (int k = 0; k < 2; ++k) {
+          float a = 0.f;
+#pragma unroll
+          for (int j = 0; j < DS_XV; ++j) a += (xv[k][j].x + xv[k][j].y) + (xv[k][j].z + xv[k][j].w);
+          a = warp_sum(a);
+          if (lane == 0) s_red[warp][k] = a;
+        }
+        __syncthreads();
+#pragma unroll
+        for (int k = 0; k < 2; ++k) {
+          float t = 0.f;
+          for (int w = 0; w < DS_WARPS; ++w) t += s_red[w][k];
+          mu[k] = t / K;
+        }
+        __syncthreads();
       }
-      __syncthreads();
-      if (tid < M) {
-        float t = 0.f;
-        for (int w = 0; w < DS_NC + 1; ++w) t += s_red[w][tid];
-        out[tid] = t / K;
+      if (p.norm_mode != NORM_COPY) {
+#pragma unroll
+        for (int k = 0; k < 2; ++k) {
+          float a = 0.f;
+#pragma unroll
+          for (int j = 0; j < DS_XV; ++j) {
+            const int v = tid + j * DS_THREADS;
+            if (v < K4) {
+              const float4 x = xv[k][j];
+              const float c0 = x.x - mu[k], c1 = x.y - mu[k], c2 = x.z - mu[k], c3 = x.w - mu[k];
+              a += (c0 * c0 + c1 * c1) + (c2 * c2 + c3 * c3);
+            }
+          }
+          a = warp_sum(a);
+          if (lane == 0) s_red[warp][k] = a;
+        }
+        __syncthreads();
+        if (tid < nr) {
+          float t = 0.f;
+          for (int w = 0; w < DS_WARPS; ++w) t += s_red[w][tid];
+          s_mu[r0 + tid] = mu[tid];
+          s_rs[r0 + tid] = rsqrtf(t / K + p.eps);
+        }
+      } else if (tid < nr) {
+        s_mu[r0 + tid] = 0.f;
+        s_rs[r0 + tid] = 1.f;
       }
-      __syncthreads();
-    };
-    if (tid < 16) {
-      s_mu[tid] = 0.f;
-      s_rs[tid] = 1.f;
     }
     __syncthreads();
-    if (p.norm_mode == NORM_LN) row_sums([](int, float x) { return x; }, s_mu);
-    if (p.norm_mode != NORM_COPY) {
-      row_sums([&](int r, float x) { const float c = x - s_mu[r]; return c * c; }, s_rs);
-      if (tid < M) s_rs[tid] = rsqrtf(s_rs[tid] + p.eps);
+#pragma unroll
+    for (int k = 0; k < 2; ++k) {
+      if (k >= nr) break;
+      const int r = r0 + k;
+      const float mu = s_mu[r], rs = s_rs[r];
+#pragma unroll
+      for (int j = 0; j < DS_XV; ++j) {
+        const int v = tid + j * DS_THREADS;
+        if (v < K4) {
+          const float4 x = xv[k][j];
+          const __nv_bfloat162 lo = __floats2bfloat162_rn((x.x - mu) * rs, (x.y - mu) * rs);
+          const __nv_bfloat162 hi = __floats2bfloat162_rn((x.z - mu) * rs, (x.w - mu) * rs);
+          uint2 u;
+          u.x = *reinterpret_cast<const uint32_t*>(&lo);
+          u.y = *reinterpret_cast<const uint32_t*>(&hi);
+          *reinterpret_cast<uint2*>(sA + (size_t)r * ap + v * 4) = u;
+        }
+      }
     }
+    __syncthreads();
   }
-  __syncthreads();
-  for (int i = tid; i < M * (K >> 2); i += DS_THREADS) {
-    const int r = i / (K >> 2), v4 = i - r * (K >> 2);
-    const float4 x = *reinterpret_cast<const float4*>(xr[r] + v4 * 4);
-    const float mu = s_mu[r], rs = s_rs[r];
-    const __nv_bfloat162 lo = __floats2bfloat162_rn((x.x - mu) * rs, (x.y - mu) * rs);
-    const __nv_bfloat162 hi = __floats2bfloat162_rn((x.z - mu) * rs, (x.w - mu) * rs);
-    uint2 u;
-    u.x = *reinterpret_cast<const uint32_t*>(&lo);
-    u.y = *reinterpret_cast<const uint32_t*>(&hi);
-    *reinterpret_cast<uint2*>(sA + (size_t)r * ap + v4 * 4) = u;
-  }
-  __syncthreads();
 }
 
 // MB: 8-token blocks of the A operand (1: M <= 8, 2: M <= 16); KIND: the epilogue kind.
 template <int MB, int KIND, int MAXG>
-__global__ void __launch_bounds__(DS_THREADS, 1) gemm_stream_kernel(const __grid_constant__ DsParams<MAXG> p) {
+__global__ void __launch_bounds__(DS_THREADS, 2) gemm_stream_kernel(const __grid_constant__ DsParams<MAXG> p) {
   KT_BEGIN();
   extern __shared__ __align__(128) uint8_t ds_smem_raw[];
   __shared__ __align__(8) uint64_t full[DS_MAX_STAGES];
   __shared__ __align__(8) uint64_t empty[DS_MAX_STAGES];
+  __shared__ __align__(8) uint64_t tb_full[2], tb_empty[2];   // tile hand-off, MMA warps -> epilogue warps
   __shared__ float s_mu[16], s_rs[16];
-  __shared__ float s_red[DS_NC + 1][16];
+  __shared__ float s_red[DS_WARPS][16];
   __shared__ int s_live[MAXG];     // problems with rows, in order
   __shared__ int s_M[MAXG], s_rb[MAXG];
   __shared__ int s_nlive, s_last;
   __shared__ int s_pos[16], s_blk[16];   // cache epilogues: each row's position and cache block
+  __shared__ int s_info[2][3];           // per hand-off buffer: live problem slot, tile, whole
+  __shared__ int s_eok[DS_NE];           // epilogue warps: still following the hand-offs
 
+  const long long wlim = wait_limit();   // the runtime wait limit, read once
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   uint8_t* smem = ds_smem_raw + ((1024 - (smem_u32(ds_smem_raw) & 1023)) & 1023);
   uint8_t* sW = smem;                                           // [S][4 chunks][32 rows][128 B], swizzled
   bf16* sA = reinterpret_cast<bf16*>(smem + p.off_a);           // [arows][apitch]
-  float* sP = reinterpret_cast<float*>(smem + p.off_p);         // [2][16][DS_RP] k halves, then [16][DS_RP] sum
-  float* sS = sP + 2 * 16 * DS_RP;
+  float* sT = reinterpret_cast<float*>(smem + p.off_p);         // [2][16][DS_RP] tile hand-off buffers
   const int S = p.stages;
+  const int nkb = p.nkb, tiles = p.tiles, Kd = p.K;   // in registers: the lambdas below take them by reference
   const long long c = blockIdx.x;
-  const long long per_prob = (long long)p.tiles * p.nkb;
-  // the units are shared by G = min(grid, units) CTAs, so that every sharing CTA has at
-  // least one unit (a tile's contributors are then exactly the CTAs between its first and
-  // its last unit's owners)
+  const long long per_prob = (long long)tiles * nkb;
 
   if (tid == 0) {
     for (int s = 0; s < S; ++s) {
       mbar_init(&full[s], 1);
       mbar_init(&empty[s], DS_NC);
     }
+    for (int b = 0; b < 2; ++b) {
+      mbar_init(&tb_full[b], DS_NC);
+      mbar_init(&tb_empty[b], DS_NE);
+    }
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
   }
+  for (int i = tid; i < 2 * 16 * DS_RP; i += DS_THREADS) sT[i] = 0.f;
   __syncthreads();
   pdl_launch_dependents();
 
@@ -380,14 +427,14 @@ __global__ void __launch_bounds__(DS_THREADS, 1) gemm_stream_kernel(const __grid
     Cur r;
     r.li = (int)(u / per_prob);
     const long long rem = u - (long long)r.li * per_prob;
-    r.t = (int)(rem / p.nkb);
-    r.kb = (int)(rem - (long long)r.t * p.nkb);
+    r.t = (int)(rem / nkb);
+    r.kb = (int)(rem - (long long)r.t * nkb);
     return r;
   };
   auto advance = [&](Cur& r) {
-    if (++r.kb == p.nkb) {
+    if (++r.kb == nkb) {
       r.kb = 0;
-      if (++r.t == p.tiles) {
+      if (++r.t == tiles) {
         r.t = 0;
         ++r.li;
       }
@@ -398,7 +445,7 @@ __global__ void __launch_bounds__(DS_THREADS, 1) gemm_stream_kernel(const __grid
     tma_load_3d(&p.wmap[q], &full[s], sW + (size_t)s * DS_STAGE, r.t * DS_BN, r.kb * (DS_KB / 64));
   };
 
-  // single problem: the partition is known before the wait; its first units are issued
+  // single problem: the partition is known before the wait and the whole ring is issued
   // before it (weights do not depend on the preceding kernel)
   long long U = p.grouped ? 0 : per_prob;
   long long G = U < (long long)gridDim.x ? U : (long long)gridDim.x;
@@ -406,8 +453,7 @@ __global__ void __launch_bounds__(DS_THREADS, 1) gemm_stream_kernel(const __grid
   int pre = 0;
   if (!p.grouped && warp == 0 && lane == 0) {
     const long long avail = u1 - u0;
-    pre = S < DS_PRE ? S : DS_PRE;
-    if ((long long)pre > avail) pre = (int)avail;
+    pre = (long long)S > avail ? (int)avail : S;
     Cur r = cur_at(u0);
     for (int g = 0; g < pre; ++g) {
       issue(r, 0, g);
@@ -418,22 +464,25 @@ __global__ void __launch_bounds__(DS_THREADS, 1) gemm_stream_kernel(const __grid
   pdl_wait();   // from here on, the preceding kernels' writes are visible
   KT_WAITED();
 
+  // The row counts (device values) and the A operand are read in parallel: every problem's
+  // rows start at row 0 (host-checked), so the launch's row bound max_m is staged without
+  // waiting for the count (rows past it feed only token columns that are never stored).
   if (tid == 0) {
     int n = 0;
     for (int q = 0; q < p.n_probs; ++q) {
-      const int b = p.rows[q].b();
-      int M = p.rows[q].e() - b;
+      int M = p.rows[q].e();
       if (M > p.max_m) {   // more rows than the launch was sized for
         atomicOr(p.err, ERRW_CONFIG);
         M = p.max_m;
       }
       s_M[q] = M;
-      s_rb[q] = b;
+      s_rb[q] = 0;
       if (M > 0) s_live[n++] = q;
     }
     s_nlive = n;
   }
-  __syncthreads();
+  ds_stage_a(p, sA, p.max_m, s_mu, s_rs, s_red);   // ends with a CTA barrier: the counts are visible
+  KT_MARK(1);
   const int nlive = s_nlive;
   if (p.grouped) {
     U = (long long)nlive * per_prob;
@@ -449,34 +498,11 @@ __global__ void __launch_bounds__(DS_THREADS, 1) gemm_stream_kernel(const __grid
     return;
   }
   const int n_units = (int)(u1 - u0);
-
-  // A operand: the rows of the launch (grouped: every problem's rows are a prefix of one
-  // shared range starting at the first live problem's begin)
-  int Ms = 0;
-  for (int k = 0; k < nlive; ++k) Ms = max(Ms, s_M[s_live[k]]);
-  const int rb0 = s_rb[s_live[0]];
-  if (KIND == EPI_QKV || KIND == EPI_KV) {
-    // each row's position and cache block, looked up once (every problem of the launch holds
-    // the same tokens in the same rows)
-    const Epi& e0 = p.epi[s_live[0]];
-    if (tid < Ms) {
-      const int tok = e0.row_tok[rb0 + tid];
-      const int pos = e0.tok_pos[tok], seq = e0.tok_seq[tok];
-      const KVCacheView& cv = e0.cache;
-      int blk = -1;
-      if (seq >= 0 && seq < cv.max_batch && pos >= 0 && pos < cv.max_blocks_per_seq * cv.block_tokens) {
-        blk = cv.block_table[seq * cv.max_blocks_per_seq + pos / cv.block_tokens];
-        if (blk < 0 || blk >= cv.n_blocks) blk = -1;
-      }
-      s_pos[tid] = pos;
-      s_blk[tid] = blk;
-    }
-  }
-  ds_stage_a(p, sA, rb0, Ms, s_mu, s_rs, s_red);
-  KT_MARK(1);
+  const long long gt_first = u0 / nkb, gt_last = (u1 - 1) / nkb;   // this CTA's first / last live-enumerated tile
+  const int n_tiles_cta = (int)(gt_last - gt_first + 1);
 
   if (warp == 0) {
-    // ---- producer: refill each slot once its four consumer warps have released it
+    // ---- producer: refill each slot once its four MMA warps have released it
     if (lane == 0) {
       bool ok = true;
       int issued = pre;
@@ -487,7 +513,7 @@ __global__ void __launch_bounds__(DS_THREADS, 1) gemm_stream_kernel(const __grid
         n = 1;
       }
       for (int g = pre; g < n_units && ok; ++g) {
-        if (n >= 1) ok = ds_wait(&empty[s], (uint32_t)((n - 1) & 1), p.err, wait_limit());
+        if (n >= 1) ok = ds_wait(&empty[s], (uint32_t)((n - 1) & 1), p.err, wlim);
         if (ok) {
           issue(r, s_live[r.li], s);
           issued = g + 1;
@@ -499,14 +525,108 @@ __global__ void __launch_bounds__(DS_THREADS, 1) gemm_stream_kernel(const __grid
         }
       }
       // before leaving, every copy this CTA issued has landed (bounded waits; immediate when
-      // the consumers have taken them)
+      // the MMA warps have taken them)
       for (int h = max(0, issued - S); h < issued; ++h)
         ds_wait(&full[h % S], (uint32_t)((h / S) & 1), p.err, DS_TIMEOUT_CYCLES);
     }
     return;
   }
 
-  // ---- consumers: warp cw = (mb, kh): features mb*16.., 64-k chunks kh, kh + 2 of a unit
+  if (warp > DS_NC) {
+    // ---- epilogue warps: finish each tile the MMA warps hand over, in order
+    const int ew = warp - 1 - DS_NC, et = tid - 32 * (1 + DS_NC);   // 0..DS_NE-1, 0..63
+    if (KIND == EPI_QKV || KIND == EPI_KV) {
+      // each row's position and cache block, looked up once while the first tile streams (every
+      // problem of the launch holds the same tokens in the same rows)
+      const Epi& e0 = p.epi[s_live[0]];
+      int Ms = 0;
+      for (int k = 0; k < nlive; ++k) Ms = max(Ms, s_M[s_live[k]]);
+      if (et < Ms) {
+        const int tok = e0.row_tok[et];
+        const int pos = e0.tok_pos[tok], seq = e0.tok_seq[tok];
+        const KVCacheView& cv = e0.cache;
+        int blk = -1;
+        if (seq >= 0 && seq < cv.max_batch && pos >= 0 && pos < cv.max_blocks_per_seq * cv.block_tokens) {
+          blk = cv.block_table[seq * cv.max_blocks_per_seq + pos / cv.block_tokens];
+          if (blk < 0 || blk >= cv.n_blocks) blk = -1;
+        }
+        s_pos[et] = pos;
+        s_blk[et] = blk;
+      }
+      epilogue_sync();
+    }
+    // one hand-off: the tile's description and sum are in buffer b
+    auto process = [&](int b) {
+      const int li = s_info[b][0], t = s_info[b][1], whole = s_info[b][2];
+      const long long gt = (long long)li * tiles + t;
+      const int q = s_live[li];
+      const int M = s_M[q], rb = s_rb[q];
+      const Epi& e = p.epi[q];
+      float* tile = sT + b * 16 * DS_RP;
+      if (whole) {
+        ds_epilogue<KIND>(e, tile, M, rb, t * DS_BN, p.N, ew, lane, s_pos, s_blk);
+        return;
+      }
+      // shared tile: publish this CTA's partial, count the arrival; the last one finishes it
+      const long long slot = 2 * c + (gt == gt_first ? 0 : 1);
+      float* mine = p.part + slot * (16 * DS_BN);
+      for (int i = et; i < M * DS_BN; i += DS_NE * 32) mine[i] = tile[(i >> 5) * DS_RP + (i & 31)];
+      __threadfence();
+      epilogue_sync();
+      const long long c_first = ds_owner(gt * nkb, U, G), c_last = ds_owner(gt * nkb + nkb - 1, U, G);
+      if (et == 0) {
+        const int old = atomicAdd(&p.cnt[(long long)q * tiles + t], 1);
+        s_last = old == (int)(c_last - c_first);
+      }
+      epilogue_sync();
+      if (!s_last) return;
+      __threadfence();
+      // the contributors' partials summed in contributor order (each thread at most 8 values)
+      float v[8];
+#pragma unroll
+      for (int k = 0; k < 8; ++k) v[k] = 0.f;
+      for (long long cc = c_first; cc <= c_last; ++cc) {
+        const long long sl = 2 * cc + (gt == ds_start(cc, U, G) / nkb ? 0 : 1);
+        const float* src = p.part + sl * (16 * DS_BN);
+#pragma unroll
+        for (int k = 0; k < 8; ++k) {
+          const int i = et + k * DS_NE * 32;
+          if (i < M * DS_BN) v[k] += __ldcg(src + i);
+        }
+      }
+#pragma unroll
+      for (int k = 0; k < 8; ++k) {
+        const int i = et + k * DS_NE * 32;
+        if (i < M * DS_BN) tile[(i >> 5) * DS_RP + (i & 31)] = v[k];
+      }
+      if (et == 0) p.cnt[(long long)q * tiles + t] = 0;
+      epilogue_sync();
+      ds_epilogue<KIND>(e, tile, M, rb, t * DS_BN, p.N, ew, lane, s_pos, s_blk);
+    };
+    bool ok = true;
+    for (int j = 0; j < n_tiles_cta; ++j) {
+      const int b = j & 1;
+      bool got = true;
+      if (lane == 0 && ok) got = ds_wait(&tb_full[b], (uint32_t)((j >> 1) & 1), p.err, wlim);
+      got = __shfl_sync(0xffffffffu, got ? 1 : 0, 0) != 0;
+      __syncwarp();     // lane 0's acquire orders the whole warp's reads of the hand-off buffer
+      // Both epilogue warps take the same decision: once either has given up, neither reads a
+      // hand-off again (its buffer and description may not have been written); they only keep
+      // releasing buffers so that the MMA warps finish (outputs undefined, error word set).
+      if (lane == 0) s_eok[ew] = (ok && got) ? 1 : 0;
+      epilogue_sync();
+      ok = s_eok[0] != 0 && s_eok[1] != 0;
+      if (ok) process(b);
+      epilogue_sync();
+      float* tile = sT + b * 16 * DS_RP;
+      for (int i = et; i < 16 * DS_RP; i += DS_NE * 32) tile[i] = 0.f;   // zero for the next hand-off
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&tb_empty[b]);
+    }
+    return;
+  }
+
+  // ---- MMA warps: warp cw = (mb, kh): features mb*16.., 64-k chunks kh, kh + 2 of a unit
   const int cw = warp - 1, mb = cw & 1, kh = cw >> 1;
   const int wrow = mb * 16 + (lane & 7) + ((lane >> 3) & 1) * 8;
   const uint32_t w_base = smem_u32(sW) + kh * DS_CHUNK + wrow * 128;
@@ -516,122 +636,107 @@ __global__ void __launch_bounds__(DS_THREADS, 1) gemm_stream_kernel(const __grid
                           kh * 128;
   const int bg = lane >> 2;
   const uint32_t b_base = smem_u32(sA) + (bg * ap + kh * 64 + (lane & 3) * 2) * 2;
-  const int ct = tid - 32;   // 0..127 among the consumers
 
-  float acc[MB][4];
+  // one accumulator set per k16 step of a 64-k chunk: four independent MMA chains per warp
+  float acc[4][MB][4];
   auto zero_acc = [&]() {
 #pragma unroll
-    for (int t = 0; t < MB; ++t) acc[t][0] = acc[t][1] = acc[t][2] = acc[t][3] = 0.f;
+    for (int k = 0; k < 4; ++k)
+#pragma unroll
+      for (int t = 0; t < MB; ++t) acc[k][t][0] = acc[k][t][1] = acc[k][t][2] = acc[k][t][3] = 0.f;
   };
   zero_acc();
   Cur r = cur_at(u0);
-  const long long gt_first = (long long)r.li * p.tiles + r.t;   // this CTA's first (live-enumerated) tile
 
-  // the tile (li, t) ends here; whole: this CTA covered all of its k-blocks
-  auto finish_tile = [&](int li, int t, bool whole) {
-    const long long gt = (long long)li * p.tiles + t;
-    const int q = s_live[li];
-    const int M = s_M[q], rb = s_rb[q];
-    const Epi& e = p.epi[q];
-    // partial tile [token][feature] of this warp into its k half, then the sum of halves
-    {
-      float* part = sP + kh * 16 * DS_RP;
-      const int gq = lane >> 2, t4 = lane & 3;
-#pragma unroll
-      for (int t2 = 0; t2 < MB; ++t2) {
-        const int tk = t2 * 8 + 2 * t4, fc = mb * 16 + gq;
-        part[tk * DS_RP + fc] = acc[t2][0];
-        part[(tk + 1) * DS_RP + fc] = acc[t2][1];
-        part[tk * DS_RP + fc + 8] = acc[t2][2];
-        part[(tk + 1) * DS_RP + fc + 8] = acc[t2][3];
-      }
-    }
-    zero_acc();
-    consumers_sync();
-    for (int i = ct; i < M * DS_BN; i += DS_NC * 32) {
-      const int j = (i >> 5) * DS_RP + (i & 31);
-      sS[j] = sP[j] + sP[16 * DS_RP + j];
-    }
-    consumers_sync();
-    if (!whole) {
-      // shared tile: publish this CTA's partial, count the arrival; the last one finishes it
-      const long long slot = 2 * c + (gt == gt_first ? 0 : 1);
-      float* mine = p.part + slot * (16 * DS_BN);
-      for (int i = ct; i < M * DS_BN; i += DS_NC * 32) mine[i] = sS[(i >> 5) * DS_RP + (i & 31)];
-      __threadfence();
-      consumers_sync();
-      const long long c_first = ds_owner(gt * p.nkb, U, G), c_last = ds_owner(gt * p.nkb + p.nkb - 1, U, G);
-      if (ct == 0) {
-        const int old = atomicAdd(&p.cnt[(long long)q * p.tiles + t], 1);
-        s_last = old == (int)(c_last - c_first);
-      }
-      consumers_sync();
-      if (!s_last) return;
-      __threadfence();
-      // the contributors' partials summed in contributor order (each thread at most 4 values)
-      float v[4] = {0.f, 0.f, 0.f, 0.f};
-      for (long long cc = c_first; cc <= c_last; ++cc) {
-        const long long sl = 2 * cc + (gt == ds_start(cc, U, G) / p.nkb ? 0 : 1);
-        const float* src = p.part + sl * (16 * DS_BN);
-#pragma unroll
-        for (int k = 0; k < 4; ++k) {
-          const int i = ct + k * DS_NC * 32;
-          if (i < M * DS_BN) v[k] += __ldcg(src + i);
-        }
-      }
-#pragma unroll
-      for (int k = 0; k < 4; ++k) {
-        const int i = ct + k * DS_NC * 32;
-        if (i < M * DS_BN) sS[(i >> 5) * DS_RP + (i & 31)] = v[k];
-      }
-      if (ct == 0) p.cnt[(long long)q * p.tiles + t] = 0;
-      consumers_sync();
-    }
-    ds_epilogue<KIND>(e, sS, M, rb, t * DS_BN, p.N, cw, lane, s_pos, s_blk);
-    consumers_sync();   // sP / sS are rewritten by the next tile
-  };
-
-  // A warp whose wait gives up stops waiting and computing but still releases its slots and
-  // takes part in every consumer barrier, so the CTA always completes (the error word is set).
+  // Lane 0 waits for each slot and broadcasts, so the decision is warp-uniform (the fragment
+  // loads and MMAs below are .aligned).  A warp whose wait gives up stops waiting, computing and
+  // releasing slots (a slot it has not seen land must not be refilled: the producer's own
+  // bounded wait then ends the stream and it drains its copies), but still hands over every
+  // tile, so the epilogue warps and the CTA complete (the error word is set).
   bool ok = true;
   bool seg_whole_start = r.kb == 0;   // the current tile's segment began at its first k-block
   int Mq = s_M[s_live[r.li]];
   int s = 0, n = 0;                   // slot and use number of unit g
+  int j = 0;                          // tile hand-offs so far
   for (int g = 0; g < n_units; ++g) {
-    if (ok) ok = ds_wait(&full[s], (uint32_t)(n & 1), p.err, wait_limit());
+    if (ok) {
+      bool landed = true;
+      if (lane == 0) landed = ds_wait(&full[s], (uint32_t)(n & 1), p.err, wlim);
+      ok = __shfl_sync(0xffffffffu, landed ? 1 : 0, 0) != 0;
+      __syncwarp();   // lane 0's acquire orders the whole warp's reads of the slot
+    }
     const int kb = r.kb;
-    const int nch = ok ? min(DS_KB, p.K - kb * DS_KB) >> 6 : 0;
+    const int nch = ok ? min(DS_KB, Kd - kb * DS_KB) >> 6 : 0;
     const uint32_t sbase = w_base + s * DS_STAGE;
     for (int q = 0; 2 * q + kh < nch; ++q) {
       const uint32_t wa = sbase + q * (2 * DS_CHUNK);
       const int kk0 = kb * DS_KB + q * 128;
       const uint32_t aa = a_base + kk0 * 2;
       const uint32_t ab = b_base + kk0 * 2;
+      // every fragment of the chunk first, then four independent MMAs
+      uint32_t a[4][4];
 #pragma unroll
-      for (int kk = 0; kk < 4; ++kk) {
-        uint32_t a[4];
-        ldsm_x4(a, wa + (((kk * 2 + wu) ^ wx) << 4));
-        if (MB == 2) {
-          uint32_t b[4];
-          ldsm_x4(b, aa + kk * 32);
-          mma_bf16(acc[0], a, b[0], b[1]);
-          mma_bf16(acc[MB - 1], a, b[2], b[3]);
-        } else {
-          uint32_t b0 = 0u, b1 = 0u;
-          if (bg < Mq) {
-            b0 = ld_shared_u32(ab + kk * 32);
-            b1 = ld_shared_u32(ab + kk * 32 + 16);
-          }
-          mma_bf16(acc[0], a, b0, b1);
+      for (int kk = 0; kk < 4; ++kk) ldsm_x4(a[kk], wa + (((kk * 2 + wu) ^ wx) << 4));
+      if (MB == 2) {
+        uint32_t bb[4][4];
+#pragma unroll
+        for (int kk = 0; kk < 4; ++kk) ldsm_x4(bb[kk], aa + kk * 32);
+#pragma unroll
+        for (int kk = 0; kk < 4; ++kk) {
+          mma_bf16(acc[kk][0], a[kk], bb[kk][0], bb[kk][1]);
+          mma_bf16(acc[kk][MB - 1], a[kk], bb[kk][2], bb[kk][3]);
         }
+      } else {
+        uint32_t b0[4], b1[4];
+#pragma unroll
+        for (int kk = 0; kk < 4; ++kk) {
+          b0[kk] = b1[kk] = 0u;
+          if (bg < Mq) {
+            b0[kk] = ld_shared_u32(ab + kk * 32);
+            b1[kk] = ld_shared_u32(ab + kk * 32 + 16);
+          }
+        }
+#pragma unroll
+        for (int kk = 0; kk < 4; ++kk) mma_bf16(acc[kk][0], a[kk], b0[kk], b1[kk]);
       }
     }
     __syncwarp();
-    if (lane == 0) mbar_arrive(&empty[s]);
+    if (lane == 0 && ok) mbar_arrive(&empty[s]);
     const bool last = g == n_units - 1;
-    // tile boundary or the end of the range: finish the tile
-    if (kb == p.nkb - 1 || last) {
-      finish_tile(r.li, r.t, seg_whole_start && kb == p.nkb - 1);
+    if (kb == nkb - 1 || last) {
+      // hand the tile over: wait until the buffer is free, add this warp's k half into it
+      // (exactly two additions per element onto zero, so the sum does not depend on their
+      // order), signal the epilogue warps
+      const int b = j & 1;
+      if (j >= 2) {
+        bool free_ok = true;
+        if (lane == 0) free_ok = ds_wait(&tb_empty[b], (uint32_t)(((j >> 1) - 1) & 1), p.err, wlim);
+        free_ok = __shfl_sync(0xffffffffu, free_ok ? 1 : 0, 0) != 0;
+        __syncwarp();
+        ok = ok && free_ok;
+      }
+      if (cw == 0 && lane == 0) {
+        s_info[b][0] = r.li;
+        s_info[b][1] = r.t;
+        s_info[b][2] = (seg_whole_start && kb == nkb - 1) ? 1 : 0;
+      }
+      float* tile = sT + b * 16 * DS_RP;
+      const int gq = lane >> 2, t4 = lane & 3;
+#pragma unroll
+      for (int t2 = 0; t2 < MB; ++t2) {
+        float a4[4];
+#pragma unroll
+        for (int jj = 0; jj < 4; ++jj) a4[jj] = (acc[0][t2][jj] + acc[1][t2][jj]) + (acc[2][t2][jj] + acc[3][t2][jj]);
+        const int tk = t2 * 8 + 2 * t4, fc = mb * 16 + gq;
+        atomicAdd(&tile[tk * DS_RP + fc], a4[0]);
+        atomicAdd(&tile[(tk + 1) * DS_RP + fc], a4[1]);
+        atomicAdd(&tile[tk * DS_RP + fc + 8], a4[2]);
+        atomicAdd(&tile[(tk + 1) * DS_RP + fc + 8], a4[3]);
+      }
+      zero_acc();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&tb_full[b]);
+      ++j;
       seg_whole_start = true;
     }
     advance(r);
@@ -694,6 +799,12 @@ bool ds_plan(const GemmProblem& q, int n_probs, int max_rows, const DgNorm* norm
   if (q.epi.tile_stats && (q.epi.kind != EPI_RESID || q.N % DS_BN)) return false;
   if (q.epi.kind < EPI_F32 || q.epi.kind > EPI_KV) return false;
   if ((long long)q.N * q.K * 2 * n_probs < DS_MIN_STREAM_BYTES) return false;
+  // narrow single problems (N < DS_MIN_N: every CTA would hold less than about two tiles and
+  // end on a shared tile's fix-up) stream faster on the cluster K-split kernel, whose partial
+  // sums meet in distributed shared memory (measured at the Llama-7B O and down projections)
+  if (n_probs == 1 && q.N < DS_MIN_N) return false;
+  if (q.rows.begin) return false;   // rows start at 0: the operand is staged before the count is read
+  if (norm && q.K > DS_XV * 4 * DS_THREADS) return false;
   if (!g_ds_sms) {
     int dev = 0;
     cudaGetDevice(&dev);
@@ -708,9 +819,9 @@ bool ds_plan(const GemmProblem& q, int n_probs, int max_rows, const DgNorm* norm
   const int arows = mb == 2 ? 16 : max_rows;
   const int apitch = q.K + 8;   // 16-byte shift per row: conflict-free fragment loads
   const int a_bytes = ((arows * apitch * 2) + 127) & ~127;
-  const int p_bytes = 3 * 16 * DS_RP * 4;
+  const int p_bytes = 2 * 16 * DS_RP * 4;   // the two tile hand-off buffers
   const int fixed = 1024 + a_bytes + p_bytes;
-  const int STATIC = 2 * DS_MAX_STAGES * 8 + 64 * 4 + (DS_NC + 1) * 64 + 3 * MAXG * 4 + 64 + 128;
+  const int STATIC = 2 * DS_MAX_STAGES * 8 + 32 + 128 + DS_WARPS * 64 + 3 * MAXG * 4 + 16 + 128 + 24 + 64;
   int stages = (DS_COHOST_SMEM - STATIC - fixed) / DS_STAGE;
   if (stages < 4) stages = (DS_SMEM_LIMIT - STATIC - fixed) / DS_STAGE;
   if (stages < 2) return false;

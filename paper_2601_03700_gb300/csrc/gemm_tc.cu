@@ -74,9 +74,10 @@ __device__ __forceinline__ bool mbar_try_wait(uint64_t* bar, uint32_t parity) {
 }
 // Bounded wait (the runtime wait limit) for the phase of `parity`; false on time-out or when
 // another role aborted.  The drains below keep the fixed TC_TIMEOUT_CYCLES.
-__device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, volatile int* abort_flag, unsigned* err) {
+__device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, volatile int* abort_flag, unsigned* err,
+                                          long long lim) {
   if (mbar_try_wait(bar, parity)) return true;
-  const long long t0 = clock64(), lim = wait_limit();
+  const long long t0 = clock64();
   while (true) {
     if (mbar_try_wait(bar, parity)) return true;
     if (*abort_flag) return false;
@@ -209,6 +210,7 @@ __global__ void __launch_bounds__(TC_THREADS, 1) gemm_tc_kernel(const __grid_con
   constexpr int B_BYTES = KC * BN * TC_BK * 2;
   constexpr uint32_t TMEM_COLS = 2 * BN;
   constexpr uint32_t IDESC = idesc_bf16<BN>();
+  const long long wlim = wait_limit();   // the runtime wait limit, read once
 
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = (uint8_t*)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
@@ -337,7 +339,7 @@ __global__ void __launch_bounds__(TC_THREADS, 1) gemm_tc_kernel(const __grid_con
         const CUtensorMap* tma_a = &G.ta;
         const CUtensorMap* tma_b = &G.tb;
         for (int kb = 0; kb < nk; ++kb) {
-          if (n_issued >= STAGES && !mbar_wait(&empty[stage], phase ^ 1, abort_flag, p.err)) break;
+          if (n_issued >= STAGES && !mbar_wait(&empty[stage], phase ^ 1, abort_flag, p.err, wlim)) break;
           ++n_issued;
           mbar_expect_tx(&full[stage], tx_bytes);
           if (KC == 1) {
@@ -383,11 +385,11 @@ __global__ void __launch_bounds__(TC_THREADS, 1) gemm_tc_kernel(const __grid_con
         locate(t, g, mb, nb);
         const int nk = (p.g[g].K + TC_BK * KC - 1) / (TC_BK * KC);
         const uint32_t a_chunk = (uint32_t)(p.g[g].a_box * TC_BK * 2);   // bytes between A chunks
-        if (!(ok = mbar_wait(&acce[ab], aph ^ 1, abort_flag, p.err))) break;
+        if (!(ok = mbar_wait(&acce[ab], aph ^ 1, abort_flag, p.err, wlim))) break;
         tc_fence_after();
         const uint32_t d = tmem + (uint32_t)(ab * BN);
         for (int kb = 0; kb < nk; ++kb) {
-          if (!(ok = mbar_wait(&full[stage], phase, abort_flag, p.err))) break;
+          if (!(ok = mbar_wait(&full[stage], phase, abort_flag, p.err, wlim))) break;
           if (t == (int)blockIdx.x && kb == 0) TC_TRACE(3);
 
           tc_fence_after();
@@ -450,7 +452,7 @@ __global__ void __launch_bounds__(TC_THREADS, 1) gemm_tc_kernel(const __grid_con
       // one lane per warp polls the barrier (128 pollers would crowd the barrier unit the
       // producer and MMA threads need); the result is broadcast to the warp
       bool got = true;
-      if (lane == 0) got = mbar_wait(&accf[ab], aph, abort_flag, p.err);
+      if (lane == 0) got = mbar_wait(&accf[ab], aph, abort_flag, p.err, wlim);
       got = __shfl_sync(0xffffffffu, got ? 1 : 0, 0) != 0;
       if (!got) break;   // warp-uniform: tcgen05.ld below is .sync.aligned
       if (t == (int)blockIdx.x && warp == 2 && lane == 0) TC_TRACE(5);

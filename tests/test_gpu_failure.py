@@ -65,9 +65,10 @@ def test_short_wait_limit_times_out_prompt_pass_and_recovers():
 
 
 def test_short_wait_limit_times_out_stream_k_generation_step_and_recovers():
-    # every GEMM of a generation step streams >= 8 MB here (the stream-K kernel)
-    cfg = synth.ModelConfig(family=synth.LLAMA, n_layers=4, d_model=2048, n_heads=16, head_dim=128, d_ffn=5504,
-                            vocab=3000, dtype="bf16", hsm_m1=4096, hsm_m2=16384, max_batch=1, max_seq=32,
+    # the wide GEMMs of a generation step (QKV, gate/up, mapper FC2, head, fills) take the
+    # stream-K kernel here
+    cfg = synth.ModelConfig(family=synth.LLAMA, n_layers=4, d_model=2048, n_heads=24, head_dim=128, d_ffn=5504,
+                            vocab=9000, dtype="bf16", hsm_m1=4096, hsm_m2=16384, max_batch=1, max_seq=32,
                             max_pass_tokens=32)
     W = synth.make_weights(cfg, seed=51, device="cuda")
     pair = Pair(cfg, weights=W)

@@ -1,10 +1,11 @@
 """The stream-K weight-streaming GEMM (generation steps and small fills) against the oracle.
 
-The model is sized so that every GEMM of a generation step streams at least 8 MB of weights
-and takes the stream-K kernel: a Llama-family decoder with D = 2048, 16 heads x 128, SwiGLU
-5504 (K = 5504 ends in a half k-block), the 36 D^2 mapper (FC widths 4096 / 16384, so FC3 has
-K = 16384 and the large-shared-memory ring), and a 3000-token vocabulary (the head's last
-32-feature tile is ragged).  Batches of 1, 5 and 12 sequences cover one and two 8-token
+The model is sized so that the wide GEMMs of a generation step (at least 8 MB of weights and
+8192 outputs) take the stream-K kernel: a Llama-family decoder with D = 2048, 24 heads x 128
+(QKV 9216 outputs), SwiGLU 5504 (gate/up 11008 outputs; K = 5504 of the down projection ends in
+a half k-block), the 36 D^2 mapper (FC2 has 16384 outputs), a 9000-token vocabulary (the head's
+last 32-feature tile is ragged) and the grouped fills (6144 outputs per layer); the narrower
+products take the cluster K-split kernel.  Batches of 1, 5 and 12 sequences cover one and two 8-token
 blocks of the A operand.  Generation steps (forced exits through every layer, the mapper,
 the grouped skipped-layer fill and the head) are compared with the oracle, with the cluster
 K-split kernel, and with themselves run again (the split tiles are summed in a fixed order, so
@@ -24,8 +25,8 @@ pytestmark = pytest.mark.gpu
 
 
 def _cfg(B):
-    return synth.ModelConfig(family=synth.LLAMA, n_layers=4, d_model=2048, n_heads=16, head_dim=128, d_ffn=5504,
-                             vocab=3000, dtype="bf16", hsm_m1=4096, hsm_m2=16384, max_batch=B, max_seq=48,
+    return synth.ModelConfig(family=synth.LLAMA, n_layers=4, d_model=2048, n_heads=24, head_dim=128, d_ffn=5504,
+                             vocab=9000, dtype="bf16", hsm_m1=4096, hsm_m2=16384, max_batch=B, max_seq=48,
                              max_pass_tokens=B * 40, block_shuffle_seed=9)
 
 
