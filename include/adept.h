@@ -234,10 +234,14 @@ ADEPT_API adept_status adept_check_device_status(adept_model* m, void* stream);
  * rows (generation steps, output heads) of bf16 models run on the weight-streaming
  * generation-step kernel, with the input standardisation fused in; 0 routes them to the
  * tcgen05 kernel after a separate standardisation launch.  DECODE_STREAM (default 1): those
- * weight-streaming GEMMs whose weights are large enough to stream (at least 8 MB) and whose
- * rows fit in shared memory run on the stream-K kernel (equal shares of the weight stream per
- * SM, split tiles finished by the last CTA to arrive); 0 keeps them on the cluster K-split
- * kernel.  EXIT_METRIC (App. H.3): 0 (default) the global similarity of Sec. 4.1,
+ * weight-streaming GEMMs that are wide (at least 8192 outputs, or a grouped fill) and large
+ * enough to stream (at least 8 MB of weights), and whose rows fit in shared memory, run on the
+ * stream-K kernel (equal shares of the weight stream per SM, split tiles finished by the last
+ * CTA to arrive); 0 keeps every one of them on the cluster K-split kernel.  DECODE_TILED (default 1): bf16 decoders keep a tile-contiguous copy of every streamed
+ * weight (layer projections, LM head, the mapper's FC weights; made at load, refreshed after
+ * each mapper training step; it doubles the weights' device memory) from which the weight-
+ * streaming kernels fetch each 32-row x 256-k unit with one contiguous bulk copy; 0 makes them
+ * read the row-major weights through tensor maps instead.  EXIT_METRIC (App. H.3): 0 (default) the global similarity of Sec. 4.1,
  * cos(s_i, sum_{d<i} s_hat_d); 1 the local similarity cos(s_i, s_{i-1}); 2 both (a token leaves
  * when both reach delta; the reported similarity is their minimum).  ALL_AT_ONCE (App. H.2):
  * 1 makes every token of a prompt take the exit decision of its sequence's last prompt token,
@@ -247,7 +251,7 @@ ADEPT_API adept_status adept_check_device_status(adept_model* m, void* stream);
  * only the tokens still active there; its mapped state still feeds the classifier.  Default 0. */
 enum { ADEPT_OPT_HSM_IDENTITY = 1, ADEPT_OPT_PROFILE = 2, ADEPT_OPT_GEMM_SIMT = 3, ADEPT_OPT_DECODE_GRAPH = 4,
        ADEPT_OPT_DECODE_GEMM = 5, ADEPT_OPT_EXIT_METRIC = 7, ADEPT_OPT_ALL_AT_ONCE = 8,
-       ADEPT_OPT_STOP_ENTIRELY = 9, ADEPT_OPT_DECODE_STREAM = 10 };
+       ADEPT_OPT_STOP_ENTIRELY = 9, ADEPT_OPT_DECODE_STREAM = 10, ADEPT_OPT_DECODE_TILED = 11 };
 ADEPT_API adept_status adept_set_option(adept_model* m, int option, int value);
 
 /* Kernel classes reported by adept_profile_read: the GEMMs of prompt passes (layer

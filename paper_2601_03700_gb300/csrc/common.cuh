@@ -317,6 +317,17 @@ struct GemmProblem {
   // rows on the device that are usually far below their bound (the prompt pass's exiting
   // rows): the tensor-core launcher may split the problem by the live count
   int split_live = 0;
+  // Optional tile-contiguous copy of B for the weight-streaming kernels (NULL: none): 16 KB
+  // units, one per (32-row tile, 256-k block), tile-major, each laid out as the kernels' shared-
+  // memory stage (four 64-k chunks of 32 rows x 128 B, 16-byte pieces XOR-swizzled by row & 7,
+  // zero past N and K), so that a unit, or a run of its chunks, is one contiguous bulk copy.
+  const void* Bt = nullptr;
+  int bt_nkb = 0;   // 256-k blocks per tile of Bt
 };
+
+static inline int cdiv_h(int a, int b) { return (a + b - 1) / b; }
+// Tile-contiguous weight layout (GemmProblem::Bt).
+constexpr int TW_ROWS = 32, TW_KB = 256, TW_UNIT = TW_ROWS * TW_KB * 2;
+static inline size_t tiled_bytes(int N, int K) { return (size_t)cdiv_h(N, TW_ROWS) * cdiv_h(K, TW_KB) * TW_UNIT; }
 
 static inline int cdiv(int a, int b) { return (a + b - 1) / b; }

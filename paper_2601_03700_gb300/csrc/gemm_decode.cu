@@ -69,6 +69,8 @@ constexpr int DG_SMEM_LIMIT = 227 * 1024 - DG_STATIC_SMEM;   // dynamic shared m
 
 struct DgParams {
   CUtensorMap wmap;     // W as {64, N, K/64}, box {64, 32, 2}, 128-byte swizzle
+  const uint8_t* bt;    // tile-contiguous copy of W (GemmProblem::Bt) or NULL
+  int bt_nkb;           // its 256-k blocks per 32-row tile
   const bf16* W;
   int ldw;
   const bf16* A;
@@ -105,10 +107,13 @@ struct DgParams {
 constexpr int DG_MAX_GROUPS = 32;
 struct DgParamsG : DgParams {
   CUtensorMap gmap[DG_MAX_GROUPS];
+  const uint8_t* gbt[DG_MAX_GROUPS];
   DevRange grows[DG_MAX_GROUPS];
   Epi gepi[DG_MAX_GROUPS];
 };
 __device__ __forceinline__ const CUtensorMap* dg_wmap(const DgParams& p) { return &p.wmap; }
+__device__ __forceinline__ const uint8_t* dg_bt(const DgParams& p) { return p.bt; }
+__device__ __forceinline__ const uint8_t* dg_bt(const DgParamsG& p) { return p.gbt[blockIdx.y]; }
 __device__ __forceinline__ const CUtensorMap* dg_wmap(const DgParamsG& p) { return &p.gmap[blockIdx.y]; }
 __device__ __forceinline__ DevRange dg_rows(const DgParams& p) { return p.rows; }
 __device__ __forceinline__ DevRange dg_rows(const DgParamsG& p) { return p.grows[blockIdx.y]; }
@@ -171,6 +176,13 @@ __device__ __forceinline__ void st_async_v4(float* dst, const float4& v, uint64_
   asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(rb) : "r"(smem_u32(bar)), "r"(rank));
   asm volatile("st.async.shared::cluster.mbarrier::complete_tx::bytes.v4.f32 [%0], {%1, %2, %3, %4}, [%5];" ::"r"(rd),
                "f"(v.x), "f"(v.y), "f"(v.z), "f"(v.w), "r"(rb)
+               : "memory");
+}
+// 1-D bulk copy of `bytes` contiguous bytes (16-byte aligned, a multiple of 16), completing on bar.
+__device__ __forceinline__ void bulk_load(void* dst, const void* src, uint32_t bytes, uint64_t* bar) {
+  asm volatile("cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(
+                   smem_u32(dst)),
+               "l"(src), "r"(bytes), "r"(smem_u32(bar))
                : "memory");
 }
 __device__ __forceinline__ void cp_async16(void* dst, const void* src) {
@@ -267,7 +279,15 @@ __global__ void __launch_bounds__(DG_THREADS, 1) gemm_decode_kernel(const __grid
     const int f = (tile0 + j * tstride) * DG_BN;
     const int s = g % S;
     mbar_expect_tx(&full[s], (uint32_t)stage_bytes);
-    tma_load_3d(dg_wmap(p), &full[s], sW + (size_t)s * stage_bytes, f, (k_lo + kb * ks) >> 6);
+    const uint8_t* bt = dg_bt(p);
+    if (bt) {   // the stage's chunks are contiguous within one 16 KB unit of the tiled copy
+      const int k = k_lo + kb * ks;
+      bulk_load(sW + (size_t)s * stage_bytes,
+                bt + ((size_t)(f >> 5) * p.bt_nkb + (k >> 8)) * (32 * 256 * 2) + ((k & 255) >> 6) * DG_CHUNK,
+                (uint32_t)stage_bytes, &full[s]);
+    } else {
+      tma_load_3d(dg_wmap(p), &full[s], sW + (size_t)s * stage_bytes, f, (k_lo + kb * ks) >> 6);
+    }
   };
   const int first = min(S, G);
   const int pre = min(p.pre, first);
@@ -533,11 +553,9 @@ __global__ void __launch_bounds__(DG_THREADS, 1) gemm_decode_kernel(const __grid
 #ifdef ADEPT_KTRACE
       const unsigned long long tw = kt_now();
 #endif
-      // lane 0 waits and broadcasts: the MMAs below are .aligned, so the warp decides as one
-      bool ok = true;
-      if (lane == 0) ok = dg_wait(&full[s], (uint32_t)((g / S) & 1), p.err, wlim);
-      ok = __shfl_sync(0xffffffffu, ok ? 1 : 0, 0) != 0;
-      __syncwarp();
+      // every lane polls (it leaves the wait as soon as the stage lands); one vote makes the
+      // outcome warp-uniform, since the MMAs below are .aligned
+      const bool ok = __all_sync(0xffffffffu, dg_wait(&full[s], (uint32_t)((g / S) & 1), p.err, wlim)) != 0;
 #ifdef ADEPT_KTRACE
       KT_ADD(7, kt_now() - tw);
 #endif
@@ -879,6 +897,14 @@ static bool dg_plan(const GemmProblem& q, int max_rows, const DgNorm* norm, int 
   return true;
 }
 
+// The problem's tile-contiguous copy when every stage of the plan lies inside one unit of it (a
+// k-range starting on a multiple of the stage width, which divides 256), else NULL.
+static const uint8_t* dg_tiled(const GemmProblem& q, const DgParams& prm) {
+  if (!q.Bt || q.bt_nkb != cdiv(q.K, 256) || ((uintptr_t)q.Bt & 15)) return nullptr;
+  if (256 % prm.ks || prm.kr % prm.ks) return nullptr;
+  return (const uint8_t*)q.Bt;
+}
+
 int decode_gemm(cudaStream_t st, const GemmProblem& q, int max_rows, const DgNorm* norm, unsigned* err) {
   thread_local DgParams prm;   // 64-byte-aligned tensor map; one per host thread
   memset(&prm, 0, sizeof prm);
@@ -886,6 +912,8 @@ int decode_gemm(cudaStream_t st, const GemmProblem& q, int max_rows, const DgNor
   size_t smem = 0;
   if (!dg_plan(q, max_rows, norm, 1, err, prm, grid, smem, mb)) return -1;
   if (!tc_encode_weight_3d(&prm.wmap, q.B, q.K, q.N, (size_t)q.ldb * 2, DG_BN, prm.ks / 64)) return -1;
+  prm.bt = dg_tiled(q, prm);
+  prm.bt_nkb = q.bt_nkb;
   const cudaError_t e = mb == 2 ? launch_kind<2>(st, prm, grid, smem) : launch_kind<1>(st, prm, grid, smem);
   return e == cudaSuccess ? 1 : -1;
 }
@@ -910,6 +938,11 @@ int decode_gemm_grouped(cudaStream_t st, const GemmProblem* probs, int n, int ma
     prm.gepi[i] = probs[i].epi;
     prm.gepi[i].tile_stats = nullptr;
   }
+  // the tiled copies, if every problem of the launch has one (all problems read the same way)
+  bool all_tiled = true;
+  for (int i = 0; i < n; ++i) all_tiled &= dg_tiled(probs[i], prm) != nullptr;
+  for (int i = 0; i < n; ++i) prm.gbt[i] = all_tiled ? dg_tiled(probs[i], prm) : nullptr;
+  prm.bt_nkb = q0.bt_nkb;
   prm.bias_aligned = 1;
   for (int i = 0; i < n; ++i) prm.bias_aligned &= ((uintptr_t)probs[i].epi.bias & 15) == 0;
   const cudaError_t e = mb == 2 ? launch_dg_grouped<2>(st, prm, grid, n, smem) : launch_dg_grouped<1>(st, prm, grid, n, smem);

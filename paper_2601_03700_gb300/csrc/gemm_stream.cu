@@ -63,6 +63,8 @@ enum : int { DS_STATS_HERE = 0, DS_STATS_ROWS = 1, DS_STATS_TILES = 2 };
 template <int MAXG>
 struct DsParams {
   CUtensorMap wmap[MAXG];   // W as {64, N, K/64}, box {64, 32, 4}, 128-byte swizzle
+  const uint8_t* bt[MAXG];  // tile-contiguous copy of W (GemmProblem::Bt) or NULL: the unit of
+                            // (tile t, k-block kb) is the 16 KB at bt + (t * nkb + kb) * 16 KB
   DevRange rows[MAXG];
   Epi epi[MAXG];
   int n_probs;
@@ -128,6 +130,13 @@ __device__ __forceinline__ void tma_load_3d(const CUtensorMap* tm, uint64_t* bar
           "r"(smem_u32(dst)),
       "l"((uint64_t)tm), "r"(0), "r"(y), "r"(z), "r"(smem_u32(bar))
       : "memory");
+}
+// 1-D bulk copy of `bytes` contiguous bytes (16-byte aligned, a multiple of 16), completing on bar.
+__device__ __forceinline__ void bulk_load(void* dst, const void* src, uint32_t bytes, uint64_t* bar) {
+  asm volatile("cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(
+                   smem_u32(dst)),
+               "l"(src), "r"(bytes), "r"(smem_u32(bar))
+               : "memory");
 }
 __device__ __forceinline__ void cp_async16(void* dst, const void* src) {
   asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(smem_u32(dst)), "l"(src) : "memory");
@@ -442,7 +451,11 @@ __global__ void __launch_bounds__(DS_THREADS, 2) gemm_stream_kernel(const __grid
   };
   auto issue = [&](const Cur& r, int q, int s) {
     mbar_expect_tx(&full[s], (uint32_t)DS_STAGE);
-    tma_load_3d(&p.wmap[q], &full[s], sW + (size_t)s * DS_STAGE, r.t * DS_BN, r.kb * (DS_KB / 64));
+    if (p.bt[q])   // one contiguous 16 KB unit of the tiled copy
+      bulk_load(sW + (size_t)s * DS_STAGE, p.bt[q] + ((size_t)r.t * nkb + r.kb) * DS_STAGE, (uint32_t)DS_STAGE,
+                &full[s]);
+    else
+      tma_load_3d(&p.wmap[q], &full[s], sW + (size_t)s * DS_STAGE, r.t * DS_BN, r.kb * (DS_KB / 64));
   };
 
   // single problem: the partition is known before the wait and the whole ring is issued
@@ -648,7 +661,7 @@ __global__ void __launch_bounds__(DS_THREADS, 2) gemm_stream_kernel(const __grid
   zero_acc();
   Cur r = cur_at(u0);
 
-  // Lane 0 waits for each slot and broadcasts, so the decision is warp-uniform (the fragment
+  // Every lane waits for each slot and one vote makes the decision warp-uniform (the fragment
   // loads and MMAs below are .aligned).  A warp whose wait gives up stops waiting, computing and
   // releasing slots (a slot it has not seen land must not be refilled: the producer's own
   // bounded wait then ends the stream and it drains its copies), but still hands over every
@@ -659,12 +672,8 @@ __global__ void __launch_bounds__(DS_THREADS, 2) gemm_stream_kernel(const __grid
   int s = 0, n = 0;                   // slot and use number of unit g
   int j = 0;                          // tile hand-offs so far
   for (int g = 0; g < n_units; ++g) {
-    if (ok) {
-      bool landed = true;
-      if (lane == 0) landed = ds_wait(&full[s], (uint32_t)(n & 1), p.err, wlim);
-      ok = __shfl_sync(0xffffffffu, landed ? 1 : 0, 0) != 0;
-      __syncwarp();   // lane 0's acquire orders the whole warp's reads of the slot
-    }
+    if (ok)   // every lane polls; one vote makes the outcome warp-uniform (.aligned MMAs below)
+      ok = __all_sync(0xffffffffu, ds_wait(&full[s], (uint32_t)(n & 1), p.err, wlim)) != 0;
     const int kb = r.kb;
     const int nch = ok ? min(DS_KB, Kd - kb * DS_KB) >> 6 : 0;
     const uint32_t sbase = w_base + s * DS_STAGE;
@@ -860,6 +869,13 @@ bool ds_plan(const GemmProblem& q, int n_probs, int max_rows, const DgNorm* norm
   return smem <= (size_t)DS_SMEM_LIMIT;
 }
 
+// The problem's tile-contiguous copy when its layout matches the launch (k-blocks per tile,
+// 16-byte alignment), else NULL (the tensor map on B is used).
+const uint8_t* ds_tiled(const GemmProblem& q, int nkb) {
+  if (!q.Bt || q.bt_nkb != nkb || ((uintptr_t)q.Bt & 15)) return nullptr;
+  return (const uint8_t*)q.Bt;
+}
+
 }  // namespace
 
 size_t stream_gemm_part_bytes(int sms) { return (size_t)2 * sms * 16 * DS_BN * sizeof(float); }
@@ -871,6 +887,7 @@ int stream_gemm(cudaStream_t st, const GemmProblem& q, int max_rows, const DgNor
   size_t smem = 0;
   if (!ds_plan(q, 1, max_rows, norm, ws, err, prm, grid, smem, mb)) return -1;
   if (!tc_encode_weight_3d(&prm.wmap[0], q.B, q.K, q.N, (size_t)q.ldb * 2, DS_BN, DS_KB / 64)) return -1;
+  prm.bt[0] = ds_tiled(q, prm.nkb);
   prm.grouped = 0;
   prm.rows[0] = q.rows;
   prm.epi[0] = q.epi;
@@ -898,6 +915,7 @@ int stream_gemm_grouped(cudaStream_t st, const GemmProblem* probs, int n, int ma
       return -1;
     prm.rows[i] = probs[i].rows;
     prm.epi[i] = probs[i].epi;
+    prm.bt[i] = ds_tiled(probs[i], prm.nkb);
   }
   prm.grouped = 1;
   const cudaError_t e = mb == 2 ? ds_launch<2, EPI_KV, DS_MAXG>(st, prm, grid, smem)

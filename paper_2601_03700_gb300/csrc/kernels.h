@@ -88,6 +88,9 @@ void launch_fill_sort(cudaStream_t st, int dt, const void* h, int n, int D, cons
 void launch_fold_rows(cudaStream_t st, int dt, void* dst, int ld_dst, const void* src, int n_rows, int K,
                       const float* gamma, const float* beta, const float* bias_in, float* bias_out, int row_mode);
 void launch_to_f32(cudaStream_t st, int dt, const void* src, float* dst, int n);
+// Writes the tile-contiguous copy (GemmProblem::Bt layout, tiled_bytes(N, K) bytes) of the
+// row-major bf16 matrix src [N][K] (row stride ld elements) into dst.
+void launch_tile_weight(cudaStream_t st, const void* src, int N, int K, int ld, void* dst);
 void launch_read_kv(cudaStream_t st, int dt, KVCacheView c, int layer0, int seq, int pos0, int n_pos, void* ko,
                     void* vo);
 

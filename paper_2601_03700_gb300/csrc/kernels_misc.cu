@@ -1590,6 +1590,32 @@ void launch_read_kv(cudaStream_t st, int dt, KVCacheView c, int layer0, int seq,
   else launch_k(read_kv_kernel<float>, n_pos, 256, 0, st, c, layer0, seq, pos0, n_pos, (float*)ko, (float*)vo);
 }
 
+// Tile-contiguous weight copy: one thread per 16-byte piece of the destination.  Piece q of
+// unit (tile t, k-block kb) sits at chunk c, row r, physical position u; it holds the 8 values of
+// row t*32 + r at k = kb*256 + c*64 + (u ^ (r & 7))*8 (the swizzle the stage's 128-byte rows
+// carry), zeros past N or K.
+__global__ void tile_weight_kernel(const bf16* __restrict__ src, int N, int K, int ld, int nkb, long long pieces,
+                                   uint4* __restrict__ dst) {
+  const long long q = (long long)blockIdx.x * blockDim.x + threadIdx.x;
+  if (q >= pieces) return;
+  const long long unit = q >> 10;           // 1024 pieces of 16 B per unit
+  const int w = (int)(q & 1023);
+  const int c = w >> 8, r = (w >> 3) & 31, u = w & 7;
+  const int t = (int)(unit / nkb), kb = (int)(unit - (long long)t * nkb);
+  const int n = t * 32 + r, k = kb * 256 + c * 64 + ((u ^ (r & 7)) << 3);
+  uint4 v = make_uint4(0u, 0u, 0u, 0u);
+  if (n < N && k < K) v = *reinterpret_cast<const uint4*>(src + (size_t)n * ld + k);   // K % 8 == 0
+  dst[q] = v;
+}
+
+void launch_tile_weight(cudaStream_t st, const void* src, int N, int K, int ld, void* dst) {
+  const int nkb = cdiv(K, TW_KB);
+  const long long pieces = (long long)cdiv(N, TW_ROWS) * nkb * (TW_UNIT / 16);
+  const int threads = 256;
+  tile_weight_kernel<<<(unsigned)((pieces + threads - 1) / threads), threads, 0, st>>>((const bf16*)src, N, K, ld, nkb,
+                                                                                       pieces, (uint4*)dst);
+}
+
 ADEPT_KTRACE_ATTACH(misc)
 
 }  // namespace adept

@@ -42,6 +42,8 @@ struct LayerW {
   void* w_down = nullptr; // [D, F]
   float* b_down = nullptr;
   float *ln1_g = nullptr, *ln1_b = nullptr, *ln2_g = nullptr, *ln2_b = nullptr;  // post-LN (encoder)
+  // tile-contiguous copies for the weight-streaming kernels (bf16 decoders; GemmProblem::Bt)
+  void *t_qkv = nullptr, *t_o = nullptr, *t_up = nullptr, *t_down = nullptr;
 };
 
 struct ProfRec {
@@ -96,6 +98,8 @@ struct adept_model {
   float *hsm_g0 = nullptr, *hsm_conv = nullptr, *hsm_g1 = nullptr, *hsm_g2 = nullptr;
   float *hsm_b1 = nullptr, *hsm_b2 = nullptr, *hsm_b3 = nullptr, *hsm_b4 = nullptr;
   void *hsm_w1 = nullptr, *hsm_w2 = nullptr, *hsm_w3 = nullptr, *hsm_w4 = nullptr;
+  // tile-contiguous copies of the head and the mapper's FC weights (bf16 decoders)
+  void *t_head = nullptr, *t_hsm1 = nullptr, *t_hsm2 = nullptr, *t_hsm3 = nullptr, *t_hsm4 = nullptr;
   float2* rope_table = nullptr;
   // paged KV cache
   void *k_pool = nullptr, *v_pool = nullptr;
@@ -146,7 +150,7 @@ struct adept_model {
   std::vector<cudaGraphExec_t> dec_graph;   // per batch size
   std::vector<int> dec_warm;                // direct runs done per batch size
   // options / instrumentation
-  int hsm_identity = 0, profile = 0, force_simt = 0, use_graph = 1, use_dg = 1, use_stream = 1;
+  int hsm_identity = 0, profile = 0, force_simt = 0, use_graph = 1, use_dg = 1, use_stream = 1, use_tiled = 1;
   int exit_metric = 0;   // EXIT_GLOBAL / EXIT_LOCAL / EXIT_BOTH
   int all_at_once = 0;   // prompt passes: sequences leave with their last prompt token
   int stop_entirely = 0; // encoders: exited tokens get no deeper K/V and leave deeper attention
@@ -324,13 +328,22 @@ static DsWork ds_work(const adept_model* m) {
 // A weight-streaming problem of at most DG_MAX_M rows: the stream-K kernel where it takes the
 // shape (weights large enough to stream, A rows fitting in shared memory), else the cluster
 // K-split kernel.  Returns the launches, or -1 when neither takes it.
-static int streaming_gemm(adept_model* m, cudaStream_t st, const GemmProblem& p, int max_rows, const DgNorm* norm) {
+static int streaming_gemm(adept_model* m, cudaStream_t st, const GemmProblem& p0, int max_rows, const DgNorm* norm) {
+  GemmProblem p = p0;
+  if (!m->use_tiled) p.Bt = nullptr;
   if (stream_gemm(st, p, max_rows, norm, ds_work(m), m->err_word) >= 0) return 1;
   return decode_gemm(st, p, max_rows, norm, m->err_word);
 }
 
 // The grouped skipped-layer fill of a few tokens on the weight-streaming kernels.
-static int streaming_gemm_grouped(adept_model* m, cudaStream_t st, const GemmProblem* probs, int n, int max_rows) {
+static int streaming_gemm_grouped(adept_model* m, cudaStream_t st, const GemmProblem* probs0, int n, int max_rows) {
+  std::vector<GemmProblem> copy;
+  const GemmProblem* probs = probs0;
+  if (!m->use_tiled) {
+    copy.assign(probs0, probs0 + n);
+    for (auto& q : copy) q.Bt = nullptr;
+    probs = copy.data();
+  }
   if (stream_gemm_grouped(st, probs, n, max_rows, ds_work(m), m->err_word) >= 0) return 1;
   return max_rows <= DG_FILL_MAX_ROWS ? decode_gemm_grouped(st, probs, n, max_rows, m->err_word) : -1;
 }
@@ -738,6 +751,50 @@ static adept_status alloc_runtime(adept_model* m) {
   return ADEPT_OK;
 }
 
+// Tile-contiguous copies of the streamed weights (bf16 decoders): every layer projection, the
+// LM head and the mapper's four FC matrices, for the weight-streaming kernels of generation
+// steps and small fills (contiguous 16 KB units instead of 32 row segments per copy).  The
+// row-major weights stay for the tensor-core prompt pass and the mapper's training.
+static adept_status tile_into(adept_model* m, cudaStream_t st, const void* src, int N, int K, void** dst) {
+  TRY(dalloc(m, dst, tiled_bytes(N, K)));
+  launch_tile_weight(st, src, N, K, K, *dst);
+  return ADEPT_OK;
+}
+
+static adept_status retile_hsm(adept_model* m, cudaStream_t st, bool alloc);
+static adept_status make_tiled(adept_model* m, cudaStream_t st) {
+  if (m->dt != ADEPT_DTYPE_BF16 || m->cfg.family == ADEPT_FAMILY_BERT) return ADEPT_OK;
+  const int D = m->D, Dq = m->Dq, Dkv = m->Dkv, F = m->F;
+  for (int l = 0; l < m->N; ++l) {
+    LayerW& w = m->L[l];
+    TRY(tile_into(m, st, w.w_qkv, Dq + 2 * Dkv, D, &w.t_qkv));
+    TRY(tile_into(m, st, w.w_o, D, Dq, &w.t_o));
+    TRY(tile_into(m, st, w.w_up, w.up_rows, D, &w.t_up));
+    TRY(tile_into(m, st, w.w_down, D, F, &w.t_down));
+  }
+  TRY(tile_into(m, st, m->w_head, m->V, D, &m->t_head));
+  return retile_hsm(m, st, true);
+}
+
+// The mapper's tiled copies from its row-major weights (at load; after every training step).
+static adept_status retile_hsm(adept_model* m, cudaStream_t st, bool alloc) {
+  if (!alloc && !m->t_hsm1) return ADEPT_OK;
+  const int D = m->D, m1 = m->m1, m2 = m->m2;
+  if (alloc) {
+    TRY(tile_into(m, st, m->hsm_w1, m1, D, &m->t_hsm1));
+    TRY(tile_into(m, st, m->hsm_w2, m2, m1, &m->t_hsm2));
+    TRY(tile_into(m, st, m->hsm_w3, m1, m2, &m->t_hsm3));
+    TRY(tile_into(m, st, m->hsm_w4, D, m1, &m->t_hsm4));
+  } else {
+    launch_tile_weight(st, m->hsm_w1, m1, D, D, m->t_hsm1);
+    launch_tile_weight(st, m->hsm_w2, m2, m1, m1, m->t_hsm2);
+    launch_tile_weight(st, m->hsm_w3, m1, m2, m2, m->t_hsm3);
+    launch_tile_weight(st, m->hsm_w4, D, m1, m1, m->t_hsm4);
+    m->launches += 4;
+  }
+  return ADEPT_OK;
+}
+
 // ---------------------------------------------------------------------------
 // sequences and KV blocks
 // ---------------------------------------------------------------------------
@@ -790,23 +847,23 @@ static void run_hsm(adept_model* m, cudaStream_t st, DevRange rows, int max_rows
   p.a_rows = a_rows;
   p.split_live = 1;   // the exiting rows of one layer: usually a small part of the pass
   // FC1: h1 = GELU(W1 c0 + b1)
-  p.A = m->c0t; p.lda = D; p.B = m->hsm_w1; p.ldb = D; p.N = m1; p.K = D;
+  p.A = m->c0t; p.lda = D; p.B = m->hsm_w1; p.ldb = D; p.N = m1; p.K = D; p.Bt = m->t_hsm1; p.bt_nkb = cdiv(D, TW_KB);
   p.epi = epi_base(); p.epi.kind = EPI_ACT; p.epi.act = ACT_GELU_ERF; p.epi.bias = m->hsm_b1;
   p.epi.out_t = m->h1t; p.epi.ld_t = m1; p.epi.out_f32 = m->h1f; p.epi.ld_f32 = m1;
   gemm(m, st, &p, 1, &max_rows, m->gemm_cls);
   // FC2: h2 = GELU(W2 h1 + b2)
-  p.A = m->h1t; p.lda = m1; p.B = m->hsm_w2; p.ldb = m1; p.N = m2; p.K = m1;
+  p.A = m->h1t; p.lda = m1; p.B = m->hsm_w2; p.ldb = m1; p.N = m2; p.K = m1; p.Bt = m->t_hsm2; p.bt_nkb = cdiv(m1, TW_KB);
   p.epi = epi_base(); p.epi.kind = EPI_ACT; p.epi.act = ACT_GELU_ERF; p.epi.bias = m->hsm_b2;
   p.epi.out_t = m->h2t; p.epi.ld_t = m2;
   gemm(m, st, &p, 1, &max_rows, m->gemm_cls);
   // FC3: h3 = W3 h2 + b3
-  p.A = m->h2t; p.lda = m2; p.B = m->hsm_w3; p.ldb = m2; p.N = m1; p.K = m2;
+  p.A = m->h2t; p.lda = m2; p.B = m->hsm_w3; p.ldb = m2; p.N = m1; p.K = m2; p.Bt = m->t_hsm3; p.bt_nkb = cdiv(m2, TW_KB);
   p.epi = epi_base(); p.epi.kind = EPI_F32; p.epi.bias = m->hsm_b3; p.epi.out_f32 = m->h3f; p.epi.ld_f32 = m1;
   gemm(m, st, &p, 1, &max_rows, m->gemm_cls);
   launch_hsm_mid(st, m->dt, m->h3f, m->h1f, rows, max_rows, m1, m->hsm_g1, eps, m->h4t);
   m->launches += 1;
   // FC4: h5 = W4 h4 + b4
-  p.A = m->h4t; p.lda = m1; p.B = m->hsm_w4; p.ldb = m1; p.N = D; p.K = m1;
+  p.A = m->h4t; p.lda = m1; p.B = m->hsm_w4; p.ldb = m1; p.N = D; p.K = m1; p.Bt = m->t_hsm4; p.bt_nkb = cdiv(m1, TW_KB);
   p.epi = epi_base(); p.epi.kind = EPI_F32; p.epi.bias = m->hsm_b4; p.epi.out_f32 = m->h5f; p.epi.ld_f32 = D;
   gemm(m, st, &p, 1, &max_rows, m->gemm_cls);
   launch_hsm_out(st, m->dt, m->h5f, m->c0f, m->hsm_s, 0, rows, max_rows, D, m->hsm_g2, eps, m->exit_tok, m->final_,
@@ -822,6 +879,10 @@ static GemmProblem kv_problem(adept_model* m, int layer0, const void* xs, int a_
   const LayerW& w = m->L[layer0];
   p.A = xs; p.lda = m->D; p.a_rows = a_rows;
   p.B = (const char*)w.w_qkv + (size_t)m->Dq * m->D * m->esz; p.ldb = m->D;
+  if (w.t_qkv && m->Dq % TW_ROWS == 0) {   // the K/V rows start at a whole tile of the copy
+    p.bt_nkb = cdiv(m->D, TW_KB);
+    p.Bt = (const char*)w.t_qkv + (size_t)(m->Dq / TW_ROWS) * p.bt_nkb * TW_UNIT;
+  }
   p.rows = rows; p.N = 2 * m->Dkv; p.K = m->D;
   p.epi = epi_base();
   p.epi.kind = EPI_KV; p.epi.bias = w.b_qkv + m->Dq;
@@ -887,7 +948,7 @@ static adept_status run_pass(adept_model* m, int n_tok, int batch, int prompt_le
     int mrs[2] = {mr, mr};
     memset(pr, 0, sizeof pr);
     pr[0].A = m->xn; pr[0].lda = D; pr[0].a_rows = n_tok; pr[0].B = w.w_qkv; pr[0].ldb = D; pr[0].rows = act;
-    pr[0].N = Dq + 2 * Dkv; pr[0].K = D;
+    pr[0].N = Dq + 2 * Dkv; pr[0].K = D; pr[0].Bt = w.t_qkv; pr[0].bt_nkb = cdiv(D, TW_KB);
     pr[0].epi = epi_base();
     pr[0].epi.kind = EPI_QKV; pr[0].epi.bias = w.b_qkv; pr[0].epi.out_t = m->q; pr[0].epi.ld_t = Dq;
     pr[0].epi.row_tok = rt; pr[0].epi.tok_seq = m->tok_seq; pr[0].epi.tok_pos = m->tok_pos;
@@ -921,6 +982,7 @@ static adept_status run_pass(adept_model* m, int n_tok, int batch, int prompt_le
     memset(&p, 0, sizeof p);
     p.a_rows = n_tok;   // the TMA view ends at this pass's rows: tiles past them read zeros, not memory
     p.A = m->att; p.lda = Dq; p.B = w.w_o; p.ldb = Dq; p.rows = act; p.N = D; p.K = Dq;
+    p.Bt = w.t_o; p.bt_nkb = cdiv(Dq, TW_KB);
     p.epi = epi_base(); p.epi.kind = EPI_RESID; p.epi.bias = w.b_o; p.epi.out_f32 = m->X_out; p.epi.ld_f32 = D;
     p.epi.resid = Xi; p.epi.ld_resid = D;
     bool ts_valid = false;   // the O projection leaves the tile statistics of X_out for the FFN input
@@ -936,6 +998,7 @@ static adept_status run_pass(adept_model* m, int n_tok, int batch, int prompt_le
     }
     // FFN (input standardised)
     p.A = m->xn; p.lda = D; p.B = w.w_up; p.ldb = D; p.N = w.up_rows; p.K = D;
+    p.Bt = w.t_up; p.bt_nkb = cdiv(D, TW_KB);
     p.epi = epi_base();
     if (fam == ADEPT_FAMILY_LLAMA) {
       p.epi.kind = EPI_SWIGLU;
@@ -946,6 +1009,7 @@ static adept_status run_pass(adept_model* m, int n_tok, int batch, int prompt_le
     p.epi.bias = w.b_up; p.epi.out_t = m->hbuf; p.epi.ld_t = m->F;
     gemm_std(m, st, p, mr, m->X_out, D, nullptr, amode, eps, m->gemm_cls, nullptr, ts_valid ? m->tile_stats : nullptr);
     p.A = m->hbuf; p.lda = m->F; p.B = w.w_down; p.ldb = m->F; p.N = D; p.K = m->F;
+    p.Bt = w.t_down; p.bt_nkb = cdiv(m->F, TW_KB);
     p.epi = epi_base(); p.epi.kind = EPI_RESID; p.epi.bias = w.b_down; p.epi.out_f32 = m->X_out; p.epi.ld_f32 = D;
     p.epi.resid = m->X_out; p.epi.ld_resid = D;
     gemm(m, st, &p, 1, &mr, m->gemm_cls);
@@ -1034,6 +1098,7 @@ static adept_status run_head(adept_model* m, int batch, int prompt_len, bool dec
   p.a_rows = batch;
   if (!enc) {
     p.A = m->xhead; p.lda = D; p.B = m->w_head; p.ldb = D; p.rows = rows; p.N = m->V; p.K = D;
+    p.Bt = m->t_head; p.bt_nkb = cdiv(D, TW_KB);
     p.epi = epi_base(); p.epi.kind = EPI_F32; p.epi.bias = m->b_head; p.epi.out_f32 = out; p.epi.ld_f32 = m->V;
     if (rows_ready)
       gemm(m, st, &p, 1, &batch, m->gemm_cls);   // rows standardised by their producers
@@ -1330,6 +1395,7 @@ static adept_status ht_backward(adept_model* m, cudaStream_t st, int n, int nspl
   a.nseg = (int)(sizeof segs / sizeof segs[0]);
   for (int i = 0; i < a.nseg; ++i) a.seg[i] = segs[i];
   ht_launch_adamw(st, dt, a);
+  TRY(retile_hsm(m, st, false));   // the generation steps' copies follow the updated weights
   // launches outside ht_gemm: prep, 2 GELU, mid, out (forward), out_bwd, mid_bwd, 2 GELU', prep_bwd,
   // 4 transposes, the column sums and AdamW, and the caller's loss launches
   m->launches += 15 + launches + cl;
@@ -1438,6 +1504,7 @@ adept_status adept_model_load(const adept_config* cfg_in, const adept_tensor_tab
   }
   adept_status s = load_weights(m, ld);
   if (s == ADEPT_OK) s = alloc_runtime(m);
+  if (s == ADEPT_OK) s = make_tiled(m, ld.st);
   if (s == ADEPT_OK) {
     cudaError_t e = cudaStreamSynchronize(ld.st);
     if (e != cudaSuccess) s = fail(m, ADEPT_ERR_CUDA, "load: %s", cudaGetErrorString(e));
@@ -1709,6 +1776,7 @@ adept_status adept_set_option(adept_model* m, int option, int value) {
     case ADEPT_OPT_DECODE_GRAPH: m->use_graph = value != 0; drop_graphs(m); return ADEPT_OK;
     case ADEPT_OPT_DECODE_GEMM: m->use_dg = value != 0; drop_graphs(m); return ADEPT_OK;
     case ADEPT_OPT_DECODE_STREAM: m->use_stream = value != 0; drop_graphs(m); return ADEPT_OK;
+    case ADEPT_OPT_DECODE_TILED: m->use_tiled = value != 0; drop_graphs(m); return ADEPT_OK;
     case ADEPT_OPT_EXIT_METRIC:
       if (value < EXIT_GLOBAL || value > EXIT_BOTH) return fail(m, ADEPT_ERR_INVALID_ARG, "exit metric %d", value);
       m->exit_metric = value;

@@ -52,12 +52,13 @@ def test_stream_gemm_generation_steps_match_oracle(B):
     pair.close()
 
 
-def _steps(cfg, W, stream, repeat=1):
+def _steps(cfg, W, stream, repeat=1, tiled=1):
     B, P = cfg.max_batch, 40
     out = []
     for _ in range(repeat):
         m = adept.Model(cfg, W)
         adept.adept_set_option(m.h, adept.OPT_DECODE_STREAM, stream)
+        adept.adept_set_option(m.h, adept.OPT_DECODE_TILED, tiled)
         tokens = synth.make_tokens(42, B, P, cfg.vocab).cuda()
         forced = synth.forced_exits_uniform(42, B * P, 2, cfg.n_layers).view(B, P).cuda()
         m.prefill(tokens, 0.9, forced)
@@ -91,6 +92,23 @@ def test_stream_gemm_matches_cluster_kernel_and_repeats_bit_for_bit(B):
         assert row_rel_err(a[2], b[2]).max() < 2e-2
     for x, y in zip(new[0][1], old[1]):
         assert row_rel_err(x.reshape(len(x), -1), y.reshape(len(y), -1)).max() < 2e-2
+
+
+@pytest.mark.parametrize("B", [1, 5])
+def test_tile_contiguous_weights_give_identical_results(B):
+    """The weight-streaming kernels reading the tile-contiguous weight copies by bulk copy equal
+    the same kernels reading the row-major weights through tensor maps bit for bit (the same
+    bytes reach the same shared-memory layout), for both the stream-K and the cluster kernel."""
+    cfg = _cfg(B)
+    W = synth.make_weights(cfg, seed=49, device="cuda")
+    for stream in (1, 0):
+        a = _steps(cfg, W, stream, tiled=1)[0]
+        b = _steps(cfg, W, stream, tiled=0)[0]
+        for x, y in zip(a[0], b[0]):
+            for u, v in zip(x, y):
+                assert np.array_equal(u, v), f"stream={stream}"
+        for u, v in zip(a[1], b[1]):
+            assert np.array_equal(u, v), f"stream={stream}"
 
 
 def test_stream_gemm_small_fills_match_oracle():
