@@ -25,6 +25,10 @@ What it follows (paper sections / equations / tables):
   similarities, and all-at-once prompt exits decided by each sequence's last token.
 * Encoder "stop entirely" (Sec. 4.3, downstream tasks): exited tokens get no deeper K/V
   and drop out of deeper attention; their s~ feeds the classifier.
+* Encoder-decoder models (Sec. 5.2, the OFA setting): the encoder runs its early-exit pass;
+  its final states (s_N, or s~_N for exited tokens) are the source of every decoder layer's
+  cross-attention; the decoder runs the same early-exit pass (its own HSM, skipped-layer
+  K/V of its self-attention), each of its layers cross-attending after self-attention.
 
 Readings where the paper is silent (each one is also listed in the design notes):
 
@@ -41,6 +45,12 @@ Readings where the paper is silent (each one is also listed in the design notes)
 * Precision contract for bf16 models: weights are bf16 values; every GEMM input
   (activations), Q and the cached K/V are rounded to bf16 (round-to-nearest-even);
   everything else stays in float64 here.  fp32 models round nothing.
+* Cross-attention sublayer (the paper names the encoder-decoder architecture but not its
+  layer): pre-LN like the decoder's other sublayers, h <- h + W_Oc attn(LN_c(h) W_Qc, E W_Kc,
+  E W_Vc) + b_Oc between self-attention and the FFN, over all source positions of the
+  token's sequence (not causal); E are the encoder's final states, projected without a
+  further norm.  An exited decoder token skips its deeper layers' cross-attention too; the
+  source K/V depend on the encoder alone and need no fill.
 """
 from __future__ import annotations
 
@@ -212,6 +222,20 @@ class OracleModel:
             q = rope(q, pos, c.rope_theta)
         return self.rb(q)
 
+    # -- cross-attention (encoder-decoder decoders)
+    def cross_q(self, i: int, h: np.ndarray):
+        c = self.cfg
+        x = self.rb(layernorm(h, self.L(i, "cross_norm.g"), self.L(i, "cross_norm.b"), c.norm_eps))
+        return self.rb(self._proj(x, i, "cwq", "cbq").reshape(len(h), c.n_heads, c.head_dim))
+
+    def cross_kv(self, i: int, e: np.ndarray):
+        """Layer i's source K and V of encoder final states e [S, D]."""
+        c = self.cfg
+        x = self.rb(e)
+        k = self._proj(x, i, "cwk", "cbk").reshape(len(e), c.n_kv_heads, c.head_dim)
+        v = self._proj(x, i, "cwv", "cbv").reshape(len(e), c.n_kv_heads, c.head_dim)
+        return self.rb(k), self.rb(v)
+
     def embed(self, tokens: np.ndarray, pos: np.ndarray) -> np.ndarray:
         c = self.cfg
         e = self.w["tok_emb"][tokens]
@@ -266,6 +290,20 @@ class OracleCache:
         self.V[i - 1][seq, pos] = v
 
 
+class CrossSource:
+    """Every decoder layer's source K/V per sequence: K[i - 1][b] is [src_len[b], Hkv, dh]."""
+
+    def __init__(self, m: "OracleModel", states):
+        """states: per sequence b, the encoder's final states [src_len[b], D] (s_N of tokens
+        that ran to full depth, s~_N of exited ones)."""
+        self.src_len = np.array([len(e) for e in states], dtype=np.int64)
+        self.K = [[None] * len(states) for _ in range(m.cfg.n_layers)]
+        self.V = [[None] * len(states) for _ in range(m.cfg.n_layers)]
+        for i in range(1, m.cfg.n_layers + 1):
+            for b, e in enumerate(states):
+                self.K[i - 1][b], self.V[i - 1][b] = m.cross_kv(i, np.asarray(e, dtype=np.float64))
+
+
 def attend(m: OracleModel, q: np.ndarray, qpos: np.ndarray, K: np.ndarray, V: np.ndarray,
            causal: bool, key_mask: Optional[np.ndarray] = None) -> np.ndarray:
     """Softmax attention of one sequence's queries q [n, H, dh] over keys K/V [L, Hkv, dh].
@@ -293,12 +331,15 @@ def attend(m: OracleModel, q: np.ndarray, qpos: np.ndarray, K: np.ndarray, V: np
 
 def layer_body(m: OracleModel, i: int, h: np.ndarray, seq: np.ndarray, pos: np.ndarray,
                cache: OracleCache, causal: bool, kv_len: np.ndarray,
-               key_active: Optional[Dict[int, np.ndarray]] = None) -> np.ndarray:
+               key_active: Optional[Dict[int, np.ndarray]] = None,
+               cross: Optional[CrossSource] = None) -> np.ndarray:
     """Everything of layer i after its K/V were cached: Q, attention, O, FFN, residuals.
 
     h: [n, D] layer inputs of the active tokens; returns their layer outputs.
     key_active (optional, "stop entirely"): per sequence, the positions whose K/V layer i
-    holds; attention sees only those keys."""
+    holds; attention sees only those keys.
+    cross (encoder-decoder decoders): the source K/V; the cross-attention sublayer runs
+    between self-attention and the FFN."""
     c, rb = m.cfg, m.rb
     q = m.q_project(i, h, pos)
     att = np.zeros((len(h), c.n_heads * c.head_dim))
@@ -316,6 +357,13 @@ def layer_body(m: OracleModel, i: int, h: np.ndarray, seq: np.ndarray, pos: np.n
         f = f @ m.L(i, "w_proj").T + m.L(i, "b_proj")
         return layernorm(h1 + f, m.L(i, "ffn_norm.g"), m.L(i, "ffn_norm.b"), c.norm_eps)
     h1 = h + o
+    if cross is not None:
+        qc = m.cross_q(i, h1)
+        ac = np.zeros((len(h), c.n_heads * c.head_dim))
+        for b in np.unique(seq):
+            sel = np.nonzero(seq == b)[0]
+            ac[sel] = attend(m, qc[sel], pos[sel], cross.K[i - 1][b], cross.V[i - 1][b], False)
+        h1 = h1 + rb(ac) @ m.L(i, "cwo").T + m.L(i, "cbo")
     if c.family == GPT2:
         x = rb(layernorm(h1, m.L(i, "ffn_norm.g"), m.L(i, "ffn_norm.b"), c.norm_eps))
         f = rb(gelu_tanh(x @ m.L(i, "w_fc").T + m.L(i, "b_fc")))
@@ -347,7 +395,8 @@ def check_forced(forced: np.ndarray, n_layers: int):
 def early_exit_pass(m: OracleModel, cache: OracleCache, s0: np.ndarray, seq: np.ndarray,
                     pos: np.ndarray, delta: float, forced: Optional[np.ndarray], causal: bool,
                     kv_len: np.ndarray, hsm_mode: str = "hsm", metric: str = "global",
-                    aao_len: int = 0, stop_entirely: bool = False) -> PassResult:
+                    aao_len: int = 0, stop_entirely: bool = False,
+                    cross: Optional[CrossSource] = None) -> PassResult:
     """Run tokens (all in parallel, App. I) through layers 1..N with token-level exits.
 
     For each layer i: (a) K/V of the active tokens from their layer input go to the
@@ -364,10 +413,13 @@ def early_exit_pass(m: OracleModel, cache: OracleCache, s0: np.ndarray, seq: np.
     stop_entirely (encoders, Sec. 4.3 on downstream tasks: computation stops beyond the exit
     layer): an exiting token gets s~ for the classifier but no K/V of deeper layers, and the
     attention of a deeper layer sees only the tokens still active there.
+    cross (encoder-decoder decoders): the source K/V of every layer's cross-attention.
     """
     if metric not in ("global", "local", "both"):
         raise ValueError(metric)
     c = m.cfg
+    if (cross is not None) != (getattr(c, "max_src", 0) > 0):
+        raise ValueError("cross-attention models take a CrossSource, other models none")
     N, T = c.n_layers, len(s0)
     forced = np.zeros(T, dtype=np.int64) if forced is None else np.asarray(forced, dtype=np.int64)
     check_forced(forced, N)
@@ -388,7 +440,7 @@ def early_exit_pass(m: OracleModel, cache: OracleCache, s0: np.ndarray, seq: np.
             key_active = {int(b): np.zeros(int(kv_len[b]), dtype=bool) for b in np.unique(seq)}
             for j in A:
                 key_active[int(seq[j])][int(pos[j])] = True
-        s_new = layer_body(m, i, s[A], seq[A], pos[A], cache, causal, kv_len, key_active)   # (b)
+        s_new = layer_body(m, i, s[A], seq[A], pos[A], cache, causal, kv_len, key_active, cross)   # (b)
         exits = np.zeros(len(A), dtype=bool)
         if 2 <= i <= N - 1:                                                # (c)
             cg = cosine(s_new, inertia[A])
@@ -423,7 +475,8 @@ def early_exit_pass(m: OracleModel, cache: OracleCache, s0: np.ndarray, seq: np.
 
 def prefill(m: OracleModel, cache: OracleCache, tokens: np.ndarray, delta: float,
             forced: Optional[np.ndarray] = None, hsm_mode: str = "hsm", metric: str = "global",
-            all_at_once: bool = False, stop_entirely: bool = False) -> PassResult:
+            all_at_once: bool = False, stop_entirely: bool = False,
+            cross: Optional[CrossSource] = None) -> PassResult:
     """Prompt pass for sequences 0..B-1 (resets them); tokens [B, P].
 
     Decoder: logits [B, V] of each sequence's last position and its greedy token
@@ -445,7 +498,7 @@ def prefill(m: OracleModel, cache: OracleCache, tokens: np.ndarray, delta: float
     kv_len = cache.lens.copy()
     res = early_exit_pass(m, cache, s0, seq, pos, delta,
                           None if forced is None else np.asarray(forced).reshape(-1),
-                          causal, kv_len, hsm_mode, metric, P if all_at_once else 0, stop_entirely)
+                          causal, kv_len, hsm_mode, metric, P if all_at_once else 0, stop_entirely, cross)
     fin = res.final.reshape(B, P, -1)
     if c.family == BERT:
         res.logits = m.cls_logits(fin[:, 0])
@@ -456,7 +509,8 @@ def prefill(m: OracleModel, cache: OracleCache, tokens: np.ndarray, delta: float
 
 
 def decode_step(m: OracleModel, cache: OracleCache, tokens: np.ndarray, delta: float,
-                forced: Optional[np.ndarray] = None, hsm_mode: str = "hsm", metric: str = "global") -> PassResult:
+                forced: Optional[np.ndarray] = None, hsm_mode: str = "hsm", metric: str = "global",
+                cross: Optional[CrossSource] = None) -> PassResult:
     """One generation step: token b of sequence b at position lens[b] (App. I, generation)."""
     c = m.cfg
     if c.family == BERT:
@@ -470,7 +524,7 @@ def decode_step(m: OracleModel, cache: OracleCache, tokens: np.ndarray, delta: f
     s0 = m.embed(tokens, pos)
     res = early_exit_pass(m, cache, s0, seq, pos, delta,
                           None if forced is None else np.asarray(forced).reshape(-1),
-                          True, kv_len, hsm_mode, metric)
+                          True, kv_len, hsm_mode, metric, cross=cross)
     res.logits = m.lm_logits(res.final)
     res.next_token = np.argmax(res.logits, axis=-1)
     return res

@@ -139,6 +139,8 @@ class ModelConfig:
     kv_pool_blocks: int = 0    # 0 -> max_batch * ceil(max_seq / kv_block_tokens)
     max_pass_tokens: int = 0   # rows of per-pass workspaces; 0 -> max_batch * max_seq
     block_shuffle_seed: int = 0  # 0: KV blocks handed out in order; else a seeded permutation
+    max_src: int = 0           # > 0 (GPT-2-family decoders): cross-attention over up to max_src
+                               # encoder states per sequence (encoder-decoder models)
 
     def __post_init__(self):
         if self.n_kv_heads == 0:
@@ -189,6 +191,20 @@ def llama7b_config(**kw) -> ModelConfig:
     return ModelConfig(**base)
 
 
+def ofa_base_configs(src_len: int = 256, tgt_len: int = 32, batch: int = 8, **kw):
+    """OFA-base-shaped encoder-decoder (6 + 6 layers, D=768, 12 heads, GELU FFN 3072, BPE
+    vocabulary 50265, bf16): a post-LN encoder with a 3-way classifier head (unused by the
+    decoder) and a pre-LN decoder whose layers cross-attend to the encoder's final states.
+    Returns (encoder config, decoder config)."""
+    enc = dict(family=BERT, n_layers=6, d_model=768, n_heads=12, head_dim=64, d_ffn=3072, vocab=50265,
+               max_pos=1024, n_classes=3, dtype="bf16", norm_eps=1e-5, max_batch=batch, max_seq=src_len)
+    dec = dict(family=GPT2, n_layers=6, d_model=768, n_heads=12, head_dim=64, d_ffn=3072, vocab=50265,
+               max_pos=1024, dtype="bf16", max_batch=batch, max_seq=tgt_len, max_src=src_len)
+    enc.update(kw)
+    dec.update(kw)
+    return ModelConfig(**enc), ModelConfig(**dec)
+
+
 def bert_base_config(**kw) -> ModelConfig:
     """BERT-base shape: 12 layers, D=768, 12 heads, GELU FFN 3072, 2 classes, bf16."""
     base = dict(family=BERT, n_layers=12, d_model=768, n_heads=12, head_dim=64, d_ffn=3072,
@@ -230,6 +246,15 @@ def weight_shapes(cfg: ModelConfig) -> Dict[str, tuple]:
         s[p + "ffn_norm.g"] = (D,)
         if cfg.family != LLAMA:
             s[p + "ffn_norm.b"] = (D,)
+        if cfg.max_src > 0:   # cross-attention sublayer (encoder-decoder decoders)
+            s[p + "cross_norm.g"] = (D,)
+            s[p + "cross_norm.b"] = (D,)
+            s[p + "cwq"] = (dq, D)
+            s[p + "cwk"] = (dkv, D)
+            s[p + "cwv"] = (dkv, D)
+            s[p + "cwo"] = (D, dq)
+            for b, n in (("cbq", dq), ("cbk", dkv), ("cbv", dkv), ("cbo", D)):
+                s[p + b] = (n,)
         if cfg.family == LLAMA:
             s[p + "w_gate"] = (F, D)
             s[p + "w_up"] = (F, D)

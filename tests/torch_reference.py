@@ -9,8 +9,9 @@ oracle's NumPy expressions.  Layers are 1-based as in the paper.
 bf16=True states the bf16 precision contract on its own: weights are bf16 values, and
 torch's own float -> bfloat16 cast (round to nearest even) is applied to every GEMM input
 (the normalised layer and head inputs, the attention output, the FFN's activated hidden
-rows, the mapper's FC inputs, the pooler's input and output), to Q and to the cached K
-and V; everything else stays float64.
+rows, the mapper's FC inputs, the pooler's input and output, the encoder states of the
+cross-attention's K/V projection), to Q and to the cached K and V (self- and cross-
+attention); everything else stays float64.
 """
 from __future__ import annotations
 
@@ -71,8 +72,30 @@ class TorchRef:
             q = self.rope(q, pos)
         return self.r(q)
 
-    def after_attn(self, i, h, a):
-        """Residual / FFN part of layer i given the attention output a [..., H*dh]."""
+    # ---------------------------------------------------------------- cross-attention
+    def cross_kv(self, i, e):
+        """Layer i's source K, V [S, Hkv, dh] of encoder final states e [S, D]."""
+        c = self.c
+        x = self.r(e)
+        k = F.linear(x, self.lw(i, "cwk"), self.lw(i, "cbk")).unflatten(-1, (c.n_kv_heads, c.head_dim))
+        v = F.linear(x, self.lw(i, "cwv"), self.lw(i, "cbv")).unflatten(-1, (c.n_kv_heads, c.head_dim))
+        return self.r(k), self.r(v)
+
+    def cross_sublayer(self, i, h1, src):
+        """h1 [..., D] of one sequence + its cross-attention over src = (K, V) [S, Hkv, dh]."""
+        c, r = self.c, self.r
+        x = r(F.layer_norm(h1, (c.d_model,), self.lw(i, "cross_norm.g"), self.lw(i, "cross_norm.b"), c.norm_eps))
+        q = r(F.linear(x, self.lw(i, "cwq"), self.lw(i, "cbq")).unflatten(-1, (c.n_heads, c.head_dim)))
+        rep = c.n_heads // c.n_kv_heads
+        k = src[0].repeat_interleave(rep, dim=1).transpose(0, 1)        # [H, S, dh]
+        v = src[1].repeat_interleave(rep, dim=1).transpose(0, 1)
+        qh = q.reshape(-1, c.n_heads, c.head_dim).transpose(0, 1)       # [H, n, dh]
+        a = F.scaled_dot_product_attention(qh, k, v).transpose(0, 1).reshape(*h1.shape[:-1], -1)
+        return h1 + F.linear(r(a), self.lw(i, "cwo"), self.lw(i, "cbo"))
+
+    def after_attn(self, i, h, a, src=None):
+        """Residual / FFN part of layer i given the attention output a [..., H*dh]; src: the
+        sequence's source K/V of layer i (encoder-decoder decoders)."""
         c, r = self.c, self.r
         o = F.linear(r(a), self.lw(i, "wo"), self.lw(i, "bo"))
         if c.family == BERT:
@@ -81,6 +104,8 @@ class TorchRef:
                          self.lw(i, "w_proj"), self.lw(i, "b_proj"))
             return F.layer_norm(h1 + f, (c.d_model,), self.lw(i, "ffn_norm.g"), self.lw(i, "ffn_norm.b"), c.norm_eps)
         h1 = h + o
+        if src is not None:
+            h1 = self.cross_sublayer(i, h1, src)
         if c.family == GPT2:
             x = r(F.layer_norm(h1, (c.d_model,), self.lw(i, "ffn_norm.g"), self.lw(i, "ffn_norm.b"), c.norm_eps))
             f = r(F.gelu(F.linear(x, self.lw(i, "w_fc"), self.lw(i, "b_fc")), approximate="tanh"))
@@ -124,8 +149,9 @@ class TorchRef:
         return F.linear(r(pooled), W["cls.w"], W["cls.b"])
 
     # ---------------------------------------------------------------- full depth, batched
-    def full_forward(self, tokens):
-        """Standard full-depth forward of [B, P] tokens with SDPA; no cache.
+    def full_forward(self, tokens, source=None):
+        """Standard full-depth forward of [B, P] tokens with SDPA; no cache.  source
+        (encoder-decoder decoders): per sequence, the encoder's final states [S_b, D].
 
         Returns final hidden states [B, P, D]."""
         c = self.c
@@ -139,18 +165,25 @@ class TorchRef:
             rep = c.n_heads // c.n_kv_heads
             k = k.repeat_interleave(rep, dim=2).transpose(1, 2)
             v = v.repeat_interleave(rep, dim=2).transpose(1, 2)
-            a = F.scaled_dot_product_attention(q, k, v, is_causal=c.family != BERT)
-            h = self.after_attn(i, h, a.transpose(1, 2).flatten(-2))
+            a = F.scaled_dot_product_attention(q, k, v, is_causal=c.family != BERT).transpose(1, 2).flatten(-2)
+            if source is None:
+                h = self.after_attn(i, h, a)
+            else:
+                h = torch.stack([self.after_attn(i, h[b], a[b], self.cross_kv(i, torch.as_tensor(source[b]).double()))
+                                 for b in range(B)])
         return h
 
     # ---------------------------------------------------------------- token-major unfold
-    def token_major(self, tokens, forced, hsm_mode="hsm"):
+    def token_major(self, tokens, forced, hsm_mode="hsm", source=None):
         """One sequence, one token at a time, each token through all of its layers before
         the next token starts.  forced[j] in [2, N] is token j's exit layer (N = none).
+        source (encoder-decoder decoders): the sequence's encoder final states [S, D].
 
         Returns (final [P, D], exit_layer [P], K dict, V dict) with K[i][j] the cached key
         of position j at layer i."""
         c = self.c
+        src = None if source is None else {i: self.cross_kv(i, torch.as_tensor(source).double())
+                                           for i in range(1, c.n_layers + 1)}
         N = c.n_layers
         tokens = torch.as_tensor(tokens).reshape(-1)
         P = len(tokens)
@@ -173,7 +206,7 @@ class TorchRef:
                 vals = vals.repeat_interleave(rep, dim=1)
                 w = torch.softmax(torch.einsum("hd,thd->ht", q, keys) / math.sqrt(c.head_dim), dim=-1)
                 a = torch.einsum("ht,thd->hd", w, vals).reshape(-1)
-                h_new = self.after_attn(i, h, a)
+                h_new = self.after_attn(i, h, a, None if src is None else src[i])
                 leave = 2 <= i <= N - 1 and int(forced[j]) == i
                 if leave:
                     st = self.hsm(h_new, h, inertia) if hsm_mode == "hsm" else h_new
