@@ -305,8 +305,7 @@ def run_fill_micro(adept, device, peaks, grid_T, grid_i, reps=3):
             args = (m.h, T, h_all[:T].contiguous(), el, seq_all[:T].contiguous(), pos_all[:T].contiguous())
             adept.adept_skip_kv_fill(*args)
             torch.cuda.synchronize()
-            adept.adept_set_option(m.h, adept.OPT_PROFILE, 1)
-            adept.adept_profile_read(m.h, adept.PROF_KV_FILL)
+            # the call as a user makes it (programmatic dependent launch, no per-launch events)
             ts = []
             for _ in range(reps):
                 flush.zero_()
@@ -316,6 +315,13 @@ def run_fill_micro(adept, device, peaks, grid_T, grid_i, reps=3):
                 e1.record(st)
                 torch.cuda.synchronize()
                 ts.append(e0.elapsed_time(e1))
+            # the GEMM launch alone, event-bracketed in a profiled call (informational)
+            adept.adept_set_option(m.h, adept.OPT_PROFILE, 1)
+            adept.adept_profile_read(m.h, adept.PROF_KV_FILL)
+            for _ in range(reps):
+                flush.zero_()
+                adept.adept_skip_kv_fill(*args)
+                torch.cuda.synchronize()
             n, kms, _, _ = adept.adept_profile_read(m.h, adept.PROF_KV_FILL)
             adept.adept_set_option(m.h, adept.OPT_PROFILE, 0)
             adept.adept_check_device_status(m.h)
@@ -390,6 +396,60 @@ def run_encoder(adept, device, B=64, P=128):
     m.close()
     torch.cuda.empty_cache()
     return {"workload": f"BERT-base shape, bf16, random-init; {B} x {P}-token classification batch", **out}
+
+
+def run_encdec(adept, device, B=8, S=256, T=8, steps=8, reps=4):
+    """OFA-base-shaped encoder-decoder (Sec. 5.2; 6 + 6 layers, D 768, 12 heads, FFN 3072,
+    bf16, random-init): B sequences of S source tokens (a text stand-in for OFA's image and
+    text source), a T-token target prompt and `steps` greedy steps.  One pass = the encoder's
+    prompt pass, the decoder's source K/V (adept_set_cross_source from the encoder's final
+    states, on the device), the decoder's prompt pass and its generation steps.  Exits ~ U{2..6}
+    per token in both stacks against full depth; tokens/s counts source + target tokens."""
+    enc, dec = synth.ofa_base_configs(src_len=S, tgt_len=T + steps, batch=B)
+    me = adept.Model(enc, synth.make_weights(enc, seed=0, device=device))
+    md = adept.Model(dec, synth.make_weights(dec, seed=1, device=device))
+    src = synth.make_tokens(0, B, S, enc.vocab).to(device)
+    tgt = synth.make_tokens(1, B, T, dec.vocab).to(device)
+    fe = synth.forced_exits_uniform(0, B * S, 2, enc.n_layers, name="forced_enc").view(B, S).to(device)
+    fd = synth.forced_exits_uniform(1, B * T, 2, dec.n_layers, name="forced_dec").view(B, T).to(device)
+    fs = synth.forced_exits_uniform(2, B * steps, 2, dec.n_layers, name="forced_steps").view(steps, B).to(device)
+    st = torch.cuda.current_stream()
+    fin = torch.empty(B * S, enc.d_model, device=device)
+
+    def one(full):
+        ex_e, _, _, _ = me.prefill(src, 0.9, torch.full_like(fe, enc.n_layers) if full else fe)
+        adept.adept_read_final_states(me.h, fin, B * S)
+        md.set_cross_source([S] * B, fin)
+        ex_d, _, nx, _ = md.prefill(tgt, 0.9, torch.full_like(fd, dec.n_layers) if full else fd)
+        for k in range(steps):
+            f = torch.full_like(fs[k], dec.n_layers) if full else fs[k]
+            _, _, nx, _ = md.decode_step(nx.view(-1).contiguous(), 0.9, f.contiguous())
+        return ex_e, ex_d
+
+    out = {}
+    for name, full in (("early_exit", False), ("full_depth", True)):
+        ts = []
+        for _ in range(reps):
+            torch.cuda.synchronize()
+            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            e0.record(st)
+            ex_e, ex_d = one(full)
+            e1.record(st)
+            torch.cuda.synchronize()
+            ts.append(e0.elapsed_time(e1))
+        t = float(np.median(ts[1:])) / 1e3
+        out[name] = {"ms": round(t * 1e3, 3), "tok_s": round(B * (S + T + steps) / t, 1),
+                     "encoder_mean_exit": round(float(ex_e.double().mean().item()), 3),
+                     "decoder_prompt_mean_exit": round(float(ex_d.double().mean().item()), 3)}
+    out["speedup"] = round(out["full_depth"]["ms"] / out["early_exit"]["ms"], 4)
+    me.check()
+    md.check()
+    me.close()
+    md.close()
+    torch.cuda.empty_cache()
+    return {"workload": f"OFA-base-shaped encoder-decoder (6 + 6 layers, D 768), bf16, random-init; {B} x {S} source "
+                        f"tokens, {T}-token target prompt + {steps} greedy steps; forced exits U{{2..6}} in both stacks",
+            **out}
 
 
 def hsm_train_flops(cfg, n, n_cls=0):
@@ -666,14 +726,17 @@ def ours(args, rank, world, device):
     e2e = replica_throughput(tok_per_step, n_e2e, world, e2e_t)
     h2d = (tok_h.numel() + fp_h.numel() + fd_h.numel()) * 4
     d2h = (nxt_h.numel() + ex_h.numel()) * 4
-    # --------------------------------------------------------------- one profiled step (per-class device time)
-    # CUDA events on the launching stream bracket every GEMM / fill / attention launch, so each
-    # bracketed kernel runs alone (it cannot overlap its neighbours as it does under
-    # programmatic dependent launch in the timed steps); generation steps run as direct
-    # launches while profiling.  Per-launch times are therefore a little pessimistic.
-    adept.adept_set_option(run.m.h, adept.OPT_PROFILE, 1)
+    # --------------------------------------------------------------- one step with the span timer (in-situ kernel time)
+    # The weight-streaming GEMM launches (the generation steps' layer, mapper and head GEMMs, and
+    # their grouped skipped-layer fills) record their spans on the device timer while the step
+    # runs as timed (programmatic dependent launch, graph replay): from the first CTA past the
+    # grid-dependency wait to the end of the last thread.  Consecutive launches' spans do not
+    # overlap, so a class's summed span never exceeds the step.
+    adept.adept_set_option(run.m.h, adept.OPT_SPAN_TIMER, 1)
+    run.step()   # graphs are captured again with the span sites
+    torch.cuda.synchronize()
     for c in range(adept.PROF_GEMM_TRAIN + 1):
-        adept.adept_profile_read(run.m.h, c)
+        adept.adept_span_read(run.m.h, c)
     flush.zero_()
     torch.cuda.synchronize()
     e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
@@ -681,20 +744,20 @@ def ours(args, rank, world, device):
     run.step()
     e1.record(st)
     torch.cuda.synchronize()
-    prof_step_ms = e0.elapsed_time(e1)
-    prof = {c: adept.adept_profile_read(run.m.h, c) for c in range(adept.PROF_GEMM_TRAIN + 1)}
-    adept.adept_set_option(run.m.h, adept.OPT_PROFILE, 0)
+    span_step_ms = e0.elapsed_time(e1)
+    spans = {c: adept.adept_span_read(run.m.h, c) for c in range(adept.PROF_GEMM_TRAIN + 1)}
+    adept.adept_set_option(run.m.h, adept.OPT_SPAN_TIMER, 0)
     adept.adept_check_device_status(run.m.h)
     # --------------------------------------------------------------- dominant kernel roofline
     e_p = run.exit_p.cpu().numpy()
     e_d = run.exit_d.cpu().numpy()
     work = class_work(cfg, e_p, e_d)
-    names = {adept.PROF_GEMM_PREFILL: "gemm_prefill", adept.PROF_GEMM_DECODE: "gemm_decode",
-             adept.PROF_KV_FILL: "kv_fill_decode", adept.PROF_ATTENTION: "attention"}
-    per_class = {names[c]: {"launches": prof[c][0], "ms_per_step": round(prof[c][1], 4)} for c in names}
-    dom_c = max((c for c in names if names[c] in work), key=lambda c: prof[c][1])
+    names = {adept.PROF_GEMM_DECODE: "gemm_decode", adept.PROF_KV_FILL: "kv_fill_decode"}
+    per_class = {names[c]: {"launches": spans[c][0], "span_ms_per_step": round(spans[c][1], 4),
+                            "share_of_step": round(spans[c][1] / span_step_ms, 4)} for c in names}
+    dom_c = max(names, key=lambda c: spans[c][1])
     dom = names[dom_c]
-    n, ms = prof[dom_c][0], prof[dom_c][1]
+    n, ms = spans[dom_c]
     fl, by = work[dom]
     t_f = fl / (peaks["bf16_tflops"] * 1e12)
     t_b = by / (peaks["hbm_gbs"] * 1e9)
@@ -706,14 +769,14 @@ def ours(args, rank, world, device):
     roof["frac"] = round(roof["achieved"] / roof["peak"], 4)
     tr = NCU_TRAFFIC_PER_LAUNCH.get(dom)
     roof["traffic"] = round(tr) if tr else None
-    roof["kernel"] = dom
+    roof["kernel"] = dom + " (stream-K and cluster K-split weight-streaming GEMM launches)"
     roof["launches"] = n
     roof["peak_source"] = (peaks_src + " (MEASURED_PEAKS.json)") if peaks_src == "measured" else peaks_src
-    roof["timing"] = ("CUDA events bracketing each launch of the class in one profiled step after the timed steps "
-                      "(each bracketed launch runs alone)")
+    roof["timing"] = ("device-timer span per launch (first CTA past the grid-dependency wait to the last thread's "
+                      "end), summed over the class in one step run as timed (PDL, graph replay) after the timed steps")
     roof["class_ms_per_step"] = round(ms, 3)
-    roof["class_share_of_step"] = round(ms / ms_per_step, 4)
-    roof["profiled_step_ms"] = round(prof_step_ms, 3)
+    roof["class_share_of_step"] = round(ms / span_step_ms, 4)
+    roof["span_step_ms"] = round(span_step_ms, 3)
     roof["work_per_launch"] = {"flop": round(fl / max(n, 1)), "bytes": round(by / max(n, 1))}
     line = {
         "metric": METRIC, "value": round(value, 2), "unit": "tokens/s", "n_gpus": world, "steps": args.steps,
@@ -752,6 +815,7 @@ def ours(args, rank, world, device):
     if rank == 0 and not args.no_llama:
         line["gpt2_small"] = run_gpt2(adept, device)
         line["encoder"] = run_encoder(adept, device)
+        line["encoder_decoder"] = run_encdec(adept, device)
         line["hsm_train"] = run_hsm_train(adept, device, peaks)
         line["hsm_train_llama7b"] = run_hsm_train(adept, device, peaks, shape="llama7b", reps=3)
         line["hsm_train_bert"] = run_hsm_train(adept, device, peaks, shape="bert")
@@ -938,6 +1002,15 @@ def kernel_case_fill_small(device):
     m.close()
 
 
+def kernel_case_fill_grid(device, grid_T, grid_i):
+    """The skipped-layer fill grid alone (Llama-7B layers), one JSON line per cell."""
+    import paper_2601_03700_gb300 as adept
+    adept.load_library()
+    peaks, _ = load_peaks()
+    for row in run_fill_micro(adept, device, peaks, grid_T, grid_i):
+        print(json.dumps({"kernel_case": "fill_grid", **row}))
+
+
 def kernel_case_llama_prefill(device):
     """Two early-exit prompt passes at the Llama-2-7B shape (2048 tokens, exits ~ N(24,4) on
     [8, 32]) for launch-list captures: the second pass is the one to capture."""
@@ -1040,7 +1113,8 @@ def kernel_case_hsm_train(device, n=8192, steps=2, shape="gpt2"):
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--kernel-case", default=None,
-                    choices=["fill_small", "llama_prefill", "gpt2_decode", "llama_decode_small", "hsm_train"])
+                    choices=["fill_small", "fill_grid", "llama_prefill", "gpt2_decode", "llama_decode_small",
+                             "hsm_train"])
     ap.add_argument("--gpus", type=int, default=1)
     ap.add_argument("--steps", type=int, default=5)
     ap.add_argument("--warmup", type=int, default=3)
@@ -1066,6 +1140,10 @@ def main():
         return
     if args.kernel_case == "fill_small":
         kernel_case_fill_small(torch.device("cuda", 0))
+        return
+    if args.kernel_case == "fill_grid":
+        kernel_case_fill_grid(torch.device("cuda", 0), [int(x) for x in args.fill_T.split(",")],
+                              [int(x) for x in args.fill_i.split(",")])
         return
     if args.kernel_case == "llama_prefill":
         kernel_case_llama_prefill(torch.device("cuda", 0))

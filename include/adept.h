@@ -76,6 +76,9 @@ typedef struct {
   int kv_pool_blocks;  /* 0 -> max_batch * ceil(max_seq / kv_block_tokens) */
   int max_pass_tokens; /* rows of the per-pass workspaces; 0 -> max_batch * max_seq */
   uint64_t block_shuffle_seed; /* 0: KV blocks handed out in order; else a seeded permutation */
+  int max_src;         /* > 0 (GPT-2 family only): an encoder-decoder decoder whose layers
+                          cross-attend to up to max_src encoder states per sequence
+                          (adept_set_cross_source); 0: no cross-attention */
 } adept_config;
 
 /* One named weight tensor.  `data` may be a host or a device pointer (it is read
@@ -89,6 +92,9 @@ typedef struct {
  *   GPT2/BERT: layers.l.w_fc [F,D], b_fc [F], w_proj [D,F], b_proj [D]
  *   LLAMA: final_norm.g [D], lm_head [V,D]; GPT2: final_norm.g/.b [D] (head tied to tok_emb)
  *   BERT: pool.w [D,D], pool.b [D], cls.w [C,D], cls.b [C]
+ *   max_src > 0 (cross-attention sublayer, pre-LN, between self-attention and the FFN):
+ *     layers.l.cross_norm.g/.b [D], cwq [D_q,D], cwk [D_kv,D], cwv [D_kv,D], cwo [D,D_q],
+ *     cbq cbk cbv cbo
  *   HSM (App. B Table S1): hsm.g0 [D], hsm.conv_w [3,3], hsm.conv_b [1],
  *     hsm.fc1_w [m1,D], hsm.fc1_b, hsm.fc2_w [m2,m1], hsm.fc2_b, hsm.fc3_w [m1,m2],
  *     hsm.fc3_b, hsm.g1 [m1], hsm.fc4_w [D,m1], hsm.fc4_b [D], hsm.g2 [D]      */
@@ -199,6 +205,21 @@ ADEPT_API adept_status adept_skip_kv_fill_noalloc(adept_model* m, int n_tokens, 
 /* Release everything the model owns (synchronises the device first).  NULL is a no-op. */
 ADEPT_API void adept_free(adept_model* m);
 
+/* Encoder-decoder models (Sec. 5.2, the OFA setting: an early-exiting encoder whose final
+ * states feed a decoder that exits token by token too).  For a decoder loaded with
+ * max_src > 0: set the source of every layer's cross-attention for sequences 0..n_seq-1.
+ * d_states: fp32 [sum_b h_src_len[b]][d_model], device, in sequence order -- the encoder's
+ * final states (s_N of tokens that ran to full depth, s~_N of exited ones; for an encoder
+ * pass of n_seq x P tokens, the rows adept_read_final_states returns, with h_src_len[b] = P).
+ * h_src_len[b] in [1, max_src].  Computes each decoder layer's source K/V (its cross K/V
+ * projection of the states, rounded to bf16 for bf16 models) into the model's source cache;
+ * later prompt passes and generation steps of these sequences cross-attend over all
+ * h_src_len[b] source positions (not causal).  The states may be released once `stream` has
+ * passed the call.  Errors: INVALID_ARG (no cross-attention, n_seq or a length out of range,
+ * NULL pointer), CUDA. */
+ADEPT_API adept_status adept_set_cross_source(adept_model* m, int n_seq, const int32_t* h_src_len,
+                                              const float* d_states, void* stream);
+
 /* ---- helpers (not part of the method; used by tests and the benchmark) ---- */
 
 /* Message of the last failing call on `m` (or of the last failed load when m is NULL). */
@@ -248,10 +269,22 @@ ADEPT_API adept_status adept_check_device_status(adept_model* m, void* stream);
  * so a sequence leaves at once (generation steps are unaffected: one token per sequence).
  * Default 0.  STOP_ENTIRELY (bf16 encoders; Sec. 4.3 on downstream tasks): 1 stops an exited
  * token's computation entirely — no K/V of deeper layers, and deeper layers' attention sees
- * only the tokens still active there; its mapped state still feeds the classifier.  Default 0. */
+ * only the tokens still active there; its mapped state still feeds the classifier.  Default 0.
+ * SPAN_TIMER (instrumentation, default 0): 1 makes the weight-streaming GEMM launches (the
+ * stream-K and the cluster K-split kernel: generation steps, output heads of short passes,
+ * fills of a few tokens) record their span on the device timer, from the first CTA past the
+ * grid-dependency wait to the end of the last CTA, summed per kernel class by a small kernel at
+ * the end of each pass (read with adept_span_read; a pass records its first 1024 such launches).
+ * Launches keep programmatic dependent launch and graph replay (graphs are captured again),
+ * so spans are taken in the step as it runs; consecutive launches' spans do not overlap.
+ * ATTN_TC (default 1): the prompt-pass attention of bf16 models (self- and cross-attention,
+ * head_dim 64 or 128) runs on the tcgen05 kernel (S and O accumulated in tensor memory, P
+ * rounded to bf16); 0 keeps the mma.sync kernel (which the encoder's stop-entirely variant
+ * always uses). */
 enum { ADEPT_OPT_HSM_IDENTITY = 1, ADEPT_OPT_PROFILE = 2, ADEPT_OPT_GEMM_SIMT = 3, ADEPT_OPT_DECODE_GRAPH = 4,
        ADEPT_OPT_DECODE_GEMM = 5, ADEPT_OPT_EXIT_METRIC = 7, ADEPT_OPT_ALL_AT_ONCE = 8,
-       ADEPT_OPT_STOP_ENTIRELY = 9, ADEPT_OPT_DECODE_STREAM = 10, ADEPT_OPT_DECODE_TILED = 11 };
+       ADEPT_OPT_STOP_ENTIRELY = 9, ADEPT_OPT_DECODE_STREAM = 10, ADEPT_OPT_DECODE_TILED = 11,
+       ADEPT_OPT_SPAN_TIMER = 12, ADEPT_OPT_ATTN_TC = 13 };
 ADEPT_API adept_status adept_set_option(adept_model* m, int option, int value);
 
 /* Kernel classes reported by adept_profile_read: the GEMMs of prompt passes (layer
@@ -266,6 +299,9 @@ enum { ADEPT_PROF_GEMM_PREFILL = 0, ADEPT_PROF_KV_FILL = 1, ADEPT_PROF_ATTENTION
  * record.  flops / bytes are reserved (returned as 0). */
 ADEPT_API adept_status adept_profile_read(adept_model* m, int cls, int64_t* launches, double* total_ms,
                                 double* flops, double* bytes);
+/* Synchronise, then return the launches of class `cls` recorded by the span timer and their
+ * summed spans in ms; resets the class total.  Zeros when the timer was never on. */
+ADEPT_API adept_status adept_span_read(adept_model* m, int cls, int64_t* launches, double* total_ms);
 
 /* ---- HSM training (Sec. 4.2; Sec. 4.3; Sec. 5.1 "Training"; App. D) -------------------
  * The Hidden State Mapper is trained with the base model frozen.  Decoders: its mapped state

@@ -21,6 +21,7 @@ STATUS_NAMES = {0: "OK", 1: "INVALID_ARG", 2: "OOM", 3: "CAPACITY", 4: "CUDA", 5
 FAMILY = {"llama": 0, "gpt2": 1, "bert": 2}
 OPT_HSM_IDENTITY, OPT_PROFILE, OPT_GEMM_SIMT, OPT_DECODE_GRAPH, OPT_DECODE_GEMM = 1, 2, 3, 4, 5
 OPT_EXIT_METRIC, OPT_ALL_AT_ONCE, OPT_STOP_ENTIRELY, OPT_DECODE_STREAM, OPT_DECODE_TILED = 7, 8, 9, 10, 11
+OPT_SPAN_TIMER, OPT_ATTN_TC = 12, 13
 EXIT_GLOBAL, EXIT_LOCAL, EXIT_BOTH = 0, 1, 2
 PROF_GEMM_PREFILL, PROF_KV_FILL, PROF_ATTENTION, PROF_GEMM_DECODE, PROF_GEMM_TRAIN = 0, 1, 2, 3, 4
 HSM_PARAMS, HSM_GRADS, HSM_MOMENT1, HSM_MOMENT2 = 0, 1, 2, 3
@@ -36,6 +37,7 @@ ABI_SYMBOLS = [
     "adept_launch_count", "adept_skip_kv_fill_noalloc",
     "adept_calibrate_threshold", "adept_hsm_train_init", "adept_hsm_train_step", "adept_hsm_train_read",
     "adept_hsm_param_numel", "adept_hsm_train_step_cls", "adept_set_wait_limit", "adept_set_alloc_fail_after",
+    "adept_span_read", "adept_set_cross_source",
 ]
 
 
@@ -54,7 +56,7 @@ class AdeptConfig(ctypes.Structure):
         ("rope_theta", ctypes.c_float), ("hsm_eps", ctypes.c_float), ("hsm_m1", ctypes.c_int),
         ("hsm_m2", ctypes.c_int), ("kv_block_tokens", ctypes.c_int), ("max_batch", ctypes.c_int),
         ("max_seq", ctypes.c_int), ("kv_pool_blocks", ctypes.c_int), ("max_pass_tokens", ctypes.c_int),
-        ("block_shuffle_seed", ctypes.c_uint64),
+        ("block_shuffle_seed", ctypes.c_uint64), ("max_src", ctypes.c_int),
     ]
 
 
@@ -103,6 +105,10 @@ def load_library(path: str = LIB_PATH):
     lib.adept_set_option.argtypes = [vp, c_int, c_int]
     lib.adept_profile_read.argtypes = [vp, c_int, ctypes.POINTER(ctypes.c_int64), ctypes.POINTER(ctypes.c_double),
                                        ctypes.POINTER(ctypes.c_double), ctypes.POINTER(ctypes.c_double)]
+    lib.adept_set_cross_source.argtypes = [vp, c_int, ctypes.POINTER(ctypes.c_int32), fp, st]
+    lib.adept_set_cross_source.restype = c_int
+    lib.adept_span_read.argtypes = [vp, c_int, ctypes.POINTER(ctypes.c_int64), ctypes.POINTER(ctypes.c_double)]
+    lib.adept_span_read.restype = c_int
     lib.adept_launch_count.argtypes = [vp]
     lib.adept_launch_count.restype = ctypes.c_int64
     lib.adept_calibrate_threshold.argtypes = [vp, c_int, c_int, i32p, c_float, c_float, c_int, c_float, c_float,
@@ -173,7 +179,7 @@ def make_config(cfg) -> AdeptConfig:
         hsm_eps=float(g("hsm_eps", 1e-6)), hsm_m1=g("hsm_m1"), hsm_m2=g("hsm_m2"),
         kv_block_tokens=g("kv_block_tokens", 16), max_batch=g("max_batch"), max_seq=g("max_seq"),
         kv_pool_blocks=g("kv_pool_blocks", 0) or 0, max_pass_tokens=g("max_pass_tokens", 0) or 0,
-        block_shuffle_seed=int(g("block_shuffle_seed", 0) or 0))
+        block_shuffle_seed=int(g("block_shuffle_seed", 0) or 0), max_src=int(g("max_src", 0) or 0))
 
 
 # ---------------------------------------------------------------------------
@@ -308,6 +314,15 @@ def adept_read_final_states(m, out: torch.Tensor, rows: int, stream=None):
     _check(lib, m, lib.adept_read_final_states(m, _ptr(out), rows, _stream(stream)))
 
 
+def adept_set_cross_source(m, src_len, states: torch.Tensor, stream=None):
+    """Cross-attention source of sequences 0..len(src_len)-1: states fp32 [sum(src_len), D] on
+    the device, in sequence order."""
+    lib = load_library()
+    n = len(src_len)
+    arr = (ctypes.c_int32 * n)(*[int(x) for x in src_len])
+    _check(lib, m, lib.adept_set_cross_source(m, n, arr, _ptr(states), _stream(stream)))
+
+
 def adept_check_device_status(m, stream=None):
     lib = load_library()
     _check(lib, m, lib.adept_check_device_status(m, _stream(stream)))
@@ -325,6 +340,15 @@ def adept_profile_read(m, cls: int):
     _check(lib, m, lib.adept_profile_read(m, cls, ctypes.byref(n), ctypes.byref(ms), ctypes.byref(fl),
                                            ctypes.byref(by)))
     return n.value, ms.value, fl.value, by.value
+
+
+def adept_span_read(m, cls: int):
+    """(launches, summed in-situ spans in ms) of class `cls` recorded by the span timer."""
+    lib = load_library()
+    n = ctypes.c_int64()
+    ms = ctypes.c_double()
+    _check(lib, m, lib.adept_span_read(m, cls, ctypes.byref(n), ctypes.byref(ms)))
+    return n.value, ms.value
 
 
 def adept_launch_count(m) -> int:
@@ -384,6 +408,9 @@ class Model:
                           None if forced is None else forced.to(torch.int32).contiguous().view(-1), ex, lg, nx, sim,
                           stream)
         return ex, lg, nx, sim
+
+    def set_cross_source(self, src_len, states: torch.Tensor, stream=None):
+        adept_set_cross_source(self.h, src_len, states.float().contiguous(), stream)
 
     def final_states(self, rows: int) -> torch.Tensor:
         out = torch.empty(rows, self.cfg.d_model, dtype=torch.float32, device="cuda")

@@ -5,6 +5,7 @@
 #define ADEPT_TU_ID 1
 #include "common.cuh"
 #include "kernels.h"
+#include "attention_tc.h"
 
 #include <algorithm>
 
@@ -869,10 +870,17 @@ static int g_ad_smem_set[4] = {0, 0, 0, 0};
 void launch_attention(cudaStream_t st, int dt, const void* q, int ld_q, void* out, int ld_out, DevRange rows,
                       int max_rows, const int* row_tok, const int* tok_seq, const int* tok_pos, const int* seq_len,
                       KVCacheView cache, int layer0, int n_heads, int causal, int decode_keys, float* ws,
-                      int* counters, unsigned* err, const int* key_exit, int kp_len) {
+                      int* counters, unsigned* err, const int* key_exit, int kp_len, int q_rows, int n_layers) {
   if (max_rows <= 0) return;
   const int dh = cache.head_dim;
   const float scale_log2 = 1.4426950408889634f / sqrtf((float)dh);
+  // prompt passes of bf16 models: the tcgen05 kernel when the caller gives the Q buffer's
+  // extent and the pools' layer count (the mma.sync kernel below keeps the key mask of the
+  // encoder's stop-entirely variant)
+  if (decode_keys == 0 && dt == 1 && !key_exit && q_rows > 0 && n_layers > 0 &&
+      launch_attention_tc(st, q, ld_q, q_rows, out, ld_out, rows, max_rows, row_tok, tok_seq, tok_pos, seq_len, cache,
+                          n_layers, layer0, n_heads, causal, scale_log2, err) >= 0)
+    return;
   if (decode_keys > 0 && ws && counters && dt == 1 && (dh == 64 || dh == 128) && cache.block_tokens == 16 &&
       (decode_keys + AD_CHUNK - 1) / AD_CHUNK <= ATTN_MAX_SPLIT && n_heads % cache.n_kv_heads == 0 &&
       n_heads / cache.n_kv_heads <= 8 &&

@@ -138,6 +138,66 @@ __device__ __forceinline__ long long wait_limit() { return g_wait_limit; }
   }
 
 namespace adept {
+// In-situ launch spans of the weight-streaming kernels (the span timer option).  A launch's
+// span runs from the first of its CTAs past the grid-dependency wait to the end of its last
+// CTA.  Every kernel of a stream passes its dependency wait only after its predecessor has
+// completed, so the spans of consecutive launches do not overlap and their sum never exceeds
+// the elapsed time of the sequence; bytes a kernel fetched before its wait (weights prefetched
+// while the predecessor still ran) fall outside its span.  Each CTA's last thread folds its
+// stamps into the launch's site with two non-returning reductions (nothing waits on them);
+// span_collect_kernel, launched at the end of the pass, adds every used site to its class total
+// and resets it.
+struct SpanSite {
+  unsigned long long t0;   // earliest post-wait stamp of the launch (all ones when idle)
+  unsigned long long t1;   // latest CTA end (0 when idle)
+  int cls;                 // kernel class of the launch
+  int pad;
+};
+struct SpanTotal {
+  unsigned long long ns, n;   // summed spans, launches
+};
+struct SpanCtx {
+  SpanSite* site;    // NULL: not recorded
+  int cls;
+};
+// The span context the weight-streaming launch functions copy into their parameters (set by
+// the runtime around a launch on the calling thread; NULL site when the timer is off).
+extern thread_local SpanCtx g_span;
+
+__device__ __forceinline__ unsigned long long global_ns() {
+  unsigned long long t;
+  asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
+  return t;
+}
+// Per-thread recorder: construct at kernel entry, call init() before the CTA's first barrier
+// and waited() right after the dependency wait; the destructor (every exit path of every
+// thread) counts the thread out, and the CTA's last thread records the CTA's stamps.
+struct SpanScope {
+  SpanCtx ctx;
+  unsigned* left;            // shared: threads of the CTA still running
+  unsigned long long* t0s;   // shared: the CTA's post-wait stamp
+  __device__ SpanScope(const SpanCtx& c, unsigned* l, unsigned long long* t) : ctx(c), left(l), t0s(t) {}
+  __device__ void init() const {
+    if (ctx.site && threadIdx.x == 0) *left = blockDim.x * blockDim.y;
+  }
+  __device__ void waited() const {
+    if (ctx.site && threadIdx.x == 0) *t0s = global_ns();
+  }
+  __device__ ~SpanScope();
+};
+// Out of line: each exit path carries only the test and the call.
+static __device__ __noinline__ void span_close(SpanCtx ctx, unsigned* left, unsigned long long* t0s) {
+  __threadfence_block();
+  if (atomicSub(left, 1u) != 1u) return;   // not the CTA's last thread
+  const unsigned long long t1 = global_ns();
+  asm volatile("red.relaxed.gpu.global.min.u64 [%0], %1;" ::"l"(&ctx.site->t0), "l"(*t0s) : "memory");
+  asm volatile("red.relaxed.gpu.global.max.u64 [%0], %1;" ::"l"(&ctx.site->t1), "l"(t1) : "memory");
+  if (blockIdx.x == 0 && blockIdx.y == 0) ctx.site->cls = ctx.cls;
+}
+__device__ __forceinline__ SpanScope::~SpanScope() {
+  if (ctx.site) span_close(ctx, left, t0s);
+}
+
 cudaError_t set_wait_limit_tc(long long cycles);
 cudaError_t set_wait_limit_dg(long long cycles);
 cudaError_t set_wait_limit_ds(long long cycles);

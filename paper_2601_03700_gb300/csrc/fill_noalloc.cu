@@ -110,10 +110,9 @@ extern "C" ADEPT_API adept_status adept_skip_kv_fill_noalloc(adept_model* m, int
   int* start = hist + (FILL_VIEW_MAX_LAYERS + 2);
   int* cursor = start + (FILL_VIEW_MAX_LAYERS + 2);
   cudaStream_t st = (cudaStream_t)stream;
-  // bucket by exit layer (the histogram is cleared here), standardise s~ once
-  launch_fill_sort(st, v.dtype, d_h_mapped, n_tokens, v.d_model, d_exit_layer, v.n_layers, hist, start, cursor,
-                   sorted_tok, xs, v.norm_mode, v.norm_eps, v.err_word);
-  model_add_launches(m, 4);
+  // bucket by exit layer (the histogram is rebuilt here), standardise s~ once
+  model_add_launches(m, launch_fill_sort(st, v.dtype, d_h_mapped, n_tokens, v.d_model, d_exit_layer, v.n_layers, hist,
+                                         start, cursor, sorted_tok, xs, v.norm_mode, v.norm_eps, v.err_word));
   // layer r's rows are the sorted prefix with i* < r; groups of at most 32 layers per launch
   GemmProblem probs[32];
   int max_rows[32];

@@ -100,6 +100,7 @@ struct DgParams {
   int bias_aligned, resid_aligned;
   Epi epi;
   unsigned* err;
+  SpanCtx span;
 };
 
 // Several problems of one launch that differ only in the weights, the row range and the
@@ -236,6 +237,9 @@ __global__ void __launch_bounds__(DG_THREADS, 1) gemm_decode_kernel(const __grid
   __shared__ EpiRow s_rr[DG_MAX_M];
   __shared__ float s_red[DG_THREADS / 32][MB * 8];
   __shared__ float s_mu[MB * 8], s_rs[MB * 8];
+  __shared__ unsigned s_span_left;
+  __shared__ unsigned long long s_span_t0;
+  SpanScope span(p.span, &s_span_left, &s_span_t0);
 
   const long long wlim = wait_limit();   // the runtime wait limit, read once
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
@@ -268,6 +272,7 @@ __global__ void __launch_bounds__(DG_THREADS, 1) gemm_decode_kernel(const __grid
     // partial tile (MB*8 rows x 32 features, whatever the row count)
     if (p.splits > 1 && rank == 0) mbar_expect_tx(&red_bar, (uint32_t)((p.splits - 1) * MB * 8 * DG_BN * 4));
   }
+  span.init();
   __syncthreads();
   pdl_launch_dependents();
 
@@ -298,6 +303,7 @@ __global__ void __launch_bounds__(DG_THREADS, 1) gemm_decode_kernel(const __grid
 
   pdl_wait();   // from here on, the preceding kernels' writes are visible
   KT_WAITED();
+  span.waited();
 
   const DevRange prow = dg_rows(p);
   const int rb = prow.b();
@@ -887,6 +893,7 @@ static bool dg_plan(const GemmProblem& q, int max_rows, const DgNorm* norm, int 
   prm.resid_aligned = ((uintptr_t)q.epi.resid & 15) == 0 && q.epi.ld_resid % 4 == 0;
   prm.epi = q.epi;
   prm.err = err;
+  prm.span = g_span;
   // a CTA whose stages fit the ring issues them all before the grid-dependency wait; a
   // longer one (large models) only its first, which bounds the weight traffic of a layer
   // whose rows have all left

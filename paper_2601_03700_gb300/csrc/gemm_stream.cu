@@ -90,6 +90,7 @@ struct DsParams {
   float* part;
   int* cnt;
   unsigned* err;
+  SpanCtx span;
 };
 
 __device__ __forceinline__ uint32_t smem_u32(const void* p) { return (uint32_t)__cvta_generic_to_shared(p); }
@@ -400,6 +401,9 @@ __global__ void __launch_bounds__(DS_THREADS, 2) gemm_stream_kernel(const __grid
   __shared__ int s_pos[16], s_blk[16];   // cache epilogues: each row's position and cache block
   __shared__ int s_info[2][3];           // per hand-off buffer: live problem slot, tile, whole
   __shared__ int s_eok[DS_NE];           // epilogue warps: still following the hand-offs
+  __shared__ unsigned s_span_left;
+  __shared__ unsigned long long s_span_t0;
+  SpanScope span(p.span, &s_span_left, &s_span_t0);
 
   const long long wlim = wait_limit();   // the runtime wait limit, read once
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
@@ -423,6 +427,7 @@ __global__ void __launch_bounds__(DS_THREADS, 2) gemm_stream_kernel(const __grid
     }
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
   }
+  span.init();
   for (int i = tid; i < 2 * 16 * DS_RP; i += DS_THREADS) sT[i] = 0.f;
   __syncthreads();
   pdl_launch_dependents();
@@ -476,6 +481,7 @@ __global__ void __launch_bounds__(DS_THREADS, 2) gemm_stream_kernel(const __grid
 
   pdl_wait();   // from here on, the preceding kernels' writes are visible
   KT_WAITED();
+  span.waited();
 
   // The row counts (device values) and the A operand are read in parallel: every problem's
   // rows start at row 0 (host-checked), so the launch's row bound max_m is staged without
@@ -865,6 +871,7 @@ bool ds_plan(const GemmProblem& q, int n_probs, int max_rows, const DgNorm* norm
   prm.part = ws.part;
   prm.cnt = ws.cnt;
   prm.err = err;
+  prm.span = g_span;
   smem = (size_t)prm.off_p + p_bytes + 1024;
   return smem <= (size_t)DS_SMEM_LIMIT;
 }
@@ -886,8 +893,9 @@ int stream_gemm(cudaStream_t st, const GemmProblem& q, int max_rows, const DgNor
   int grid = 0, mb = 1;
   size_t smem = 0;
   if (!ds_plan(q, 1, max_rows, norm, ws, err, prm, grid, smem, mb)) return -1;
-  if (!tc_encode_weight_3d(&prm.wmap[0], q.B, q.K, q.N, (size_t)q.ldb * 2, DS_BN, DS_KB / 64)) return -1;
-  prm.bt[0] = ds_tiled(q, prm.nkb);
+  prm.bt[0] = ds_tiled(q, prm.nkb);   // the tensor map is read only without the tiled copy
+  if (!prm.bt[0] && !tc_encode_weight_3d(&prm.wmap[0], q.B, q.K, q.N, (size_t)q.ldb * 2, DS_BN, DS_KB / 64))
+    return -1;
   prm.grouped = 0;
   prm.rows[0] = q.rows;
   prm.epi[0] = q.epi;
@@ -910,12 +918,13 @@ int stream_gemm_grouped(cudaStream_t st, const GemmProblem* probs, int n, int ma
   size_t smem = 0;
   if (!ds_plan(q0, n, max_rows, nullptr, ws, err, prm, grid, smem, mb)) return -1;
   for (int i = 0; i < n; ++i) {
-    if (((uintptr_t)probs[i].B & 15) ||
-        !tc_encode_weight_3d(&prm.wmap[i], probs[i].B, q0.K, q0.N, (size_t)q0.ldb * 2, DS_BN, DS_KB / 64))
+    prm.bt[i] = ds_tiled(probs[i], prm.nkb);   // the tensor map is read only without the tiled copy
+    if (!prm.bt[i] && (((uintptr_t)probs[i].B & 15) ||
+                       !tc_encode_weight_3d(&prm.wmap[i], probs[i].B, q0.K, q0.N, (size_t)q0.ldb * 2, DS_BN,
+                                            DS_KB / 64)))
       return -1;
     prm.rows[i] = probs[i].rows;
     prm.epi[i] = probs[i].epi;
-    prm.bt[i] = ds_tiled(probs[i], prm.nkb);
   }
   prm.grouped = 1;
   const cudaError_t e = mb == 2 ? ds_launch<2, EPI_KV, DS_MAXG>(st, prm, grid, smem)

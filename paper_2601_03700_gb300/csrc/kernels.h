@@ -50,6 +50,7 @@ bool launch_exit_small(cudaStream_t st, const float* Xin, const float* Xout, con
                        bf16* xhat_next, int smode, float seps, int metric, int aao_len, const int* tok_pos,
                        unsigned* err);
 void launch_set_float(cudaStream_t st, float* p, float v);
+void launch_span_collect(cudaStream_t st, SpanSite* sites, int n, SpanTotal* tot, int n_cls);
 // Generation-step staging of the caller's inputs (forced NULL -> zeros) and outputs (each
 // output optional).
 void launch_stage_in(cudaStream_t st, float* d_delta, float delta, const int* tokens, int* dec_tok, const int* forced,
@@ -82,9 +83,10 @@ void launch_hsm_out(cudaStream_t st, int dt, const float* h5, const float* c0f, 
 // Greedy token per row (lowest index on ties); part_v / part_i: rows * 32 partials.
 int launch_argmax(cudaStream_t st, const float* logits, int V, int rows, int* out, float* part_v, int* part_i);
 void launch_head_rows(cudaStream_t st, int batch, int prompt_len, int last, int* rows);
-void launch_fill_sort(cudaStream_t st, int dt, const void* h, int n, int D, const int* exit_layer, int n_layers,
-                      int* hist, int* start, int* cursor, int* sorted_tok, void* xs, int mode, float eps,
-                      unsigned* err);
+// Returns the number of launches (1 for calls of at most 32 tokens, else 2).
+int launch_fill_sort(cudaStream_t st, int dt, const void* h, int n, int D, const int* exit_layer, int n_layers,
+                     int* hist, int* start, int* cursor, int* sorted_tok, void* xs, int mode, float eps,
+                     unsigned* err);
 void launch_fold_rows(cudaStream_t st, int dt, void* dst, int ld_dst, const void* src, int n_rows, int K,
                       const float* gamma, const float* beta, const float* bias_in, float* bias_out, int row_mode);
 void launch_to_f32(cudaStream_t st, int dt, const void* src, float* dst, int n);
@@ -107,6 +109,7 @@ constexpr int ATTN_MAX_SPLIT = 32;
 void launch_attention(cudaStream_t st, int dt, const void* q, int ld_q, void* out, int ld_out, DevRange rows,
                       int max_rows, const int* row_tok, const int* tok_seq, const int* tok_pos, const int* seq_len,
                       KVCacheView cache, int layer0, int n_heads, int causal, int decode_keys, float* ws,
-                      int* counters, unsigned* err, const int* key_exit = nullptr, int kp_len = 0);
+                      int* counters, unsigned* err, const int* key_exit = nullptr, int kp_len = 0,
+                      int q_rows = 0, int n_layers = 0);
 
 }  // namespace adept

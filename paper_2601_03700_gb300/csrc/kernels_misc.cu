@@ -99,6 +99,22 @@ __global__ void embed_kernel(const int* tokens, int n_tok, const int* tok_pos, c
   for (int d = threadIdx.x; d < D; d += blockDim.x) x[d] = (x[d] - mu) * rstd * g[d] + b[d];
 }
 
+// Grid of the row kernels whose live row count is a device value, usually far below its
+// bound in a prompt pass (the mapper's rows, the standardisation, the exit moves): the rows are
+// taken in turn by at most per_sm CTAs per SM, so a pass whose bound is thousands of rows does
+// not launch thousands of CTAs that find no row.
+static int row_grid(int max_rows, int per_sm) {
+  static int sms = 0;
+  if (!sms) {
+    int dev = 0;
+    cudaGetDevice(&dev);
+    cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+    if (sms <= 0) sms = 1;
+  }
+  return std::min(max_rows, per_sm * sms);
+}
+static int hsm_grid(int max_rows) { return row_grid(max_rows, 2); }
+
 // ---------------------------------------------------------------------------
 // standardisation of a layer input (gains folded into the next GEMM)
 // ---------------------------------------------------------------------------
@@ -107,14 +123,14 @@ __global__ void standardize_kernel(const float* X, int ldx, const int* in_rows, 
                                    float eps, T* out, int ld_out) {
   PDL_ENTRY();
   __shared__ float red[32];
-  const int r = rows.b() + blockIdx.x;
-  if (r >= rows.e()) return;
+  const int rb = rows.b(), re = rows.e();
+  for (int r = rb + blockIdx.x; r < re; r += gridDim.x) {   // rows of the live range, in turn
   const int src = in_rows ? in_rows[r] : r;
   const float* x = X + (size_t)src * ldx;
   T* o = out + (size_t)r * ld_out;
   if (mode == NORM_COPY) {
     for (int d = threadIdx.x; d < D; d += blockDim.x) o[d] = from_f<T>(x[d]);
-    return;
+    continue;
   }
   float mu = 0.f;
   if (mode == NORM_LN) {
@@ -129,6 +145,7 @@ __global__ void standardize_kernel(const float* X, int ldx, const int* in_rows, 
   }
   const float rstd = rsqrtf(block_sum(s2, red) / D + eps);
   for (int d = threadIdx.x; d < D; d += blockDim.x) o[d] = from_f<T>((x[d] - mu) * rstd);
+  }
 }
 
 // In-place LayerNorm with gain and shift (the post-LN encoder's residual stream).
@@ -273,8 +290,8 @@ __global__ void exit_move_kernel(const float* Xin, const float* Xout, const floa
                                  const int* n_rows, const int* dst, const float* inv_norm, float* Xnext, float* Inext,
                                  float* hsm_s, float* hsm_prev, float* hsm_I) {
   PDL_ENTRY();
-  const int r = blockIdx.x;
-  if (r >= *n_rows) return;
+  const int n = *n_rows;
+  for (int r = blockIdx.x; r < n; r += gridDim.x) {
   const int d0 = dst[r];
   const float* s = Xout + (size_t)r * D;
   const float* in = I + (size_t)r * D;
@@ -295,6 +312,7 @@ __global__ void exit_move_kernel(const float* Xin, const float* Xout, const floa
       hsm_prev[k * D + d] = sp[d];
       hsm_I[k * D + d] = in[d];
     }
+  }
   }
 }
 
@@ -634,6 +652,26 @@ __global__ void set_float_kernel(float* p, float v) {
   PDL_ENTRY(); *p = v; }
 void launch_set_float(cudaStream_t st, float* p, float v) { launch_k(set_float_kernel, 1, 1, 0, st, p, v); }
 
+// Span timer: every used launch site's span into its class total; the site is reset.
+__global__ void span_collect_kernel(SpanSite* sites, int n, SpanTotal* tot, int n_cls) {
+  PDL_ENTRY();
+  for (int i = threadIdx.x; i < n; i += blockDim.x) {
+    SpanSite& s = sites[i];
+    const unsigned long long t0 = s.t0, t1 = s.t1;
+    if (t0 == ~0ull) continue;
+    if (t1 > t0 && s.cls >= 0 && s.cls < n_cls) {
+      atomicAdd(&tot[s.cls].ns, t1 - t0);
+      atomicAdd(&tot[s.cls].n, 1ull);
+    }
+    s.t0 = ~0ull;
+    s.t1 = 0ull;
+  }
+}
+
+void launch_span_collect(cudaStream_t st, SpanSite* sites, int n, SpanTotal* tot, int n_cls) {
+  launch_k(span_collect_kernel, 1, 1024, 0, st, sites, n, tot, n_cls);
+}
+
 // Generation-step staging: the caller's inputs into the library's fixed buffers (the captured
 // step reads only those), in one launch instead of a kernel and two copies.
 __global__ void stage_in_kernel(float* d_delta, float delta, const int* tokens, int* dec_tok, const int* forced,
@@ -819,8 +857,8 @@ __global__ void __launch_bounds__(256) hsm_prep_kernel(const float* hs, const fl
   PDL_ENTRY();
   extern __shared__ float s_xn[];
   __shared__ float red[32 * 3];
-  const int k = rows.b() + blockIdx.x;
-  if (k >= rows.e()) return;
+  const int kb = rows.b(), ke = rows.e();
+  for (int k = kb + blockIdx.x; k < ke; k += gridDim.x) {   // rows of the live range, in turn
   float xa[EPT], xb[EPT], xc[EPT], g[EPT];
   hsm_load_row(hs + (size_t)k * D, D, xa);
   hsm_load_row(hp + (size_t)k * D, D, xb);
@@ -864,6 +902,7 @@ __global__ void __launch_bounds__(256) hsm_prep_kernel(const float* hs, const fl
     c0f[(size_t)k * D + t] = acc;
     c0t[(size_t)k * D + t] = from_f<T>(acc);
   }
+  }
 }
 
 // h4 = RMSNorm_g1(h3) + h1 (the MLP's addition), rounded for FC4.
@@ -872,8 +911,8 @@ __global__ void __launch_bounds__(1024) hsm_mid_kernel(const float* h3, const fl
                                T* h4) {
   PDL_ENTRY();
   __shared__ float red[32];
-  const int k = rows.b() + blockIdx.x;
-  if (k >= rows.e()) return;
+  const int kb = rows.b(), ke = rows.e();
+  for (int k = kb + blockIdx.x; k < ke; k += gridDim.x) {
   float a[EPT], b[EPT];
   hsm_load_row(h3 + (size_t)k * m1, m1, a);
   hsm_load_row(h1 + (size_t)k * m1, m1, b);
@@ -887,6 +926,7 @@ __global__ void __launch_bounds__(1024) hsm_mid_kernel(const float* h3, const fl
     const int d = threadIdx.x + j * blockDim.x;
     if (d < m1) h4[(size_t)k * m1 + d] = from_f<T>(a[j] * sc * g1[d] + b[j]);
   }
+  }
 }
 
 // s~ = RMSNorm_g2(h5) + c0 (the final addition); written to the token's final state,
@@ -899,8 +939,8 @@ __global__ void __launch_bounds__(1024) hsm_out_kernel(const float* h5, const fl
                                int fill_mode, float norm_eps, T* xhead) {
   PDL_ENTRY();
   __shared__ float red[32];
-  const int k = rows.b() + blockIdx.x;
-  if (k >= rows.e()) return;
+  const int kb = rows.b(), ke = rows.e();
+  for (int k = kb + blockIdx.x; k < ke; k += gridDim.x) {
   const int tok = exit_tok[k];
   float f[EPT];
   if (identity) {
@@ -933,7 +973,7 @@ __global__ void __launch_bounds__(1024) hsm_out_kernel(const float* h5, const fl
       const int d = threadIdx.x + j * blockDim.x;
       if (d < D) o[d] = from_f<T>(f[j]);
     }
-    return;
+    continue;
   }
   float mu = 0.f;
   if (fill_mode == NORM_LN) {
@@ -961,6 +1001,7 @@ __global__ void __launch_bounds__(1024) hsm_out_kernel(const float* h5, const fl
       o[d] = x;
       if (oh) oh[d] = x;
     }
+  }
   }
 }
 
@@ -1161,28 +1202,73 @@ __global__ void head_rows_kernel(int batch, int prompt_len, int last, int* rows)
 // skipped-layer fill input: bucket tokens by exit layer (ascending) so that the rows of
 // skipped layer r (tokens with i* < r) are a prefix, and standardise s~ once.
 // ---------------------------------------------------------------------------
-__global__ void fill_hist_kernel(const int* exit_layer, int n, int n_layers, int* hist, unsigned* err) {
+// The histogram and the scan in one CTA (histogram in shared memory): one launch instead of
+// a memset and two kernels ahead of the scatter.  Calls of at most FILL_PLAN_ROWS tokens
+// (generation steps, small fills) also place and standardise the rows here, one warp per row,
+// so that the whole pre-pass is this one launch.
+constexpr int FILL_PLAN_ROWS = 32;
+template <typename T>
+__global__ void __launch_bounds__(1024) fill_plan_kernel(const T* h, int D, const int* exit_layer, int n, int n_layers,
+                                                         int* hist, int* start, int* cursor, int* sorted_tok, T* xs,
+                                                         int mode, float eps, unsigned* err) {
   PDL_ENTRY();
-  const int j = blockIdx.x * blockDim.x + threadIdx.x;
-  if (j >= n) return;
-  int l = exit_layer[j];
-  if (l < 1 || l > n_layers) {
-    atomicOr(err, ERRW_EXIT_LAYER);
-    l = n_layers;
+  extern __shared__ int s_hist[];   // [n_layers + 2] counts, then [n_layers + 2] running slots
+  int* s_cur = s_hist + n_layers + 2;
+  __shared__ int s_slot[FILL_PLAN_ROWS];
+  for (int l = threadIdx.x; l < n_layers + 2; l += blockDim.x) s_hist[l] = 0;
+  __syncthreads();
+  bool bad = false;
+  for (int j = threadIdx.x; j < n; j += blockDim.x) {
+    int l = exit_layer[j];
+    if (l < 1 || l > n_layers) {
+      bad = true;
+      l = n_layers;
+    }
+    atomicAdd(&s_hist[l], 1);
   }
-  atomicAdd(&hist[l], 1);
-}
-
-// hist[1..N] -> start[l] (exclusive prefix) and prefix[r] = #(i* < r) = start[r].
-__global__ void fill_scan_kernel(const int* hist, int n_layers, int* start, int* cursor) {
-  PDL_ENTRY();
-  if (threadIdx.x != 0 || blockIdx.x != 0) return;
-  int acc = 0;
-  for (int l = 0; l <= n_layers + 1; ++l) {
-    start[l] = acc;
-    cursor[l] = 0;
-    if (l >= 1 && l <= n_layers) acc += hist[l];
+  if (bad) atomicOr(err, ERRW_EXIT_LAYER);
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    int acc = 0;
+    for (int l = 0; l <= n_layers + 1; ++l) {
+      start[l] = acc;
+      s_cur[l] = acc;
+      cursor[l] = 0;
+      hist[l] = s_hist[l];
+      if (l >= 1 && l <= n_layers) acc += s_hist[l];
+    }
   }
+  if (n > FILL_PLAN_ROWS) return;
+  __syncthreads();
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  if (threadIdx.x < n) {
+    int l = exit_layer[threadIdx.x];
+    if (l < 1 || l > n_layers) l = n_layers;
+    const int slot = atomicAdd(&s_cur[l], 1);
+    s_slot[threadIdx.x] = slot;
+    sorted_tok[slot] = threadIdx.x;
+  }
+  __syncthreads();
+  if (warp >= n) return;
+  const T* x = h + (size_t)warp * D;
+  T* o = xs + (size_t)s_slot[warp] * D;
+  if (mode == NORM_COPY) {
+    for (int d = lane; d < D; d += 32) o[d] = x[d];
+    return;
+  }
+  float mu = 0.f;
+  if (mode == NORM_LN) {
+    float sm = 0.f;
+    for (int d = lane; d < D; d += 32) sm += to_f(x[d]);
+    mu = warp_sum(sm) / D;
+  }
+  float s2 = 0.f;
+  for (int d = lane; d < D; d += 32) {
+    const float c = to_f(x[d]) - mu;
+    s2 += c * c;
+  }
+  const float rstd = rsqrtf(warp_sum(s2) / D + eps);
+  for (int d = lane; d < D; d += 32) o[d] = from_f<T>((to_f(x[d]) - mu) * rstd);
 }
 
 template <typename T>
@@ -1316,9 +1402,9 @@ void launch_standardize(cudaStream_t st, int dt, const float* X, int ldx, const 
                         int max_rows, int D, int mode, float eps, void* out, int ld_out) {
   if (max_rows <= 0) return;
   if (dt == 1)
-    launch_k(standardize_kernel<bf16>, max_rows, 256, 0, st, X, ldx, in_rows, rows, D, mode, eps, (bf16*)out, ld_out);
+    launch_k(standardize_kernel<bf16>, row_grid(max_rows, 8), 256, 0, st, X, ldx, in_rows, rows, D, mode, eps, (bf16*)out, ld_out);
   else
-    launch_k(standardize_kernel<float>, max_rows, 256, 0, st, X, ldx, in_rows, rows, D, mode, eps, (float*)out, ld_out);
+    launch_k(standardize_kernel<float>, row_grid(max_rows, 8), 256, 0, st, X, ldx, in_rows, rows, D, mode, eps, (float*)out, ld_out);
 }
 
 void launch_layernorm_inplace(cudaStream_t st, float* X, DevRange rows, int max_rows, int D, const float* g,
@@ -1347,7 +1433,7 @@ void launch_exit_move(cudaStream_t st, const float* Xin, const float* Xout, cons
                       const int* n_rows, int max_rows, const int* dst, const float* inv_norm, float* Xnext,
                       float* Inext, float* hsm_s, float* hsm_prev, float* hsm_I) {
   if (max_rows <= 0) return;
-  launch_k(exit_move_kernel, max_rows, 256, 0, st, Xin, Xout, I, first, D, n_rows, dst, inv_norm, Xnext, Inext, hsm_s,
+  launch_k(exit_move_kernel, row_grid(max_rows, 8), 256, 0, st, Xin, Xout, I, first, D, n_rows, dst, inv_norm, Xnext, Inext, hsm_s,
                                              hsm_prev, hsm_I);
 }
 
@@ -1376,7 +1462,8 @@ static void hsm_prep_go(cudaStream_t st, int thr, const float* hs, const float* 
     cudaFuncSetAttribute(hsm_prep_kernel<T, EPT>, cudaFuncAttributeMaxDynamicSharedMemorySize, 3 * 16 * 256 * 4);
     attr = true;
   }
-  launch_k(hsm_prep_kernel<T, EPT>, max_rows, thr, smem, st, hs, hp, hI, rows, D, g0, conv, eps, c0f, (T*)c0t);
+  launch_k(hsm_prep_kernel<T, EPT>, hsm_grid(max_rows), thr, smem, st, hs, hp, hI, rows, D, g0, conv, eps, c0f,
+           (T*)c0t);
 }
 
 void launch_hsm_prep(cudaStream_t st, int dt, const float* hs, const float* hp, const float* hI, DevRange rows,
@@ -1412,11 +1499,11 @@ void launch_hsm_mid(cudaStream_t st, int dt, const float* h3, const float* h1, D
   }
   const bool small = m1 <= 4 * 256;
   if (dt == 1) {
-    if (small) launch_k(hsm_mid_kernel<bf16, 4>, max_rows, thr, 0, st, h3, h1, rows, m1, g1, eps, (bf16*)h4);
-    else launch_k(hsm_mid_kernel<bf16, 8>, max_rows, thr, 0, st, h3, h1, rows, m1, g1, eps, (bf16*)h4);
+    if (small) launch_k(hsm_mid_kernel<bf16, 4>, hsm_grid(max_rows), thr, 0, st, h3, h1, rows, m1, g1, eps, (bf16*)h4);
+    else launch_k(hsm_mid_kernel<bf16, 8>, hsm_grid(max_rows), thr, 0, st, h3, h1, rows, m1, g1, eps, (bf16*)h4);
   } else {
-    if (small) launch_k(hsm_mid_kernel<float, 4>, max_rows, thr, 0, st, h3, h1, rows, m1, g1, eps, (float*)h4);
-    else launch_k(hsm_mid_kernel<float, 8>, max_rows, thr, 0, st, h3, h1, rows, m1, g1, eps, (float*)h4);
+    if (small) launch_k(hsm_mid_kernel<float, 4>, hsm_grid(max_rows), thr, 0, st, h3, h1, rows, m1, g1, eps, (float*)h4);
+    else launch_k(hsm_mid_kernel<float, 8>, hsm_grid(max_rows), thr, 0, st, h3, h1, rows, m1, g1, eps, (float*)h4);
   }
 }
 
@@ -1436,7 +1523,7 @@ void launch_hsm_out(cudaStream_t st, int dt, const float* h5, const float* c0f, 
   }
   const bool small = D <= 4 * 256;
 #define HSM_OUT(T, E)                                                                                              \
-  launch_k(hsm_out_kernel<T, E>, max_rows, thr, 0, st, h5, c0f, hs, identity, rows, D, g2, eps, exit_tok, final_, \
+  launch_k(hsm_out_kernel<T, E>, hsm_grid(max_rows), thr, 0, st, h5, c0f, hs, identity, rows, D, g2, eps, exit_tok, final_, \
            (T*)xfill, fill_mode, norm_eps, (T*)xhead)
   if (dt == 1) {
     if (small) HSM_OUT(bf16, 4);
@@ -1552,19 +1639,24 @@ void launch_head_rows(cudaStream_t st, int batch, int prompt_len, int last, int*
   launch_k(head_rows_kernel, cdiv(batch, 128), 128, 0, st, batch, prompt_len, last, rows);
 }
 
-void launch_fill_sort(cudaStream_t st, int dt, const void* h, int n, int D, const int* exit_layer, int n_layers,
-                      int* hist, int* start, int* cursor, int* sorted_tok, void* xs, int mode, float eps,
-                      unsigned* err) {
-  cudaMemsetAsync(hist, 0, sizeof(int) * (n_layers + 2), st);
-  if (n > 0) launch_k(fill_hist_kernel, cdiv(n, 256), 256, 0, st, exit_layer, n, n_layers, hist, err);
-  launch_k(fill_scan_kernel, 1, 32, 0, st, hist, n_layers, start, cursor);
-  if (n <= 0) return;
+int launch_fill_sort(cudaStream_t st, int dt, const void* h, int n, int D, const int* exit_layer, int n_layers,
+                     int* hist, int* start, int* cursor, int* sorted_tok, void* xs, int mode, float eps,
+                     unsigned* err) {
+  const size_t smem = (size_t)2 * (n_layers + 2) * sizeof(int);
+  if (dt == 1)
+    launch_k(fill_plan_kernel<bf16>, 1, 1024, smem, st, (const bf16*)h, D, exit_layer, n, n_layers, hist, start, cursor,
+             sorted_tok, (bf16*)xs, mode, eps, err);
+  else
+    launch_k(fill_plan_kernel<float>, 1, 1024, smem, st, (const float*)h, D, exit_layer, n, n_layers, hist, start,
+             cursor, sorted_tok, (float*)xs, mode, eps, err);
+  if (n <= FILL_PLAN_ROWS) return 1;   // placed and standardised by the plan kernel
   if (dt == 1)
     launch_k(fill_scatter_kernel<bf16>, n, 256, 0, st, (const bf16*)h, n, D, exit_layer, n_layers, start, cursor,
                                                  sorted_tok, (bf16*)xs, mode, eps);
   else
     launch_k(fill_scatter_kernel<float>, n, 256, 0, st, (const float*)h, n, D, exit_layer, n_layers, start, cursor,
                                                   sorted_tok, (float*)xs, mode, eps);
+  return 2;
 }
 
 void launch_fold_rows(cudaStream_t st, int dt, void* dst, int ld_dst, const void* src, int n_rows, int K,

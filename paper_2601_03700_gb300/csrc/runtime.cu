@@ -25,6 +25,7 @@ using namespace adept;
 
 namespace adept {
 thread_local bool g_pdl = false;
+thread_local SpanCtx g_span = {nullptr, 0};
 }
 
 namespace {
@@ -44,6 +45,11 @@ struct LayerW {
   float *ln1_g = nullptr, *ln1_b = nullptr, *ln2_g = nullptr, *ln2_b = nullptr;  // post-LN (encoder)
   // tile-contiguous copies for the weight-streaming kernels (bf16 decoders; GemmProblem::Bt)
   void *t_qkv = nullptr, *t_o = nullptr, *t_up = nullptr, *t_down = nullptr;
+  // cross-attention sublayer (max_src > 0): W_Qc with the LN_c gain / shift folded in, the
+  // source K/V projection [2 D_kv, D] (K rows, then V rows), W_Oc
+  void *w_cq = nullptr, *w_ckv = nullptr, *w_co = nullptr;
+  float *b_cq = nullptr, *b_ckv = nullptr, *b_co = nullptr;
+  void *t_cq = nullptr, *t_co = nullptr;
 };
 
 struct ProfRec {
@@ -108,6 +114,15 @@ struct adept_model {
   std::vector<int> h_block_table, free_list, h_seq_len;
   std::vector<std::vector<int>> seq_blocks;
   int* d_seq_len = nullptr;
+  // source cache of the cross-attention (max_src > 0): per layer, max_src positions per
+  // sequence in 16-position blocks (sequence b owns blocks b * cs_blocks_per_seq ...)
+  void *ck_pool = nullptr, *cv_pool = nullptr;
+  int cs_blocks_per_seq = 0;
+  int* d_cblock_table = nullptr;
+  int* d_src_len = nullptr;          // source positions per sequence (0: not set)
+  std::vector<int> h_src_len;
+  int *cs_seq = nullptr, *cs_pos = nullptr, *cs_iota = nullptr;   // source row -> (sequence, position)
+  void* cs_x = nullptr;              // source states in the GEMM input type
   // pass workspaces (T_max rows)
   int T_max = 0;
   float *X_in[2] = {nullptr, nullptr}, *X_out = nullptr, *I[2] = {nullptr, nullptr};
@@ -151,6 +166,7 @@ struct adept_model {
   std::vector<int> dec_warm;                // direct runs done per batch size
   // options / instrumentation
   int hsm_identity = 0, profile = 0, force_simt = 0, use_graph = 1, use_dg = 1, use_stream = 1, use_tiled = 1;
+  int use_attn_tc = 1;   // prompt-pass attention on the tcgen05 kernel
   int exit_metric = 0;   // EXIT_GLOBAL / EXIT_LOCAL / EXIT_BOTH
   int all_at_once = 0;   // prompt passes: sequences leave with their last prompt token
   int stop_entirely = 0; // encoders: exited tokens get no deeper K/V and leave deeper attention
@@ -165,7 +181,14 @@ struct adept_model {
   adept_status deferred = ADEPT_OK;   // an error met inside a launch sequence, reported by check_launch
   int64_t graph_launches = 0;   // kernels in one captured generation step
   ProfRec prof[ADEPT_PROF_NCLASS];
+  // in-situ spans of the weight-streaming launches (ADEPT_OPT_SPAN_TIMER)
+  int span_on = 0;
+  SpanSite* span_sites = nullptr;   // SPAN_SITES launch sites, taken in turn (a pass uses fewer)
+  SpanTotal* span_tot = nullptr;    // per kernel class
+  unsigned span_next = 0;
+  unsigned span_in_pass = 0;        // sites taken since the last collect (at most SPAN_SITES)
 };
+constexpr unsigned SPAN_SITES = 1024;
 
 // ---------------------------------------------------------------------------
 // small helpers
@@ -257,6 +280,20 @@ static KVCacheView cache_view(const adept_model* m) {
   return c;
 }
 
+static KVCacheView cross_view(const adept_model* m) {
+  KVCacheView c;
+  c.k = m->ck_pool;
+  c.v = m->cv_pool;
+  c.block_table = m->d_cblock_table;
+  c.max_blocks_per_seq = m->cs_blocks_per_seq;
+  c.n_blocks = m->cfg.max_batch * m->cs_blocks_per_seq;
+  c.n_kv_heads = m->Hkv;
+  c.head_dim = m->dh;
+  c.block_tokens = m->cfg.kv_block_tokens;
+  c.max_batch = m->cfg.max_batch;
+  return c;
+}
+
 static Epi epi_base() {
   Epi e;
   memset(&e, 0, sizeof e);
@@ -325,10 +362,39 @@ static DsWork ds_work(const adept_model* m) {
   return w;
 }
 
+// Sets g_span for the weight-streaming launch of one call (class cls) while the span timer
+// is on; consecutive launches take different sites.
+struct SpanGuard {
+  SpanCtx prev;
+  SpanGuard(adept_model* m, int cls) : prev(g_span) {
+    if (m->span_on && m->span_sites && m->span_in_pass < SPAN_SITES) {
+      // a site is used once between two collects (a pass with more launches records its first
+      // SPAN_SITES only)
+      g_span = SpanCtx{m->span_sites + (m->span_next++ % SPAN_SITES), cls};
+      m->span_in_pass += 1;
+    } else {
+      g_span = SpanCtx{nullptr, 0};
+    }
+  }
+  ~SpanGuard() { g_span = prev; }
+  SpanGuard(const SpanGuard&) = delete;
+  SpanGuard& operator=(const SpanGuard&) = delete;
+};
+
 // A weight-streaming problem of at most DG_MAX_M rows: the stream-K kernel where it takes the
 // shape (weights large enough to stream, A rows fitting in shared memory), else the cluster
 // K-split kernel.  Returns the launches, or -1 when neither takes it.
-static int streaming_gemm(adept_model* m, cudaStream_t st, const GemmProblem& p0, int max_rows, const DgNorm* norm) {
+// End of a pass with the span timer on: the pass's sites into the class totals.
+static void span_collect(adept_model* m, cudaStream_t st) {
+  if (!m->span_on || !m->span_sites) return;
+  launch_span_collect(st, m->span_sites, (int)SPAN_SITES, m->span_tot, ADEPT_PROF_NCLASS);
+  m->launches += 1;
+  m->span_in_pass = 0;
+}
+
+static int streaming_gemm(adept_model* m, cudaStream_t st, const GemmProblem& p0, int max_rows, const DgNorm* norm,
+                          int cls) {
+  SpanGuard sg(m, cls);
   GemmProblem p = p0;
   if (!m->use_tiled) p.Bt = nullptr;
   if (stream_gemm(st, p, max_rows, norm, ds_work(m), m->err_word) >= 0) return 1;
@@ -337,6 +403,7 @@ static int streaming_gemm(adept_model* m, cudaStream_t st, const GemmProblem& p0
 
 // The grouped skipped-layer fill of a few tokens on the weight-streaming kernels.
 static int streaming_gemm_grouped(adept_model* m, cudaStream_t st, const GemmProblem* probs0, int n, int max_rows) {
+  SpanGuard sg(m, ADEPT_PROF_KV_FILL);
   std::vector<GemmProblem> copy;
   const GemmProblem* probs = probs0;
   if (!m->use_tiled) {
@@ -352,7 +419,7 @@ static void gemm(adept_model* m, cudaStream_t st, const GemmProblem* probs, int 
                  int cls, double flops = 0, double bytes = 0) {
   cudaEvent_t b = nullptr;
   prof_begin(m, cls, st, &b);
-  if (dg_takes(m, n_probs, probs[0], max_rows[0], nullptr) && streaming_gemm(m, st, probs[0], max_rows[0], nullptr) >= 0) {
+  if (dg_takes(m, n_probs, probs[0], max_rows[0], nullptr) && streaming_gemm(m, st, probs[0], max_rows[0], nullptr, cls) >= 0) {
     m->launches += 1;
     prof_end(m, cls, st, b, flops, bytes);
     return;
@@ -393,7 +460,7 @@ static void gemm_std(adept_model* m, cudaStream_t st, const GemmProblem& p, int 
   if (dg_takes(m, 1, p, max_rows, &nrm)) {
     cudaEvent_t b = nullptr;
     prof_begin(m, cls, st, &b);
-    if (streaming_gemm(m, st, p, max_rows, &nrm) >= 0) {
+    if (streaming_gemm(m, st, p, max_rows, &nrm, cls) >= 0) {
       m->launches += 1;
       prof_end(m, cls, st, b, 0, 0);
       return;
@@ -504,6 +571,10 @@ static adept_status validate_cfg(adept_config* c) {
     return fail(nullptr, ADEPT_ERR_INVALID_ARG, "encoder needs n_classes >= 1");
   if ((long long)c->max_batch * c->max_seq > (1LL << 26))
     return fail(nullptr, ADEPT_ERR_INVALID_ARG, "max_batch * max_seq too large");
+  if (c->max_src < 0 || (c->max_src > 0 && c->family != ADEPT_FAMILY_GPT2))
+    return fail(nullptr, ADEPT_ERR_INVALID_ARG, "cross-attention (max_src > 0) is defined for GPT-2-family decoders");
+  if ((long long)c->max_batch * c->max_src > (1LL << 24))
+    return fail(nullptr, ADEPT_ERR_INVALID_ARG, "max_batch * max_src too large");
   return ADEPT_OK;
 }
 
@@ -597,6 +668,24 @@ static adept_status load_weights(adept_model* m, Loader& ld) {
         TRY(ld.vec_f32(p + "ffn_norm.b", D, &w.ln2_b));
       }
     }
+    if (c.max_src > 0) {
+      // cross-attention: LN_c folded into W_Qc (like the layer's input norm into W_qkv)
+      float *cbq = nullptr, *cbk = nullptr, *cbv = nullptr, *cg = nullptr, *cb = nullptr;
+      TRY(ld.vec_f32(p + "cbq", Dq, &cbq));
+      TRY(ld.vec_f32(p + "cbk", Dkv, &cbk));
+      TRY(ld.vec_f32(p + "cbv", Dkv, &cbv));
+      TRY(ld.tmp_f32(p + "cross_norm.g", D, 0, &cg));
+      TRY(ld.tmp_f32(p + "cross_norm.b", D, 1, &cb));
+      TRY(dalloc(m, &w.w_cq, (size_t)Dq * D * m->esz));
+      TRY(dalloc_t(m, &w.b_cq, Dq));
+      TRY(ld.fold(p + "cwq", Dq, D, w.w_cq, 0, cg, cb, cbq, w.b_cq));
+      TRY(dalloc(m, &w.w_ckv, (size_t)2 * Dkv * D * m->esz));
+      TRY(dalloc_t(m, &w.b_ckv, 2 * Dkv));
+      TRY(ld.fold(p + "cwk", Dkv, D, w.w_ckv, 0, nullptr, nullptr, cbk, w.b_ckv));
+      TRY(ld.fold(p + "cwv", Dkv, D, w.w_ckv, Dkv, nullptr, nullptr, cbv, w.b_ckv));
+      TRY(ld.upload(p + "cwo", (int64_t)D * Dq, &w.w_co));
+      TRY(ld.vec_f32(p + "cbo", D, &w.b_co));
+    }
   }
   // output heads (final norm gain / shift folded into the head)
   if (fam == ADEPT_FAMILY_LLAMA) {
@@ -682,6 +771,27 @@ static adept_status alloc_runtime(adept_model* m) {
   m->h_seq_len.assign(c.max_batch, 0);
   TRY(dalloc_t(m, &m->d_seq_len, c.max_batch));
   CUDA_TRY(m, cudaMemset(m->d_seq_len, 0, c.max_batch * sizeof(int)));
+  if (c.max_src > 0) {
+    // source cache: every sequence owns its blocks (b * per_seq + k), so the table is fixed
+    m->cs_blocks_per_seq = cdiv(c.max_src, c.kv_block_tokens);
+    const int nb = c.max_batch * m->cs_blocks_per_seq;
+    const size_t cper = (size_t)nb * m->Hkv * c.kv_block_tokens * m->dh;
+    TRY(dalloc(m, &m->ck_pool, cper * m->N * m->esz));
+    TRY(dalloc(m, &m->cv_pool, cper * m->N * m->esz));
+    std::vector<int> tab(nb), iota((size_t)c.max_batch * c.max_src);
+    for (int i = 0; i < nb; ++i) tab[i] = i;
+    for (size_t i = 0; i < iota.size(); ++i) iota[i] = (int)i;
+    TRY(dalloc_t(m, &m->d_cblock_table, nb));
+    CUDA_TRY(m, cudaMemcpy(m->d_cblock_table, tab.data(), nb * sizeof(int), cudaMemcpyHostToDevice));
+    TRY(dalloc_t(m, &m->cs_iota, iota.size()));
+    CUDA_TRY(m, cudaMemcpy(m->cs_iota, iota.data(), iota.size() * sizeof(int), cudaMemcpyHostToDevice));
+    TRY(dalloc_t(m, &m->cs_seq, iota.size()));
+    TRY(dalloc_t(m, &m->cs_pos, iota.size()));
+    TRY(dalloc(m, &m->cs_x, iota.size() * D * m->esz));
+    TRY(dalloc_t(m, &m->d_src_len, c.max_batch));
+    CUDA_TRY(m, cudaMemset(m->d_src_len, 0, c.max_batch * sizeof(int)));
+    m->h_src_len.assign(c.max_batch, 0);
+  }
   // pass workspaces
   const size_t TD = (size_t)T * D;
   for (int k = 0; k < 2; ++k) {
@@ -771,6 +881,10 @@ static adept_status make_tiled(adept_model* m, cudaStream_t st) {
     TRY(tile_into(m, st, w.w_o, D, Dq, &w.t_o));
     TRY(tile_into(m, st, w.w_up, w.up_rows, D, &w.t_up));
     TRY(tile_into(m, st, w.w_down, D, F, &w.t_down));
+    if (w.w_cq) {
+      TRY(tile_into(m, st, w.w_cq, Dq, D, &w.t_cq));
+      TRY(tile_into(m, st, w.w_co, D, Dq, &w.t_co));
+    }
   }
   TRY(tile_into(m, st, m->w_head, m->V, D, &m->t_head));
   return retile_hsm(m, st, true);
@@ -907,6 +1021,7 @@ static adept_status run_pass(adept_model* m, int n_tok, int batch, int prompt_le
   // encoder "stop entirely" (Sec. 4.3, downstream tasks): exits are recorded in tok_exit
   // (the attention leaves out keys of tokens gone before its layer) and get no fills
   const bool stop = fam == ADEPT_FAMILY_BERT && m->stop_entirely && !decode;
+  const bool cross = c.max_src > 0;   // encoder-decoder decoder: a cross-attention sublayer per layer
   // generation steps of bf16 decoders: the producers of the final states (the last layer's
   // row scatter, the HSM's output step) also write them standardised for the head, so the
   // head GEMM streams its weights against ready bf16 rows
@@ -973,7 +1088,7 @@ static adept_status run_pass(adept_model* m, int n_tok, int batch, int prompt_le
       prof_begin(m, ADEPT_PROF_ATTENTION, st, &b);
       launch_attention(st, m->dt, m->q, Dq, m->att, Dq, act, mr, rt, m->tok_seq, m->tok_pos, m->d_seq_len, cv, l0,
                        m->H, causal, decode_keys, m->attn_ws, m->attn_ctr, m->err_word, stop ? m->tok_exit : nullptr,
-                       prompt_len);
+                       prompt_len, m->use_attn_tc ? m->T_max : 0, N);
       prof_end(m, ADEPT_PROF_ATTENTION, st, b, 0, 0);
       m->launches += 1;
     }
@@ -995,6 +1110,40 @@ static adept_status run_pass(adept_model* m, int n_tok, int batch, int prompt_le
     if (fam == ADEPT_FAMILY_BERT) {
       launch_layernorm_inplace(st, m->X_out, act, mr, D, w.ln1_g, w.ln1_b, eps);
       m->launches += 1;
+    }
+    if (cross) {
+      // cross-attention sublayer (encoder-decoder decoders, Sec. 5.2): Q of LN_c(X_out) (gain
+      // and shift folded into W_Qc), attention over all source positions of the token's
+      // sequence (the source cache, not causal), W_Oc + residual into X_out
+      GemmProblem pc;
+      memset(&pc, 0, sizeof pc);
+      pc.a_rows = n_tok;
+      pc.A = m->xn; pc.lda = D; pc.B = w.w_cq; pc.ldb = D; pc.rows = act; pc.N = Dq; pc.K = D;
+      pc.Bt = w.t_cq; pc.bt_nkb = cdiv(D, TW_KB);
+      pc.epi = epi_base(); pc.epi.kind = EPI_ACT; pc.epi.act = ACT_NONE; pc.epi.bias = w.b_cq;
+      pc.epi.out_t = m->q; pc.epi.ld_t = Dq;
+      gemm_std(m, st, pc, mr, m->X_out, D, nullptr, amode, eps, m->gemm_cls, nullptr,
+               ts_valid ? m->tile_stats : nullptr);
+      {
+        cudaEvent_t b = nullptr;
+        prof_begin(m, ADEPT_PROF_ATTENTION, st, &b);
+        launch_attention(st, m->dt, m->q, Dq, m->att, Dq, act, mr, rt, m->tok_seq, m->tok_pos, m->d_src_len,
+                         cross_view(m), l0, m->H, 0, decode ? m->cs_blocks_per_seq * c.kv_block_tokens : 0,
+                         m->attn_ws, m->attn_ctr, m->err_word, nullptr, 0, m->use_attn_tc ? m->T_max : 0, N);
+        prof_end(m, ADEPT_PROF_ATTENTION, st, b, 0, 0);
+        m->launches += 1;
+      }
+      pc.A = m->att; pc.lda = Dq; pc.B = w.w_co; pc.ldb = Dq; pc.N = D; pc.K = Dq;
+      pc.Bt = w.t_co; pc.bt_nkb = cdiv(Dq, TW_KB);
+      pc.epi = epi_base(); pc.epi.kind = EPI_RESID; pc.epi.bias = w.b_co; pc.epi.out_f32 = m->X_out;
+      pc.epi.ld_f32 = D; pc.epi.resid = m->X_out; pc.epi.ld_resid = D;
+      ts_valid = false;   // the statistics of the FFN input now come from this product
+      if (dgrows) {
+        pc.epi.tile_stats = m->tile_stats;
+        ts_valid = dg_takes(m, 1, pc, mr, nullptr);
+        if (!ts_valid) pc.epi.tile_stats = nullptr;
+      }
+      gemm(m, st, &pc, 1, &mr, m->gemm_cls);
     }
     // FFN (input standardised)
     p.A = m->xn; p.lda = D; p.B = w.w_up; p.ldb = D; p.N = w.up_rows; p.K = D;
@@ -1535,6 +1684,14 @@ void adept_free(adept_model* m) {
   delete m;
 }
 
+static adept_status check_cross_set(adept_model* m, int batch) {
+  if (m->cfg.max_src <= 0) return ADEPT_OK;
+  for (int b = 0; b < batch; ++b)
+    if (m->h_src_len[b] <= 0)
+      return fail(m, ADEPT_ERR_INVALID_ARG, "sequence %d has no cross-attention source (adept_set_cross_source)", b);
+  return ADEPT_OK;
+}
+
 adept_status adept_prefill(adept_model* m, int batch, int prompt_len, const int32_t* d_tokens, float delta,
                            const int32_t* d_forced_exit, int32_t* d_exit_layer_out, float* d_logits_out,
                            int32_t* d_next_token_out, float* d_sim_out, void* stream) {
@@ -1549,6 +1706,7 @@ adept_status adept_prefill(adept_model* m, int batch, int prompt_len, const int3
   if ((long long)batch * prompt_len > m->T_max)
     return fail(m, ADEPT_ERR_CAPACITY, "batch * prompt_len %d above the pass workspace (%d rows)", batch * prompt_len,
                 m->T_max);
+  TRY(check_cross_set(m, batch));
   cudaStream_t st = (cudaStream_t)stream;
   std::vector<int> lens(batch, prompt_len);
   TRY(reserve_seqs(m, batch, lens.data(), st));
@@ -1557,6 +1715,55 @@ adept_status adept_prefill(adept_model* m, int batch, int prompt_len, const int3
   TRY(run_pass(m, batch * prompt_len, batch, prompt_len, false, d_tokens, d_forced_exit, d_exit_layer_out, d_sim_out,
                st));
   TRY(run_head(m, batch, prompt_len, false, d_logits_out, d_next_token_out, st));
+  span_collect(m, st);
+  return check_launch(m);
+}
+
+adept_status adept_set_cross_source(adept_model* m, int n_seq, const int32_t* h_src_len, const float* d_states,
+                                    void* stream) {
+  if (!m) return ADEPT_ERR_INVALID_ARG;
+  const adept_config& c = m->cfg;
+  if (c.max_src <= 0) return fail(m, ADEPT_ERR_INVALID_ARG, "the model has no cross-attention (max_src = 0)");
+  if (!h_src_len || !d_states) return fail(m, ADEPT_ERR_INVALID_ARG, "NULL source lengths or states");
+  if (n_seq < 1 || n_seq > c.max_batch) return fail(m, ADEPT_ERR_INVALID_ARG, "n_seq %d out of range", n_seq);
+  std::vector<int> seq, pos;
+  for (int b = 0; b < n_seq; ++b) {
+    if (h_src_len[b] < 1 || h_src_len[b] > c.max_src)
+      return fail(m, ADEPT_ERR_INVALID_ARG, "source length %d of sequence %d outside [1, %d]", h_src_len[b], b, c.max_src);
+    for (int p = 0; p < h_src_len[b]; ++p) {
+      seq.push_back(b);
+      pos.push_back(p);
+    }
+  }
+  PdlScope pdl(!m->profile);
+  cudaStream_t st = (cudaStream_t)stream;
+  const int n = (int)seq.size(), D = m->D;
+  CUDA_TRY(m, cudaMemcpyAsync(m->cs_seq, seq.data(), n * sizeof(int), cudaMemcpyHostToDevice, st));
+  CUDA_TRY(m, cudaMemcpyAsync(m->cs_pos, pos.data(), n * sizeof(int), cudaMemcpyHostToDevice, st));
+  // the states in the GEMM input type, then every layer's source K/V in one grouped launch
+  launch_standardize(st, m->dt, d_states, D, nullptr, DevRange{nullptr, nullptr, n}, n, D, NORM_COPY, 0.f, m->cs_x, D);
+  m->launches += 1;
+  std::vector<GemmProblem> probs(m->N);
+  std::vector<int> mrs(m->N, n);
+  const KVCacheView cv = cross_view(m);
+  for (int l = 0; l < m->N; ++l) {
+    GemmProblem& p = probs[l];
+    memset(&p, 0, sizeof p);
+    p.A = m->cs_x; p.lda = D; p.a_rows = n;
+    p.B = m->L[l].w_ckv; p.ldb = D; p.N = 2 * m->Dkv; p.K = D;
+    p.rows = DevRange{nullptr, nullptr, n};
+    p.epi = epi_base();
+    p.epi.kind = EPI_KV; p.epi.bias = m->L[l].b_ckv;
+    p.epi.row_tok = m->cs_iota; p.epi.tok_seq = m->cs_seq; p.epi.tok_pos = m->cs_pos;
+    p.epi.cache = cv; p.epi.layer0 = l;
+    p.epi.n_q_cols = 0; p.epi.n_kv_cols = m->Dkv; p.epi.head_dim = m->dh;
+  }
+  gemm(m, st, probs.data(), m->N, mrs.data(), ADEPT_PROF_GEMM_PREFILL);
+  // the lengths last: a copy on the stream starts after the projection has completed, so no
+  // later kernel's early (pre-dependency-wait) reads of the source cache can overlap it
+  for (int b = 0; b < n_seq; ++b) m->h_src_len[b] = h_src_len[b];
+  CUDA_TRY(m, cudaMemcpyAsync(m->d_src_len, m->h_src_len.data(), n_seq * sizeof(int), cudaMemcpyHostToDevice, st));
+  CUDA_TRY(m, cudaStreamSynchronize(st));   // the host vectors above are released on return
   return check_launch(m);
 }
 
@@ -1569,6 +1776,7 @@ adept_status adept_decode_step(adept_model* m, int batch, const int32_t* d_token
   if (!d_tokens) return fail(m, ADEPT_ERR_INVALID_ARG, "d_tokens is NULL");
   if (batch < 1 || batch > m->cfg.max_batch) return fail(m, ADEPT_ERR_CAPACITY, "batch %d out of range", batch);
   if (std::isnan(delta)) return fail(m, ADEPT_ERR_INVALID_ARG, "delta is NaN");
+  TRY(check_cross_set(m, batch));
   for (int b = 0; b < batch; ++b) {
     if (m->seq_blocks[b].empty()) return fail(m, ADEPT_ERR_INVALID_ARG, "sequence %d has no prompt", b);
     if (m->h_seq_len[b] >= m->max_blocks_per_seq * m->cfg.kv_block_tokens || m->h_seq_len[b] >= m->cfg.max_seq)
@@ -1580,7 +1788,9 @@ adept_status adept_decode_step(adept_model* m, int batch, const int32_t* d_token
   m->launches += 1;
   auto body = [&](cudaStream_t s) -> adept_status {
     TRY(run_pass(m, batch, batch, 1, true, m->dec_tok, m->dec_forced, m->dec_exit, m->dec_sim, s));
-    return run_head(m, batch, 1, true, m->logits_ws, m->dec_next, s);
+    TRY(run_head(m, batch, 1, true, m->logits_ws, m->dec_next, s));
+    span_collect(m, s);
+    return ADEPT_OK;
   };
   const bool graph_ok = m->use_graph && !m->profile;
   if (graph_ok && m->dec_warm[batch] >= 1) {
@@ -1687,9 +1897,9 @@ adept_status adept_skip_kv_fill(adept_model* m, int n_tokens, const void* d_h_ma
     }
     m->fill_cap = cap;
   }
-  launch_fill_sort(st, m->dt, d_h_mapped, n_tokens, m->D, d_exit_layer, m->N, m->fill_hist, m->fill_start,
-                   m->fill_cursor, m->fill_tok, m->fill_x, attn_norm_mode(m), m->cfg.norm_eps, m->err_word);
-  m->launches += 4;
+  m->launches += launch_fill_sort(st, m->dt, d_h_mapped, n_tokens, m->D, d_exit_layer, m->N, m->fill_hist,
+                                  m->fill_start, m->fill_cursor, m->fill_tok, m->fill_x, attn_norm_mode(m),
+                                  m->cfg.norm_eps, m->err_word);
   std::vector<GemmProblem> probs;
   std::vector<int> mrs;
   for (int r = 2; r <= m->N; ++r) {
@@ -1707,6 +1917,7 @@ adept_status adept_skip_kv_fill(adept_model* m, int n_tokens, const void* d_h_ma
     if (done) m->launches += 1;
   }
   if (!done) gemm(m, st, probs.data(), (int)probs.size(), mrs.data(), ADEPT_PROF_KV_FILL);
+  span_collect(m, st);
   return check_launch(m);
 }
 
@@ -1772,11 +1983,23 @@ adept_status adept_set_option(adept_model* m, int option, int value) {
   switch (option) {
     case ADEPT_OPT_HSM_IDENTITY: m->hsm_identity = value != 0; drop_graphs(m); return ADEPT_OK;
     case ADEPT_OPT_PROFILE: m->profile = value != 0; return ADEPT_OK;
+    case ADEPT_OPT_SPAN_TIMER:
+      if (value && !m->span_sites) {
+        TRY(dalloc_t(m, &m->span_sites, SPAN_SITES));
+        TRY(dalloc_t(m, &m->span_tot, ADEPT_PROF_NCLASS));
+        const std::vector<SpanSite> idle(SPAN_SITES, SpanSite{~0ull, 0ull, 0, 0});
+        CUDA_TRY(m, cudaMemcpy(m->span_sites, idle.data(), SPAN_SITES * sizeof(SpanSite), cudaMemcpyHostToDevice));
+        CUDA_TRY(m, cudaMemset(m->span_tot, 0, ADEPT_PROF_NCLASS * sizeof(SpanTotal)));
+      }
+      m->span_on = value != 0;
+      drop_graphs(m);   // captured steps carry their launches' span sites
+      return ADEPT_OK;
     case ADEPT_OPT_GEMM_SIMT: m->force_simt = value != 0; drop_graphs(m); return ADEPT_OK;
     case ADEPT_OPT_DECODE_GRAPH: m->use_graph = value != 0; drop_graphs(m); return ADEPT_OK;
     case ADEPT_OPT_DECODE_GEMM: m->use_dg = value != 0; drop_graphs(m); return ADEPT_OK;
     case ADEPT_OPT_DECODE_STREAM: m->use_stream = value != 0; drop_graphs(m); return ADEPT_OK;
     case ADEPT_OPT_DECODE_TILED: m->use_tiled = value != 0; drop_graphs(m); return ADEPT_OK;
+    case ADEPT_OPT_ATTN_TC: m->use_attn_tc = value != 0; return ADEPT_OK;
     case ADEPT_OPT_EXIT_METRIC:
       if (value < EXIT_GLOBAL || value > EXIT_BOTH) return fail(m, ADEPT_ERR_INVALID_ARG, "exit metric %d", value);
       m->exit_metric = value;
@@ -1791,6 +2014,20 @@ adept_status adept_set_option(adept_model* m, int option, int value) {
       return ADEPT_OK;
   }
   return fail(m, ADEPT_ERR_INVALID_ARG, "unknown option %d", option);
+}
+
+adept_status adept_span_read(adept_model* m, int cls, int64_t* launches, double* total_ms) {
+  if (!m || cls < 0 || cls >= ADEPT_PROF_NCLASS) return ADEPT_ERR_INVALID_ARG;
+  if (launches) *launches = 0;
+  if (total_ms) *total_ms = 0;
+  if (!m->span_tot) return ADEPT_OK;
+  CUDA_TRY(m, cudaDeviceSynchronize());
+  SpanTotal t{};
+  CUDA_TRY(m, cudaMemcpy(&t, m->span_tot + cls, sizeof t, cudaMemcpyDeviceToHost));
+  CUDA_TRY(m, cudaMemset(m->span_tot + cls, 0, sizeof t));
+  if (launches) *launches = (int64_t)t.n;
+  if (total_ms) *total_ms = (double)t.ns * 1e-6;
+  return ADEPT_OK;
 }
 
 adept_status adept_profile_read(adept_model* m, int cls, int64_t* launches, double* total_ms, double* flops,

@@ -38,6 +38,7 @@ class Pair:
         self.om = O.OracleModel(cfg, self.W)
         self.gm = adept.Model(cfg, self.W)
         self.tol = TOL[cfg.dtype]
+        self.cross = None   # encoder-decoder decoders: the oracle's O.CrossSource
 
     def close(self):
         self.gm.close()
@@ -85,7 +86,7 @@ def run_prefill(pair: Pair, tokens: np.ndarray, delta: float, forced=None, hsm_i
     B, P = tokens.shape
     cache = O.OracleCache(cfg, cfg.max_batch, cfg.max_seq)
     ores = O.prefill(pair.om, cache, tokens, delta, forced, hsm_mode="identity" if hsm_identity else "hsm",
-                     metric=metric, all_at_once=all_at_once, stop_entirely=stop_entirely)
+                     metric=metric, all_at_once=all_at_once, stop_entirely=stop_entirely, cross=pair.cross)
     if cfg.family == synth.BERT:
         adept.adept_set_option(pair.gm.h, adept.OPT_STOP_ENTIRELY, int(stop_entirely))
     adept.adept_set_option(pair.gm.h, adept.OPT_EXIT_METRIC, {"global": 0, "local": 1, "both": 2}[metric])
@@ -175,7 +176,8 @@ def compare_decode(pair: Pair, cache: O.OracleCache, first_tokens, steps: int, d
     tok = np.asarray(first_tokens)
     for s in range(steps):
         f = None if forced_steps is None else np.asarray(forced_steps[s])
-        o = O.decode_step(pair.om, cache, tok, delta, f, hsm_mode="identity" if hsm_identity else "hsm", metric=metric)
+        o = O.decode_step(pair.om, cache, tok, delta, f, hsm_mode="identity" if hsm_identity else "hsm", metric=metric,
+                          cross=pair.cross)
         use_forced = f
         if f is None and band_tokens(o.sim, delta).any():
             use_forced = o.exit_layer

@@ -139,3 +139,47 @@ def test_stream_gemm_small_fills_match_oracle():
                 checked += len(rows)
         assert checked >= n - int(np.sum(el == cfg.n_layers))
     pair.close()
+
+
+def test_span_timer_sums_within_the_step_and_changes_nothing():
+    """With the span timer on, the weight-streaming launches of generation steps record their
+    in-situ spans: every step records the same launches, the summed spans stay within the steps'
+    elapsed time, and the results equal those of the same steps without the timer bit for bit."""
+    cfg = _cfg(2)
+    W = synth.make_weights(cfg, seed=50, device="cuda")
+    B, P = cfg.max_batch, 40
+    res = []
+    for timer in (0, 1):
+        m = adept.Model(cfg, W)
+        adept.adept_set_option(m.h, adept.OPT_SPAN_TIMER, timer)
+        tokens = synth.make_tokens(50, B, P, cfg.vocab).cuda()
+        forced = synth.forced_exits_uniform(50, B * P, 2, cfg.n_layers).view(B, P).cuda()
+        m.prefill(tokens, 0.9, forced)
+        adept.adept_span_read(m.h, adept.PROF_GEMM_DECODE)
+        adept.adept_span_read(m.h, adept.PROF_KV_FILL)
+        ts = synth.make_tokens(51, 5, B, cfg.vocab).cuda()
+        fs = torch.full((B,), 3, dtype=torch.int32, device="cuda")
+        out, counts = [], []
+        for s in range(5):   # direct launches first, then graph replays
+            torch.cuda.synchronize()
+            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            e0.record()
+            ex, lg, nx, _ = m.decode_step(ts[s].contiguous(), 0.9, fs)
+            e1.record()
+            torch.cuda.synchronize()
+            n_g, ms_g = adept.adept_span_read(m.h, adept.PROF_GEMM_DECODE)
+            n_f, ms_f = adept.adept_span_read(m.h, adept.PROF_KV_FILL)
+            counts.append((n_g, n_f))
+            if timer:
+                assert n_g > 0 and n_f == 1
+                assert 0 < ms_g + ms_f <= e0.elapsed_time(e1), (ms_g, ms_f, e0.elapsed_time(e1))
+            else:
+                assert n_g == 0 and n_f == 0
+            out.append((ex.cpu().numpy(), lg.cpu().numpy(), m.final_states(B).cpu().numpy()))
+        m.check()
+        assert len(set(counts)) == 1, counts
+        res.append(out)
+        m.close()
+    for a, b in zip(res[0], res[1]):
+        for x, y in zip(a, b):
+            assert np.array_equal(x, y)

@@ -60,7 +60,7 @@ def test_noalloc_fill_matches_allocating_fill_and_oracle_on_two_calls(sizes):
         adept.adept_skip_kv_fill(ref.h, n, hd, el, seq, pos)
         adept.adept_launch_count(new.h)
         adept.adept_skip_kv_fill_noalloc(new.h, n, hd, el, seq, pos)
-        assert adept.adept_launch_count(new.h) >= 5     # the bucket sort (4) and at least one GEMM
+        assert adept.adept_launch_count(new.h) >= 2     # the bucket sort (1 or 2) and at least one GEMM
         ref.check()
         new.check()
         want = O.skip_kv_fill(om, h.double().numpy(), el_h, pos_h)
