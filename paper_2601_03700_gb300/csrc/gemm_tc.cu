@@ -577,6 +577,14 @@ static int pick_bn(const GemmProblem* probs, int n_probs, const int* max_rows, l
       pick = k;
       break;
     }
+  // wave quantisation: the next narrower width (down to 128) when its whole waves of tiles take
+  // at least 10 % less work per SM (e.g. 512 tiles of 256 are 4 waves of 256 columns on 152 SMs,
+  // 1024 tiles of 128 are 7 waves of 128)
+  if (pick < 3 && bns[pick + 1] >= 128) {
+    const long long w0 = (tiles[pick] + g_num_sms - 1) / g_num_sms * bns[pick];
+    const long long w1 = (tiles[pick + 1] + g_num_sms - 1) / g_num_sms * bns[pick + 1];
+    if (w1 * 10 <= w0 * 9) ++pick;
+  }
   *tiles_out = tiles[pick];
   return bns[pick];
 }

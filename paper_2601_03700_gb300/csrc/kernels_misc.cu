@@ -1207,8 +1207,73 @@ __global__ void head_rows_kernel(int batch, int prompt_len, int last, int* rows)
 // (generation steps, small fills) also place and standardise the rows here, one warp per row,
 // so that the whole pre-pass is this one launch.
 constexpr int FILL_PLAN_ROWS = 32;
+// One row standardised (the attention-input normalisation of the family) by one warp.
 template <typename T>
-__global__ void __launch_bounds__(1024) fill_plan_kernel(const T* h, int D, const int* exit_layer, int n, int n_layers,
+__device__ __forceinline__ void plan_row(const T* x, T* o, int D, int mode, float eps, int lane) {
+  constexpr int E = 16 / sizeof(T);   // elements per 16-byte piece
+  const int nch = D / (32 * E);       // pieces per lane
+  if (D % (32 * E) == 0 && nch <= 16 && (((uintptr_t)x | (uintptr_t)o) & 15) == 0) {
+    // the row in registers, every load issued before the first reduction (one memory round
+    // trip instead of one per strided loop iteration)
+    uint4 r[16];
+#pragma unroll
+    for (int i = 0; i < 16; ++i)
+      if (i < nch) r[i] = reinterpret_cast<const uint4*>(x)[lane + 32 * i];
+    auto val = [&](int i, int e) { return to_f(reinterpret_cast<const T*>(&r[i])[e]); };
+    float mu = 0.f, s2 = 0.f;
+    if (mode == NORM_LN) {
+#pragma unroll
+      for (int i = 0; i < 16; ++i)
+        if (i < nch)
+#pragma unroll
+          for (int e = 0; e < E; ++e) mu += val(i, e);
+      mu = warp_sum(mu) / D;
+    }
+    float rstd = 1.f;
+    if (mode != NORM_COPY) {
+#pragma unroll
+      for (int i = 0; i < 16; ++i)
+        if (i < nch)
+#pragma unroll
+          for (int e = 0; e < E; ++e) {
+            const float c = val(i, e) - mu;
+            s2 += c * c;
+          }
+      rstd = rsqrtf(warp_sum(s2) / D + eps);
+    }
+#pragma unroll
+    for (int i = 0; i < 16; ++i)
+      if (i < nch) {
+        uint4 w;
+        T* wt = reinterpret_cast<T*>(&w);
+#pragma unroll
+        for (int e = 0; e < E; ++e) wt[e] = mode == NORM_COPY ? reinterpret_cast<const T*>(&r[i])[e]
+                                                             : from_f<T>((val(i, e) - mu) * rstd);
+        reinterpret_cast<uint4*>(o)[lane + 32 * i] = w;
+      }
+    return;
+  }
+  if (mode == NORM_COPY) {
+    for (int d = lane; d < D; d += 32) o[d] = x[d];
+    return;
+  }
+  float mu = 0.f;
+  if (mode == NORM_LN) {
+    float sm = 0.f;
+    for (int d = lane; d < D; d += 32) sm += to_f(x[d]);
+    mu = warp_sum(sm) / D;
+  }
+  float s2 = 0.f;
+  for (int d = lane; d < D; d += 32) {
+    const float c = to_f(x[d]) - mu;
+    s2 += c * c;
+  }
+  const float rstd = rsqrtf(warp_sum(s2) / D + eps);
+  for (int d = lane; d < D; d += 32) o[d] = from_f<T>((to_f(x[d]) - mu) * rstd);
+}
+
+template <typename T>
+__global__ void __launch_bounds__(512) fill_plan_kernel(const T* h, int D, const int* exit_layer, int n, int n_layers,
                                                          int* hist, int* start, int* cursor, int* sorted_tok, T* xs,
                                                          int mode, float eps, unsigned* err) {
   PDL_ENTRY();
@@ -1249,26 +1314,8 @@ __global__ void __launch_bounds__(1024) fill_plan_kernel(const T* h, int D, cons
     sorted_tok[slot] = threadIdx.x;
   }
   __syncthreads();
-  if (warp >= n) return;
-  const T* x = h + (size_t)warp * D;
-  T* o = xs + (size_t)s_slot[warp] * D;
-  if (mode == NORM_COPY) {
-    for (int d = lane; d < D; d += 32) o[d] = x[d];
-    return;
-  }
-  float mu = 0.f;
-  if (mode == NORM_LN) {
-    float sm = 0.f;
-    for (int d = lane; d < D; d += 32) sm += to_f(x[d]);
-    mu = warp_sum(sm) / D;
-  }
-  float s2 = 0.f;
-  for (int d = lane; d < D; d += 32) {
-    const float c = to_f(x[d]) - mu;
-    s2 += c * c;
-  }
-  const float rstd = rsqrtf(warp_sum(s2) / D + eps);
-  for (int d = lane; d < D; d += 32) o[d] = from_f<T>((to_f(x[d]) - mu) * rstd);
+  for (int row = warp; row < n; row += blockDim.x >> 5)
+    plan_row(h + (size_t)row * D, xs + (size_t)s_slot[row] * D, D, mode, eps, lane);
 }
 
 template <typename T>
@@ -1644,10 +1691,10 @@ int launch_fill_sort(cudaStream_t st, int dt, const void* h, int n, int D, const
                      unsigned* err) {
   const size_t smem = (size_t)2 * (n_layers + 2) * sizeof(int);
   if (dt == 1)
-    launch_k(fill_plan_kernel<bf16>, 1, 1024, smem, st, (const bf16*)h, D, exit_layer, n, n_layers, hist, start, cursor,
+    launch_k(fill_plan_kernel<bf16>, 1, 512, smem, st, (const bf16*)h, D, exit_layer, n, n_layers, hist, start, cursor,
              sorted_tok, (bf16*)xs, mode, eps, err);
   else
-    launch_k(fill_plan_kernel<float>, 1, 1024, smem, st, (const float*)h, D, exit_layer, n, n_layers, hist, start,
+    launch_k(fill_plan_kernel<float>, 1, 512, smem, st, (const float*)h, D, exit_layer, n, n_layers, hist, start,
              cursor, sorted_tok, (float*)xs, mode, eps, err);
   if (n <= FILL_PLAN_ROWS) return 1;   // placed and standardised by the plan kernel
   if (dt == 1)
