@@ -40,10 +40,12 @@ import torch  # noqa: E402
 import synth  # noqa: E402
 
 PEAKS_FALLBACK = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
-# DRAM bytes (read + write) per launch of a kernel class from one ncu capture at the
-# workload's shapes, scaled to a launch of the workload (profiles/); None until a capture of
-# the current kernel exists.
-NCU_TRAFFIC_PER_LAUNCH = {}
+# DRAM bytes (read + write) over algorithmic bytes of a kernel class, from one ncu capture of
+# the current kernel at the workload's layer shapes (profiles/gemm_stream_llama_layer_shapes.md:
+# the QKV and gate/up launches of a generation step, 104.39 + 183.87 MB of DRAM traffic for
+# 100.69 + 180.39 MB of weights, rows and outputs); the line's traffic is this ratio times the
+# class's algorithmic bytes per launch (traffic grows with the weight bytes streamed).
+NCU_TRAFFIC_RATIO = {"gemm_decode": (104.39 + 183.87) / (100.69 + 180.39)}
 METRIC = "early-exit prefill+decode tokens/s at 1 GB300; skipped-layer KV-fill % of roofline"
 # Llama-7B headline workload: one prompt of LP tokens, LSTEPS greedy steps, exits ~ N(24, 4) on [8, 32]
 LP, LSTEPS, LMEAN, LSD, LLO, LHI = 2048, 256, 24.0, 4.0, 8, 32
@@ -770,8 +772,9 @@ def ours(args, rank, world, device):
     else:
         roof = {"bound": "hbm", "achieved": round(by / (ms / 1e3) / 1e9, 2), "peak": peaks["hbm_gbs"], "unit": "GB/s"}
     roof["frac"] = round(roof["achieved"] / roof["peak"], 4)
-    tr = NCU_TRAFFIC_PER_LAUNCH.get(dom)
-    roof["traffic"] = round(tr) if tr else None
+    tr = NCU_TRAFFIC_RATIO.get(dom)
+    roof["traffic"] = round(tr * by / max(n, 1)) if tr else None
+    roof["traffic_source"] = "ncu DRAM bytes / algorithmic bytes of the captured launches x algorithmic bytes per launch"
     roof["kernel"] = dom + " (stream-K and cluster K-split weight-streaming GEMM launches)"
     roof["launches"] = n
     roof["peak_source"] = (peaks_src + " (MEASURED_PEAKS.json)") if peaks_src == "measured" else peaks_src
