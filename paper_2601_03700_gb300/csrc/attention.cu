@@ -469,7 +469,8 @@ static void attn_dispatch(cudaStream_t st, const void* q, int ld_q, void* out, i
 // then clears its counter for the next launch.
 // ---------------------------------------------------------------------------
 constexpr int AD_CHUNK = 128;
-constexpr int AD_THREADS = 128;
+constexpr int AD_THREADS = 256;
+constexpr int AD_WARPS = AD_THREADS / 32;
 constexpr long long AD_TIMEOUT_CYCLES = 4000000000LL;   // ~2 s at 2 GHz
 
 __device__ __forceinline__ uint32_t ad_smem_u32(const void* p) { return (uint32_t)__cvta_generic_to_shared(p); }
@@ -525,7 +526,7 @@ __global__ void __launch_bounds__(AD_THREADS)
   KT_BEGIN();
   constexpr int PARTS = DH / 8;                    // 16-byte pieces of a K / V row
   constexpr int KPI = 32 / PARTS;                  // keys per warp instruction
-  constexpr int KIT = AD_CHUNK / (4 * KPI);        // key groups per warp
+  constexpr int KIT = AD_CHUNK / (AD_WARPS * KPI); // key groups per warp
   extern __shared__ __align__(128) uint8_t ad_smem[];
   bf16* sK = reinterpret_cast<bf16*>(ad_smem);   // [AD_CHUNK][DH]
   bf16* sV = sK + AD_CHUNK * DH;                  // [AD_CHUNK][DH]
@@ -665,7 +666,7 @@ __global__ void __launch_bounds__(AD_THREADS)
       uint4 kr[KIT];
 #pragma unroll
       for (int it = 0; it < KIT; ++it)
-        kr[it] = *reinterpret_cast<const uint4*>(sK + (warp * KPI + it * 4 * KPI + slot) * DH + part * 8);
+        kr[it] = *reinterpret_cast<const uint4*>(sK + (warp * KPI + it * AD_WARPS * KPI + slot) * DH + part * 8);
       float d[KIT];
 #pragma unroll
       for (int it = 0; it < KIT; ++it) {
@@ -686,7 +687,7 @@ __global__ void __launch_bounds__(AD_THREADS)
       if (part == 0) {
 #pragma unroll
         for (int it = 0; it < KIT; ++it) {
-          const int key = warp * KPI + it * 4 * KPI + slot;
+          const int key = warp * KPI + it * AD_WARPS * KPI + slot;
           s_p[key] = key < nkc ? d[it] : -INFINITY;
         }
       }
@@ -700,7 +701,9 @@ __global__ void __launch_bounds__(AD_THREADS)
     mx = warp_max(mx);
     if (lane == 0) s_red[warp] = mx;
     __syncthreads();
-    const float M = fmaxf(fmaxf(s_red[0], s_red[1]), fmaxf(s_red[2], s_red[3]));
+    float M = s_red[0];
+#pragma unroll
+    for (int w = 1; w < AD_WARPS; ++w) M = fmaxf(M, s_red[w]);
     float ls = 0.f;
 #pragma unroll
     for (int k = tid; k < AD_CHUNK; k += AD_THREADS) {
@@ -721,7 +724,7 @@ __global__ void __launch_bounds__(AD_THREADS)
       float pr[KIT];
 #pragma unroll
       for (int it = 0; it < KIT; ++it) {
-        const int key = warp * KPI + it * 4 * KPI + slot;
+        const int key = warp * KPI + it * AD_WARPS * KPI + slot;
         vr[it] = *reinterpret_cast<const uint4*>(sV + key * DH + part * 8);
         pr[it] = s_p[key];
       }
@@ -757,11 +760,15 @@ __global__ void __launch_bounds__(AD_THREADS)
 #pragma unroll
         for (int c = 0; c < 4; ++c) {
           const int d = q4 * 4 + c;
-          vv[c] = nkc == 0 ? (d == DH ? -INFINITY : 0.f)
-                           : d < DH ? s_o[0][d] + s_o[1][d] + s_o[2][d] + s_o[3][d]
-                           : d == DH ? M
-                           : d == DH + 1 ? s_red[0] + s_red[1] + s_red[2] + s_red[3]
-                                         : 0.f;
+          float sum = 0.f;
+          if (d < DH) {
+#pragma unroll
+            for (int w = 0; w < AD_WARPS; ++w) sum += s_o[w][d];
+          } else if (d == DH + 1) {
+#pragma unroll
+            for (int w = 0; w < AD_WARPS; ++w) sum += s_red[w];
+          }
+          vv[c] = nkc == 0 ? (d == DH ? -INFINITY : 0.f) : d == DH ? M : sum;
         }
         if (split == 0) {
           *reinterpret_cast<float4*>(slot + q4 * 4) = v;
@@ -780,10 +787,18 @@ __global__ void __launch_bounds__(AD_THREADS)
     }
     // chunk partial -> workspace [(row, head), split]: o[DH], m, l
     float* w = ws + ((size_t)rh * n_split + split) * (DH + 2);
-    for (int d = tid; d < DH; d += AD_THREADS) w[d] = s_o[0][d] + s_o[1][d] + s_o[2][d] + s_o[3][d];
+    for (int d = tid; d < DH; d += AD_THREADS) {
+      float sum = 0.f;
+#pragma unroll
+      for (int w2 = 0; w2 < AD_WARPS; ++w2) sum += s_o[w2][d];
+      w[d] = sum;
+    }
     if (tid == 0) {
+      float sum = 0.f;
+#pragma unroll
+      for (int w2 = 0; w2 < AD_WARPS; ++w2) sum += s_red[w2];
       w[DH] = M;
-      w[DH + 1] = s_red[0] + s_red[1] + s_red[2] + s_red[3];
+      w[DH + 1] = sum;
     }
     __threadfence();
     __syncthreads();
