@@ -13,9 +13,12 @@
 //    16 KB slots, completing on the slot's full barrier; four consumer warps release a slot
 //    through its empty barrier (one arrival per warp), so a warp never waits for the other
 //    warps before the producer can refill.  Weights do not depend on the preceding kernel,
-//    so the first slots are issued before the programmatic-dependent-launch wait.  The CTA
-//    is sized (about 112 KB of shared memory) so that the next launch's CTA fits beside it
-//    on the SM and its first copies overlap this launch's tail.
+//    so the first slots are issued before the programmatic-dependent-launch wait.
+//  * One CTA per SM: the CTA takes just over half an SM's shared memory.  Consecutive
+//    launches overlap (their CTAs are placed wherever there is room), and two CTAs of this
+//    kernel on one SM would each stream at half rate while another SM idles, so the launch's
+//    equal shares would end at twice the time; a five-slot ring leaves room beside the CTA
+//    for one CTA of the neighbouring kernels (attention, cluster K-split GEMM).
 //  * A operand: after the wait the launch's token rows (all of K) are staged once in shared
 //    memory, copied (bf16) or standardised from the fp32 residual stream with row statistics
 //    computed here or handed over by the producer of the rows.
@@ -51,9 +54,9 @@ constexpr int DS_NE = 2;                          // epilogue warps
 constexpr int DS_WARPS = 1 + DS_NC + DS_NE;       // + the producer warp
 constexpr int DS_THREADS = 32 * DS_WARPS;
 constexpr int DS_MAX_STAGES = 12;
+constexpr int DS_RING_STAGES = 5;                 // ring depth (measured at the Llama-7B shapes: 3-7 tried)
 constexpr int DS_RP = DS_BN + 1;                  // floats per token row of a partial tile
 constexpr int DS_MAXG = 32;
-constexpr int DS_COHOST_SMEM = 113 * 1024;        // two launches' CTAs fit on one SM (228 KB, 1 KB each reserved)
 constexpr int DS_SMEM_LIMIT = 200 * 1024;
 constexpr long long DS_TIMEOUT_CYCLES = 4000000000LL;   // ~2 s at 2 GHz
 constexpr long long DS_MIN_STREAM_BYTES = 8ll << 20;    // below: the cluster K-split kernel
@@ -765,6 +768,7 @@ __global__ void __launch_bounds__(DS_THREADS, 2) gemm_stream_kernel(const __grid
 }
 
 int g_ds_sms = 0;
+int g_ds_sm_smem = 0;   // shared memory per SM (bytes)
 
 template <int MB, int KIND, int MAXG>
 cudaError_t ds_launch(cudaStream_t st, const DsParams<MAXG>& prm, int grid, size_t smem) {
@@ -824,6 +828,7 @@ bool ds_plan(const GemmProblem& q, int n_probs, int max_rows, const DgNorm* norm
     int dev = 0;
     cudaGetDevice(&dev);
     cudaDeviceGetAttribute(&g_ds_sms, cudaDevAttrMultiProcessorCount, dev);
+    cudaDeviceGetAttribute(&g_ds_sm_smem, cudaDevAttrMaxSharedMemoryPerMultiprocessor, dev);
     if (g_ds_sms <= 0) g_ds_sms = 1;
   }
   grid = g_ds_sms;
@@ -837,10 +842,8 @@ bool ds_plan(const GemmProblem& q, int n_probs, int max_rows, const DgNorm* norm
   const int p_bytes = 2 * 16 * DS_RP * 4;   // the two tile hand-off buffers
   const int fixed = 1024 + a_bytes + p_bytes;
   const int STATIC = 2 * DS_MAX_STAGES * 8 + 32 + 128 + DS_WARPS * 64 + 3 * MAXG * 4 + 16 + 128 + 24 + 64;
-  int stages = (DS_COHOST_SMEM - STATIC - fixed) / DS_STAGE;
-  if (stages < 4) stages = (DS_SMEM_LIMIT - STATIC - fixed) / DS_STAGE;
+  const int stages = std::min(DS_RING_STAGES, (DS_SMEM_LIMIT - STATIC - fixed) / DS_STAGE);
   if (stages < 2) return false;
-  stages = std::min(stages, DS_MAX_STAGES);
   memset(&prm, 0, sizeof prm);
   prm.n_probs = n_probs;
   prm.tiles = tiles;
@@ -873,6 +876,7 @@ bool ds_plan(const GemmProblem& q, int n_probs, int max_rows, const DgNorm* norm
   prm.err = err;
   prm.span = g_span;
   smem = (size_t)prm.off_p + p_bytes + 1024;
+  smem = std::max(smem, (size_t)g_ds_sm_smem / 2 + 1024);   // no second CTA of this kernel on the SM
   return smem <= (size_t)DS_SMEM_LIMIT;
 }
 
