@@ -56,7 +56,8 @@ constexpr int DS_THREADS = 32 * DS_WARPS;
 constexpr int DS_MAX_STAGES = 12;
 constexpr int DS_RING_STAGES = 5;                 // ring depth (measured at the Llama-7B shapes: 3-7 tried)
 constexpr int DS_RP = DS_BN + 1;                  // floats per token row of a partial tile
-constexpr int DS_MAXG = 32;
+constexpr int DS_MAXG = 32;                       // problems of a grouped launch (one warp's lanes)
+static_assert(DS_MAXG <= 32, "the row counts of a launch are read by one warp");
 constexpr int DS_SMEM_LIMIT = 200 * 1024;
 constexpr long long DS_TIMEOUT_CYCLES = 4000000000LL;   // ~2 s at 2 GHz
 constexpr long long DS_MIN_STREAM_BYTES = 8ll << 20;    // below: the cluster K-split kernel
@@ -489,19 +490,23 @@ __global__ void __launch_bounds__(DS_THREADS, 2) gemm_stream_kernel(const __grid
   // The row counts (device values) and the A operand are read in parallel: every problem's
   // rows start at row 0 (host-checked), so the launch's row bound max_m is staged without
   // waiting for the count (rows past it feed only token columns that are never stored).
-  if (tid == 0) {
-    int n = 0;
-    for (int q = 0; q < p.n_probs; ++q) {
-      int M = p.rows[q].e();
+  if (warp == 0) {
+    // lane q reads problem q's count (all loads at once; MAXG <= 32), the live problems are
+    // listed in problem order
+    const int q = lane;
+    int M = 0;
+    if (q < p.n_probs) {
+      M = p.rows[q].e();
       if (M > p.max_m) {   // more rows than the launch was sized for
         atomicOr(p.err, ERRW_CONFIG);
         M = p.max_m;
       }
       s_M[q] = M;
       s_rb[q] = 0;
-      if (M > 0) s_live[n++] = q;
     }
-    s_nlive = n;
+    const unsigned live = __ballot_sync(0xffffffffu, q < p.n_probs && M > 0);
+    if (q < p.n_probs && M > 0) s_live[__popc(live & ((1u << q) - 1u))] = q;
+    if (lane == 0) s_nlive = __popc(live);
   }
   ds_stage_a(p, sA, p.max_m, s_mu, s_rs, s_red);   // ends with a CTA barrier: the counts are visible
   KT_MARK(1);
