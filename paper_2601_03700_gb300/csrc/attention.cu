@@ -517,7 +517,13 @@ __device__ __forceinline__ bool ad_wait(uint64_t* bar, unsigned* err) {
 // copied after it.  The token's row among this layer's active rows is found after the wait;
 // a token that left at an earlier layer lets its copies land and leaves.  The copy barrier
 // takes two arrivals (before and after the wait), so it cannot complete between them.
-template <int DH, bool CL>
+//
+// SV (one query head per KV head): the first half of the chunk's V rows has its own slots and
+// the second half is copied into the K slots once the scores are formed, so a CTA holds 1.5
+// chunks of rows instead of 2 (48 KB at d_h = 128): four CTAs fit on an SM and the grid of a
+// 2-4 k-token context runs in one wave; the second half's copy overlaps the softmax and the
+// first half's sum.
+template <int DH, bool CL, bool SV>
 __global__ void __launch_bounds__(AD_THREADS)
     attn_decode_kernel(const bf16* __restrict__ q, int ld_q, DevRange rows, const int* row_tok, const int* tok_seq,
                        const int* tok_pos, const int* seq_len, KVCacheView cache, int layer0, int n_heads, int causal,
@@ -528,9 +534,11 @@ __global__ void __launch_bounds__(AD_THREADS)
   constexpr int KPI = 32 / PARTS;                  // keys per warp instruction
   constexpr int KIT = AD_CHUNK / (AD_WARPS * KPI); // key groups per warp
   extern __shared__ __align__(128) uint8_t ad_smem[];
-  bf16* sK = reinterpret_cast<bf16*>(ad_smem);   // [AD_CHUNK][DH]
-  bf16* sV = sK + AD_CHUNK * DH;                  // [AD_CHUNK][DH]
+  constexpr int HB = AD_CHUNK / 32;               // SV: cache blocks of the chunk's first half
+  bf16* sK = reinterpret_cast<bf16*>(ad_smem);   // [AD_CHUNK][DH]; SV: then V rows HB*16..
+  bf16* sV = sK + AD_CHUNK * DH;                  // [AD_CHUNK][DH]; SV: [AD_CHUNK / 2][DH]
   __shared__ __align__(8) uint64_t bar;
+  __shared__ __align__(8) uint64_t bar2;          // SV: the second half of V
   __shared__ float s_p[AD_CHUNK];
   __shared__ float s_red[AD_THREADS / 32];
   __shared__ float s_o[AD_THREADS / 32][DH];
@@ -547,17 +555,22 @@ __global__ void __launch_bounds__(AD_THREADS)
   const int sq = tok_seq[t], pos = tok_pos[t];
   const int nk = causal ? pos + 1 : seq_len[sq];
   const int n_eff = (nk + AD_CHUNK - 1) / AD_CHUNK;   // chunks holding keys of this token
+  if (SV && group != 1) {   // (uniform over the grid) the K slots would be needed again
+    if (tid == 0) atomicOr(err, ERRW_CONFIG);
+    return;
+  }
   if (!CL && split >= n_eff) return;   // (a cluster's CTAs all stay: they push empty partials)
   const int k_lo = split * AD_CHUNK, nkc = max(0, min(nk - k_lo, AD_CHUNK));
   const int nb = (nkc + 15) >> 4;                      // cache blocks of the chunk
   // blocks of the chunk below the block of the token's own position: written before this step
   const int n_pre = max(0, min(nb, (pos >> 4) - (k_lo >> 4)));
-  float* sPart = reinterpret_cast<float*>(ad_smem + 2 * AD_CHUNK * DH * 2);   // CL: [group][n_split][PW]
+  float* sPart = reinterpret_cast<float*>(ad_smem + (SV ? 3 * AD_CHUNK / 2 : 2 * AD_CHUNK) * DH * 2);   // CL: [group][n_split][PW]
   constexpr int BLOCK_BYTES = 16 * DH * 2;
   KT_MARK(0);
 
   if (tid == 0) {
     asm volatile("mbarrier.init.shared::cta.b64 [%0], 2;" ::"r"(ad_smem_u32(&bar)) : "memory");
+    if (SV) asm volatile("mbarrier.init.shared::cta.b64 [%0], 1;" ::"r"(ad_smem_u32(&bar2)) : "memory");
     if (CL) {
       asm volatile("mbarrier.init.shared::cta.b64 [%0], 1;" ::"r"(ad_smem_u32(&red_bar)) : "memory");
     }
@@ -568,8 +581,9 @@ __global__ void __launch_bounds__(AD_THREADS)
                    : "memory");
   }
   __syncthreads();
-  // copy of block lane of the chunk (lane < nb) into its K / V slots
-  auto copy_block = [&](int b) {
+  // copy of block b of the chunk (b < nb) into its K slots and (V: !SV or b < HB) its V slots;
+  // v_only (SV): block b >= HB's V rows into K slots (b - HB), completing on bar2
+  auto copy_block = [&](int b, bool v_only) {
     const int bi = (k_lo >> 4) + b;
     int blk = (sq >= 0 && sq < cache.max_batch && bi < cache.max_blocks_per_seq)
                   ? cache.block_table[sq * cache.max_blocks_per_seq + bi]
@@ -579,22 +593,34 @@ __global__ void __launch_bounds__(AD_THREADS)
       blk = 0;
     }
     const size_t off = (((size_t)layer0 * cache.n_blocks + blk) * Hkv + kvh) * (size_t)(16 * DH);
+    if (SV && v_only) {
+      asm volatile("cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(
+                       ad_smem_u32(sK + (b - HB) * 16 * DH)),
+                   "l"((const bf16*)cache.v + off), "r"((uint32_t)BLOCK_BYTES), "r"(ad_smem_u32(&bar2))
+                   : "memory");
+      return;
+    }
     asm volatile("cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(
                      ad_smem_u32(sK + b * 16 * DH)),
                  "l"((const bf16*)cache.k + off), "r"((uint32_t)BLOCK_BYTES), "r"(ad_smem_u32(&bar))
                  : "memory");
-    asm volatile("cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(
-                     ad_smem_u32(sV + b * 16 * DH)),
-                 "l"((const bf16*)cache.v + off), "r"((uint32_t)BLOCK_BYTES), "r"(ad_smem_u32(&bar))
-                 : "memory");
+    if (!SV || b < HB)
+      asm volatile("cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(
+                       ad_smem_u32(sV + b * 16 * DH)),
+                   "l"((const bf16*)cache.v + off), "r"((uint32_t)BLOCK_BYTES), "r"(ad_smem_u32(&bar))
+                   : "memory");
+  };
+  // bytes of the phase-one copies of blocks [b0, b1)
+  auto phase1_bytes = [&](int b0, int b1) {
+    return (uint32_t)(((b1 - b0) + (SV ? max(0, min(b1, HB) - min(b0, HB)) : (b1 - b0))) * BLOCK_BYTES);
   };
   if (warp == 0) {
     if (lane == 0)
       asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(ad_smem_u32(&bar)),
-                   "r"((uint32_t)(2 * n_pre * BLOCK_BYTES))
+                   "r"(phase1_bytes(0, n_pre))
                    : "memory");
     __syncwarp();
-    if (lane < n_pre) copy_block(lane);
+    if (lane < n_pre) copy_block(lane, false);
   }
   pdl_wait();
   KT_WAITED();
@@ -617,13 +643,13 @@ __global__ void __launch_bounds__(AD_THREADS)
     if (lane == 0) {
       if (r >= 0)
         asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(ad_smem_u32(&bar)),
-                     "r"((uint32_t)(2 * (nb - n_pre) * BLOCK_BYTES))
+                     "r"(phase1_bytes(n_pre, nb))
                      : "memory");
       else
         asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(ad_smem_u32(&bar)) : "memory");
     }
     __syncwarp();
-    if (r >= 0 && lane >= n_pre && lane < nb) copy_block(lane);
+    if (r >= 0 && lane >= n_pre && lane < nb) copy_block(lane, false);
   }
   if (r < 0) {
     // the token left at an earlier layer (uniform over the cluster): let the copies land, leave
@@ -694,6 +720,16 @@ __global__ void __launch_bounds__(AD_THREADS)
     }
     __syncthreads();
     KT_MARK(3);
+    if (SV && nb > HB && warp == 0) {
+      // every read of the K slots is done: the second half of V into them
+      asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+      if (lane == 0)
+        asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(ad_smem_u32(&bar2)),
+                     "r"((uint32_t)((nb - HB) * BLOCK_BYTES))
+                     : "memory");
+      __syncwarp();
+      if (lane >= HB && lane < nb) copy_block(lane, true);
+    }
     // chunk max, probabilities, chunk sum
     float mx = -INFINITY;
 #pragma unroll
@@ -719,17 +755,22 @@ __global__ void __launch_bounds__(AD_THREADS)
     float o[8];
 #pragma unroll
     for (int i = 0; i < 8; ++i) o[i] = 0.f;
-    {
+    // key groups [it0, it1) of the warp (SV: the first half's groups read sV, the second's
+    // the K slots after their copy has landed; key = ... + it * AD_WARPS * KPI, so groups below
+    // KIT / 2 hold the keys below AD_CHUNK / 2)
+    auto pv = [&](int it0, int it1, const bf16* base, int key0) {
       uint4 vr[KIT];
       float pr[KIT];
 #pragma unroll
       for (int it = 0; it < KIT; ++it) {
+        if (it < it0 || it >= it1) continue;
         const int key = warp * KPI + it * AD_WARPS * KPI + slot;
-        vr[it] = *reinterpret_cast<const uint4*>(sV + key * DH + part * 8);
+        vr[it] = *reinterpret_cast<const uint4*>(base + (key - key0) * DH + part * 8);
         pr[it] = s_p[key];
       }
 #pragma unroll
       for (int it = 0; it < KIT; ++it) {
+        if (it < it0 || it >= it1) continue;
         const __nv_bfloat162* b = reinterpret_cast<const __nv_bfloat162*>(&vr[it]);
 #pragma unroll
         for (int i = 0; i < 4; ++i) {
@@ -738,6 +779,16 @@ __global__ void __launch_bounds__(AD_THREADS)
           o[2 * i] += pr[it] != 0.f ? pr[it] * f.x : 0.f;
           o[2 * i + 1] += pr[it] != 0.f ? pr[it] * f.y : 0.f;
         }
+      }
+    };
+    if (!SV) {
+      pv(0, KIT, sV, 0);
+    } else {
+      pv(0, KIT / 2, sV, 0);
+      if (nb > HB) {
+        bool ok = ad_wait(&bar2, err);
+        if (!ok) ad_wait(&bar2, err);   // second bounded wait for the copies in flight; results flagged
+        pv(KIT / 2, KIT, sK, AD_CHUNK / 2);
       }
     }
 #pragma unroll
@@ -880,7 +931,7 @@ __global__ void __launch_bounds__(AD_THREADS)
 }
 
 static int g_attn_smem_set[2] = {0, 0};
-static int g_ad_smem_set[4] = {0, 0, 0, 0};
+static int g_ad_smem_set[8] = {0, 0, 0, 0, 0, 0, 0, 0};
 
 void launch_attention(cudaStream_t st, int dt, const void* q, int ld_q, void* out, int ld_out, DevRange rows,
                       int max_rows, const int* row_tok, const int* tok_seq, const int* tok_pos, const int* seq_len,
@@ -904,14 +955,19 @@ void launch_attention(cudaStream_t st, int dt, const void* q, int ld_q, void* ou
     const dim3 grid(max_rows * cache.n_kv_heads, n_split);
     const int group = n_heads / cache.n_kv_heads;
     const bool cl = n_split > 1 && n_split <= 8;   // chunks of a (row, kv head) merged in a cluster
-    const int smem = 2 * AD_CHUNK * dh * 2 + (cl ? group * n_split * (dh + 4) * 4 : 0);
-    const int vi = (dh == 64 ? 0 : 2) + (cl ? 1 : 0);
+    const bool sv = group == 1;                     // one query head per KV head: 1.5 chunks of rows
+    const int smem = (sv ? 3 * AD_CHUNK / 2 : 2 * AD_CHUNK) * dh * 2 + (cl ? group * n_split * (dh + 4) * 4 : 0);
+    const int vi = (dh == 64 ? 0 : 4) + (cl ? 1 : 0) + (sv ? 2 : 0);
     void (*kern)(const bf16*, int, DevRange, const int*, const int*, const int*, const int*, KVCacheView, int, int, int,
                  float, int, float*, int*, bf16*, int, unsigned*) =
-        vi == 0 ? attn_decode_kernel<64, false>
-        : vi == 1 ? attn_decode_kernel<64, true>
-        : vi == 2 ? attn_decode_kernel<128, false>
-                  : attn_decode_kernel<128, true>;
+        vi == 0 ? attn_decode_kernel<64, false, false>
+        : vi == 1 ? attn_decode_kernel<64, true, false>
+        : vi == 2 ? attn_decode_kernel<64, false, true>
+        : vi == 3 ? attn_decode_kernel<64, true, true>
+        : vi == 4 ? attn_decode_kernel<128, false, false>
+        : vi == 5 ? attn_decode_kernel<128, true, false>
+        : vi == 6 ? attn_decode_kernel<128, false, true>
+                  : attn_decode_kernel<128, true, true>;
     if (g_ad_smem_set[vi] < smem) {
       cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
       g_ad_smem_set[vi] = smem;
