@@ -97,6 +97,7 @@ struct DgParams {
   const float2* tile_stats;   // DG_STATS_TILES: [row][n_stiles] (mean, M2) of 32-column tiles
   int n_stiles;
   int off_a, off_x, off_t, off_p;   // dynamic shared-memory offsets (bytes)
+  int off_r;                        // rotary epilogues: the rows' (cos, sin) table rows [DG_MAX_M][DG_ROPE_HALF]
   int bias_aligned, resid_aligned;
   Epi epi;
   unsigned* err;
@@ -233,7 +234,6 @@ __global__ void __launch_bounds__(DG_THREADS, 1) gemm_decode_kernel(const __grid
   __shared__ __align__(8) uint64_t red_bar;          // leader: one arrival per other split
   __shared__ __align__(16) float s_bias[DG_BN];
   __shared__ __align__(16) float s_res[DG_MAX_M][DG_BN];
-  __shared__ __align__(16) float2 s_rope[DG_MAX_M][DG_ROPE_HALF];
   __shared__ EpiRow s_rr[DG_MAX_M];
   __shared__ float s_red[DG_THREADS / 32][MB * 8];
   __shared__ float s_mu[MB * 8], s_rs[MB * 8];
@@ -262,6 +262,9 @@ __global__ void __launch_bounds__(DG_THREADS, 1) gemm_decode_kernel(const __grid
   constexpr int SLOT = DG_MAX_M * DG_RP;
   float* sP = reinterpret_cast<float*>(dg_smem + p.off_p);              // [2][DG_MAX_M][DG_RP]: own k halves
   float* sR = sP + 2 * SLOT;                                            // [splits - 1][DG_MAX_M][32]: pushed
+  // rotary epilogues only (kept out of the other kernels' footprint, so that more of their
+  // CTAs fit beside a neighbouring launch's)
+  float2 (*s_rope)[DG_ROPE_HALF] = reinterpret_cast<float2 (*)[DG_ROPE_HALF]>(dg_smem + p.off_r);
   const uint32_t rank = p.splits > 1 ? cluster_rank() : 0u;
 
   if (tid == 0) {
@@ -866,7 +869,8 @@ static bool dg_plan(const GemmProblem& q, int max_rows, const DgNorm* norm, int 
   // rings; several splits -> one CTA per (tile, split)
   const int arows = mb == 2 ? 16 : max_rows;   // A-slice rows held in shared memory
   const int tst = prm.stat_mode == DG_STATS_TILES ? prm.n_stiles : 0;
-  const int fixed0 = dg_layout(0, arows, kr, prm.xrows, prm.xk, tst, splits).total + 1024;
+  const int rope_bytes = q.epi.rope ? DG_MAX_M * DG_ROPE_HALF * (int)sizeof(float2) : 0;
+  const int fixed0 = ((dg_layout(0, arows, kr, prm.xrows, prm.xk, tst, splits).total + 15) & ~15) + rope_bytes + 1024;
   int grid = tiles * splits;
   if (splits == 1 && groups == 1) {
     // as many CTAs as can be resident with a ring of at least four stages, each with the
@@ -882,13 +886,15 @@ static bool dg_plan(const GemmProblem& q, int max_rows, const DgNorm* norm, int 
   int stages = (227 * 1024 / per_sm - DG_STATIC_SMEM - fixed0) / stage_bytes;
   stages = std::max(1, std::min(stages, std::min(DG_MAX_STAGES, cta_stages)));
   const DgLayout L = dg_layout(stages * stage_bytes, arows, kr, prm.xrows, prm.xk, tst, splits);
-  const size_t smem = (size_t)L.total + 1024;   // + slack to align the ring to 1024 bytes
+  const int off_r = (L.total + 15) & ~15;
+  const size_t smem = (size_t)off_r + rope_bytes + 1024;   // + slack to align the ring to 1024 bytes
   if (smem > (size_t)DG_SMEM_LIMIT) return false;
   prm.stages = stages;
   prm.off_a = L.off_a;
   prm.off_x = L.off_x;
   prm.off_t = L.off_t;
   prm.off_p = L.off_p;
+  prm.off_r = off_r;
   prm.bias_aligned = ((uintptr_t)q.epi.bias & 15) == 0;
   prm.resid_aligned = ((uintptr_t)q.epi.resid & 15) == 0 && q.epi.ld_resid % 4 == 0;
   prm.epi = q.epi;
@@ -931,7 +937,7 @@ int decode_gemm_grouped(cudaStream_t st, const GemmProblem* probs, int n, int ma
   for (int i = 0; i < n; ++i) {
     const GemmProblem& q = probs[i];
     if (q.epi.kind != EPI_KV || q.A != q0.A || q.lda != q0.lda || q.N != q0.N || q.K != q0.K || q.ldb != q0.ldb ||
-        q.rows.begin != nullptr || !decode_gemm_supported(q, max_rows, nullptr))
+        q.epi.rope != q0.epi.rope || q.rows.begin != nullptr || !decode_gemm_supported(q, max_rows, nullptr))
       return -1;
   }
   thread_local DgParamsG prm;   // one per host thread
