@@ -42,10 +42,10 @@ import synth  # noqa: E402
 PEAKS_FALLBACK = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
 # DRAM bytes (read + write) over algorithmic bytes of a kernel class, from one ncu capture of
 # the current kernel at the workload's layer shapes (profiles/gemm_stream_llama_layer_shapes.md:
-# the QKV and gate/up launches of a generation step, 104.39 + 183.87 MB of DRAM traffic for
+# the QKV and gate/up launches of a generation step, 104.36 + 184.19 MB of DRAM traffic for
 # 100.69 + 180.39 MB of weights, rows and outputs); the line's traffic is this ratio times the
 # class's algorithmic bytes per launch (traffic grows with the weight bytes streamed).
-NCU_TRAFFIC_RATIO = {"gemm_decode": (104.39 + 183.87) / (100.69 + 180.39)}
+NCU_TRAFFIC_RATIO = {"gemm_decode": (104.36 + 184.19) / (100.69 + 180.39)}
 METRIC = "early-exit prefill+decode tokens/s at 1 GB300; skipped-layer KV-fill % of roofline"
 # Llama-7B headline workload: one prompt of LP tokens, LSTEPS greedy steps, exits ~ N(24, 4) on [8, 32]
 LP, LSTEPS, LMEAN, LSD, LLO, LHI = 2048, 256, 24.0, 4.0, 8, 32
