@@ -424,7 +424,10 @@ __global__ void __launch_bounds__(256) exit_small_kernel(const float* Xin, const
 // row per 512 >> rshift threads), the decision and compaction run on the reduced sums,
 // and the moves are written from the registers.
 constexpr int EXD_THREADS = 512;
-constexpr int EXD_V = 4;   // float4 per thread per row vector
+constexpr int EXD_V = 4;   // most float4 per thread per row vector
+// V: float4 per thread per row vector, the fewest that cover a row (the kernel runs cold in
+// every layer of a generation step, so its unrolled code is kept to what the rows need)
+template <int V>
 __global__ void __launch_bounds__(EXD_THREADS)
     exit_decode_kernel(const float* __restrict__ Xin, const float* __restrict__ Xout, const float* __restrict__ I,
                        int first, int D, int* ctr, int par, const int* row_tok, int* row_tok_next, const int* forced,
@@ -454,13 +457,13 @@ __global__ void __launch_bounds__(EXD_THREADS)
   const int forced_r = forced && (int)threadIdx.x < max_rows ? forced[tok_r] : 0;   // the decider's forced layer
   const float delta = *delta_p;
   const int D4 = D >> 2;
-  float4 xs[EXD_V], xi[EXD_V], xp[EXD_V];
+  float4 xs[V], xi[V], xp[V];
   float ns = 0.f, ni = 0.f, dot = 0.f, sx = 0.f, np_ = 0.f, dp = 0.f;
   if (row < max_rows) {
     const float4* i4 = reinterpret_cast<const float4*>(I + (size_t)row * D);
     const float4* p4 = reinterpret_cast<const float4*>(Xin + (size_t)row * D);
 #pragma unroll
-    for (int j = 0; j < EXD_V; ++j) {
+    for (int j = 0; j < V; ++j) {
       const int v = sub + j * tpr;
       if (v < D4) {
         xi[j] = first ? make_float4(0.f, 0.f, 0.f, 0.f) : i4[v];
@@ -474,12 +477,12 @@ __global__ void __launch_bounds__(EXD_THREADS)
   if (row < max_rows) {
     const float4* s4 = reinterpret_cast<const float4*>(Xout + (size_t)row * D);
 #pragma unroll
-    for (int j = 0; j < EXD_V; ++j) {
+    for (int j = 0; j < V; ++j) {
       const int v = sub + j * tpr;
       if (v < D4) xs[j] = s4[v];
     }
 #pragma unroll
-    for (int j = 0; j < EXD_V; ++j) {
+    for (int j = 0; j < V; ++j) {
       if (row < n && sub + j * tpr < D4) {
         const float4 a = xs[j], c = xi[j];
         ns += a.x * a.x + a.y * a.y + a.z * a.z + a.w * a.w;
@@ -564,7 +567,7 @@ __global__ void __launch_bounds__(EXD_THREADS)
     float c2 = 0.f;
     if (row < n) {
 #pragma unroll
-      for (int j = 0; j < EXD_V; ++j)
+      for (int j = 0; j < V; ++j)
         if (sub + j * tpr < D4) {
           const float4 a = xs[j];
           c2 += (a.x - mu) * (a.x - mu) + (a.y - mu) * (a.y - mu) + (a.z - mu) * (a.z - mu) + (a.w - mu) * (a.w - mu);
@@ -580,7 +583,7 @@ __global__ void __launch_bounds__(EXD_THREADS)
       const float m0 = smode == NORM_COPY ? 0.f : mu;
       uint2* o = reinterpret_cast<uint2*>(xhat_next + (size_t)s_dst[row] * D);
 #pragma unroll
-      for (int j = 0; j < EXD_V; ++j) {
+      for (int j = 0; j < V; ++j) {
         const int v = sub + j * tpr;
         if (v < D4) {
           const float4 a = xs[j];
@@ -601,7 +604,7 @@ __global__ void __launch_bounds__(EXD_THREADS)
     float4* xn = reinterpret_cast<float4*>(Xnext + (size_t)d0 * D);
     float4* inn = reinterpret_cast<float4*>(Inext + (size_t)d0 * D);
 #pragma unroll
-    for (int j = 0; j < EXD_V; ++j) {
+    for (int j = 0; j < V; ++j) {
       const int v = sub + j * tpr;
       if (v < D4) {
         const float4 a = xs[j], c = xi[j];
@@ -615,7 +618,7 @@ __global__ void __launch_bounds__(EXD_THREADS)
     float4* hp = reinterpret_cast<float4*>(hsm_prev + kk * D);
     float4* hi = reinterpret_cast<float4*>(hsm_I + kk * D);
 #pragma unroll
-    for (int j = 0; j < EXD_V; ++j) {
+    for (int j = 0; j < V; ++j) {
       const int v = sub + j * tpr;
       if (v < D4) {
         hs[v] = xs[j];
@@ -637,7 +640,8 @@ bool launch_exit_small(cudaStream_t st, const float* Xin, const float* Xout, con
   const bool aligned = ((uintptr_t)Xin | (uintptr_t)Xout | (uintptr_t)I | (uintptr_t)Xnext | (uintptr_t)Inext |
                         (uintptr_t)hsm_s | (uintptr_t)hsm_prev | (uintptr_t)hsm_I) % 16 == 0;
   if (max_rows <= 16 && D % 4 == 0 && D / 4 <= EXD_V * (EXD_THREADS >> rshift) && aligned) {
-    launch_k(exit_decode_kernel, 1, EXD_THREADS, 0, st, Xin, Xout, I, first, D, ctr, par, row_tok, row_tok_next, forced,
+    auto* kern = D / 4 <= 2 * (EXD_THREADS >> rshift) ? exit_decode_kernel<2> : exit_decode_kernel<EXD_V>;
+    launch_k(kern, 1, EXD_THREADS, 0, st, Xin, Xout, I, first, D, ctr, par, row_tok, row_tok_next, forced,
              layer, n_layers, delta_p, test, sim, exit_tok, exit_layer_out, Xnext, Inext, hsm_s, hsm_prev, hsm_I,
              rshift, max_rows, xhat_next, smode, seps, metric, aao_len, tok_pos, err);
     return true;
