@@ -280,11 +280,16 @@ ADEPT_API adept_status adept_check_device_status(adept_model* m, void* stream);
  * ATTN_TC (default 1): the prompt-pass attention of bf16 models (self- and cross-attention,
  * head_dim 64 or 128) runs on the tcgen05 kernel (S and O accumulated in tensor memory, P
  * rounded to bf16); 0 keeps the mma.sync kernel (which the encoder's stop-entirely variant
- * always uses). */
+ * always uses).  FUSED_EXIT (default 1): in generation steps of at most 4 sequences whose QKV
+ * product runs on the stream-K kernel (decoders without cross-attention, global exit
+ * similarity), the exit step of layer i (test, inertia update, compaction) is taken by layer
+ * i+1's QKV launch: every CTA reduces the layer's rows and takes the same decisions, so the
+ * separate exit kernel and its launch leave the step; 0 launches the exit kernel after every
+ * layer. */
 enum { ADEPT_OPT_HSM_IDENTITY = 1, ADEPT_OPT_PROFILE = 2, ADEPT_OPT_GEMM_SIMT = 3, ADEPT_OPT_DECODE_GRAPH = 4,
        ADEPT_OPT_DECODE_GEMM = 5, ADEPT_OPT_EXIT_METRIC = 7, ADEPT_OPT_ALL_AT_ONCE = 8,
        ADEPT_OPT_STOP_ENTIRELY = 9, ADEPT_OPT_DECODE_STREAM = 10, ADEPT_OPT_DECODE_TILED = 11,
-       ADEPT_OPT_SPAN_TIMER = 12, ADEPT_OPT_ATTN_TC = 13 };
+       ADEPT_OPT_SPAN_TIMER = 12, ADEPT_OPT_ATTN_TC = 13, ADEPT_OPT_FUSED_EXIT = 14 };
 ADEPT_API adept_status adept_set_option(adept_model* m, int option, int value);
 
 /* Kernel classes reported by adept_profile_read: the GEMMs of prompt passes (layer

@@ -21,7 +21,7 @@ STATUS_NAMES = {0: "OK", 1: "INVALID_ARG", 2: "OOM", 3: "CAPACITY", 4: "CUDA", 5
 FAMILY = {"llama": 0, "gpt2": 1, "bert": 2}
 OPT_HSM_IDENTITY, OPT_PROFILE, OPT_GEMM_SIMT, OPT_DECODE_GRAPH, OPT_DECODE_GEMM = 1, 2, 3, 4, 5
 OPT_EXIT_METRIC, OPT_ALL_AT_ONCE, OPT_STOP_ENTIRELY, OPT_DECODE_STREAM, OPT_DECODE_TILED = 7, 8, 9, 10, 11
-OPT_SPAN_TIMER, OPT_ATTN_TC = 12, 13
+OPT_SPAN_TIMER, OPT_ATTN_TC, OPT_FUSED_EXIT = 12, 13, 14
 EXIT_GLOBAL, EXIT_LOCAL, EXIT_BOTH = 0, 1, 2
 PROF_GEMM_PREFILL, PROF_KV_FILL, PROF_ATTENTION, PROF_GEMM_DECODE, PROF_GEMM_TRAIN = 0, 1, 2, 3, 4
 HSM_PARAMS, HSM_GRADS, HSM_MOMENT1, HSM_MOMENT2 = 0, 1, 2, 3

@@ -36,6 +36,7 @@
 #include "gemm_stream.h"
 #include "epilogue.cuh"
 #include "gemm_tc.h"
+#include "kernels.h"
 
 #include <cuda.h>
 
@@ -95,6 +96,8 @@ struct DsParams {
   int* cnt;
   unsigned* err;
   SpanCtx span;
+  int exit_on;   // EPI_QKV, one problem: the previous layer's exit step first (ex)
+  DsExit ex;
 };
 
 __device__ __forceinline__ uint32_t smem_u32(const void* p) { return (uint32_t)__cvta_generic_to_shared(p); }
@@ -389,6 +392,200 @@ __device__ void ds_stage_a(const DsParams<MAXG>& p, bf16* sA, int Ms, float* s_m
   }
 }
 
+// What the exit step reads before the grid-dependency wait: everything the previous layer's exit
+// step wrote (it finished several launches earlier), i.e. the layer's row count and exit count,
+// the threshold, the first row's token, forced layer and inertia (from HBM by now); only s_i
+// (the preceding kernel's output) is read after the wait.
+struct DsExitPre {
+  float4 xi[DS_XV];
+  int n, base, tok0, f0;
+  float delta;
+};
+template <int MAXG>
+__device__ __forceinline__ void ds_exit_prefetch(const DsParams<MAXG>& p, DsExitPre& e) {
+  const DsExit& x = p.ex;
+  const int tid = threadIdx.x, K4 = p.K >> 2;
+  e.n = x.ctr[CTR_ACTIVE + x.par];
+  e.base = x.ctr[CTR_PREFIX + x.layer - 1];
+  e.delta = *x.delta;
+  e.tok0 = x.row_tok[0];
+  e.f0 = (x.forced && tid == 0) ? x.forced[e.tok0] : 0;
+  const float4* i4 = reinterpret_cast<const float4*>(x.I);
+  const float4 z4 = make_float4(0.f, 0.f, 0.f, 0.f);
+#pragma unroll
+  for (int j = 0; j < DS_XV; ++j) {
+    const int v = tid + j * DS_THREADS;
+    e.xi[j] = (v < K4 && !x.first) ? i4[v] : z4;
+  }
+}
+
+// The previous layer's exit step inside the QKV launch (DsExit; the global similarity of Sec.
+// 4.1), rows one at a time: s_i and the inertia read once into registers, the four sums reduced
+// over the CTA in a fixed order (every CTA of the launch decides alike), the decision (a forced
+// layer, else similarity >= delta), then from the registers the kept row standardised into the A
+// operand at its compacted index, and this CTA's slice of the moved rows (a leaving row's s_{i-1}
+// copied from memory).  Rows past the kept ones are zeroed.  Ends with a CTA barrier; s_M /
+// s_live / s_nlive describe the kept rows.
+template <int MAXG>
+__device__ void ds_exit_stage(const DsParams<MAXG>& p, const DsExitPre& pre, bf16* sA, float (*s_red)[16], int* s_M,
+                              int* s_live, int* s_nlive, int* s_tokk, float* s_bc) {
+  const DsExit& x = p.ex;
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  const int K = p.K, K4 = K >> 2, ap = p.apitch;
+  const int G = gridDim.x, c = blockIdx.x;
+  const int n_all = pre.n;
+  const int n = min(n_all, p.max_m);
+  const int base = pre.base;
+  const float delta = pre.delta;
+  if (n_all > p.max_m && c == 0 && tid == 0) atomicOr(x.err, ERRW_CONFIG);
+  // this CTA's slice of every moved row: float4 indices [v0, v1)
+  const int v0 = (int)((long long)c * K4 / G), v1 = (int)((long long)(c + 1) * K4 / G);
+  const float4 z4 = make_float4(0.f, 0.f, 0.f, 0.f);
+  int k = 0, e = 0;   // rows kept / left so far (the same in every thread)
+  for (int r = 0; r < n; ++r) {
+    const float4* s4 = reinterpret_cast<const float4*>(x.Xout + (size_t)r * K);
+    const float4* i4 = reinterpret_cast<const float4*>(x.I + (size_t)r * K);
+    const float4* p4 = reinterpret_cast<const float4*>(x.Xin + (size_t)r * K);
+    const int tok = r == 0 ? pre.tok0 : x.row_tok[r];
+    float4 xs[DS_XV], xi[DS_XV];
+#pragma unroll
+    for (int j = 0; j < DS_XV; ++j) {   // every load first (the first row's inertia: read before the wait)
+      const int v = tid + j * DS_THREADS;
+      xs[j] = v < K4 ? s4[v] : z4;
+      xi[j] = r == 0 ? pre.xi[j] : (v < K4 && !x.first) ? i4[v] : z4;
+    }
+    float ns = 0.f, ni = 0.f, dot = 0.f, sx = 0.f;
+#pragma unroll
+    for (int j = 0; j < DS_XV; ++j) {
+      const float4 a = xs[j], b = xi[j];
+      ns += a.x * a.x + a.y * a.y + a.z * a.z + a.w * a.w;
+      ni += b.x * b.x + b.y * b.y + b.z * b.z + b.w * b.w;
+      dot += a.x * b.x + a.y * b.y + a.z * b.z + a.w * b.w;
+      sx += a.x + a.y + a.z + a.w;
+    }
+    ns = warp_sum(ns);
+    ni = warp_sum(ni);
+    dot = warp_sum(dot);
+    sx = warp_sum(sx);
+    if (lane == 0) {
+      s_red[warp][0] = ns;
+      s_red[warp][1] = ni;
+      s_red[warp][2] = dot;
+      s_red[warp][3] = sx;
+    }
+    __syncthreads();
+    if (tid == 0) {
+      float a = 0.f, b = 0.f, cc = 0.f, m = 0.f;
+      for (int w = 0; w < DS_WARPS; ++w) {
+        a += s_red[w][0];
+        b += s_red[w][1];
+        cc += s_red[w][2];
+        m += s_red[w][3];
+      }
+      int ex = 0;
+      if (x.test) {
+        const float cs = exit_similarity(EXIT_GLOBAL, a, b, cc, 0.f, 0.f);
+        if (x.sim && c == 0) x.sim[(size_t)tok * x.n_layers + (x.layer - 1)] = cs;
+        const int f = r == 0 ? pre.f0 : x.forced ? x.forced[tok] : 0;
+        if (f != 0 && (f < 2 || f > x.n_layers) && c == 0) atomicOr(x.err, ERRW_FORCED);
+        ex = (f > 0) ? (f == x.layer) : (cs >= delta);
+      }
+      s_bc[0] = ex ? 1.f : 0.f;
+      s_bc[1] = a > 0.f ? rsqrtf(a) : 0.f;                 // inertia step weight 1 / |s_i|
+      s_bc[2] = x.norm_mode == NORM_LN ? m / K : 0.f;       // the row's mean (LayerNorm)
+      s_bc[3] = a;                                          // sum of squares (RMSNorm)
+    }
+    __syncthreads();
+    const bool left = s_bc[0] != 0.f;
+    const float w = s_bc[1], mu = s_bc[2];
+    if (!left) {
+      // the kept row standardised (as the standardisation kernel: LayerNorm two-pass from the
+      // registers, RMSNorm from the sum of squares) into A row k, bf16
+      float rs = 1.f, m0 = 0.f;
+      if (x.norm_mode == NORM_LN) {
+        float c2 = 0.f;
+#pragma unroll
+        for (int j = 0; j < DS_XV; ++j)
+          if (tid + j * DS_THREADS < K4) {
+            const float4 a = xs[j];
+            c2 += (a.x - mu) * (a.x - mu) + (a.y - mu) * (a.y - mu) + (a.z - mu) * (a.z - mu) +
+                  (a.w - mu) * (a.w - mu);
+          }
+        c2 = warp_sum(c2);
+        if (lane == 0) s_red[warp][6] = c2;
+        __syncthreads();
+        float t = 0.f;
+        for (int w2 = 0; w2 < DS_WARPS; ++w2) t += s_red[w2][6];
+        rs = rsqrtf(t / K + x.eps);
+        m0 = mu;
+      } else if (x.norm_mode == NORM_RMS) {
+        rs = rsqrtf(s_bc[3] / K + x.eps);
+      }
+      float4* xn = reinterpret_cast<float4*>(x.Xnext + (size_t)k * K);
+      float4* in = reinterpret_cast<float4*>(x.Inext + (size_t)k * K);
+#pragma unroll
+      for (int j = 0; j < DS_XV; ++j) {
+        const int v = tid + j * DS_THREADS;
+        if (v < K4) {
+          const float4 a = xs[j], b = xi[j];
+          const __nv_bfloat162 lo = __floats2bfloat162_rn((a.x - m0) * rs, (a.y - m0) * rs);
+          const __nv_bfloat162 hi = __floats2bfloat162_rn((a.z - m0) * rs, (a.w - m0) * rs);
+          uint2 u;
+          u.x = *reinterpret_cast<const uint32_t*>(&lo);
+          u.y = *reinterpret_cast<const uint32_t*>(&hi);
+          *reinterpret_cast<uint2*>(sA + (size_t)k * ap + v * 4) = u;
+          if (v >= v0 && v < v1) {
+            xn[v] = a;
+            in[v] = make_float4(b.x + a.x * w, b.y + a.y * w, b.z + a.z * w, b.w + a.w * w);
+          }
+        }
+      }
+      if (tid == 0) {
+        s_tokk[k] = tok;
+        if (c == 0) x.row_tok_next[k] = tok;
+      }
+      ++k;
+    } else {
+      // the leaving row's mapper inputs at its exit slot
+      const size_t slot = (size_t)(base + e);
+      float4* hs = reinterpret_cast<float4*>(x.hsm_s + slot * K);
+      float4* hp = reinterpret_cast<float4*>(x.hsm_prev + slot * K);
+      float4* hi = reinterpret_cast<float4*>(x.hsm_I + slot * K);
+#pragma unroll
+      for (int j = 0; j < DS_XV; ++j) {
+        const int v = tid + j * DS_THREADS;
+        if (v < K4 && v >= v0 && v < v1) {
+          hs[v] = xs[j];
+          hp[v] = p4[v];
+          hi[v] = xi[j];
+        }
+      }
+      if (tid == 0 && c == 0) {
+        x.exit_tok[base + e] = tok;
+        if (x.exit_layer) x.exit_layer[tok] = x.layer;
+      }
+      ++e;
+    }
+    __syncthreads();   // s_red / s_bc are reused by the next row
+  }
+  // rows past the kept ones stay zero (they feed only token columns that are never stored)
+  for (int i = tid; i < (p.arows - k) * (ap >> 3); i += DS_THREADS) {
+    const int rr = k + i / (ap >> 3), cc = i % (ap >> 3);
+    *reinterpret_cast<uint4*>(sA + (size_t)rr * ap + cc * 8) = make_uint4(0, 0, 0, 0);
+  }
+  if (tid == 0) {
+    if (c == 0) {
+      x.ctr[CTR_ACTIVE + (x.par ^ 1)] = k;
+      x.ctr[CTR_EXITED] = base + e;
+      x.ctr[CTR_PREFIX + x.layer] = base + e;
+    }
+    s_M[0] = k;
+    s_live[0] = 0;
+    *s_nlive = k > 0 ? 1 : 0;
+  }
+  __syncthreads();
+}
+
 // MB: 8-token blocks of the A operand (1: M <= 8, 2: M <= 16); KIND: the epilogue kind.
 template <int MB, int KIND, int MAXG>
 __global__ void __launch_bounds__(DS_THREADS, 2) gemm_stream_kernel(const __grid_constant__ DsParams<MAXG> p) {
@@ -403,6 +600,8 @@ __global__ void __launch_bounds__(DS_THREADS, 2) gemm_stream_kernel(const __grid
   __shared__ int s_M[MAXG], s_rb[MAXG];
   __shared__ int s_nlive, s_last;
   __shared__ int s_pos[16], s_blk[16];   // cache epilogues: each row's position and cache block
+  __shared__ int s_tokk[16];             // exit step: the kept rows' tokens
+  __shared__ float s_bc[4];              // exit step: one row's decision, weight, mean, sum of squares
   __shared__ int s_info[2][3];           // per hand-off buffer: live problem slot, tile, whole
   __shared__ int s_eok[DS_NE];           // epilogue warps: still following the hand-offs
   __shared__ unsigned s_span_left;
@@ -483,32 +682,41 @@ __global__ void __launch_bounds__(DS_THREADS, 2) gemm_stream_kernel(const __grid
     }
   }
 
+  DsExitPre xpre;
+  if (KIND == EPI_QKV && p.exit_on) ds_exit_prefetch(p, xpre);
+
   pdl_wait();   // from here on, the preceding kernels' writes are visible
   KT_WAITED();
   span.waited();
 
-  // The row counts (device values) and the A operand are read in parallel: every problem's
-  // rows start at row 0 (host-checked), so the launch's row bound max_m is staged without
-  // waiting for the count (rows past it feed only token columns that are never stored).
-  if (warp == 0) {
-    // lane q reads problem q's count (all loads at once; MAXG <= 32), the live problems are
-    // listed in problem order
-    const int q = lane;
-    int M = 0;
-    if (q < p.n_probs) {
-      M = p.rows[q].e();
-      if (M > p.max_m) {   // more rows than the launch was sized for
-        atomicOr(p.err, ERRW_CONFIG);
-        M = p.max_m;
+  if (KIND == EPI_QKV && p.exit_on) {
+    // the previous layer's exit step first: its kept rows are this launch's rows
+    if (tid == 0) s_rb[0] = 0;
+    ds_exit_stage(p, xpre, sA, s_red, s_M, s_live, &s_nlive, s_tokk, s_bc);
+  } else {
+    // The row counts (device values) and the A operand are read in parallel: every problem's
+    // rows start at row 0 (host-checked), so the launch's row bound max_m is staged without
+    // waiting for the count (rows past it feed only token columns that are never stored).
+    if (warp == 0) {
+      // lane q reads problem q's count (all loads at once; MAXG <= 32), the live problems are
+      // listed in problem order
+      const int q = lane;
+      int M = 0;
+      if (q < p.n_probs) {
+        M = p.rows[q].e();
+        if (M > p.max_m) {   // more rows than the launch was sized for
+          atomicOr(p.err, ERRW_CONFIG);
+          M = p.max_m;
+        }
+        s_M[q] = M;
+        s_rb[q] = 0;
       }
-      s_M[q] = M;
-      s_rb[q] = 0;
+      const unsigned live = __ballot_sync(0xffffffffu, q < p.n_probs && M > 0);
+      if (q < p.n_probs && M > 0) s_live[__popc(live & ((1u << q) - 1u))] = q;
+      if (lane == 0) s_nlive = __popc(live);
     }
-    const unsigned live = __ballot_sync(0xffffffffu, q < p.n_probs && M > 0);
-    if (q < p.n_probs && M > 0) s_live[__popc(live & ((1u << q) - 1u))] = q;
-    if (lane == 0) s_nlive = __popc(live);
+    ds_stage_a(p, sA, p.max_m, s_mu, s_rs, s_red);   // ends with a CTA barrier: the counts are visible
   }
-  ds_stage_a(p, sA, p.max_m, s_mu, s_rs, s_red);   // ends with a CTA barrier: the counts are visible
   KT_MARK(1);
   const int nlive = s_nlive;
   if (p.grouped) {
@@ -569,7 +777,7 @@ __global__ void __launch_bounds__(DS_THREADS, 2) gemm_stream_kernel(const __grid
       int Ms = 0;
       for (int k = 0; k < nlive; ++k) Ms = max(Ms, s_M[s_live[k]]);
       if (et < Ms) {
-        const int tok = e0.row_tok[et];
+        const int tok = (KIND == EPI_QKV && p.exit_on) ? s_tokk[et] : e0.row_tok[et];
         const int pos = e0.tok_pos[tok], seq = e0.tok_seq[tok];
         const KVCacheView& cv = e0.cache;
         int blk = -1;
@@ -909,6 +1117,33 @@ int stream_gemm(cudaStream_t st, const GemmProblem& q, int max_rows, const DgNor
   prm.rows[0] = q.rows;
   prm.epi[0] = q.epi;
   const cudaError_t e = mb == 2 ? ds_launch_kind<2, 1>(st, prm, grid, smem) : ds_launch_kind<1, 1>(st, prm, grid, smem);
+  return e == cudaSuccess ? 1 : -1;
+}
+
+int stream_gemm_exit(cudaStream_t st, const GemmProblem& q, int max_rows, const DsExit& ex, const DsWork& ws,
+                     unsigned* err) {
+  if (q.epi.kind != EPI_QKV || max_rows < 1 || max_rows > DS_EXIT_MAX_ROWS) return -1;
+  if (q.K % 4 || q.K / 4 > DS_XV * DS_THREADS || ex.layer < 1 || ex.layer >= ex.n_layers) return -1;
+  if (ex.metric != EXIT_GLOBAL) return -1;   // the local rules also need s_{i-1}'s sums
+  if (!ex.Xin || !ex.Xout || !ex.I || !ex.Xnext || !ex.Inext || !ex.hsm_s || !ex.hsm_prev || !ex.hsm_I || !ex.ctr ||
+      !ex.row_tok || !ex.row_tok_next || !ex.delta || !ex.exit_tok)
+    return -1;
+  const uintptr_t al = (uintptr_t)ex.Xin | (uintptr_t)ex.Xout | (uintptr_t)ex.I | (uintptr_t)ex.Xnext |
+                       (uintptr_t)ex.Inext | (uintptr_t)ex.hsm_s | (uintptr_t)ex.hsm_prev | (uintptr_t)ex.hsm_I;
+  if (al & 15) return -1;
+  thread_local DsParams<1> prm;   // one per host thread
+  int grid = 0, mb = 1;
+  size_t smem = 0;
+  if (!ds_plan(q, 1, max_rows, nullptr, ws, err, prm, grid, smem, mb)) return -1;
+  prm.bt[0] = ds_tiled(q, prm.nkb);
+  if (!prm.bt[0] && !tc_encode_weight_3d(&prm.wmap[0], q.B, q.K, q.N, (size_t)q.ldb * 2, DS_BN, DS_KB / 64))
+    return -1;
+  prm.grouped = 0;
+  prm.rows[0] = q.rows;
+  prm.epi[0] = q.epi;
+  prm.exit_on = 1;
+  prm.ex = ex;
+  const cudaError_t e = mb == 2 ? ds_launch<2, EPI_QKV, 1>(st, prm, grid, smem) : ds_launch<1, EPI_QKV, 1>(st, prm, grid, smem);
   return e == cudaSuccess ? 1 : -1;
 }
 

@@ -15,6 +15,18 @@ enum : int {
 };
 __host__ __device__ static inline int ctr_words(int n_layers) { return CTR_PREFIX + n_layers + 2; }
 
+// The similarity the exit test compares with delta: global cos(s_i, I) (Eq. 7), local
+// cos(s_i, s_{i-1}) or both (their minimum: both must reach delta), App. H.3; from the sums
+// ns = |s_i|^2, ni = |I|^2, dot = <s_i, I>, np = |s_{i-1}|^2, dp = <s_i, s_{i-1}>.  A zero
+// norm gives -inf (never exits).
+static __device__ __forceinline__ float exit_similarity(int metric, float ns, float ni, float dot, float np_,
+                                                       float dp) {
+  const float g = (ns > 0.f && ni > 0.f) ? dot / sqrtf(ns * ni) : -INFINITY;
+  if (metric == EXIT_GLOBAL) return g;
+  const float l = (ns > 0.f && np_ > 0.f) ? dp / sqrtf(ns * np_) : -INFINITY;
+  return metric == EXIT_LOCAL ? l : fminf(g, l);
+}
+
 // Token -> (sequence, position) maps, identity row map, the pass's counters (all rows
 // active), if sim is given NaN for every (token, layer) similarity, and if tok_exit is
 // given N as every token's exit layer so far.

@@ -170,16 +170,6 @@ __global__ void layernorm_inplace_kernel(float* X, DevRange rows, int D, const f
 // ---------------------------------------------------------------------------
 // exit test (Sec. 4.1): c = <s_i, I> / (|s_i| |I|) vs delta, or the forced layer
 // ---------------------------------------------------------------------------
-// The similarity the exit test compares with delta: global cos(s_i, I) (Eq. 7), local
-// cos(s_i, s_{i-1}) or both (their minimum: both must reach delta), App. H.3; from the sums
-// ns = |s_i|^2, ni = |I|^2, dot = <s_i, I>, np = |s_{i-1}|^2, dp = <s_i, s_{i-1}>.  A zero
-// norm gives -inf (never exits).
-__device__ __forceinline__ float exit_similarity(int metric, float ns, float ni, float dot, float np_, float dp) {
-  const float g = (ns > 0.f && ni > 0.f) ? dot / sqrtf(ns * ni) : -INFINITY;
-  if (metric == EXIT_GLOBAL) return g;
-  const float l = (ns > 0.f && np_ > 0.f) ? dp / sqrtf(ns * np_) : -INFINITY;
-  return metric == EXIT_LOCAL ? l : fminf(g, l);
-}
 
 __global__ void exit_decide_kernel(const float* Xout, const float* I, const float* Xin, int D, DevRange rows,
                                    const int* row_tok, const int* forced, int layer, int n_layers,

@@ -167,6 +167,7 @@ struct adept_model {
   // options / instrumentation
   int hsm_identity = 0, profile = 0, force_simt = 0, use_graph = 1, use_dg = 1, use_stream = 1, use_tiled = 1;
   int use_attn_tc = 1;   // prompt-pass attention on the tcgen05 kernel
+  int use_fused_exit = 1;   // generation steps: layer i's exit step inside layer i+1's QKV launch
   int exit_metric = 0;   // EXIT_GLOBAL / EXIT_LOCAL / EXIT_BOTH
   int all_at_once = 0;   // prompt passes: sequences leave with their last prompt token
   int stop_entirely = 0; // encoders: exited tokens get no deeper K/V and leave deeper attention
@@ -413,6 +414,24 @@ static int streaming_gemm_grouped(adept_model* m, cudaStream_t st, const GemmPro
   }
   if (stream_gemm_grouped(st, probs, n, max_rows, ds_work(m), m->err_word) >= 0) return 1;
   return max_rows <= DG_FILL_MAX_ROWS ? decode_gemm_grouped(st, probs, n, max_rows, m->err_word) : -1;
+}
+
+// The QKV product of a generation step with the previous layer's exit step in the same launch
+// (stream-K kernel); -1 when that launch does not take it.
+static int streaming_gemm_exit(adept_model* m, cudaStream_t st, const GemmProblem& p0, int max_rows,
+                               const DsExit& ex, int cls) {
+  if (!m->use_stream || !m->use_dg || m->force_simt || m->dt != ADEPT_DTYPE_BF16) return -1;
+  cudaEvent_t b = nullptr;
+  prof_begin(m, cls, st, &b);
+  int r;
+  {
+    SpanGuard sg(m, cls);
+    GemmProblem p = p0;
+    if (!m->use_tiled) p.Bt = nullptr;
+    r = stream_gemm_exit(st, p, max_rows, ex, ds_work(m), m->err_word);
+  }
+  prof_end(m, cls, st, b, 0, 0);
+  return r;
 }
 
 static void gemm(adept_model* m, cudaStream_t st, const GemmProblem* probs, int n_probs, const int* max_rows,
@@ -1048,6 +1067,17 @@ static adept_status run_pass(adept_model* m, int n_tok, int batch, int prompt_le
   // all-at-once exits apply to prompt passes (a generation step holds one token per sequence)
   const int aao_len = !decode && m->all_at_once ? prompt_len : 0;
   (void)batch;
+  // generation steps of a few sequences: layer i's exit step is taken by layer i+1's QKV launch
+  // (or, if that launch declines, launched on its own just before it)
+  const bool fuse_exit = decode && dgrows && !cross && !stop && m->use_fused_exit && m->use_stream &&
+                         n_tok <= DS_EXIT_MAX_ROWS && aao_len == 0;
+  struct {
+    bool on;
+    int layer, par;
+    float* Xi;
+    float* Ii;
+    int* rt;
+  } pend = {false, 0, 0, nullptr, nullptr, nullptr};
   int par = 0;
   for (int i = 1; i <= N; ++i) {
     const int l0 = i - 1;
@@ -1077,10 +1107,38 @@ static adept_status run_pass(adept_model* m, int n_tok, int batch, int prompt_le
       m->launches += 1;
       gemm(m, st, pr, 2, mrs, m->gemm_cls);
     } else {
-      if (xn_valid)
-        gemm(m, st, pr, 1, mrs, m->gemm_cls);
-      else
-        gemm_std(m, st, pr[0], mr, Xi, D, nullptr, amode, eps, m->gemm_cls);
+      bool done = false;
+      if (pend.on) {
+        pend.on = false;
+        const int pl = pend.layer, pp = pend.par;
+        DsExit ex;
+        ex.Xin = pend.Xi; ex.Xout = m->X_out; ex.I = pend.Ii; ex.Xnext = m->X_in[pp ^ 1]; ex.Inext = m->I[pp ^ 1];
+        ex.hsm_s = m->hsm_s; ex.hsm_prev = m->hsm_prev; ex.hsm_I = m->hsm_I;
+        ex.ctr = m->ctr; ex.row_tok = pend.rt; ex.row_tok_next = m->row_tok[pp ^ 1];
+        ex.forced = forced; ex.delta = m->d_delta; ex.sim = sim_out; ex.exit_tok = m->exit_tok;
+        ex.exit_layer = exit_w; ex.err = m->err_word;
+        ex.par = pp; ex.layer = pl; ex.n_layers = N; ex.first = pl == 1; ex.test = pl >= 2;
+        ex.metric = m->exit_metric; ex.norm_mode = amode; ex.eps = eps;
+        done = streaming_gemm_exit(m, st, pr[0], mr, ex, m->gemm_cls) >= 0;
+        if (done) {
+          m->launches += 1;
+        } else {
+          // not taken: the exit step on its own first, then the product
+          xn_valid = launch_exit_small(st, pend.Xi, m->X_out, pend.Ii, pl == 1, D, m->ctr, pp, pend.rt,
+                                       m->row_tok[pp ^ 1], forced, pl, N, m->d_delta, pl >= 2, sim_out, m->exit_tok,
+                                       exit_w, m->X_in[pp ^ 1], m->I[pp ^ 1], m->hsm_s, m->hsm_prev, m->hsm_I, mr,
+                                       dgrows ? (bf16*)m->xn : nullptr, amode, eps, m->exit_metric, aao_len,
+                                       m->tok_pos, m->err_word) &&
+                     dgrows;
+          m->launches += 1;
+        }
+      }
+      if (!done) {
+        if (xn_valid)
+          gemm(m, st, pr, 1, mrs, m->gemm_cls);
+        else
+          gemm_std(m, st, pr[0], mr, Xi, D, nullptr, amode, eps, m->gemm_cls);
+      }
     }
     // attention over every cached position of layer i
     {
@@ -1169,7 +1227,10 @@ static adept_status run_pass(adept_model* m, int n_tok, int batch, int prompt_le
     if (i < N) {
       // exit test (Sec. 4.1) for 2 <= i <= N-1, inertia update, compaction (App. I)
       const int test = i >= 2;
-      if (n_tok <= EXIT_SMALL_MAX) {
+      if (fuse_exit) {
+        pend = {true, i, par, Xi, Ii, rt};
+        xn_valid = false;
+      } else if (n_tok <= EXIT_SMALL_MAX) {
         xn_valid = launch_exit_small(st, Xi, m->X_out, Ii, i == 1, D, m->ctr, par, rt, m->row_tok[par ^ 1], forced, i,
                                      N, m->d_delta, test, sim_out, m->exit_tok, exit_w, m->X_in[par ^ 1],
                                      m->I[par ^ 1], m->hsm_s, m->hsm_prev, m->hsm_I, mr,
@@ -2000,6 +2061,7 @@ adept_status adept_set_option(adept_model* m, int option, int value) {
     case ADEPT_OPT_DECODE_STREAM: m->use_stream = value != 0; drop_graphs(m); return ADEPT_OK;
     case ADEPT_OPT_DECODE_TILED: m->use_tiled = value != 0; drop_graphs(m); return ADEPT_OK;
     case ADEPT_OPT_ATTN_TC: m->use_attn_tc = value != 0; return ADEPT_OK;
+    case ADEPT_OPT_FUSED_EXIT: m->use_fused_exit = value != 0; drop_graphs(m); return ADEPT_OK;
     case ADEPT_OPT_EXIT_METRIC:
       if (value < EXIT_GLOBAL || value > EXIT_BOTH) return fail(m, ADEPT_ERR_INVALID_ARG, "exit metric %d", value);
       m->exit_metric = value;
