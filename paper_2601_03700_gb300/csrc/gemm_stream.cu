@@ -693,6 +693,9 @@ __global__ void __launch_bounds__(DS_THREADS, 2) gemm_stream_kernel(const __grid
     // the previous layer's exit step first: its kept rows are this launch's rows
     if (tid == 0) s_rb[0] = 0;
     ds_exit_stage(p, xpre, sA, s_red, s_M, s_live, &s_nlive, s_tokk, s_bc);
+    // the span of the product starts here: the exit step (with the standardised rows it writes)
+    // is the previous layer's work, as when it ran as its own kernel before this launch
+    span.waited();
   } else {
     // The row counts (device values) and the A operand are read in parallel: every problem's
     // rows start at row 0 (host-checked), so the launch's row bound max_m is staged without

@@ -85,6 +85,41 @@ def test_llama7b_layer_shapes_threshold(llama_layers):
 
 
 @pytest.fixture(scope="module")
+def llama_layers_b3():
+    cfg = synth.llama7b_config(n_layers=5, max_batch=3, max_seq=24, max_pass_tokens=48, block_shuffle_seed=6)
+    W = synth.make_weights(cfg, seed=3, device="cuda")
+    pair = Pair(cfg, weights=W)
+    del W
+    torch.cuda.empty_cache()
+    yield pair
+    pair.close()
+    torch.cuda.empty_cache()
+
+
+@pytest.mark.parametrize("fused_exit", [1, 0])
+def test_llama7b_layer_shapes_three_sequences_exit_step(llama_layers_b3, fused_exit):
+    """Three sequences per generation step at the Llama-7B layer shapes, forced exits that differ
+    between the sequences of a step (every step keeps some rows and drops others at each layer),
+    then a threshold step: with the exit step inside the next layer's QKV launch (several rows
+    reduced and compacted by every CTA, records written by one) and with the separate exit
+    kernel, each against the oracle; every cached K/V entry at the end."""
+    pair = llama_layers_b3
+    cfg = pair.cfg
+    adept.adept_set_option(pair.gm.h, adept.OPT_FUSED_EXIT, fused_exit)
+    try:
+        B, P = 3, 12
+        tokens = synth.make_tokens(10 + fused_exit, B, P, cfg.vocab).numpy()
+        forced = synth.forced_exits_uniform(10, B * P, 2, cfg.n_layers).numpy().reshape(B, P)
+        ores, cache, g = compare_prefill(pair, tokens, 0.9, forced)
+        fd = np.array([[2, 4, 5], [5, 3, 2], [3, 5, 4], [4, 2, 3]])
+        compare_decode(pair, cache, ores.next_token, 4, 0.9, fd)
+        compare_decode(pair, cache, ores.next_token, 1, 0.9995)
+        pair.compare_cache(cache, B, P + 5)
+    finally:
+        adept.adept_set_option(pair.gm.h, adept.OPT_FUSED_EXIT, 1)
+
+
+@pytest.fixture(scope="module")
 def bert_base():
     cfg = synth.bert_base_config(max_batch=64, max_seq=128, max_pass_tokens=64 * 128)
     W = synth.make_weights(cfg, seed=0, device="cuda")
