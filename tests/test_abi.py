@@ -37,6 +37,16 @@ def test_library_exports_every_declared_symbol(lib):
     assert sorted(adept.ABI_SYMBOLS) == names
 
 
+def test_option_numbers_match_the_header():
+    """Every ADEPT_OPT_* of include/adept.h has the same number as the binding's OPT_*."""
+    import paper_2601_03700_gb300 as adept
+    src = open(os.path.join(ROOT, "include", "adept.h")).read()
+    opts = dict(re.findall(r"ADEPT_OPT_(\w+)\s*=\s*(\d+)", src))
+    assert len(opts) >= 13
+    for name, val in opts.items():
+        assert getattr(adept, "OPT_" + name) == int(val), name
+
+
 def test_status_strings_and_load_validation_without_gpu(lib):
     import synth
     import paper_2601_03700_gb300 as adept
