@@ -21,7 +21,9 @@
 //    for one CTA of the neighbouring kernels (attention, cluster K-split GEMM).
 //  * A operand: after the wait the launch's token rows (all of K) are staged once in shared
 //    memory, copied (bf16) or standardised from the fp32 residual stream with row statistics
-//    computed here or handed over by the producer of the rows.
+//    computed here or handed over by the producer of the rows.  A QKV launch of a generation step
+//    may first take the previous layer's exit step (ds_exit_stage): its kept rows, standardised,
+//    are then the operand.
 //  * MMA: mma.sync m16n8k16 with the weight features as the m16 operand and the token rows
 //    as the n8 operand (the contraction is far below the tensor-core ridge; only bytes count).
 //  * Split tiles: a tile shared by several CTAs is finished by the last one to arrive: each
