@@ -1089,6 +1089,31 @@ def kernel_case_llama_decode_small(device):
     m.close()
 
 
+def kernel_case_llama_decode_ctx(device):
+    """Generation steps at Llama-2-7B layer shapes after the headline workload's 2048-token
+    prompt (2 layers, a 1024-token vocabulary, a small HSM, batch 1, room for 2304 positions as
+    in the headline: the attention grid of 32 heads x 18 key chunks), 3 steps: about 1 GB on the
+    device."""
+    import paper_2601_03700_gb300 as adept
+    adept.load_library()
+    P = 2048
+    cfg = synth.llama7b_config(n_layers=2, vocab=1024, hsm_m1=512, hsm_m2=512, max_batch=1, max_seq=P + 256,
+                               max_pass_tokens=P)
+    W = synth.make_weights(cfg, seed=0, device=device)
+    m = adept.Model(cfg, W)
+    del W
+    tok = synth.make_tokens(0, 1, P, cfg.vocab).to(device)
+    nxt = torch.empty(4, 1, dtype=torch.int32, device=device)
+    full = torch.full((P,), 2, dtype=torch.int32, device=device)
+    adept.adept_prefill(m.h, 1, P, tok.view(-1), DELTA, full, None, None, nxt[0], None)
+    for s in range(3):
+        adept.adept_decode_step(m.h, 1, nxt[s], DELTA, full[:1], None, None, nxt[s + 1], None)
+    torch.cuda.synchronize()
+    m.check()
+    print(json.dumps({"kernel_case": "llama_decode_ctx", "prompt": P, "steps": 3, "ok": True}))
+    m.close()
+
+
 def kernel_case_hsm_train(device, n=8192, steps=2, shape="gpt2"):
     """HSM training steps at GPT-2-small shapes (the bench section's workload; about 5 GB on
     the device), Llama-2-7B shapes (about 25 GB) or BERT-base shapes (the encoder step, n / 128
@@ -1123,7 +1148,7 @@ def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--kernel-case", default=None,
                     choices=["fill_small", "fill_grid", "llama_prefill", "gpt2_decode", "llama_decode_small",
-                             "hsm_train"])
+                             "llama_decode_ctx", "hsm_train"])
     ap.add_argument("--gpus", type=int, default=1)
     ap.add_argument("--steps", type=int, default=5)
     ap.add_argument("--warmup", type=int, default=3)
@@ -1162,6 +1187,9 @@ def main():
         return
     if args.kernel_case == "llama_decode_small":
         kernel_case_llama_decode_small(torch.device("cuda", 0))
+        return
+    if args.kernel_case == "llama_decode_ctx":
+        kernel_case_llama_decode_ctx(torch.device("cuda", 0))
         return
     if args.kernel_case == "hsm_train":
         kernel_case_hsm_train(torch.device("cuda", 0), n=args.hsm_n, shape=args.hsm_shape)
