@@ -95,3 +95,33 @@ def test_hsm_train_flops():
     assert bench.hsm_train_flops(g, 10) == pytest.approx(10 * (6.0 * fc + 4.0 * 768 * g.vocab), rel=1e-12)
     e = synth.bert_base_config()
     assert bench.hsm_train_flops(e, 10, 2) == pytest.approx(10 * 6.0 * fc + 2 * 4.0 * 768 ** 2, rel=1e-12)
+
+
+def test_fill_micro_work_counts_the_oracles_fill():
+    """The fill grid's numerators (bench.fill_micro_work) against a count over what the oracle's
+    skipped-layer fill computes (Sec. 4.3) on a small Llama-shaped model with the grid's law (all
+    T tokens leaving at i*): every produced (token, layer) entry is two products of the layer's
+    K and V weight shapes; each filled layer's W_K / W_V is read once, each s~ once, each entry
+    written once (bf16 throughout)."""
+    from oracle import adept_oracle as O
+    cfg = synth.ModelConfig(family=synth.LLAMA, n_layers=6, d_model=16, n_heads=2, n_kv_heads=1, head_dim=8,
+                            d_ffn=32, vocab=50, max_pos=64, dtype="f32", max_batch=2, max_seq=16)
+    assert cfg.n_kv_heads * cfg.head_dim != cfg.d_model   # D_kv and D told apart
+    m = O.OracleModel(cfg, synth.make_weights(cfg, seed=5))
+    shapes = synth.weight_shapes(cfg)
+    for T, istar in ((1, 2), (3, 4), (5, 6), (2, 1)):
+        out = O.skip_kv_fill(m, np.ones((T, cfg.d_model)), np.full(T, istar), np.arange(T))
+        flops = bytes_ = 0
+        for r, (k, v, sel) in out.items():
+            wk, wv = shapes[f"layers.{r - 1}.wk"], shapes[f"layers.{r - 1}.wv"]   # [D_kv, D] each
+            flops += len(sel) * 2 * (wk[0] * wk[1] + wv[0] * wv[1])
+            bytes_ += (wk[0] * wk[1] + wv[0] * wv[1]) * 2 + len(sel) * (wk[0] + wv[0]) * 2
+            assert k.shape == v.shape == (len(sel), cfg.n_kv_heads, cfg.head_dim)
+        bytes_ += T * cfg.d_model * 2
+        want_f, want_b = bench.fill_micro_work(T, istar, n_layers=cfg.n_layers, d=cfg.d_model,
+                                               dkv=cfg.n_kv_heads * cfg.head_dim)
+        if istar == cfg.n_layers:   # nothing to fill: no product and no weight read
+            assert not out and want_f == 0
+            continue
+        assert flops == want_f, (T, istar)
+        assert bytes_ == want_b, (T, istar)
